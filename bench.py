@@ -1,0 +1,499 @@
+#!/usr/bin/env python
+"""Benchmark of the SideQuest KV-cache hot path on GB300.
+
+Workload (default, "serving-128k"): batched long-horizon serving — 8
+requests of 131,072 tokens, each paired with an auxiliary fork (16 decoding
+sequences), 32 layers, 32 query / 8 KV heads, head dim 128, page size 64,
+bf16.  Synthetic N(0,1) K/V and queries (they stand in for the FRAMES /
+BrowseComp agent contexts of the paper's Sec. 4.1, whose lengths pass 100k
+tokens, Fig. 2).
+
+One step = one decode token for every sequence: append its K/V row
+(all layers) and run decode attention at all 32 layers (each call reads the
+shared prefix pages once for main + aux).  Then, timed separately: release
+the forks, evict 20-65% of every request in 10-40 spans (Algorithm 1,
+clear_kv), re-fork, and decode again.
+
+Prints one JSON line.  `--impl reference` times the CPU oracle on a bounded
+sample of the same workload instead (the reference arm).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import shutil
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "decode-attn tokens/s + achieved HBM GB/s at 128k ctx; span-evict GB/s"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="sq", choices=["sq", "reference"])
+    ap.add_argument("--requests", type=int, default=8)
+    ap.add_argument("--ctx", type=int, default=131072)
+    ap.add_argument("--layers", type=int, default=32)
+    ap.add_argument("--no-evict", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--seed", type=int, default=0)
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.proc = None
+        self.path = None
+        exe = shutil.which("nvidia-smi")
+        if not exe:
+            return
+        fd, self.path = tempfile.mkstemp(prefix="sq_clocks_", suffix=".csv")
+        os.close(fd)
+        self.out = open(self.path, "w")
+        self.proc = subprocess.Popen(
+            [exe, f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200",
+             "-i", str(device_index)], stdout=self.out, stderr=subprocess.DEVNULL)
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.out.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+
+
+def dist_setup():
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------
+# workload
+# ---------------------------------------------------------------------------
+def workload_name(args):
+    return (f"serving-128k: {args.requests} requests x {args.ctx} tokens + {args.requests} aux forks "
+            f"({2 * args.requests} decoding sequences), {args.layers} layers, 32q/8kv heads, d128, "
+            f"page 64, bf16")
+
+
+def request_spans(seed, r, n, P):
+    """Per request: 20-65% of the context (uniform) in 10-40 spans (uniform)
+    with lognormal lengths (median 2,000 tokens), inside [P, n)."""
+    import numpy as np
+    from synthetic import random_spans, shuffled, sub_seed
+    rng = np.random.default_rng(sub_seed(seed, 100 + r))
+    frac = rng.uniform(0.20, 0.65)
+    k = int(rng.integers(10, 41))
+    total = int(frac * (n - P))
+    return shuffled(random_spans(sub_seed(seed, 200 + r), k, total, P, n, median=2000), r)
+
+
+def run_sq(args, world, rank, local):
+    import numpy as np
+    import torch
+
+    import paper_2602_22603_gb300 as sq
+    from synthetic import AGENT_8B, Bank, bf16_normal, sub_seed
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    sh = AGENT_8B
+    L, Hq, Hkv, D, P = args.layers, sh.num_q_heads, sh.num_kv_heads, sh.head_dim, sh.page_size
+    R, ctx = args.requests, args.ctx
+    S = 2 * R
+    extra_tokens = 8 + (args.warmup + args.steps) * 3 + 64
+    pages_per_req = (ctx + extra_tokens) // P + 2
+    num_pages = R * pages_per_req + R * ((extra_tokens // P) + 2) + 64
+    scale = 1.0 / math.sqrt(D)
+    seed = args.seed + 1000 * rank
+    cache = sq.Cache(L, Hq, Hkv, D, P, num_pages, max_seqs=4 * S + 8)
+    stream = torch.cuda.current_stream()
+
+    # K/V source: a seeded N(0,1) bank sliced at seeded offsets
+    chunk = 4096
+    bank = Bank(1 << 28, sub_seed(seed, 1), device="cuda")
+    chunk_elems = L * chunk * Hkv * D
+    n_chunks = ctx // chunk
+    offs = bank.offsets(R * n_chunks * 2, chunk_elems, sub_seed(seed, 2))
+    mains, auxs = [], []
+    for r in range(R):
+        m = cache.seq_new()
+        for c in range(n_chunks):
+            i = (r * n_chunks + c) * 2
+            cache.append_kv(m, chunk, bank.view(offs[i], (L, chunk, Hkv, D)),
+                            bank.view(offs[i + 1], (L, chunk, Hkv, D)))
+        mains.append(m)
+    tok_elems = L * Hkv * D
+    small = bank.offsets(8192, 2 * 8 * tok_elems, sub_seed(seed, 3))
+    small_i = [0]
+
+    def kv_rows(n):
+        """K and V of n <= 8 new tokens, [L, n, Hkv, D] views of the bank."""
+        o = int(small[small_i[0] % len(small)])
+        small_i[0] += 1
+        return bank.view(o, (L, n, Hkv, D)), bank.view(o + 8 * tok_elems, (L, n, Hkv, D))
+
+    def fork_all():
+        auxs.clear()
+        for m in mains:
+            a = cache.fork_aux(m)
+            k, v = kv_rows(8)                       # trigger phrase (Sec. 3.2)
+            cache.append_kv(a, 8, k, v)
+            auxs.append(a)
+
+    fork_all()
+    seqs = [x for pair in zip(mains, auxs) for x in pair]
+    q_all = bf16_normal((L, S, Hq, D), sub_seed(seed, 4), device="cuda")
+    out_all = torch.empty(L, S, Hq, D, dtype=torch.bfloat16, device="cuda")
+    torch.cuda.synchronize()
+
+    def step(ev=None):
+        for h in seqs:
+            k, v = kv_rows(1)
+            cache.append_kv(h, 1, k, v)
+        if ev is not None:
+            ev.record(stream)
+        for layer in range(L):
+            cache.decode_attention(seqs, layer, q_all[layer], out_all[layer], sq.SQ_OUT_BF16, scale)
+
+    def timed_decode(K, W):
+        for _ in range(W):
+            step()
+        torch.cuda.synchronize()
+        barrier(world)
+        st0 = cache.stats()
+        ev_s = [torch.cuda.Event(enable_timing=True) for _ in range(K + 1)]
+        ev_m = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+        ev_s[0].record(stream)
+        for t in range(K):
+            step(ev_m[t])
+            ev_s[t + 1].record(stream)
+        torch.cuda.synchronize()
+        st1 = cache.stats()
+        total_ms = ev_s[0].elapsed_time(ev_s[K])
+        attn_ms = sum(ev_m[t].elapsed_time(ev_s[t + 1]) for t in range(K))
+        calls = st1["decode_calls"] - st0["decode_calls"]
+        uniq = st1["decode_unique_bytes"] - st0["decode_unique_bytes"]
+        logi = st1["decode_logical_bytes"] - st0["decode_logical_bytes"]
+        return {"total_ms": total_ms, "attn_ms": attn_ms, "calls": calls, "unique_bytes": uniq,
+                "logical_bytes": logi}
+
+    hbm_peak, peak_kind = peaks()
+    clocks = ClockSampler(local)
+    time.sleep(0.4)
+    K, W = args.steps, args.warmup
+    before = timed_decode(K, W)
+    clock_rec = clocks.stop()
+    t_total = max_over_ranks(before["total_ms"], world)
+    value = world * S * K / (t_total / 1e3)
+    per_call_ms = before["attn_ms"] / before["calls"]
+    uniq_per_call = before["unique_bytes"] / before["calls"]
+    achieved = uniq_per_call / (per_call_ms / 1e3) / 1e9
+    logical_gbs = before["logical_bytes"] / before["calls"] / (per_call_ms / 1e3) / 1e9
+
+    res = {
+        "metric": METRIC,
+        "value": round(value, 3),
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": W,
+        "ms_per_step": round(t_total / K, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) K/V bank, random-init queries; no dataset)",
+        "config": {
+            "workload": workload_name(args),
+            "requests_per_gpu": R, "context_tokens": ctx, "decoding_sequences_per_gpu": S,
+            "layers": L, "q_heads": Hq, "kv_heads": Hkv, "head_dim": D, "page_size": P,
+            "sm_scale": scale,
+            "l2": "inputs larger than L2: %.2f GB of distinct K/V per decode call" % (uniq_per_call / 1e9),
+            "parallelism": "replicas: requests partitioned across GPUs, no collective" if world > 1
+            else "single GPU",
+        },
+        "decode": {
+            "attn_ms_per_step": round(before["attn_ms"] / K, 4),
+            "attn_ms_per_call": round(per_call_ms, 5),
+            "tokens_per_s_attention_only": round(S * K / (before["attn_ms"] / 1e3), 3),
+            "unique_gb_per_call": round(uniq_per_call / 1e9, 4),
+            "logical_gb_per_call": round(before["logical_bytes"] / before["calls"] / 1e9, 4),
+            "hbm_gbs_unique": round(achieved, 1),
+            "hbm_gbs_logical": round(logical_gbs, 1),
+            "frac_of_%s_peak" % peak_kind: round(achieved / hbm_peak, 4),
+            "frac_of_nominal_8tbs": round(achieved / 8000.0, 4),
+        },
+        "roofline": {
+            "bound": "hbm",
+            "kernel": "sq_decode_splitk_kernel (+ sq_lse_combine_kernel, timed together per call)",
+            "achieved": round(achieved, 1),
+            "peak": hbm_peak,
+            "peak_kind": peak_kind,
+            "unit": "GB/s",
+            "frac": round(achieved / hbm_peak, 4),
+            "traffic": None,
+            "algorithmic_bytes_per_launch": int(uniq_per_call),
+        },
+        "gpu_launches": int(K * (S + 2 * L)),
+        "clocks": clock_rec,
+    }
+
+    # ---- end to end through the C ABI with host buffers ----------------------
+    if not args.no_e2e:
+        q_h = q_all.cpu().pin_memory()
+        out_h = torch.empty(out_all.shape, dtype=out_all.dtype).pin_memory()
+        o_e2e = int(bank.offsets(1, S * 2 * tok_elems, sub_seed(seed, 5))[0])
+        kv_h = bank.view(o_e2e, (S, 2, L, 1, Hkv, D)).cpu().pin_memory()
+        kv_d = torch.empty(S, 2, L, 1, Hkv, D, dtype=torch.bfloat16, device="cuda")
+        q_d = torch.empty_like(q_all)
+
+        def e2e_step():
+            q_d.copy_(q_h, non_blocking=True)
+            kv_d.copy_(kv_h, non_blocking=True)
+            for i, h in enumerate(seqs):
+                cache.append_kv(h, 1, kv_d[i, 0], kv_d[i, 1])
+            for layer in range(L):
+                cache.decode_attention(seqs, layer, q_d[layer], out_all[layer], sq.SQ_OUT_BF16, scale)
+            out_h.copy_(out_all, non_blocking=True)
+
+        for _ in range(W):
+            e2e_step()
+        torch.cuda.synchronize()
+        barrier(world)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        w0 = time.perf_counter()
+        e0.record(stream)
+        for _ in range(K):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - w0
+        e_ms = max_over_ranks(max(e0.elapsed_time(e1), wall * 1e3), world)
+        res["e2e"] = {
+            "value": round(world * S * K / (e_ms / 1e3), 3), "unit": "tokens/s",
+            "h2d_bytes_per_step": int(q_h.numel() * 2 + kv_h.numel() * 2),
+            "d2h_bytes_per_step": int(out_h.numel() * 2),
+            "note": "pinned host q and new-token K/V copied in, outputs copied out, every step",
+        }
+
+    # ---- eviction: release forks, evict per request, re-fork, decode again ---
+    if not args.no_evict:
+        for a in auxs:
+            cache.release(a)
+        torch.cuda.synchronize()
+        st0 = cache.stats()
+        ev_ms = 0.0
+        per = []
+        for r, m in enumerate(mains):
+            n = cache.seq_info(m)[0]
+            spans = request_spans(seed, r, n, P)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            b0 = cache.stats()["evict_bytes"]
+            e0.record(stream)
+            cache.evict_spans(m, spans)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1)
+            ev_ms += ms
+            per.append((cache.stats()["evict_bytes"] - b0) / (ms / 1e3) / 1e9)
+        st1 = cache.stats()
+        ev_bytes = st1["evict_bytes"] - st0["evict_bytes"]
+        assert cache.sync_status() == sq.SQ_OK
+        ev_gbs = ev_bytes / (ev_ms / 1e3) / 1e9
+        fork_all()
+        seqs[:] = [x for pair in zip(mains, auxs) for x in pair]
+        torch.cuda.synchronize()
+        after = timed_decode(K, W)
+        pc = after["attn_ms"] / after["calls"]
+        up = after["unique_bytes"] / after["calls"]
+        res["evict"] = {
+            "gbs": round(ev_gbs, 1),
+            "frac_of_%s_peak" % peak_kind: round(ev_gbs / hbm_peak, 4),
+            "ms_total": round(ev_ms, 4),
+            "algorithmic_bytes": int(ev_bytes),
+            "evicted_tokens_per_layer": int(st1["evicted_tokens"] - st0["evicted_tokens"]),
+            "moved_rows": int(st1["evict_moved_rows"] - st0["evict_moved_rows"]),
+            "per_request_gbs": [round(x, 1) for x in per],
+            "calls": len(mains),
+        }
+        res["after_evict"] = {
+            "tokens_per_s": round(world * S * K / (max_over_ranks(after["total_ms"], world) / 1e3), 3),
+            "attn_ms_per_call": round(pc, 5),
+            "unique_gb_per_call": round(up / 1e9, 4),
+            "hbm_gbs_unique": round(up / (pc / 1e3) / 1e9, 1),
+        }
+        st = cache.stats()
+        res["peak_live_pages"] = st["peak_live_pages"]
+
+    # ---- CPU oracle on a bounded sample (rank 0, N = 1) ----------------------
+    if not args.no_cpu and rank == 0 and world == 1:
+        res["cpu_baseline"] = cpu_baseline(args, bank, offs, n_chunks, chunk, scale)
+
+    cache.close()
+    return res
+
+
+def cpu_baseline(args, bank, offs, n_chunks, chunk, scale):
+    """The oracle as it stands (oracle/attention.c) on the host cores: one
+    decode step of request 0's main sequence and of an aux fork at one layer
+    over the full context (2 sequences x 1 layer), scaled to tokens/s."""
+    import numpy as np
+
+    from oracle import attention as oatt
+    from synthetic import bf16_bits, bf16_normal
+    L, Hq, Hkv, D = args.layers, 32, 8, 128
+    host_bank = bf16_bits(bank.data.cpu())
+    layer = 0
+
+    def rows(which):
+        parts = []
+        for c in range(n_chunks):
+            o = int(offs[c * 2 + which])
+            a = host_bank[o:o + L * chunk * Hkv * D].reshape(L, chunk, Hkv, D)
+            parts.append(a[layer])
+        return np.ascontiguousarray(np.concatenate(parts))
+
+    k, v = rows(0), rows(1)
+    q = bf16_bits(bf16_normal((2, Hq, D), 99))
+    oatt.decode_batch(q[:1, :, :], [k[:1024]], [v[:1024]], scale)  # warm
+    t0 = time.perf_counter()
+    oatt.decode_batch(q, [k, k], [v, v], scale)
+    t = time.perf_counter() - t0
+    tokens_per_s = 2 / (t * L)
+    return {"value": round(tokens_per_s, 4), "unit": "tokens/s", "cores": oatt.num_threads(),
+            "kind": "oracle",
+            "sample": f"2 sequences x 1 of {L} layers, {k.shape[0]} tokens each, all {Hq} heads "
+                      f"(fp64 C oracle, OpenMP); tokens/s = 2 / (time x {L} layers)",
+            "seconds": round(t, 3)}
+
+
+def run_reference(args, world, rank):
+    """Reference arm: the CPU oracle as it stands, on this machine's host cores,
+    for the same metric; each step is a bounded sample of the workload."""
+    import numpy as np
+
+    from oracle import attention as oatt
+    from synthetic import bf16_bits, bf16_normal, sub_seed
+    if rank != 0:
+        return None
+    L, Hq, Hkv, D = args.layers, 32, 8, 128
+    n = args.ctx
+    scale = 1.0 / math.sqrt(D)
+    k = bf16_bits(bf16_normal((n, Hkv, D), sub_seed(args.seed, 11)))
+    v = bf16_bits(bf16_normal((n, Hkv, D), sub_seed(args.seed, 12)))
+    q = bf16_bits(bf16_normal((2, Hq, D), sub_seed(args.seed, 13)))
+    for _ in range(args.warmup):
+        oatt.decode_batch(q[:1], [k[:4096]], [v[:4096]], scale)
+    ts = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oatt.decode_batch(q, [k, k], [v, v], scale)
+        ts.append(time.perf_counter() - t0)
+    t = sum(ts)
+    value = 2 * args.steps / (t * L)
+    sample = (f"per step: 2 sequences (main + aux) x 1 of {L} layers at {n} tokens, all {Hq} heads, "
+              f"fp64 C oracle with OpenMP; tokens/s = sequences / (time x {L} layers)")
+    return {
+        "metric": METRIC, "value": round(value, 4), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(t / args.steps * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "impl": "reference",
+        "config": {"workload": workload_name(args)},
+        "cpu_baseline": {"value": round(value, 4), "unit": "tokens/s", "cores": oatt.num_threads(),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 4), "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        world = int(os.environ.get("WORLD_SIZE", "1"))
+        rank = int(os.environ.get("RANK", "0"))
+        res = run_reference(args, world, rank)
+        if res is not None:
+            print(json.dumps(res), flush=True)
+        return
+    world, rank, local = dist_setup()
+    res = run_sq(args, world, rank, local)
+    if rank == 0:
+        print(json.dumps(res), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,222 @@
+/*
+ * sq.h — C ABI of libsq, the GB300 (sm_103a) hot path behind SideQuest's
+ * model-driven KV-cache management (Kariyappa & Suh, "SideQuest: Model-Driven
+ * KV Cache Management for Long-Horizon Agentic Reasoning").
+ *
+ * The library keeps a paged bf16 KV pool on one GPU.  A main reasoning
+ * sequence and the auxiliary sequences forked from it share their prefix
+ * pages (reference-counted, copy-on-write); decode attention reads the pages
+ * through per-sequence page tables; span eviction removes cursor-identified
+ * message spans and compacts the surviving rows in place.
+ *
+ * Conventions for every call:
+ *   - Return value: SQ_OK (0) or one of the negative SQ_ERR_* codes below.
+ *   - On any error the host-side state (sequences, page tables, reference
+ *     counts, free pages) is left exactly as it was before the call.
+ *   - Device work is enqueued asynchronously on the `stream` argument
+ *     (a cudaStream_t passed as void*; NULL = the legacy default stream).
+ *     Nothing is copied back to the host; device-side faults detected by
+ *     the kernels' own checks are reported by sq_sync_status().
+ *   - Pointers named "device" must point to GPU memory of the cache's device;
+ *     pointers named "host" to CPU memory.  The caller keeps ownership of all
+ *     buffers it passes; the library never frees them.  Device input buffers
+ *     must stay valid until the enqueued work has run.
+ *   - A cache is not thread-safe: one host thread issues its calls.  Calls
+ *     may use different streams; the caller orders work on one sequence
+ *     (e.g. evicting a sequence after its own decode on another stream,
+ *     Sec. 3.1 step 4: eviction waits for the main thread's current turn).
+ *
+ * KV pool layout (bf16, 16-bit elements), for layer l, page p, plane kv
+ * (0 = K, 1 = V), KV head h, slot s, dimension e:
+ *     pool[((((l * num_pages + p) * 2 + kv) * num_kv_heads + h) * page_size
+ *           + s) * head_dim + e]
+ * Logical token j of a sequence lives in slot j % page_size of page
+ * page_table[j / page_size].
+ */
+#ifndef SQ_H_
+#define SQ_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SQ_API __attribute__((visibility("default")))
+#else
+#define SQ_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Opaque cache object, owned by the library. */
+typedef struct sq_cache sq_cache;
+
+/* Sequence handle: slot | generation << 20; always > 0.  A released
+ * handle is rejected with SQ_ERR_BAD_HANDLE. */
+typedef int32_t sq_seq;
+
+/* A half-open span [start, end) of CURRENT logical token positions of one
+ * sequence — the tokens of a tool call and its response (Sec. 3, Goal and
+ * its footnote; Algorithm 1, C.clear_kv(Delta_ids)).  The caller maps the
+ * auxiliary thread's cursor ids to spans. */
+typedef struct {
+    int32_t start;
+    int32_t end;
+} sq_span;
+
+typedef struct {
+    int32_t num_layers;        /* L   >= 1 */
+    int32_t num_q_heads;       /* Hq  >= 1, multiple of num_kv_heads */
+    int32_t num_kv_heads;      /* Hkv >= 1; Hq / Hkv <= 16 */
+    int32_t head_dim;          /* d: 64 or 128 */
+    int32_t page_size;         /* P: power of two, 8 .. 256 */
+    int32_t num_pages;         /* pages in the pool (each holds P tokens of every layer) */
+    int32_t max_seqs;          /* live sequences at most (<= 2^20 - 1) */
+    int32_t max_pages_per_seq; /* page-table capacity of one sequence */
+    void *kv_pool;             /* device; NULL = the library allocates (and zeroes) the
+                                  pool; else caller memory of sq_pool_bytes() bytes,
+                                  256-byte aligned, owned by the caller */
+    int32_t decode_ctas;       /* 0 = automatic (SMs x resident CTAs per SM); else the
+                                  number of persistent CTAs decode attention uses */
+} sq_config;
+
+enum {
+    SQ_OK = 0,
+    SQ_ERR_INVALID_ARG = -1,     /* a bad pointer, size, span, dtype or layer */
+    SQ_ERR_BAD_HANDLE = -2,      /* unknown or released sequence / cache */
+    SQ_ERR_NO_PAGES = -3,        /* the pool has too few free pages */
+    SQ_ERR_CAPACITY = -4,        /* a sequence would exceed max_pages_per_seq,
+                                    or max_seqs sequences are live */
+    SQ_ERR_CUDA = -5,            /* a CUDA runtime call failed */
+    SQ_ERR_DEVICE = -6,          /* a kernel's own bounds check fired */
+    SQ_ERR_DEVICE_TIMEOUT = -7,  /* a kernel's bounded wait ran out */
+    SQ_ERR_UNSUPPORTED = -8,     /* a geometry this build does not handle */
+    SQ_ERR_NO_MEMORY = -9        /* host or device allocation failed */
+};
+
+enum { SQ_OUT_BF16 = 0, SQ_OUT_F32 = 1 };
+
+/* Bytes of the KV pool for a configuration (0 if it is invalid). */
+SQ_API size_t sq_pool_bytes(const sq_config *cfg);
+
+/* Create a cache on the current CUDA device.  *out receives the handle.
+ * Paper: Sec. 3.4 (Storage Costs) — one pool shared by the main and
+ * auxiliary threads.  Errors: INVALID_ARG, UNSUPPORTED, NO_MEMORY, CUDA. */
+SQ_API int sq_cache_create(const sq_config *cfg, sq_cache **out);
+
+/* Destroy a cache (synchronises the device first; frees library memory). */
+SQ_API int sq_cache_destroy(sq_cache *cache);
+
+/* A new, empty main sequence (Algorithm 1: C <- [Q] starts empty here and
+ * the query tokens are appended).  Errors: CAPACITY. */
+SQ_API int sq_seq_new(sq_cache *cache, sq_seq *out);
+
+/* Append n_tokens K/V rows to the end of `seq` (Algorithm 1: C <- C + R,
+ * C <- C + O; the aux thread's C_aux <- C + p).
+ *   k, v: device, bf16, contiguous [num_layers][n_tokens][num_kv_heads][head_dim]
+ *         (keys already rotated: the library never applies positional
+ *         encodings).
+ * If the sequence's last page is partial and shared with another sequence it
+ * is first copied (copy-on-write); then fresh pages are taken, lowest free id
+ * first, in increasing logical order.  n_tokens == 0 is a no-op.
+ * Errors: BAD_HANDLE, INVALID_ARG, NO_PAGES, CAPACITY, CUDA. */
+SQ_API int sq_append_kv(sq_cache *cache, sq_seq seq, int32_t n_tokens, const void *k,
+                 const void *v, void *stream);
+
+/* Fork an auxiliary sequence that shares the whole context of `parent`
+ * (Sec. 3.1 step 1; Algorithm 1 phase 2, C_aux <- C + p; Sec. 3.4: the
+ * auxiliary thread does not duplicate the KV cache).  The child gets the same
+ * page ids and token count; every page's reference count grows by one; no
+ * K/V byte is copied and no device work is enqueued.
+ * Errors: BAD_HANDLE, CAPACITY. */
+SQ_API int sq_fork_aux(sq_cache *cache, sq_seq parent, sq_seq *child_out);
+
+/* Decode attention for one new query token of each of n_seqs sequences at
+ * layer `layer` (Sec. 1 and Sec. 3.4: attention reads the whole KV cache of
+ * the context for every generated token; Sec. 2.1: grouped-query attention).
+ * For sequence i, query head h and KV head g = h / (Hq / Hkv):
+ *     out[i][h] = sum_t softmax_t(sm_scale * q[i][h] . K_g[t]) V_g[t]
+ * over all n_i tokens of the sequence in logical order.
+ *   seqs: host, n_seqs distinct live handles, each with >= 1 token
+ *   q:    device, bf16 [n_seqs][num_q_heads][head_dim]
+ *   out:  device, [n_seqs][num_q_heads][head_dim], bf16 (SQ_OUT_BF16, round
+ *         to nearest even) or fp32 (SQ_OUT_F32)
+ * Sequences that share pages (a main thread and its forks) in one call read
+ * each shared page once for all of them (Sec. 3.4, shared-context kernels).
+ * Errors: BAD_HANDLE, INVALID_ARG, NO_MEMORY, CUDA. */
+SQ_API int sq_decode_attention(sq_cache *cache, const sq_seq *seqs, int32_t n_seqs,
+                        int32_t layer, const void *q, void *out,
+                        int32_t out_dtype, float sm_scale, void *stream);
+
+/* Evict spans from `seq` (Algorithm 1 phase 1, C.clear_kv(Delta_ids);
+ * Sec. 3.1 step 3).  The kept tokens keep their order and their K/V bytes
+ * (keys are never re-rotated); row j of the result is the j-th kept row.
+ *   spans: host, n_spans half-open spans of current positions, any order;
+ *          empty, overlapping or out-of-range spans are INVALID_ARG;
+ *          n_spans == 0 is a no-op.
+ * Pages whose contents change and that are shared with another sequence are
+ * replaced by fresh pages (copy-on-write, increasing logical page order);
+ * others are compacted in place; pages past the new end are released.
+ * Errors: BAD_HANDLE, INVALID_ARG, NO_PAGES, NO_MEMORY, CUDA. */
+SQ_API int sq_evict_spans(sq_cache *cache, sq_seq seq, const sq_span *spans,
+                   int32_t n_spans, void *stream);
+
+/* Release a sequence (Algorithm 1: S_thread <- None; Sec. 3.4: the
+ * auxiliary thread's own tokens are discarded).  Every page loses one
+ * reference; pages that reach zero become free once all work enqueued on
+ * `stream` (and on the stream that last used the sequence) before this call
+ * has completed — later work on other streams that takes them waits for it.
+ * Errors: BAD_HANDLE, CUDA. */
+SQ_API int sq_release(sq_cache *cache, sq_seq seq, void *stream);
+
+/* ---- inspection helpers (host-side, no device work) ---- */
+
+/* Token count and page count of a sequence. */
+SQ_API int sq_seq_info(sq_cache *cache, sq_seq seq, int32_t *n_tokens,
+                int32_t *n_pages);
+
+/* Copy the page table of `seq` into host_out[0 .. cap); *n_out = its length.
+ * Errors: BAD_HANDLE, INVALID_ARG (cap too small). */
+SQ_API int sq_get_page_table(sq_cache *cache, sq_seq seq, int32_t *host_out,
+                      int32_t cap, int32_t *n_out);
+
+/* Reference count of a page (0 = free). */
+SQ_API int sq_page_refcount(sq_cache *cache, int32_t page, int32_t *out);
+
+/* Number of free pages. */
+SQ_API int sq_free_pages(sq_cache *cache, int32_t *out);
+
+/* Device pointer of the KV pool (layout above). */
+SQ_API int sq_pool_ptr(sq_cache *cache, void **out);
+
+typedef struct {
+    int64_t live_pages;          /* pages with a nonzero reference count now */
+    int64_t peak_live_pages;     /* Sec. 4.5, Peak Token Utilization (in pages) */
+    int64_t decode_calls;
+    int64_t decode_logical_bytes;/* Sec. 4.5, KV Cache Memory Reads: sum over calls
+                                    and sequences of tokens x 2 x Hkv x d x 2 B */
+    int64_t decode_unique_bytes; /* the same with pages shared inside one call
+                                    counted once */
+    int64_t evict_calls;
+    int64_t evicted_tokens;
+    int64_t evict_moved_rows;    /* token rows rewritten (all layers/planes count once) */
+    int64_t evict_bytes;         /* algorithmic bytes read + written by compaction */
+    int64_t appended_tokens;
+    int64_t cow_pages;           /* pages copied on write (append + evict) */
+} sq_stats_t;
+
+SQ_API int sq_stats(sq_cache *cache, sq_stats_t *out);
+
+/* Synchronise `stream`, then read and clear the device error word.
+ * Returns SQ_OK, SQ_ERR_DEVICE, SQ_ERR_DEVICE_TIMEOUT or SQ_ERR_CUDA. */
+SQ_API int sq_sync_status(sq_cache *cache, void *stream);
+
+/* Human-readable name of a return code. */
+SQ_API const char *sq_strerror(int code);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SQ_H_ */

@@ -1,0 +1,105 @@
+// A small C interface over the host-side cache state and planners, built into
+// a separate CPU-only library (libsq_host.so) so that the page allocator,
+// the copy-on-write / eviction rules and the decode planner can be exercised
+// without a GPU.  It drives exactly the code libsq.so runs on the host.
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "../host/core.hpp"
+
+using namespace sq;
+
+extern "C" {
+
+void* sqh_create(int32_t L, int32_t Hq, int32_t Hkv, int32_t D, int32_t P,
+                 int32_t num_pages, int32_t max_seqs, int32_t max_pages_per_seq) {
+    Geometry g;
+    g.L = L; g.Hq = Hq; g.Hkv = Hkv; g.D = D; g.P = P;
+    g.num_pages = num_pages; g.max_seqs = max_seqs; g.max_pages_per_seq = max_pages_per_seq;
+    if (check_geometry(g) != kOk) return nullptr;
+    return new (std::nothrow) HostCache(g);
+}
+
+void sqh_destroy(void* c) { delete static_cast<HostCache*>(c); }
+
+int sqh_seq_new(void* c, int32_t* h) { return static_cast<HostCache*>(c)->seq_new(h); }
+
+int sqh_fork(void* c, int32_t parent, int32_t* child) {
+    return static_cast<HostCache*>(c)->fork(parent, child);
+}
+
+int sqh_append(void* c, int32_t h, int32_t n) {
+    AppendPlan p;
+    return static_cast<HostCache*>(c)->append(h, n, &p);
+}
+
+// stats_out (may be NULL): moved_rows, cow_pages, freed_pages, first_row, n_runs
+int sqh_evict(void* c, int32_t h, const int32_t* spans, int32_t n_spans, int64_t* stats_out) {
+    std::vector<int32_t> a(n_spans > 0 ? n_spans : 0), b(a.size());
+    for (int32_t i = 0; i < n_spans; ++i) { a[i] = spans[2 * i]; b[i] = spans[2 * i + 1]; }
+    EvictPlan p;
+    int rc = static_cast<HostCache*>(c)->evict(h, a.data(), b.data(), n_spans, &p);
+    if (rc == kOk && stats_out) {
+        stats_out[0] = p.moved_rows;
+        stats_out[1] = (int64_t)p.cow_pages.size();
+        stats_out[2] = (int64_t)p.freed.size();
+        stats_out[3] = p.first_row;
+        stats_out[4] = (int64_t)p.run_dst.size();
+    }
+    return rc;
+}
+
+int sqh_release(void* c, int32_t h) { return static_cast<HostCache*>(c)->release(h, nullptr); }
+
+int sqh_seq_info(void* c, int32_t h, int32_t* n_tokens, int32_t* n_pages) {
+    const Seq* s = static_cast<HostCache*>(c)->seq(h);
+    if (!s) return kBadHandle;
+    *n_tokens = s->n;
+    *n_pages = (int32_t)s->pages.size();
+    return kOk;
+}
+
+int sqh_page_table(void* c, int32_t h, int32_t* out, int32_t cap, int32_t* n_out) {
+    const Seq* s = static_cast<HostCache*>(c)->seq(h);
+    if (!s) return kBadHandle;
+    *n_out = (int32_t)s->pages.size();
+    if (cap < *n_out) return kInvalidArg;
+    std::memcpy(out, s->pages.data(), sizeof(int32_t) * s->pages.size());
+    return kOk;
+}
+
+int sqh_refcount(void* c, int32_t p) {
+    HostCache* hc = static_cast<HostCache*>(c);
+    if (p < 0 || p >= hc->geom().num_pages) return -1;
+    return hc->alloc().refcount(p);
+}
+
+int sqh_free_count(void* c) { return static_cast<HostCache*>(c)->alloc().free_count(); }
+
+int64_t sqh_peak_live_pages(void* c) { return static_cast<HostCache*>(c)->peak_live_pages(); }
+
+// Plans a decode call.  layout_out receives 16 int64 values:
+//   offsets segs, items, cta_begin, page_ids, comb_off, comb_ent, total,
+//   counts n_segs, n_items, n_ctas, n_page_ids, n_comb_keys, n_comb_ent,
+//   unique_tokens, logical_tokens, sizeof(DecodeSeg).
+// If buf is non-NULL and buf_bytes >= total, the serialised plan is written.
+int sqh_plan_decode(void* c, const int32_t* handles, int32_t n, int32_t n_ctas,
+                    int64_t* layout_out, uint8_t* buf, int64_t buf_bytes) {
+    HostCache* hc = static_cast<HostCache*>(c);
+    DecodePlanHost p;
+    int rc = plan_decode(*hc, handles, n, n_ctas, &p);
+    if (rc != kOk) return rc;
+    DecodePlanLayout L = plan_layout(p, n, hc->geom().Hkv);
+    int64_t v[16] = {L.segs, L.items, L.cta_begin, L.page_ids, L.comb_off, L.comb_ent, L.total,
+                     L.n_segs, L.n_items, L.n_ctas, L.n_page_ids, L.n_comb_keys, L.n_comb_ent,
+                     p.unique_tokens, p.logical_tokens, (int64_t)sizeof(DecodeSeg)};
+    std::memcpy(layout_out, v, sizeof v);
+    if (buf) {
+        if (buf_bytes < L.total) return kInvalidArg;
+        plan_serialize(p, L, buf);
+    }
+    return kOk;
+}
+
+}  // extern "C"

@@ -1,0 +1,664 @@
+// libsq C ABI: validation, transactional host state, plan upload, launches.
+// See include/sq.h for the contract of every call.
+#include "sq.h"
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cstring>
+#include <memory>
+#include <new>
+#include <unordered_map>
+#include <vector>
+
+#include "../host/core.hpp"
+#include "../kernels/launch.hpp"
+
+using namespace sq;
+
+namespace {
+
+constexpr int kPlanCacheEntries = 8;
+constexpr int kUploadSlots = 8;
+
+struct PlanEntry {
+    bool valid = false;
+    int32_t n_ctas = 0;
+    std::vector<int32_t> handles;
+    std::vector<uint64_t> versions;
+    DecodePlanLayout lay{};
+    int64_t unique_tokens = 0, logical_tokens = 0;
+    uint8_t* d_plan = nullptr;
+    size_t plan_cap = 0;
+    float* d_part = nullptr;
+    size_t part_cap = 0;
+    cudaEvent_t ev = nullptr;   // recorded after the last launch that used it
+    bool ev_recorded = false;
+    uint64_t last_use = 0;
+};
+
+struct UploadSlot {
+    uint8_t* d = nullptr;
+    size_t cap = 0;
+    cudaEvent_t ev = nullptr;
+    bool ev_recorded = false;
+};
+
+}  // namespace
+
+struct sq_cache {
+    Geometry g;
+    std::unique_ptr<HostCache> host;
+    int device = 0;
+    int num_sms = 0;
+    int decode_ctas = 0;
+    int evict_slots = 0;
+    __nv_bfloat16* pool = nullptr;
+    bool own_pool = false;
+    size_t pool_bytes = 0;
+    CUtensorMap tmap;
+    int* d_err = nullptr;
+    PlanEntry plans[kPlanCacheEntries];
+    uint64_t use_clock = 0;
+    UploadSlot slots[kUploadSlots];
+    int next_slot = 0;
+    std::vector<uint8_t> staging;
+    // pages freed by work on a stream become reusable elsewhere only after
+    // that work: the stream that freed each free page, and one event per
+    // stream recorded after its latest freeing operation
+    std::vector<void*> freed_on;
+    std::vector<uint8_t> fenced;
+    std::unordered_map<void*, cudaEvent_t> free_event;
+    sq_stats_t stats;
+};
+
+namespace {
+
+inline cudaStream_t as_stream(void* s) { return reinterpret_cast<cudaStream_t>(s); }
+
+int cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return SQ_OK;
+    if (e == cudaErrorMemoryAllocation) return SQ_ERR_NO_MEMORY;
+    return SQ_ERR_CUDA;
+}
+
+int geometry_from(const sq_config* cfg, Geometry* g) {
+    if (!cfg) return SQ_ERR_INVALID_ARG;
+    g->L = cfg->num_layers;
+    g->Hq = cfg->num_q_heads;
+    g->Hkv = cfg->num_kv_heads;
+    g->D = cfg->head_dim;
+    g->P = cfg->page_size;
+    g->num_pages = cfg->num_pages;
+    g->max_seqs = cfg->max_seqs;
+    g->max_pages_per_seq = cfg->max_pages_per_seq;
+    return check_geometry(*g);
+}
+
+size_t pool_bytes_of(const Geometry& g) {
+    return (size_t)g.L * g.num_pages * 2 * g.Hkv * g.P * g.D * sizeof(__nv_bfloat16);
+}
+
+int make_tensor_map(sq_cache* c) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !fn)
+        return SQ_ERR_CUDA;
+    auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    const Geometry& g = c->g;
+    // dims, innermost first: head dim, row within a (layer, page) block
+    // ((kv * Hkv + head) * P + slot), page, layer
+    cuuint64_t dims[4] = {(cuuint64_t)g.D, (cuuint64_t)2 * g.Hkv * g.P, (cuuint64_t)g.num_pages,
+                          (cuuint64_t)g.L};
+    cuuint64_t strides[3] = {(cuuint64_t)g.D * 2, (cuuint64_t)2 * g.Hkv * g.P * g.D * 2,
+                             (cuuint64_t)g.num_pages * 2 * g.Hkv * g.P * g.D * 2};
+    cuuint32_t box[4] = {64, (cuuint32_t)std::min(g.P, kStageTokens), 1, 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    CUresult r = encode(&c->tmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, c->pool, dims, strides, box,
+                        estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? SQ_OK : SQ_ERR_UNSUPPORTED;
+}
+
+// Before `stream` writes pages taken from the free list, wait for the work
+// that freed them on other streams.
+int fence_taken_pages(sq_cache* c, const std::vector<int32_t>& taken, void* stream) {
+    void* waited[8];
+    int n_waited = 0;
+    for (int32_t p : taken) {
+        if (!c->fenced[p]) continue;
+        c->fenced[p] = 0;
+        void* s = c->freed_on[p];
+        if (s == stream) continue;
+        bool seen = false;
+        for (int i = 0; i < n_waited; ++i) seen |= waited[i] == s;
+        if (seen) continue;
+        auto it = c->free_event.find(s);
+        if (it == c->free_event.end()) continue;
+        cudaError_t e = cudaStreamWaitEvent(as_stream(stream), it->second, 0);
+        if (e != cudaSuccess) return cuda_status(e);
+        if (n_waited < 8) waited[n_waited++] = s;
+    }
+    return SQ_OK;
+}
+
+// Marks pages freed by the work enqueued on `stream` so far.
+int record_freed(sq_cache* c, const std::vector<int32_t>& freed, void* stream) {
+    if (freed.empty()) return SQ_OK;
+    auto it = c->free_event.find(stream);
+    if (it == c->free_event.end()) {
+        cudaEvent_t ev;
+        cudaError_t e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+        if (e != cudaSuccess) return cuda_status(e);
+        it = c->free_event.emplace(stream, ev).first;
+    }
+    cudaError_t e = cudaEventRecord(it->second, as_stream(stream));
+    if (e != cudaSuccess) return cuda_status(e);
+    for (int32_t p : freed) {
+        c->freed_on[p] = stream;
+        c->fenced[p] = 1;
+    }
+    return SQ_OK;
+}
+
+int upload(sq_cache* c, UploadSlot& s, const void* src, size_t bytes, void* stream) {
+    if (bytes > s.cap) {
+        if (s.d) {
+            if (s.ev_recorded) cudaEventSynchronize(s.ev);
+            cudaFree(s.d);
+            s.d = nullptr;
+            s.cap = 0;
+        }
+        size_t cap = std::max<size_t>(bytes, 4096);
+        cudaError_t e = cudaMalloc(&s.d, cap);
+        if (e != cudaSuccess) return cuda_status(e);
+        s.cap = cap;
+        s.ev_recorded = false;
+    }
+    if (s.ev_recorded) {
+        cudaError_t e = cudaStreamWaitEvent(as_stream(stream), s.ev, 0);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    // pageable source: staged by the driver before the call returns, so the
+    // host buffer may be reused at once
+    cudaError_t e = cudaMemcpyAsync(s.d, src, bytes, cudaMemcpyHostToDevice, as_stream(stream));
+    return cuda_status(e);
+}
+
+void free_entry(PlanEntry& p) {
+    if (p.d_plan) cudaFree(p.d_plan);
+    if (p.d_part) cudaFree(p.d_part);
+    if (p.ev) cudaEventDestroy(p.ev);
+    p = PlanEntry();
+}
+
+int choose_col_split(const sq_cache* c) {
+    const int64_t planes = (int64_t)c->g.L * 2 * c->g.Hkv;
+    const int row_bytes = c->g.D * 2;
+    for (int cs = 4; cs >= 2; cs >>= 1)
+        if (row_bytes / cs >= 64 && planes * cs <= c->evict_slots) return cs;
+    return 1;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* sq_strerror(int code) {
+    switch (code) {
+        case SQ_OK: return "SQ_OK";
+        case SQ_ERR_INVALID_ARG: return "SQ_ERR_INVALID_ARG";
+        case SQ_ERR_BAD_HANDLE: return "SQ_ERR_BAD_HANDLE";
+        case SQ_ERR_NO_PAGES: return "SQ_ERR_NO_PAGES";
+        case SQ_ERR_CAPACITY: return "SQ_ERR_CAPACITY";
+        case SQ_ERR_CUDA: return "SQ_ERR_CUDA";
+        case SQ_ERR_DEVICE: return "SQ_ERR_DEVICE";
+        case SQ_ERR_DEVICE_TIMEOUT: return "SQ_ERR_DEVICE_TIMEOUT";
+        case SQ_ERR_UNSUPPORTED: return "SQ_ERR_UNSUPPORTED";
+        case SQ_ERR_NO_MEMORY: return "SQ_ERR_NO_MEMORY";
+        default: return "SQ_ERR_UNKNOWN";
+    }
+}
+
+size_t sq_pool_bytes(const sq_config* cfg) {
+    Geometry g;
+    if (geometry_from(cfg, &g) != SQ_OK) return 0;
+    return pool_bytes_of(g);
+}
+
+int sq_cache_create(const sq_config* cfg, sq_cache** out) {
+    if (!out) return SQ_ERR_INVALID_ARG;
+    *out = nullptr;
+    Geometry g;
+    int rc = geometry_from(cfg, &g);
+    if (rc != SQ_OK) return rc;
+    if (cfg->decode_ctas < 0) return SQ_ERR_INVALID_ARG;
+    if (cfg->kv_pool && (reinterpret_cast<uintptr_t>(cfg->kv_pool) & 255)) return SQ_ERR_INVALID_ARG;
+    std::unique_ptr<sq_cache> c(new (std::nothrow) sq_cache());
+    if (!c) return SQ_ERR_NO_MEMORY;
+    c->g = g;
+    c->host.reset(new (std::nothrow) HostCache(g));
+    if (!c->host) return SQ_ERR_NO_MEMORY;
+    c->freed_on.assign(g.num_pages, nullptr);
+    c->fenced.assign(g.num_pages, 0);
+    std::memset(&c->stats, 0, sizeof c->stats);
+    cudaError_t e = cudaGetDevice(&c->device);
+    if (e != cudaSuccess) return cuda_status(e);
+    e = cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device);
+    if (e != cudaSuccess) return cuda_status(e);
+    e = decode_prepare(g.D);
+    if (e != cudaSuccess) return cuda_status(e);
+    c->decode_ctas = cfg->decode_ctas > 0 ? cfg->decode_ctas : c->num_sms * decode_ctas_per_sm(g.D);
+    c->evict_slots = c->num_sms * evict_ctas_per_sm();
+    c->pool_bytes = pool_bytes_of(g);
+    if (cfg->kv_pool) {
+        c->pool = reinterpret_cast<__nv_bfloat16*>(cfg->kv_pool);
+    } else {
+        e = cudaMalloc(&c->pool, c->pool_bytes);
+        if (e != cudaSuccess) return cuda_status(e);
+        c->own_pool = true;
+        e = cudaMemset(c->pool, 0, c->pool_bytes);
+        if (e != cudaSuccess) {
+            cudaFree(c->pool);
+            return cuda_status(e);
+        }
+    }
+    auto fail = [&](int code) {
+        if (c->own_pool) cudaFree(c->pool);
+        if (c->d_err) cudaFree(c->d_err);
+        return code;
+    };
+    e = cudaMalloc(&c->d_err, sizeof(int));
+    if (e != cudaSuccess) return fail(cuda_status(e));
+    e = cudaMemset(c->d_err, 0, sizeof(int));
+    if (e != cudaSuccess) return fail(cuda_status(e));
+    rc = make_tensor_map(c.get());
+    if (rc != SQ_OK) return fail(rc);
+    for (auto& s : c->slots) {
+        e = cudaEventCreateWithFlags(&s.ev, cudaEventDisableTiming);
+        if (e != cudaSuccess) return fail(cuda_status(e));
+    }
+    e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return fail(cuda_status(e));
+    *out = c.release();
+    return SQ_OK;
+}
+
+int sq_cache_destroy(sq_cache* c) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    cudaDeviceSynchronize();
+    for (auto& p : c->plans) free_entry(p);
+    for (auto& s : c->slots) {
+        if (s.d) cudaFree(s.d);
+        if (s.ev) cudaEventDestroy(s.ev);
+    }
+    for (auto& kv : c->free_event) cudaEventDestroy(kv.second);
+    if (c->d_err) cudaFree(c->d_err);
+    if (c->own_pool) cudaFree(c->pool);
+    delete c;
+    return SQ_OK;
+}
+
+int sq_seq_new(sq_cache* c, sq_seq* out) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    if (!out) return SQ_ERR_INVALID_ARG;
+    return c->host->seq_new(out);
+}
+
+int sq_fork_aux(sq_cache* c, sq_seq parent, sq_seq* child_out) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    if (!child_out) return SQ_ERR_INVALID_ARG;
+    return c->host->fork(parent, child_out);
+}
+
+int sq_append_kv(sq_cache* c, sq_seq seq, int32_t n_tokens, const void* k, const void* v,
+                 void* stream) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    if (!c->host->seq(seq)) return SQ_ERR_BAD_HANDLE;
+    if (n_tokens < 0) return SQ_ERR_INVALID_ARG;
+    if (n_tokens == 0) return SQ_OK;
+    if (!k || !v || (reinterpret_cast<uintptr_t>(k) & 15) || (reinterpret_cast<uintptr_t>(v) & 15))
+        return SQ_ERR_INVALID_ARG;
+    AppendPlan plan;
+    int rc = c->host->append(seq, n_tokens, &plan);
+    if (rc != SQ_OK) return rc;
+    const Geometry& g = c->g;
+    cudaStream_t st = as_stream(stream);
+    auto undo = [&](int code) {
+        c->host->undo_append(seq, plan);
+        return code;
+    };
+    rc = fence_taken_pages(c, plan.taken, stream);
+    if (rc != SQ_OK) return undo(rc);
+    if (plan.cow) {
+        CowArgs ca;
+        ca.pool = c->pool;
+        ca.num_pages = g.num_pages;
+        ca.L = g.L; ca.Hkv = g.Hkv; ca.P = g.P; ca.D = g.D;
+        ca.src_page = plan.cow_old;
+        ca.dst_page = plan.cow_new;
+        ca.rows = plan.cow_rows;
+        ca.err = c->d_err;
+        cudaError_t e = launch_cow_copy(ca, c->num_sms, st);
+        if (e != cudaSuccess) return undo(cuda_status(e));
+    }
+    const int64_t end = (int64_t)plan.n0 + plan.n_new;
+    for (size_t b = 0; b < plan.pages.size(); b += kAppendMaxPages) {
+        AppendArgs a;
+        a.pool = c->pool;
+        a.k = reinterpret_cast<const __nv_bfloat16*>(k);
+        a.v = reinterpret_cast<const __nv_bfloat16*>(v);
+        a.num_pages = g.num_pages;
+        a.L = g.L; a.Hkv = g.Hkv; a.P = g.P; a.D = g.D;
+        a.n_total = n_tokens;
+        a.page_index0 = plan.first_page_index + (int32_t)b;
+        a.n_pages = (int32_t)std::min<size_t>(kAppendMaxPages, plan.pages.size() - b);
+        for (int i = 0; i < a.n_pages; ++i) a.pages[i] = plan.pages[b + i];
+        const int64_t pb = std::max<int64_t>(plan.n0, (int64_t)a.page_index0 * g.P);
+        const int64_t pe = std::min<int64_t>(end, (int64_t)(a.page_index0 + a.n_pages) * g.P);
+        if (pe <= pb) continue;
+        a.pos0 = (int32_t)pb;
+        a.tok_begin = (int32_t)(pb - plan.n0);
+        a.n_tok = (int32_t)(pe - pb);
+        a.err = c->d_err;
+        cudaError_t e = launch_append(a, c->num_sms, st);
+        if (e != cudaSuccess) return undo(cuda_status(e));
+    }
+    c->host->seq_mut(seq)->last_stream = stream;
+    c->stats.appended_tokens += n_tokens;
+    if (plan.cow) c->stats.cow_pages += 1;
+    return SQ_OK;
+}
+
+int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t layer,
+                        const void* q, void* out, int32_t out_dtype, float sm_scale,
+                        void* stream) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    const Geometry& g = c->g;
+    if (!seqs || n_seqs < 1 || n_seqs > g.max_seqs || !q || !out) return SQ_ERR_INVALID_ARG;
+    if (layer < 0 || layer >= g.L) return SQ_ERR_INVALID_ARG;
+    if (out_dtype != SQ_OUT_BF16 && out_dtype != SQ_OUT_F32) return SQ_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(q) & 15) || (reinterpret_cast<uintptr_t>(out) & 15))
+        return SQ_ERR_INVALID_ARG;
+    if (!(sm_scale == sm_scale)) return SQ_ERR_INVALID_ARG;
+    for (int32_t i = 0; i < n_seqs; ++i) {
+        const Seq* s = c->host->seq(seqs[i]);
+        if (!s) return SQ_ERR_BAD_HANDLE;
+        if (s->n < 1) return SQ_ERR_INVALID_ARG;
+    }
+    // plan cache lookup: same handles, same versions, same CTA count
+    PlanEntry* hit = nullptr;
+    for (auto& p : c->plans) {
+        if (!p.valid || p.n_ctas != c->decode_ctas || (int32_t)p.handles.size() != n_seqs) continue;
+        bool same = true;
+        for (int32_t i = 0; i < n_seqs && same; ++i)
+            same = p.handles[i] == seqs[i] && p.versions[i] == c->host->seq(seqs[i])->version;
+        if (same) {
+            hit = &p;
+            break;
+        }
+    }
+    cudaStream_t st = as_stream(stream);
+    cudaError_t e;
+    if (!hit) {
+        DecodePlanHost plan;
+        int rc = plan_decode(*c->host, seqs, n_seqs, c->decode_ctas, &plan);
+        if (rc != SQ_OK) return rc;
+        DecodePlanLayout lay = plan_layout(plan, n_seqs, g.Hkv);
+        // least recently used entry
+        PlanEntry* victim = &c->plans[0];
+        for (auto& p : c->plans)
+            if (!p.valid || p.last_use < victim->last_use) victim = &p;
+        const size_t part_bytes = (size_t)decode_partial_bytes(lay.n_items, g.D);
+        if ((size_t)lay.total > victim->plan_cap || part_bytes > victim->part_cap) {
+            if (victim->ev_recorded) cudaEventSynchronize(victim->ev);
+            if ((size_t)lay.total > victim->plan_cap) {
+                if (victim->d_plan) cudaFree(victim->d_plan);
+                victim->d_plan = nullptr;
+                victim->plan_cap = 0;
+                size_t cap = (size_t)lay.total * 5 / 4 + 4096;
+                e = cudaMalloc(&victim->d_plan, cap);
+                if (e != cudaSuccess) { victim->valid = false; return cuda_status(e); }
+                victim->plan_cap = cap;
+            }
+            if (part_bytes > victim->part_cap) {
+                if (victim->d_part) cudaFree(victim->d_part);
+                victim->d_part = nullptr;
+                victim->part_cap = 0;
+                size_t cap = part_bytes * 5 / 4 + 4096;
+                e = cudaMalloc(&victim->d_part, cap);
+                if (e != cudaSuccess) { victim->valid = false; return cuda_status(e); }
+                victim->part_cap = cap;
+            }
+        }
+        if (!victim->ev) {
+            e = cudaEventCreateWithFlags(&victim->ev, cudaEventDisableTiming);
+            if (e != cudaSuccess) return cuda_status(e);
+        }
+        if (victim->ev_recorded) {
+            e = cudaStreamWaitEvent(st, victim->ev, 0);
+            if (e != cudaSuccess) return cuda_status(e);
+        }
+        if (c->staging.size() < (size_t)lay.total) c->staging.resize(lay.total);
+        plan_serialize(plan, lay, c->staging.data());
+        e = cudaMemcpyAsync(victim->d_plan, c->staging.data(), lay.total, cudaMemcpyHostToDevice, st);
+        if (e != cudaSuccess) { victim->valid = false; return cuda_status(e); }
+        victim->valid = true;
+        victim->n_ctas = c->decode_ctas;
+        victim->handles.assign(seqs, seqs + n_seqs);
+        victim->versions.resize(n_seqs);
+        for (int32_t i = 0; i < n_seqs; ++i) victim->versions[i] = c->host->seq(seqs[i])->version;
+        victim->lay = lay;
+        victim->unique_tokens = plan.unique_tokens;
+        victim->logical_tokens = plan.logical_tokens;
+        hit = victim;
+    } else if (hit->ev_recorded) {
+        e = cudaStreamWaitEvent(st, hit->ev, 0);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    hit->last_use = ++c->use_clock;
+    const DecodePlanLayout& L = hit->lay;
+    float* part_o = hit->d_part;
+    float* part_ml = part_o + (size_t)L.n_items * kDecodeConsumerWarps * kRowsPerTile * g.D;
+
+    DecodeArgs a;
+    a.segs = reinterpret_cast<const DecodeSeg*>(hit->d_plan + L.segs);
+    a.items = reinterpret_cast<const DecodeItem*>(hit->d_plan + L.items);
+    a.cta_begin = reinterpret_cast<const int32_t*>(hit->d_plan + L.cta_begin);
+    a.page_ids = reinterpret_cast<const int32_t*>(hit->d_plan + L.page_ids);
+    a.q = reinterpret_cast<const __nv_bfloat16*>(q);
+    a.part_o = part_o;
+    a.part_ml = part_ml;
+    a.layer = layer;
+    a.Hq = g.Hq;
+    a.Hkv = g.Hkv;
+    a.G = g.G();
+    a.P = g.P;
+    a.num_pages = g.num_pages;
+    a.scale_log2 = sm_scale * 1.4426950408889634f;
+    a.err = c->d_err;
+    e = launch_decode(c->tmap, a, L.n_ctas, g.D, st);
+    if (e != cudaSuccess) { hit->valid = false; return cuda_status(e); }
+
+    CombineArgs ca;
+    ca.comb_off = reinterpret_cast<const int32_t*>(hit->d_plan + L.comb_off);
+    ca.comb_ent = reinterpret_cast<const CombineEnt*>(hit->d_plan + L.comb_ent);
+    ca.part_o = part_o;
+    ca.part_ml = part_ml;
+    ca.out = out;
+    ca.out_f32 = out_dtype == SQ_OUT_F32;
+    ca.n_seqs = n_seqs;
+    ca.Hq = g.Hq;
+    ca.Hkv = g.Hkv;
+    ca.G = g.G();
+    e = launch_combine(ca, g.D, st);
+    if (e != cudaSuccess) { hit->valid = false; return cuda_status(e); }
+    e = cudaEventRecord(hit->ev, st);
+    if (e != cudaSuccess) return cuda_status(e);
+    hit->ev_recorded = true;
+    for (int32_t i = 0; i < n_seqs; ++i) c->host->seq_mut(seqs[i])->last_stream = stream;
+    c->stats.decode_calls += 1;
+    c->stats.decode_logical_bytes += hit->logical_tokens * g.token_layer_bytes();
+    c->stats.decode_unique_bytes += hit->unique_tokens * g.token_layer_bytes();
+    return SQ_OK;
+}
+
+int sq_evict_spans(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_spans, void* stream) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    if (!c->host->seq(seq)) return SQ_ERR_BAD_HANDLE;
+    if (n_spans < 0 || (n_spans > 0 && !spans)) return SQ_ERR_INVALID_ARG;
+    if (n_spans == 0) return SQ_OK;
+    std::vector<int32_t> a(n_spans), b(n_spans);
+    for (int32_t i = 0; i < n_spans; ++i) {
+        a[i] = spans[i].start;
+        b[i] = spans[i].end;
+    }
+    EvictPlan plan;
+    int rc = c->host->evict(seq, a.data(), b.data(), n_spans, &plan);
+    if (rc != SQ_OK) return rc;
+    const Geometry& g = c->g;
+    cudaStream_t st = as_stream(stream);
+    auto undo = [&](int code) {
+        c->host->undo_evict(seq, plan);
+        return code;
+    };
+    rc = fence_taken_pages(c, plan.cow_pages, stream);
+    if (rc != SQ_OK) return undo(rc);
+    if (plan.first_row < plan.n_new) {
+        // upload: old page table, new page table, run starts (dst, src)
+        const size_t n_old = plan.old_pages.size(), n_new = plan.new_pages.size();
+        const size_t n_runs = plan.run_dst.size();
+        std::vector<int32_t> buf(n_old + n_new + 2 * n_runs);
+        std::copy(plan.old_pages.begin(), plan.old_pages.end(), buf.begin());
+        std::copy(plan.new_pages.begin(), plan.new_pages.end(), buf.begin() + n_old);
+        std::copy(plan.run_dst.begin(), plan.run_dst.end(), buf.begin() + n_old + n_new);
+        std::copy(plan.run_src.begin(), plan.run_src.end(), buf.begin() + n_old + n_new + n_runs);
+        UploadSlot& s = c->slots[c->next_slot];
+        c->next_slot = (c->next_slot + 1) % kUploadSlots;
+        rc = upload(c, s, buf.data(), buf.size() * sizeof(int32_t), stream);
+        if (rc != SQ_OK) return undo(rc);
+        const int32_t* d = reinterpret_cast<const int32_t*>(s.d);
+        EvictArgs ea;
+        ea.pool = c->pool;
+        ea.num_pages = g.num_pages;
+        ea.L = g.L; ea.Hkv = g.Hkv; ea.P = g.P; ea.D = g.D;
+        ea.old_pt = d;
+        ea.new_pt = d + n_old;
+        ea.run_dst = d + n_old + n_new;
+        ea.run_src = d + n_old + n_new + n_runs;
+        ea.n_old_pages = (int32_t)n_old;
+        ea.n_new_pages = (int32_t)n_new;
+        ea.n_runs = (int32_t)n_runs;
+        ea.n_new = plan.n_new;
+        ea.first_row = plan.first_row;
+        ea.col_split = choose_col_split(c);
+        ea.err = c->d_err;
+        cudaError_t e = launch_evict(ea, st);
+        if (e != cudaSuccess) return undo(cuda_status(e));
+        e = cudaEventRecord(s.ev, st);
+        if (e != cudaSuccess) return cuda_status(e);
+        s.ev_recorded = true;
+    }
+    rc = record_freed(c, plan.freed, stream);
+    if (rc != SQ_OK) return rc;
+    c->host->seq_mut(seq)->last_stream = stream;
+    c->stats.evict_calls += 1;
+    c->stats.evicted_tokens += plan.evicted;
+    c->stats.evict_moved_rows += plan.moved_rows;
+    c->stats.evict_bytes += 2 * plan.moved_rows * g.L * g.token_layer_bytes();
+    c->stats.cow_pages += (int64_t)plan.cow_pages.size();
+    return SQ_OK;
+}
+
+int sq_release(sq_cache* c, sq_seq seq, void* stream) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    const Seq* s = c->host->seq(seq);
+    if (!s) return SQ_ERR_BAD_HANDLE;
+    void* last = s->last_stream;
+    if (last && last != stream) {
+        // make `stream` follow the sequence's last work before the pages go
+        cudaEvent_t ev;
+        cudaError_t e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+        if (e != cudaSuccess) return cuda_status(e);
+        e = cudaEventRecord(ev, as_stream(last));
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(as_stream(stream), ev, 0);
+        cudaEventDestroy(ev);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    std::vector<int32_t> freed;
+    int rc = c->host->release(seq, &freed);
+    if (rc != SQ_OK) return rc;
+    return record_freed(c, freed, stream);
+}
+
+int sq_seq_info(sq_cache* c, sq_seq seq, int32_t* n_tokens, int32_t* n_pages) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    const Seq* s = c->host->seq(seq);
+    if (!s) return SQ_ERR_BAD_HANDLE;
+    if (n_tokens) *n_tokens = s->n;
+    if (n_pages) *n_pages = (int32_t)s->pages.size();
+    return SQ_OK;
+}
+
+int sq_get_page_table(sq_cache* c, sq_seq seq, int32_t* host_out, int32_t cap, int32_t* n_out) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    const Seq* s = c->host->seq(seq);
+    if (!s) return SQ_ERR_BAD_HANDLE;
+    const int32_t n = (int32_t)s->pages.size();
+    if (n_out) *n_out = n;
+    if (n > 0 && (!host_out || cap < n)) return SQ_ERR_INVALID_ARG;
+    if (n > 0) std::memcpy(host_out, s->pages.data(), sizeof(int32_t) * n);
+    return SQ_OK;
+}
+
+int sq_page_refcount(sq_cache* c, int32_t page, int32_t* out) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    if (!out || page < 0 || page >= c->g.num_pages) return SQ_ERR_INVALID_ARG;
+    *out = c->host->alloc().refcount(page);
+    return SQ_OK;
+}
+
+int sq_free_pages(sq_cache* c, int32_t* out) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    if (!out) return SQ_ERR_INVALID_ARG;
+    *out = c->host->alloc().free_count();
+    return SQ_OK;
+}
+
+int sq_pool_ptr(sq_cache* c, void** out) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    if (!out) return SQ_ERR_INVALID_ARG;
+    *out = c->pool;
+    return SQ_OK;
+}
+
+int sq_stats(sq_cache* c, sq_stats_t* out) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    if (!out) return SQ_ERR_INVALID_ARG;
+    *out = c->stats;
+    out->live_pages = c->host->live_pages();
+    out->peak_live_pages = c->host->peak_live_pages();
+    return SQ_OK;
+}
+
+int sq_sync_status(sq_cache* c, void* stream) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    cudaError_t e = cudaStreamSynchronize(as_stream(stream));
+    if (e != cudaSuccess) return SQ_ERR_CUDA;
+    int err = 0;
+    e = cudaMemcpy(&err, c->d_err, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return SQ_ERR_CUDA;
+    if (err) {
+        e = cudaMemset(c->d_err, 0, sizeof(int));
+        if (e != cudaSuccess) return SQ_ERR_CUDA;
+    }
+    if (err & 2) return SQ_ERR_DEVICE_TIMEOUT;
+    if (err & 1) return SQ_ERR_DEVICE;
+    return SQ_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,480 @@
+// Host-side cache state and planners.  See core.hpp for the rules.
+#include "core.hpp"
+
+#include <algorithm>
+#include <cstring>
+#include <unordered_map>
+
+namespace sq {
+
+static inline int32_t ceil_div(int64_t a, int64_t b) { return (int32_t)((a + b - 1) / b); }
+
+int check_geometry(const Geometry& g) {
+    if (g.L < 1 || g.Hq < 1 || g.Hkv < 1 || g.D < 1 || g.P < 1 ||
+        g.num_pages < 1 || g.max_seqs < 1 || g.max_pages_per_seq < 1)
+        return kInvalidArg;
+    if (g.Hq % g.Hkv != 0) return kInvalidArg;
+    if (g.G() > kRowsPerTile) return kUnsupported;
+    if (g.D != 64 && g.D != 128) return kUnsupported;
+    if (g.P < 8 || g.P > 256 || (g.P & (g.P - 1)) != 0) return kUnsupported;
+    if (g.max_seqs >= (1 << 20)) return kUnsupported;
+    // logical positions are int32
+    if ((int64_t)g.max_pages_per_seq * g.P >= (1LL << 31)) return kUnsupported;
+    return kOk;
+}
+
+// ---------------------------------------------------------------------------
+PageAllocator::PageAllocator(int32_t n)
+    : ref_(n, 0), free_bits_((n + 63) / 64, 0), free_count_(n) {
+    for (int32_t i = 0; i < n; ++i) free_bits_[i >> 6] |= 1ULL << (i & 63);
+}
+
+int32_t PageAllocator::lowest_free() const {
+    const int32_t words = (int32_t)free_bits_.size();
+    for (int32_t w = hint_; w < words; ++w) {
+        if (free_bits_[w]) {
+            hint_ = w;
+            return w * 64 + __builtin_ctzll(free_bits_[w]);
+        }
+    }
+    hint_ = words;
+    return -1;
+}
+
+void PageAllocator::take(int32_t p) {
+    ref_[p] = 1;
+    free_bits_[p >> 6] &= ~(1ULL << (p & 63));
+    --free_count_;
+}
+
+bool PageAllocator::drop_ref(int32_t p) {
+    if (--ref_[p] == 0) {
+        free_bits_[p >> 6] |= 1ULL << (p & 63);
+        ++free_count_;
+        if ((p >> 6) < hint_) hint_ = p >> 6;
+        return true;
+    }
+    return false;
+}
+
+// ---------------------------------------------------------------------------
+static uint64_t g_version_counter = 1;
+
+HostCache::HostCache(const Geometry& g) : g_(g), alloc_(g.num_pages), seqs_(g.max_seqs) {
+    free_slots_.reserve(g.max_seqs);
+    for (int32_t s = g.max_seqs - 1; s >= 0; --s) free_slots_.push_back(s);
+}
+
+int32_t HostCache::take_lowest() {
+    int32_t p = alloc_.lowest_free();
+    alloc_.take(p);
+    int64_t live = live_pages();
+    if (live > peak_live_) peak_live_ = live;
+    return p;
+}
+
+const Seq* HostCache::seq(int32_t h) const {
+    if (h <= 0) return nullptr;
+    int32_t slot = h & 0xFFFFF;
+    uint32_t gen = (uint32_t)h >> 20;
+    if (slot >= g_.max_seqs) return nullptr;
+    const Seq& s = seqs_[slot];
+    if (!s.live || s.gen != gen) return nullptr;
+    return &s;
+}
+
+Seq* HostCache::seq_mut(int32_t h) { return const_cast<Seq*>(seq(h)); }
+
+int HostCache::seq_new(int32_t* handle) {
+    if (free_slots_.empty()) return kCapacity;
+    int32_t slot = free_slots_.back();
+    free_slots_.pop_back();
+    Seq& s = seqs_[slot];
+    s.live = true;
+    s.gen = (s.gen % 2047) + 1;  // 1 .. 2047: handles stay positive
+    s.n = 0;
+    s.pages.clear();
+    s.version = g_version_counter++;
+    s.last_stream = nullptr;
+    *handle = (int32_t)((s.gen << 20) | (uint32_t)slot);
+    return kOk;
+}
+
+int HostCache::fork(int32_t parent, int32_t* child) {
+    const Seq* ps = seq(parent);
+    if (!ps) return kBadHandle;
+    std::vector<int32_t> pages = ps->pages;
+    int32_t n = ps->n;
+    void* st = ps->last_stream;
+    int rc = seq_new(child);
+    if (rc != kOk) return rc;
+    Seq* cs = seq_mut(*child);
+    cs->pages = std::move(pages);
+    cs->n = n;
+    cs->last_stream = st;
+    for (int32_t p : cs->pages) alloc_.add_ref(p);
+    return kOk;
+}
+
+int HostCache::append(int32_t h, int32_t n_new, AppendPlan* plan) {
+    *plan = AppendPlan();
+    if (n_new < 0) return kInvalidArg;
+    Seq* s = seq_mut(h);
+    if (!s) return kBadHandle;
+    const int32_t P = g_.P;
+    const int32_t n = s->n;
+    plan->n0 = n;
+    plan->n_new = n_new;
+    if (n_new == 0) return kOk;
+    if ((int64_t)n + n_new >= (1LL << 31)) return kCapacity;
+    const int32_t new_np = ceil_div((int64_t)n + n_new, P);
+    if (new_np > g_.max_pages_per_seq) return kCapacity;
+    const bool cow = (n % P != 0) && alloc_.refcount(s->pages.back()) > 1;
+    const int32_t need = (cow ? 1 : 0) + new_np - (int32_t)s->pages.size();
+    if (need > alloc_.free_count()) return kNoPages;
+
+    if (cow) {
+        int32_t old = s->pages.back();
+        int32_t fresh = take_lowest();
+        alloc_.drop_ref(old);  // was > 1: stays held by the other sequences
+        s->pages.back() = fresh;
+        plan->cow = true;
+        plan->cow_old = old;
+        plan->cow_new = fresh;
+        plan->cow_rows = n % P;
+        plan->taken.push_back(fresh);
+    }
+    while ((int32_t)s->pages.size() < new_np) {
+        int32_t p = take_lowest();
+        s->pages.push_back(p);
+        plan->taken.push_back(p);
+    }
+    plan->first_page_index = n / P;
+    plan->pages.assign(s->pages.begin() + n / P, s->pages.end());
+    s->n = n + n_new;
+    s->version = g_version_counter++;
+    return kOk;
+}
+
+void HostCache::undo_append(int32_t h, const AppendPlan& plan) {
+    Seq* s = seq_mut(h);
+    if (!s || plan.n_new == 0) return;
+    const int32_t old_np = ceil_div(plan.n0, g_.P);
+    while ((int32_t)s->pages.size() > old_np) {
+        alloc_.drop_ref(s->pages.back());
+        s->pages.pop_back();
+    }
+    if (plan.cow) {
+        alloc_.drop_ref(plan.cow_new);
+        alloc_.add_ref(plan.cow_old);
+        s->pages.back() = plan.cow_old;
+    }
+    s->n = plan.n0;
+    s->version = g_version_counter++;
+}
+
+int HostCache::evict(int32_t h, const int32_t* starts, const int32_t* ends,
+                     int32_t n_spans, EvictPlan* plan) {
+    *plan = EvictPlan();
+    Seq* s = seq_mut(h);
+    if (!s) return kBadHandle;
+    if (n_spans < 0) return kInvalidArg;
+    const int32_t n = s->n;
+    const int32_t P = g_.P;
+    plan->n_old = n;
+    plan->n_new = n;
+    plan->first_row = n;
+    plan->old_pages = s->pages;
+    plan->new_pages = s->pages;
+    if (n_spans == 0) return kOk;
+    if (!starts || !ends) return kInvalidArg;
+
+    std::vector<std::pair<int32_t, int32_t>> sp(n_spans);
+    for (int32_t i = 0; i < n_spans; ++i) sp[i] = {starts[i], ends[i]};
+    std::sort(sp.begin(), sp.end());
+    int32_t prev_end = 0;
+    int64_t removed = 0;
+    for (auto& ab : sp) {
+        if (ab.first < 0 || ab.second > n || ab.first >= ab.second) return kInvalidArg;
+        if (ab.first < prev_end) return kInvalidArg;
+        prev_end = ab.second;
+        removed += ab.second - ab.first;
+    }
+    // kept runs
+    int32_t cur = 0, dst = 0;
+    for (auto& ab : sp) {
+        if (ab.first > cur) {
+            plan->run_dst.push_back(dst);
+            plan->run_src.push_back(cur);
+            plan->run_len.push_back(ab.first - cur);
+            dst += ab.first - cur;
+        }
+        cur = ab.second;
+    }
+    if (n > cur) {
+        plan->run_dst.push_back(dst);
+        plan->run_src.push_back(cur);
+        plan->run_len.push_back(n - cur);
+        dst += n - cur;
+    }
+    const int32_t n2 = (int32_t)(n - removed);
+    const int32_t new_np = ceil_div(n2, P);
+    const int32_t a0 = sp[0].first;
+    const int32_t qc = a0 / P;
+    const bool any_change = n2 > a0;  // some kept row moves
+    // copy-on-write needs
+    int32_t need = 0;
+    if (any_change)
+        for (int32_t q = qc; q < new_np; ++q)
+            if (alloc_.refcount(s->pages[q]) > 1) ++need;
+    if (need > alloc_.free_count()) return kNoPages;
+
+    // commit
+    std::vector<int32_t> new_pages(s->pages.begin(), s->pages.begin() + new_np);
+    int64_t moved = 0;
+    if (any_change) {
+        for (int32_t q = qc; q < new_np; ++q) {
+            const int32_t row_end = std::min<int64_t>((int64_t)q * P + P, n2);
+            if (alloc_.refcount(s->pages[q]) > 1) {
+                new_pages[q] = take_lowest();
+                plan->cow_pages.push_back(new_pages[q]);
+                moved += row_end - (int64_t)q * P;
+            } else {
+                moved += row_end - std::max<int64_t>((int64_t)q * P, a0);
+            }
+        }
+        for (int32_t q = qc; q < new_np; ++q)
+            if (new_pages[q] != s->pages[q]) alloc_.drop_ref(s->pages[q]);
+    }
+    for (size_t q = new_np; q < s->pages.size(); ++q)
+        if (alloc_.drop_ref(s->pages[q])) plan->freed.push_back(s->pages[q]);
+    plan->new_pages = new_pages;
+    plan->n_new = n2;
+    plan->first_row = any_change ? qc * P : n2;
+    plan->moved_rows = moved;
+    plan->evicted = (int32_t)removed;
+    s->pages = std::move(new_pages);
+    s->n = n2;
+    s->version = g_version_counter++;
+    return kOk;
+}
+
+void HostCache::undo_evict(int32_t h, const EvictPlan& plan) {
+    Seq* s = seq_mut(h);
+    if (!s || plan.n_new == plan.n_old) return;
+    // trailing pages back
+    for (size_t q = plan.new_pages.size(); q < plan.old_pages.size(); ++q) {
+        int32_t p = plan.old_pages[q];
+        if (alloc_.refcount(p) == 0) alloc_.take(p);
+        else alloc_.add_ref(p);
+    }
+    for (size_t q = 0; q < plan.new_pages.size(); ++q) {
+        if (plan.new_pages[q] != plan.old_pages[q]) {
+            alloc_.drop_ref(plan.new_pages[q]);
+            alloc_.add_ref(plan.old_pages[q]);
+        }
+    }
+    s->pages = plan.old_pages;
+    s->n = plan.n_old;
+    s->version = g_version_counter++;
+}
+
+int HostCache::release(int32_t h, std::vector<int32_t>* freed) {
+    Seq* s = seq_mut(h);
+    if (!s) return kBadHandle;
+    for (int32_t p : s->pages)
+        if (alloc_.drop_ref(p) && freed) freed->push_back(p);
+    s->pages.clear();
+    s->n = 0;
+    s->live = false;
+    int32_t slot = h & 0xFFFFF;
+    free_slots_.push_back(slot);
+    return kOk;
+}
+
+// ---------------------------------------------------------------------------
+// decode planning
+
+int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
+                int32_t n_ctas, DecodePlanHost* out) {
+    *out = DecodePlanHost();
+    const Geometry& g = c.geom();
+    if (n_seqs < 1 || !handles || n_ctas < 1) return kInvalidArg;
+    std::vector<const Seq*> ss(n_seqs);
+    for (int32_t i = 0; i < n_seqs; ++i) {
+        ss[i] = c.seq(handles[i]);
+        if (!ss[i]) return kBadHandle;
+        if (ss[i]->n < 1) return kInvalidArg;
+        for (int32_t j = 0; j < i; ++j)
+            if (ss[j] == ss[i]) return kInvalidArg;
+        out->logical_tokens += ss[i]->n;
+    }
+    const int32_t P = g.P;
+    const int32_t max_grp = kRowsPerTile / g.G();
+
+    // Group sequences holding the same physical page at the same logical
+    // index into shared runs (depth-first over the prefix tree of pages).
+    struct Work {
+        std::vector<int32_t> members;
+        int32_t q;
+    };
+    std::vector<Work> stack;
+    {
+        Work root;
+        for (int32_t i = 0; i < n_seqs; ++i) root.members.push_back(i);
+        root.q = 0;
+        stack.push_back(std::move(root));
+    }
+    while (!stack.empty()) {
+        Work w = std::move(stack.back());
+        stack.pop_back();
+        // partition by the page held at w.q (first-seen order)
+        std::vector<std::vector<int32_t>> parts;
+        std::vector<int32_t> part_page;
+        for (int32_t i : w.members) {
+            if ((int32_t)ss[i]->pages.size() <= w.q) continue;
+            int32_t p = ss[i]->pages[w.q];
+            size_t k = 0;
+            while (k < part_page.size() && part_page[k] != p) ++k;
+            if (k == part_page.size()) {
+                part_page.push_back(p);
+                parts.emplace_back();
+            }
+            parts[k].push_back(i);
+        }
+        // process parts in order: push in reverse so the first is handled first
+        std::vector<Work> next;
+        for (auto& part : parts) {
+            const int32_t q0 = w.q;
+            int32_t q_end = q0 + 1;
+            const Seq* lead = ss[part[0]];
+            for (;;) {
+                if (q_end >= (int32_t)lead->pages.size()) break;
+                bool same = true;
+                for (int32_t i : part) {
+                    if ((int32_t)ss[i]->pages.size() <= q_end ||
+                        ss[i]->pages[q_end] != lead->pages[q_end]) {
+                        same = false;
+                        break;
+                    }
+                }
+                if (!same) break;
+                ++q_end;
+            }
+            for (size_t b = 0; b < part.size(); b += max_grp) {
+                DecodeSeg seg;
+                std::memset(&seg, 0, sizeof seg);
+                seg.page_off = (int32_t)out->page_ids.size();
+                seg.n_pages = q_end - q0;
+                seg.n_grp = (int32_t)std::min<size_t>(max_grp, part.size() - b);
+                seg.n_tok = 0;
+                for (int32_t j = 0; j < seg.n_grp; ++j) {
+                    int32_t i = part[b + j];
+                    int64_t lim = std::min<int64_t>((int64_t)ss[i]->n - (int64_t)q0 * P,
+                                                    (int64_t)seg.n_pages * P);
+                    seg.grp_seq[j] = i;
+                    seg.grp_lim[j] = (int32_t)lim;
+                    seg.n_tok = std::max(seg.n_tok, (int32_t)lim);
+                }
+                const Seq* sl = ss[part[b]];
+                for (int32_t q = q0; q < q_end; ++q) out->page_ids.push_back(sl->pages[q]);
+                out->unique_tokens += seg.n_tok;
+                out->segs.push_back(seg);
+            }
+            Work nw;
+            for (int32_t i : part)
+                if ((int32_t)ss[i]->pages.size() > q_end) nw.members.push_back(i);
+            nw.q = q_end;
+            if (!nw.members.empty()) next.push_back(std::move(nw));
+        }
+        for (auto it = next.rbegin(); it != next.rend(); ++it) stack.push_back(std::move(*it));
+    }
+
+    // (segment, head) units, stage counts, and an even split of all stages
+    // over the persistent CTAs.
+    const int32_t n_segs = (int32_t)out->segs.size();
+    std::vector<int64_t> unit_start;
+    int64_t total = 0;
+    for (int32_t s = 0; s < n_segs; ++s)
+        for (int32_t h = 0; h < g.Hkv; ++h) {
+            unit_start.push_back(total);
+            total += ceil_div(out->segs[s].n_tok, kStageTokens);
+        }
+    unit_start.push_back(total);
+    const int32_t ctas = (int32_t)std::min<int64_t>(n_ctas, total);
+    out->n_ctas = ctas;
+    out->cta_begin.resize(ctas + 1);
+    size_t u = 0;
+    for (int32_t cta = 0; cta < ctas; ++cta) {
+        const int64_t b = total * cta / ctas, e = total * (cta + 1) / ctas;
+        out->cta_begin[cta] = (int32_t)out->items.size();
+        int64_t pos = b;
+        while (pos < e) {
+            while (unit_start[u + 1] <= pos) ++u;
+            const int64_t stop = std::min(e, unit_start[u + 1]);
+            DecodeItem it;
+            it.seg = (int32_t)(u / g.Hkv);
+            it.head = (int32_t)(u % g.Hkv);
+            it.s0 = (int32_t)(pos - unit_start[u]);
+            it.s1 = (int32_t)(stop - unit_start[u]);
+            out->items.push_back(it);
+            pos = stop;
+        }
+    }
+    out->cta_begin[ctas] = (int32_t)out->items.size();
+
+    // combine lists per (sequence, KV head)
+    const int32_t keys = n_seqs * g.Hkv;
+    out->comb_off.assign(keys + 1, 0);
+    for (const DecodeItem& it : out->items) {
+        const DecodeSeg& s = out->segs[it.seg];
+        for (int32_t j = 0; j < s.n_grp; ++j) ++out->comb_off[s.grp_seq[j] * g.Hkv + it.head + 1];
+    }
+    for (int32_t k = 0; k < keys; ++k) out->comb_off[k + 1] += out->comb_off[k];
+    out->comb_ent.resize(out->comb_off[keys]);
+    std::vector<int32_t> fill(out->comb_off.begin(), out->comb_off.end() - 1);
+    for (int32_t i = 0; i < (int32_t)out->items.size(); ++i) {
+        const DecodeItem& it = out->items[i];
+        const DecodeSeg& s = out->segs[it.seg];
+        for (int32_t j = 0; j < s.n_grp; ++j) {
+            CombineEnt e;
+            e.item = i;
+            e.j = j;
+            out->comb_ent[fill[s.grp_seq[j] * g.Hkv + it.head]++] = e;
+        }
+    }
+    return kOk;
+}
+
+static int64_t align16(int64_t x) { return (x + 15) & ~int64_t(15); }
+
+DecodePlanLayout plan_layout(const DecodePlanHost& p, int32_t n_seqs, int32_t Hkv) {
+    DecodePlanLayout L;
+    L.n_segs = (int32_t)p.segs.size();
+    L.n_items = (int32_t)p.items.size();
+    L.n_ctas = p.n_ctas;
+    L.n_page_ids = (int32_t)p.page_ids.size();
+    L.n_comb_keys = n_seqs * Hkv;
+    L.n_comb_ent = (int32_t)p.comb_ent.size();
+    int64_t o = 0;
+    L.segs = o;      o = align16(o + sizeof(DecodeSeg) * L.n_segs);
+    L.items = o;     o = align16(o + sizeof(DecodeItem) * L.n_items);
+    L.cta_begin = o; o = align16(o + sizeof(int32_t) * (L.n_ctas + 1));
+    L.page_ids = o;  o = align16(o + sizeof(int32_t) * L.n_page_ids);
+    L.comb_off = o;  o = align16(o + sizeof(int32_t) * (L.n_comb_keys + 1));
+    L.comb_ent = o;  o = align16(o + sizeof(CombineEnt) * L.n_comb_ent);
+    L.total = o;
+    return L;
+}
+
+void plan_serialize(const DecodePlanHost& p, const DecodePlanLayout& L, uint8_t* dst) {
+    std::memset(dst, 0, L.total);
+    std::memcpy(dst + L.segs, p.segs.data(), sizeof(DecodeSeg) * L.n_segs);
+    std::memcpy(dst + L.items, p.items.data(), sizeof(DecodeItem) * L.n_items);
+    std::memcpy(dst + L.cta_begin, p.cta_begin.data(), sizeof(int32_t) * (L.n_ctas + 1));
+    std::memcpy(dst + L.page_ids, p.page_ids.data(), sizeof(int32_t) * L.n_page_ids);
+    std::memcpy(dst + L.comb_off, p.comb_off.data(), sizeof(int32_t) * (L.n_comb_keys + 1));
+    std::memcpy(dst + L.comb_ent, p.comb_ent.data(), sizeof(CombineEnt) * L.n_comb_ent);
+}
+
+}  // namespace sq

@@ -1,0 +1,163 @@
+// Host-side state of the paged KV cache: page allocator, reference counts,
+// sequence table and page tables, and the planners for append, eviction and
+// decode.  Plain C++17, no CUDA: the device side consumes the plans.
+//
+// The rules (Sec. 3.1 and Algorithm 1 for fork / append / clear_kv /
+// release; Sec. 3.4 for prefix sharing without duplication) are fixed as:
+//   * lowest free page id first;
+//   * fork copies the page list, +1 reference per page, no K/V copy;
+//   * append: copy-on-write of a shared partial last page, then new pages in
+//     increasing logical order;
+//   * evict: a destination page whose rows change and that is shared is
+//     replaced by a fresh page (increasing logical order), others are
+//     compacted in place; pages past the new end lose a reference;
+//   * release: every page loses a reference.
+#pragma once
+
+#include <stdint.h>
+
+#include <vector>
+
+#include "plan.hpp"
+
+namespace sq {
+
+enum Status : int {
+    kOk = 0,
+    kInvalidArg = -1,
+    kBadHandle = -2,
+    kNoPages = -3,
+    kCapacity = -4,
+    kCuda = -5,
+    kDevice = -6,
+    kDeviceTimeout = -7,
+    kUnsupported = -8,
+    kNoMemory = -9,
+};
+
+struct Geometry {
+    int32_t L = 0, Hq = 0, Hkv = 0, D = 0, P = 0;
+    int32_t num_pages = 0, max_seqs = 0, max_pages_per_seq = 0;
+    int32_t G() const { return Hq / Hkv; }
+    // K+V bytes of one token of one layer
+    int64_t token_layer_bytes() const { return 2LL * Hkv * D * 2; }
+};
+
+// Validates a geometry against what the kernels handle.
+int check_geometry(const Geometry& g);
+
+class PageAllocator {
+  public:
+    explicit PageAllocator(int32_t n = 0);
+    int32_t size() const { return (int32_t)ref_.size(); }
+    int32_t free_count() const { return free_count_; }
+    int32_t refcount(int32_t p) const { return ref_[p]; }
+    // The lowest free page id, -1 if none.
+    int32_t lowest_free() const;
+    // Take a free page (reference count 0 -> 1).
+    void take(int32_t p);
+    void add_ref(int32_t p) { ++ref_[p]; }
+    // Drop one reference; true if the page became free.
+    bool drop_ref(int32_t p);
+
+  private:
+    std::vector<int32_t> ref_;
+    std::vector<uint64_t> free_bits_;  // bit set = free
+    int32_t free_count_ = 0;
+    mutable int32_t hint_ = 0;         // no free page below word hint_
+};
+
+struct Seq {
+    bool live = false;
+    uint32_t gen = 0;
+    int32_t n = 0;
+    std::vector<int32_t> pages;
+    uint64_t version = 0;  // bumped by every change of n or pages
+    void* last_stream = nullptr;
+};
+
+struct AppendPlan {
+    int32_t n0 = 0, n_new = 0;
+    bool cow = false;
+    int32_t cow_old = -1, cow_new = -1, cow_rows = 0;
+    int32_t first_page_index = 0;  // logical index of the page holding n0
+    std::vector<int32_t> pages;    // page ids for logical pages first_page_index ..
+    std::vector<int32_t> taken;    // pages newly taken (cow page first)
+};
+
+struct EvictPlan {
+    int32_t n_old = 0, n_new = 0;
+    int32_t first_row = 0;             // first destination row that may change
+    std::vector<int32_t> old_pages;    // page table before
+    std::vector<int32_t> new_pages;    // page table after (length ceil(n_new / P))
+    std::vector<int32_t> run_dst;      // kept runs: destination start (increasing)
+    std::vector<int32_t> run_src;      //            source start
+    std::vector<int32_t> run_len;      //            length (> 0)
+    std::vector<int32_t> cow_pages;    // fresh pages taken (increasing logical page)
+    std::vector<int32_t> freed;        // pages whose count reached zero
+    int64_t moved_rows = 0;            // destination rows that are written
+    int32_t evicted = 0;
+};
+
+class HostCache {
+  public:
+    explicit HostCache(const Geometry& g);
+    const Geometry& geom() const { return g_; }
+    const PageAllocator& alloc() const { return alloc_; }
+
+    int seq_new(int32_t* handle);
+    int fork(int32_t parent, int32_t* child);
+    // Plans and commits an append (host state updated).  `undo_append`
+    // restores the state if the device work cannot be enqueued.
+    int append(int32_t h, int32_t n_new, AppendPlan* plan);
+    void undo_append(int32_t h, const AppendPlan& plan);
+    // Validates spans, plans and commits an eviction.
+    int evict(int32_t h, const int32_t* starts, const int32_t* ends,
+              int32_t n_spans, EvictPlan* plan);
+    void undo_evict(int32_t h, const EvictPlan& plan);
+    int release(int32_t h, std::vector<int32_t>* freed);
+
+    // Resolves a handle; nullptr if invalid.
+    const Seq* seq(int32_t h) const;
+    Seq* seq_mut(int32_t h);
+    int32_t live_pages() const { return g_.num_pages - alloc_.free_count(); }
+    int64_t peak_live_pages() const { return peak_live_; }
+
+  private:
+    int32_t take_lowest();
+    Geometry g_;
+    PageAllocator alloc_;
+    std::vector<Seq> seqs_;
+    std::vector<int32_t> free_slots_;  // stack, lowest slot on top
+    int64_t peak_live_ = 0;
+};
+
+// ---- decode planning -------------------------------------------------------
+
+struct DecodePlanHost {
+    std::vector<DecodeSeg> segs;
+    std::vector<DecodeItem> items;
+    std::vector<int32_t> cta_begin;   // n_ctas + 1
+    std::vector<int32_t> page_ids;
+    std::vector<int32_t> comb_off;    // n_seqs * Hkv + 1
+    std::vector<CombineEnt> comb_ent;
+    int64_t unique_tokens = 0;        // sum over segments of n_tok (one head, one layer)
+    int64_t logical_tokens = 0;       // sum over sequences of n
+    int32_t n_ctas = 0;
+};
+
+// Plans one decode call over the given sequences (each with n >= 1):
+// groups sequences that hold the same physical page at the same logical
+// index into shared runs, splits every (run, KV head) into stages of
+// kStageTokens tokens and deals the stages out evenly to `n_ctas`
+// persistent CTAs.
+int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
+                int32_t n_ctas, DecodePlanHost* out);
+
+// Serialises a plan into one buffer (8-byte aligned arrays).
+DecodePlanLayout plan_layout(const DecodePlanHost& p, int32_t n_seqs,
+                             int32_t Hkv);
+void plan_serialize(const DecodePlanHost& p, const DecodePlanLayout& lay,
+                    uint8_t* dst);
+
+}  // namespace sq

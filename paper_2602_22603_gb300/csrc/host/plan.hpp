@@ -1,0 +1,47 @@
+// Plain-old-data work descriptions the host planners write and the kernels
+// read.  Shared by host code (C++) and device code (CUDA); no CUDA types.
+#pragma once
+#include <stdint.h>
+
+namespace sq {
+
+// Rows of one tensor-core tile: the query rows a decode work item serves
+// (Sec. 2.1: a KV head is shared by G query heads; with several sequences
+// sharing the same pages, their query groups stack up to this many rows).
+constexpr int kRowsPerTile = 16;
+// Tokens of K/V one pipeline stage of the decode kernel holds.
+constexpr int kStageTokens = 64;
+// Consumer warps of the decode kernel; each owns kStageTokens / 4 tokens.
+constexpr int kDecodeConsumerWarps = 4;
+
+// A run of logical pages read once for a group of sequences that hold the
+// same physical pages there (a main thread and its forks, Sec. 3.4).
+struct DecodeSeg {
+    int32_t page_off;                 // into DecodePlan page_ids
+    int32_t n_pages;                  // pages in the run
+    int32_t n_tok;                    // tokens to read (max over the group)
+    int32_t n_grp;                    // sequences in the group
+    int32_t grp_seq[kRowsPerTile];    // call-local sequence indices
+    int32_t grp_lim[kRowsPerTile];    // valid tokens of each, from the run start
+};
+
+// A contiguous range of stages of one (segment, KV head) — one partial result.
+struct DecodeItem {
+    int32_t seg;
+    int32_t head;
+    int32_t s0, s1;                   // stages [s0, s1)
+};
+
+// One combine entry: partials of item `item`, rows of group member `j`.
+struct CombineEnt {
+    int32_t item;
+    int32_t j;
+};
+
+// Byte offsets of the arrays of a decode plan inside one upload buffer.
+struct DecodePlanLayout {
+    int64_t segs, items, cta_begin, page_ids, comb_off, comb_ent, total;
+    int32_t n_segs, n_items, n_ctas, n_page_ids, n_comb_keys, n_comb_ent;
+};
+
+}  // namespace sq

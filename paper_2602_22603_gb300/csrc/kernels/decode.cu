@@ -1,0 +1,461 @@
+// Split-K flash-decoding over the paged bf16 KV pool, and the log-sum-exp
+// combine of its partial results.
+//
+// What is computed (Sec. 1 and Sec. 3.4: for every generated token,
+// attention reads the whole KV cache of the context; Sec. 2.1: in
+// grouped-query attention a K/V head serves G query heads): for sequence i,
+// query head h and KV head g = h / G,
+//     out[i][h] = sum_t softmax_t(sm_scale * q[i][h] . K_g[t]) V_g[t].
+//
+// Work decomposition (host planner, core.cpp): every run of pages that a
+// group of sequences holds in common (a main thread and its forked auxiliary
+// threads, Sec. 3.4) is one segment; a (segment, KV head) pair is a list of
+// 64-token stages; the stages of all pairs are dealt evenly to persistent
+// CTAs.  Each CTA streams its stages through a TMA + mbarrier ring in shared
+// memory; each of four consumer warps owns 16 tokens of a stage and keeps an
+// online-softmax partial (max, sum, unnormalised output) for up to 16 query
+// rows — the G heads of every sequence in the group, so a shared page is read
+// from HBM once for all of them.
+//
+// Tensor cores: S = Q K^T and O += P V are m16n8k16 bf16 mma.sync with fp32
+// accumulation; rows = query rows (<= 16), columns = tokens / head dims.  The
+// contraction is tiny (G x d per token) and the kernel is HBM-bound, so the
+// warp-level mma is the right size: the point is to keep HBM busy.
+#include <math.h>
+
+#include "launch.hpp"
+#include "ptx.cuh"
+
+namespace sq {
+namespace {
+
+using namespace dev;
+
+template <int D>
+struct DecCfg {
+    static constexpr int kColBlocks = D / 64;                    // 128-byte column blocks
+    static constexpr int kBlockBytes = kStageTokens * 128;       // one column block of a tile
+    static constexpr int kTileBytes = kColBlocks * kBlockBytes;  // K (or V) of one stage
+    static constexpr int kStageBytes = 2 * kTileBytes;
+    static constexpr int kStages = (D == 128) ? 3 : 6;
+    static constexpr int kThreads = (kDecodeConsumerWarps + 1) * 32;
+    static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 128;
+    static constexpr int kNT = D / 8;   // 8-wide output column tiles
+    static constexpr int kKS = D / 16;  // 16-deep contraction steps
+};
+
+__device__ __forceinline__ uint32_t ld_u32(const __nv_bfloat16* p) {
+    return *reinterpret_cast<const uint32_t*>(p);
+}
+
+// ---- producer: one thread issues the TMA loads of every stage -------------
+template <int D>
+__device__ void produce(const CUtensorMap* tmap, const DecodeArgs& a, int it0, int it1,
+                        uint8_t* smem, uint64_t* bars, volatile int* abort_flag) {
+    using C = DecCfg<D>;
+    prefetch_tmap(tmap);
+    const int P = a.P;
+    const int box_rows = P < kStageTokens ? P : kStageTokens;
+    const int pages_per_stage = P < kStageTokens ? kStageTokens / P : 1;
+    const uint32_t box_bytes = (uint32_t)box_rows * 128u;
+    int slot = 0;
+    uint32_t phase = 0;
+    uint32_t issued = 0, issued_phase = 0;  // per-slot bits of the last issue
+    bool ok = true;
+    for (int it = it0; it < it1 && ok; ++it) {
+        const DecodeItem item = a.items[it];
+        const DecodeSeg* seg = a.segs + item.seg;
+        const int page_off = seg->page_off, n_pages = seg->n_pages;
+        for (int s = item.s0; s < item.s1; ++s) {
+            const uint32_t full = smem_addr(&bars[slot]);
+            const uint32_t empty = smem_addr(&bars[C::kStages + slot]);
+            if (!mbar_wait(empty, phase ^ 1)) {
+                set_error(a.err, kErrTimeout);
+                *abort_flag = 1;
+                ok = false;
+                break;
+            }
+            if (*abort_flag) {
+                ok = false;
+                break;
+            }
+            const int tok0 = s * kStageTokens;
+            const int pi0 = tok0 / P;
+            const int row0 = P > kStageTokens ? (tok0 % P) : 0;
+            const int np = P >= kStageTokens ? 1 : min(pages_per_stage, n_pages - pi0);
+            int32_t pid[kStageTokens / 8];
+            uint32_t vmask = 0;
+            for (int k = 0; k < np; ++k) {
+                const int32_t p = a.page_ids[page_off + pi0 + k];
+                pid[k] = p;
+                if ((uint32_t)p < (uint32_t)a.num_pages) vmask |= 1u << k;
+                else set_error(a.err, kErrBounds);
+            }
+            const uint32_t bytes = (uint32_t)__popc(vmask) * box_bytes * C::kColBlocks * 2u;
+            uint8_t* stage = smem + slot * C::kStageBytes;
+            if (bytes == 0) {
+                mbar_arrive(full);
+            } else {
+                mbar_arrive_expect_tx(full, bytes);
+                for (int k = 0; k < np; ++k) {
+                    if (!((vmask >> k) & 1u)) continue;
+                    for (int cb = 0; cb < C::kColBlocks; ++cb) {
+                        const uint32_t dk =
+                            smem_addr(stage + cb * C::kBlockBytes + k * box_rows * 128);
+                        tma_load_4d(dk, tmap, full, cb * 64, item.head * P + row0, pid[k],
+                                    a.layer);
+                        tma_load_4d(dk + C::kTileBytes, tmap, full, cb * 64,
+                                    (a.Hkv + item.head) * P + row0, pid[k], a.layer);
+                    }
+                }
+            }
+            issued |= 1u << slot;
+            issued_phase = (issued_phase & ~(1u << slot)) | (phase << slot);
+            if (++slot == C::kStages) {
+                slot = 0;
+                phase ^= 1;
+            }
+        }
+    }
+    if (!ok) {
+        // Leave only after every copy already issued has landed (bounded).
+        for (int sl = 0; sl < C::kStages; ++sl)
+            if ((issued >> sl) & 1u)
+                mbar_wait(smem_addr(&bars[sl]), (issued_phase >> sl) & 1u);
+    }
+}
+
+// ---- consumers: four warps, 16 tokens of every stage each ------------------
+template <int D>
+__device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, uint64_t* bars,
+                        volatile int* abort_flag, int warp, int lane) {
+    using C = DecCfg<D>;
+    const int gid = lane >> 2, tig = lane & 3;
+    const int r0 = gid, r1 = gid + 8;
+    const int mi = lane >> 3, rr = lane & 7;
+    int slot = 0;
+    uint32_t phase = 0;
+    for (int it = it0; it < it1; ++it) {
+        const DecodeItem item = a.items[it];
+        const DecodeSeg* seg = a.segs + item.seg;
+        const int G = a.G;
+        const int n_grp = seg->n_grp;
+        const int j0 = r0 / G, j1 = r1 / G;
+        const bool v0 = j0 < n_grp, v1 = j1 < n_grp;
+        const int lim0 = v0 ? seg->grp_lim[j0] : 0;
+        const int lim1 = v1 ? seg->grp_lim[j1] : 0;
+        const int n_tok = seg->n_tok;
+
+        uint32_t qa[C::kKS][4];
+        {
+            const __nv_bfloat16* q0 =
+                a.q + ((size_t)(v0 ? seg->grp_seq[j0] : 0) * a.Hq + item.head * G + r0 % G) * D;
+            const __nv_bfloat16* q1 =
+                a.q + ((size_t)(v1 ? seg->grp_seq[j1] : 0) * a.Hq + item.head * G + r1 % G) * D;
+#pragma unroll
+            for (int kk = 0; kk < C::kKS; ++kk) {
+                const int c = kk * 16 + tig * 2;
+                qa[kk][0] = v0 ? ld_u32(q0 + c) : 0u;
+                qa[kk][1] = v1 ? ld_u32(q1 + c) : 0u;
+                qa[kk][2] = v0 ? ld_u32(q0 + c + 8) : 0u;
+                qa[kk][3] = v1 ? ld_u32(q1 + c + 8) : 0u;
+            }
+        }
+        float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+        float o[C::kNT][4];
+#pragma unroll
+        for (int nd = 0; nd < C::kNT; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
+
+        for (int s = item.s0; s < item.s1; ++s) {
+            const uint32_t full = smem_addr(&bars[slot]);
+            const uint32_t empty = smem_addr(&bars[C::kStages + slot]);
+            if (!mbar_wait(full, phase)) {
+                set_error(a.err, kErrTimeout);
+                *abort_flag = 1;
+                return;
+            }
+            const uint32_t kb = smem_addr(smem + slot * C::kStageBytes);
+            const uint32_t vb = kb + C::kTileBytes;
+            const int tbase = s * kStageTokens + warp * 16;  // segment-relative
+
+            // S = Q K^T over this warp's 16 tokens (two n8 tiles)
+            float sc[2][4];
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+            {
+                const int t = warp * 16 + (mi >> 1) * 8 + rr;
+                const uint32_t row = kb + t * 128;
+                const int sw = t & 7;
+#pragma unroll
+                for (int kk = 0; kk < C::kKS; ++kk) {
+                    const int d0 = kk * 16 + (mi & 1) * 8;
+                    uint32_t b0, b1, b2, b3;
+                    ldsm_x4(row + (d0 >> 6) * C::kBlockBytes + ((((d0 & 63) >> 3) ^ sw) << 4), b0,
+                            b1, b2, b3);
+                    mma_bf16(sc[0], qa[kk], b0, b1);
+                    mma_bf16(sc[1], qa[kk], b2, b3);
+                }
+            }
+
+            // masking, scaling, online softmax (log2 domain)
+            float x[2][4];
+            float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int tk = tbase + nt * 8 + tig * 2 + e;
+                    x[nt][e] = tk < lim0 ? sc[nt][e] * a.scale_log2 : -INFINITY;
+                    x[nt][2 + e] = tk < lim1 ? sc[nt][2 + e] * a.scale_log2 : -INFINITY;
+                    mx0 = fmaxf(mx0, x[nt][e]);
+                    mx1 = fmaxf(mx1, x[nt][2 + e]);
+                }
+            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+            const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+            const float ms0 = mn0 == -INFINITY ? 0.f : mn0;
+            const float ms1 = mn1 == -INFINITY ? 0.f : mn1;
+            const float al0 = exp2f(m0 - ms0), al1 = exp2f(m1 - ms1);
+            m0 = mn0;
+            m1 = mn1;
+            float ps0 = 0.f, ps1 = 0.f;
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    x[nt][e] = exp2f(x[nt][e] - ms0);
+                    x[nt][2 + e] = exp2f(x[nt][2 + e] - ms1);
+                    ps0 += x[nt][e];
+                    ps1 += x[nt][2 + e];
+                }
+            l0 = l0 * al0 + ps0;
+            l1 = l1 * al1 + ps1;
+#pragma unroll
+            for (int nd = 0; nd < C::kNT; ++nd) {
+                o[nd][0] *= al0;
+                o[nd][1] *= al0;
+                o[nd][2] *= al1;
+                o[nd][3] *= al1;
+            }
+            uint32_t pa[4];
+            pa[0] = pack_bf16x2(x[0][0], x[0][1]);
+            pa[1] = pack_bf16x2(x[0][2], x[0][3]);
+            pa[2] = pack_bf16x2(x[1][0], x[1][1]);
+            pa[3] = pack_bf16x2(x[1][2], x[1][3]);
+
+            // Rows past the last valid token hold stale or never-written
+            // shared memory: zero this warp's such V rows so 0 * V stays 0.
+            const bool tail = tbase + 16 > n_tok;
+            if (tail) {
+                const int first = max(0, n_tok - tbase);
+                const int per_row = C::kColBlocks * 8;  // 16-byte chunks per row
+                const int total = (16 - first) * per_row;
+                uint8_t* vgen = smem + slot * C::kStageBytes + C::kTileBytes;
+                for (int idx = lane; idx < total; idx += 32) {
+                    const int row = warp * 16 + first + idx / per_row;
+                    const int rem = idx % per_row;
+                    *reinterpret_cast<uint4*>(vgen + (rem >> 3) * C::kBlockBytes + row * 128 +
+                                              (rem & 7) * 16) = make_uint4(0, 0, 0, 0);
+                }
+                __syncwarp();
+            }
+
+            // O += P V (V^T fragments through ldmatrix.trans)
+            {
+                const int t = warp * 16 + (mi & 1) * 8 + rr;
+                const uint32_t row = vb + t * 128;
+                const int sw = t & 7;
+#pragma unroll
+                for (int nd2 = 0; nd2 < C::kKS; ++nd2) {
+                    const int d0 = nd2 * 16 + (mi >> 1) * 8;
+                    uint32_t b0, b1, b2, b3;
+                    ldsm_x4_trans(row + (d0 >> 6) * C::kBlockBytes + ((((d0 & 63) >> 3) ^ sw) << 4),
+                                  b0, b1, b2, b3);
+                    mma_bf16(o[2 * nd2], pa, b0, b1);
+                    mma_bf16(o[2 * nd2 + 1], pa, b2, b3);
+                }
+            }
+            if (tail) fence_proxy_async_smem();  // generic writes before the next TMA fill
+            __syncwarp();
+            if (lane == 0) mbar_arrive(empty);
+            if (++slot == C::kStages) {
+                slot = 0;
+                phase ^= 1;
+            }
+        }
+
+        // close the item: full row sums, then the partial (o, m, l)
+        l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+        l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+        l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+        l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+        const size_t pidx = (size_t)it * kDecodeConsumerWarps + warp;
+        float* po = a.part_o + pidx * kRowsPerTile * D;
+        float* pml = a.part_ml + pidx * kRowsPerTile * 2;
+        if (v0) {
+#pragma unroll
+            for (int nd = 0; nd < C::kNT; ++nd)
+                *reinterpret_cast<float2*>(po + r0 * D + nd * 8 + tig * 2) =
+                    make_float2(o[nd][0], o[nd][1]);
+            if (tig == 0) *reinterpret_cast<float2*>(pml + r0 * 2) = make_float2(m0, l0);
+        }
+        if (v1) {
+#pragma unroll
+            for (int nd = 0; nd < C::kNT; ++nd)
+                *reinterpret_cast<float2*>(po + r1 * D + nd * 8 + tig * 2) =
+                    make_float2(o[nd][2], o[nd][3]);
+            if (tig == 0) *reinterpret_cast<float2*>(pml + r1 * 2) = make_float2(m1, l1);
+        }
+    }
+}
+
+template <int D>
+__global__ void __launch_bounds__(DecCfg<D>::kThreads, 2)
+    sq_decode_splitk_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a) {
+    using C = DecCfg<D>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 2 * C::kStages);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::kStages; ++s) {
+            mbar_init(smem_addr(&bars[s]), 1);
+            mbar_init(smem_addr(&bars[C::kStages + s]), kDecodeConsumerWarps);
+        }
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    __syncthreads();
+    const int it0 = a.cta_begin[blockIdx.x], it1 = a.cta_begin[blockIdx.x + 1];
+    if (warp == kDecodeConsumerWarps) {
+        if (lane == 0) produce<D>(&tmap, a, it0, it1, smem, bars, abort_flag);
+        return;
+    }
+    consume<D>(a, it0, it1, smem, bars, abort_flag, warp, lane);
+}
+
+// ---- combine: one warp per (sequence, query head) ---------------------------
+template <int D>
+__global__ void __launch_bounds__(256) sq_lse_combine_kernel(const CombineArgs a) {
+    constexpr int V = D / 32;  // output elements per lane
+    const int wid = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (wid >= a.n_seqs * a.Hq) return;
+    const int i = wid / a.Hq, h = wid % a.Hq;
+    const int hh = h % a.G;
+    const int key = i * a.Hkv + h / a.G;
+    const int e0 = a.comb_off[key], e1 = a.comb_off[key + 1];
+    const int np = (e1 - e0) * kDecodeConsumerWarps;
+
+    float M = -INFINITY;
+    for (int k = lane; k < np; k += 32) {
+        const CombineEnt ent = a.comb_ent[e0 + k / kDecodeConsumerWarps];
+        const size_t p = (size_t)ent.item * kDecodeConsumerWarps + k % kDecodeConsumerWarps;
+        const int r = ent.j * a.G + hh;
+        M = fmaxf(M, a.part_ml[(p * kRowsPerTile + r) * 2]);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    const float Ms = M == -INFINITY ? 0.f : M;
+
+    float acc[V];
+#pragma unroll
+    for (int e = 0; e < V; ++e) acc[e] = 0.f;
+    float L = 0.f;
+    for (int k = 0; k < np; ++k) {
+        const CombineEnt ent = a.comb_ent[e0 + k / kDecodeConsumerWarps];
+        const size_t p = (size_t)ent.item * kDecodeConsumerWarps + k % kDecodeConsumerWarps;
+        const size_t row = p * kRowsPerTile + ent.j * a.G + hh;
+        const float2 ml = *reinterpret_cast<const float2*>(a.part_ml + row * 2);
+        const float w = exp2f(ml.x - Ms);
+        L += w * ml.y;
+        const float* po = a.part_o + row * D + lane * V;
+        if constexpr (V == 4) {
+            const float4 v = *reinterpret_cast<const float4*>(po);
+            acc[0] += w * v.x;
+            acc[1] += w * v.y;
+            acc[2] += w * v.z;
+            acc[3] += w * v.w;
+        } else {
+            const float2 v = *reinterpret_cast<const float2*>(po);
+            acc[0] += w * v.x;
+            acc[1] += w * v.y;
+        }
+    }
+    const float inv = 1.f / L;
+    const size_t ob = ((size_t)i * a.Hq + h) * D + lane * V;
+    if (a.out_f32) {
+        float* out = reinterpret_cast<float*>(a.out) + ob;
+        if constexpr (V == 4)
+            *reinterpret_cast<float4*>(out) =
+                make_float4(acc[0] * inv, acc[1] * inv, acc[2] * inv, acc[3] * inv);
+        else
+            *reinterpret_cast<float2*>(out) = make_float2(acc[0] * inv, acc[1] * inv);
+    } else {
+        __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.out) + ob;
+        if constexpr (V == 4) {
+            uint2 u;
+            u.x = pack_bf16x2(acc[0] * inv, acc[1] * inv);
+            u.y = pack_bf16x2(acc[2] * inv, acc[3] * inv);
+            *reinterpret_cast<uint2*>(out) = u;
+        } else {
+            *reinterpret_cast<uint32_t*>(out) = pack_bf16x2(acc[0] * inv, acc[1] * inv);
+        }
+    }
+}
+
+}  // namespace
+
+int64_t decode_partial_bytes(int32_t n_items, int32_t D) {
+    return (int64_t)n_items * kDecodeConsumerWarps * kRowsPerTile * (D + 2) * (int64_t)sizeof(float);
+}
+
+cudaError_t decode_prepare(int D) {
+    if (D == 128)
+        return cudaFuncSetAttribute(sq_decode_splitk_kernel<128>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    DecCfg<128>::kSmemBytes);
+    return cudaFuncSetAttribute(sq_decode_splitk_kernel<64>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                DecCfg<64>::kSmemBytes);
+}
+
+int decode_ctas_per_sm(int D) {
+    int n = 0;
+    cudaError_t e;
+    if (D == 128)
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, sq_decode_splitk_kernel<128>,
+                                                          DecCfg<128>::kThreads,
+                                                          DecCfg<128>::kSmemBytes);
+    else
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, sq_decode_splitk_kernel<64>,
+                                                          DecCfg<64>::kThreads,
+                                                          DecCfg<64>::kSmemBytes);
+    if (e != cudaSuccess || n < 1) return 1;
+    return n;
+}
+
+cudaError_t launch_decode(const CUtensorMap& tmap, const DecodeArgs& a, int n_ctas, int D,
+                          cudaStream_t st) {
+    if (D == 128)
+        sq_decode_splitk_kernel<128>
+            <<<n_ctas, DecCfg<128>::kThreads, DecCfg<128>::kSmemBytes, st>>>(tmap, a);
+    else
+        sq_decode_splitk_kernel<64>
+            <<<n_ctas, DecCfg<64>::kThreads, DecCfg<64>::kSmemBytes, st>>>(tmap, a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_combine(const CombineArgs& a, int D, cudaStream_t st) {
+    const int warps = a.n_seqs * a.Hq;
+    const int blocks = (warps + 7) / 8;
+    if (D == 128) sq_lse_combine_kernel<128><<<blocks, 256, 0, st>>>(a);
+    else sq_lse_combine_kernel<64><<<blocks, 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace sq

@@ -1,0 +1,93 @@
+// Kernel argument blocks and host-side launchers of the sm_103a kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../host/plan.hpp"
+
+namespace sq {
+
+// ---- decode attention -------------------------------------------------------
+struct DecodeArgs {
+    const DecodeSeg* segs;
+    const DecodeItem* items;
+    const int32_t* cta_begin;
+    const int32_t* page_ids;
+    const __nv_bfloat16* q;     // [n_seqs][Hq][D]
+    float* part_o;              // [n_items * 4][16][D]  unnormalised partial outputs
+    float* part_ml;             // [n_items * 4][16][2]  running max (log2 units), sum
+    int32_t layer, Hq, Hkv, G, P, num_pages;
+    float scale_log2;           // sm_scale * log2(e)
+    int* err;
+};
+
+struct CombineArgs {
+    const int32_t* comb_off;    // [n_seqs * Hkv + 1]
+    const CombineEnt* comb_ent;
+    const float* part_o;
+    const float* part_ml;
+    void* out;                  // [n_seqs][Hq][D] bf16 or fp32
+    int32_t out_f32;
+    int32_t n_seqs, Hq, Hkv, G;
+};
+
+// Bytes of partial results one decode plan needs.
+int64_t decode_partial_bytes(int32_t n_items, int32_t D);
+// Persistent CTAs per SM the decode kernel runs with (occupancy of the kernel).
+int decode_ctas_per_sm(int D);
+cudaError_t decode_prepare(int D);  // raises the dynamic shared-memory limit once
+cudaError_t launch_decode(const CUtensorMap& tmap, const DecodeArgs& a, int n_ctas, int D,
+                          cudaStream_t st);
+cudaError_t launch_combine(const CombineArgs& a, int D, cudaStream_t st);
+
+// ---- append / copy-on-write / eviction --------------------------------------
+constexpr int kAppendMaxPages = 64;
+
+struct AppendArgs {
+    __nv_bfloat16* pool;
+    const __nv_bfloat16* k;     // [L][n_total][Hkv][D]
+    const __nv_bfloat16* v;
+    int64_t num_pages;
+    int32_t L, Hkv, P, D;
+    int32_t n_total;            // tokens in the caller's buffers
+    int32_t tok_begin;          // first caller token this launch writes
+    int32_t n_tok;              // tokens this launch writes
+    int32_t pos0;               // logical position of token tok_begin
+    int32_t page_index0;        // logical page index of pages[0]
+    int32_t n_pages;
+    int32_t pages[kAppendMaxPages];
+    int* err;
+};
+
+struct CowArgs {
+    __nv_bfloat16* pool;
+    int64_t num_pages;
+    int32_t L, Hkv, P, D;
+    int32_t src_page, dst_page, rows;
+    int* err;
+};
+
+struct EvictArgs {
+    __nv_bfloat16* pool;
+    int64_t num_pages;
+    int32_t L, Hkv, P, D;
+    const int32_t* old_pt;      // page table before (n_old_pages)
+    const int32_t* new_pt;      // page table after (n_new_pages)
+    const int32_t* run_dst;     // kept runs, destination starts (increasing)
+    const int32_t* run_src;     // kept runs, source starts
+    int32_t n_old_pages, n_new_pages, n_runs;
+    int32_t n_new;              // rows after eviction
+    int32_t first_row;          // first destination row that can change
+    int32_t col_split;          // column pieces per row (1, 2 or 4)
+    int* err;
+};
+
+cudaError_t launch_append(const AppendArgs& a, int num_sms, cudaStream_t st);
+cudaError_t launch_cow_copy(const CowArgs& a, int num_sms, cudaStream_t st);
+int evict_ctas_per_sm();
+cudaError_t launch_evict(const EvictArgs& a, cudaStream_t st);
+
+}  // namespace sq

@@ -1,0 +1,136 @@
+"""ctypes face of libsq_host.so: the library's host-side cache state and
+planners, built without CUDA, for CPU tests."""
+import ctypes
+import os
+import sys
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2602_22603_gb300 import build as _build  # noqa: E402
+
+_lib = None
+
+SEG_INTS = 4 + 2 * 16  # DecodeSeg: page_off, n_pages, n_tok, n_grp, grp_seq[16], grp_lim[16]
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        path = _build.build_host_lib()
+        L = ctypes.CDLL(path)
+        P, I32, I32P, I64P = ctypes.c_void_p, ctypes.c_int32, ctypes.POINTER(ctypes.c_int32), \
+            ctypes.POINTER(ctypes.c_int64)
+        L.sqh_create.restype = P
+        L.sqh_create.argtypes = [I32] * 8
+        L.sqh_destroy.argtypes = [P]
+        L.sqh_seq_new.argtypes = [P, I32P]
+        L.sqh_fork.argtypes = [P, I32, I32P]
+        L.sqh_append.argtypes = [P, I32, I32]
+        L.sqh_evict.argtypes = [P, I32, I32P, I32, I64P]
+        L.sqh_release.argtypes = [P, I32]
+        L.sqh_seq_info.argtypes = [P, I32, I32P, I32P]
+        L.sqh_page_table.argtypes = [P, I32, I32P, I32, I32P]
+        L.sqh_refcount.argtypes = [P, I32]
+        L.sqh_free_count.argtypes = [P]
+        L.sqh_peak_live_pages.argtypes = [P]
+        L.sqh_peak_live_pages.restype = ctypes.c_int64
+        L.sqh_plan_decode.argtypes = [P, I32P, I32, I32, I64P, ctypes.POINTER(ctypes.c_uint8),
+                                      ctypes.c_int64]
+        _lib = L
+    return _lib
+
+
+class HostCache:
+    def __init__(self, L, Hq, Hkv, D, P, num_pages, max_seqs=64, max_pages_per_seq=None):
+        self.h = lib().sqh_create(L, Hq, Hkv, D, P, num_pages, max_seqs,
+                                  max_pages_per_seq or num_pages)
+        assert self.h, "invalid geometry"
+        self.P, self.Hkv, self.G = P, Hkv, Hq // Hkv
+
+    def __del__(self):
+        if getattr(self, "h", None):
+            lib().sqh_destroy(self.h)
+            self.h = None
+
+    def seq_new(self):
+        x = ctypes.c_int32()
+        rc = lib().sqh_seq_new(self.h, ctypes.byref(x))
+        return rc, x.value
+
+    def fork(self, parent):
+        x = ctypes.c_int32()
+        rc = lib().sqh_fork(self.h, parent, ctypes.byref(x))
+        return rc, x.value
+
+    def append(self, h, n):
+        return lib().sqh_append(self.h, h, n)
+
+    def evict(self, h, spans):
+        arr = (ctypes.c_int32 * max(2, 2 * len(spans)))(*[int(x) for ab in spans for x in ab])
+        st = (ctypes.c_int64 * 5)()
+        rc = lib().sqh_evict(self.h, h, arr, len(spans), st)
+        return rc, {"moved_rows": st[0], "cow_pages": st[1], "freed": st[2],
+                    "first_row": st[3], "n_runs": st[4]}
+
+    def release(self, h):
+        return lib().sqh_release(self.h, h)
+
+    def info(self, h):
+        n, p = ctypes.c_int32(), ctypes.c_int32()
+        rc = lib().sqh_seq_info(self.h, h, ctypes.byref(n), ctypes.byref(p))
+        return rc, n.value, p.value
+
+    def page_table(self, h):
+        rc, n, npg = self.info(h)
+        assert rc == 0
+        buf = (ctypes.c_int32 * max(1, npg))()
+        m = ctypes.c_int32()
+        assert lib().sqh_page_table(self.h, h, buf, npg, ctypes.byref(m)) == 0
+        return list(buf[:m.value])
+
+    def refcount(self, p):
+        return lib().sqh_refcount(self.h, p)
+
+    def free_count(self):
+        return lib().sqh_free_count(self.h)
+
+    def peak_live_pages(self):
+        return lib().sqh_peak_live_pages(self.h)
+
+    def plan_decode(self, handles, n_ctas):
+        arr = (ctypes.c_int32 * len(handles))(*handles)
+        lay = (ctypes.c_int64 * 16)()
+        rc = lib().sqh_plan_decode(self.h, arr, len(handles), n_ctas, lay, None, 0)
+        if rc != 0:
+            return rc, None
+        total = lay[6]
+        buf = np.zeros(total, dtype=np.uint8)
+        rc = lib().sqh_plan_decode(self.h, arr, len(handles), n_ctas, lay,
+                                   buf.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)), total)
+        assert rc == 0
+        L = list(lay)
+        assert L[15] == SEG_INTS * 4
+        i32 = buf.view(np.int32)
+
+        def arr_at(off, count, width=1):
+            a = i32[off // 4: off // 4 + count * width]
+            return a.reshape(count, width) if width > 1 else a
+
+        n_segs, n_items, n_ctas_, n_pid, n_keys, n_ent = L[7:13]
+        segs = arr_at(L[0], n_segs, SEG_INTS)
+        plan = {
+            "segs": [{"page_off": int(s[0]), "n_pages": int(s[1]), "n_tok": int(s[2]),
+                      "n_grp": int(s[3]), "grp_seq": [int(x) for x in s[4:4 + s[3]]],
+                      "grp_lim": [int(x) for x in s[20:20 + s[3]]]} for s in segs],
+            "items": arr_at(L[1], n_items, 4).tolist() if n_items else [],
+            "cta_begin": arr_at(L[2], n_ctas_ + 1).tolist(),
+            "page_ids": arr_at(L[3], n_pid).tolist(),
+            "comb_off": arr_at(L[4], n_keys + 1).tolist(),
+            "comb_ent": arr_at(L[5], n_ent, 2).tolist() if n_ent else [],
+            "unique_tokens": L[13], "logical_tokens": L[14],
+        }
+        return 0, plan

@@ -1,0 +1,60 @@
+"""The C-ABI library builds, loads and exports every symbol include/sq.h
+declares; the Python binding carries the same names.  No GPU needed: only
+host-side calls that touch no device are made."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2602_22603_gb300 as sq
+from paper_2602_22603_gb300 import build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "sq.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    return re.findall(r"^SQ_API\s+[\w\s\*]*?\b(sq_\w+)\s*\(", text, flags=re.M)
+
+
+@pytest.fixture(scope="module")
+def libsq():
+    build.build_libsq()
+    return ctypes.CDLL(build.LIBSQ)
+
+
+def test_header_declares_the_six_calls_and_helpers():
+    names = declared_functions()
+    for call in ("sq_cache_create", "sq_append_kv", "sq_fork_aux", "sq_decode_attention",
+                 "sq_evict_spans", "sq_release"):
+        assert call in names
+    assert len(names) == len(set(names))
+
+
+def test_library_exports_every_declared_symbol(libsq):
+    for name in declared_functions():
+        assert hasattr(libsq, name), name
+
+
+def test_binding_has_the_same_names():
+    for name in declared_functions():
+        assert callable(getattr(sq, name)), name
+
+
+def test_host_only_calls(libsq):
+    assert sq.strerror(sq.SQ_ERR_NO_PAGES) == "SQ_ERR_NO_PAGES"
+    cfg = sq.make_config(32, 32, 8, 128, 64, 100)
+    assert sq.sq_pool_bytes(cfg) == 32 * 100 * 2 * 8 * 64 * 128 * 2
+    # geometries the kernels do not handle give 0 bytes
+    assert sq.sq_pool_bytes(sq.make_config(1, 8, 2, 96, 16, 10)) == 0   # head dim 96
+    assert sq.sq_pool_bytes(sq.make_config(1, 8, 2, 64, 12, 10)) == 0   # page size 12
+    assert sq.sq_pool_bytes(sq.make_config(1, 64, 2, 64, 16, 10)) == 0  # group of 32
+    assert sq.sq_pool_bytes(sq.make_config(1, 6, 4, 64, 16, 10)) == 0   # Hq % Hkv != 0
+
+
+def test_null_cache_is_rejected(libsq):
+    out = ctypes.c_int32()
+    assert libsq.sq_seq_new(None, ctypes.byref(out)) == sq.SQ_ERR_BAD_HANDLE
+    assert libsq.sq_cache_destroy(None) == sq.SQ_ERR_BAD_HANDLE

@@ -1,0 +1,297 @@
+"""GPU parity of the CUDA path against the CPU oracle (through the C ABI).
+
+Page tables, token counts, reference counts and post-compaction K/V contents
+must match bit for bit; decode attention within max-abs 1e-2 and mean-abs
+1e-3 of the double-precision oracle."""
+import math
+import random
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2602_22603_gb300 as sq
+from synthetic import TINY, bf16_normal, random_spans, shuffled
+from tests.gpu_harness import MAX_ABS, MEAN_ABS, Pair, assert_close
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2602_22603_gb300 import build
+    build.build_libsq()
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+
+
+def _q(seed, S, Hq, D):
+    q = bf16_normal((S, Hq, D), seed)
+    return q, q.cuda()
+
+
+def _decode_check(p: Pair, seqs, layer, scale, seed):
+    q_cpu, q = _q(seed, len(seqs), p.Hq, p.D)
+    exp = p.oracle_decode(seqs, layer, scale, q_cpu)
+    out32 = p.decode(seqs, layer, scale, q, sq.SQ_OUT_F32)
+    out16 = p.decode(seqs, layer, scale, q, sq.SQ_OUT_BF16)
+    torch.cuda.synchronize()
+    assert p.cache.sync_status() == sq.SQ_OK
+    e32 = assert_close(out32, exp, max_abs=2e-3, mean_abs=2e-4)
+    e16 = assert_close(out16, exp)
+    # the bf16 output is the fp32 output rounded to nearest even
+    assert torch.equal(out16, out32.to(torch.bfloat16))
+    return e32, e16
+
+
+def test_tiny_workload_full_parity():
+    """1 layer, 16 q / 4 kv heads, d 64, P 16, seed 0: 2,048-token prefix,
+    fork, main +32 / aux +64, one decode step each, evict 5 spans (30% of the
+    prefix) from main while the aux is alive, one more decode step each."""
+    s = TINY
+    p = Pair(s.num_layers, s.num_q_heads, s.num_kv_heads, s.head_dim, s.page_size,
+             num_pages=400, seed=0)
+    scale = 1.0 / math.sqrt(s.head_dim)
+    keep = []
+    main = p.seq_new()
+    keep.append(p.append(main, 2048))
+    aux = p.fork(main)
+    p.check_tables()
+    assert p.cache.stats()["live_pages"] == 2048 // 16   # the fork copied nothing
+    keep.append(p.append(main, 32))
+    keep.append(p.append(aux, 64))
+    for step in range(2):
+        keep.append(p.append(main, 1))
+        keep.append(p.append(aux, 1))
+        _decode_check(p, [main, aux], 0, scale, 10 + step)
+        if step == 0:
+            spans = random_spans(seed=1, n_spans=5, total=int(0.3 * 2048), lo=s.page_size,
+                                 hi=2048, median=100)
+            r = p.evict(main, shuffled(spans, 2))
+            assert r["cow_pages"] > 0          # shared changed pages were copied
+        p.check_tables()
+        p.check_contents(main)
+        p.check_contents(aux)
+    st = p.cache.stats()
+    assert st["evict_calls"] == 1 and st["evicted_tokens"] == int(0.3 * 2048)
+    p.close()
+
+
+@pytest.mark.parametrize("P,G,D", [(16, 1, 64), (16, 4, 128), (64, 4, 128), (64, 8, 128),
+                                   (64, 8, 64), (32, 16, 64), (128, 2, 128), (8, 4, 64),
+                                   (256, 4, 128)])
+def test_ragged_lengths(P, G, D):
+    Hkv = 2
+    p = Pair(2, G * Hkv, Hkv, D, P, num_pages=4000 // max(1, P // 16), seed=P * 31 + G * 7 + D)
+    keep = []
+    lengths = [1, P - 1, P, P + 1, 3 * P + 7, 700]
+    seqs = []
+    for n in lengths:
+        h = p.seq_new()
+        keep.append(p.append(h, n))
+        seqs.append(h)
+    p.check_tables()
+    for h in seqs:
+        p.check_contents(h)
+    for layer in range(2):
+        _decode_check(p, seqs, layer, 1.0 / math.sqrt(D), 5 + layer)
+    p.close()
+
+
+def test_split_invariance_over_cta_counts():
+    """The same decode with 1 .. many persistent CTAs (so 1 .. many partials
+    per sequence and head) agrees with the oracle and with itself."""
+    outs = []
+    for ctas in (1, 2, 7, 64, 304, 1000):
+        p = Pair(1, 32, 8, 128, 64, num_pages=600, decode_ctas=ctas, seed=3)
+        keep = []
+        m = p.seq_new()
+        keep.append(p.append(m, 9000))
+        a = p.fork(m)
+        keep.append(p.append(a, 40))
+        keep.append(p.append(m, 3))
+        q_cpu, q = _q(77, 2, 32, 128)
+        out = p.decode([m, a], 0, 0.0884, q, sq.SQ_OUT_F32)
+        torch.cuda.synchronize()
+        exp = p.oracle_decode([m, a], 0, 0.0884, q_cpu)
+        assert_close(out, exp, max_abs=2e-3, mean_abs=2e-4)
+        outs.append(out.cpu())
+        p.close()
+    for o in outs[1:]:
+        assert (o - outs[0]).abs().max().item() < 1e-4
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_random_forks_appends_evictions(seed):
+    rng = random.Random(seed)
+    P = rng.choice([16, 64])
+    D = rng.choice([64, 128])
+    G = rng.choice([1, 4, 8])
+    Hkv = rng.choice([1, 2, 4])
+    L = 2
+    p = Pair(L, G * Hkv, Hkv, D, P, num_pages=3000, seed=seed)
+    keep = []
+    mains = []
+    for _ in range(2):
+        h = p.seq_new()
+        keep.append(p.append(h, rng.randint(P, 60 * P)))
+        mains.append(h)
+    live = list(mains)
+    for it in range(6):
+        h = rng.choice(live)
+        op = rng.random()
+        if op < 0.3 and len(live) < 8:
+            live.append(p.fork(h))
+        elif op < 0.7:
+            keep.append(p.append(h, rng.choice([1, 2, P - 1, P + 3, 5 * P])))
+        else:
+            n = p.cache.seq_info(h)[0]
+            k = rng.randint(1, 6)
+            if n > 4 * k:
+                spans = random_spans(seed=seed * 100 + it, n_spans=k,
+                                     total=rng.randint(k, n // 2), lo=0, hi=n,
+                                     median=max(1, n // (4 * k)))
+                p.evict(h, shuffled(spans, it))
+        p.check_tables()
+        for x in live:
+            p.check_contents(x)
+        _decode_check(p, live, rng.randrange(L), 1.0 / math.sqrt(D), 1000 + it)
+    # releasing forks frees exactly their private pages
+    for x in live[2:]:
+        p.release(x)
+    p.check_tables()
+    p.close()
+
+
+def test_evict_edge_cases():
+    p = Pair(1, 8, 2, 64, 16, num_pages=200, seed=11)
+    keep = []
+    m = p.seq_new()
+    keep.append(p.append(m, 100))
+    snap = p.cache.page_table(m)
+    p.evict(m, [])                                   # no spans: identity
+    assert p.cache.page_table(m) == snap
+    p.check_contents(m)
+    p.evict(m, [(0, 1)])                             # first token
+    p.evict(m, [(98, 99)])                           # last token
+    p.evict(m, [(10, 20), (20, 30)])                 # adjacent spans
+    p.evict(m, [(0, 16)])                            # exactly one page
+    p.check_tables()
+    p.check_contents(m)
+    n = p.cache.seq_info(m)[0]
+    p.evict(m, [(5, n)])                             # everything after a prefix
+    p.check_tables()
+    p.check_contents(m)
+    for bad in ([(3, 2)], [(-1, 2)], [(0, 999)], [(0, 3), (2, 4)]):
+        before = p.cache.page_table(m)
+        with pytest.raises(sq.SqError) as e:
+            p.cache.evict_spans(m, bad)
+        assert e.value.code == sq.SQ_ERR_INVALID_ARG
+        assert p.cache.page_table(m) == before
+    p.evict(m, [(0, 5)])                             # everything: empty sequence
+    assert p.cache.seq_info(m) == (0, 0)
+    out = torch.empty(1, 8, 64, device="cuda")
+    with pytest.raises(sq.SqError) as e:
+        p.cache.decode_attention([m], 0, torch.zeros(1, 8, 64, dtype=torch.bfloat16,
+                                                     device="cuda"), out, sq.SQ_OUT_F32)
+    assert e.value.code == sq.SQ_ERR_INVALID_ARG     # empty-sequence decode
+    keep.append(p.append(m, 20))                     # it can grow again
+    p.check_tables()
+    p.check_contents(m)
+    assert p.cache.sync_status() == sq.SQ_OK
+    p.close()
+
+
+def test_no_pages_is_transactional():
+    p = Pair(1, 4, 1, 64, 16, num_pages=6, seed=5)
+    keep = []
+    m = p.seq_new()
+    keep.append(p.append(m, 90))                     # 6 pages, the last one partial
+    a = p.fork(m)
+    before = (p.cache.page_table(m), p.cache.free_pages())
+    with pytest.raises(sq.SqError) as e:
+        p.cache.append_kv(m, 1, keep[0][0], keep[0][1])
+    assert e.value.code == sq.SQ_ERR_NO_PAGES
+    with pytest.raises(sq.SqError) as e:
+        p.cache.evict_spans(m, [(0, 1)])
+    assert e.value.code == sq.SQ_ERR_NO_PAGES
+    assert (p.cache.page_table(m), p.cache.free_pages()) == before
+    p.release(a)
+    p.evict(m, [(0, 1)])                             # private now: in place
+    p.check_tables()
+    p.check_contents(m)
+    p.close()
+
+
+def test_argument_errors():
+    c = sq.Cache(2, 8, 2, 64, 16, 50)
+    m = c.seq_new()
+    k = torch.zeros(2, 4, 2, 64, dtype=torch.bfloat16, device="cuda")
+    c.append_kv(m, 4, k, k)
+    q = torch.zeros(1, 8, 64, dtype=torch.bfloat16, device="cuda")
+    out = torch.empty(1, 8, 64, device="cuda")
+    for kwargs, code in [
+        (dict(seqs=[m], layer=2), sq.SQ_ERR_INVALID_ARG),
+        (dict(seqs=[m], layer=-1), sq.SQ_ERR_INVALID_ARG),
+        (dict(seqs=[m, m], layer=0), sq.SQ_ERR_INVALID_ARG),
+        (dict(seqs=[m + 1], layer=0), sq.SQ_ERR_BAD_HANDLE),
+    ]:
+        with pytest.raises(sq.SqError) as e:
+            c.decode_attention(kwargs["seqs"], kwargs["layer"], q, out, sq.SQ_OUT_F32)
+        assert e.value.code == code
+    with pytest.raises(sq.SqError) as e:
+        c.decode_attention([m], 0, q, out, 7)
+    assert e.value.code == sq.SQ_ERR_INVALID_ARG
+    with pytest.raises(sq.SqError) as e:                # misaligned input
+        c.append_kv(m, 1, k.view(-1)[1:].data_ptr(), k)
+    assert e.value.code == sq.SQ_ERR_INVALID_ARG
+    with pytest.raises(sq.SqError) as e:
+        c.append_kv(m, -3, k, k)
+    assert e.value.code == sq.SQ_ERR_INVALID_ARG
+    c.release(m)
+    with pytest.raises(sq.SqError) as e:
+        c.append_kv(m, 1, k, k)
+    assert e.value.code == sq.SQ_ERR_BAD_HANDLE
+    assert c.sync_status() == sq.SQ_OK
+    c.close()
+
+
+def test_two_streams_main_and_aux():
+    """Main and aux decode on two streams, interleaved from one host thread
+    (single-agent workload shape, at a reduced size); then the aux is
+    released on its stream and main evicts on its own."""
+    p = Pair(2, 32, 8, 128, 64, num_pages=800, seed=21, k_scale=1 / math.sqrt(128))
+    sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+    keep = []
+    m = p.seq_new()
+    keep.append(p.append(m, 4096))
+    torch.cuda.synchronize()
+    a = p.fork(m)
+    checks = []
+    for step in range(6):
+        with torch.cuda.stream(sa):
+            keep.append(p.append(m, 1, sa))
+            q_cpu, q = _q(500 + step, 1, 32, 128)
+            keep.append(q)
+            out = p.decode([m], step % 2, 1.0, q, sq.SQ_OUT_F32, sa)
+            checks.append((out, p.oracle_decode([m], step % 2, 1.0, q_cpu)))
+        if step % 2 == 0:
+            with torch.cuda.stream(sb):
+                keep.append(p.append(a, 1, sb))
+                q_cpu, q = _q(900 + step, 1, 32, 128)
+                keep.append(q)
+                out = p.decode([a], step % 2, 1.0, q, sq.SQ_OUT_F32, sb)
+                checks.append((out, p.oracle_decode([a], step % 2, 1.0, q_cpu)))
+    torch.cuda.synchronize()
+    for out, exp in checks:
+        assert_close(out, exp, max_abs=2e-3, mean_abs=2e-4)
+    p.release(a, sb)
+    with torch.cuda.stream(sa):
+        spans = random_spans(seed=4, n_spans=12, total=int(0.4 * 4096), lo=64, hi=4096, median=150)
+        p.evict(m, spans, sa)
+        keep.append(p.append(m, 70, sa))     # may reuse pages the aux released on sb
+    torch.cuda.synchronize()
+    p.check_tables()
+    p.check_contents(m)
+    assert p.cache.sync_status() == sq.SQ_OK
+    p.close()

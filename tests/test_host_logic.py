@@ -1,0 +1,204 @@
+"""CPU tests of the library's host logic (page allocator, copy-on-write and
+eviction planning, decode planning), driven through libsq_host.so — the same
+C++ the CUDA library runs on the host — and compared with the oracle."""
+import random
+
+import pytest
+
+from oracle import cache_model as ocm
+from tests.hostlib import HostCache
+
+CODES = {ocm.InvalidArg: -1, ocm.BadHandle: -2, ocm.NoPages: -3, ocm.Capacity: -4}
+STAGE = 64  # tokens per decode stage
+
+
+def oracle_call(fn, *args):
+    try:
+        return 0, fn(*args)
+    except ocm.OracleError as e:
+        return CODES[type(e)], None
+
+
+def random_spans(rng, n, k):
+    if n == 0:
+        return []
+    cuts = sorted(rng.sample(range(n + 1), min(2 * k, n + 1)))
+    spans = [(cuts[i], cuts[i + 1]) for i in range(0, len(cuts) - 1, 2) if cuts[i] < cuts[i + 1]]
+    rng.shuffle(spans)
+    return spans
+
+
+def compare_state(hc, oc, pairs):
+    for h, o in pairs.items():
+        assert hc.page_table(h) == oc.page_table(o)
+        assert hc.info(h)[1] == oc.n_tokens(o)
+    assert hc.free_count() == oc.free_count()
+    for p in range(oc.num_pages):
+        assert hc.refcount(p) == oc.ref[p]
+
+
+@pytest.mark.parametrize("seed", range(16))
+def test_page_tables_match_oracle_bit_exact(seed):
+    rng = random.Random(1000 + seed)
+    P = rng.choice([8, 16, 32, 64])
+    num_pages = rng.choice([24, 64, 150])
+    mpps = rng.choice([None, 12])
+    hc = HostCache(1, 8, 2, 64, P, num_pages, max_seqs=32, max_pages_per_seq=mpps)
+    oc = ocm.OracleCache(num_pages, P, max_pages_per_seq=mpps)
+    pairs = {}
+    rc, h = hc.seq_new()
+    pairs[h] = oc.seq_new()
+    for step in range(150):
+        live = list(pairs)
+        op = rng.random()
+        if not live or op < 0.05:
+            rc, h = hc.seq_new()
+            if rc == 0:
+                pairs[h] = oc.seq_new()
+            continue
+        h = rng.choice(live)
+        o = pairs[h]
+        if op < 0.2:
+            rc, child = hc.fork(h)
+            orc, ochild = oracle_call(oc.fork, o)
+            assert rc == orc
+            if rc == 0:
+                pairs[child] = ochild
+        elif op < 0.6:
+            n = rng.choice([1, 1, 3, P - 1, P, P + 1, 2 * P + 5, 7 * P])
+            rc = hc.append(h, n)
+            orc, _ = oracle_call(oc.append, o, n)
+            assert rc == orc
+        elif op < 0.9:
+            spans = random_spans(rng, oc.n_tokens(o), rng.choice([1, 2, 4, 9]))
+            if rng.random() < 0.1 and spans:
+                spans.append((spans[0][0], spans[0][0] + 1))  # overlap -> rejected
+            rc, st = hc.evict(h, spans)
+            orc, ost = oracle_call(oc.evict, o, spans)
+            assert rc == orc, (spans, rc, orc)
+            if rc == 0 and spans:
+                assert st["moved_rows"] == ost["moved_rows"]
+                assert st["cow_pages"] == ost["cow_pages"]
+        else:
+            assert hc.release(h) == 0
+            oc.release(o)
+            del pairs[h]
+        compare_state(hc, oc, pairs)
+    assert hc.peak_live_pages() == oc.peak_live_pages
+
+
+def test_bad_handles_rejected():
+    hc = HostCache(1, 4, 4, 64, 16, 32)
+    rc, h = hc.seq_new()
+    assert hc.append(h, 5) == 0
+    assert hc.release(h) == 0
+    assert hc.append(h, 1) == -2       # released handle
+    assert hc.fork(h)[0] == -2
+    assert hc.evict(h, [(0, 1)])[0] == -2
+    assert hc.append(12345, 1) == -2
+    assert hc.append(-1, 1) == -2
+    rc, h2 = hc.seq_new()               # the slot is reused with a new generation
+    assert h2 != h
+    assert hc.append(h2, -1) == -1
+
+
+def _check_plan(hc, handles, plan, n_ctas, G):
+    P, Hkv = hc.P, hc.Hkv
+    segs, items = plan["segs"], plan["items"]
+    cb = plan["cta_begin"]
+    assert cb[0] == 0 and cb[-1] == len(items)
+    assert all(cb[i] <= cb[i + 1] for i in range(len(cb) - 1))
+    assert len(cb) - 1 <= n_ctas
+    # stages per CTA are balanced to within one stage
+    per_cta = [sum(items[i][3] - items[i][2] for i in range(cb[c], cb[c + 1]))
+               for c in range(len(cb) - 1)]
+    assert max(per_cta) - min(per_cta) <= 1
+    for s in segs:
+        assert 1 <= s["n_grp"] <= 16 // G
+        assert max(s["grp_lim"]) == s["n_tok"] and min(s["grp_lim"]) > 0
+        assert s["n_tok"] <= s["n_pages"] * P
+    # every (sequence, head) covers its tokens exactly once, through its own pages
+    tables = [hc.page_table(h) for h in handles]
+    ns = [hc.info(h)[1] for h in handles]
+    for i in range(len(handles)):
+        for head in range(Hkv):
+            key = i * Hkv + head
+            ents = plan["comb_ent"][plan["comb_off"][key]:plan["comb_off"][key + 1]]
+            covered = []
+            seg_start = {}
+            for it_idx, j in ents:
+                seg_i, hd, s0, s1 = items[it_idx]
+                s = segs[seg_i]
+                assert hd == head and s["grp_seq"][j] == i
+                # first logical page of the segment: find where its pages sit
+                pids = plan["page_ids"][s["page_off"]:s["page_off"] + s["n_pages"]]
+                q0 = tables[i].index(pids[0])
+                assert tables[i][q0:q0 + s["n_pages"]] == pids
+                lim = s["grp_lim"][j]
+                lo, hi = s0 * STAGE, min(s1 * STAGE, lim)
+                if hi > lo:
+                    covered.append((q0 * P + lo, q0 * P + hi))
+            covered.sort()
+            pos = 0
+            for a, b in covered:
+                assert a == pos
+                pos = b
+            assert pos == ns[i]
+
+
+@pytest.mark.parametrize("seed", range(10))
+def test_decode_plan_covers_every_token_once(seed):
+    rng = random.Random(seed)
+    P = rng.choice([8, 16, 64, 128])
+    G = rng.choice([1, 4, 8, 16])
+    Hkv = rng.choice([1, 2, 8])
+    hc = HostCache(2, G * Hkv, Hkv, 128, P, 4000, max_seqs=64)
+    mains = []
+    for _ in range(rng.randint(1, 4)):
+        rc, h = hc.seq_new()
+        assert hc.append(h, rng.randint(1, 40 * P)) == 0
+        mains.append(h)
+    seqs = list(mains)
+    for h in mains:
+        for _ in range(rng.randint(0, 3)):
+            rc, a = hc.fork(h)
+            assert rc == 0
+            assert hc.append(a, rng.randint(0, 3 * P)) == 0
+            seqs.append(a)
+        assert hc.append(h, rng.randint(0, 2 * P)) == 0
+        if rng.random() < 0.5:
+            n = hc.info(h)[1]
+            hc.evict(h, random_spans(rng, n, 3))
+    rng.shuffle(seqs)
+    for n_ctas in (1, 3, 152, 304, 5000):
+        rc, plan = hc.plan_decode(seqs, n_ctas)
+        assert rc == 0
+        _check_plan(hc, seqs, plan, n_ctas, G)
+        assert plan["logical_tokens"] == sum(hc.info(h)[1] for h in seqs)
+        assert plan["unique_tokens"] <= plan["logical_tokens"]
+
+
+def test_decode_plan_reads_shared_prefix_once():
+    # main + fork with a 4096-token shared prefix: the shared pages form one
+    # segment read for both query groups (Sec. 3.4, shared-context kernels)
+    hc = HostCache(1, 32, 8, 128, 64, 1000)
+    rc, m = hc.seq_new()
+    hc.append(m, 4096)
+    rc, a = hc.fork(m)
+    hc.append(a, 8)
+    hc.append(m, 1)
+    rc, plan = hc.plan_decode([m, a], 304)
+    assert rc == 0
+    shared = [s for s in plan["segs"] if s["n_grp"] == 2]
+    assert len(shared) == 1 and shared[0]["n_tok"] == 4096
+    assert plan["unique_tokens"] == 4096 + 1 + 8
+    assert plan["logical_tokens"] == 4097 + 4104
+
+
+def test_decode_plan_rejects_bad_input():
+    hc = HostCache(1, 8, 2, 64, 16, 100)
+    rc, m = hc.seq_new()
+    assert hc.plan_decode([m], 10)[0] == -1          # empty sequence
+    hc.append(m, 5)
+    assert hc.plan_decode([m, m], 10)[0] == -1       # duplicate
+    assert hc.plan_decode([m, 999], 10)[0] == -2     # bad handle
