@@ -48,6 +48,11 @@ __device__ __forceinline__ uint32_t ld_u32(const __nv_bfloat16* p) {
     return *reinterpret_cast<const uint32_t*>(p);
 }
 
+// Sum of the two bf16 halves of a packed pair, in fp32.
+__device__ __forceinline__ float bf16x2_sum(uint32_t v) {
+    return __uint_as_float(v << 16) + __uint_as_float(v & 0xffff0000u);
+}
+
 // ---- producer: one thread issues the TMA loads of every stage -------------
 template <int D>
 __device__ void produce(const CUtensorMap* tmap, const DecodeArgs& a, int it0, int it1,
@@ -220,16 +225,22 @@ __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, ui
             const float al0 = exp2f(m0 - ms0), al1 = exp2f(m1 - ms1);
             m0 = mn0;
             m1 = mn1;
-            float ps0 = 0.f, ps1 = 0.f;
 #pragma unroll
             for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
                 for (int e = 0; e < 2; ++e) {
                     x[nt][e] = exp2f(x[nt][e] - ms0);
                     x[nt][2 + e] = exp2f(x[nt][2 + e] - ms1);
-                    ps0 += x[nt][e];
-                    ps1 += x[nt][2 + e];
                 }
+            // P in bf16 for the PV product; the normaliser sums the same
+            // rounded weights, so the output is an exact convex combination
+            uint32_t pa[4];
+            pa[0] = pack_bf16x2(x[0][0], x[0][1]);
+            pa[1] = pack_bf16x2(x[0][2], x[0][3]);
+            pa[2] = pack_bf16x2(x[1][0], x[1][1]);
+            pa[3] = pack_bf16x2(x[1][2], x[1][3]);
+            const float ps0 = bf16x2_sum(pa[0]) + bf16x2_sum(pa[2]);
+            const float ps1 = bf16x2_sum(pa[1]) + bf16x2_sum(pa[3]);
             l0 = l0 * al0 + ps0;
             l1 = l1 * al1 + ps1;
 #pragma unroll
@@ -239,11 +250,6 @@ __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, ui
                 o[nd][2] *= al1;
                 o[nd][3] *= al1;
             }
-            uint32_t pa[4];
-            pa[0] = pack_bf16x2(x[0][0], x[0][1]);
-            pa[1] = pack_bf16x2(x[0][2], x[0][3]);
-            pa[2] = pack_bf16x2(x[1][0], x[1][1]);
-            pa[3] = pack_bf16x2(x[1][2], x[1][3]);
 
             // Rows past the last valid token hold stale or never-written
             // shared memory: zero this warp's such V rows so 0 * V stays 0.
