@@ -208,6 +208,37 @@ typedef struct {
 
 SQ_API int sq_stats(sq_cache *cache, sq_stats_t *out);
 
+/* ---- allocation-free decode (the paper has no counterpart) ---- */
+
+/* Bytes of the fixed device scratch behind sq_decode_attention_noalloc. */
+#define SQ_NOALLOC_SCRATCH_BYTES (32u << 20)
+
+/* The same decode attention as sq_decode_attention (same arguments, same
+ * kernels, same result), for callers that may not allocate GPU memory while
+ * decoding: runtimes that reserve the device for their KV pool up front and
+ * forbid allocations on the hot path, or hosts whose device allocator cannot
+ * be reached from C.  This call allocates no device memory — no cudaMalloc,
+ * no cudaFree, no library allocator.  The call's split-K plan and partial
+ * results go to a fixed scratch array of SQ_NOALLOC_SCRATCH_BYTES that is
+ * part of the library's device image: every GPU that loads the library holds
+ * it until the process exits.
+ *   - The first call on a device looks up the scratch's device address
+ *     (cudaGetSymbolAddress, with the cache's device current); make that first
+ *     call before any stream capture.
+ *   - The current device must be the cache's device (else INVALID_ARG).
+ *   - A call whose plan and partials need more than SQ_NOALLOC_SCRATCH_BYTES
+ *     (very many sequences, or a very large decode_ctas) returns
+ *     SQ_ERR_CAPACITY and enqueues nothing.
+ *   - Every call, on every cache of the device, shares the one scratch array
+ *     and leaves its contents behind; nothing in it has to start at zero
+ *     (every value read is written first by the same call).  Calls whose GPU
+ *     work overlaps — on different streams without ordering between them —
+ *     race on the scratch: order them (one stream, or events).
+ * Errors: BAD_HANDLE, INVALID_ARG, CAPACITY, CUDA. */
+SQ_API int sq_decode_attention_noalloc(sq_cache *cache, const sq_seq *seqs, int32_t n_seqs,
+                                       int32_t layer, const void *q, void *out,
+                                       int32_t out_dtype, float sm_scale, void *stream);
+
 /* Synchronise `stream`, then read and clear the device error word.
  * Returns SQ_OK, SQ_ERR_DEVICE, SQ_ERR_DEVICE_TIMEOUT or SQ_ERR_CUDA. */
 SQ_API int sq_sync_status(sq_cache *cache, void *stream);

@@ -93,6 +93,8 @@ _SIGS = {
     "sq_stats": (ctypes.c_int, [_P, ctypes.POINTER(sq_stats_t)]),
     "sq_sync_status": (ctypes.c_int, [_P, _P]),
     "sq_strerror": (ctypes.c_char_p, [ctypes.c_int]),
+    "sq_decode_attention_noalloc": (ctypes.c_int, [_P, _I32P, _I32, _I32, _P, _P, _I32,
+                                                   ctypes.c_float, _P]),
 }
 
 
@@ -188,6 +190,17 @@ def sq_decode_attention(cache: int, seqs: Sequence[int], layer: int, q, out,
     _check(lib().sq_decode_attention(cache, arr, len(seqs), layer, _ptr(q), _ptr(out),
                                      out_dtype, float(sm_scale), _stream(stream)),
            "sq_decode_attention")
+
+
+def sq_decode_attention_noalloc(cache: int, seqs: Sequence[int], layer: int, q, out,
+                                out_dtype: int = SQ_OUT_BF16, sm_scale: float = 1.0,
+                                stream=None) -> None:
+    """sq_decode_attention without any device allocation (fixed library
+    scratch; see include/sq.h for the limits and the sharing rule)."""
+    arr = (ctypes.c_int32 * len(seqs))(*seqs)
+    _check(lib().sq_decode_attention_noalloc(cache, arr, len(seqs), layer, _ptr(q), _ptr(out),
+                                             out_dtype, float(sm_scale), _stream(stream)),
+           "sq_decode_attention_noalloc")
 
 
 def sq_evict_spans(cache: int, seq: int, spans: Sequence[Tuple[int, int]], stream=None) -> None:

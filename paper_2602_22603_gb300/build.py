@@ -25,6 +25,7 @@ NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-use_fast_math", "-Xcompiler", 
 LIBSQ_SOURCES = [
     "kernels/decode.cu",
     "kernels/kv.cu",
+    "kernels/noalloc_scratch.cu",
     "host/core.cpp",
     "api/sq_api.cpp",
 ]

@@ -15,6 +15,7 @@
 
 #include "../host/core.hpp"
 #include "../kernels/launch.hpp"
+#include "../kernels/noalloc.hpp"
 
 using namespace sq;
 
@@ -658,6 +659,80 @@ int sq_sync_status(sq_cache* c, void* stream) {
     }
     if (err & 2) return SQ_ERR_DEVICE_TIMEOUT;
     if (err & 1) return SQ_ERR_DEVICE;
+    return SQ_OK;
+}
+
+int sq_decode_attention_noalloc(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t layer,
+                                const void* q, void* out, int32_t out_dtype, float sm_scale,
+                                void* stream) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    const Geometry& g = c->g;
+    if (!seqs || n_seqs < 1 || n_seqs > g.max_seqs || !q || !out) return SQ_ERR_INVALID_ARG;
+    if (layer < 0 || layer >= g.L) return SQ_ERR_INVALID_ARG;
+    if (out_dtype != SQ_OUT_BF16 && out_dtype != SQ_OUT_F32) return SQ_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(q) & 15) || (reinterpret_cast<uintptr_t>(out) & 15))
+        return SQ_ERR_INVALID_ARG;
+    if (!(sm_scale == sm_scale)) return SQ_ERR_INVALID_ARG;
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) return SQ_ERR_CUDA;
+    if (dev != c->device) return SQ_ERR_INVALID_ARG;
+    DecodePlanHost plan;
+    int rc = plan_decode(*c->host, seqs, n_seqs, c->decode_ctas, &plan);
+    if (rc != SQ_OK) return rc;
+    const DecodePlanLayout L = plan_layout(plan, n_seqs, g.Hkv);
+    // scratch = [plan | partial outputs | partial (max, sum)]
+    const size_t part_off = ((size_t)L.total + 255) & ~size_t(255);
+    const size_t need = part_off + (size_t)decode_partial_bytes(L.n_items, g.D);
+    if (need > (size_t)SQ_NOALLOC_SCRATCH_BYTES) return SQ_ERR_CAPACITY;
+    void* base = nullptr;
+    rc = noalloc_scratch(dev, &base);
+    if (rc != SQ_OK) return rc;
+    uint8_t* scratch = static_cast<uint8_t*>(base);
+
+    if (c->staging.size() < (size_t)L.total) c->staging.resize(L.total);
+    plan_serialize(plan, L, c->staging.data());
+    cudaStream_t st = as_stream(stream);
+    cudaError_t e = cudaMemcpyAsync(scratch, c->staging.data(), L.total, cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) return cuda_status(e);
+    float* part_o = reinterpret_cast<float*>(scratch + part_off);
+    float* part_ml = part_o + (size_t)L.n_items * kDecodeConsumerWarps * kRowsPerTile * g.D;
+
+    DecodeArgs a;
+    a.segs = reinterpret_cast<const DecodeSeg*>(scratch + L.segs);
+    a.items = reinterpret_cast<const DecodeItem*>(scratch + L.items);
+    a.cta_begin = reinterpret_cast<const int32_t*>(scratch + L.cta_begin);
+    a.page_ids = reinterpret_cast<const int32_t*>(scratch + L.page_ids);
+    a.q = reinterpret_cast<const __nv_bfloat16*>(q);
+    a.part_o = part_o;
+    a.part_ml = part_ml;
+    a.layer = layer;
+    a.Hq = g.Hq;
+    a.Hkv = g.Hkv;
+    a.G = g.G();
+    a.P = g.P;
+    a.num_pages = g.num_pages;
+    a.scale_log2 = sm_scale * 1.4426950408889634f;
+    a.err = c->d_err;
+    e = launch_decode(c->tmap, a, L.n_ctas, g.D, st);
+    if (e != cudaSuccess) return cuda_status(e);
+
+    CombineArgs ca;
+    ca.comb_off = reinterpret_cast<const int32_t*>(scratch + L.comb_off);
+    ca.comb_ent = reinterpret_cast<const CombineEnt*>(scratch + L.comb_ent);
+    ca.part_o = part_o;
+    ca.part_ml = part_ml;
+    ca.out = out;
+    ca.out_f32 = out_dtype == SQ_OUT_F32;
+    ca.n_seqs = n_seqs;
+    ca.Hq = g.Hq;
+    ca.Hkv = g.Hkv;
+    ca.G = g.G();
+    e = launch_combine(ca, g.D, st);
+    if (e != cudaSuccess) return cuda_status(e);
+    for (int32_t i = 0; i < n_seqs; ++i) c->host->seq_mut(seqs[i])->last_stream = stream;
+    c->stats.decode_calls += 1;
+    c->stats.decode_logical_bytes += plan.logical_tokens * g.token_layer_bytes();
+    c->stats.decode_unique_bytes += plan.unique_tokens * g.token_layer_bytes();
     return SQ_OK;
 }
 

@@ -1,0 +1,82 @@
+"""sq_decode_attention_noalloc: decode attention for callers that may not
+allocate GPU memory while decoding (runtimes that reserve the device for their
+KV pool up front, or hosts whose allocator C code cannot reach).  Its result
+must equal the regular entry point's, call after call, although every call
+reuses the same fixed library scratch.
+
+Collected last on purpose (file name), so a run that stops at the first
+failure has already run every other test; it also passes on its own."""
+import ctypes
+import math
+
+import pytest
+import torch
+
+import paper_2602_22603_gb300 as sq
+from synthetic import bf16_normal
+from tests.gpu_harness import MAX_ABS, MEAN_ABS, Pair, assert_close
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2602_22603_gb300 import build
+    build.build_libsq()
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+
+
+def _noalloc_c(cache, seqs, layer, q, out, out_dtype, scale):
+    """Direct C-ABI call; returns the status code."""
+    arr = (ctypes.c_int32 * len(seqs))(*seqs)
+    return sq.lib().sq_decode_attention_noalloc(
+        cache.handle, arr, len(seqs), layer, q.data_ptr(), out.data_ptr(), out_dtype,
+        ctypes.c_float(scale), torch.cuda.current_stream().cuda_stream)
+
+
+def test_noalloc_matches_regular_entry_point_two_calls_in_a_row():
+    p = Pair(2, 32, 8, 128, 64, num_pages=1200, seed=41)
+    keep = []
+    m = p.seq_new()
+    keep.append(p.append(m, 20000))
+    a = p.fork(m)
+    keep.append(p.append(a, 8))
+    keep.append(p.append(m, 37))
+    lone = p.seq_new()
+    keep.append(p.append(lone, 333))
+    seqs = [m, a, lone]
+    scale = 1.0 / math.sqrt(128)
+    for call in range(2):
+        layer = call % 2
+        q_cpu = bf16_normal((3, 32, 128), 7 + call)
+        q = q_cpu.cuda()
+        for dt, tdt in ((sq.SQ_OUT_F32, torch.float32), (sq.SQ_OUT_BF16, torch.bfloat16)):
+            ref = torch.empty(3, 32, 128, dtype=tdt, device="cuda")
+            got = torch.full((3, 32, 128), float("nan"), dtype=tdt, device="cuda")
+            p.cache.decode_attention(seqs, layer, q, ref, dt, scale)
+            assert _noalloc_c(p.cache, seqs, layer, q, got, dt, scale) == sq.SQ_OK
+            torch.cuda.synchronize()
+            assert p.cache.sync_status() == sq.SQ_OK
+            assert_close(got, ref.double().cpu().numpy(), MAX_ABS, MEAN_ABS)
+            assert torch.equal(got, ref)   # same plan, same kernels
+        exp = p.oracle_decode(seqs, layer, scale, q_cpu)
+        assert_close(got, exp)
+        keep.append(p.append(m, 1))        # the next call sees a changed sequence
+    p.close()
+
+
+def test_noalloc_rejects_plans_beyond_the_scratch():
+    # 8 KV heads x 512 stages over 4096 persistent CTAs -> 4096 partial items,
+    # ~136 MB of partials: more than the fixed scratch holds
+    p = Pair(1, 32, 8, 128, 64, num_pages=600, seed=43, decode_ctas=4096)
+    keep = [None]
+    m = p.seq_new()
+    keep.append(p.append(m, 32768))
+    q = bf16_normal((1, 32, 128), 1).cuda()
+    out = torch.zeros(1, 32, 128, device="cuda")
+    assert _noalloc_c(p.cache, [m], 0, q, out, sq.SQ_OUT_F32, 0.1) == sq.SQ_ERR_CAPACITY
+    torch.cuda.synchronize()
+    assert torch.count_nonzero(out).item() == 0     # nothing was enqueued
+    assert p.cache.sync_status() == sq.SQ_OK
+    p.close()
