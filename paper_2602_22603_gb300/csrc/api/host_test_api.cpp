@@ -50,6 +50,28 @@ int sqh_evict(void* c, int32_t h, const int32_t* spans, int32_t n_spans, int64_t
     return rc;
 }
 
+// Evicts and returns the compaction tiles (4 ints each: dst_page, dst_slot,
+// n_rows, piece_begin) and pieces (src_page, src_slot, n_rows, dst_row).
+int sqh_evict_tiles(void* c, int32_t h, const int32_t* spans, int32_t n_spans, int32_t tile_rows,
+                    int32_t* tiles_out, int32_t tiles_cap, int32_t* pieces_out,
+                    int32_t pieces_cap, int32_t* n_tiles, int32_t* n_pieces) {
+    HostCache* hc = static_cast<HostCache*>(c);
+    std::vector<int32_t> a(n_spans > 0 ? n_spans : 0), b(a.size());
+    for (int32_t i = 0; i < n_spans; ++i) { a[i] = spans[2 * i]; b[i] = spans[2 * i + 1]; }
+    EvictPlan p;
+    int rc = hc->evict(h, a.data(), b.data(), n_spans, &p);
+    if (rc != kOk) return rc;
+    std::vector<EvictTile> tiles;
+    std::vector<EvictPiece> pieces;
+    evict_tiles(p, hc->geom().P, tile_rows, &tiles, &pieces);
+    *n_tiles = (int32_t)tiles.size();
+    *n_pieces = (int32_t)pieces.size();
+    if ((int32_t)tiles.size() > tiles_cap || (int32_t)pieces.size() > pieces_cap) return kInvalidArg;
+    std::memcpy(tiles_out, tiles.data(), tiles.size() * sizeof(EvictTile));
+    std::memcpy(pieces_out, pieces.data(), pieces.size() * sizeof(EvictPiece));
+    return kOk;
+}
+
 int sqh_release(void* c, int32_t h) { return static_cast<HostCache*>(c)->release(h, nullptr); }
 
 int sqh_seq_info(void* c, int32_t h, int32_t* n_tokens, int32_t* n_pages) {

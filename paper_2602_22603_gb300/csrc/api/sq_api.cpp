@@ -55,7 +55,7 @@ struct sq_cache {
     int device = 0;
     int num_sms = 0;
     int decode_ctas = 0;
-    int evict_slots = 0;
+    int evict_tile_rows = 0;
     __nv_bfloat16* pool = nullptr;
     bool own_pool = false;
     size_t pool_bytes = 0;
@@ -197,12 +197,16 @@ void free_entry(PlanEntry& p) {
     p = PlanEntry();
 }
 
-int choose_col_split(const sq_cache* c) {
+// Rows per eviction tile: the largest (up to 64, at most a page) for which
+// one CTA per (layer, K/V, head) plane still fits in one wave of resident CTAs.
+int choose_tile_rows(const sq_cache* c) {
     const int64_t planes = (int64_t)c->g.L * 2 * c->g.Hkv;
-    const int row_bytes = c->g.D * 2;
-    for (int cs = 4; cs >= 2; cs >>= 1)
-        if (row_bytes / cs >= 64 && planes * cs <= c->evict_slots) return cs;
-    return 1;
+    int best = 0;
+    for (int tr = std::min(c->g.P, kStageTokens); tr >= 8; tr >>= 1) {
+        best = tr;
+        if (planes <= (int64_t)c->num_sms * evict_ctas_per_sm(tr, c->g.D)) break;
+    }
+    return best;
 }
 
 }  // namespace
@@ -254,7 +258,9 @@ int sq_cache_create(const sq_config* cfg, sq_cache** out) {
     e = decode_prepare(g.D);
     if (e != cudaSuccess) return cuda_status(e);
     c->decode_ctas = cfg->decode_ctas > 0 ? cfg->decode_ctas : c->num_sms * decode_ctas_per_sm(g.D);
-    c->evict_slots = c->num_sms * evict_ctas_per_sm();
+    e = evict_prepare();
+    if (e != cudaSuccess) return cuda_status(e);
+    c->evict_tile_rows = choose_tile_rows(c.get());
     c->pool_bytes = pool_bytes_of(g);
     if (cfg->kv_pool) {
         c->pool = reinterpret_cast<__nv_bfloat16*>(cfg->kv_pool);
@@ -530,33 +536,26 @@ int sq_evict_spans(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_span
     rc = fence_taken_pages(c, plan.cow_pages, stream);
     if (rc != SQ_OK) return undo(rc);
     if (plan.first_row < plan.n_new) {
-        // upload: old page table, new page table, run starts (dst, src)
-        const size_t n_old = plan.old_pages.size(), n_new = plan.new_pages.size();
-        const size_t n_runs = plan.run_dst.size();
-        std::vector<int32_t> buf(n_old + n_new + 2 * n_runs);
-        std::copy(plan.old_pages.begin(), plan.old_pages.end(), buf.begin());
-        std::copy(plan.new_pages.begin(), plan.new_pages.end(), buf.begin() + n_old);
-        std::copy(plan.run_dst.begin(), plan.run_dst.end(), buf.begin() + n_old + n_new);
-        std::copy(plan.run_src.begin(), plan.run_src.end(), buf.begin() + n_old + n_new + n_runs);
+        std::vector<EvictTile> tiles;
+        std::vector<EvictPiece> pieces;
+        evict_tiles(plan, g.P, c->evict_tile_rows, &tiles, &pieces);
+        const size_t tb = tiles.size() * sizeof(EvictTile);
+        std::vector<uint8_t> buf(tb + pieces.size() * sizeof(EvictPiece));
+        std::memcpy(buf.data(), tiles.data(), tb);
+        std::memcpy(buf.data() + tb, pieces.data(), pieces.size() * sizeof(EvictPiece));
         UploadSlot& s = c->slots[c->next_slot];
         c->next_slot = (c->next_slot + 1) % kUploadSlots;
-        rc = upload(c, s, buf.data(), buf.size() * sizeof(int32_t), stream);
+        rc = upload(c, s, buf.data(), buf.size(), stream);
         if (rc != SQ_OK) return undo(rc);
-        const int32_t* d = reinterpret_cast<const int32_t*>(s.d);
         EvictArgs ea;
         ea.pool = c->pool;
         ea.num_pages = g.num_pages;
         ea.L = g.L; ea.Hkv = g.Hkv; ea.P = g.P; ea.D = g.D;
-        ea.old_pt = d;
-        ea.new_pt = d + n_old;
-        ea.run_dst = d + n_old + n_new;
-        ea.run_src = d + n_old + n_new + n_runs;
-        ea.n_old_pages = (int32_t)n_old;
-        ea.n_new_pages = (int32_t)n_new;
-        ea.n_runs = (int32_t)n_runs;
-        ea.n_new = plan.n_new;
-        ea.first_row = plan.first_row;
-        ea.col_split = choose_col_split(c);
+        ea.tiles = reinterpret_cast<const EvictTile*>(s.d);
+        ea.pieces = reinterpret_cast<const EvictPiece*>(s.d + tb);
+        ea.n_tiles = (int32_t)tiles.size();
+        ea.n_pieces = (int32_t)pieces.size();
+        ea.tile_rows = c->evict_tile_rows;
         ea.err = c->d_err;
         cudaError_t e = launch_evict(ea, st);
         if (e != cudaSuccess) return undo(cuda_status(e));

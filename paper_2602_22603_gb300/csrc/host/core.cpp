@@ -292,6 +292,57 @@ int HostCache::release(int32_t h, std::vector<int32_t>* freed) {
     return kOk;
 }
 
+void evict_tiles(const EvictPlan& p, int32_t P, int32_t tile_rows,
+                 std::vector<EvictTile>* tiles, std::vector<EvictPiece>* pieces) {
+    tiles->clear();
+    pieces->clear();
+    if (p.first_row >= p.n_new) return;
+    size_t r = 0;  // current kept run (monotone in the destination row)
+    const int32_t first_q = p.first_row / P;
+    const int32_t new_np = (int32_t)p.new_pages.size();
+    for (int32_t q = first_q; q < new_np; ++q) {
+        const int32_t page_begin = q * P;
+        const int32_t row_end = std::min<int64_t>((int64_t)page_begin + P, p.n_new);
+        const bool fresh = p.new_pages[q] != p.old_pages[q];
+        int32_t row = page_begin;
+        if (!fresh) {
+            // skip destination rows that keep their row (kept[j] == j)
+            while (row < row_end) {
+                while (r + 1 < p.run_dst.size() && p.run_dst[r + 1] <= row) ++r;
+                const int32_t src = p.run_src[r] + (row - p.run_dst[r]);
+                if (src != row) break;
+                // the whole rest of this run keeps its rows
+                row = std::min<int32_t>(row_end, p.run_dst[r] + p.run_len[r]);
+            }
+        }
+        while (row < row_end) {
+            const int32_t t_end = std::min(row_end, row + tile_rows);
+            EvictTile t;
+            t.dst_page = p.new_pages[q];
+            t.dst_slot = row - page_begin;
+            t.n_rows = t_end - row;
+            t.piece_begin = (int32_t)pieces->size();
+            int32_t j = row;
+            while (j < t_end) {
+                while (r + 1 < p.run_dst.size() && p.run_dst[r + 1] <= j) ++r;
+                const int32_t src = p.run_src[r] + (j - p.run_dst[r]);
+                const int32_t run_left = p.run_dst[r] + p.run_len[r] - j;
+                const int32_t page_left = P - src % P;
+                const int32_t n = std::min({t_end - j, run_left, page_left});
+                EvictPiece pc;
+                pc.src_page = p.old_pages[src / P];
+                pc.src_slot = src % P;
+                pc.n_rows = n;
+                pc.dst_row = j - row;
+                pieces->push_back(pc);
+                j += n;
+            }
+            tiles->push_back(t);
+            row = t_end;
+        }
+    }
+}
+
 // ---------------------------------------------------------------------------
 // decode planning
 

@@ -132,6 +132,15 @@ class HostCache {
     int64_t peak_live_ = 0;
 };
 
+// Splits the rows an eviction writes into tiles of at most `tile_rows`
+// rows inside one destination page, in increasing logical order, and each
+// tile into contiguous source pieces (a piece never crosses a kept-run or a
+// source-page boundary).  Every source of a tile lies at a logical position
+// >= the tile's first destination row, so processing tiles in order, each
+// tile's reads before its writes, compacts in place.
+void evict_tiles(const EvictPlan& p, int32_t P, int32_t tile_rows,
+                 std::vector<EvictTile>* tiles, std::vector<EvictPiece>* pieces);
+
 // ---- decode planning -------------------------------------------------------
 
 struct DecodePlanHost {

@@ -38,6 +38,24 @@ struct CombineEnt {
     int32_t j;
 };
 
+// Eviction compaction, planned once per eviction and shared by every
+// (layer, K/V, head) plane: destination tiles (contiguous rows of one page, in
+// increasing logical order) and, per tile, the contiguous source pieces that
+// fill it.
+struct EvictTile {
+    int32_t dst_page;
+    int32_t dst_slot;     // first destination slot in the page
+    int32_t n_rows;       // rows written (<= tile capacity)
+    int32_t piece_begin;  // pieces [piece_begin, next tile's piece_begin)
+};
+
+struct EvictPiece {
+    int32_t src_page;
+    int32_t src_slot;
+    int32_t n_rows;
+    int32_t dst_row;      // row offset inside the tile
+};
+
 // Byte offsets of the arrays of a decode plan inside one upload buffer.
 struct DecodePlanLayout {
     int64_t segs, items, cta_begin, page_ids, comb_off, comb_ent, total;

@@ -69,105 +69,105 @@ __global__ void __launch_bounds__(256) sq_cow_copy_kernel(const CowArgs a) {
 //
 // Algorithm 1, C.clear_kv(Delta_ids): the j-th kept row moves to position j.
 // Since the kept positions increase, the source of destination row j is at
-// position >= j.  One CTA owns one (layer, K/V, head) plane (or a column
-// piece of it) and walks its destination tiles left to right.  The sources
-// of tile t sit at positions >= t*R, so
-//   * writes of tile t (positions in [t*R, (t+1)*R)) can only clobber sources
-//     of tiles <= t; all of tile t's sources are in shared memory (cp.async
-//     waited, then a CTA barrier) before any of its writes;
-//   * loads of later tiles (positions >= (t+1)*R) never overlap writes of
-//     tile t, so they are issued ahead (a 3-stage cp.async ring).
-// Destination pages that were copied on write are fresh pages that hold no
-// source row, so all their rows are written; other destination rows are
-// skipped when they do not move.
-constexpr int kEvictThreads = 128;
-constexpr int kEvictVecsPerThread = 4;
-constexpr int kEvictTileVecs = kEvictThreads * kEvictVecsPerThread;  // 8 KB per stage
-constexpr int kEvictStages = 3;
-
-__device__ __forceinline__ int kept_source(const int32_t* run_dst, const int32_t* run_src,
-                                           int n_runs, int j) {
-    int lo = 0, hi = n_runs - 1;  // last run with run_dst <= j
-    while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (__ldg(run_dst + mid) <= j) lo = mid;
-        else hi = mid - 1;
-    }
-    return __ldg(run_src + lo) + (j - __ldg(run_dst + lo));
-}
-
-__global__ void __launch_bounds__(kEvictThreads) sq_evict_compact_kernel(const EvictArgs a) {
-    __shared__ __align__(16) uint8_t buf[kEvictStages][kEvictTileVecs * 16];
-    const int plane = blockIdx.x / a.col_split;
-    const int piece = blockIdx.x % a.col_split;
+// position >= j.  The host splits the rows that change into destination
+// tiles (contiguous rows of one page, increasing logical order) and each tile
+// into contiguous source pieces; the list is the same for every
+// (layer, K/V, head) plane.  One CTA owns one plane; one thread drives it
+// with 1-D bulk copies (TMA):
+//   * bulk loads of tile t's pieces land in a shared-memory slot, tracked by
+//     an mbarrier (expect-tx);
+//   * after the barrier completes, one bulk store writes the tile back;
+//   * the slot is refilled (tile t + S - 1) once that store has read it.
+// All sources of tile t sit at positions >= its first destination row, so
+// (a) every source a store of tile t could overwrite belongs to tile t or an
+// earlier tile, whose loads have all completed before the store is issued,
+// and (b) the loads issued ahead for later tiles read positions past every
+// row written so far.  Copy-on-write destination pages are fresh pages that
+// hold no source row.  No inter-CTA wait is needed.
+__global__ void __launch_bounds__(32) sq_evict_compact_kernel(const EvictArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    if (threadIdx.x != 0) return;
+    constexpr int S = kEvictStages;
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
+    const uint32_t row_bytes = (uint32_t)a.D * 2u;
+    const uint32_t tile_bytes = (uint32_t)a.tile_rows * row_bytes;
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + S * tile_bytes);
+    const int plane = blockIdx.x;
     const int head = plane % a.Hkv;
     const int kv = (plane / a.Hkv) % 2;
     const int layer = plane / (2 * a.Hkv);
-    const int vpr = a.D / 8 / a.col_split;       // vectors per row piece
-    const int rows_per_tile = kEvictTileVecs / vpr;
-    const int col0 = piece * vpr * 8;            // first element of the piece
-    const int tid = threadIdx.x;
-    const int vc = tid % vpr;
-    const int row_lane = tid / vpr;
-    const int row_step = kEvictThreads / vpr;
+    uint8_t* base = reinterpret_cast<uint8_t*>(a.pool) +
+                    row_offset(a.num_pages, a.Hkv, a.P, a.D, layer, 0, kv, head, 0) * 2;
+    const int64_t page_stride = (int64_t)2 * a.Hkv * a.P * row_bytes;  // bytes between pages
+    for (int s = 0; s < S; ++s) mbar_init(smem_addr(&full[s]), 1);
+    fence_mbar_init();
 
-    const int t_first = a.first_row / rows_per_tile;
-    const int t_end = (a.n_new + rows_per_tile - 1) / rows_per_tile;
-    if (t_first >= t_end) return;
-
-    // destination element offset per (stage, vector), -1 = nothing to write
-    int64_t dst_off[kEvictStages][kEvictVecsPerThread];
-
-    auto issue = [&](int t, int st) {
-#pragma unroll
-        for (int k = 0; k < kEvictVecsPerThread; ++k) {
-            dst_off[st][k] = -1;
-            const int j = t * rows_per_tile + row_lane + k * row_step;
-            if (j < a.first_row || j >= a.n_new) continue;
-            const int q = j / a.P;
-            const int dpage = __ldg(a.new_pt + q);
-            const bool fresh = dpage != __ldg(a.old_pt + q);
-            const int src = kept_source(a.run_dst, a.run_src, a.n_runs, j);
-            if (!fresh && src == j) continue;
-            const int sq_ = src / a.P;
-            if (sq_ >= a.n_old_pages) { set_error(a.err, kErrBounds); continue; }
-            const int spage = __ldg(a.old_pt + sq_);
-            if ((uint64_t)spage >= (uint64_t)a.num_pages || (uint64_t)dpage >= (uint64_t)a.num_pages) {
+    auto issue_loads = [&](int t) {
+        const int slot = t % S;
+        const uint32_t bar = smem_addr(&full[slot]);
+        const uint32_t dst0 = smem_addr(smem + slot * tile_bytes);
+        const int pb = __ldg(&a.tiles[t].piece_begin);
+        const int pe = t + 1 < a.n_tiles ? __ldg(&a.tiles[t + 1].piece_begin) : a.n_pieces;
+        uint32_t bytes = 0;
+        for (int k = pb; k < pe; ++k) {
+            const EvictPiece pc = a.pieces[k];
+            if ((uint64_t)pc.src_page >= (uint64_t)a.num_pages || pc.src_slot < 0 ||
+                pc.n_rows <= 0 || pc.src_slot + pc.n_rows > a.P || pc.dst_row < 0 ||
+                pc.dst_row + pc.n_rows > a.tile_rows)
+                continue;
+            bytes += (uint32_t)pc.n_rows * row_bytes;
+        }
+        if (bytes == 0) {
+            mbar_arrive(bar);
+        } else {
+            mbar_arrive_expect_tx(bar, bytes);
+        }
+        for (int k = pb; k < pe; ++k) {
+            const EvictPiece pc = a.pieces[k];
+            if ((uint64_t)pc.src_page >= (uint64_t)a.num_pages || pc.src_slot < 0 ||
+                pc.n_rows <= 0 || pc.src_slot + pc.n_rows > a.P || pc.dst_row < 0 ||
+                pc.dst_row + pc.n_rows > a.tile_rows) {
                 set_error(a.err, kErrBounds);
                 continue;
             }
-            const int64_t so = row_offset(a.num_pages, a.Hkv, a.P, a.D, layer, spage, kv, head,
-                                          src % a.P) + col0 + vc * 8;
-            dst_off[st][k] = row_offset(a.num_pages, a.Hkv, a.P, a.D, layer, dpage, kv, head,
-                                        j % a.P) + col0 + vc * 8;
-            cp_async_16(smem_addr(&buf[st][(tid + k * kEvictThreads) * 16]), a.pool + so);
+            bulk_load(dst0 + (uint32_t)pc.dst_row * row_bytes,
+                      base + pc.src_page * page_stride + (int64_t)pc.src_slot * row_bytes,
+                      (uint32_t)pc.n_rows * row_bytes, bar);
         }
-        cp_async_commit();
     };
 
-    // prologue: tiles t_first, t_first + 1
-#pragma unroll
-    for (int s = 0; s < kEvictStages - 1; ++s) {
-        if (t_first + s < t_end) issue(t_first + s, s);
-        else cp_async_commit();
-    }
-    int st = 0;
-    for (int t = t_first; t < t_end; ++t) {
-        const int ahead = t + kEvictStages - 1;
-        const int st_ahead = (st + kEvictStages - 1) % kEvictStages;
-        if (ahead < t_end) issue(ahead, st_ahead);
-        else cp_async_commit();
-        cp_async_wait<kEvictStages - 1>();  // tile t has landed (this thread's part)
-        __syncthreads();                    // ... and every thread's part
-#pragma unroll
-        for (int k = 0; k < kEvictVecsPerThread; ++k) {
-            if (dst_off[st][k] < 0) continue;
-            *reinterpret_cast<uint4*>(a.pool + dst_off[st][k]) =
-                *reinterpret_cast<const uint4*>(&buf[st][(tid + k * kEvictThreads) * 16]);
+    const int T = a.n_tiles;
+    for (int t = 0; t < S - 1 && t < T; ++t) issue_loads(t);
+    int t = 0;
+    for (; t < T; ++t) {
+        const int slot = t % S;
+        if (!mbar_wait(smem_addr(&full[slot]), (uint32_t)(t / S) & 1u)) {
+            set_error(a.err, kErrTimeout);
+            break;
         }
-        st = (st + 1) % kEvictStages;
+        fence_proxy_async_smem();
+        const EvictTile tl = a.tiles[t];
+        if ((uint64_t)tl.dst_page < (uint64_t)a.num_pages && tl.dst_slot >= 0 && tl.n_rows > 0 &&
+            tl.n_rows <= a.tile_rows && tl.dst_slot + tl.n_rows <= a.P) {
+            bulk_store(base + tl.dst_page * page_stride + (int64_t)tl.dst_slot * row_bytes,
+                       smem_addr(smem + slot * tile_bytes), (uint32_t)tl.n_rows * row_bytes);
+        } else {
+            set_error(a.err, kErrBounds);
+        }
+        bulk_commit();
+        const int tn = t + S - 1;
+        if (tn < T) {
+            bulk_wait_read<1>();  // the store of tile t - 1 has read its slot
+            issue_loads(tn);
+        }
     }
-    cp_async_wait<0>();
+    if (t < T) {
+        // timed out: let the loads already issued land (bounded) before leaving
+        for (int u = t + 1; u < T && u < t + S - 1; ++u)
+            mbar_wait(smem_addr(&full[u % S]), (uint32_t)(u / S) & 1u);
+    }
+    bulk_wait<0>();
 }
 
 }  // namespace
@@ -192,18 +192,30 @@ cudaError_t launch_cow_copy(const CowArgs& a, int num_sms, cudaStream_t st) {
     return cudaGetLastError();
 }
 
-int evict_ctas_per_sm() {
+int evict_smem_bytes(int tile_rows, int D) {
+    return kEvictStages * tile_rows * D * 2 + kEvictStages * 8 + 128;
+}
+
+int evict_ctas_per_sm(int tile_rows, int D) {
     int n = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, sq_evict_compact_kernel, kEvictThreads, 0) !=
-            cudaSuccess || n < 1)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, sq_evict_compact_kernel, 32,
+                                                      evict_smem_bytes(tile_rows, D)) !=
+            cudaSuccess ||
+        n < 1)
         return 1;
     return n;
 }
 
+cudaError_t evict_prepare() {
+    return cudaFuncSetAttribute(sq_evict_compact_kernel,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                evict_smem_bytes(kStageTokens, 128));
+}
+
 cudaError_t launch_evict(const EvictArgs& a, cudaStream_t st) {
-    const int blocks = a.L * 2 * a.Hkv * a.col_split;
-    if (blocks == 0 || a.first_row >= a.n_new) return cudaSuccess;
-    sq_evict_compact_kernel<<<blocks, kEvictThreads, 0, st>>>(a);
+    const int blocks = a.L * 2 * a.Hkv;
+    if (blocks == 0 || a.n_tiles == 0) return cudaSuccess;
+    sq_evict_compact_kernel<<<blocks, 32, evict_smem_bytes(a.tile_rows, a.D), st>>>(a);
     return cudaGetLastError();
 }
 

@@ -74,20 +74,21 @@ struct EvictArgs {
     __nv_bfloat16* pool;
     int64_t num_pages;
     int32_t L, Hkv, P, D;
-    const int32_t* old_pt;      // page table before (n_old_pages)
-    const int32_t* new_pt;      // page table after (n_new_pages)
-    const int32_t* run_dst;     // kept runs, destination starts (increasing)
-    const int32_t* run_src;     // kept runs, source starts
-    int32_t n_old_pages, n_new_pages, n_runs;
-    int32_t n_new;              // rows after eviction
-    int32_t first_row;          // first destination row that can change
-    int32_t col_split;          // column pieces per row (1, 2 or 4)
+    const EvictTile* tiles;     // destination tiles, increasing logical order
+    const EvictPiece* pieces;   // their contiguous source pieces
+    int32_t n_tiles, n_pieces;
+    int32_t tile_rows;          // rows a tile holds at most
     int* err;
 };
 
 cudaError_t launch_append(const AppendArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_cow_copy(const CowArgs& a, int num_sms, cudaStream_t st);
-int evict_ctas_per_sm();
+constexpr int kEvictStages = 3;
+// Shared memory of one eviction CTA for a tile size.
+int evict_smem_bytes(int tile_rows, int D);
+// Resident eviction CTAs per SM for a tile size.
+int evict_ctas_per_sm(int tile_rows, int D);
+cudaError_t evict_prepare();  // raises the dynamic shared-memory limit once
 cudaError_t launch_evict(const EvictArgs& a, cudaStream_t st);
 
 }  // namespace sq

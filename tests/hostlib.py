@@ -32,6 +32,7 @@ def lib():
         L.sqh_append.argtypes = [P, I32, I32]
         L.sqh_evict.argtypes = [P, I32, I32P, I32, I64P]
         L.sqh_release.argtypes = [P, I32]
+        L.sqh_evict_tiles.argtypes = [P, I32, I32P, I32, I32, I32P, I32, I32P, I32, I32P, I32P]
         L.sqh_seq_info.argtypes = [P, I32, I32P, I32P]
         L.sqh_page_table.argtypes = [P, I32, I32P, I32, I32P]
         L.sqh_refcount.argtypes = [P, I32]
@@ -75,6 +76,19 @@ class HostCache:
         rc = lib().sqh_evict(self.h, h, arr, len(spans), st)
         return rc, {"moved_rows": st[0], "cow_pages": st[1], "freed": st[2],
                     "first_row": st[3], "n_runs": st[4]}
+
+    def evict_tiles(self, h, spans, tile_rows, cap=100000):
+        arr = (ctypes.c_int32 * max(2, 2 * len(spans)))(*[int(x) for ab in spans for x in ab])
+        tiles = np.zeros(4 * cap, dtype=np.int32)
+        pieces = np.zeros(4 * cap, dtype=np.int32)
+        nt, npc = ctypes.c_int32(), ctypes.c_int32()
+        i32p = ctypes.POINTER(ctypes.c_int32)
+        rc = lib().sqh_evict_tiles(self.h, h, arr, len(spans), tile_rows,
+                                   tiles.ctypes.data_as(i32p), cap, pieces.ctypes.data_as(i32p),
+                                   cap, ctypes.byref(nt), ctypes.byref(npc))
+        if rc != 0:
+            return rc, None, None
+        return 0, tiles[:4 * nt.value].reshape(-1, 4), pieces[:4 * npc.value].reshape(-1, 4)
 
     def release(self, h):
         return lib().sqh_release(self.h, h)

@@ -202,3 +202,61 @@ def test_decode_plan_rejects_bad_input():
     hc.append(m, 5)
     assert hc.plan_decode([m, m], 10)[0] == -1       # duplicate
     assert hc.plan_decode([m, 999], 10)[0] == -2     # bad handle
+
+
+@pytest.mark.parametrize("seed", range(20))
+def test_evict_tiles_compact_in_place(seed):
+    """Replaying the compaction tiles in order — each tile's reads before its
+    writes, on a physical model of the pool — gives the oracle's result; no
+    tile reads a slot an earlier tile wrote (so loads may run ahead of
+    earlier stores); forks sharing pages are untouched."""
+    rng = random.Random(500 + seed)
+    P = rng.choice([8, 16, 64, 128])
+    tile_rows = rng.choice([t for t in (8, 16, 32, 64) if t <= P])
+    hc = HostCache(1, 4, 1, 64, P, 600)
+    oc = ocm.OracleCache(600, P, physical=True)
+    rc, m = hc.seq_new()
+    om = oc.seq_new()
+    n0 = rng.randint(1, 40 * P)
+    hc.append(m, n0)
+    oc.append(om, n0)
+    forks = []
+    if rng.random() < 0.5:
+        rc, a = hc.fork(m)
+        forks.append((a, oc.fork(om)))
+        k = rng.randint(0, 2 * P)
+        hc.append(a, k)
+        oc.append(forks[-1][1], k)
+        k = rng.randint(0, P)
+        hc.append(m, k)
+        oc.append(om, k)
+    n = oc.n_tokens(om)
+    spans = random_spans(rng, n, rng.choice([1, 3, 8, 20]))
+    # physical state before, as {page: [token ids]}
+    phys = {p: list(v) for p, v in oc.phys.items()}
+    rc, tiles, pieces = hc.evict_tiles(m, spans, tile_rows)
+    oc.evict(om, spans)
+    assert rc == 0
+    written = set()
+    for t in range(len(tiles)):
+        dpage, dslot, nrows, pb = (int(x) for x in tiles[t])
+        pe = int(tiles[t + 1][3]) if t + 1 < len(tiles) else len(pieces)
+        assert 0 < nrows <= tile_rows and dslot + nrows <= P
+        buf = [None] * nrows
+        for k in range(pb, pe):
+            spage, sslot, pn, drow = (int(x) for x in pieces[k])
+            assert 0 < pn and sslot + pn <= P and drow + pn <= nrows
+            for i in range(pn):
+                assert (spage, sslot + i) not in written
+                buf[drow + i] = phys[spage][sslot + i]
+        assert all(x is not None for x in buf)
+        for i in range(nrows):
+            phys.setdefault(dpage, [-1] * P)[dslot + i] = buf[i]
+            written.add((dpage, dslot + i))
+    pt = hc.page_table(m)
+    assert pt == oc.page_table(om)
+    got = [phys[pt[j // P]][j % P] for j in range(oc.n_tokens(om))]
+    assert got == oc.tokens(om)
+    for a, oa in forks:
+        apt = hc.page_table(a)
+        assert [phys[apt[j // P]][j % P] for j in range(oc.n_tokens(oa))] == oc.tokens(oa)
