@@ -64,6 +64,43 @@ def peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+KERNEL_SOURCES = {
+    "sq_decode_splitk_kernel": ["kernels/decode.cu", "kernels/ptx.cuh", "kernels/launch.hpp",
+                                "host/plan.hpp"],
+    "sq_evict_compact_kernel": ["kernels/kv.cu", "kernels/ptx.cuh", "kernels/launch.hpp",
+                                "host/plan.hpp"],
+}
+
+
+def sources_hash(kernel: str) -> str:
+    import hashlib
+    m = hashlib.sha256()
+    for rel in KERNEL_SOURCES[kernel]:
+        with open(os.path.join(ROOT, "paper_2602_22603_gb300", "csrc", rel), "rb") as f:
+            m.update(f.read())
+    return m.hexdigest()[:16]
+
+
+def recorded_traffic_ratio(kernel: str):
+    """DRAM traffic per algorithmic byte from the ncu capture summarised in
+    profiles/, if that capture was taken of the current kernel sources
+    (else None)."""
+    import re
+    pdir = os.path.join(ROOT, "profiles")
+    if not os.path.isdir(pdir):
+        return None, None
+    cur = sources_hash(kernel)
+    for name in sorted(os.listdir(pdir)):
+        if not name.endswith(".md"):
+            continue
+        with open(os.path.join(pdir, name)) as f:
+            for line in f:
+                mt = re.search(r"traffic: kernel=(\S+) ratio=([0-9.]+) sources_sha256=([0-9a-f]+)", line)
+                if mt and mt.group(1) == kernel and mt.group(3) == cur:
+                    return float(mt.group(2)), "profiles/" + name
+    return None, None
+
+
 class ClockSampler:
     """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
 
@@ -146,24 +183,12 @@ def workload_name(args):
             f"page 64, bf16")
 
 
-def request_spans(seed, r, n, P):
-    """Per request: 20-65% of the context (uniform) in 10-40 spans (uniform)
-    with lognormal lengths (median 2,000 tokens), inside [P, n)."""
-    import numpy as np
-    from synthetic import random_spans, shuffled, sub_seed
-    rng = np.random.default_rng(sub_seed(seed, 100 + r))
-    frac = rng.uniform(0.20, 0.65)
-    k = int(rng.integers(10, 41))
-    total = int(frac * (n - P))
-    return shuffled(random_spans(sub_seed(seed, 200 + r), k, total, P, n, median=2000), r)
-
-
 def run_sq(args, world, rank, local):
     import numpy as np
     import torch
 
     import paper_2602_22603_gb300 as sq
-    from synthetic import AGENT_8B, Bank, bf16_normal, sub_seed
+    from synthetic import AGENT_8B, Bank, bf16_normal, request_spans, sub_seed
 
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
@@ -197,11 +222,14 @@ def run_sq(args, world, rank, local):
     small = bank.offsets(8192, 2 * 8 * tok_elems, sub_seed(seed, 3))
     small_i = [0]
 
+    bank_ptr = bank.data.data_ptr()
+
     def kv_rows(n):
-        """K and V of n <= 8 new tokens, [L, n, Hkv, D] views of the bank."""
+        """Device addresses of the K and V of n <= 8 new tokens
+        ([L, n, Hkv, D] slices of the bank)."""
         o = int(small[small_i[0] % len(small)])
         small_i[0] += 1
-        return bank.view(o, (L, n, Hkv, D)), bank.view(o + 8 * tok_elems, (L, n, Hkv, D))
+        return bank_ptr + 2 * o, bank_ptr + 2 * (o + 8 * tok_elems)
 
     def fork_all():
         auxs.clear()
@@ -217,14 +245,28 @@ def run_sq(args, world, rank, local):
     out_all = torch.empty(L, S, Hq, D, dtype=torch.bfloat16, device="cuda")
     torch.cuda.synchronize()
 
+    # per-call arguments resolved once: raw pointers, one stream handle
+    st_h = int(stream.cuda_stream)
+    q_ptr = [q_all[layer].data_ptr() for layer in range(L)]
+    o_ptr = [out_all[layer].data_ptr() for layer in range(L)]
+    seq_arr = [None]
+
+    def set_seqs():
+        import ctypes
+        seq_arr[0] = (ctypes.c_int32 * len(seqs))(*seqs)
+
+    set_seqs()
+
     def step(ev=None):
         for h in seqs:
             k, v = kv_rows(1)
-            cache.append_kv(h, 1, k, v)
+            cache.append_kv(h, 1, k, v, st_h)
         if ev is not None:
             ev.record(stream)
+        arr = seq_arr[0]
         for layer in range(L):
-            cache.decode_attention(seqs, layer, q_all[layer], out_all[layer], sq.SQ_OUT_BF16, scale)
+            sq.sq_decode_attention(cache.handle, arr, layer, q_ptr[layer], o_ptr[layer],
+                                   sq.SQ_OUT_BF16, scale, st_h)
 
     def timed_decode(K, W):
         for _ in range(W):
@@ -261,6 +303,7 @@ def run_sq(args, world, rank, local):
     achieved = uniq_per_call / (per_call_ms / 1e3) / 1e9
     logical_gbs = before["logical_bytes"] / before["calls"] / (per_call_ms / 1e3) / 1e9
 
+    ratio, ratio_src = recorded_traffic_ratio("sq_decode_splitk_kernel")
     res = {
         "metric": METRIC,
         "value": round(value, 3),
@@ -302,7 +345,9 @@ def run_sq(args, world, rank, local):
             "peak_kind": peak_kind,
             "unit": "GB/s",
             "frac": round(achieved / hbm_peak, 4),
-            "traffic": None,
+            "traffic": int(ratio * uniq_per_call) if ratio else None,
+            "traffic_source": (ratio_src + ": small-case DRAM bytes per algorithmic byte, scaled "
+                               "to this launch's algorithmic bytes") if ratio else None,
             "algorithmic_bytes_per_launch": int(uniq_per_call),
         },
         "gpu_launches": int(K * (S + 2 * L)),
@@ -357,7 +402,7 @@ def run_sq(args, world, rank, local):
         per = []
         for r, m in enumerate(mains):
             n = cache.seq_info(m)[0]
-            spans = request_spans(seed, r, n, P)
+            spans = request_spans(seed, r, n, P)  # 20-65% in 10-40 spans, median 2,000
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             b0 = cache.stats()["evict_bytes"]
             e0.record(stream)
@@ -373,12 +418,17 @@ def run_sq(args, world, rank, local):
         ev_gbs = ev_bytes / (ev_ms / 1e3) / 1e9
         fork_all()
         seqs[:] = [x for pair in zip(mains, auxs) for x in pair]
+        set_seqs()
         torch.cuda.synchronize()
         after = timed_decode(K, W)
         pc = after["attn_ms"] / after["calls"]
         up = after["unique_bytes"] / after["calls"]
+        ev_ratio, ev_src = recorded_traffic_ratio("sq_evict_compact_kernel")
         res["evict"] = {
+            "kernel": "sq_evict_compact_kernel",
             "gbs": round(ev_gbs, 1),
+            "traffic_per_call": int(ev_ratio * ev_bytes / len(mains)) if ev_ratio else None,
+            "traffic_source": ev_src,
             "frac_of_%s_peak" % peak_kind: round(ev_gbs / hbm_peak, 4),
             "ms_total": round(ev_ms, 4),
             "algorithmic_bytes": int(ev_bytes),

@@ -186,7 +186,7 @@ def sq_fork_aux(cache: int, parent: int) -> int:
 def sq_decode_attention(cache: int, seqs: Sequence[int], layer: int, q, out,
                         out_dtype: int = SQ_OUT_BF16, sm_scale: float = 1.0,
                         stream=None) -> None:
-    arr = (ctypes.c_int32 * len(seqs))(*seqs)
+    arr = seqs if isinstance(seqs, ctypes.Array) else (ctypes.c_int32 * len(seqs))(*seqs)
     _check(lib().sq_decode_attention(cache, arr, len(seqs), layer, _ptr(q), _ptr(out),
                                      out_dtype, float(sm_scale), _stream(stream)),
            "sq_decode_attention")

@@ -47,6 +47,18 @@ struct UploadSlot {
     bool ev_recorded = false;
 };
 
+// Pinned host staging for uploads: a copy from pageable memory may wait for
+// the stream's earlier work (draining the GPU between calls); from pinned
+// memory it is a plain asynchronous DMA.  A buffer is refilled only after the
+// copy that last used it has run.
+constexpr int kPinnedSlots = 8;
+struct PinnedSlot {
+    uint8_t* h = nullptr;
+    size_t cap = 0;
+    cudaEvent_t ev = nullptr;
+    bool ev_recorded = false;
+};
+
 }  // namespace
 
 struct sq_cache {
@@ -65,6 +77,8 @@ struct sq_cache {
     uint64_t use_clock = 0;
     UploadSlot slots[kUploadSlots];
     int next_slot = 0;
+    PinnedSlot pinned[kPinnedSlots];
+    int next_pinned = 0;
     std::vector<uint8_t> staging;
     // pages freed by work on a stream become reusable elsewhere only after
     // that work: the stream that freed each free page, and one event per
@@ -166,6 +180,38 @@ int record_freed(sq_cache* c, const std::vector<int32_t>& freed, void* stream) {
     return SQ_OK;
 }
 
+// Asynchronous host -> device copy of `bytes` from `src` through a pinned
+// staging buffer; `src` may be reused as soon as this returns.
+int staged_copy(sq_cache* c, void* dst, const void* src, size_t bytes, void* stream) {
+    PinnedSlot& p = c->pinned[c->next_pinned];
+    c->next_pinned = (c->next_pinned + 1) % kPinnedSlots;
+    cudaError_t e;
+    if (!p.ev) {
+        e = cudaEventCreateWithFlags(&p.ev, cudaEventDisableTiming);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    if (p.ev_recorded) {
+        e = cudaEventSynchronize(p.ev);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    if (bytes > p.cap) {
+        if (p.h) cudaFreeHost(p.h);
+        p.h = nullptr;
+        p.cap = 0;
+        const size_t cap = std::max<size_t>(bytes * 5 / 4, 64 << 10);
+        e = cudaHostAlloc(reinterpret_cast<void**>(&p.h), cap, cudaHostAllocDefault);
+        if (e != cudaSuccess) return cuda_status(e);
+        p.cap = cap;
+    }
+    std::memcpy(p.h, src, bytes);
+    e = cudaMemcpyAsync(dst, p.h, bytes, cudaMemcpyHostToDevice, as_stream(stream));
+    if (e != cudaSuccess) return cuda_status(e);
+    e = cudaEventRecord(p.ev, as_stream(stream));
+    if (e != cudaSuccess) return cuda_status(e);
+    p.ev_recorded = true;
+    return SQ_OK;
+}
+
 int upload(sq_cache* c, UploadSlot& s, const void* src, size_t bytes, void* stream) {
     if (bytes > s.cap) {
         if (s.d) {
@@ -184,10 +230,7 @@ int upload(sq_cache* c, UploadSlot& s, const void* src, size_t bytes, void* stre
         cudaError_t e = cudaStreamWaitEvent(as_stream(stream), s.ev, 0);
         if (e != cudaSuccess) return cuda_status(e);
     }
-    // pageable source: staged by the driver before the call returns, so the
-    // host buffer may be reused at once
-    cudaError_t e = cudaMemcpyAsync(s.d, src, bytes, cudaMemcpyHostToDevice, as_stream(stream));
-    return cuda_status(e);
+    return staged_copy(c, s.d, src, bytes, stream);
 }
 
 void free_entry(PlanEntry& p) {
@@ -302,6 +345,10 @@ int sq_cache_destroy(sq_cache* c) {
     for (auto& s : c->slots) {
         if (s.d) cudaFree(s.d);
         if (s.ev) cudaEventDestroy(s.ev);
+    }
+    for (auto& p : c->pinned) {
+        if (p.h) cudaFreeHost(p.h);
+        if (p.ev) cudaEventDestroy(p.ev);
     }
     for (auto& kv : c->free_event) cudaEventDestroy(kv.second);
     if (c->d_err) cudaFree(c->d_err);
@@ -452,8 +499,8 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
         }
         if (c->staging.size() < (size_t)lay.total) c->staging.resize(lay.total);
         plan_serialize(plan, lay, c->staging.data());
-        e = cudaMemcpyAsync(victim->d_plan, c->staging.data(), lay.total, cudaMemcpyHostToDevice, st);
-        if (e != cudaSuccess) { victim->valid = false; return cuda_status(e); }
+        int urc = staged_copy(c, victim->d_plan, c->staging.data(), lay.total, stream);
+        if (urc != SQ_OK) { victim->valid = false; return urc; }
         victim->valid = true;
         victim->n_ctas = c->decode_ctas;
         victim->handles.assign(seqs, seqs + n_seqs);

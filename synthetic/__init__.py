@@ -167,3 +167,15 @@ def shuffled(spans: Sequence[Tuple[int, int]], seed: int) -> List[Tuple[int, int
     rng = np.random.default_rng(seed)
     idx = rng.permutation(len(spans))
     return [tuple(spans[int(i)]) for i in idx]
+
+
+def request_spans(seed: int, r: int, n: int, P: int, frac=(0.20, 0.65), count=(10, 40),
+                  median: float = 2000.0) -> List[Tuple[int, int]]:
+    """Spans for one request of the batched-serving workload: a uniform
+    fraction of the context in a uniform number of spans with lognormal
+    lengths, inside [P, n), in shuffled order."""
+    rng = np.random.default_rng(sub_seed(seed, 100 + r))
+    f = rng.uniform(*frac)
+    k = int(rng.integers(count[0], count[1] + 1))
+    total = int(f * (n - P))
+    return shuffled(random_spans(sub_seed(seed, 200 + r), k, total, P, n, median=median), r)

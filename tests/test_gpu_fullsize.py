@@ -1,0 +1,139 @@
+"""Parity at the benchmark's full sizes, in the launch configuration bench.py
+times (all decoding sequences of a step in one call, default persistent CTA
+count): attention outputs on sampled sequences and layers against the oracle,
+complete page tables, and sampled (layer, K/V, head) planes of the pool bit
+for bit after eviction."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2602_22603_gb300 as sq
+from oracle import attention as oatt
+from synthetic import bf16_bits, bf16_normal, random_spans, request_spans, shuffled
+from tests.bankfill import BankPair
+from tests.gpu_harness import assert_close
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2602_22603_gb300 import build
+    build.build_libsq()
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+
+
+def _decode_and_check(bp, seqs, layer, scale, seed, sample):
+    S = len(seqs)
+    q_cpu = bf16_normal((S, bp.Hq, bp.D), seed)
+    out = torch.empty(S, bp.Hq, bp.D, dtype=torch.float32, device="cuda")
+    bp.cache.decode_attention(seqs, layer, q_cpu.cuda(), out, sq.SQ_OUT_F32, scale)
+    torch.cuda.synchronize()
+    assert bp.cache.sync_status() == sq.SQ_OK
+    qb = bf16_bits(q_cpu)
+    for i in sample:
+        K, V = bp.rows(seqs[i], layer)
+        exp = oatt.decode(qb[i], K, V, scale)
+        assert_close(out[i], exp)
+
+
+def test_serving_128k_full_size():
+    """8 requests x 131,072 tokens + 8 forks (16 decoding sequences), 32
+    layers, 32q/8kv, d128, P64; evict 20-65% per request in 10-40 spans."""
+    L, Hq, Hkv, D, P = 32, 32, 8, 128, 64
+    R, ctx = 8, 131072
+    bp = BankPair(L, Hq, Hkv, D, P, num_pages=R * (ctx // P + 4) + R * 4 + 64, seed=0)
+    try:
+        scale = 1.0 / math.sqrt(D)
+        mains = []
+        for r in range(R):
+            m = bp.seq_new()
+            bp.fill(m, ctx, 4096)
+            mains.append(m)
+        auxs = []
+        for m in mains:
+            a = bp.fork(m)
+            bp.append(a, 8)
+            auxs.append(a)
+        seqs = [x for pair in zip(mains, auxs) for x in pair]
+        for h in seqs:
+            bp.append(h, 1)
+        bp.check_tables(seqs)
+        st = bp.cache.stats()
+        assert st["live_pages"] == bp.oracle.live_pages()
+        for layer, sample in ((0, (0, 1)), (13, (9,)), (31, (14, 15))):
+            _decode_and_check(bp, seqs, layer, scale, 100 + layer, sample)
+        # the shared prefix is read once per call
+        st2 = bp.cache.stats()
+        calls = st2["decode_calls"] - st["decode_calls"]
+        uniq = (st2["decode_unique_bytes"] - st["decode_unique_bytes"]) / calls
+        logi = (st2["decode_logical_bytes"] - st["decode_logical_bytes"]) / calls
+        assert uniq < 0.51 * logi
+        # Algorithm 1: release the aux threads, then evict
+        for a in auxs:
+            bp.release(a)
+        for r, m in enumerate(mains):
+            n = bp.cache.seq_info(m)[0]
+            bp.evict(m, request_spans(0, r, n, P))
+        bp.check_tables(mains)
+        for r, layer, kv, head in ((0, 0, 0, 0), (3, 31, 1, 7), (7, 15, 0, 4), (5, 1, 1, 2)):
+            bp.check_plane(mains[r], layer, kv, head)
+        auxs = []
+        for m in mains:
+            a = bp.fork(m)
+            bp.append(a, 8)
+            auxs.append(a)
+        seqs = [x for pair in zip(mains, auxs) for x in pair]
+        for h in seqs:
+            bp.append(h, 1)
+        _decode_and_check(bp, seqs, 5, scale, 999, (0, 7, 10))
+        bp.check_tables(seqs)
+    finally:
+        bp.close()
+
+
+def test_large_ragged_full_size():
+    """64q/8kv (G = 8), d128, 80 layers, P64: requests of 32k, 96k, 192k and
+    262,144 tokens, each with a fork; evict 50% of each in 25 spans — the
+    32k one while its fork is alive (copy-on-write of every changed page)."""
+    L, Hq, Hkv, D, P = 80, 64, 8, 128, 64
+    ctxs = [32768, 98304, 196608, 262144]
+    pages = sum(c // P for c in ctxs) + 4 * 8 + 64 + ctxs[0] // P  # + CoW room
+    bp = BankPair(L, Hq, Hkv, D, P, num_pages=pages, seed=3)
+    try:
+        scale = 1.0 / math.sqrt(D)
+        mains = []
+        for n in ctxs:
+            m = bp.seq_new()
+            bp.fill(m, n, 2048)
+            mains.append(m)
+        auxs = []
+        for m in mains:
+            a = bp.fork(m)
+            bp.append(a, 8)
+            auxs.append(a)
+        seqs = [x for pair in zip(mains, auxs) for x in pair]
+        for h in seqs:
+            bp.append(h, 1)
+        bp.check_tables(seqs)
+        _decode_and_check(bp, seqs, 0, scale, 7, (6, 1))
+        _decode_and_check(bp, seqs, 79, scale, 8, (7, 2))
+        for r in range(1, 4):
+            bp.release(auxs[r])
+        for r, m in enumerate(mains):
+            n = bp.cache.seq_info(m)[0]
+            spans = shuffled(random_spans(500 + r, 25, n // 2, P, n, median=n / 50), r)
+            bp.evict(m, spans)
+        kept = [mains[0], auxs[0], mains[1], mains[2], mains[3]]
+        bp.check_tables(kept)
+        for h, layer, kv, head in ((mains[3], 79, 1, 7), (mains[2], 40, 0, 3), (auxs[0], 40, 0, 3),
+                                   (mains[0], 0, 1, 0), (mains[0], 61, 0, 5)):
+            bp.check_plane(h, layer, kv, head)
+        for h in kept:
+            bp.append(h, 1)
+        _decode_and_check(bp, kept, 33, scale, 9, (0, 1, 4))
+    finally:
+        bp.close()
