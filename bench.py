@@ -454,66 +454,94 @@ def run_sq(args, world, rank, local):
     return res
 
 
+def _oracle_rows(host_bank, offs, n_chunks, chunk, L, Hkv, D, layer, which):
+    """K (which = 0) or V (1) bits [n, Hkv, D] of one main sequence at one
+    layer, rebuilt from its bank chunks."""
+    import numpy as np
+    parts = []
+    for c in range(n_chunks):
+        o = int(offs[c * 2 + which])
+        a = host_bank[o:o + L * chunk * Hkv * D].reshape(L, chunk, Hkv, D)
+        parts.append(a[layer])
+    return np.ascontiguousarray(np.concatenate(parts))
+
+
 def cpu_baseline(args, bank, offs, n_chunks, chunk, scale):
-    """The oracle as it stands (oracle/attention.c) on the host cores: one
-    decode step of request 0's main sequence and of an aux fork at one layer
-    over the full context (2 sequences x 1 layer), scaled to tokens/s."""
+    """The oracle as it stands (oracle/attention.c, fp64, OpenMP) on the host
+    cores: one decode call of the whole batch (the 8 main sequences and their
+    forks, every head) at 2 of the layers, over the full context; scaled to
+    tokens/s = sequences / (time per layer x layers)."""
     import numpy as np
 
     from oracle import attention as oatt
     from synthetic import bf16_bits, bf16_normal
     L, Hq, Hkv, D = args.layers, 32, 8, 128
+    R = args.requests
     host_bank = bf16_bits(bank.data.cpu())
-    layer = 0
-
-    def rows(which):
-        parts = []
-        for c in range(n_chunks):
-            o = int(offs[c * 2 + which])
-            a = host_bank[o:o + L * chunk * Hkv * D].reshape(L, chunk, Hkv, D)
-            parts.append(a[layer])
-        return np.ascontiguousarray(np.concatenate(parts))
-
-    k, v = rows(0), rows(1)
-    q = bf16_bits(bf16_normal((2, Hq, D), 99))
-    oatt.decode_batch(q[:1, :, :], [k[:1024]], [v[:1024]], scale)  # warm
-    t0 = time.perf_counter()
-    oatt.decode_batch(q, [k, k], [v, v], scale)
-    t = time.perf_counter() - t0
-    tokens_per_s = 2 / (t * L)
-    return {"value": round(tokens_per_s, 4), "unit": "tokens/s", "cores": oatt.num_threads(),
-            "kind": "oracle",
-            "sample": f"2 sequences x 1 of {L} layers, {k.shape[0]} tokens each, all {Hq} heads "
-                      f"(fp64 C oracle, OpenMP); tokens/s = 2 / (time x {L} layers)",
-            "seconds": round(t, 3)}
+    layers = (0, L - 1) if L > 1 else (0,)
+    total = 0.0
+    n_tok = 0
+    for layer in layers:
+        ks, vs = [], []
+        for r in range(R):
+            sub = offs[r * n_chunks * 2:(r + 1) * n_chunks * 2]
+            k = _oracle_rows(host_bank, sub, n_chunks, chunk, L, Hkv, D, layer, 0)
+            v = _oracle_rows(host_bank, sub, n_chunks, chunk, L, Hkv, D, layer, 1)
+            ks += [k, k]   # main and its fork read the same prefix rows
+            vs += [v, v]
+        n_tok = ks[0].shape[0]
+        q = bf16_bits(bf16_normal((2 * R, Hq, D), 99 + layer))
+        t0 = time.perf_counter()
+        oatt.decode_batch(q, ks, vs, scale)
+        total += time.perf_counter() - t0
+    per_layer = total / len(layers)
+    return {"value": round(2 * R / (per_layer * L), 4), "unit": "tokens/s",
+            "cores": oatt.num_threads(), "kind": "oracle",
+            "sample": f"one decode call of all {2 * R} sequences ({n_tok} tokens each, {Hq} heads) "
+                      f"at {len(layers)} of {L} layers; tokens/s = sequences / "
+                      f"(seconds per layer x {L} layers)",
+            "seconds": round(total, 3)}
 
 
 def run_reference(args, world, rank):
     """Reference arm: the CPU oracle as it stands, on this machine's host cores,
-    for the same metric; each step is a bounded sample of the workload."""
+    for the same metric; each step is one decode call of the whole batch at
+    one layer (a bounded sample of the workload)."""
     import numpy as np
 
     from oracle import attention as oatt
-    from synthetic import bf16_bits, bf16_normal, sub_seed
+    from synthetic import Bank, bf16_bits, bf16_normal, sub_seed
     if rank != 0:
         return None
     L, Hq, Hkv, D = args.layers, 32, 8, 128
-    n = args.ctx
+    R, n = args.requests, args.ctx
     scale = 1.0 / math.sqrt(D)
-    k = bf16_bits(bf16_normal((n, Hkv, D), sub_seed(args.seed, 11)))
-    v = bf16_bits(bf16_normal((n, Hkv, D), sub_seed(args.seed, 12)))
-    q = bf16_bits(bf16_normal((2, Hq, D), sub_seed(args.seed, 13)))
+    bank = bf16_bits(Bank(1 << 27, sub_seed(args.seed, 11)).data)
+    rng = np.random.default_rng(sub_seed(args.seed, 12))
+    row = Hkv * D
+
+    def rows():
+        o = int(rng.integers(0, (bank.size - n * row) // 8)) * 8
+        return bank[o:o + n * row].reshape(n, Hkv, D)
+
+    ks, vs = [], []
+    for _ in range(R):
+        k, v = rows(), rows()
+        ks += [k, k]
+        vs += [v, v]
+    q = bf16_bits(bf16_normal((2 * R, Hq, D), sub_seed(args.seed, 13)))
     for _ in range(args.warmup):
-        oatt.decode_batch(q[:1], [k[:4096]], [v[:4096]], scale)
+        oatt.decode_batch(q[:1], [ks[0][:4096]], [vs[0][:4096]], scale)
     ts = []
     for _ in range(args.steps):
         t0 = time.perf_counter()
-        oatt.decode_batch(q, [k, k], [v, v], scale)
+        oatt.decode_batch(q, ks, vs, scale)
         ts.append(time.perf_counter() - t0)
     t = sum(ts)
-    value = 2 * args.steps / (t * L)
-    sample = (f"per step: 2 sequences (main + aux) x 1 of {L} layers at {n} tokens, all {Hq} heads, "
-              f"fp64 C oracle with OpenMP; tokens/s = sequences / (time x {L} layers)")
+    value = 2 * R * args.steps / (t * L)
+    sample = (f"per step: one decode call of all {2 * R} sequences (main + fork) x 1 of {L} layers "
+              f"at {n} tokens, all {Hq} heads, fp64 C oracle with OpenMP; "
+              f"tokens/s = sequences / (seconds per layer x {L} layers)")
     return {
         "metric": METRIC, "value": round(value, 4), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(t / args.steps * 1e3, 3),
