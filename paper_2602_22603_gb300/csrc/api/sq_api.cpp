@@ -517,7 +517,7 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
     hit->last_use = ++c->use_clock;
     const DecodePlanLayout& L = hit->lay;
     float* part_o = hit->d_part;
-    float* part_ml = part_o + (size_t)L.n_items * kDecodeConsumerWarps * kRowsPerTile * g.D;
+    float* part_ml = part_o + (size_t)L.n_items * kRowsPerTile * g.D;
 
     DecodeArgs a;
     a.segs = reinterpret_cast<const DecodeSeg*>(hit->d_plan + L.segs);
@@ -741,7 +741,7 @@ int sq_decode_attention_noalloc(sq_cache* c, const sq_seq* seqs, int32_t n_seqs,
     cudaError_t e = cudaMemcpyAsync(scratch, c->staging.data(), L.total, cudaMemcpyHostToDevice, st);
     if (e != cudaSuccess) return cuda_status(e);
     float* part_o = reinterpret_cast<float*>(scratch + part_off);
-    float* part_ml = part_o + (size_t)L.n_items * kDecodeConsumerWarps * kRowsPerTile * g.D;
+    float* part_ml = part_o + (size_t)L.n_items * kRowsPerTile * g.D;
 
     DecodeArgs a;
     a.segs = reinterpret_cast<const DecodeSeg*>(scratch + L.segs);

@@ -441,35 +441,39 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
         for (auto it = next.rbegin(); it != next.rend(); ++it) stack.push_back(std::move(*it));
     }
 
-    // (segment, head) units, stage counts, and an even split of all stages
-    // over the persistent CTAs.
+    // (segment, head) units and an even split of their cost over the
+    // persistent CTAs.  On the cost line a unit occupies kUnitCostStages
+    // (its start-up) followed by its stages; an item is the overlap of a
+    // CTA's share with a unit's stages.
     const int32_t n_segs = (int32_t)out->segs.size();
-    std::vector<int64_t> unit_start;
+    std::vector<int64_t> unit_start;  // where the unit's stages begin on the cost line
+    std::vector<int64_t> unit_end;
     int64_t total = 0;
     for (int32_t s = 0; s < n_segs; ++s)
         for (int32_t h = 0; h < g.Hkv; ++h) {
+            total += kUnitCostStages;
             unit_start.push_back(total);
             total += ceil_div(out->segs[s].n_tok, kStageTokens);
+            unit_end.push_back(total);
         }
-    unit_start.push_back(total);
-    const int32_t ctas = (int32_t)std::min<int64_t>(n_ctas, total);
+    const int64_t n_units = (int64_t)unit_start.size();
+    const int32_t ctas = (int32_t)std::min<int64_t>(n_ctas, total - n_units * kUnitCostStages);
     out->n_ctas = ctas;
     out->cta_begin.resize(ctas + 1);
-    size_t u = 0;
+    int64_t u = 0;
     for (int32_t cta = 0; cta < ctas; ++cta) {
         const int64_t b = total * cta / ctas, e = total * (cta + 1) / ctas;
         out->cta_begin[cta] = (int32_t)out->items.size();
-        int64_t pos = b;
-        while (pos < e) {
-            while (unit_start[u + 1] <= pos) ++u;
-            const int64_t stop = std::min(e, unit_start[u + 1]);
+        while (u < n_units && unit_end[u] <= b) ++u;
+        for (int64_t v = u; v < n_units && unit_start[v] - kUnitCostStages < e; ++v) {
+            const int64_t lo = std::max(b, unit_start[v]), hi = std::min(e, unit_end[v]);
+            if (hi <= lo) continue;
             DecodeItem it;
-            it.seg = (int32_t)(u / g.Hkv);
-            it.head = (int32_t)(u % g.Hkv);
-            it.s0 = (int32_t)(pos - unit_start[u]);
-            it.s1 = (int32_t)(stop - unit_start[u]);
+            it.seg = (int32_t)(v / g.Hkv);
+            it.head = (int32_t)(v % g.Hkv);
+            it.s0 = (int32_t)(lo - unit_start[v]);
+            it.s1 = (int32_t)(hi - unit_start[v]);
             out->items.push_back(it);
-            pos = stop;
         }
     }
     out->cta_begin[ctas] = (int32_t)out->items.size();

@@ -13,6 +13,11 @@ constexpr int kRowsPerTile = 16;
 constexpr int kStageTokens = 64;
 // Consumer warps of the decode kernel; each owns kStageTokens / 4 tokens.
 constexpr int kDecodeConsumerWarps = 4;
+// Fixed cost of starting a work unit, in stages: its query reload and its
+// item-end merge.  The planner balances stages plus this cost per unit, so a
+// CTA that gets many short units (e.g. the few-token tails of several forks)
+// is not the one every other CTA waits for.
+constexpr int kUnitCostStages = 2;
 
 // A run of logical pages read once for a group of sequences that hold the
 // same physical pages there (a main thread and its forks, Sec. 3.4).

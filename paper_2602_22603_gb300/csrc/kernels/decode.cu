@@ -39,7 +39,13 @@ struct DecCfg {
     static constexpr int kStageBytes = 2 * kTileBytes;
     static constexpr int kStages = (D == 128) ? 3 : 6;
     static constexpr int kThreads = (kDecodeConsumerWarps + 1) * 32;
-    static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 128;
+    // item-end merge of the four consumer warps: per-warp row max / sum,
+    // and one 16-row output tile
+    static constexpr int kMergeStride = D + 8;  // floats per merge row (padded: fewer bank conflicts)
+    static constexpr int kMergeBytes = 2 * kDecodeConsumerWarps * kRowsPerTile * 4 +
+                                       kRowsPerTile * kMergeStride * 4;
+    // + 1024 alignment slack + 256 for the mbarriers and flags
+    static constexpr int kSmemBytes = kStages * kStageBytes + kMergeBytes + 1024 + 256;
     static constexpr int kNT = D / 8;   // 8-wide output column tiles
     static constexpr int kKS = D / 16;  // 16-deep contraction steps
 };
@@ -74,8 +80,8 @@ __device__ void produce(const CUtensorMap* tmap, const DecodeArgs& a, int it0, i
         for (int s = item.s0; s < item.s1; ++s) {
             const uint32_t full = smem_addr(&bars[slot]);
             const uint32_t empty = smem_addr(&bars[C::kStages + slot]);
-            if (!mbar_wait(empty, phase ^ 1)) {
-                set_error(a.err, kErrTimeout);
+            if (!mbar_wait(empty, phase ^ 1, abort_flag)) {
+                if (!*abort_flag) set_error(a.err, kErrTimeout);
                 *abort_flag = 1;
                 ok = false;
                 break;
@@ -131,15 +137,22 @@ __device__ void produce(const CUtensorMap* tmap, const DecodeArgs& a, int it0, i
 }
 
 // ---- consumers: four warps, 16 tokens of every stage each ------------------
+// Every consumer warp runs every item and every stage and reaches every
+// named barrier of every item, also after a wait ran out (it then skips the
+// work only), so the barriers never miss a participant.
 template <int D>
 __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, uint64_t* bars,
-                        volatile int* abort_flag, int warp, int lane) {
+                        volatile int* abort_flag, float* merge, int warp, int lane) {
     using C = DecCfg<D>;
     const int gid = lane >> 2, tig = lane & 3;
     const int r0 = gid, r1 = gid + 8;
     const int mi = lane >> 3, rr = lane & 7;
+    float* red_m = merge;                                          // [4][16]
+    float* red_l = merge + kDecodeConsumerWarps * kRowsPerTile;    // [4][16]
+    float* red_o = merge + 2 * kDecodeConsumerWarps * kRowsPerTile;  // [16][kMergeStride]
     int slot = 0;
     uint32_t phase = 0;
+    bool dead = false;  // warp-uniform: a wait ran out or the CTA aborted
     for (int it = it0; it < it1; ++it) {
         const DecodeItem item = a.items[it];
         const DecodeSeg* seg = a.segs + item.seg;
@@ -174,146 +187,192 @@ __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, ui
         for (int s = item.s0; s < item.s1; ++s) {
             const uint32_t full = smem_addr(&bars[slot]);
             const uint32_t empty = smem_addr(&bars[C::kStages + slot]);
-            if (!mbar_wait(full, phase)) {
-                set_error(a.err, kErrTimeout);
-                *abort_flag = 1;
-                return;
-            }
-            const uint32_t kb = smem_addr(smem + slot * C::kStageBytes);
-            const uint32_t vb = kb + C::kTileBytes;
-            const int tbase = s * kStageTokens + warp * 16;  // segment-relative
-
-            // S = Q K^T over this warp's 16 tokens (two n8 tiles)
-            float sc[2][4];
-#pragma unroll
-            for (int nt = 0; nt < 2; ++nt) sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
-            {
-                const int t = warp * 16 + (mi >> 1) * 8 + rr;
-                const uint32_t row = kb + t * 128;
-                const int sw = t & 7;
-#pragma unroll
-                for (int kk = 0; kk < C::kKS; ++kk) {
-                    const int d0 = kk * 16 + (mi & 1) * 8;
-                    uint32_t b0, b1, b2, b3;
-                    ldsm_x4(row + (d0 >> 6) * C::kBlockBytes + ((((d0 & 63) >> 3) ^ sw) << 4), b0,
-                            b1, b2, b3);
-                    mma_bf16(sc[0], qa[kk], b0, b1);
-                    mma_bf16(sc[1], qa[kk], b2, b3);
+            if (!dead) {
+                const bool ok = mbar_wait(full, phase, abort_flag);
+                if (!__all_sync(0xffffffffu, ok)) {
+                    if (lane == 0 && !*abort_flag) set_error(a.err, kErrTimeout);
+                    *abort_flag = 1;
+                    dead = true;
                 }
             }
+            if (!dead) {
+                const uint32_t kb = smem_addr(smem + slot * C::kStageBytes);
+                const uint32_t vb = kb + C::kTileBytes;
+                const int tbase = s * kStageTokens + warp * 16;  // segment-relative
 
-            // masking, scaling, online softmax (log2 domain)
-            float x[2][4];
-            float mx0 = -INFINITY, mx1 = -INFINITY;
+                // S = Q K^T over this warp's 16 tokens (two n8 tiles)
+                float sc[2][4];
 #pragma unroll
-            for (int nt = 0; nt < 2; ++nt)
+                for (int nt = 0; nt < 2; ++nt) sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+                {
+                    const int t = warp * 16 + (mi >> 1) * 8 + rr;
+                    const uint32_t row = kb + t * 128;
+                    const int sw = t & 7;
 #pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const int tk = tbase + nt * 8 + tig * 2 + e;
-                    x[nt][e] = tk < lim0 ? sc[nt][e] * a.scale_log2 : -INFINITY;
-                    x[nt][2 + e] = tk < lim1 ? sc[nt][2 + e] * a.scale_log2 : -INFINITY;
-                    mx0 = fmaxf(mx0, x[nt][e]);
-                    mx1 = fmaxf(mx1, x[nt][2 + e]);
+                    for (int kk = 0; kk < C::kKS; ++kk) {
+                        const int d0 = kk * 16 + (mi & 1) * 8;
+                        uint32_t b0, b1, b2, b3;
+                        ldsm_x4(row + (d0 >> 6) * C::kBlockBytes + ((((d0 & 63) >> 3) ^ sw) << 4), b0,
+                                b1, b2, b3);
+                        mma_bf16(sc[0], qa[kk], b0, b1);
+                        mma_bf16(sc[1], qa[kk], b2, b3);
+                    }
                 }
-            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-            const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-            const float ms0 = mn0 == -INFINITY ? 0.f : mn0;
-            const float ms1 = mn1 == -INFINITY ? 0.f : mn1;
-            const float al0 = exp2f(m0 - ms0), al1 = exp2f(m1 - ms1);
-            m0 = mn0;
-            m1 = mn1;
-#pragma unroll
-            for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    x[nt][e] = exp2f(x[nt][e] - ms0);
-                    x[nt][2 + e] = exp2f(x[nt][2 + e] - ms1);
-                }
-            // P in bf16 for the PV product; the normaliser sums the same
-            // rounded weights, so the output is an exact convex combination
-            uint32_t pa[4];
-            pa[0] = pack_bf16x2(x[0][0], x[0][1]);
-            pa[1] = pack_bf16x2(x[0][2], x[0][3]);
-            pa[2] = pack_bf16x2(x[1][0], x[1][1]);
-            pa[3] = pack_bf16x2(x[1][2], x[1][3]);
-            const float ps0 = bf16x2_sum(pa[0]) + bf16x2_sum(pa[2]);
-            const float ps1 = bf16x2_sum(pa[1]) + bf16x2_sum(pa[3]);
-            l0 = l0 * al0 + ps0;
-            l1 = l1 * al1 + ps1;
-#pragma unroll
-            for (int nd = 0; nd < C::kNT; ++nd) {
-                o[nd][0] *= al0;
-                o[nd][1] *= al0;
-                o[nd][2] *= al1;
-                o[nd][3] *= al1;
-            }
 
-            // Rows past the last valid token hold stale or never-written
-            // shared memory: zero this warp's such V rows so 0 * V stays 0.
-            const bool tail = tbase + 16 > n_tok;
-            if (tail) {
-                const int first = max(0, n_tok - tbase);
-                const int per_row = C::kColBlocks * 8;  // 16-byte chunks per row
-                const int total = (16 - first) * per_row;
-                uint8_t* vgen = smem + slot * C::kStageBytes + C::kTileBytes;
-                for (int idx = lane; idx < total; idx += 32) {
-                    const int row = warp * 16 + first + idx / per_row;
-                    const int rem = idx % per_row;
-                    *reinterpret_cast<uint4*>(vgen + (rem >> 3) * C::kBlockBytes + row * 128 +
-                                              (rem & 7) * 16) = make_uint4(0, 0, 0, 0);
+                // masking, scaling, online softmax (log2 domain)
+                float x[2][4];
+                float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+                for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        const int tk = tbase + nt * 8 + tig * 2 + e;
+                        x[nt][e] = tk < lim0 ? sc[nt][e] * a.scale_log2 : -INFINITY;
+                        x[nt][2 + e] = tk < lim1 ? sc[nt][2 + e] * a.scale_log2 : -INFINITY;
+                        mx0 = fmaxf(mx0, x[nt][e]);
+                        mx1 = fmaxf(mx1, x[nt][2 + e]);
+                    }
+                mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+                mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+                mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+                mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+                const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+                const float ms0 = mn0 == -INFINITY ? 0.f : mn0;
+                const float ms1 = mn1 == -INFINITY ? 0.f : mn1;
+                const float al0 = exp2f(m0 - ms0), al1 = exp2f(m1 - ms1);
+                m0 = mn0;
+                m1 = mn1;
+#pragma unroll
+                for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        x[nt][e] = exp2f(x[nt][e] - ms0);
+                        x[nt][2 + e] = exp2f(x[nt][2 + e] - ms1);
+                    }
+                // P in bf16 for the PV product; the normaliser sums the same
+                // rounded weights, so the output is an exact convex combination
+                uint32_t pa[4];
+                pa[0] = pack_bf16x2(x[0][0], x[0][1]);
+                pa[1] = pack_bf16x2(x[0][2], x[0][3]);
+                pa[2] = pack_bf16x2(x[1][0], x[1][1]);
+                pa[3] = pack_bf16x2(x[1][2], x[1][3]);
+                const float ps0 = bf16x2_sum(pa[0]) + bf16x2_sum(pa[2]);
+                const float ps1 = bf16x2_sum(pa[1]) + bf16x2_sum(pa[3]);
+                l0 = l0 * al0 + ps0;
+                l1 = l1 * al1 + ps1;
+#pragma unroll
+                for (int nd = 0; nd < C::kNT; ++nd) {
+                    o[nd][0] *= al0;
+                    o[nd][1] *= al0;
+                    o[nd][2] *= al1;
+                    o[nd][3] *= al1;
                 }
+
+                // Rows past the last valid token hold stale or never-written
+                // shared memory: zero this warp's such V rows so 0 * V stays 0.
+                const bool tail = tbase + 16 > n_tok;
+                if (tail) {
+                    const int first = max(0, n_tok - tbase);
+                    const int per_row = C::kColBlocks * 8;  // 16-byte chunks per row
+                    const int total = (16 - first) * per_row;
+                    uint8_t* vgen = smem + slot * C::kStageBytes + C::kTileBytes;
+                    for (int idx = lane; idx < total; idx += 32) {
+                        const int row = warp * 16 + first + idx / per_row;
+                        const int rem = idx % per_row;
+                        *reinterpret_cast<uint4*>(vgen + (rem >> 3) * C::kBlockBytes + row * 128 +
+                                                  (rem & 7) * 16) = make_uint4(0, 0, 0, 0);
+                    }
+                    __syncwarp();
+                }
+
+                // O += P V (V^T fragments through ldmatrix.trans)
+                {
+                    const int t = warp * 16 + (mi & 1) * 8 + rr;
+                    const uint32_t row = vb + t * 128;
+                    const int sw = t & 7;
+#pragma unroll
+                    for (int nd2 = 0; nd2 < C::kKS; ++nd2) {
+                        const int d0 = nd2 * 16 + (mi >> 1) * 8;
+                        uint32_t b0, b1, b2, b3;
+                        ldsm_x4_trans(row + (d0 >> 6) * C::kBlockBytes + ((((d0 & 63) >> 3) ^ sw) << 4),
+                                      b0, b1, b2, b3);
+                        mma_bf16(o[2 * nd2], pa, b0, b1);
+                        mma_bf16(o[2 * nd2 + 1], pa, b2, b3);
+                    }
+                }
+                if (tail) fence_proxy_async_smem();  // generic writes before the next TMA fill
                 __syncwarp();
+                if (lane == 0) mbar_arrive(empty);
             }
-
-            // O += P V (V^T fragments through ldmatrix.trans)
-            {
-                const int t = warp * 16 + (mi & 1) * 8 + rr;
-                const uint32_t row = vb + t * 128;
-                const int sw = t & 7;
-#pragma unroll
-                for (int nd2 = 0; nd2 < C::kKS; ++nd2) {
-                    const int d0 = nd2 * 16 + (mi >> 1) * 8;
-                    uint32_t b0, b1, b2, b3;
-                    ldsm_x4_trans(row + (d0 >> 6) * C::kBlockBytes + ((((d0 & 63) >> 3) ^ sw) << 4),
-                                  b0, b1, b2, b3);
-                    mma_bf16(o[2 * nd2], pa, b0, b1);
-                    mma_bf16(o[2 * nd2 + 1], pa, b2, b3);
-                }
-            }
-            if (tail) fence_proxy_async_smem();  // generic writes before the next TMA fill
-            __syncwarp();
-            if (lane == 0) mbar_arrive(empty);
             if (++slot == C::kStages) {
                 slot = 0;
                 phase ^= 1;
             }
         }
 
-        // close the item: full row sums, then the partial (o, m, l)
+        // close the item: merge the four warps' (m, l, o) in shared memory,
+        // then write one partial (unnormalised o, m, l) for the item
         l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
         l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
         l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
         l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-        const size_t pidx = (size_t)it * kDecodeConsumerWarps + warp;
-        float* po = a.part_o + pidx * kRowsPerTile * D;
-        float* pml = a.part_ml + pidx * kRowsPerTile * 2;
-        if (v0) {
-#pragma unroll
-            for (int nd = 0; nd < C::kNT; ++nd)
-                *reinterpret_cast<float2*>(po + r0 * D + nd * 8 + tig * 2) =
-                    make_float2(o[nd][0], o[nd][1]);
-            if (tig == 0) *reinterpret_cast<float2*>(pml + r0 * 2) = make_float2(m0, l0);
+        if (tig == 0) {
+            red_m[warp * kRowsPerTile + r0] = dead ? -INFINITY : m0;
+            red_m[warp * kRowsPerTile + r1] = dead ? -INFINITY : m1;
+            red_l[warp * kRowsPerTile + r0] = dead ? 0.f : l0;
+            red_l[warp * kRowsPerTile + r1] = dead ? 0.f : l1;
         }
-        if (v1) {
+        named_bar_sync(1, kDecodeConsumerWarps * 32);
+        float M0 = -INFINITY, M1 = -INFINITY;
 #pragma unroll
-            for (int nd = 0; nd < C::kNT; ++nd)
-                *reinterpret_cast<float2*>(po + r1 * D + nd * 8 + tig * 2) =
-                    make_float2(o[nd][2], o[nd][3]);
-            if (tig == 0) *reinterpret_cast<float2*>(pml + r1 * 2) = make_float2(m1, l1);
+        for (int w = 0; w < kDecodeConsumerWarps; ++w) {
+            M0 = fmaxf(M0, red_m[w * kRowsPerTile + r0]);
+            M1 = fmaxf(M1, red_m[w * kRowsPerTile + r1]);
         }
+        const float Ms0 = M0 == -INFINITY ? 0.f : M0, Ms1 = M1 == -INFINITY ? 0.f : M1;
+        const float f0 = dead ? 0.f : exp2f(m0 - Ms0), f1 = dead ? 0.f : exp2f(m1 - Ms1);
+        for (int w = 0; w < kDecodeConsumerWarps; ++w) {
+            if (w == warp) {
+#pragma unroll
+                for (int nd = 0; nd < C::kNT; ++nd) {
+                    float2* p0 = reinterpret_cast<float2*>(red_o + r0 * C::kMergeStride + nd * 8 + tig * 2);
+                    float2* p1 = reinterpret_cast<float2*>(red_o + r1 * C::kMergeStride + nd * 8 + tig * 2);
+                    float2 a0 = dead ? make_float2(0.f, 0.f) : make_float2(o[nd][0] * f0, o[nd][1] * f0);
+                    float2 a1 = dead ? make_float2(0.f, 0.f) : make_float2(o[nd][2] * f1, o[nd][3] * f1);
+                    if (w > 0) {
+                        const float2 b0 = *p0, b1 = *p1;
+                        a0.x += b0.x; a0.y += b0.y;
+                        a1.x += b1.x; a1.y += b1.y;
+                    }
+                    *p0 = a0;
+                    *p1 = a1;
+                }
+            }
+            named_bar_sync(1, kDecodeConsumerWarps * 32);
+        }
+        // the merged tile: rows of the group's query heads, plus their (M, L)
+        const int rows = n_grp * G;
+        float* po = a.part_o + (size_t)it * kRowsPerTile * D;
+        constexpr int kVecRow = D / 4;  // float4 per row
+        for (int v = threadIdx.x; v < rows * kVecRow; v += kDecodeConsumerWarps * 32)
+            reinterpret_cast<float4*>(po)[v] = *reinterpret_cast<const float4*>(
+                red_o + (v / kVecRow) * C::kMergeStride + (v % kVecRow) * 4);
+        if (threadIdx.x < rows) {
+            const int r = threadIdx.x;
+            float M = -INFINITY;
+#pragma unroll
+            for (int w = 0; w < kDecodeConsumerWarps; ++w) M = fmaxf(M, red_m[w * kRowsPerTile + r]);
+            const float Ms = M == -INFINITY ? 0.f : M;
+            float L = 0.f;
+#pragma unroll
+            for (int w = 0; w < kDecodeConsumerWarps; ++w)
+                L += red_l[w * kRowsPerTile + r] * exp2f(red_m[w * kRowsPerTile + r] - Ms);
+            *reinterpret_cast<float2*>(a.part_ml + ((size_t)it * kRowsPerTile + r) * 2) =
+                make_float2(M, L);
+        }
+        // the merge buffers are rewritten by the next item only after every
+        // warp has copied them out
+        named_bar_sync(1, kDecodeConsumerWarps * 32);
     }
 }
 
@@ -326,6 +385,7 @@ __global__ void __launch_bounds__(DecCfg<D>::kThreads, 2)
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 2 * C::kStages);
+    float* merge = reinterpret_cast<float*>(smem + C::kStages * C::kStageBytes + 256);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::kStages; ++s) {
@@ -341,13 +401,16 @@ __global__ void __launch_bounds__(DecCfg<D>::kThreads, 2)
         if (lane == 0) produce<D>(&tmap, a, it0, it1, smem, bars, abort_flag);
         return;
     }
-    consume<D>(a, it0, it1, smem, bars, abort_flag, warp, lane);
+    consume<D>(a, it0, it1, smem, bars, abort_flag, merge, warp, lane);
 }
 
 // ---- combine: one warp per (sequence, query head) ---------------------------
+// Max of the partial maxima, weights 2^(m_c - M), weighted sums of the
+// unnormalised outputs and of the sums; loads of up to 8 partials in flight.
 template <int D>
 __global__ void __launch_bounds__(256) sq_lse_combine_kernel(const CombineArgs a) {
     constexpr int V = D / 32;  // output elements per lane
+    constexpr int U = 8;       // partials per batch of loads
     const int wid = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
     if (wid >= a.n_seqs * a.Hq) return;
@@ -355,14 +418,12 @@ __global__ void __launch_bounds__(256) sq_lse_combine_kernel(const CombineArgs a
     const int hh = h % a.G;
     const int key = i * a.Hkv + h / a.G;
     const int e0 = a.comb_off[key], e1 = a.comb_off[key + 1];
-    const int np = (e1 - e0) * kDecodeConsumerWarps;
+    const int np = e1 - e0;
 
     float M = -INFINITY;
     for (int k = lane; k < np; k += 32) {
-        const CombineEnt ent = a.comb_ent[e0 + k / kDecodeConsumerWarps];
-        const size_t p = (size_t)ent.item * kDecodeConsumerWarps + k % kDecodeConsumerWarps;
-        const int r = ent.j * a.G + hh;
-        M = fmaxf(M, a.part_ml[(p * kRowsPerTile + r) * 2]);
+        const CombineEnt ent = a.comb_ent[e0 + k];
+        M = fmaxf(M, a.part_ml[((size_t)ent.item * kRowsPerTile + ent.j * a.G + hh) * 2]);
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
@@ -372,25 +433,34 @@ __global__ void __launch_bounds__(256) sq_lse_combine_kernel(const CombineArgs a
 #pragma unroll
     for (int e = 0; e < V; ++e) acc[e] = 0.f;
     float L = 0.f;
-    for (int k = 0; k < np; ++k) {
-        const CombineEnt ent = a.comb_ent[e0 + k / kDecodeConsumerWarps];
-        const size_t p = (size_t)ent.item * kDecodeConsumerWarps + k % kDecodeConsumerWarps;
-        const size_t row = p * kRowsPerTile + ent.j * a.G + hh;
-        const float2 ml = *reinterpret_cast<const float2*>(a.part_ml + row * 2);
-        const float w = exp2f(ml.x - Ms);
-        L += w * ml.y;
-        const float* po = a.part_o + row * D + lane * V;
-        if constexpr (V == 4) {
-            const float4 v = *reinterpret_cast<const float4*>(po);
-            acc[0] += w * v.x;
-            acc[1] += w * v.y;
-            acc[2] += w * v.z;
-            acc[3] += w * v.w;
-        } else {
-            const float2 v = *reinterpret_cast<const float2*>(po);
-            acc[0] += w * v.x;
-            acc[1] += w * v.y;
+    for (int k0 = 0; k0 < np; k0 += U) {
+        float w[U];
+        float vals[U][V];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            w[u] = 0.f;
+#pragma unroll
+            for (int e = 0; e < V; ++e) vals[u][e] = 0.f;
+            if (k0 + u < np) {
+                const CombineEnt ent = a.comb_ent[e0 + k0 + u];
+                const size_t row = (size_t)ent.item * kRowsPerTile + ent.j * a.G + hh;
+                const float2 ml = *reinterpret_cast<const float2*>(a.part_ml + row * 2);
+                w[u] = exp2f(ml.x - Ms);
+                L += w[u] * ml.y;
+                const float* po = a.part_o + row * D + lane * V;
+                if constexpr (V == 4) {
+                    const float4 v = *reinterpret_cast<const float4*>(po);
+                    vals[u][0] = v.x; vals[u][1] = v.y; vals[u][2] = v.z; vals[u][3] = v.w;
+                } else {
+                    const float2 v = *reinterpret_cast<const float2*>(po);
+                    vals[u][0] = v.x; vals[u][1] = v.y;
+                }
+            }
         }
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+#pragma unroll
+            for (int e = 0; e < V; ++e) acc[e] += w[u] * vals[u][e];
     }
     const float inv = 1.f / L;
     const size_t ob = ((size_t)i * a.Hq + h) * D + lane * V;
@@ -417,18 +487,22 @@ __global__ void __launch_bounds__(256) sq_lse_combine_kernel(const CombineArgs a
 }  // namespace
 
 int64_t decode_partial_bytes(int32_t n_items, int32_t D) {
-    return (int64_t)n_items * kDecodeConsumerWarps * kRowsPerTile * (D + 2) * (int64_t)sizeof(float);
+    return (int64_t)n_items * kRowsPerTile * (D + 2) * (int64_t)sizeof(float);
 }
 
-cudaError_t decode_prepare(int D) {
-    if (D == 128)
-        return cudaFuncSetAttribute(sq_decode_splitk_kernel<128>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    DecCfg<128>::kSmemBytes);
-    return cudaFuncSetAttribute(sq_decode_splitk_kernel<64>,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                DecCfg<64>::kSmemBytes);
+template <int D>
+static cudaError_t prepare_one() {
+    cudaError_t e = cudaFuncSetAttribute(sq_decode_splitk_kernel<D>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         DecCfg<D>::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    // the largest shared-memory carveout, so that two CTAs fit on an SM
+    return cudaFuncSetAttribute(sq_decode_splitk_kernel<D>,
+                                cudaFuncAttributePreferredSharedMemoryCarveout,
+                                cudaSharedmemCarveoutMaxShared);
 }
+
+cudaError_t decode_prepare(int D) { return D == 128 ? prepare_one<128>() : prepare_one<64>(); }
 
 int decode_ctas_per_sm(int D) {
     int n = 0;

@@ -17,8 +17,8 @@ struct DecodeArgs {
     const int32_t* cta_begin;
     const int32_t* page_ids;
     const __nv_bfloat16* q;     // [n_seqs][Hq][D]
-    float* part_o;              // [n_items * 4][16][D]  unnormalised partial outputs
-    float* part_ml;             // [n_items * 4][16][2]  running max (log2 units), sum
+    float* part_o;              // [n_items][16][D]  unnormalised partial outputs
+    float* part_ml;             // [n_items][16][2]  max (log2 units), sum
     int32_t layer, Hq, Hkv, G, P, num_pages;
     float scale_log2;           // sm_scale * log2(e)
     int* err;

@@ -109,10 +109,13 @@ def _check_plan(hc, handles, plan, n_ctas, G):
     assert cb[0] == 0 and cb[-1] == len(items)
     assert all(cb[i] <= cb[i + 1] for i in range(len(cb) - 1))
     assert len(cb) - 1 <= n_ctas
-    # stages per CTA are balanced to within one stage
-    per_cta = [sum(items[i][3] - items[i][2] for i in range(cb[c], cb[c + 1]))
+    # work per CTA (stages + a fixed cost per item) is balanced: within one
+    # unit start-up cost plus one stage
+    C = 2
+    per_cta = [sum(items[i][3] - items[i][2] + C for i in range(cb[c], cb[c + 1]))
                for c in range(len(cb) - 1)]
-    assert max(per_cta) - min(per_cta) <= 1
+    busy = [x for x in per_cta if x > 0]
+    assert max(busy) - min(busy) <= 2 * C + 1
     for s in segs:
         assert 1 <= s["n_grp"] <= 16 // G
         assert max(s["grp_lim"]) == s["n_tok"] and min(s["grp_lim"]) > 0
