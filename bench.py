@@ -183,6 +183,28 @@ def workload_name(args):
             f"page 64, bf16")
 
 
+def read_probe(cache, stream, nbytes=8 << 30, reps=5):
+    """Read-only HBM bandwidth of this GPU in this run (sq_probe_read over
+    8 GiB, best of 5), reported next to the copy peak."""
+    import torch
+
+    import paper_2602_22603_gb300 as sq
+    buf = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    st_h = int(stream.cuda_stream)
+    sq.sq_probe_read(cache.handle, buf, nbytes, st_h)
+    best = 0.0
+    for _ in range(reps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        sq.sq_probe_read(cache.handle, buf, nbytes, st_h)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        best = max(best, nbytes / (e0.elapsed_time(e1) / 1e3) / 1e9)
+    del buf
+    torch.cuda.empty_cache()
+    return best
+
+
 def run_sq(args, world, rank, local):
     import numpy as np
     import torch
@@ -291,6 +313,7 @@ def run_sq(args, world, rank, local):
                 "logical_bytes": logi}
 
     hbm_peak, peak_kind = peaks()
+    probe_gbs = read_probe(cache, stream)
     clocks = ClockSampler(local)
     time.sleep(0.4)
     K, W = args.steps, args.warmup
@@ -345,6 +368,8 @@ def run_sq(args, world, rank, local):
             "peak_kind": peak_kind,
             "unit": "GB/s",
             "frac": round(achieved / hbm_peak, 4),
+            "read_probe_gbs": round(probe_gbs, 1),
+            "frac_of_read_probe": round(achieved / probe_gbs, 4),
             "traffic": int(ratio * uniq_per_call) if ratio else None,
             "traffic_source": (ratio_src + ": small-case DRAM bytes per algorithmic byte, scaled "
                                "to this launch's algorithmic bytes") if ratio else None,

@@ -239,6 +239,12 @@ SQ_API int sq_decode_attention_noalloc(sq_cache *cache, const sq_seq *seqs, int3
                                        int32_t layer, const void *q, void *out,
                                        int32_t out_dtype, float sm_scale, void *stream);
 
+/* Measurement helper: streams `bytes` (a multiple of 16, 16-byte aligned)
+ * of device memory at `buf` once with plain loads and no writes, so that the
+ * caller can time the read-only HBM bandwidth of this GPU next to the
+ * library's kernels.  Not part of the method.  Errors: INVALID_ARG, CUDA. */
+SQ_API int sq_probe_read(sq_cache *cache, const void *buf, size_t bytes, void *stream);
+
 /* Synchronise `stream`, then read and clear the device error word.
  * Returns SQ_OK, SQ_ERR_DEVICE, SQ_ERR_DEVICE_TIMEOUT or SQ_ERR_CUDA. */
 SQ_API int sq_sync_status(sq_cache *cache, void *stream);

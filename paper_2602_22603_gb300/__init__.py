@@ -93,6 +93,7 @@ _SIGS = {
     "sq_stats": (ctypes.c_int, [_P, ctypes.POINTER(sq_stats_t)]),
     "sq_sync_status": (ctypes.c_int, [_P, _P]),
     "sq_strerror": (ctypes.c_char_p, [ctypes.c_int]),
+    "sq_probe_read": (ctypes.c_int, [_P, _P, ctypes.c_size_t, _P]),
     "sq_decode_attention_noalloc": (ctypes.c_int, [_P, _I32P, _I32, _I32, _P, _P, _I32,
                                                    ctypes.c_float, _P]),
 }
@@ -248,6 +249,10 @@ def sq_stats(cache: int) -> dict:
     st = sq_stats_t()
     _check(lib().sq_stats(cache, ctypes.byref(st)), "sq_stats")
     return st.as_dict()
+
+
+def sq_probe_read(cache: int, buf, nbytes: int, stream=None) -> None:
+    _check(lib().sq_probe_read(cache, _ptr(buf), nbytes, _stream(stream)), "sq_probe_read")
 
 
 def sq_sync_status(cache: int, stream=None) -> int:

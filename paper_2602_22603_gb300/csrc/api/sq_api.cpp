@@ -322,9 +322,10 @@ int sq_cache_create(const sq_config* cfg, sq_cache** out) {
         if (c->d_err) cudaFree(c->d_err);
         return code;
     };
-    e = cudaMalloc(&c->d_err, sizeof(int));
+    // [0] device error word, [1] sink of the read probe
+    e = cudaMalloc(&c->d_err, 4 * sizeof(int));
     if (e != cudaSuccess) return fail(cuda_status(e));
-    e = cudaMemset(c->d_err, 0, sizeof(int));
+    e = cudaMemset(c->d_err, 0, 4 * sizeof(int));
     if (e != cudaSuccess) return fail(cuda_status(e));
     rc = make_tensor_map(c.get());
     if (rc != SQ_OK) return fail(rc);
@@ -690,6 +691,15 @@ int sq_stats(sq_cache* c, sq_stats_t* out) {
     out->live_pages = c->host->live_pages();
     out->peak_live_pages = c->host->peak_live_pages();
     return SQ_OK;
+}
+
+int sq_probe_read(sq_cache* c, const void* buf, size_t bytes, void* stream) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    if (!buf || bytes == 0 || (bytes & 15) || (reinterpret_cast<uintptr_t>(buf) & 15))
+        return SQ_ERR_INVALID_ARG;
+    cudaError_t e = launch_read_probe(buf, bytes, reinterpret_cast<unsigned int*>(c->d_err) + 1,
+                                      c->num_sms, as_stream(stream));
+    return cuda_status(e);
 }
 
 int sq_sync_status(sq_cache* c, void* stream) {

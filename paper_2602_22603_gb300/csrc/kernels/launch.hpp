@@ -91,4 +91,8 @@ int evict_ctas_per_sm(int tile_rows, int D);
 cudaError_t evict_prepare();  // raises the dynamic shared-memory limit once
 cudaError_t launch_evict(const EvictArgs& a, cudaStream_t st);
 
+// Read-only streaming probe over `bytes` (multiple of 16) at `buf`.
+cudaError_t launch_read_probe(const void* buf, size_t bytes, unsigned int* sink, int num_sms,
+                              cudaStream_t st);
+
 }  // namespace sq
