@@ -245,6 +245,17 @@ SQ_API int sq_decode_attention_noalloc(sq_cache *cache, const sq_seq *seqs, int3
  * library's kernels.  Not part of the method.  Errors: INVALID_ARG, CUDA. */
 SQ_API int sq_probe_read(sq_cache *cache, const void *buf, size_t bytes, void *stream);
 
+/* Test hook for failure detection (no counterpart in the paper).
+ * SQ_DEBUG_DROP_DECODE_STAGE: in the next decode call, the first persistent
+ * CTA leaves its first pipeline stage unsignalled, so that CTA's consumer
+ * warps wait on a barrier nothing completes.  Their wait is bounded: after
+ * about 2 s they give up, the CTA winds down without faulting, the output of
+ * that call is undefined, and sq_sync_status returns SQ_ERR_DEVICE_TIMEOUT;
+ * the cache and the CUDA context stay usable.  The flag clears itself after
+ * one call.  0 clears it.  Errors: BAD_HANDLE, INVALID_ARG. */
+enum { SQ_DEBUG_DROP_DECODE_STAGE = 1 };
+SQ_API int sq_debug_set(sq_cache *cache, int32_t flags);
+
 /* Synchronise `stream`, then read and clear the device error word.
  * Returns SQ_OK, SQ_ERR_DEVICE, SQ_ERR_DEVICE_TIMEOUT or SQ_ERR_CUDA. */
 SQ_API int sq_sync_status(sq_cache *cache, void *stream);

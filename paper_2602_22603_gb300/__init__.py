@@ -32,6 +32,7 @@ SQ_ERR_UNSUPPORTED = -8
 SQ_ERR_NO_MEMORY = -9
 SQ_OUT_BF16 = 0
 SQ_OUT_F32 = 1
+SQ_DEBUG_DROP_DECODE_STAGE = 1
 
 
 class sq_config(ctypes.Structure):
@@ -94,6 +95,7 @@ _SIGS = {
     "sq_sync_status": (ctypes.c_int, [_P, _P]),
     "sq_strerror": (ctypes.c_char_p, [ctypes.c_int]),
     "sq_probe_read": (ctypes.c_int, [_P, _P, ctypes.c_size_t, _P]),
+    "sq_debug_set": (ctypes.c_int, [_P, _I32]),
     "sq_decode_attention_noalloc": (ctypes.c_int, [_P, _I32P, _I32, _I32, _P, _P, _I32,
                                                    ctypes.c_float, _P]),
 }
@@ -253,6 +255,10 @@ def sq_stats(cache: int) -> dict:
 
 def sq_probe_read(cache: int, buf, nbytes: int, stream=None) -> None:
     _check(lib().sq_probe_read(cache, _ptr(buf), nbytes, _stream(stream)), "sq_probe_read")
+
+
+def sq_debug_set(cache: int, flags: int) -> None:
+    _check(lib().sq_debug_set(cache, flags), "sq_debug_set")
 
 
 def sq_sync_status(cache: int, stream=None) -> int:

@@ -31,6 +31,7 @@ struct PlanEntry {
     std::vector<uint64_t> versions;
     DecodePlanLayout lay{};
     int64_t unique_tokens = 0, logical_tokens = 0;
+    int32_t first_busy_cta = 0;  // lowest CTA with work (target of the test hook)
     uint8_t* d_plan = nullptr;
     size_t plan_cap = 0;
     float* d_part = nullptr;
@@ -86,6 +87,7 @@ struct sq_cache {
     std::vector<void*> freed_on;
     std::vector<uint8_t> fenced;
     std::unordered_map<void*, cudaEvent_t> free_event;
+    int32_t debug_flags = 0;
     sq_stats_t stats;
 };
 
@@ -510,6 +512,10 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
         victim->lay = lay;
         victim->unique_tokens = plan.unique_tokens;
         victim->logical_tokens = plan.logical_tokens;
+        victim->first_busy_cta = 0;
+        while (victim->first_busy_cta + 1 < (int32_t)plan.cta_begin.size() &&
+               plan.cta_begin[victim->first_busy_cta + 1] == plan.cta_begin[victim->first_busy_cta])
+            ++victim->first_busy_cta;
         hit = victim;
     } else if (hit->ev_recorded) {
         e = cudaStreamWaitEvent(st, hit->ev, 0);
@@ -535,6 +541,8 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
     a.P = g.P;
     a.num_pages = g.num_pages;
     a.scale_log2 = sm_scale * 1.4426950408889634f;
+    a.debug_drop_cta = (c->debug_flags & SQ_DEBUG_DROP_DECODE_STAGE) ? hit->first_busy_cta : -1;
+    c->debug_flags &= ~SQ_DEBUG_DROP_DECODE_STAGE;
     a.err = c->d_err;
     e = launch_decode(c->tmap, a, L.n_ctas, g.D, st);
     if (e != cudaSuccess) { hit->valid = false; return cuda_status(e); }
@@ -702,6 +710,13 @@ int sq_probe_read(sq_cache* c, const void* buf, size_t bytes, void* stream) {
     return cuda_status(e);
 }
 
+int sq_debug_set(sq_cache* c, int32_t flags) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    if (flags & ~SQ_DEBUG_DROP_DECODE_STAGE) return SQ_ERR_INVALID_ARG;
+    c->debug_flags = flags;
+    return SQ_OK;
+}
+
 int sq_sync_status(sq_cache* c, void* stream) {
     if (!c) return SQ_ERR_BAD_HANDLE;
     cudaError_t e = cudaStreamSynchronize(as_stream(stream));
@@ -768,6 +783,11 @@ int sq_decode_attention_noalloc(sq_cache* c, const sq_seq* seqs, int32_t n_seqs,
     a.P = g.P;
     a.num_pages = g.num_pages;
     a.scale_log2 = sm_scale * 1.4426950408889634f;
+    int32_t busy = 0;
+    while (busy + 1 < (int32_t)plan.cta_begin.size() && plan.cta_begin[busy + 1] == plan.cta_begin[busy])
+        ++busy;
+    a.debug_drop_cta = (c->debug_flags & SQ_DEBUG_DROP_DECODE_STAGE) ? busy : -1;
+    c->debug_flags &= ~SQ_DEBUG_DROP_DECODE_STAGE;
     a.err = c->d_err;
     e = launch_decode(c->tmap, a, L.n_ctas, g.D, st);
     if (e != cudaSuccess) return cuda_status(e);

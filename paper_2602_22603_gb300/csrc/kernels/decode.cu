@@ -90,6 +90,15 @@ __device__ void produce(const CUtensorMap* tmap, const DecodeArgs& a, int it0, i
                 ok = false;
                 break;
             }
+            if ((int)blockIdx.x == a.debug_drop_cta && it == it0 && s == item.s0) {
+                // test hook: leave this stage unsignalled (the consumers'
+                // bounded wait runs out; nothing is in flight for it)
+                if (++slot == C::kStages) {
+                    slot = 0;
+                    phase ^= 1;
+                }
+                continue;
+            }
             const int tok0 = s * kStageTokens;
             const int pi0 = tok0 / P;
             const int row0 = P > kStageTokens ? (tok0 % P) : 0;

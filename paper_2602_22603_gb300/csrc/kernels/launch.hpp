@@ -21,6 +21,7 @@ struct DecodeArgs {
     float* part_ml;             // [n_items][16][2]  max (log2 units), sum
     int32_t layer, Hq, Hkv, G, P, num_pages;
     float scale_log2;           // sm_scale * log2(e)
+    int32_t debug_drop_cta;     // test hook: this CTA leaves its first stage unsignalled (-1: none)
     int* err;
 };
 
