@@ -295,3 +295,87 @@ def test_two_streams_main_and_aux():
     p.check_contents(m)
     assert p.cache.sync_status() == sq.SQ_OK
     p.close()
+
+
+@pytest.mark.parametrize("sm_scale", [1.0, 1.0 / math.sqrt(128)])
+def test_agent_shape_key_scaling_readings(sm_scale):
+    """Single-agent shape with keys N(0,1)/sqrt(128): the reading taken
+    (sm_scale 1, the 1/sqrt(d) folded into the keys) and the alternate one
+    (1/sqrt(d) applied again at decode) both match the oracle."""
+    p = Pair(2, 32, 8, 128, 64, num_pages=400, seed=31, k_scale=1 / math.sqrt(128))
+    keep = []
+    m = p.seq_new()
+    keep.append(p.append(m, 5000))
+    a = p.fork(m)
+    keep.append(p.append(a, 8))
+    for layer in range(2):
+        _decode_check(p, [m, a], layer, sm_scale, 40 + layer)
+    p.close()
+
+
+def test_short_agent_loop_trace():
+    """Algorithm 1 at a reduced size: 2 agents x 9 turns; every turn 6 main
+    decode steps then a tool response; every 4 turns an aux fork (trigger +
+    3 steps, decoded with the mains in one call); at the next turn release
+    it and evict whole tool responses older than 2 turns until >= 60% of
+    their tokens are covered.  Page tables, contents and attention outputs
+    are checked against the oracle along the way."""
+    rng = random.Random(77)
+    P = 16
+    p = Pair(2, 16, 4, 64, P, num_pages=3000, seed=77)
+    keep = []
+    mains = [p.seq_new() for _ in range(2)]
+    for m in mains:
+        keep.append(p.append(m, 40))            # the user query
+    responses = {m: [] for m in mains}          # (turn, start, end)
+    auxs = []
+    for t in range(9):
+        if auxs:
+            for x in auxs:
+                p.release(x)
+            auxs = []
+            for m in mains:
+                old = [r for r in responses[m] if r[0] < t - 2]
+                if not old:
+                    continue
+                rng.shuffle(old)
+                total = sum(e - s for _, s, e in old)
+                chosen, cov = [], 0
+                for r in old:
+                    if cov >= 0.6 * total:
+                        break
+                    chosen.append(r)
+                    cov += r[2] - r[1]
+                p.evict(m, [(s, e) for _, s, e in chosen])
+                gone = sorted((s, e) for _, s, e in chosen)
+                kept = []
+                for r in responses[m]:
+                    if r in chosen:
+                        continue
+                    sh = sum(e - s for s, e in gone if e <= r[1])
+                    kept.append((r[0], r[1] - sh, r[2] - sh))
+                responses[m] = kept
+            p.check_tables()
+            for m in mains:
+                p.check_contents(m)
+        if t % 4 == 0:
+            for m in mains:
+                a = p.fork(m)
+                keep.append(p.append(a, 8))
+                auxs.append(a)
+        for s_ in range(6):
+            seqs = mains + (auxs if s_ < 3 else [])
+            for h in seqs:
+                keep.append(p.append(h, 1))
+            if s_ in (0, 5):
+                _decode_check(p, seqs, s_ % 2, 0.125, 1000 * t + s_)
+        for m in mains:
+            n = p.cache.seq_info(m)[0]
+            ln = rng.choice([17, 60, 150, 333])
+            keep.append(p.append(m, ln))
+            responses[m].append((t, n, n + ln))
+    p.check_tables()
+    for h in mains + auxs:
+        p.check_contents(h)
+    assert p.cache.sync_status() == sq.SQ_OK
+    p.close()
