@@ -802,6 +802,24 @@ def run_trace(args, world, rank, local):
     return res
 
 
+def cpu_model() -> str:
+    import platform
+    try:
+        fields = {}
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if ":" in line:
+                    k, v = line.split(":", 1)
+                    fields.setdefault(k.strip().lower(), v.strip())
+        if "model name" in fields:
+            return fields["model name"]
+        if "cpu part" in fields:
+            return f"{platform.machine()} (CPU implementer {fields.get('cpu implementer', '?')}, part {fields['cpu part']})"
+    except OSError:
+        pass
+    return platform.machine()
+
+
 def _oracle_rows(host_bank, offs, n_chunks, chunk, L, Hkv, D, layer, which):
     """K (which = 0) or V (1) bits [n, Hkv, D] of one main sequence at one
     layer, rebuilt from its bank chunks."""
@@ -827,6 +845,7 @@ def cpu_baseline(args, bank, offs, n_chunks, chunk, scale):
     R = args.requests
     host_bank = bf16_bits(bank.data.cpu())
     layers = (0, L - 1) if L > 1 else (0,)
+    oatt_threads = oatt.num_threads()
     total = 0.0
     n_tok = 0
     for layer in layers:
@@ -843,8 +862,16 @@ def cpu_baseline(args, bank, offs, n_chunks, chunk, scale):
         oatt.decode_batch(q, ks, vs, scale)
         total += time.perf_counter() - t0
     per_layer = total / len(layers)
+    # the same oracle on one thread, over the first sequence only
+    oatt.set_threads(1)
+    t0 = time.perf_counter()
+    oatt.decode_batch(q[:1], ks[:1], vs[:1], scale)
+    t1 = time.perf_counter() - t0
+    oatt.set_threads(oatt_threads)
+    single = round(1 / (t1 * L), 5)
     return {"value": round(2 * R / (per_layer * L), 4), "unit": "tokens/s",
-            "cores": oatt.num_threads(), "kind": "oracle",
+            "cores": oatt_threads, "kind": "oracle", "cpu_model": cpu_model(),
+            "single_thread_value": single,
             "sample": f"one decode call of all {2 * R} sequences ({n_tok} tokens each, {Hq} heads) "
                       f"at {len(layers)} of {L} layers; tokens/s = sequences / "
                       f"(seconds per layer x {L} layers)",

@@ -141,6 +141,15 @@ int oracle_decode_batch_f64(int n_seqs, const int *ns, int Hq, int Hkv, int d,
     return status;
 }
 
+/* Sets the number of OpenMP threads (timing runs only; no effect on results). */
+void oracle_set_threads(int n) {
+#ifdef _OPENMP
+    if (n > 0) omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}
+
 /* Number of OpenMP threads the two entry points above run with. */
 int oracle_num_threads(void) {
     int n = 1;

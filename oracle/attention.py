@@ -53,6 +53,8 @@ def lib():
             L.oracle_decode_batch_f64.restype = ctypes.c_int
             L.oracle_num_threads.argtypes = []
             L.oracle_num_threads.restype = ctypes.c_int
+            L.oracle_set_threads.argtypes = [ctypes.c_int]
+            L.oracle_set_threads.restype = None
             _lib = L
     return _lib
 
@@ -64,6 +66,10 @@ def _u16(a: np.ndarray):
 
 def num_threads() -> int:
     return int(lib().oracle_num_threads())
+
+
+def set_threads(n: int) -> None:
+    lib().oracle_set_threads(int(n))
 
 
 def decode(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float,
