@@ -306,10 +306,15 @@ def run_sq(args, world, rank, local):
 
     set_seqs()
 
+    # new-token K/V of a step: [L][S][Hkv][D] slices of the bank (one batched append)
+    step_rows = bank.offsets(512, 2 * S * tok_elems, sub_seed(seed, 6))
+    step_i = [0]
+
     def step(ev=None):
-        for h in seqs:
-            k, v = kv_rows(1)
-            cache.append_kv(h, 1, k, v, st_h)
+        o = int(step_rows[step_i[0] % len(step_rows)])
+        step_i[0] += 1
+        sq.sq_append_kv_batch(cache.handle, seq_arr[0], bank_ptr + 2 * o,
+                              bank_ptr + 2 * (o + S * tok_elems), st_h)
         if ev is not None:
             ev.record(stream)
         arr = seq_arr[0]
@@ -402,7 +407,7 @@ def run_sq(args, world, rank, local):
                                "to this launch's algorithmic bytes") if ratio else None,
             "algorithmic_bytes_per_launch": int(uniq_per_call),
         },
-        "gpu_launches": int(K * (S + 2 * L)),
+        "gpu_launches": int(K * (1 + 2 * L)),
         "clocks": clock_rec,
     }
 
@@ -411,15 +416,14 @@ def run_sq(args, world, rank, local):
         q_h = q_all.cpu().pin_memory()
         out_h = torch.empty(out_all.shape, dtype=out_all.dtype).pin_memory()
         o_e2e = int(bank.offsets(1, S * 2 * tok_elems, sub_seed(seed, 5))[0])
-        kv_h = bank.view(o_e2e, (S, 2, L, 1, Hkv, D)).cpu().pin_memory()
-        kv_d = torch.empty(S, 2, L, 1, Hkv, D, dtype=torch.bfloat16, device="cuda")
+        kv_h = bank.view(o_e2e, (2, L, S, Hkv, D)).cpu().pin_memory()
+        kv_d = torch.empty(2, L, S, Hkv, D, dtype=torch.bfloat16, device="cuda")
         q_d = torch.empty_like(q_all)
 
         def e2e_step():
             q_d.copy_(q_h, non_blocking=True)
             kv_d.copy_(kv_h, non_blocking=True)
-            for i, h in enumerate(seqs):
-                cache.append_kv(h, 1, kv_d[i, 0], kv_d[i, 1])
+            sq.sq_append_kv_batch(cache.handle, seq_arr[0], kv_d[0], kv_d[1], st_h)
             for layer in range(L):
                 cache.decode_attention(seqs, layer, q_d[layer], out_all[layer], sq.SQ_OUT_BF16, scale)
             out_h.copy_(out_all, non_blocking=True)
@@ -736,11 +740,10 @@ def run_trace(args, world, rank, local):
         for s_ in range(256):
             seqs = mains + (auxs if (auxs and s_ < 128) else [])
             ea = _timed(st)
-            for h in seqs:
-                o = int(small[ctr["small"] % len(small)]); ctr["small"] += 1
-                cache.append_kv(h, 1, bp + 2 * o, bp + 2 * (o + 8 * tok), sh_)
-            eb = _timed(st)
             arr = (ctypes.c_int32 * len(seqs))(*seqs)
+            o = int(small[ctr["small"] % len(small)]); ctr["small"] += 1
+            sq.sq_append_kv_batch(cache.handle, arr, bp + 2 * o, bp + 2 * (o + 8 * tok), sh_)
+            eb = _timed(st)
             for layer in range(L):
                 sq.sq_decode_attention(cache.handle, arr, layer, qp[layer], op[layer],
                                        sq.SQ_OUT_BF16, scale, sh_)

@@ -124,6 +124,17 @@ SQ_API int sq_seq_new(sq_cache *cache, sq_seq *out);
 SQ_API int sq_append_kv(sq_cache *cache, sq_seq seq, int32_t n_tokens, const void *k,
                  const void *v, void *stream);
 
+/* Append one token to each of n_seqs sequences in one launch (a decode step
+ * of a batch; Algorithm 1: C <- C + R one generated token at a time).
+ *   seqs: host, n_seqs distinct live handles
+ *   k, v: device, bf16, contiguous [num_layers][n_seqs][num_kv_heads][head_dim]:
+ *         row i belongs to seqs[i]
+ * Same page rules as sq_append_kv, sequence by sequence in the order given;
+ * all or nothing: on any error no sequence changes.
+ * Errors: BAD_HANDLE, INVALID_ARG, NO_PAGES, CAPACITY, CUDA. */
+SQ_API int sq_append_kv_batch(sq_cache *cache, const sq_seq *seqs, int32_t n_seqs,
+                              const void *k, const void *v, void *stream);
+
 /* Fork an auxiliary sequence that shares the whole context of `parent`
  * (Sec. 3.1 step 1; Algorithm 1 phase 2, C_aux <- C + p; Sec. 3.4: the
  * auxiliary thread does not duplicate the KV cache).  The child gets the same

@@ -83,6 +83,7 @@ _SIGS = {
     "sq_seq_new": (ctypes.c_int, [_P, _I32P]),
     "sq_append_kv": (ctypes.c_int, [_P, _I32, _I32, _P, _P, _P]),
     "sq_fork_aux": (ctypes.c_int, [_P, _I32, _I32P]),
+    "sq_append_kv_batch": (ctypes.c_int, [_P, _I32P, _I32, _P, _P, _P]),
     "sq_decode_attention": (ctypes.c_int, [_P, _I32P, _I32, _I32, _P, _P, _I32, ctypes.c_float, _P]),
     "sq_evict_spans": (ctypes.c_int, [_P, _I32, ctypes.POINTER(sq_span), _I32, _P]),
     "sq_release": (ctypes.c_int, [_P, _I32, _P]),
@@ -178,6 +179,12 @@ def sq_seq_new(cache: int) -> int:
 def sq_append_kv(cache: int, seq: int, n_tokens: int, k, v, stream=None) -> None:
     _check(lib().sq_append_kv(cache, seq, n_tokens, _ptr(k), _ptr(v), _stream(stream)),
            "sq_append_kv")
+
+
+def sq_append_kv_batch(cache: int, seqs, k, v, stream=None) -> None:
+    arr = seqs if isinstance(seqs, ctypes.Array) else (ctypes.c_int32 * len(seqs))(*seqs)
+    _check(lib().sq_append_kv_batch(cache, arr, len(seqs), _ptr(k), _ptr(v), _stream(stream)),
+           "sq_append_kv_batch")
 
 
 def sq_fork_aux(cache: int, parent: int) -> int:
@@ -308,6 +315,7 @@ class Cache:
     seq_new = lambda self: sq_seq_new(self.handle)
     append_kv = lambda self, seq, n, k, v, stream=None: sq_append_kv(self.handle, seq, n, k, v, stream)
     fork_aux = lambda self, parent: sq_fork_aux(self.handle, parent)
+    append_kv_batch = lambda self, seqs, k, v, stream=None: sq_append_kv_batch(self.handle, seqs, k, v, stream)
     decode_attention = (lambda self, seqs, layer, q, out, out_dtype=SQ_OUT_BF16, sm_scale=1.0,
                         stream=None: sq_decode_attention(self.handle, seqs, layer, q, out,
                                                          out_dtype, sm_scale, stream))

@@ -431,6 +431,73 @@ int sq_append_kv(sq_cache* c, sq_seq seq, int32_t n_tokens, const void* k, const
     return SQ_OK;
 }
 
+int sq_append_kv_batch(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, const void* k,
+                       const void* v, void* stream) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    if (n_seqs < 0 || (n_seqs > 0 && !seqs)) return SQ_ERR_INVALID_ARG;
+    if (n_seqs == 0) return SQ_OK;
+    if (!k || !v || (reinterpret_cast<uintptr_t>(k) & 15) || (reinterpret_cast<uintptr_t>(v) & 15))
+        return SQ_ERR_INVALID_ARG;
+    for (int32_t i = 0; i < n_seqs; ++i) {
+        if (!c->host->seq(seqs[i])) return SQ_ERR_BAD_HANDLE;
+        for (int32_t j = 0; j < i; ++j)
+            if (seqs[j] == seqs[i]) return SQ_ERR_INVALID_ARG;
+    }
+    const Geometry& g = c->g;
+    std::vector<AppendPlan> plans(n_seqs);
+    auto undo = [&](int32_t upto, int code) {
+        for (int32_t j = upto - 1; j >= 0; --j) c->host->undo_append(seqs[j], plans[j]);
+        return code;
+    };
+    std::vector<int32_t> taken;
+    for (int32_t i = 0; i < n_seqs; ++i) {
+        int rc = c->host->append(seqs[i], 1, &plans[i]);
+        if (rc != SQ_OK) return undo(i, rc);
+        taken.insert(taken.end(), plans[i].taken.begin(), plans[i].taken.end());
+    }
+    cudaStream_t st = as_stream(stream);
+    int rc = fence_taken_pages(c, taken, stream);
+    if (rc != SQ_OK) return undo(n_seqs, rc);
+    for (int32_t i = 0; i < n_seqs; ++i) {
+        if (!plans[i].cow) continue;
+        CowArgs ca;
+        ca.pool = c->pool;
+        ca.num_pages = g.num_pages;
+        ca.L = g.L; ca.Hkv = g.Hkv; ca.P = g.P; ca.D = g.D;
+        ca.src_page = plans[i].cow_old;
+        ca.dst_page = plans[i].cow_new;
+        ca.rows = plans[i].cow_rows;
+        ca.err = c->d_err;
+        cudaError_t e = launch_cow_copy(ca, c->num_sms, st);
+        if (e != cudaSuccess) return undo(n_seqs, cuda_status(e));
+    }
+    for (int32_t b = 0; b < n_seqs; b += kAppendBatchMax) {
+        AppendBatchArgs a;
+        a.pool = c->pool;
+        a.k = reinterpret_cast<const __nv_bfloat16*>(k);
+        a.v = reinterpret_cast<const __nv_bfloat16*>(v);
+        a.num_pages = g.num_pages;
+        a.L = g.L; a.Hkv = g.Hkv; a.P = g.P; a.D = g.D;
+        a.n_total = n_seqs;
+        a.row0 = b;
+        a.n = std::min(kAppendBatchMax, n_seqs - b);
+        for (int32_t i = 0; i < a.n; ++i) {
+            const AppendPlan& pl = plans[b + i];
+            a.page[i] = pl.pages[0];                 // the page holding position n0
+            a.slot[i] = pl.n0 % g.P;
+        }
+        a.err = c->d_err;
+        cudaError_t e = launch_append_batch(a, c->num_sms, st);
+        if (e != cudaSuccess) return undo(n_seqs, cuda_status(e));
+    }
+    for (int32_t i = 0; i < n_seqs; ++i) {
+        c->host->seq_mut(seqs[i])->last_stream = stream;
+        if (plans[i].cow) c->stats.cow_pages += 1;
+    }
+    c->stats.appended_tokens += n_seqs;
+    return SQ_OK;
+}
+
 int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t layer,
                         const void* q, void* out, int32_t out_dtype, float sm_scale,
                         void* stream) {

@@ -42,6 +42,31 @@ __global__ void __launch_bounds__(256) sq_append_kv_kernel(const AppendArgs a) {
     }
 }
 
+// ---- one new token for each of a batch of sequences --------------------------
+__global__ void __launch_bounds__(256) sq_append_kv_batch_kernel(const AppendBatchArgs a) {
+    const int vpr = a.D / 8;
+    const int64_t total = (int64_t)a.L * a.n * 2 * a.Hkv * vpr;
+    for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+         idx += (int64_t)gridDim.x * blockDim.x) {
+        int64_t r = idx;
+        const int vc = (int)(r % vpr); r /= vpr;
+        const int head = (int)(r % a.Hkv); r /= a.Hkv;
+        const int kv = (int)(r % 2); r /= 2;
+        const int i = (int)(r % a.n);
+        const int layer = (int)(r / a.n);
+        const int page = a.page[i], slot = a.slot[i];
+        if ((uint64_t)page >= (uint64_t)a.num_pages || slot < 0 || slot >= a.P) {
+            set_error(a.err, kErrBounds);
+            continue;
+        }
+        const __nv_bfloat16* src = (kv ? a.v : a.k) +
+            (((int64_t)layer * a.n_total + a.row0 + i) * a.Hkv + head) * a.D + vc * 8;
+        __nv_bfloat16* dst = a.pool +
+            row_offset(a.num_pages, a.Hkv, a.P, a.D, layer, page, kv, head, slot) + vc * 8;
+        *reinterpret_cast<uint4*>(dst) = __ldg(reinterpret_cast<const uint4*>(src));
+    }
+}
+
 // ---- copy-on-write of the first `rows` rows of a page, every plane ----------
 __global__ void __launch_bounds__(256) sq_cow_copy_kernel(const CowArgs a) {
     const int vpr = a.D / 8;
@@ -179,6 +204,16 @@ cudaError_t launch_append(const AppendArgs& a, int num_sms, cudaStream_t st) {
     const int64_t cap = (int64_t)num_sms * 8;
     if (blocks > cap) blocks = cap;
     sq_append_kv_kernel<<<(unsigned)blocks, 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_append_batch(const AppendBatchArgs& a, int num_sms, cudaStream_t st) {
+    const int64_t total = (int64_t)a.L * a.n * 2 * a.Hkv * (a.D / 8);
+    if (total == 0) return cudaSuccess;
+    int64_t blocks = (total + 255) / 256;
+    const int64_t cap = (int64_t)num_sms * 8;
+    if (blocks > cap) blocks = cap;
+    sq_append_kv_batch_kernel<<<(unsigned)blocks, 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 

@@ -63,6 +63,23 @@ struct AppendArgs {
     int* err;
 };
 
+// One new token for each of up to kAppendBatchMax sequences.
+constexpr int kAppendBatchMax = 128;
+
+struct AppendBatchArgs {
+    __nv_bfloat16* pool;
+    const __nv_bfloat16* k;     // [L][n_total][Hkv][D]
+    const __nv_bfloat16* v;
+    int64_t num_pages;
+    int32_t L, Hkv, P, D;
+    int32_t n_total;            // rows in the caller's buffers (sequences of the call)
+    int32_t row0;               // first row this launch writes
+    int32_t n;                  // rows this launch writes
+    int32_t page[kAppendBatchMax];
+    int32_t slot[kAppendBatchMax];
+    int* err;
+};
+
 struct CowArgs {
     __nv_bfloat16* pool;
     int64_t num_pages;
@@ -83,6 +100,7 @@ struct EvictArgs {
 };
 
 cudaError_t launch_append(const AppendArgs& a, int num_sms, cudaStream_t st);
+cudaError_t launch_append_batch(const AppendBatchArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_cow_copy(const CowArgs& a, int num_sms, cudaStream_t st);
 constexpr int kEvictStages = 3;
 // Shared memory of one eviction CTA for a tile size.

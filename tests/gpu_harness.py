@@ -90,6 +90,19 @@ class Pair:
         self.cache.append_kv(h, n, kd, vd, stream)
         return kd, vd  # keep alive until the stream has run
 
+    def append_batch(self, hs, stream=None):
+        """One new token for each sequence of hs, in one library call."""
+        S = len(hs)
+        s = self._next_seed()
+        k = bf16_normal((self.L, S, self.Hkv, self.D), s, scale=self.k_scale)
+        v = bf16_normal((self.L, S, self.Hkv, self.D), s + 50000)
+        ids = [self.oracle.append(self.o[h], 1)[0] for h in hs]
+        assert ids == list(range(ids[0], ids[0] + S))
+        self.store.add(ids[0], bf16_bits(k), bf16_bits(v))
+        kd, vd = k.cuda(), v.cuda()
+        self.cache.append_kv_batch(list(hs), kd, vd, stream)
+        return kd, vd
+
     def evict(self, h: int, spans, stream=None):
         r = self.oracle.evict(self.o[h], spans)
         self.cache.evict_spans(h, spans, stream)

@@ -379,3 +379,34 @@ def test_short_agent_loop_trace():
         p.check_contents(h)
     assert p.cache.sync_status() == sq.SQ_OK
     p.close()
+
+
+def test_batched_single_token_append():
+    """sq_append_kv_batch = one sq_append_kv of one token per sequence, in the
+    order given: same page tables (including the copy-on-write of a shared
+    partial last page right after a fork), same contents."""
+    P = 16
+    p = Pair(2, 8, 2, 64, P, num_pages=400, seed=61)
+    keep = []
+    seqs = []
+    for n in (1, P - 1, P, 37):
+        h = p.seq_new()
+        keep.append(p.append(h, n))
+        seqs.append(h)
+    seqs.append(p.fork(seqs[3]))            # shares a partial last page
+    for step in range(2 * P + 3):
+        keep.append(p.append_batch(seqs))
+    p.check_tables()
+    for h in seqs:
+        p.check_contents(h)
+    _decode_check(p, seqs, 1, 0.125, 7)
+    # all or nothing: a bad handle in the batch changes nothing
+    before = [p.cache.page_table(h) for h in seqs]
+    with pytest.raises(sq.SqError) as e:
+        p.cache.append_kv_batch(seqs + [123456789], keep[-1][0], keep[-1][1])
+    assert e.value.code == sq.SQ_ERR_BAD_HANDLE
+    with pytest.raises(sq.SqError) as e:
+        p.cache.append_kv_batch([seqs[0], seqs[0]], keep[-1][0], keep[-1][1])
+    assert e.value.code == sq.SQ_ERR_INVALID_ARG
+    assert before == [p.cache.page_table(h) for h in seqs]
+    p.close()
