@@ -405,6 +405,10 @@ __global__ void __launch_bounds__(DecCfg<D>::kThreads, 2)
         fence_mbar_init();
     }
     __syncthreads();
+    // Launched as a programmatic dependent: the set-up above overlapped the
+    // previous kernel's tail; nothing it may have written is read before here.
+    grid_dependency_wait();
+    grid_launch_dependents();  // the combine may be scheduled as CTAs retire
     const int it0 = a.cta_begin[blockIdx.x], it1 = a.cta_begin[blockIdx.x + 1];
     if (warp == kDecodeConsumerWarps) {
         if (lane == 0) produce<D>(&tmap, a, it0, it1, smem, bars, abort_flag);
@@ -420,6 +424,9 @@ template <int D>
 __global__ void __launch_bounds__(256) sq_lse_combine_kernel(const CombineArgs a) {
     constexpr int V = D / 32;  // output elements per lane
     constexpr int U = 8;       // partials per batch of loads
+    // programmatic dependent of the decode kernel: wait for its partials
+    grid_dependency_wait();
+    grid_launch_dependents();
     const int wid = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
     if (wid >= a.n_seqs * a.Hq) return;
@@ -528,23 +535,45 @@ int decode_ctas_per_sm(int D) {
     return n;
 }
 
+// Both kernels are launched as programmatic dependents of whatever precedes
+// them on the stream: each waits (griddepcontrol.wait) before it reads
+// anything, so the launch latency overlaps the previous kernel's tail.
+static cudaLaunchAttribute pdl_attr() {
+    cudaLaunchAttribute at;
+    at.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at.val.programmaticStreamSerializationAllowed = 1;
+    return at;
+}
+
 cudaError_t launch_decode(const CUtensorMap& tmap, const DecodeArgs& a, int n_ctas, int D,
                           cudaStream_t st) {
-    if (D == 128)
-        sq_decode_splitk_kernel<128>
-            <<<n_ctas, DecCfg<128>::kThreads, DecCfg<128>::kSmemBytes, st>>>(tmap, a);
-    else
-        sq_decode_splitk_kernel<64>
-            <<<n_ctas, DecCfg<64>::kThreads, DecCfg<64>::kSmemBytes, st>>>(tmap, a);
-    return cudaGetLastError();
+    cudaLaunchAttribute at = pdl_attr();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(n_ctas);
+    cfg.stream = st;
+    cfg.attrs = &at;
+    cfg.numAttrs = 1;
+    if (D == 128) {
+        cfg.blockDim = dim3(DecCfg<128>::kThreads);
+        cfg.dynamicSmemBytes = DecCfg<128>::kSmemBytes;
+        return cudaLaunchKernelEx(&cfg, sq_decode_splitk_kernel<128>, tmap, a);
+    }
+    cfg.blockDim = dim3(DecCfg<64>::kThreads);
+    cfg.dynamicSmemBytes = DecCfg<64>::kSmemBytes;
+    return cudaLaunchKernelEx(&cfg, sq_decode_splitk_kernel<64>, tmap, a);
 }
 
 cudaError_t launch_combine(const CombineArgs& a, int D, cudaStream_t st) {
     const int warps = a.n_seqs * a.Hq;
-    const int blocks = (warps + 7) / 8;
-    if (D == 128) sq_lse_combine_kernel<128><<<blocks, 256, 0, st>>>(a);
-    else sq_lse_combine_kernel<64><<<blocks, 256, 0, st>>>(a);
-    return cudaGetLastError();
+    cudaLaunchAttribute at = pdl_attr();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((warps + 7) / 8);
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cfg.attrs = &at;
+    cfg.numAttrs = 1;
+    if (D == 128) return cudaLaunchKernelEx(&cfg, sq_lse_combine_kernel<128>, a);
+    return cudaLaunchKernelEx(&cfg, sq_lse_combine_kernel<64>, a);
 }
 
 }  // namespace sq
