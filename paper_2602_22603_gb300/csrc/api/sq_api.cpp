@@ -5,6 +5,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <algorithm>
 #include <cstring>
@@ -20,6 +21,13 @@
 using namespace sq;
 
 namespace {
+
+// An NVTX range around every C-ABI call, so that a timeline tool shows the
+// library's calls next to their kernels (no cost without an attached tool).
+struct TraceRange {
+    explicit TraceRange(const char* name) { nvtxRangePushA(name); }
+    ~TraceRange() { nvtxRangePop(); }
+};
 
 constexpr int kPlanCacheEntries = 8;
 constexpr int kUploadSlots = 8;
@@ -281,6 +289,7 @@ size_t sq_pool_bytes(const sq_config* cfg) {
 }
 
 int sq_cache_create(const sq_config* cfg, sq_cache** out) {
+    TraceRange trace_("sq_cache_create");
     if (!out) return SQ_ERR_INVALID_ARG;
     *out = nullptr;
     Geometry g;
@@ -367,6 +376,7 @@ int sq_seq_new(sq_cache* c, sq_seq* out) {
 }
 
 int sq_fork_aux(sq_cache* c, sq_seq parent, sq_seq* child_out) {
+    TraceRange trace_("sq_fork_aux");
     if (!c) return SQ_ERR_BAD_HANDLE;
     if (!child_out) return SQ_ERR_INVALID_ARG;
     return c->host->fork(parent, child_out);
@@ -374,6 +384,7 @@ int sq_fork_aux(sq_cache* c, sq_seq parent, sq_seq* child_out) {
 
 int sq_append_kv(sq_cache* c, sq_seq seq, int32_t n_tokens, const void* k, const void* v,
                  void* stream) {
+    TraceRange trace_("sq_append_kv");
     if (!c) return SQ_ERR_BAD_HANDLE;
     if (!c->host->seq(seq)) return SQ_ERR_BAD_HANDLE;
     if (n_tokens < 0) return SQ_ERR_INVALID_ARG;
@@ -433,6 +444,7 @@ int sq_append_kv(sq_cache* c, sq_seq seq, int32_t n_tokens, const void* k, const
 
 int sq_append_kv_batch(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, const void* k,
                        const void* v, void* stream) {
+    TraceRange trace_("sq_append_kv_batch");
     if (!c) return SQ_ERR_BAD_HANDLE;
     if (n_seqs < 0 || (n_seqs > 0 && !seqs)) return SQ_ERR_INVALID_ARG;
     if (n_seqs == 0) return SQ_OK;
@@ -501,6 +513,7 @@ int sq_append_kv_batch(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, const vo
 int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t layer,
                         const void* q, void* out, int32_t out_dtype, float sm_scale,
                         void* stream) {
+    TraceRange trace_("sq_decode_attention");
     if (!c) return SQ_ERR_BAD_HANDLE;
     const Geometry& g = c->g;
     if (!seqs || n_seqs < 1 || n_seqs > g.max_seqs || !q || !out) return SQ_ERR_INVALID_ARG;
@@ -638,6 +651,7 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
 }
 
 int sq_evict_spans(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_spans, void* stream) {
+    TraceRange trace_("sq_evict_spans");
     if (!c) return SQ_ERR_BAD_HANDLE;
     if (!c->host->seq(seq)) return SQ_ERR_BAD_HANDLE;
     if (n_spans < 0 || (n_spans > 0 && !spans)) return SQ_ERR_INVALID_ARG;
@@ -698,6 +712,7 @@ int sq_evict_spans(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_span
 }
 
 int sq_release(sq_cache* c, sq_seq seq, void* stream) {
+    TraceRange trace_("sq_release");
     if (!c) return SQ_ERR_BAD_HANDLE;
     const Seq* s = c->host->seq(seq);
     if (!s) return SQ_ERR_BAD_HANDLE;
@@ -803,6 +818,7 @@ int sq_sync_status(sq_cache* c, void* stream) {
 int sq_decode_attention_noalloc(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t layer,
                                 const void* q, void* out, int32_t out_dtype, float sm_scale,
                                 void* stream) {
+    TraceRange trace_("sq_decode_attention_noalloc");
     if (!c) return SQ_ERR_BAD_HANDLE;
     const Geometry& g = c->g;
     if (!seqs || n_seqs < 1 || n_seqs > g.max_seqs || !q || !out) return SQ_ERR_INVALID_ARG;

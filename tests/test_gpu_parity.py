@@ -79,7 +79,7 @@ def test_tiny_workload_full_parity():
 
 @pytest.mark.parametrize("P,G,D", [(16, 1, 64), (16, 4, 128), (64, 4, 128), (64, 8, 128),
                                    (64, 8, 64), (32, 16, 64), (128, 2, 128), (8, 4, 64),
-                                   (256, 4, 128)])
+                                   (256, 4, 128), (64, 3, 64), (16, 6, 128), (32, 5, 128)])
 def test_ragged_lengths(P, G, D):
     Hkv = 2
     p = Pair(2, G * Hkv, Hkv, D, P, num_pages=4000 // max(1, P // 16), seed=P * 31 + G * 7 + D)
@@ -409,4 +409,24 @@ def test_batched_single_token_append():
         p.cache.append_kv_batch([seqs[0], seqs[0]], keep[-1][0], keep[-1][1])
     assert e.value.code == sq.SQ_ERR_INVALID_ARG
     assert before == [p.cache.page_table(h) for h in seqs]
+    p.close()
+
+
+def test_many_sequences_in_one_call():
+    """64 sequences of mixed lengths (some sharing prefixes) in one decode
+    call: many segments, items and combine lists."""
+    rng = random.Random(5)
+    p = Pair(1, 32, 8, 128, 64, num_pages=4000, max_seqs=128, seed=55)
+    keep = []
+    seqs = []
+    for i in range(40):
+        h = p.seq_new()
+        keep.append(p.append(h, rng.choice([1, 63, 64, 65, 500, 3000])))
+        seqs.append(h)
+    for i in range(24):
+        a = p.fork(seqs[i])
+        keep.append(p.append(a, rng.choice([1, 7, 70])))
+        seqs.append(a)
+    rng.shuffle(seqs)
+    _decode_check(p, seqs, 0, 0.0884, 3)
     p.close()
