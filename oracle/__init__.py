@@ -11,7 +11,9 @@ Contents:
   cache_model  paged cache as an integer state machine (fork, append, evict,
                release; lowest-free-id allocation; copy-on-write rules).
   attention    decode attention in double precision over bf16 inputs
-               (plain C, oracle/attention.c), with optional token mask.
+               (plain C, oracle/attention.c), with optional token mask;
+               masked prefill attention (causal, span tokens removed:
+               Algorithm 2's BuildMask) built on the same per-query routine.
 
 Parity status: every function here is pinned by tests/test_oracle_pins.py
 against closed forms, invariants, brute force and library routines; nothing

@@ -141,6 +141,48 @@ int oracle_decode_batch_f64(int n_seqs, const int *ns, int Hq, int Hkv, int d,
     return status;
 }
 
+/*
+ * Masked prefill attention (Algorithm 2, BuildMask; Sec. 3.3: the auxiliary
+ * training traces see the context with the closed cursors' tokens masked
+ * out).  The last n_q tokens of a sequence of n tokens are the queries; query
+ * i sits at logical position p = n - n_q + i and attends to the tokens
+ * t = 0 .. p (causal) that are not removed (removed[t] != 0).  Per query and
+ * head this is exactly the decode above over the rows 0 .. p with the
+ * removal mask.  A query that sees no token gets a zero output and a log-sum-
+ * exp of -infinity (a reading: the paper never masks a whole prefix).
+ *   q:   [n_q][Hq][d] bf16 bits       k, v: [n][Hkv][d] bf16 bits
+ *   removed: [n] or NULL              out: [n_q][Hq][d] double
+ *   lse: [n_q][Hq] or NULL (natural log of sum_t exp(s_t))
+ * Returns 0, or -1 on an invalid shape.
+ */
+int oracle_prefill_f64(int n, int n_q, int Hq, int Hkv, int d, const uint16_t *q,
+                       const uint16_t *k, const uint16_t *v, double scale,
+                       const uint8_t *removed, double *out, double *lse) {
+    if (n <= 0 || n_q <= 0 || n_q > n || Hq <= 0 || Hkv <= 0 || d <= 0 ||
+        Hq % Hkv != 0)
+        return -1;
+    int G = Hq / Hkv;
+    int status = 0;
+    long total = (long)n_q * Hq;
+#pragma omp parallel for schedule(dynamic, 4) reduction(min : status)
+    for (long w = 0; w < total; ++w) {
+        int i = (int)(w / Hq), h = (int)(w % Hq);
+        int p = n - n_q + i;
+        double *o = out + ((size_t)i * Hq + h) * d;
+        double l_se = 0.0;
+        int rc = one_head(p + 1, Hkv, d, h / G, q + ((size_t)i * Hq + h) * d, k, v,
+                          scale, removed, o, NULL, &l_se);
+        if (rc == -1) {  /* every visible token removed */
+            for (int e = 0; e < d; ++e) o[e] = 0.0;
+            l_se = -INFINITY;
+            rc = 0;
+        }
+        if (lse) lse[(size_t)i * Hq + h] = l_se;
+        if (rc < status) status = rc;
+    }
+    return status;
+}
+
 /* Sets the number of OpenMP threads (timing runs only; no effect on results). */
 void oracle_set_threads(int n) {
 #ifdef _OPENMP

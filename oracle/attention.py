@@ -51,6 +51,11 @@ def lib():
                 ctypes.c_int, ctypes.c_int, u16p,
                 ctypes.POINTER(u16p), ctypes.POINTER(u16p), ctypes.c_double, f64p]
             L.oracle_decode_batch_f64.restype = ctypes.c_int
+            L.oracle_prefill_f64.argtypes = [
+                ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                u16p, u16p, u16p, ctypes.c_double,
+                ctypes.POINTER(ctypes.c_uint8), f64p, f64p]
+            L.oracle_prefill_f64.restype = ctypes.c_int
             L.oracle_num_threads.argtypes = []
             L.oracle_num_threads.restype = ctypes.c_int
             L.oracle_set_threads.argtypes = [ctypes.c_int]
@@ -132,3 +137,39 @@ def decode_batch(q: np.ndarray, ks: Sequence[np.ndarray], vs: Sequence[np.ndarra
     if rc != 0:
         raise ValueError(f"oracle_decode_batch_f64 rejected the input (rc={rc})")
     return out
+
+
+def removed_mask(n: int, spans: Sequence[Tuple[int, int]]) -> np.ndarray:
+    """uint8 [n]: 1 for tokens inside any half-open span (start, end)."""
+    m = np.zeros(n, dtype=np.uint8)
+    for a, b in spans:
+        m[int(a):int(b)] = 1
+    return m
+
+
+def prefill(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float,
+            spans: Sequence[Tuple[int, int]] = (), want_lse: bool = False):
+    """Masked prefill attention (Algorithm 2's BuildMask): the last n_q tokens
+    of the sequence query it causally with the spans' tokens removed.
+
+    q: uint16 bf16 bits [n_q, Hq, d]; k, v: uint16 [n, Hkv, d] in logical
+    order; spans: half-open (start, end) token ranges to remove.
+    Returns out float64 [n_q, Hq, d] (and lse [n_q, Hq], natural log, -inf
+    for a query that sees no token)."""
+    q = np.ascontiguousarray(q, dtype=np.uint16)
+    k = np.ascontiguousarray(k, dtype=np.uint16)
+    v = np.ascontiguousarray(v, dtype=np.uint16)
+    n_q, Hq, d = q.shape
+    n, Hkv, d2 = k.shape
+    assert d2 == d and v.shape == k.shape
+    m = removed_mask(n, spans)
+    out = np.zeros((n_q, Hq, d), dtype=np.float64)
+    lse = np.zeros((n_q, Hq), dtype=np.float64)
+    f64p = ctypes.POINTER(ctypes.c_double)
+    rc = lib().oracle_prefill_f64(n, n_q, Hq, Hkv, d, _u16(q), _u16(k), _u16(v),
+                                  float(scale),
+                                  m.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)),
+                                  out.ctypes.data_as(f64p), lse.ctypes.data_as(f64p))
+    if rc != 0:
+        raise ValueError(f"oracle_prefill_f64 rejected the input (rc={rc})")
+    return (out, lse) if want_lse else out

@@ -442,3 +442,123 @@ def test_forked_aux_attends_exactly_like_parent():
     mask[5:20] = 1
     o_m2 = oatt.decode(q, rows_k[c.tokens(m)], rows_v[c.tokens(m)], 0.17)
     assert np.array_equal(o_m2, oatt.decode(q, km, rows_v[ids], 0.17, mask=mask))
+
+
+# ---------------------------------------------------------------------------
+# masked prefill attention (Algorithm 2, BuildMask)
+# ---------------------------------------------------------------------------
+def prefill_reference_f64(q, k, v, scale, spans):
+    """Causal attention with the spans' tokens removed, written with torch
+    float64 ops: an explicit [n_q, n] mask and torch's SDPA (library routine),
+    and the log-sum-exp from torch.logsumexp over the masked logits."""
+    n_q, Hq, d = q.shape
+    n, Hkv, _ = k.shape
+    G = Hq // Hkv
+    pos = torch.arange(n - n_q, n).view(n_q, 1)
+    key = torch.arange(n).view(1, n)
+    allowed = key <= pos
+    for a, b in spans:
+        allowed[:, a:b] = False
+    qt = torch.from_numpy(widen(q)).permute(1, 0, 2)                               # [Hq, n_q, d]
+    kt = torch.from_numpy(widen(k)).permute(1, 0, 2).repeat_interleave(G, dim=0)  # [Hq, n, d]
+    vt = torch.from_numpy(widen(v)).permute(1, 0, 2).repeat_interleave(G, dim=0)
+    logits = scale * qt @ kt.transpose(1, 2)                                       # [Hq, n_q, n]
+    logits = logits.masked_fill(~allowed, -math.inf)
+    lse = torch.logsumexp(logits, dim=-1)                                          # [Hq, n_q]
+    rows = allowed.any(dim=1)
+    am = torch.zeros(n_q, n, dtype=torch.float64).masked_fill(~allowed, -math.inf)
+    am[~rows] = 0.0  # keep SDPA finite on rows with nothing to see; zeroed below
+    o = torch.nn.functional.scaled_dot_product_attention(
+        qt.unsqueeze(0), kt.unsqueeze(0), vt.unsqueeze(0), attn_mask=am, scale=scale)[0]
+    o[:, ~rows] = 0.0
+    return o.permute(1, 0, 2).numpy(), lse.permute(1, 0).numpy()
+
+
+def rand_prefill(seed, n, n_q, Hq, Hkv, d):
+    q = bf16_bits(bf16_normal((n_q, Hq, d), seed))
+    k = bf16_bits(bf16_normal((n, Hkv, d), seed + 1))
+    v = bf16_bits(bf16_normal((n, Hkv, d), seed + 2))
+    return q, k, v
+
+
+@pytest.mark.parametrize("n,n_q,Hq,Hkv,d,spans", [
+    (1, 1, 4, 4, 16, []),                              # one token, G = 1
+    (40, 40, 4, 4, 32, []),                            # textbook causal MHA
+    (40, 40, 8, 2, 32, [(5, 9), (20, 33)]),            # GQA, full prefill
+    (97, 13, 16, 4, 64, [(60, 90), (2, 3), (95, 97)]),  # queries at the tail
+    (64, 64, 6, 2, 16, [(0, 10)]),                     # a masked prefix: empty rows
+    (150, 7, 12, 4, 64, [(143, 146)]),                 # spans among the queries
+])
+def test_prefill_matches_masked_causal_sdpa(n, n_q, Hq, Hkv, d, spans):
+    q, k, v = rand_prefill(n * 7 + n_q, n, n_q, Hq, Hkv, d)
+    out, lse = oatt.prefill(q, k, v, 0.21, spans, want_lse=True)
+    ref, ref_lse = prefill_reference_f64(q, k, v, 0.21, spans)
+    np.testing.assert_allclose(out, ref, rtol=1e-10, atol=1e-12)
+    fin = np.isfinite(ref_lse)
+    assert np.array_equal(np.isfinite(lse), fin)
+    np.testing.assert_allclose(lse[fin], ref_lse[fin], rtol=1e-12, atol=1e-12)
+
+
+def test_prefill_causal_reach_is_exact():
+    # Changing token t's K/V changes exactly the queries at positions >= t,
+    # and none when t lies in a masked span.
+    n, n_q, Hq, Hkv, d = 30, 30, 4, 2, 16
+    q, k, v = rand_prefill(5, n, n_q, Hq, Hkv, d)
+    spans = [(11, 14)]
+    base = oatt.prefill(q, k, v, 0.3, spans)
+    for t in (0, 7, 12, 29):
+        k2, v2 = k.copy(), v.copy()
+        k2[t] = bf16_bits(bf16_normal((Hkv, d), 90 + t))
+        v2[t] = bf16_bits(bf16_normal((Hkv, d), 190 + t))
+        out = oatt.prefill(q, k2, v2, 0.3, spans)
+        changed = [i for i in range(n_q) if not np.array_equal(out[i], base[i])]
+        expect = [] if 11 <= t < 14 else list(range(t, n))
+        assert changed == expect, t
+
+
+def test_prefill_single_visible_key_and_empty_rows():
+    # spans [1, n): every query sees token 0 only -> output = V[0] of its
+    # group exactly, lse = its logit; spans [0, n): nothing -> zeros, -inf.
+    n, Hq, Hkv, d = 20, 8, 2, 16
+    q, k, v = rand_prefill(11, n, n, Hq, Hkv, d)
+    out, lse = oatt.prefill(q, k, v, 0.5, [(1, n)], want_lse=True)
+    vw, kw, qw = widen(v), widen(k), widen(q)
+    for h in range(Hq):
+        g = h // (Hq // Hkv)
+        assert np.array_equal(out[:, h], np.broadcast_to(vw[0, g], (n, d)))
+        np.testing.assert_allclose(lse[:, h], 0.5 * qw[:, h] @ kw[0, g], rtol=1e-13)
+    out, lse = oatt.prefill(q, k, v, 0.5, [(0, n)], want_lse=True)
+    assert not out.any() and np.all(lse == -np.inf)
+
+
+def test_prefill_last_row_equals_decode_after_eviction():
+    # Algorithm 2 masks the closed cursors' tokens while training; Algorithm 1
+    # evicts them at inference.  The last query of a masked prefill must equal
+    # decode over the evicted cache, up to the order of the sums.
+    Hq, Hkv, d, P = 8, 2, 32, 4
+    c = ocm.OracleCache(num_pages=64, page_size=P)
+    m = c.seq_new()
+    ids = c.append(m, 90)
+    k = bf16_bits(bf16_normal((90, Hkv, d), 21))
+    v = bf16_bits(bf16_normal((90, Hkv, d), 22))
+    q = bf16_bits(bf16_normal((1, Hq, d), 23))
+    spans = [(30, 41), (4, 9), (60, 88)]
+    pre = oatt.prefill(q, k[ids], v[ids], 0.2, spans)
+    c.evict(m, spans)
+    kept = c.tokens(m)
+    dec = oatt.decode(q[0], k[kept], v[kept], 0.2)
+    np.testing.assert_allclose(pre[0], dec, rtol=1e-12, atol=1e-13)
+
+
+def test_prefill_constant_values():
+    n, Hq, Hkv, d = 50, 4, 1, 8
+    q, k, _ = rand_prefill(3, n, 25, Hq, Hkv, d)
+    v = np.full((n, Hkv, d), bf16_bits(torch.tensor([0.375], dtype=torch.bfloat16))[0], dtype=np.uint16)
+    out = oatt.prefill(q, k, v, 0.4, [(26, 31)])
+    np.testing.assert_allclose(out, 0.375, rtol=1e-14)
+
+
+def test_prefill_rejects_bad_shapes():
+    q, k, v = rand_prefill(1, 10, 11, 4, 2, 8)
+    with pytest.raises(ValueError):
+        oatt.prefill(q, k, v, 1.0)
