@@ -173,6 +173,35 @@ SQ_API int sq_decode_attention(sq_cache *cache, const sq_seq *seqs, int32_t n_se
 SQ_API int sq_evict_spans(sq_cache *cache, sq_seq seq, const sq_span *spans,
                    int32_t n_spans, void *stream);
 
+/* Masked prefill attention (Algorithm 2, BuildMask; Sec. 3.3): the
+ * training-time counterpart of span eviction.  The last n_q tokens of `seq`
+ * (already appended) are the queries; query i sits at logical position
+ * p = n - n_q + i and attends causally to the sequence's tokens 0 .. p,
+ * except the tokens inside `spans`, which no query sees (a closed cursor's
+ * tokens masked out for the whole trace).  With GQA, query head h reads KV
+ * head floor(h / G):
+ *     o[i][h] = sum_j softmax_j(sm_scale * q[i][h] . K[j]) V[j]   over visible j
+ *   q:   device bf16 [n_q][Hq][head_dim], 16-byte aligned, caller-owned;
+ *        row i is the query of position n - n_q + i (post-RoPE, like K);
+ *   out: device [n_q][Hq][head_dim], SQ_OUT_BF16 (round to nearest even) or
+ *        SQ_OUT_F32, 16-byte aligned;
+ *   lse: NULL, or device float [n_q][Hq], 4-byte aligned: the natural log of
+ *        sum_j exp(sm_scale * q . K[j]) over the visible keys (for a backward
+ *        pass or for merging with other key ranges);
+ *   sm_scale: finite, >= 0;
+ *   spans: host, n_spans half-open spans of current positions, any order;
+ *          empty, overlapping or out-of-range spans are INVALID_ARG;
+ *          n_spans == 0 is plain causal attention.
+ * A query that sees no token (every key up to it masked) gets a zero output
+ * and lse = -infinity.  The sequence and the cache are not modified.  The
+ * kernel runs on the tensor cores (bf16 products, fp32 accumulation; the
+ * softmax weights are rounded to bf16 before the value product).
+ * Errors: BAD_HANDLE, INVALID_ARG, NO_MEMORY, CUDA. */
+SQ_API int sq_prefill_attention(sq_cache *cache, sq_seq seq, int32_t layer, int32_t n_q,
+                                const void *q, void *out, int32_t out_dtype, float *lse,
+                                float sm_scale, const sq_span *spans, int32_t n_spans,
+                                void *stream);
+
 /* Release a sequence (Algorithm 1: S_thread <- None; Sec. 3.4: the
  * auxiliary thread's own tokens are discarded).  Every page loses one
  * reference; pages that reach zero become free once all work enqueued on
@@ -215,6 +244,9 @@ typedef struct {
     int64_t evict_bytes;         /* algorithmic bytes read + written by compaction */
     int64_t appended_tokens;
     int64_t cow_pages;           /* pages copied on write (append + evict) */
+    int64_t prefill_calls;
+    int64_t prefill_pairs;       /* visible (query, key) pairs per query head,
+                                    summed over prefill calls */
 } sq_stats_t;
 
 SQ_API int sq_stats(sq_cache *cache, sq_stats_t *out);

@@ -58,7 +58,7 @@ class sq_stats_t(ctypes.Structure):
     _fields_ = [(name, ctypes.c_int64) for name in (
         "live_pages", "peak_live_pages", "decode_calls", "decode_logical_bytes",
         "decode_unique_bytes", "evict_calls", "evicted_tokens", "evict_moved_rows",
-        "evict_bytes", "appended_tokens", "cow_pages")]
+        "evict_bytes", "appended_tokens", "cow_pages", "prefill_calls", "prefill_pairs")]
 
     def as_dict(self):
         return {name: int(getattr(self, name)) for name, _ in self._fields_}
@@ -86,6 +86,8 @@ _SIGS = {
     "sq_append_kv_batch": (ctypes.c_int, [_P, _I32P, _I32, _P, _P, _P]),
     "sq_decode_attention": (ctypes.c_int, [_P, _I32P, _I32, _I32, _P, _P, _I32, ctypes.c_float, _P]),
     "sq_evict_spans": (ctypes.c_int, [_P, _I32, ctypes.POINTER(sq_span), _I32, _P]),
+    "sq_prefill_attention": (ctypes.c_int, [_P, _I32, _I32, _I32, _P, _P, _I32, _P, ctypes.c_float,
+                                            ctypes.POINTER(sq_span), _I32, _P]),
     "sq_release": (ctypes.c_int, [_P, _I32, _P]),
     "sq_seq_info": (ctypes.c_int, [_P, _I32, _I32P, _I32P]),
     "sq_get_page_table": (ctypes.c_int, [_P, _I32, _I32P, _I32, _I32P]),
@@ -218,6 +220,16 @@ def sq_evict_spans(cache: int, seq: int, spans: Sequence[Tuple[int, int]], strea
     _check(lib().sq_evict_spans(cache, seq, arr, len(spans), _stream(stream)), "sq_evict_spans")
 
 
+def sq_prefill_attention(cache: int, seq: int, layer: int, n_q: int, q, out,
+                         out_dtype: int = SQ_OUT_BF16, lse=None, sm_scale: float = 1.0,
+                         spans: Sequence[Tuple[int, int]] = (), stream=None) -> None:
+    arr = (sq_span * max(1, len(spans)))(*[sq_span(int(a), int(b)) for a, b in spans])
+    _check(lib().sq_prefill_attention(cache, seq, layer, n_q, _ptr(q), _ptr(out), out_dtype,
+                                      _ptr(lse), float(sm_scale), arr, len(spans),
+                                      _stream(stream)),
+           "sq_prefill_attention")
+
+
 def sq_release(cache: int, seq: int, stream=None) -> None:
     _check(lib().sq_release(cache, seq, _stream(stream)), "sq_release")
 
@@ -320,6 +332,10 @@ class Cache:
                         stream=None: sq_decode_attention(self.handle, seqs, layer, q, out,
                                                          out_dtype, sm_scale, stream))
     evict_spans = lambda self, seq, spans, stream=None: sq_evict_spans(self.handle, seq, spans, stream)
+    prefill_attention = (lambda self, seq, layer, n_q, q, out, out_dtype=SQ_OUT_BF16, lse=None,
+                         sm_scale=1.0, spans=(), stream=None:
+                         sq_prefill_attention(self.handle, seq, layer, n_q, q, out, out_dtype, lse,
+                                              sm_scale, spans, stream))
     release = lambda self, seq, stream=None: sq_release(self.handle, seq, stream)
     seq_info = lambda self, seq: sq_seq_info(self.handle, seq)
     page_table = lambda self, seq: sq_get_page_table(self.handle, seq)

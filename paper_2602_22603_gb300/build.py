@@ -26,6 +26,7 @@ LIBSQ_SOURCES = [
     "kernels/decode.cu",
     "kernels/kv.cu",
     "kernels/noalloc_scratch.cu",
+    "kernels/prefill.cu",
     "kernels/probe.cu",
     "host/core.cpp",
     "api/sq_api.cpp",

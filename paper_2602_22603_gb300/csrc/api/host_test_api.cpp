@@ -124,4 +124,39 @@ int sqh_plan_decode(void* c, const int32_t* handles, int32_t n, int32_t n_ctas,
     return kOk;
 }
 
+// Plans a masked prefill over a sequence of n tokens (G = Hq / Hkv; spans as
+// start, end pairs).  info_out receives 6 int64 values: n_tiles, BP, n_qt,
+// n_split, visible_pairs, sizeof(PrefillTile).  If tiles_out is non-NULL,
+// up to `cap` tiles are written as 6 int32 each: key0, flags, vis[4].
+int sqh_plan_prefill(int32_t Hq, int32_t Hkv, int32_t n, int32_t n_q, const int32_t* spans,
+                     int32_t n_spans, int32_t target_ctas, int64_t* info_out, int32_t* tiles_out,
+                     int32_t cap) {
+    Geometry g;
+    g.L = 1; g.Hq = Hq; g.Hkv = Hkv; g.D = 128; g.P = 64;
+    g.num_pages = 1; g.max_seqs = 1; g.max_pages_per_seq = 1;
+    if (Hkv < 1 || Hq % Hkv != 0) return kInvalidArg;
+    std::vector<int32_t> a(n_spans > 0 ? n_spans : 0), b(a.size());
+    for (int32_t i = 0; i < n_spans; ++i) {
+        a[i] = spans[2 * i];
+        b[i] = spans[2 * i + 1];
+    }
+    PrefillPlanHost p;
+    int rc = plan_prefill(g, n, n_q, a.data(), b.data(), n_spans, target_ctas, &p);
+    if (rc != kOk) return rc;
+    int64_t v[6] = {(int64_t)p.tiles.size(), p.BP, p.n_qt, p.n_split, p.visible_pairs,
+                    (int64_t)sizeof(PrefillTile)};
+    std::memcpy(info_out, v, sizeof v);
+    if (tiles_out) {
+        const int32_t m = std::min<int32_t>(cap, (int32_t)p.tiles.size());
+        for (int32_t i = 0; i < m; ++i) {
+            const PrefillTile& t = p.tiles[i];
+            int32_t* o = tiles_out + 6 * i;
+            o[0] = t.key0;
+            o[1] = t.flags;
+            for (int w = 0; w < 4; ++w) o[2 + w] = (int32_t)t.vis[w];
+        }
+    }
+    return kOk;
+}
+
 }  // extern "C"

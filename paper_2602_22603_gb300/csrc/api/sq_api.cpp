@@ -81,7 +81,13 @@ struct sq_cache {
     bool own_pool = false;
     size_t pool_bytes = 0;
     CUtensorMap tmap;
+    void* encode_fn = nullptr;  // cuTensorMapEncodeTiled
     int* d_err = nullptr;
+    // prefill split-K partials, reused by every call (grown on demand)
+    float* pre_part = nullptr;
+    size_t pre_part_cap = 0;
+    cudaEvent_t pre_ev = nullptr;
+    bool pre_ev_recorded = false;
     PlanEntry plans[kPlanCacheEntries];
     uint64_t use_clock = 0;
     UploadSlot slots[kUploadSlots];
@@ -133,6 +139,7 @@ int make_tensor_map(sq_cache* c) {
                                          &q) != cudaSuccess ||
         q != cudaDriverEntryPointSuccess || !fn)
         return SQ_ERR_CUDA;
+    c->encode_fn = fn;
     auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     const Geometry& g = c->g;
     // dims, innermost first: head dim, row within a (layer, page) block
@@ -314,6 +321,8 @@ int sq_cache_create(const sq_config* cfg, sq_cache** out) {
     c->decode_ctas = cfg->decode_ctas > 0 ? cfg->decode_ctas : c->num_sms * decode_ctas_per_sm(g.D);
     e = evict_prepare();
     if (e != cudaSuccess) return cuda_status(e);
+    e = prefill_prepare(g.D);
+    if (e != cudaSuccess) return cuda_status(e);
     c->evict_tile_rows = choose_tile_rows(c.get());
     c->pool_bytes = pool_bytes_of(g);
     if (cfg->kv_pool) {
@@ -363,6 +372,8 @@ int sq_cache_destroy(sq_cache* c) {
         if (p.ev) cudaEventDestroy(p.ev);
     }
     for (auto& kv : c->free_event) cudaEventDestroy(kv.second);
+    if (c->pre_part) cudaFree(c->pre_part);
+    if (c->pre_ev) cudaEventDestroy(c->pre_ev);
     if (c->d_err) cudaFree(c->d_err);
     if (c->own_pool) cudaFree(c->pool);
     delete c;
@@ -708,6 +719,132 @@ int sq_evict_spans(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_span
     c->stats.evict_moved_rows += plan.moved_rows;
     c->stats.evict_bytes += 2 * plan.moved_rows * g.L * g.token_layer_bytes();
     c->stats.cow_pages += (int64_t)plan.cow_pages.size();
+    return SQ_OK;
+}
+
+int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, const void* q,
+                         void* out, int32_t out_dtype, float* lse, float sm_scale,
+                         const sq_span* spans, int32_t n_spans, void* stream) {
+    TraceRange trace_("sq_prefill_attention");
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    const Seq* s = c->host->seq(seq);
+    if (!s) return SQ_ERR_BAD_HANDLE;
+    const Geometry& g = c->g;
+    if (layer < 0 || layer >= g.L || n_q < 1 || n_q > s->n || !q || !out)
+        return SQ_ERR_INVALID_ARG;
+    if (out_dtype != SQ_OUT_BF16 && out_dtype != SQ_OUT_F32) return SQ_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(q) & 15) || (reinterpret_cast<uintptr_t>(out) & 15) ||
+        (reinterpret_cast<uintptr_t>(lse) & 3))
+        return SQ_ERR_INVALID_ARG;
+    if (!(sm_scale >= 0.f) || sm_scale > 3.0e38f) return SQ_ERR_INVALID_ARG;
+    if (n_spans < 0 || (n_spans > 0 && !spans)) return SQ_ERR_INVALID_ARG;
+    std::vector<int32_t> sa(n_spans), sb(n_spans);
+    for (int32_t i = 0; i < n_spans; ++i) {
+        sa[i] = spans[i].start;
+        sb[i] = spans[i].end;
+    }
+    PrefillPlanHost plan;
+    int rc = plan_prefill(g, s->n, n_q, sa.data(), sb.data(), n_spans, c->num_sms, &plan);
+    if (rc != SQ_OK) return rc;
+    cudaStream_t st = as_stream(stream);
+    cudaError_t e;
+    // upload: key tiles, then the page table
+    const size_t tb = plan.tiles.size() * sizeof(PrefillTile);
+    const size_t pb = s->pages.size() * sizeof(int32_t);
+    if (c->staging.size() < tb + pb) c->staging.resize(tb + pb);
+    if (tb) std::memcpy(c->staging.data(), plan.tiles.data(), tb);
+    std::memcpy(c->staging.data() + tb, s->pages.data(), pb);
+    UploadSlot& slot = c->slots[c->next_slot];
+    c->next_slot = (c->next_slot + 1) % kUploadSlots;
+    rc = upload(c, slot, c->staging.data(), tb + pb, stream);
+    if (rc != SQ_OK) return rc;
+    const int64_t grid = (int64_t)plan.n_qt * g.Hkv * plan.n_split;
+    if (plan.n_split > 1) {
+        const size_t need = (size_t)grid * kPrefillRows * (g.D + 1) * sizeof(float);
+        if (!c->pre_ev) {
+            e = cudaEventCreateWithFlags(&c->pre_ev, cudaEventDisableTiming);
+            if (e != cudaSuccess) return cuda_status(e);
+        }
+        if (need > c->pre_part_cap) {
+            if (c->pre_ev_recorded) cudaEventSynchronize(c->pre_ev);
+            if (c->pre_part) cudaFree(c->pre_part);
+            c->pre_part = nullptr;
+            c->pre_part_cap = 0;
+            e = cudaMalloc(&c->pre_part, need * 5 / 4);
+            if (e != cudaSuccess) return cuda_status(e);
+            c->pre_part_cap = need * 5 / 4;
+            c->pre_ev_recorded = false;
+        }
+        if (c->pre_ev_recorded) {
+            e = cudaStreamWaitEvent(st, c->pre_ev, 0);
+            if (e != cudaSuccess) return cuda_status(e);
+        }
+    }
+    // queries: {D, Hq, n_q}, one box = the G heads of a KV head x BP positions
+    CUtensorMap qmap;
+    {
+        auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(c->encode_fn);
+        cuuint64_t dims[3] = {(cuuint64_t)g.D, (cuuint64_t)g.Hq, (cuuint64_t)n_q};
+        cuuint64_t strides[2] = {(cuuint64_t)g.D * 2, (cuuint64_t)g.Hq * g.D * 2};
+        cuuint32_t box[3] = {64, (cuuint32_t)g.G(), (cuuint32_t)plan.BP};
+        cuuint32_t estr[3] = {1, 1, 1};
+        CUresult r = encode(&qmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), dims,
+                            strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) return SQ_ERR_INVALID_ARG;
+    }
+    PrefillArgs a;
+    a.tiles = reinterpret_cast<const PrefillTile*>(slot.d);
+    a.page_ids = reinterpret_cast<const int32_t*>(slot.d + tb);
+    a.n_tiles = (int32_t)plan.tiles.size();
+    a.n_pages_seq = (int32_t)s->pages.size();
+    a.n = s->n;
+    a.n_q = n_q;
+    a.layer = layer;
+    a.Hq = g.Hq;
+    a.Hkv = g.Hkv;
+    a.G = g.G();
+    a.P = g.P;
+    a.num_pages = g.num_pages;
+    a.BP = plan.BP;
+    a.n_qt = plan.n_qt;
+    a.n_split = plan.n_split;
+    a.scale_log2 = sm_scale * 1.4426950408889634f;
+    a.out = out;
+    a.out_f32 = out_dtype == SQ_OUT_F32;
+    a.lse = lse;
+    a.part_o = c->pre_part;
+    a.part_ml = c->pre_part ? c->pre_part + (size_t)grid * kPrefillRows * g.D : nullptr;
+    a.err = c->d_err;
+    e = launch_prefill(c->tmap, qmap, a, g.D, st);
+    if (e != cudaSuccess) return cuda_status(e);
+    if (plan.n_split > 1) {
+        PrefillCombineArgs ca;
+        ca.part_o = a.part_o;
+        ca.part_ml = a.part_ml;
+        ca.out = out;
+        ca.out_f32 = a.out_f32;
+        ca.lse = lse;
+        ca.n_q = n_q;
+        ca.Hq = g.Hq;
+        ca.Hkv = g.Hkv;
+        ca.G = g.G();
+        ca.BP = plan.BP;
+        ca.n_qt = plan.n_qt;
+        ca.n_split = plan.n_split;
+        e = launch_prefill_combine(ca, g.D, st);
+        if (e != cudaSuccess) return cuda_status(e);
+        e = cudaEventRecord(c->pre_ev, st);
+        if (e != cudaSuccess) return cuda_status(e);
+        c->pre_ev_recorded = true;
+    }
+    e = cudaEventRecord(slot.ev, st);
+    if (e != cudaSuccess) return cuda_status(e);
+    slot.ev_recorded = true;
+    c->host->seq_mut(seq)->last_stream = stream;
+    c->stats.prefill_calls += 1;
+    c->stats.prefill_pairs += plan.visible_pairs;
     return SQ_OK;
 }
 

@@ -23,6 +23,27 @@ int check_geometry(const Geometry& g) {
     return kOk;
 }
 
+int sorted_spans(int32_t n, const int32_t* starts, const int32_t* ends, int32_t n_spans,
+                 std::vector<std::pair<int32_t, int32_t>>* out) {
+    out->clear();
+    if (n_spans < 0) return kInvalidArg;
+    if (n_spans == 0) return kOk;
+    if (!starts || !ends) return kInvalidArg;
+    auto& sp = *out;
+    sp.resize(n_spans);
+    for (int32_t i = 0; i < n_spans; ++i) sp[i] = {starts[i], ends[i]};
+    std::sort(sp.begin(), sp.end());
+    int32_t prev_end = 0;
+    for (auto& ab : sp) {
+        if (ab.first < 0 || ab.second > n || ab.first >= ab.second || ab.first < prev_end) {
+            out->clear();
+            return kInvalidArg;
+        }
+        prev_end = ab.second;
+    }
+    return kOk;
+}
+
 // ---------------------------------------------------------------------------
 PageAllocator::PageAllocator(int32_t n)
     : ref_(n, 0), free_bits_((n + 63) / 64, 0), free_count_(n) {
@@ -189,17 +210,11 @@ int HostCache::evict(int32_t h, const int32_t* starts, const int32_t* ends,
     if (n_spans == 0) return kOk;
     if (!starts || !ends) return kInvalidArg;
 
-    std::vector<std::pair<int32_t, int32_t>> sp(n_spans);
-    for (int32_t i = 0; i < n_spans; ++i) sp[i] = {starts[i], ends[i]};
-    std::sort(sp.begin(), sp.end());
-    int32_t prev_end = 0;
+    std::vector<std::pair<int32_t, int32_t>> sp;
+    int rc = sorted_spans(n, starts, ends, n_spans, &sp);
+    if (rc != kOk) return rc;
     int64_t removed = 0;
-    for (auto& ab : sp) {
-        if (ab.first < 0 || ab.second > n || ab.first >= ab.second) return kInvalidArg;
-        if (ab.first < prev_end) return kInvalidArg;
-        prev_end = ab.second;
-        removed += ab.second - ab.first;
-    }
+    for (auto& ab : sp) removed += ab.second - ab.first;
     // kept runs
     int32_t cur = 0, dst = 0;
     for (auto& ab : sp) {
@@ -530,6 +545,66 @@ void plan_serialize(const DecodePlanHost& p, const DecodePlanLayout& L, uint8_t*
     std::memcpy(dst + L.page_ids, p.page_ids.data(), sizeof(int32_t) * L.n_page_ids);
     std::memcpy(dst + L.comb_off, p.comb_off.data(), sizeof(int32_t) * (L.n_comb_keys + 1));
     std::memcpy(dst + L.comb_ent, p.comb_ent.data(), sizeof(CombineEnt) * L.n_comb_ent);
+}
+
+// ---------------------------------------------------------------------------
+// Masked prefill planning.  Visibility of key j to the query at position p:
+// j <= p (causal) and j in no span (Algorithm 2: a closed cursor's tokens are
+// masked for every later token).  The kernel applies the causal part; the
+// plan carries the span part as one bit per key, per key tile.
+int plan_prefill(const Geometry& g, int32_t n, int32_t n_q, const int32_t* starts,
+                 const int32_t* ends, int32_t n_spans, int32_t target_ctas,
+                 PrefillPlanHost* out) {
+    *out = PrefillPlanHost();
+    if (n < 1 || n_q < 1 || n_q > n) return kInvalidArg;
+    std::vector<std::pair<int32_t, int32_t>> sp;
+    int rc = sorted_spans(n, starts, ends, n_spans, &sp);
+    if (rc != kOk) return rc;
+    const int32_t n_kt = ceil_div(n, kPrefillKeys);
+    std::vector<uint32_t> vis((size_t)n_kt * 4, 0);
+    for (int32_t j = 0; j < n; j += 32) {
+        const int32_t m = std::min(32, n - j);
+        vis[j >> 5] = m == 32 ? 0xffffffffu : ((1u << m) - 1u);
+    }
+    for (auto& ab : sp)
+        for (int32_t j = ab.first; j < ab.second; ++j) vis[j >> 5] &= ~(1u << (j & 31));
+    for (int32_t t = 0; t < n_kt; ++t) {
+        PrefillTile tile{};
+        tile.key0 = t * kPrefillKeys;
+        bool any = false, full = true;
+        for (int w = 0; w < 4; ++w) {
+            tile.vis[w] = vis[(size_t)t * 4 + w];
+            any |= tile.vis[w] != 0;
+            full &= tile.vis[w] == 0xffffffffu;
+        }
+        if (!any) continue;
+        tile.flags = full ? kPrefillTileFull : 0;
+        out->tiles.push_back(tile);
+    }
+    // visible keys of each query: the visible keys among 0 .. p
+    int64_t seen = 0, pairs = 0;
+    const int32_t q0 = n - n_q;
+    for (int32_t j = 0; j < n; ++j) {
+        seen += (vis[j >> 5] >> (j & 31)) & 1u;
+        if (j >= q0) pairs += seen;
+    }
+    out->visible_pairs = pairs;
+    out->n = n;
+    out->n_q = n_q;
+    out->BP = kPrefillRows / g.G();
+    out->n_qt = ceil_div(n_q, out->BP);
+    const int64_t units = (int64_t)out->n_qt * g.Hkv;
+    const int32_t n_tiles = (int32_t)out->tiles.size();
+    int32_t split = 1;
+    if (units < target_ctas && n_tiles > 0) {
+        // at least kMinTiles key tiles per split, at most kMaxSplit splits
+        constexpr int32_t kMinTiles = 4, kMaxSplit = 64;
+        split = (int32_t)std::min<int64_t>((target_ctas + units - 1) / units,
+                                           std::max<int32_t>(1, n_tiles / kMinTiles));
+        split = std::max(1, std::min(split, kMaxSplit));
+    }
+    out->n_split = split;
+    return kOk;
 }
 
 }  // namespace sq

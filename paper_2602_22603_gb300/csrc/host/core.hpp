@@ -16,6 +16,7 @@
 
 #include <stdint.h>
 
+#include <utility>
 #include <vector>
 
 #include "plan.hpp"
@@ -45,6 +46,11 @@ struct Geometry {
 
 // Validates a geometry against what the kernels handle.
 int check_geometry(const Geometry& g);
+
+// Checks half-open spans against a sequence of n tokens (each non-empty,
+// inside [0, n), no two overlapping; any order) and returns them sorted.
+int sorted_spans(int32_t n, const int32_t* starts, const int32_t* ends, int32_t n_spans,
+                 std::vector<std::pair<int32_t, int32_t>>* out);
 
 class PageAllocator {
   public:
@@ -168,5 +174,24 @@ DecodePlanLayout plan_layout(const DecodePlanHost& p, int32_t n_seqs,
                              int32_t Hkv);
 void plan_serialize(const DecodePlanHost& p, const DecodePlanLayout& lay,
                     uint8_t* dst);
+
+// ---- masked prefill planning ----------------------------------------------
+
+struct PrefillPlanHost {
+    std::vector<PrefillTile> tiles;   // key tiles with a visible key, increasing key0
+    int32_t n = 0, n_q = 0;
+    int32_t BP = 0;                   // query positions per tile
+    int32_t n_qt = 0;                 // query tiles per KV head
+    int32_t n_split = 1;              // key-range splits per query tile
+    int64_t visible_pairs = 0;        // sum over queries of the keys each sees
+};
+
+// Plans masked prefill attention over a sequence of n tokens whose last n_q
+// tokens are the queries: validates the spans, builds the per-tile visibility
+// bitmaps, and splits each query tile's key range in n_split parts when the
+// query tiles alone would fill fewer than `target_ctas` CTAs.
+int plan_prefill(const Geometry& g, int32_t n, int32_t n_q, const int32_t* starts,
+                 const int32_t* ends, int32_t n_spans, int32_t target_ctas,
+                 PrefillPlanHost* out);
 
 }  // namespace sq

@@ -61,6 +61,22 @@ struct EvictPiece {
     int32_t dst_row;      // row offset inside the tile
 };
 
+// Masked prefill attention (Algorithm 2, BuildMask).  A query tile holds
+// kPrefillRows rows: floor(kPrefillRows / G) consecutive query positions times
+// the G query heads of one KV head (Sec. 2.1), so one K/V tile serves them all.
+// Keys are taken kPrefillKeys at a time, aligned to kPrefillKeys.
+constexpr int kPrefillRows = 128;
+constexpr int kPrefillKeys = 128;
+constexpr int32_t kPrefillTileFull = 1;  // every key of the tile exists and is visible
+
+// One key tile that holds at least one visible key of the sequence.
+struct PrefillTile {
+    int32_t key0;      // first key position (a multiple of kPrefillKeys)
+    int32_t flags;     // kPrefillTileFull or 0
+    uint32_t vis[4];   // bit c of word w: key key0 + 32 w + c exists and lies in no span
+    int32_t pad[2];
+};
+
 // Byte offsets of the arrays of a decode plan inside one upload buffer.
 struct DecodePlanLayout {
     int64_t segs, items, cta_begin, page_ids, comb_off, comb_ent, total;

@@ -44,6 +44,41 @@ cudaError_t launch_decode(const CUtensorMap& tmap, const DecodeArgs& a, int n_ct
                           cudaStream_t st);
 cudaError_t launch_combine(const CombineArgs& a, int D, cudaStream_t st);
 
+// ---- masked prefill attention -------------------------------------------------
+struct PrefillArgs {
+    const PrefillTile* tiles;   // key tiles with a visible key, increasing key0
+    const int32_t* page_ids;    // the sequence's page table
+    int32_t n_tiles, n_pages_seq;
+    int32_t n, n_q;             // sequence tokens; queries = its last n_q tokens
+    int32_t layer, Hq, Hkv, G, P, num_pages;
+    int32_t BP;                 // query positions per tile (kPrefillRows / G)
+    int32_t n_qt, n_split;
+    float scale_log2;           // sm_scale * log2(e), >= 0
+    void* out;                  // [n_q][Hq][D] bf16 or fp32 (n_split == 1)
+    int32_t out_f32;
+    float* lse;                 // [n_q][Hq] or null (n_split == 1)
+    float* part_o;              // [grid][kPrefillRows][D] normalised partials (n_split > 1)
+    float* part_ml;             // [grid][kPrefillRows] log2-sum-exp of each partial
+    int* err;
+};
+
+struct PrefillCombineArgs {
+    const float* part_o;
+    const float* part_ml;
+    void* out;
+    int32_t out_f32;
+    float* lse;
+    int32_t n_q, Hq, Hkv, G, BP, n_qt, n_split;
+};
+
+// Dynamic shared memory of the prefill kernel.
+int prefill_smem_bytes(int D);
+cudaError_t prefill_prepare(int D);
+// qmap: 3-D map of the queries {D, Hq, n_q}, box {64, G, BP}, 128-byte swizzle.
+cudaError_t launch_prefill(const CUtensorMap& pool_map, const CUtensorMap& qmap,
+                           const PrefillArgs& a, int D, cudaStream_t st);
+cudaError_t launch_prefill_combine(const PrefillCombineArgs& a, int D, cudaStream_t st);
+
 // ---- append / copy-on-write / eviction --------------------------------------
 constexpr int kAppendMaxPages = 64;
 

@@ -1,0 +1,558 @@
+// Masked prefill attention on the 5th-generation tensor cores.
+//
+// What it computes (Algorithm 2, BuildMask; Sec. 3.3): the last n_q tokens of
+// a sequence attend causally to its tokens, with the tokens of the given spans
+// (closed cursors) removed from every query's view:
+//   query at position p, query head h, KV head g = floor(h / G):
+//     s_j = sm_scale * q_h . k_{g,j}   for visible keys j (j <= p, j in no span)
+//     o_h = sum_j softmax_j(s) v_{g,j}
+//
+// One CTA owns a tile of 128 query rows: floor(128 / G) consecutive query
+// positions times the G query heads of one KV head (Sec. 2.1), so every K/V
+// tile it loads serves all of them.  Keys go 128 at a time, aligned to 128;
+// tiles whose keys are all masked are never loaded (the host lists the
+// others with a visibility bitmap).  Per key tile j:
+//   S_j = Q K_j^T            tcgen05.mma, Q and K from shared memory, S in TMEM
+//   P_j = exp2(S_j - m)       softmax warps: tcgen05.ld of S, mask, bf16 P to smem
+//   O  += P_j V_j             tcgen05.mma, V read token-major (MN-major B)
+// S is double-buffered in TMEM so that S_{j+1} is computed while the softmax
+// warps work on S_j.  The running maximum m is raised lazily: O (in TMEM) is
+// rescaled only when a row's maximum grows by more than 2^8, so the weights
+// stay below 256 and most tiles need no rescale.
+//
+// Warp roles (192 threads): warp 0 loads (TMA), lane 0 of warp 1 issues the
+// MMAs and warp 1 owns the TMEM allocation, warps 2-5 run the softmax and the
+// epilogue (warp w reads TMEM lanes 32 (w mod 4) .. +31, one row per thread).
+// Every wait is bounded; a wait that runs out sets the error word and the CTA
+// winds down after its copies and MMAs in flight have completed.
+#include "launch.hpp"
+#include "ptx.cuh"
+#include "tc.cuh"
+
+namespace sq {
+namespace dev {
+namespace {
+
+template <int D>
+struct PreCfg {
+    static constexpr int kThreads = 192;
+    static constexpr int kColBlocks = D / 64;                 // 64-column (128-byte) blocks
+    static constexpr int kBlockBytes = kPrefillRows * 128;     // one block of a 128-row tile
+    static constexpr int kQBytes = kColBlocks * kBlockBytes;
+    static constexpr int kKVBytes = kColBlocks * kBlockBytes;  // 128 keys of K (or V)
+    static constexpr int kPBytes = 2 * kBlockBytes;            // 128 x 128 bf16 weights
+    static constexpr int kStages = D == 128 ? 2 : 3;
+    static constexpr int kOffQ = 0;
+    static constexpr int kOffK = kOffQ + kQBytes;
+    static constexpr int kOffV = kOffK + kStages * kKVBytes;
+    static constexpr int kOffP = kOffV + kStages * kKVBytes;
+    static constexpr int kOffBar = kOffP + 2 * kPBytes;
+    static constexpr int kBarQ = 0;
+    static constexpr int kBarK = 1;                     // [kStages] K tile landed
+    static constexpr int kBarV = kBarK + kStages;       // [kStages] V tile ready
+    static constexpr int kBarEmpty = kBarV + kStages;   // [kStages] stage consumed by the MMAs
+    static constexpr int kBarS = kBarEmpty + kStages;   // [2] S buffer written
+    static constexpr int kBarP = kBarS + 2;             // [2] P buffer written (128 arrivals)
+    static constexpr int kBarPV = kBarP + 2;            // [2] O += P V done
+    static constexpr int kBarVfix = kBarPV + 2;         // V of the last key tile landed
+    static constexpr int kBarDone = kBarVfix + 1;       // every MMA of the CTA done
+    static constexpr int kNumBars = kBarDone + 1;
+    static constexpr int kOffMisc = kOffBar + kNumBars * 8;
+    static constexpr int kSmemBytes = kOffMisc + 32 + 1024;  // + alignment slack
+    static constexpr uint32_t kTmemCols = 512;
+    static constexpr uint32_t kColS = 0;    // S_j at columns 128 (j mod 2)
+    static constexpr uint32_t kColO = 256;  // O at columns 256 .. 256 + D
+    static constexpr uint32_t kIdescQK = mma_idesc_bf16(128, kPrefillKeys, false);
+    static constexpr uint32_t kIdescPV = mma_idesc_bf16(128, D, true);
+    static_assert(kSmemBytes <= 232448, "shared memory");
+};
+
+struct Smem {
+    uint32_t base;  // shared address of the 1024-aligned region
+    uint8_t* ptr;
+    template <int D>
+    __device__ uint32_t bar(int i) const {
+        return base + PreCfg<D>::kOffBar + 8 * i;
+    }
+};
+
+// Bits 0 .. x of a word (x < 0: none; x >= 31: all).
+__device__ __forceinline__ uint32_t low_bits_through(int x) {
+    return x >= 31 ? 0xffffffffu : (x < 0 ? 0u : ((2u << x) - 1u));
+}
+
+template <int D>
+__device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* qmap,
+                                const PrefillArgs& a, const Smem& sm, int g, int pos_lo, int t0,
+                                int T, volatile int* abort_flag, int lane) {
+    using C = PreCfg<D>;
+    if (lane == 0) {
+        prefetch_tmap(pool_map);
+        prefetch_tmap(qmap);
+        mbar_arrive_expect_tx(sm.bar<D>(C::kBarQ), C::kColBlocks * a.BP * a.G * 128);
+        for (int cb = 0; cb < C::kColBlocks; ++cb)
+            tma_load_3d(sm.base + C::kOffQ + cb * C::kBlockBytes, qmap, sm.bar<D>(C::kBarQ),
+                        cb * 64, g * a.G, pos_lo);
+    }
+    const int br = a.P < 64 ? a.P : 64;  // rows of one TMA box
+    const int n_pieces = kPrefillKeys / br;
+    int issued = 0;
+    bool tail_issued = false;
+    for (int j = 0; j < T; ++j) {
+        const int s = j % C::kStages;
+        const int use = j / C::kStages;
+        if (use > 0) {
+            bool ok = mbar_wait(sm.bar<D>(C::kBarEmpty + s), (use - 1) & 1, abort_flag);
+            if (!__all_sync(0xffffffffu, ok)) {
+                if (lane == 0) {
+                    set_error(a.err, kErrTimeout);
+                    *abort_flag = 1;
+                }
+                break;
+            }
+        }
+        const int key0 = __ldg(&a.tiles[t0 + j].key0);
+        const bool tail = key0 + kPrefillKeys > a.n;
+        if (lane == 0) {
+            // pieces that hold tokens of the sequence and a page inside the pool
+            uint32_t pmask = 0;
+            for (int i = 0; i < n_pieces; ++i) {
+                const int key = key0 + i * br;
+                if (key >= a.n) break;
+                const int32_t page = __ldg(&a.page_ids[key / a.P]);
+                if ((uint32_t)page < (uint32_t)a.num_pages) pmask |= 1u << i;
+                else set_error(a.err, kErrBounds);
+            }
+            const uint32_t bytes = (uint32_t)__popc(pmask) * br * 128 * C::kColBlocks;
+            const uint32_t kb = sm.bar<D>(C::kBarK + s);
+            const uint32_t vb = tail ? sm.bar<D>(C::kBarVfix) : sm.bar<D>(C::kBarV + s);
+            mbar_arrive_expect_tx(kb, bytes);
+            mbar_arrive_expect_tx(vb, bytes);
+            const uint32_t ks = sm.base + C::kOffK + s * C::kKVBytes;
+            const uint32_t vs = sm.base + C::kOffV + s * C::kKVBytes;
+            for (int i = 0; i < n_pieces; ++i) {
+                if (!((pmask >> i) & 1u)) continue;
+                const int key = key0 + i * br;
+                const int32_t page = __ldg(&a.page_ids[key / a.P]);
+                const int row0 = key % a.P;
+                for (int cb = 0; cb < C::kColBlocks; ++cb) {
+                    const uint32_t off = cb * C::kBlockBytes + i * br * 128;
+                    tma_load_4d(ks + off, pool_map, kb, cb * 64, g * a.P + row0, page, a.layer);
+                    tma_load_4d(vs + off, pool_map, vb, cb * 64, (a.Hkv + g) * a.P + row0, page,
+                                a.layer);
+                }
+            }
+        }
+        issued = j + 1;
+        if (tail) {
+            // The last key tile: its rows past the sequence's end hold stale
+            // or never-written data.  Their weights are zero, but 0 * NaN is
+            // not, so zero those V rows before the MMAs read the stage.
+            tail_issued = true;
+            bool ok = mbar_wait(sm.bar<D>(C::kBarVfix), 0, abort_flag);
+            if (!__all_sync(0xffffffffu, ok)) {
+                if (lane == 0) {
+                    set_error(a.err, kErrTimeout);
+                    *abort_flag = 1;
+                }
+                break;
+            }
+            const int r0 = a.n - key0;  // 1 .. 127
+            const int chunks = (kPrefillKeys - r0) * 8;
+            uint8_t* vsp = sm.ptr + C::kOffV + s * C::kKVBytes;
+            for (int cb = 0; cb < C::kColBlocks; ++cb)
+                for (int c = lane; c < chunks; c += 32)
+                    *reinterpret_cast<uint4*>(vsp + cb * C::kBlockBytes + (r0 + (c >> 3)) * 128 +
+                                              (c & 7) * 16) = make_uint4(0, 0, 0, 0);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(sm.bar<D>(C::kBarV + s));
+        }
+    }
+    // Drain: every copy this CTA issued lands before the CTA exits (immediate
+    // unless a consumer gave up early).
+    if (lane == 0) {
+        mbar_wait(sm.bar<D>(C::kBarQ), 0);
+        for (int j = issued > C::kStages ? issued - C::kStages : 0; j < issued; ++j) {
+            const int s = j % C::kStages;
+            mbar_wait(sm.bar<D>(C::kBarK + s), (j / C::kStages) & 1);
+            const bool is_tail = tail_issued && j == issued - 1;
+            if (is_tail) mbar_wait(sm.bar<D>(C::kBarVfix), 0);
+            else mbar_wait(sm.bar<D>(C::kBarV + s), (j / C::kStages) & 1);
+        }
+    }
+}
+
+template <int D>
+__device__ __forceinline__ bool issue_qk(const Smem& sm, uint32_t tmem, int j,
+                                         volatile int* abort_flag) {
+    using C = PreCfg<D>;
+    const int s = j % C::kStages;
+    if (!mbar_wait(sm.bar<D>(C::kBarK + s), (j / C::kStages) & 1, abort_flag)) return false;
+    const uint32_t qa = sm.base + C::kOffQ;
+    const uint32_t ka = sm.base + C::kOffK + s * C::kKVBytes;
+    const uint32_t dt = tmem + C::kColS + (uint32_t)(j & 1) * kPrefillKeys;
+#pragma unroll
+    for (int ks = 0; ks < D / 16; ++ks) {
+        const uint32_t off = (ks >> 2) * C::kBlockBytes + (ks & 3) * 32;
+        mma_bf16_ss(dt, smem_desc_sw128(qa + off, 16, 1024), smem_desc_sw128(ka + off, 16, 1024),
+                    C::kIdescQK, ks > 0);
+    }
+    mma_commit(sm.bar<D>(C::kBarS + (j & 1)));
+    return true;
+}
+
+template <int D>
+__device__ void prefill_mma(const PrefillArgs& a, const Smem& sm, uint32_t tmem, int T,
+                            volatile int* abort_flag) {
+    using C = PreCfg<D>;
+    bool ok = mbar_wait(sm.bar<D>(C::kBarQ), 0, abort_flag);
+    bool any = false;
+    if (ok && T > 0) {
+        tc_fence_after();
+        ok = issue_qk<D>(sm, tmem, 0, abort_flag);
+        any = ok;
+        for (int j = 0; ok && j < T; ++j) {
+            const int s = j % C::kStages;
+            if (j + 1 < T && !(ok = issue_qk<D>(sm, tmem, j + 1, abort_flag))) break;
+            if (!(ok = mbar_wait(sm.bar<D>(C::kBarP + (j & 1)), (j >> 1) & 1, abort_flag))) break;
+            tc_fence_after();
+            if (!(ok = mbar_wait(sm.bar<D>(C::kBarV + s), (j / C::kStages) & 1, abort_flag))) break;
+            const uint32_t pa = sm.base + C::kOffP + (j & 1) * C::kPBytes;
+            const uint32_t va = sm.base + C::kOffV + s * C::kKVBytes;
+#pragma unroll
+            for (int ks = 0; ks < kPrefillKeys / 16; ++ks) {
+                const uint32_t aoff = (ks >> 2) * C::kBlockBytes + (ks & 3) * 32;
+                mma_bf16_ss(tmem + C::kColO, smem_desc_sw128(pa + aoff, 16, 1024),
+                            smem_desc_sw128(va + ks * 16 * 128, C::kBlockBytes, 1024),
+                            C::kIdescPV, (j > 0 || ks > 0) ? 1u : 0u);
+            }
+            mma_commit(sm.bar<D>(C::kBarPV + (j & 1)));
+            mma_commit(sm.bar<D>(C::kBarEmpty + s));
+        }
+    }
+    if (!ok) {
+        set_error(a.err, kErrTimeout);
+        *abort_flag = 1;
+    }
+    if (any) {
+        // every MMA issued here completes before TMEM is released
+        mma_commit(sm.bar<D>(C::kBarDone));
+        mbar_wait(sm.bar<D>(C::kBarDone), 0);
+    }
+}
+
+template <int D>
+__device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t tmem, int rest,
+                                int g, int pos_lo, int t0, int T, volatile int* abort_flag,
+                                int warp, int lane) {
+    using C = PreCfg<D>;
+    const int wq = warp & 3;
+    const int row = wq * 32 + lane;
+    const int qi = pos_lo + row / a.G;
+    const bool valid = row < a.BP * a.G && qi < a.n_q;
+    const int p_row = a.n - a.n_q + qi;
+    const uint32_t tl = tmem + ((uint32_t)(wq * 32) << 16);
+    const float sc = a.scale_log2;
+    float m_run = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < T; ++j) {
+        const int4* tp = reinterpret_cast<const int4*>(a.tiles + t0 + j);
+        const int4 w0 = __ldg(tp), w1 = __ldg(tp + 1);
+        const int key0 = w0.x;
+        const uint32_t vis[4] = {(uint32_t)w0.z, (uint32_t)w0.w, (uint32_t)w1.x, (uint32_t)w1.y};
+        ok = __all_sync(0xffffffffu,
+                        mbar_wait(sm.bar<D>(C::kBarS + (j & 1)), (j >> 1) & 1, abort_flag));
+        if (!ok) break;
+        tc_fence_after();
+        float x[kPrefillKeys];
+        {
+            uint32_t u[kPrefillKeys];
+#pragma unroll
+            for (int c = 0; c < kPrefillKeys / 32; ++c)
+                tmem_ld32(tl + C::kColS + (uint32_t)(j & 1) * kPrefillKeys + c * 32,
+                          *reinterpret_cast<uint32_t(*)[32]>(&u[c * 32]));
+            tmem_wait_ld();
+#pragma unroll
+            for (int c = 0; c < kPrefillKeys; ++c) x[c] = __uint_as_float(u[c]) * sc;
+        }
+        const int lim = p_row - key0;  // keys key0 + c with c <= lim are causal
+        if (!(valid && (w0.y & kPrefillTileFull) && lim >= kPrefillKeys - 1)) {
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+                const uint32_t mw = valid ? (vis[w] & low_bits_through(lim - 32 * w)) : 0u;
+#pragma unroll
+                for (int c = 0; c < 32; ++c)
+                    if (!((mw >> c) & 1u)) x[32 * w + c] = -INFINITY;
+            }
+        }
+        float mt = x[0];
+#pragma unroll
+        for (int c = 1; c < kPrefillKeys; ++c) mt = fmaxf(mt, x[c]);
+        const bool need = mt > m_run + 8.f;
+        float alpha = 1.f;
+        if (need) {
+            alpha = exp2f(m_run - mt);
+            m_run = mt;
+            l *= alpha;
+        }
+        if (j > 0 && __any_sync(0xffffffffu, need)) {
+            // O holds P_{j-1} V_{j-1} once that MMA is done: rescale it in place
+            ok = __all_sync(0xffffffffu, mbar_wait(sm.bar<D>(C::kBarPV + ((j - 1) & 1)),
+                                                   ((j - 1) >> 1) & 1, abort_flag));
+            if (!ok) break;
+            tc_fence_after();
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t o[32];
+                tmem_ld32(tl + C::kColO + c * 32, o);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+                tmem_st32(tl + C::kColO + c * 32, o);
+            }
+            tmem_wait_st();
+        }
+        if (j >= 2) {
+            // P buffer (j mod 2) was last read by the MMAs of tile j - 2
+            ok = __all_sync(0xffffffffu, mbar_wait(sm.bar<D>(C::kBarPV + (j & 1)),
+                                                   ((j - 2) >> 1) & 1, abort_flag));
+            if (!ok) break;
+        }
+        const float mu = m_run == -INFINITY ? 0.f : m_run;
+        uint8_t* prow = sm.ptr + C::kOffP + (j & 1) * C::kPBytes + row * 128;
+#pragma unroll
+        for (int k = 0; k < kPrefillKeys / 8; ++k) {
+            uint32_t w[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const __nv_bfloat162 h =
+                    __floats2bfloat162_rn(exp2f(x[8 * k + 2 * e] - mu), exp2f(x[8 * k + 2 * e + 1] - mu));
+                w[e] = *reinterpret_cast<const uint32_t*>(&h);
+                l += __uint_as_float(w[e] << 16) + __uint_as_float(w[e] & 0xffff0000u);
+            }
+            const int cb = k >> 3, ch = (k & 7) ^ (row & 7);
+            *reinterpret_cast<uint4*>(prow + cb * C::kBlockBytes + ch * 16) =
+                make_uint4(w[0], w[1], w[2], w[3]);
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        mbar_arrive(sm.bar<D>(C::kBarP + (j & 1)));
+    }
+    if (ok && T > 0)
+        ok = __all_sync(0xffffffffu, mbar_wait(sm.bar<D>(C::kBarPV + ((T - 1) & 1)),
+                                               ((T - 1) >> 1) & 1, abort_flag));
+    if (!ok) {
+        if (lane == 0) {
+            set_error(a.err, kErrTimeout);
+            *abort_flag = 1;
+        }
+        return;
+    }
+    tc_fence_after();
+    const float inv = l > 0.f ? 1.f / l : 0.f;
+    const float lse2 = l > 0.f ? m_run + __log2f(l) : -INFINITY;
+    const int h = g * a.G + row % a.G;
+    float* part_row = nullptr;
+    uint8_t* out_row = nullptr;
+    if (a.n_split > 1) {
+        part_row = a.part_o + ((size_t)blockIdx.x * kPrefillRows + row) * D;
+        if (valid) a.part_ml[(size_t)blockIdx.x * kPrefillRows + row] = lse2;
+    } else {
+        out_row = reinterpret_cast<uint8_t*>(a.out) +
+                  ((size_t)qi * a.Hq + h) * D * (a.out_f32 ? 4 : 2);
+        if (valid && a.lse) a.lse[(size_t)qi * a.Hq + h] = lse2 * 0.69314718055994531f;
+    }
+#pragma unroll
+    for (int c = 0; c < D / 32; ++c) {
+        uint32_t o[32];
+        if (T > 0) {
+            tmem_ld32(tl + C::kColO + c * 32, o);
+            tmem_wait_ld();
+        } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] = 0u;
+        }
+        if (!valid) continue;
+        float f[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) f[i] = __uint_as_float(o[i]) * inv;
+        if (part_row || a.out_f32) {
+            float4* dst = reinterpret_cast<float4*>(part_row ? part_row + c * 32
+                                                             : reinterpret_cast<float*>(out_row) + c * 32);
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                dst[i] = make_float4(f[4 * i], f[4 * i + 1], f[4 * i + 2], f[4 * i + 3]);
+        } else {
+            uint4* dst = reinterpret_cast<uint4*>(out_row + c * 64);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                uint32_t w[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const __nv_bfloat162 hb = __floats2bfloat162_rn(f[8 * i + 2 * e], f[8 * i + 2 * e + 1]);
+                    w[e] = *reinterpret_cast<const uint32_t*>(&hb);
+                }
+                dst[i] = make_uint4(w[0], w[1], w[2], w[3]);
+            }
+        }
+    }
+    (void)rest;
+}
+
+template <int D>
+__global__ void __launch_bounds__(192, 1)
+    sq_prefill_kernel(const __grid_constant__ CUtensorMap pool_map,
+                      const __grid_constant__ CUtensorMap qmap, const PrefillArgs a) {
+    using C = PreCfg<D>;
+    extern __shared__ uint8_t smem_raw[];
+    Smem sm;
+    sm.ptr = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                        ~static_cast<uintptr_t>(1023));
+    sm.base = smem_addr(sm.ptr);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm.ptr + C::kOffMisc);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(sm.ptr + C::kOffMisc + 4);
+    int* sched = reinterpret_cast<int*>(sm.ptr + C::kOffMisc + 8);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // heaviest query tiles (latest positions) first
+    const int split = blockIdx.x % a.n_split;
+    const int rest = blockIdx.x / a.n_split;
+    const int g = rest % a.Hkv;
+    const int qt = a.n_qt - 1 - rest / a.Hkv;
+    const int pos_lo = qt * a.BP;
+    const int q_pos = min(a.BP, a.n_q - pos_lo);
+    if (threadIdx.x == 0) {
+        mbar_init(sm.bar<D>(C::kBarQ), 1);
+        for (int s = 0; s < C::kStages; ++s) {
+            mbar_init(sm.bar<D>(C::kBarK + s), 1);
+            mbar_init(sm.bar<D>(C::kBarV + s), 1);
+            mbar_init(sm.bar<D>(C::kBarEmpty + s), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(sm.bar<D>(C::kBarS + b), 1);
+            mbar_init(sm.bar<D>(C::kBarP + b), 128);
+            mbar_init(sm.bar<D>(C::kBarPV + b), 1);
+        }
+        mbar_init(sm.bar<D>(C::kBarVfix), 1);
+        mbar_init(sm.bar<D>(C::kBarDone), 1);
+        fence_mbar_init();
+        *abort_flag = 0;
+        // key tiles up to the last query position, split evenly
+        const int p_last = a.n - a.n_q + pos_lo + q_pos - 1;
+        int lo = 0, hi = a.n_tiles;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (__ldg(&a.tiles[mid].key0) <= p_last) lo = mid + 1;
+            else hi = mid;
+        }
+        const int t0 = (int)((int64_t)lo * split / a.n_split);
+        sched[0] = t0;
+        sched[1] = (int)((int64_t)lo * (split + 1) / a.n_split) - t0;
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_addr(tmem_slot), C::kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const int t0 = sched[0], T = sched[1];
+    if (warp == 0) {
+        prefill_produce<D>(&pool_map, &qmap, a, sm, g, pos_lo, t0, T, abort_flag, lane);
+    } else if (warp == 1) {
+        if (lane == 0) prefill_mma<D>(a, sm, tmem, T, abort_flag);
+        __syncwarp();
+    } else {
+        prefill_softmax<D>(a, sm, tmem, rest, g, pos_lo, t0, T, abort_flag, warp, lane);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, C::kTmemCols);
+    }
+}
+
+// Merges the key-range splits of each query row: weights 2^(lse_s - max).
+template <int D>
+__global__ void __launch_bounds__(256) sq_prefill_combine_kernel(const PrefillCombineArgs a) {
+    const int gw = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+    const int lane = threadIdx.x & 31;
+    const int units = a.n_qt * a.Hkv;
+    if (gw >= units * kPrefillRows) return;
+    const int rest = gw / kPrefillRows, row = gw % kPrefillRows;
+    const int g = rest % a.Hkv, qt = a.n_qt - 1 - rest / a.Hkv;
+    const int qi = qt * a.BP + row / a.G;
+    if (row >= a.BP * a.G || qi >= a.n_q) return;
+    const int h = g * a.G + row % a.G;
+    float M = -INFINITY;
+    for (int s = 0; s < a.n_split; ++s)
+        M = fmaxf(M, a.part_ml[((size_t)rest * a.n_split + s) * kPrefillRows + row]);
+    float W = 0.f, acc[D / 32];
+#pragma unroll
+    for (int e = 0; e < D / 32; ++e) acc[e] = 0.f;
+    if (M != -INFINITY) {
+        for (int s = 0; s < a.n_split; ++s) {
+            const size_t pr = ((size_t)rest * a.n_split + s) * kPrefillRows + row;
+            const float ml = a.part_ml[pr];
+            if (ml == -INFINITY) continue;
+            const float w = exp2f(ml - M);
+            W += w;
+            const float* po = a.part_o + pr * D;
+#pragma unroll
+            for (int e = 0; e < D / 32; ++e) acc[e] += w * po[lane + 32 * e];
+        }
+    }
+    const float inv = W > 0.f ? 1.f / W : 0.f;
+    const size_t o = ((size_t)qi * a.Hq + h) * D;
+#pragma unroll
+    for (int e = 0; e < D / 32; ++e) {
+        const float v = acc[e] * inv;
+        if (a.out_f32) reinterpret_cast<float*>(a.out)[o + lane + 32 * e] = v;
+        else reinterpret_cast<__nv_bfloat16*>(a.out)[o + lane + 32 * e] = __float2bfloat16_rn(v);
+    }
+    if (lane == 0 && a.lse)
+        a.lse[(size_t)qi * a.Hq + h] = W > 0.f ? (M + __log2f(W)) * 0.69314718055994531f : -INFINITY;
+}
+
+}  // namespace
+}  // namespace dev
+
+int prefill_smem_bytes(int D) {
+    return D == 128 ? dev::PreCfg<128>::kSmemBytes : dev::PreCfg<64>::kSmemBytes;
+}
+
+cudaError_t prefill_prepare(int D) {
+    if (D == 128)
+        return cudaFuncSetAttribute(dev::sq_prefill_kernel<128>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    dev::PreCfg<128>::kSmemBytes);
+    return cudaFuncSetAttribute(dev::sq_prefill_kernel<64>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                dev::PreCfg<64>::kSmemBytes);
+}
+
+cudaError_t launch_prefill(const CUtensorMap& pool_map, const CUtensorMap& qmap,
+                           const PrefillArgs& a, int D, cudaStream_t st) {
+    const unsigned grid = (unsigned)(a.n_qt * a.Hkv * a.n_split);
+    if (grid == 0) return cudaSuccess;
+    if (D == 128)
+        dev::sq_prefill_kernel<128><<<grid, dev::PreCfg<128>::kThreads,
+                                      dev::PreCfg<128>::kSmemBytes, st>>>(pool_map, qmap, a);
+    else
+        dev::sq_prefill_kernel<64><<<grid, dev::PreCfg<64>::kThreads, dev::PreCfg<64>::kSmemBytes,
+                                     st>>>(pool_map, qmap, a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_prefill_combine(const PrefillCombineArgs& a, int D, cudaStream_t st) {
+    const int64_t warps = (int64_t)a.n_qt * a.Hkv * kPrefillRows;
+    const unsigned grid = (unsigned)((warps * 32 + 255) / 256);
+    if (grid == 0) return cudaSuccess;
+    if (D == 128) dev::sq_prefill_combine_kernel<128><<<grid, 256, 0, st>>>(a);
+    else dev::sq_prefill_combine_kernel<64><<<grid, 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace sq

@@ -1,0 +1,202 @@
+"""Masked prefill attention (Algorithm 2, BuildMask) on the GPU against the
+oracle: every output row and log-sum-exp at small sizes that still span
+several query and key tiles with ragged tails, across GQA groups, head dims,
+page sizes, span layouts (including a masked prefix and masked queries), the
+split-key path for short query blocks, forked sequences and evicted ones."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2602_22603_gb300 as sq
+from oracle import attention as oatt
+from synthetic import bf16_bits, bf16_normal, random_spans
+from tests.gpu_harness import Pair, assert_close
+
+pytestmark = pytest.mark.gpu
+
+LSE_ABS = 1e-2
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2602_22603_gb300 import build
+    build.build_libsq()
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+
+
+def run_prefill(p: Pair, h, layer, n_q, spans, seed, scale, out_dtype=sq.SQ_OUT_F32):
+    q_cpu = bf16_normal((n_q, p.Hq, p.D), seed)
+    dt = torch.float32 if out_dtype == sq.SQ_OUT_F32 else torch.bfloat16
+    out = torch.full((n_q, p.Hq, p.D), float("nan"), dtype=dt, device="cuda")
+    lse = torch.full((n_q, p.Hq), float("nan"), dtype=torch.float32, device="cuda")
+    p.cache.prefill_attention(h, layer, n_q, q_cpu.cuda(), out, out_dtype, lse, scale, spans)
+    torch.cuda.synchronize()
+    assert p.cache.sync_status() == sq.SQ_OK
+    return q_cpu, out, lse
+
+
+def oracle_prefill(p: Pair, h, layer, q_cpu, spans, scale):
+    k, v = p.store.rows(p.oracle.tokens(p.o[h]), layer)
+    return oatt.prefill(bf16_bits(q_cpu), k, v, scale, spans, want_lse=True)
+
+
+def check(p, h, layer, n_q, spans, seed, scale=None, out_dtype=sq.SQ_OUT_F32):
+    scale = scale if scale is not None else 1.0 / math.sqrt(p.D)
+    q_cpu, out, lse = run_prefill(p, h, layer, n_q, spans, seed, scale, out_dtype)
+    exp, exp_lse = oracle_prefill(p, h, layer, q_cpu, spans, scale)
+    assert_close(out, exp)
+    got_lse = lse.cpu().numpy().astype(np.float64)
+    fin = np.isfinite(exp_lse)
+    assert np.array_equal(np.isfinite(got_lse), fin)
+    if fin.any():
+        assert np.abs(got_lse[fin] - exp_lse[fin]).max() <= LSE_ABS
+    return out, lse
+
+
+def spans_for(n, k, seed):
+    if n < 4 or k == 0:
+        return []
+    total = max(k, n // 3)
+    return random_spans(seed, k, total, 0, n, median=max(1.0, total / k))
+
+
+@pytest.mark.parametrize("Hq,Hkv,D,P", [
+    (16, 4, 64, 16),    # G = 4, the tiny shape
+    (32, 8, 128, 64),   # G = 4, d = 128, the 8B-class shape
+    (8, 8, 64, 8),      # G = 1: textbook MHA, 8-token pages
+    (6, 2, 128, 256),   # G = 3: padded query tiles, 256-token pages
+    (32, 2, 64, 32),    # G = 16: 8 positions per query tile
+])
+@pytest.mark.parametrize("n,n_q,k", [(1, 1, 0), (129, 129, 2), (300, 37, 3), (517, 517, 5)])
+def test_prefill_matches_oracle(Hq, Hkv, D, P, n, n_q, k):
+    p = Pair(2, Hq, Hkv, D, P, num_pages=(n + P - 1) // P + 8, seed=n + Hq)
+    try:
+        h = p.seq_new()
+        p.append(h, n)
+        spans = spans_for(n, k, n * 3 + k)
+        check(p, h, 1, n_q, spans, seed=n + 7)
+    finally:
+        p.close()
+
+
+def test_prefill_bf16_output_and_long_ragged_sequence():
+    p = Pair(1, 32, 8, 128, 64, num_pages=40, seed=5)
+    try:
+        h = p.seq_new()
+        for chunk in (700, 1, 1000, 333):   # several appends, a ragged last page
+            p.append(h, chunk)
+        n = 2034
+        spans = random_spans(9, 6, 800, 64, n, median=130)
+        check(p, h, 0, n, spans, seed=11, out_dtype=sq.SQ_OUT_BF16)
+    finally:
+        p.close()
+
+
+def test_prefill_split_key_ranges():
+    # 8 query positions over 3000 keys: one query tile per KV head, so the key
+    # range is split across CTAs and merged by the combine kernel.
+    p = Pair(1, 32, 8, 128, 64, num_pages=60, seed=6)
+    try:
+        h = p.seq_new()
+        p.append(h, 3000)
+        spans = random_spans(4, 10, 1200, 0, 3000, median=120)
+        check(p, h, 0, 8, spans, seed=3)
+        check(p, h, 0, 8, [], seed=4, out_dtype=sq.SQ_OUT_BF16)
+    finally:
+        p.close()
+
+
+def test_prefill_masked_prefix_gives_empty_rows():
+    # spans covering [0, 200): the first 200 queries see nothing (zeros,
+    # -inf), later ones see only the unmasked suffix
+    p = Pair(1, 16, 4, 64, 16, num_pages=40, seed=8)
+    try:
+        h = p.seq_new()
+        p.append(h, 400)
+        out, lse = check(p, h, 0, 400, [(0, 150), (150, 200)], seed=1)
+        assert not out[:200].any()
+        assert torch.isinf(lse[:200]).all() and (lse[:200] < 0).all()
+        # only the last token visible: the last query sees itself, the rest nothing
+        out, _ = check(p, h, 0, 400, [(0, 399)], seed=2)
+    finally:
+        p.close()
+
+
+def test_prefill_on_fork_and_after_eviction():
+    # the aux thread's prefill reads the shared pages; after the main thread
+    # evicts, the aux keeps its view and the main thread's masked prefill over
+    # the evicted context equals decode over it
+    p = Pair(2, 32, 8, 128, 64, num_pages=80, seed=9)
+    try:
+        m = p.seq_new()
+        p.append(m, 1500)
+        a = p.fork(m)
+        p.append(a, 24)                       # trigger + aux tokens
+        check(p, a, 1, 24, [], seed=5)        # aux prefill over the shared context
+        spans = [(100, 400), (700, 710), (900, 1300)]
+        p.evict(m, spans)
+        p.append(m, 1)
+        check(p, a, 1, 24, [(64, 128)], seed=6)
+        n = p.cache.seq_info(m)[0]
+        q_cpu, out, _ = run_prefill(p, m, 0, 1, [], 7, 0.088)
+        dec = p.decode([m], 0, 0.088, q_cpu.cuda())
+        torch.cuda.synchronize()
+        assert (out[0] - dec[0]).abs().max().item() < 2e-3
+        exp = p.oracle_decode([m], 0, 0.088, q_cpu)
+        assert_close(out, exp)
+        assert n == 1500 - 710 + 1
+    finally:
+        p.close()
+
+
+def test_prefill_masked_equals_evicted():
+    # Algorithm 2 (mask) vs Algorithm 1 (evict): the masked prefill's last
+    # query over the full context equals prefill's last query after the spans
+    # are evicted, both on the GPU.
+    p = Pair(1, 16, 4, 64, 16, num_pages=80, seed=10)
+    try:
+        m = p.seq_new()
+        p.append(m, 900)
+        spans = [(17, 90), (300, 301), (500, 870)]
+        q_cpu = bf16_normal((1, 16, 64), 77)
+        out_mask = torch.empty(1, 16, 64, dtype=torch.float32, device="cuda")
+        p.cache.prefill_attention(m, 0, 1, q_cpu.cuda(), out_mask, sq.SQ_OUT_F32, None, 0.125, spans)
+        p.evict(m, spans)
+        out_evict = torch.empty_like(out_mask)
+        p.cache.prefill_attention(m, 0, 1, q_cpu.cuda(), out_evict, sq.SQ_OUT_F32, None, 0.125, [])
+        torch.cuda.synchronize()
+        assert (out_mask - out_evict).abs().max().item() < 2e-3
+    finally:
+        p.close()
+
+
+def test_prefill_rejects_bad_arguments():
+    p = Pair(1, 16, 4, 64, 16, num_pages=20, seed=11)
+    try:
+        h = p.seq_new()
+        p.append(h, 100)
+        q = torch.zeros(10, 16, 64, dtype=torch.bfloat16, device="cuda")
+        out = torch.zeros(10, 16, 64, dtype=torch.float32, device="cuda")
+        c = p.cache
+        bad = [
+            dict(n_q=101), dict(n_q=0), dict(layer=1), dict(spans=[(5, 5)]),
+            dict(spans=[(5, 9), (8, 12)]), dict(spans=[(90, 101)]), dict(sm_scale=-1.0),
+            dict(sm_scale=float("nan")), dict(out_dtype=7),
+        ]
+        for kw in bad:
+            args = dict(seq=h, layer=0, n_q=10, q=q, out=out, out_dtype=sq.SQ_OUT_F32,
+                        lse=None, sm_scale=0.1, spans=[])
+            args.update(kw)
+            with pytest.raises(sq.SqError) as ei:
+                c.prefill_attention(**args)
+            assert ei.value.code == sq.SQ_ERR_INVALID_ARG, kw
+        with pytest.raises(sq.SqError) as ei:
+            c.prefill_attention(123456789, 0, 10, q, out, sq.SQ_OUT_F32, None, 0.1, [])
+        assert ei.value.code == sq.SQ_ERR_BAD_HANDLE
+        torch.cuda.synchronize()
+        assert c.sync_status() == sq.SQ_OK
+    finally:
+        p.close()

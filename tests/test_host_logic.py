@@ -263,3 +263,73 @@ def test_evict_tiles_compact_in_place(seed):
     for a, oa in forks:
         apt = hc.page_table(a)
         assert [phys[apt[j // P]][j % P] for j in range(oc.n_tokens(oa))] == oc.tokens(oa)
+
+
+# ---------------------------------------------------------------------------
+# masked prefill planning (Algorithm 2, BuildMask)
+# ---------------------------------------------------------------------------
+def _brute_prefill_plan(n, n_q, spans):
+    removed = [False] * n
+    for a, b in spans:
+        for j in range(a, b):
+            removed[j] = True
+    tiles = []
+    for key0 in range(0, n, 128):
+        bits = [key0 + c < n and not removed[key0 + c] for c in range(128)]
+        if any(bits):
+            words = [sum(1 << c for c in range(32) if bits[32 * w + c]) for w in range(4)]
+            tiles.append((key0, int(all(bits)), words))
+    pairs = sum(sum(1 for j in range(p + 1) if not removed[j]) for p in range(n - n_q, n))
+    return tiles, pairs
+
+
+@pytest.mark.parametrize("seed", range(10))
+def test_prefill_plan_visibility_matches_brute_force(seed):
+    from tests.hostlib import plan_prefill
+    rng = random.Random(seed)
+    n = rng.choice([1, 5, 127, 128, 129, 700, 1500])
+    n_q = rng.choice([1, n, max(1, n // 3)])
+    Hkv = rng.choice([1, 2, 8])
+    G = rng.choice([1, 3, 4, 16])
+    k = rng.randint(0, 6)
+    cuts = sorted(rng.sample(range(n + 1), min(2 * k, n + 1)))
+    spans = [(cuts[i], cuts[i + 1]) for i in range(0, len(cuts) - 1, 2) if cuts[i] < cuts[i + 1]]
+    rng.shuffle(spans)
+    rc, info, tiles = plan_prefill(G * Hkv, Hkv, n, n_q, spans)
+    assert rc == 0
+    exp_tiles, exp_pairs = _brute_prefill_plan(n, n_q, spans)
+    assert info["tile_bytes"] == 32
+    assert info["n_tiles"] == len(exp_tiles)
+    for got, (key0, full, words) in zip(tiles, exp_tiles):
+        assert got[0] == key0 and got[1] == full and list(got[2:]) == words
+    assert info["visible_pairs"] == exp_pairs
+    assert info["BP"] == 128 // G
+    assert info["n_qt"] == -(-n_q // (128 // G))
+    units = info["n_qt"] * Hkv
+    assert info["n_split"] >= 1
+    if units >= 152:
+        assert info["n_split"] == 1
+    else:
+        assert info["n_split"] <= max(1, len(exp_tiles) // 4)
+
+
+def test_prefill_plan_rejects_bad_input():
+    from tests.hostlib import plan_prefill
+    assert plan_prefill(8, 2, 100, 101, [])[0] == -1      # more queries than tokens
+    assert plan_prefill(8, 2, 100, 0, [])[0] == -1
+    assert plan_prefill(8, 2, 100, 10, [(5, 5)])[0] == -1      # empty span
+    assert plan_prefill(8, 2, 100, 10, [(5, 9), (8, 12)])[0] == -1  # overlap
+    assert plan_prefill(8, 2, 100, 10, [(90, 101)])[0] == -1   # past the end
+    assert plan_prefill(8, 2, 100, 10, [(-1, 3)])[0] == -1
+    rc, info, _ = plan_prefill(8, 2, 100, 10, [(0, 100)])      # everything masked
+    assert rc == 0 and info["n_tiles"] == 0 and info["visible_pairs"] == 0
+
+
+def test_prefill_plan_splits_short_query_blocks():
+    # 8 trigger tokens over a long context: one query tile per KV head, so the
+    # key range is split to fill the GPU; a full prefill is not split.
+    from tests.hostlib import plan_prefill
+    rc, info, _ = plan_prefill(32, 8, 131072, 8, [])
+    assert rc == 0 and info["n_qt"] == 1 and info["n_split"] == 19
+    rc, info, _ = plan_prefill(32, 8, 32768, 32768, [(100, 5000)])
+    assert rc == 0 and info["n_split"] == 1 and info["n_qt"] == 1024
