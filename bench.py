@@ -35,6 +35,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "decode-attn tokens/s + achieved HBM GB/s at 128k ctx; span-evict GB/s"
+PREFILL_METRIC = "masked-prefill attention tokens/s at 32k ctx (all layers) + achieved bf16 TFLOP/s"
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -45,7 +46,8 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="sq", choices=["sq", "reference"])
     ap.add_argument("--workload", default="serving-128k",
-                    choices=["serving-128k", "large-ragged", "agent-32k", "trace"])
+                    choices=["serving-128k", "large-ragged", "agent-32k", "trace", "prefill-32k"])
+    ap.add_argument("--prefill-ctx", type=int, default=32768, help="prefill-32k: context tokens")
     ap.add_argument("--turns", type=int, default=50, help="trace: turns per agent")
     ap.add_argument("--requests", type=int, default=8)
     ap.add_argument("--ctx", type=int, default=131072)
@@ -55,6 +57,17 @@ def parse_args():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--seed", type=int, default=0)
     return ap.parse_args()
+
+
+def tensor_peak():
+    """Sustained cuBLAS bf16 TFLOP/s (for a kernel timed inside a long step)."""
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["bf16_tflops_sustained"]), "measured (sustained)"
+    except Exception:
+        return 1700.0, "fallback (sustained)"
 
 
 def peaks():
@@ -72,6 +85,8 @@ KERNEL_SOURCES = {
                                 "host/plan.hpp"],
     "sq_evict_compact_kernel": ["kernels/kv.cu", "kernels/ptx.cuh", "kernels/launch.hpp",
                                 "host/plan.hpp"],
+    "sq_prefill_kernel": ["kernels/prefill.cu", "kernels/ptx.cuh", "kernels/tc.cuh",
+                          "kernels/launch.hpp", "host/plan.hpp"],
 }
 
 
@@ -805,6 +820,229 @@ def run_trace(args, world, rank, local):
     return res
 
 
+def prefill_spans(seed, n, P):
+    """Closed cursors of the prefill workload: 12 spans holding 40% of the
+    context (lognormal lengths, median 1,500), inside [P, n), shuffled."""
+    from synthetic import random_spans, shuffled, sub_seed
+    return shuffled(random_spans(sub_seed(seed, 20), 12, int(0.4 * n), P, n, median=1500), 1)
+
+
+def prefill_tile_flops(n, n_q, spans, G, Hkv, D):
+    """FLOPs the tile loop issues (every 128 x 128 tile it computes, masked
+    parts included) for one call: 4 x 128 x 128 x D per (query tile, key
+    tile) pair."""
+    import numpy as np
+    vis = np.ones(n, dtype=bool)
+    for a, b in spans:
+        vis[a:b] = False
+    n_kt = (n + 127) // 128
+    tile_has = np.array([vis[t * 128:(t + 1) * 128].any() for t in range(n_kt)])
+    key0 = np.nonzero(tile_has)[0] * 128
+    BP = 128 // G
+    n_qt = (n_q + BP - 1) // BP
+    total = 0
+    for qt in range(n_qt):
+        p_last = n - n_q + min((qt + 1) * BP, n_q) - 1
+        total += int(np.searchsorted(key0, p_last, side="right"))
+    return total * Hkv * 4 * 128 * 128 * D
+
+
+def run_prefill(args, world, rank, local):
+    """Masked prefill attention (Algorithm 2, BuildMask): one 32,768-token
+    agent context (8B-class GQA, 32 layers), 40% of it in 12 closed-cursor
+    spans that no query sees; every token is a query (a training-style
+    forward).  One step = the attention of all layers."""
+    import numpy as np
+    import torch
+
+    import paper_2602_22603_gb300 as sq
+    from synthetic import AGENT_8B, Bank, sub_seed
+    torch.cuda.set_device(local)
+    sh = AGENT_8B
+    L, Hq, Hkv, D, P = args.layers, sh.num_q_heads, sh.num_kv_heads, sh.head_dim, sh.page_size
+    G = Hq // Hkv
+    n = args.prefill_ctx
+    seed = args.seed + 1000 * rank
+    scale = 1.0 / math.sqrt(D)
+    cache = sq.Cache(L, Hq, Hkv, D, P, n // P + 64, max_seqs=4)
+    bank = Bank(1 << 28, sub_seed(seed, 1), device="cuda")
+    chunk = 2048
+    sizes = [chunk] * (n // chunk) + ([n % chunk] if n % chunk else [])
+    offs = bank.offsets(2 * len(sizes), L * chunk * Hkv * D, sub_seed(seed, 2))
+    m = cache.seq_new()
+    for i, c in enumerate(sizes):
+        cache.append_kv(m, c, bank.view(offs[2 * i], (L, c, Hkv, D)),
+                        bank.view(offs[2 * i + 1], (L, c, Hkv, D)))
+    spans = prefill_spans(seed, n, P)
+    q_offs = bank.offsets(L, n * Hq * D, sub_seed(seed, 4))
+    q_ptr = [bank.data.data_ptr() + 2 * int(o) for o in q_offs]
+    out = torch.empty(n, Hq, D, dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty(n, Hq, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    st_h = int(stream.cuda_stream)
+    torch.cuda.synchronize()
+
+    def step(evs=None):
+        for layer in range(L):
+            if evs is not None:
+                evs[2 * layer].record(stream)
+            sq.sq_prefill_attention(cache.handle, m, layer, n, q_ptr[layer], out, sq.SQ_OUT_BF16,
+                                    lse, scale, spans, st_h)
+            if evs is not None:
+                evs[2 * layer + 1].record(stream)
+
+    K, W = args.steps, args.warmup
+    for _ in range(W):
+        step()
+    torch.cuda.synchronize()
+    assert cache.sync_status() == sq.SQ_OK
+    barrier(world)
+    clocks = ClockSampler(local)
+    time.sleep(0.4)
+    st0 = cache.stats()
+    e_begin, e_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    call_evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2 * L)] for _ in range(K)]
+    e_begin.record(stream)
+    for t in range(K):
+        step(call_evs[t])
+    e_end.record(stream)
+    torch.cuda.synchronize()
+    clock_rec = clocks.stop()
+    st1 = cache.stats()
+    assert cache.sync_status() == sq.SQ_OK
+    total_ms = max_over_ranks(e_begin.elapsed_time(e_end), world)
+    call_ms = [call_evs[t][2 * l].elapsed_time(call_evs[t][2 * l + 1]) for t in range(K) for l in range(L)]
+    calls = st1["prefill_calls"] - st0["prefill_calls"]
+    pairs = (st1["prefill_pairs"] - st0["prefill_pairs"]) / calls
+    flops = 4.0 * D * Hq * pairs                       # per call, visible pairs only
+    tile_flops = prefill_tile_flops(n, n, spans, G, Hkv, D)
+    mean_call = statistics.mean(call_ms)
+    achieved = flops / (mean_call / 1e3) / 1e12
+    peak, peak_kind = tensor_peak()
+    value = world * n * K / (total_ms / 1e3)
+    ratio, ratio_src = recorded_traffic_ratio("sq_prefill_kernel")
+    kv_bytes = n * Hkv * D * 2 * 2                    # K and V of one layer
+    res = {
+        "metric": PREFILL_METRIC,
+        "value": round(value, 2),
+        "unit": "tokens/s",
+        "n_gpus": world, "steps": K, "warmup": W,
+        "ms_per_step": round(total_ms / K, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) K/V and queries from a bank; no dataset)",
+        "config": {
+            "workload": (f"prefill-32k: one {n}-token agent context, every token a query, "
+                         f"{L} layers, 32q/8kv, d128, page 64, bf16; 12 closed-cursor spans "
+                         f"({sum(b - a for a, b in spans)} tokens, 40%) masked for every query"),
+            "layers": L, "q_heads": Hq, "kv_heads": Hkv, "head_dim": D, "page_size": P,
+            "context_tokens": n, "queries": n, "sm_scale": scale,
+            "masked_tokens": int(sum(b - a for a, b in spans)), "spans": len(spans),
+            "l2": "each call reads %.2f GB of distinct K/V + %.2f GB of queries (inputs larger than L2)"
+                  % (kv_bytes / 1e9, n * Hq * D * 2 / 1e9),
+            "parallelism": "replicas" if world > 1 else "single GPU",
+        },
+        "prefill": {
+            "ms_per_call": round(mean_call, 4),
+            "ms_per_call_min": round(min(call_ms), 4),
+            "visible_pairs_per_head": int(pairs),
+            "algorithmic_tflop_per_call": round(flops / 1e12, 4),
+            "tile_tflop_per_call": round(tile_flops / 1e12, 4),
+            "tile_tflops": round(tile_flops / (mean_call / 1e3) / 1e12, 1),
+            "useful_fraction_of_tiles": round(flops / tile_flops, 4),
+        },
+        "roofline": {
+            "bound": "tensor",
+            "kernel": "sq_prefill_kernel",
+            "achieved": round(achieved, 1),
+            "peak": peak,
+            "peak_kind": peak_kind,
+            "unit": "TFLOP/s",
+            "frac": round(achieved / peak, 4),
+            "traffic": int(ratio * kv_bytes) if ratio else None,
+            "traffic_source": (ratio_src + ": DRAM bytes per byte of the layer's K/V, from the "
+                               "capture") if ratio else None,
+            "algorithmic_flops_per_launch": int(flops),
+        },
+        "gpu_launches": int(K * L),
+        "clocks": clock_rec,
+    }
+    if not args.no_e2e:
+        # through the C ABI with host buffers: each layer's queries copied in
+        # from pinned memory, its outputs and log-sum-exp copied back
+        q_h = bank.view(int(q_offs[0]), (n, Hq, D)).cpu().pin_memory()
+        q_d = torch.empty(n, Hq, D, dtype=torch.bfloat16, device="cuda")
+        out_h = torch.empty(n, Hq, D, dtype=torch.bfloat16).pin_memory()
+        lse_h = torch.empty(n, Hq, dtype=torch.float32).pin_memory()
+        Ke = min(K, 5)
+
+        def e2e_step():
+            for layer in range(L):
+                q_d.copy_(q_h, non_blocking=True)
+                cache.prefill_attention(m, layer, n, q_d, out, sq.SQ_OUT_BF16, lse, scale, spans)
+                out_h.copy_(out, non_blocking=True)
+                lse_h.copy_(lse, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize()
+        barrier(world)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        w0 = time.perf_counter()
+        e0.record(stream)
+        for _ in range(Ke):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - w0
+        e_ms = max_over_ranks(max(e0.elapsed_time(e1), wall * 1e3), world)
+        res["e2e"] = {
+            "value": round(world * n * Ke / (e_ms / 1e3), 2), "unit": "tokens/s",
+            "h2d_bytes_per_step": int(L * q_h.numel() * 2),
+            "d2h_bytes_per_step": int(L * (out_h.numel() * 2 + lse_h.numel() * 4)),
+            "steps": Ke,
+            "note": "per layer: pinned host queries in, outputs and log-sum-exp out",
+        }
+    if not args.no_cpu and rank == 0 and world == 1:
+        res["cpu_baseline"] = prefill_cpu_baseline(bank, offs, sizes, q_offs, spans, L, Hq, Hkv, D,
+                                                   n, scale)
+    cache.close()
+    return res
+
+
+def prefill_cpu_baseline(bank, offs, sizes, q_offs, spans, L, Hq, Hkv, D, n, scale):
+    """The oracle as it stands (oracle/attention.c prefill, fp64, OpenMP) on
+    the host cores: the last 48 queries of the context at 2 layers, every
+    head; tokens/s = queries / (seconds per layer x layers)."""
+    import numpy as np
+
+    from oracle import attention as oatt
+    from synthetic import bf16_bits
+    host = bf16_bits(bank.data.cpu())
+    n_sample = 48
+    layers = (0, L - 1) if L > 1 else (0,)
+    total = 0.0
+    for layer in layers:
+        ks, vs = [], []
+        for i, c in enumerate(sizes):
+            for which, dst in ((0, ks), (1, vs)):
+                o = int(offs[2 * i + which])
+                a = host[o:o + L * c * Hkv * D].reshape(L, c, Hkv, D)
+                dst.append(a[layer])
+        k = np.ascontiguousarray(np.concatenate(ks))
+        v = np.ascontiguousarray(np.concatenate(vs))
+        qo = int(q_offs[layer])
+        q = host[qo:qo + n * Hq * D].reshape(n, Hq, D)[n - n_sample:]
+        t0 = time.perf_counter()
+        oatt.prefill(np.ascontiguousarray(q), k, v, scale, spans)
+        total += time.perf_counter() - t0
+    per_layer = total / len(layers)
+    return {"value": round(n_sample / (per_layer * L), 4), "unit": "tokens/s",
+            "cores": oatt.num_threads(), "kind": "oracle", "cpu_model": cpu_model(),
+            "sample": f"the last {n_sample} queries of the {n}-token context, all {Hq} heads, at "
+                      f"{len(layers)} of {L} layers; tokens/s = queries / (seconds per layer x {L})",
+            "seconds": round(total, 3)}
+
+
 def cpu_model() -> str:
     import platform
     try:
@@ -947,6 +1185,8 @@ def main():
         res = run_agent(args, world, rank, local)
     elif args.workload == "trace":
         res = run_trace(args, world, rank, local)
+    elif args.workload == "prefill-32k":
+        res = run_prefill(args, world, rank, local)
     else:
         res = run_sq(args, world, rank, local)
     if rank == 0:

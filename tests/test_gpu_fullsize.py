@@ -137,3 +137,38 @@ def test_large_ragged_full_size():
         _decode_and_check(bp, kept, 33, scale, 9, (0, 1, 4))
     finally:
         bp.close()
+
+
+def test_prefill_32k_full_size():
+    """Masked prefill at the bench's size and launch configuration: one
+    32,768-token context, 32 layers, 32q/8kv, d128, P64, 12 spans holding 40%
+    of it masked, every token a query.  Sampled query rows (masked and
+    unmasked positions, tile edges, the first and last) of two layers, with
+    their log-sum-exp, against the oracle."""
+    L, Hq, Hkv, D, P = 32, 32, 8, 128, 64
+    n = 32768
+    bp = BankPair(L, Hq, Hkv, D, P, num_pages=n // P + 64, seed=4)
+    try:
+        m = bp.seq_new()
+        bp.fill(m, n, 2048)
+        spans = shuffled(random_spans(21, 12, int(0.4 * n), P, n, median=1500), 1)
+        scale = 1.0 / math.sqrt(D)
+        inside = spans[0][0] + 3
+        for layer in (0, 31):
+            q = bf16_normal((n, Hq, D), 400 + layer, device="cuda")
+            out = torch.empty(n, Hq, D, dtype=torch.float32, device="cuda")
+            lse = torch.empty(n, Hq, dtype=torch.float32, device="cuda")
+            bp.cache.prefill_attention(m, layer, n, q, out, sq.SQ_OUT_F32, lse, scale, spans)
+            torch.cuda.synchronize()
+            assert bp.cache.sync_status() == sq.SQ_OK
+            qb = bf16_bits(q.cpu())
+            K, V = bp.rows(m, layer)
+            for p in (0, 31, 32, 127, 128, 4095, inside, 20000, n - 129, n - 1):
+                vis = [(a, min(b, p + 1)) for a, b in spans if a < p + 1]
+                exp, exp_lse = oatt.prefill(qb[p:p + 1], K[:p + 1], V[:p + 1], scale, vis,
+                                            want_lse=True)
+                assert_close(out[p:p + 1], exp)
+                got = lse[p].cpu().numpy().astype(np.float64)
+                assert np.abs(got - exp_lse[0]).max() <= 1e-2, p
+    finally:
+        bp.close()
