@@ -127,10 +127,11 @@ int sqh_plan_decode(void* c, const int32_t* handles, int32_t n, int32_t n_ctas,
 // Plans a masked prefill over a sequence of n tokens (G = Hq / Hkv; spans as
 // start, end pairs).  info_out receives 6 int64 values: n_tiles, BP, n_qt,
 // n_split, visible_pairs, sizeof(PrefillTile).  If tiles_out is non-NULL,
-// up to `cap` tiles are written as 6 int32 each: key0, flags, vis[4].
+// up to `cap` tiles are written as 6 int32 each: key0, flags, vis[4]; if
+// qt_out is non-NULL, up to qt_cap per-query-tile tile counts.
 int sqh_plan_prefill(int32_t Hq, int32_t Hkv, int32_t n, int32_t n_q, const int32_t* spans,
                      int32_t n_spans, int32_t target_ctas, int64_t* info_out, int32_t* tiles_out,
-                     int32_t cap) {
+                     int32_t cap, int32_t* qt_out, int32_t qt_cap) {
     Geometry g;
     g.L = 1; g.Hq = Hq; g.Hkv = Hkv; g.D = 128; g.P = 64;
     g.num_pages = 1; g.max_seqs = 1; g.max_pages_per_seq = 1;
@@ -155,6 +156,10 @@ int sqh_plan_prefill(int32_t Hq, int32_t Hkv, int32_t n, int32_t n_q, const int3
             o[1] = t.flags;
             for (int w = 0; w < 4; ++w) o[2 + w] = (int32_t)t.vis[w];
         }
+    }
+    if (qt_out) {
+        const int32_t m = std::min<int32_t>(qt_cap, (int32_t)p.qt_tiles.size());
+        for (int32_t i = 0; i < m; ++i) qt_out[i] = p.qt_tiles[i];
     }
     return kOk;
 }

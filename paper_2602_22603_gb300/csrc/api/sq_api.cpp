@@ -748,15 +748,17 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
     if (rc != SQ_OK) return rc;
     cudaStream_t st = as_stream(stream);
     cudaError_t e;
-    // upload: key tiles, then the page table
+    // upload: key tiles, per-query-tile counts, then the page table
     const size_t tb = plan.tiles.size() * sizeof(PrefillTile);
+    const size_t qb = plan.qt_tiles.size() * sizeof(int32_t);
     const size_t pb = s->pages.size() * sizeof(int32_t);
-    if (c->staging.size() < tb + pb) c->staging.resize(tb + pb);
+    if (c->staging.size() < tb + qb + pb) c->staging.resize(tb + qb + pb);
     if (tb) std::memcpy(c->staging.data(), plan.tiles.data(), tb);
-    std::memcpy(c->staging.data() + tb, s->pages.data(), pb);
+    std::memcpy(c->staging.data() + tb, plan.qt_tiles.data(), qb);
+    std::memcpy(c->staging.data() + tb + qb, s->pages.data(), pb);
     UploadSlot& slot = c->slots[c->next_slot];
     c->next_slot = (c->next_slot + 1) % kUploadSlots;
-    rc = upload(c, slot, c->staging.data(), tb + pb, stream);
+    rc = upload(c, slot, c->staging.data(), tb + qb + pb, stream);
     if (rc != SQ_OK) return rc;
     const int64_t grid = (int64_t)plan.n_qt * g.Hkv * plan.n_split;
     if (plan.n_split > 1) {
@@ -796,7 +798,8 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
     }
     PrefillArgs a;
     a.tiles = reinterpret_cast<const PrefillTile*>(slot.d);
-    a.page_ids = reinterpret_cast<const int32_t*>(slot.d + tb);
+    a.qt_tiles = reinterpret_cast<const int32_t*>(slot.d + tb);
+    a.page_ids = reinterpret_cast<const int32_t*>(slot.d + tb + qb);
     a.n_tiles = (int32_t)plan.tiles.size();
     a.n_pages_seq = (int32_t)s->pages.size();
     a.n = s->n;
@@ -810,7 +813,9 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
     a.BP = plan.BP;
     a.n_qt = plan.n_qt;
     a.n_split = plan.n_split;
-    a.scale_log2 = sm_scale * 1.4426950408889634f;
+    // the kernel keeps the scale inside the exponent (s * scale - m); a zero
+    // scale runs as 1e-30, whose weights 2^(s * 1e-30 - m) are exactly 1
+    a.scale_log2 = std::max(sm_scale * 1.4426950408889634f, 1e-30f);
     a.out = out;
     a.out_f32 = out_dtype == SQ_OUT_F32;
     a.lse = lse;

@@ -593,6 +593,13 @@ int plan_prefill(const Geometry& g, int32_t n, int32_t n_q, const int32_t* start
     out->n_q = n_q;
     out->BP = kPrefillRows / g.G();
     out->n_qt = ceil_div(n_q, out->BP);
+    // each query tile reaches the key tiles up to its last query position
+    out->qt_tiles.resize(out->n_qt);
+    for (int32_t qt = 0, t = 0; qt < out->n_qt; ++qt) {
+        const int32_t p_last = q0 + std::min((qt + 1) * out->BP, n_q) - 1;
+        while (t < (int32_t)out->tiles.size() && out->tiles[t].key0 <= p_last) ++t;
+        out->qt_tiles[qt] = t;
+    }
     const int64_t units = (int64_t)out->n_qt * g.Hkv;
     const int32_t n_tiles = (int32_t)out->tiles.size();
     int32_t split = 1;

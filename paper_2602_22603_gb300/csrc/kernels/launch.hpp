@@ -47,6 +47,7 @@ cudaError_t launch_combine(const CombineArgs& a, int D, cudaStream_t st);
 // ---- masked prefill attention -------------------------------------------------
 struct PrefillArgs {
     const PrefillTile* tiles;   // key tiles with a visible key, increasing key0
+    const int32_t* qt_tiles;    // [n_qt] key tiles each query tile reaches (a prefix of tiles)
     const int32_t* page_ids;    // the sequence's page table
     int32_t n_tiles, n_pages_seq;
     int32_t n, n_q;             // sequence tokens; queries = its last n_q tokens

@@ -13,15 +13,20 @@
 // tiles whose keys are all masked are never loaded (the host lists the
 // others with a visibility bitmap).  Per key tile j:
 //   S_j = Q K_j^T            tcgen05.mma, Q and K from shared memory, S in TMEM
-//   P_j = exp2(S_j - m)       softmax warps: tcgen05.ld of S, mask, bf16 P to smem
-//   O  += P_j V_j             tcgen05.mma, V read token-major (MN-major B)
-// S is double-buffered in TMEM so that S_{j+1} is computed while the softmax
-// warps work on S_j.  The running maximum m is raised lazily: O (in TMEM) is
-// rescaled only when a row's maximum grows by more than 2^8, so the weights
-// stay below 256 and most tiles need no rescale.
+//   P_j = exp2(S_j - m)       softmax warps: tcgen05.ld of S, mask, bf16 P back
+//                             to TMEM with tcgen05.st
+//   O  += P_j V_j             tcgen05.mma with A = P read from TMEM and V read
+//                             token-major from shared memory (MN-major B)
+// S and P are double-buffered in TMEM, so S_{j+1} is computed while the
+// softmax warps work on S_j.  K and V tiles stream through one ring of
+// shared-memory slots (K_0, V_0, K_1, V_1, ...); a K slot is released as soon
+// as its S has been computed, a V slot once its PV product is done, which
+// keeps about three key tiles in flight.  The running maximum m is raised
+// lazily: O (in TMEM) is rescaled only when a row's maximum grows by more
+// than 2^8, so the weights stay below 256 and most tiles need no rescale.
 //
-// Warp roles (192 threads): warp 0 loads (TMA), lane 0 of warp 1 issues the
-// MMAs and warp 1 owns the TMEM allocation, warps 2-5 run the softmax and the
+// Warp roles (192 threads): warp 0 loads (lane 0 issues the TMA copies),
+// lane 0 of warp 1 issues the MMAs and warp 1 owns the TMEM allocation, warps 2-5 run the softmax and the
 // epilogue (warp w reads TMEM lanes 32 (w mod 4) .. +31, one row per thread).
 // Every wait is bounded; a wait that runs out sets the error word and the CTA
 // winds down after its copies and MMAs in flight have completed.
@@ -36,35 +41,38 @@ namespace {
 template <int D>
 struct PreCfg {
     static constexpr int kThreads = 192;
-    static constexpr int kColBlocks = D / 64;                 // 64-column (128-byte) blocks
-    static constexpr int kBlockBytes = kPrefillRows * 128;     // one block of a 128-row tile
+    static constexpr int kColBlocks = D / 64;                  // 64-column (128-byte) blocks
+    static constexpr int kBlockBytes = kPrefillRows * 128;      // one block of a 128-row tile
     static constexpr int kQBytes = kColBlocks * kBlockBytes;
-    static constexpr int kKVBytes = kColBlocks * kBlockBytes;  // 128 keys of K (or V)
-    static constexpr int kPBytes = 2 * kBlockBytes;            // 128 x 128 bf16 weights
-    static constexpr int kStages = D == 128 ? 2 : 3;
+    static constexpr int kSlotBytes = kColBlocks * kBlockBytes;  // 128 keys of K or of V
+    static constexpr int kSlots = D == 128 ? 6 : 12;
     static constexpr int kOffQ = 0;
-    static constexpr int kOffK = kOffQ + kQBytes;
-    static constexpr int kOffV = kOffK + kStages * kKVBytes;
-    static constexpr int kOffP = kOffV + kStages * kKVBytes;
-    static constexpr int kOffBar = kOffP + 2 * kPBytes;
+    static constexpr int kOffRing = kOffQ + kQBytes;
+    static constexpr int kOffBar = kOffRing + kSlots * kSlotBytes;
     static constexpr int kBarQ = 0;
-    static constexpr int kBarK = 1;                     // [kStages] K tile landed
-    static constexpr int kBarV = kBarK + kStages;       // [kStages] V tile ready
-    static constexpr int kBarEmpty = kBarV + kStages;   // [kStages] stage consumed by the MMAs
-    static constexpr int kBarS = kBarEmpty + kStages;   // [2] S buffer written
+    static constexpr int kBarFull = 1;                  // [kSlots] tile landed (V: and ready)
+    static constexpr int kBarEmpty = kBarFull + kSlots; // [kSlots] slot consumed by the MMAs
+    static constexpr int kBarS = kBarEmpty + kSlots;    // [2] S buffer written
     static constexpr int kBarP = kBarS + 2;             // [2] P buffer written (128 arrivals)
     static constexpr int kBarPV = kBarP + 2;            // [2] O += P V done
     static constexpr int kBarVfix = kBarPV + 2;         // V of the last key tile landed
     static constexpr int kBarDone = kBarVfix + 1;       // every MMA of the CTA done
     static constexpr int kNumBars = kBarDone + 1;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
-    static constexpr int kSmemBytes = kOffMisc + 32 + 1024;  // + alignment slack
+    // producer's table of the next kMetaTiles key tiles: first key, then the
+    // page of each of up to 16 pieces
+    static constexpr int kMetaTiles = 16;
+    static constexpr int kOffMeta = kOffMisc + 32;
+    static constexpr int kMetaBytes = kMetaTiles * 17 * 4;
+    static constexpr int kSmemBytes = kOffMeta + kMetaBytes + 1024;  // + alignment slack
     static constexpr uint32_t kTmemCols = 512;
-    static constexpr uint32_t kColS = 0;    // S_j at columns 128 (j mod 2)
-    static constexpr uint32_t kColO = 256;  // O at columns 256 .. 256 + D
+    static constexpr uint32_t kColS = 0;    // S_j (fp32) at columns 128 (j mod 2)
+    static constexpr uint32_t kColO = 256;  // O (fp32) at columns 256 .. 256 + D
+    static constexpr uint32_t kColP = 384;  // P_j (bf16 pairs) at columns 384 + 64 (j mod 2)
     static constexpr uint32_t kIdescQK = mma_idesc_bf16(128, kPrefillKeys, false);
     static constexpr uint32_t kIdescPV = mma_idesc_bf16(128, D, true);
     static_assert(kSmemBytes <= 232448, "shared memory");
+    static_assert(kColO + D <= kColP, "TMEM columns");
 };
 
 struct Smem {
@@ -81,6 +89,10 @@ __device__ __forceinline__ uint32_t low_bits_through(int x) {
     return x >= 31 ? 0xffffffffu : (x < 0 ? 0u : ((2u << x) - 1u));
 }
 
+// The producer warp: Q once, then K_j and V_j of every key tile into the ring
+// (load u = 2 j is K_j, u = 2 j + 1 is V_j, slot u mod kSlots).  Lane 0 waits
+// and issues the copies; the warp fills the table of tile keys and pages and
+// zeroes the tail rows.
 template <int D>
 __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* qmap,
                                 const PrefillArgs& a, const Smem& sm, int g, int pos_lo, int t0,
@@ -95,62 +107,85 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
                         cb * 64, g * a.G, pos_lo);
     }
     const int br = a.P < 64 ? a.P : 64;  // rows of one TMA box
-    const int n_pieces = kPrefillKeys / br;
+    const int n_pieces = kPrefillKeys / br;  // <= 16
     int issued = 0;
-    bool tail_issued = false;
-    for (int j = 0; j < T; ++j) {
-        const int s = j % C::kStages;
-        const int use = j / C::kStages;
-        if (use > 0) {
-            bool ok = mbar_wait(sm.bar<D>(C::kBarEmpty + s), (use - 1) & 1, abort_flag);
-            if (!__all_sync(0xffffffffu, ok)) {
-                if (lane == 0) {
-                    set_error(a.err, kErrTimeout);
-                    *abort_flag = 1;
-                }
-                break;
+    int tail_u = -1;          // the load that used the fix-up barrier
+    bool tail_done = false;   // ... and was handed over on its slot's barrier
+    // The first key and the pages of the next kMetaTiles tiles are read into
+    // a small shared table ahead of use (rolled loops keep this warp's code
+    // small), so that no global-memory latency sits between a free slot and
+    // the copy that refills it.
+    int32_t* meta_key0 = reinterpret_cast<int32_t*>(sm.ptr + C::kOffMeta);
+    int32_t* meta_page = meta_key0 + C::kMetaTiles;  // [kMetaTiles][16]
+    int batch = -1;
+    int key0 = 0;
+    for (int u = 0; u < 2 * T; ++u) {
+        const int j = u >> 1;
+        const bool is_v = (u & 1) != 0;
+        const int slot = u % C::kSlots;
+        const int use = u / C::kSlots;
+        if (j / C::kMetaTiles != batch) {
+            batch = j / C::kMetaTiles;
+            const int tb = batch * C::kMetaTiles;
+            if (lane < C::kMetaTiles && tb + lane < T)
+                meta_key0[lane] = __ldg(&a.tiles[t0 + tb + lane].key0);
+            __syncwarp();
+#pragma unroll 1
+            for (int idx = lane; idx < C::kMetaTiles * n_pieces; idx += 32) {
+                const int t = idx / n_pieces, i = idx - t * n_pieces;
+                if (tb + t >= T) continue;
+                const int key = meta_key0[t] + i * br;
+                meta_page[t * 16 + i] = key < a.n ? __ldg(&a.page_ids[key / a.P]) : -1;
             }
+            __syncwarp();
         }
-        const int key0 = __ldg(&a.tiles[t0 + j].key0);
-        const bool tail = key0 + kPrefillKeys > a.n;
+        bool ok = true;
+        if (use > 0 && lane == 0)
+            ok = mbar_wait(sm.bar<D>(C::kBarEmpty + slot), (use - 1) & 1, abort_flag);
+        if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) {
+            if (lane == 0) {
+                set_error(a.err, kErrTimeout);
+                *abort_flag = 1;
+            }
+            break;
+        }
+        const int mt = j % C::kMetaTiles;
+        key0 = meta_key0[mt];
+        const bool tail = is_v && key0 + kPrefillKeys > a.n;
+        const uint32_t dst = sm.base + C::kOffRing + slot * C::kSlotBytes;
         if (lane == 0) {
             // pieces that hold tokens of the sequence and a page inside the pool
             uint32_t pmask = 0;
-            for (int i = 0; i < n_pieces; ++i) {
-                const int key = key0 + i * br;
-                if (key >= a.n) break;
-                const int32_t page = __ldg(&a.page_ids[key / a.P]);
-                if ((uint32_t)page < (uint32_t)a.num_pages) pmask |= 1u << i;
+#pragma unroll 1
+            for (int i = 0; i < n_pieces && key0 + i * br < a.n; ++i) {
+                if ((uint32_t)meta_page[mt * 16 + i] < (uint32_t)a.num_pages) pmask |= 1u << i;
                 else set_error(a.err, kErrBounds);
             }
             const uint32_t bytes = (uint32_t)__popc(pmask) * br * 128 * C::kColBlocks;
-            const uint32_t kb = sm.bar<D>(C::kBarK + s);
-            const uint32_t vb = tail ? sm.bar<D>(C::kBarVfix) : sm.bar<D>(C::kBarV + s);
-            mbar_arrive_expect_tx(kb, bytes);
-            mbar_arrive_expect_tx(vb, bytes);
-            const uint32_t ks = sm.base + C::kOffK + s * C::kKVBytes;
-            const uint32_t vs = sm.base + C::kOffV + s * C::kKVBytes;
+            const uint32_t fb = tail ? sm.bar<D>(C::kBarVfix) : sm.bar<D>(C::kBarFull + slot);
+            mbar_arrive_expect_tx(fb, bytes);
+            const int head_row = (is_v ? a.Hkv + g : g) * a.P;
+#pragma unroll 1
             for (int i = 0; i < n_pieces; ++i) {
                 if (!((pmask >> i) & 1u)) continue;
                 const int key = key0 + i * br;
-                const int32_t page = __ldg(&a.page_ids[key / a.P]);
-                const int row0 = key % a.P;
-                for (int cb = 0; cb < C::kColBlocks; ++cb) {
-                    const uint32_t off = cb * C::kBlockBytes + i * br * 128;
-                    tma_load_4d(ks + off, pool_map, kb, cb * 64, g * a.P + row0, page, a.layer);
-                    tma_load_4d(vs + off, pool_map, vb, cb * 64, (a.Hkv + g) * a.P + row0, page,
-                                a.layer);
-                }
+                const int32_t page = meta_page[mt * 16 + i];
+#pragma unroll
+                for (int cb = 0; cb < C::kColBlocks; ++cb)
+                    tma_load_4d(dst + cb * C::kBlockBytes + i * br * 128, pool_map, fb, cb * 64,
+                                head_row + key % a.P, page, a.layer);
             }
         }
-        issued = j + 1;
+        __syncwarp();
+        issued = u + 1;
         if (tail) {
-            // The last key tile: its rows past the sequence's end hold stale
+            // The last key tile: its V rows past the sequence's end hold stale
             // or never-written data.  Their weights are zero, but 0 * NaN is
-            // not, so zero those V rows before the MMAs read the stage.
-            tail_issued = true;
-            bool ok = mbar_wait(sm.bar<D>(C::kBarVfix), 0, abort_flag);
-            if (!__all_sync(0xffffffffu, ok)) {
+            // not, so zero those rows before the MMAs read the slot.
+            tail_u = u;
+            ok = true;
+            if (lane == 0) ok = mbar_wait(sm.bar<D>(C::kBarVfix), 0, abort_flag);
+            if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) {
                 if (lane == 0) {
                     set_error(a.err, kErrTimeout);
                     *abort_flag = 1;
@@ -159,38 +194,37 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
             }
             const int r0 = a.n - key0;  // 1 .. 127
             const int chunks = (kPrefillKeys - r0) * 8;
-            uint8_t* vsp = sm.ptr + C::kOffV + s * C::kKVBytes;
+            uint8_t* vsp = sm.ptr + C::kOffRing + slot * C::kSlotBytes;
             for (int cb = 0; cb < C::kColBlocks; ++cb)
                 for (int c = lane; c < chunks; c += 32)
                     *reinterpret_cast<uint4*>(vsp + cb * C::kBlockBytes + (r0 + (c >> 3)) * 128 +
                                               (c & 7) * 16) = make_uint4(0, 0, 0, 0);
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) mbar_arrive(sm.bar<D>(C::kBarV + s));
+            if (lane == 0) mbar_arrive(sm.bar<D>(C::kBarFull + slot));
+            tail_done = true;
         }
     }
     // Drain: every copy this CTA issued lands before the CTA exits (immediate
     // unless a consumer gave up early).
     if (lane == 0) {
         mbar_wait(sm.bar<D>(C::kBarQ), 0);
-        for (int j = issued > C::kStages ? issued - C::kStages : 0; j < issued; ++j) {
-            const int s = j % C::kStages;
-            mbar_wait(sm.bar<D>(C::kBarK + s), (j / C::kStages) & 1);
-            const bool is_tail = tail_issued && j == issued - 1;
-            if (is_tail) mbar_wait(sm.bar<D>(C::kBarVfix), 0);
-            else mbar_wait(sm.bar<D>(C::kBarV + s), (j / C::kStages) & 1);
+        for (int u = issued > C::kSlots ? issued - C::kSlots : 0; u < issued; ++u) {
+            if (u == tail_u && !tail_done) mbar_wait(sm.bar<D>(C::kBarVfix), 0);
+            else mbar_wait(sm.bar<D>(C::kBarFull + u % C::kSlots), (u / C::kSlots) & 1);
         }
     }
 }
 
+// S_j = Q K_j^T into S buffer j mod 2; releases K_j's slot when done.
 template <int D>
 __device__ __forceinline__ bool issue_qk(const Smem& sm, uint32_t tmem, int j,
                                          volatile int* abort_flag) {
     using C = PreCfg<D>;
-    const int s = j % C::kStages;
-    if (!mbar_wait(sm.bar<D>(C::kBarK + s), (j / C::kStages) & 1, abort_flag)) return false;
+    const int u = 2 * j, slot = u % C::kSlots;
+    if (!mbar_wait(sm.bar<D>(C::kBarFull + slot), (u / C::kSlots) & 1, abort_flag)) return false;
     const uint32_t qa = sm.base + C::kOffQ;
-    const uint32_t ka = sm.base + C::kOffK + s * C::kKVBytes;
+    const uint32_t ka = sm.base + C::kOffRing + slot * C::kSlotBytes;
     const uint32_t dt = tmem + C::kColS + (uint32_t)(j & 1) * kPrefillKeys;
 #pragma unroll
     for (int ks = 0; ks < D / 16; ++ks) {
@@ -199,6 +233,7 @@ __device__ __forceinline__ bool issue_qk(const Smem& sm, uint32_t tmem, int j,
                     C::kIdescQK, ks > 0);
     }
     mma_commit(sm.bar<D>(C::kBarS + (j & 1)));
+    mma_commit(sm.bar<D>(C::kBarEmpty + slot));
     return true;
 }
 
@@ -213,22 +248,22 @@ __device__ void prefill_mma(const PrefillArgs& a, const Smem& sm, uint32_t tmem,
         ok = issue_qk<D>(sm, tmem, 0, abort_flag);
         any = ok;
         for (int j = 0; ok && j < T; ++j) {
-            const int s = j % C::kStages;
+            // S buffer (j + 1) mod 2 last held S_{j-1}, read before P_{j-1} was signalled
             if (j + 1 < T && !(ok = issue_qk<D>(sm, tmem, j + 1, abort_flag))) break;
             if (!(ok = mbar_wait(sm.bar<D>(C::kBarP + (j & 1)), (j >> 1) & 1, abort_flag))) break;
             tc_fence_after();
-            if (!(ok = mbar_wait(sm.bar<D>(C::kBarV + s), (j / C::kStages) & 1, abort_flag))) break;
-            const uint32_t pa = sm.base + C::kOffP + (j & 1) * C::kPBytes;
-            const uint32_t va = sm.base + C::kOffV + s * C::kKVBytes;
+            const int u = 2 * j + 1, slot = u % C::kSlots;
+            if (!(ok = mbar_wait(sm.bar<D>(C::kBarFull + slot), (u / C::kSlots) & 1, abort_flag)))
+                break;
+            const uint32_t pa = tmem + C::kColP + (uint32_t)(j & 1) * (kPrefillKeys / 2);
+            const uint32_t va = sm.base + C::kOffRing + slot * C::kSlotBytes;
 #pragma unroll
-            for (int ks = 0; ks < kPrefillKeys / 16; ++ks) {
-                const uint32_t aoff = (ks >> 2) * C::kBlockBytes + (ks & 3) * 32;
-                mma_bf16_ss(tmem + C::kColO, smem_desc_sw128(pa + aoff, 16, 1024),
-                            smem_desc_sw128(va + ks * 16 * 128, C::kBlockBytes, 1024),
-                            C::kIdescPV, (j > 0 || ks > 0) ? 1u : 0u);
-            }
+            for (int ks = 0; ks < kPrefillKeys / 16; ++ks)
+                mma_bf16_ts(tmem + C::kColO, pa + ks * 8,
+                            smem_desc_sw128(va + ks * 16 * 128, C::kBlockBytes, 1024), C::kIdescPV,
+                            (j > 0 || ks > 0) ? 1u : 0u);
             mma_commit(sm.bar<D>(C::kBarPV + (j & 1)));
-            mma_commit(sm.bar<D>(C::kBarEmpty + s));
+            mma_commit(sm.bar<D>(C::kBarEmpty + slot));
         }
     }
     if (!ok) {
@@ -242,10 +277,21 @@ __device__ void prefill_mma(const PrefillArgs& a, const Smem& sm, uint32_t tmem,
     }
 }
 
+// One lane of the warp polls the barrier; the others wait at the shuffle.
+// Returns the warp-uniform result.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, const volatile int* abort,
+                                          int lane) {
+    bool ok = true;
+    if (lane == 0) ok = mbar_wait(bar, parity, abort);
+    ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+    __syncwarp();
+    return ok;
+}
+
 template <int D>
-__device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t tmem, int rest,
-                                int g, int pos_lo, int t0, int T, volatile int* abort_flag,
-                                int warp, int lane) {
+__device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t tmem, int g,
+                                int pos_lo, int t0, int T, volatile int* abort_flag, int warp,
+                                int lane) {
     using C = PreCfg<D>;
     const int wq = warp & 3;
     const int row = wq * 32 + lane;
@@ -253,18 +299,29 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
     const bool valid = row < a.BP * a.G && qi < a.n_q;
     const int p_row = a.n - a.n_q + qi;
     const uint32_t tl = tmem + ((uint32_t)(wq * 32) << 16);
-    const float sc = a.scale_log2;
+    const float sc = a.scale_log2;  // > 0 (the host raises a zero scale to a tiny one)
     float m_run = -INFINITY, l = 0.f;
     bool ok = true;
+    int4 n0 = make_int4(0, 0, 0, 0), n1 = n0;
+    if (T > 0) {
+        const int4* tp = reinterpret_cast<const int4*>(a.tiles + t0);
+        n0 = __ldg(tp);
+        n1 = __ldg(tp + 1);
+    }
     for (int j = 0; j < T; ++j) {
-        const int4* tp = reinterpret_cast<const int4*>(a.tiles + t0 + j);
-        const int4 w0 = __ldg(tp), w1 = __ldg(tp + 1);
+        // this tile's record; the next one is fetched while this tile is worked on
+        const int4 w0 = n0, w1 = n1;
+        if (j + 1 < T) {
+            const int4* tp = reinterpret_cast<const int4*>(a.tiles + t0 + j + 1);
+            n0 = __ldg(tp);
+            n1 = __ldg(tp + 1);
+        }
         const int key0 = w0.x;
         const uint32_t vis[4] = {(uint32_t)w0.z, (uint32_t)w0.w, (uint32_t)w1.x, (uint32_t)w1.y};
-        ok = __all_sync(0xffffffffu,
-                        mbar_wait(sm.bar<D>(C::kBarS + (j & 1)), (j >> 1) & 1, abort_flag));
+        ok = warp_wait(sm.bar<D>(C::kBarS + (j & 1)), (j >> 1) & 1, abort_flag, lane);
         if (!ok) break;
         tc_fence_after();
+        // raw logits q.k (the scale is applied inside the exponent; it is > 0)
         float x[kPrefillKeys];
         {
             uint32_t u[kPrefillKeys];
@@ -274,7 +331,7 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
                           *reinterpret_cast<uint32_t(*)[32]>(&u[c * 32]));
             tmem_wait_ld();
 #pragma unroll
-            for (int c = 0; c < kPrefillKeys; ++c) x[c] = __uint_as_float(u[c]) * sc;
+            for (int c = 0; c < kPrefillKeys; ++c) x[c] = __uint_as_float(u[c]);
         }
         const int lim = p_row - key0;  // keys key0 + c with c <= lim are causal
         if (!(valid && (w0.y & kPrefillTileFull) && lim >= kPrefillKeys - 1)) {
@@ -286,9 +343,14 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
                     if (!((mw >> c) & 1u)) x[32 * w + c] = -INFINITY;
             }
         }
-        float mt = x[0];
+        // row maximum: eight independent chains, then a tree
+        float mx[8];
 #pragma unroll
-        for (int c = 1; c < kPrefillKeys; ++c) mt = fmaxf(mt, x[c]);
+        for (int c = 0; c < 8; ++c) mx[c] = x[c];
+#pragma unroll
+        for (int c = 8; c < kPrefillKeys; ++c) mx[c & 7] = fmaxf(mx[c & 7], x[c]);
+        const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) * sc;
         const bool need = mt > m_run + 8.f;
         float alpha = 1.f;
         if (need) {
@@ -298,8 +360,8 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
         }
         if (j > 0 && __any_sync(0xffffffffu, need)) {
             // O holds P_{j-1} V_{j-1} once that MMA is done: rescale it in place
-            ok = __all_sync(0xffffffffu, mbar_wait(sm.bar<D>(C::kBarPV + ((j - 1) & 1)),
-                                                   ((j - 1) >> 1) & 1, abort_flag));
+            ok = warp_wait(sm.bar<D>(C::kBarPV + ((j - 1) & 1)), ((j - 1) >> 1) & 1, abort_flag,
+                           lane);
             if (!ok) break;
             tc_fence_after();
 #pragma unroll
@@ -315,33 +377,39 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
         }
         if (j >= 2) {
             // P buffer (j mod 2) was last read by the MMAs of tile j - 2
-            ok = __all_sync(0xffffffffu, mbar_wait(sm.bar<D>(C::kBarPV + (j & 1)),
-                                                   ((j - 2) >> 1) & 1, abort_flag));
+            ok = warp_wait(sm.bar<D>(C::kBarPV + (j & 1)), ((j - 2) >> 1) & 1, abort_flag, lane);
             if (!ok) break;
+            tc_fence_after();
         }
-        const float mu = m_run == -INFINITY ? 0.f : m_run;
-        uint8_t* prow = sm.ptr + C::kOffP + (j & 1) * C::kPBytes + row * 128;
+        // weights 2^(s * scale - m), rounded to bf16 and stored to TMEM as the A
+        // operand of the value product; the normaliser sums the same rounded
+        // weights (eight chains), so the output is a weighted mean of V rows
+        // with weights summing to one
+        const float nmu = m_run == -INFINITY ? 0.f : -m_run;
+        float ls[8];
 #pragma unroll
-        for (int k = 0; k < kPrefillKeys / 8; ++k) {
-            uint32_t w[4];
+        for (int c = 0; c < 8; ++c) ls[c] = 0.f;
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const __nv_bfloat162 h =
-                    __floats2bfloat162_rn(exp2f(x[8 * k + 2 * e] - mu), exp2f(x[8 * k + 2 * e + 1] - mu));
-                w[e] = *reinterpret_cast<const uint32_t*>(&h);
-                l += __uint_as_float(w[e] << 16) + __uint_as_float(w[e] & 0xffff0000u);
+        for (int h = 0; h < 2; ++h) {
+            uint32_t w[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                const int c = 64 * h + 2 * i;
+                const __nv_bfloat162 hb = __floats2bfloat162_rn(exp2f(fmaf(x[c], sc, nmu)),
+                                                                exp2f(fmaf(x[c + 1], sc, nmu)));
+                w[i] = *reinterpret_cast<const uint32_t*>(&hb);
+                ls[(2 * i) & 7] += __uint_as_float(w[i] << 16);
+                ls[(2 * i + 1) & 7] += __uint_as_float(w[i] & 0xffff0000u);
             }
-            const int cb = k >> 3, ch = (k & 7) ^ (row & 7);
-            *reinterpret_cast<uint4*>(prow + cb * C::kBlockBytes + ch * 16) =
-                make_uint4(w[0], w[1], w[2], w[3]);
+            tmem_st32(tl + C::kColP + (uint32_t)(j & 1) * (kPrefillKeys / 2) + 32 * h, w);
         }
-        fence_proxy_async_smem();
+        l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
+        tmem_wait_st();
         tc_fence_before();
         mbar_arrive(sm.bar<D>(C::kBarP + (j & 1)));
     }
     if (ok && T > 0)
-        ok = __all_sync(0xffffffffu, mbar_wait(sm.bar<D>(C::kBarPV + ((T - 1) & 1)),
-                                               ((T - 1) >> 1) & 1, abort_flag));
+        ok = warp_wait(sm.bar<D>(C::kBarPV + ((T - 1) & 1)), ((T - 1) >> 1) & 1, abort_flag, lane);
     if (!ok) {
         if (lane == 0) {
             set_error(a.err, kErrTimeout);
@@ -397,7 +465,6 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
             }
         }
     }
-    (void)rest;
 }
 
 template <int D>
@@ -420,12 +487,10 @@ __global__ void __launch_bounds__(192, 1)
     const int g = rest % a.Hkv;
     const int qt = a.n_qt - 1 - rest / a.Hkv;
     const int pos_lo = qt * a.BP;
-    const int q_pos = min(a.BP, a.n_q - pos_lo);
     if (threadIdx.x == 0) {
         mbar_init(sm.bar<D>(C::kBarQ), 1);
-        for (int s = 0; s < C::kStages; ++s) {
-            mbar_init(sm.bar<D>(C::kBarK + s), 1);
-            mbar_init(sm.bar<D>(C::kBarV + s), 1);
+        for (int s = 0; s < C::kSlots; ++s) {
+            mbar_init(sm.bar<D>(C::kBarFull + s), 1);
             mbar_init(sm.bar<D>(C::kBarEmpty + s), 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -438,13 +503,7 @@ __global__ void __launch_bounds__(192, 1)
         fence_mbar_init();
         *abort_flag = 0;
         // key tiles up to the last query position, split evenly
-        const int p_last = a.n - a.n_q + pos_lo + q_pos - 1;
-        int lo = 0, hi = a.n_tiles;
-        while (lo < hi) {
-            const int mid = (lo + hi) >> 1;
-            if (__ldg(&a.tiles[mid].key0) <= p_last) lo = mid + 1;
-            else hi = mid;
-        }
+        const int lo = __ldg(&a.qt_tiles[qt]);
         const int t0 = (int)((int64_t)lo * split / a.n_split);
         sched[0] = t0;
         sched[1] = (int)((int64_t)lo * (split + 1) / a.n_split) - t0;
@@ -464,7 +523,7 @@ __global__ void __launch_bounds__(192, 1)
         if (lane == 0) prefill_mma<D>(a, sm, tmem, T, abort_flag);
         __syncwarp();
     } else {
-        prefill_softmax<D>(a, sm, tmem, rest, g, pos_lo, t0, T, abort_flag, warp, lane);
+        prefill_softmax<D>(a, sm, tmem, g, pos_lo, t0, T, abort_flag, warp, lane);
     }
     tc_fence_before();
     __syncthreads();

@@ -305,6 +305,11 @@ def test_prefill_plan_visibility_matches_brute_force(seed):
     assert info["visible_pairs"] == exp_pairs
     assert info["BP"] == 128 // G
     assert info["n_qt"] == -(-n_q // (128 // G))
+    # each query tile reaches the listed tiles up to its last query position
+    BP = 128 // G
+    for qt, cnt in enumerate(info["qt_tiles"]):
+        p_last = n - n_q + min((qt + 1) * BP, n_q) - 1
+        assert cnt == sum(1 for t in exp_tiles if t[0] <= p_last), qt
     units = info["n_qt"] * Hkv
     assert info["n_split"] >= 1
     if units >= 152:
