@@ -830,7 +830,8 @@ def prefill_spans(seed, n, P):
 def prefill_tile_flops(n, n_q, spans, G, Hkv, D):
     """FLOPs the tile loop issues (every 128 x 128 tile it computes, masked
     parts included) for one call: 4 x 128 x 128 x D per (query tile, key
-    tile) pair."""
+    tile) pair; a CTA's two query tiles both run over the key tiles its
+    later tile reaches."""
     import numpy as np
     vis = np.ones(n, dtype=bool)
     for a, b in spans:
@@ -838,12 +839,12 @@ def prefill_tile_flops(n, n_q, spans, G, Hkv, D):
     n_kt = (n + 127) // 128
     tile_has = np.array([vis[t * 128:(t + 1) * 128].any() for t in range(n_kt)])
     key0 = np.nonzero(tile_has)[0] * 128
-    BP = 128 // G
-    n_qt = (n_q + BP - 1) // BP
+    span = 2 * (128 // G)
+    n_qt = (n_q + span - 1) // span
     total = 0
     for qt in range(n_qt):
-        p_last = n - n_q + min((qt + 1) * BP, n_q) - 1
-        total += int(np.searchsorted(key0, p_last, side="right"))
+        p_last = n - n_q + min((qt + 1) * span, n_q) - 1
+        total += 2 * int(np.searchsorted(key0, p_last, side="right"))
     return total * Hkv * 4 * 128 * 128 * D
 
 

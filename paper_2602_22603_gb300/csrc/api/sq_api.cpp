@@ -762,7 +762,8 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
     if (rc != SQ_OK) return rc;
     const int64_t grid = (int64_t)plan.n_qt * g.Hkv * plan.n_split;
     if (plan.n_split > 1) {
-        const size_t need = (size_t)grid * kPrefillRows * (g.D + 1) * sizeof(float);
+        const size_t need =
+            (size_t)grid * kPrefillQTiles * kPrefillRows * (g.D + 1) * sizeof(float);
         if (!c->pre_ev) {
             e = cudaEventCreateWithFlags(&c->pre_ev, cudaEventDisableTiming);
             if (e != cudaSuccess) return cuda_status(e);
@@ -820,7 +821,9 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
     a.out_f32 = out_dtype == SQ_OUT_F32;
     a.lse = lse;
     a.part_o = c->pre_part;
-    a.part_ml = c->pre_part ? c->pre_part + (size_t)grid * kPrefillRows * g.D : nullptr;
+    a.part_ml = c->pre_part
+                    ? c->pre_part + (size_t)grid * kPrefillQTiles * kPrefillRows * g.D
+                    : nullptr;
     a.err = c->d_err;
     e = launch_prefill(c->tmap, qmap, a, g.D, st);
     if (e != cudaSuccess) return cuda_status(e);

@@ -592,11 +592,12 @@ int plan_prefill(const Geometry& g, int32_t n, int32_t n_q, const int32_t* start
     out->n = n;
     out->n_q = n_q;
     out->BP = kPrefillRows / g.G();
-    out->n_qt = ceil_div(n_q, out->BP);
-    // each query tile reaches the key tiles up to its last query position
+    const int32_t span = out->BP * kPrefillQTiles;  // query positions per CTA
+    out->n_qt = ceil_div(n_q, span);
+    // each CTA tile reaches the key tiles up to its last query position
     out->qt_tiles.resize(out->n_qt);
     for (int32_t qt = 0, t = 0; qt < out->n_qt; ++qt) {
-        const int32_t p_last = q0 + std::min((qt + 1) * out->BP, n_q) - 1;
+        const int32_t p_last = q0 + std::min((qt + 1) * span, n_q) - 1;
         while (t < (int32_t)out->tiles.size() && out->tiles[t].key0 <= p_last) ++t;
         out->qt_tiles[qt] = t;
     }

@@ -179,10 +179,10 @@ void plan_serialize(const DecodePlanHost& p, const DecodePlanLayout& lay,
 
 struct PrefillPlanHost {
     std::vector<PrefillTile> tiles;   // key tiles with a visible key, increasing key0
-    std::vector<int32_t> qt_tiles;    // per query tile: tiles with key0 <= its last position
+    std::vector<int32_t> qt_tiles;    // per CTA tile: key tiles with key0 <= its last position
     int32_t n = 0, n_q = 0;
-    int32_t BP = 0;                   // query positions per tile
-    int32_t n_qt = 0;                 // query tiles per KV head
+    int32_t BP = 0;                   // query positions per query tile
+    int32_t n_qt = 0;                 // CTA tiles (kPrefillQTiles query tiles each) per KV head
     int32_t n_split = 1;              // key-range splits per query tile
     int64_t visible_pairs = 0;        // sum over queries of the keys each sees
 };

@@ -67,6 +67,8 @@ struct EvictPiece {
 // Keys are taken kPrefillKeys at a time, aligned to kPrefillKeys.
 constexpr int kPrefillRows = 128;
 constexpr int kPrefillKeys = 128;
+// Query tiles one CTA owns; they share every K/V tile it loads.
+constexpr int kPrefillQTiles = 2;
 constexpr int32_t kPrefillTileFull = 1;  // every key of the tile exists and is visible
 
 // One key tile that holds at least one visible key of the sequence.

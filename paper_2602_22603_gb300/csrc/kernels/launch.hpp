@@ -47,19 +47,20 @@ cudaError_t launch_combine(const CombineArgs& a, int D, cudaStream_t st);
 // ---- masked prefill attention -------------------------------------------------
 struct PrefillArgs {
     const PrefillTile* tiles;   // key tiles with a visible key, increasing key0
-    const int32_t* qt_tiles;    // [n_qt] key tiles each query tile reaches (a prefix of tiles)
+    const int32_t* qt_tiles;    // [n_qt] key tiles each CTA tile reaches (a prefix of tiles)
     const int32_t* page_ids;    // the sequence's page table
     int32_t n_tiles, n_pages_seq;
     int32_t n, n_q;             // sequence tokens; queries = its last n_q tokens
     int32_t layer, Hq, Hkv, G, P, num_pages;
-    int32_t BP;                 // query positions per tile (kPrefillRows / G)
+    int32_t BP;                 // query positions per query tile (kPrefillRows / G)
     int32_t n_qt, n_split;
     float scale_log2;           // sm_scale * log2(e), >= 0
     void* out;                  // [n_q][Hq][D] bf16 or fp32 (n_split == 1)
     int32_t out_f32;
     float* lse;                 // [n_q][Hq] or null (n_split == 1)
-    float* part_o;              // [grid][kPrefillRows][D] normalised partials (n_split > 1)
-    float* part_ml;             // [grid][kPrefillRows] log2-sum-exp of each partial
+    float* part_o;              // [grid][kPrefillQTiles][kPrefillRows][D] normalised partials
+                                // (n_split > 1)
+    float* part_ml;             // [grid][kPrefillQTiles][kPrefillRows] their log2-sum-exp
     int* err;
 };
 

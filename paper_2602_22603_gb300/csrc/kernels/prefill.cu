@@ -7,29 +7,34 @@
 //     s_j = sm_scale * q_h . k_{g,j}   for visible keys j (j <= p, j in no span)
 //     o_h = sum_j softmax_j(s) v_{g,j}
 //
-// One CTA owns a tile of 128 query rows: floor(128 / G) consecutive query
-// positions times the G query heads of one KV head (Sec. 2.1), so every K/V
-// tile it loads serves all of them.  Keys go 128 at a time, aligned to 128;
-// tiles whose keys are all masked are never loaded (the host lists the
-// others with a visibility bitmap).  Per key tile j:
-//   S_j = Q K_j^T            tcgen05.mma, Q and K from shared memory, S in TMEM
-//   P_j = exp2(S_j - m)       softmax warps: tcgen05.ld of S, mask, bf16 P back
-//                             to TMEM with tcgen05.st
-//   O  += P_j V_j             tcgen05.mma with A = P read from TMEM and V read
+// A query tile is 128 rows: floor(128 / G) consecutive query positions times
+// the G query heads of one KV head (Sec. 2.1).  One CTA owns two consecutive
+// query tiles (a, b) of the same KV head, and every K/V tile it loads serves
+// both, which halves the loads per tensor-core FLOP.  Keys go 128 at a time,
+// aligned to 128; tiles whose keys are all masked are never loaded (the host
+// lists the others with a visibility bitmap).  Per key tile j and query tile t:
+//   S_t = Q_t K_j^T           tcgen05.mma, Q and K from shared memory, S in TMEM
+//   P_t = exp2(S_t - m)       softmax warpgroup t: tcgen05.ld of S, mask, bf16 P
+//                             stored back over the first half of S_t
+//   O_t += P_t V_j            tcgen05.mma with A = P from TMEM and V read
 //                             token-major from shared memory (MN-major B)
-// S and P are double-buffered in TMEM, so S_{j+1} is computed while the
-// softmax warps work on S_j.  K and V tiles stream through one ring of
-// shared-memory slots (K_0, V_0, K_1, V_1, ...); a K slot is released as soon
-// as its S has been computed, a V slot once its PV product is done, which
-// keeps about three key tiles in flight.  The running maximum m is raised
-// lazily: O (in TMEM) is rescaled only when a row's maximum grows by more
-// than 2^8, so the weights stay below 256 and most tiles need no rescale.
+// The MMA issuer interleaves the two tiles (PV_a(j), S_a(j+1), PV_b(j),
+// S_b(j+1)), so while one warpgroup turns S into P the tensor core works for
+// the other.  P_t(j) shares TMEM with S_t: S_t(j+1) is issued after PV_t(j),
+// and tcgen05.mma operations of one thread execute in issue order.  The same
+// order means that when S_t(j) is ready, PV_t(j-1) is complete, so a
+// warpgroup may rescale O_t then without another wait.  The running maximum
+// is raised lazily: O is rescaled only when a row's maximum grows by more than
+// 2^8, so the weights stay below 256.  K and V stream through one ring of
+// shared-memory slots (K_0, V_0, K_1, ...); a K slot is released once both S
+// products are done, a V slot once both PV products are.
 //
-// Warp roles (192 threads): warp 0 loads (lane 0 issues the TMA copies),
-// lane 0 of warp 1 issues the MMAs and warp 1 owns the TMEM allocation, warps 2-5 run the softmax and the
-// epilogue (warp w reads TMEM lanes 32 (w mod 4) .. +31, one row per thread).
-// Every wait is bounded; a wait that runs out sets the error word and the CTA
-// winds down after its copies and MMAs in flight have completed.
+// Warp roles (320 threads): warp 0 loads (lane 0 issues the TMA copies), lane
+// 0 of warp 1 issues the MMAs and warp 1 owns the TMEM allocation, warps 2-5
+// are the softmax warpgroup of tile a and warps 6-9 that of tile b (warp w
+// reads TMEM lanes 32 (w mod 4) .. +31, one row per thread).  Every wait is
+// bounded; a wait that runs out sets the error word and the CTA winds down
+// after its copies and MMAs in flight have completed.
 #include "launch.hpp"
 #include "ptx.cuh"
 #include "tc.cuh"
@@ -40,22 +45,22 @@ namespace {
 
 template <int D>
 struct PreCfg {
-    static constexpr int kThreads = 192;
+    static constexpr int kThreads = 320;
     static constexpr int kColBlocks = D / 64;                  // 64-column (128-byte) blocks
     static constexpr int kBlockBytes = kPrefillRows * 128;      // one block of a 128-row tile
-    static constexpr int kQBytes = kColBlocks * kBlockBytes;
+    static constexpr int kQBytes = kColBlocks * kBlockBytes;    // one query tile
     static constexpr int kSlotBytes = kColBlocks * kBlockBytes;  // 128 keys of K or of V
-    static constexpr int kSlots = D == 128 ? 6 : 12;
+    static constexpr int kSlots = D == 128 ? 5 : 12;
     static constexpr int kOffQ = 0;
-    static constexpr int kOffRing = kOffQ + kQBytes;
+    static constexpr int kOffRing = kOffQ + kPrefillQTiles * kQBytes;
     static constexpr int kOffBar = kOffRing + kSlots * kSlotBytes;
     static constexpr int kBarQ = 0;
     static constexpr int kBarFull = 1;                  // [kSlots] tile landed (V: and ready)
     static constexpr int kBarEmpty = kBarFull + kSlots; // [kSlots] slot consumed by the MMAs
-    static constexpr int kBarS = kBarEmpty + kSlots;    // [2] S buffer written
-    static constexpr int kBarP = kBarS + 2;             // [2] P buffer written (128 arrivals)
-    static constexpr int kBarPV = kBarP + 2;            // [2] O += P V done
-    static constexpr int kBarVfix = kBarPV + 2;         // V of the last key tile landed
+    static constexpr int kBarS = kBarEmpty + kSlots;    // [2] S_t written (and PV_t before it done)
+    static constexpr int kBarP = kBarS + 2;             // [2] P_t written (128 arrivals)
+    static constexpr int kBarO = kBarP + 2;             // [2] last PV_t done
+    static constexpr int kBarVfix = kBarO + 2;          // V of the last key tile landed
     static constexpr int kBarDone = kBarVfix + 1;       // every MMA of the CTA done
     static constexpr int kNumBars = kBarDone + 1;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
@@ -66,13 +71,12 @@ struct PreCfg {
     static constexpr int kMetaBytes = kMetaTiles * 17 * 4;
     static constexpr int kSmemBytes = kOffMeta + kMetaBytes + 1024;  // + alignment slack
     static constexpr uint32_t kTmemCols = 512;
-    static constexpr uint32_t kColS = 0;    // S_j (fp32) at columns 128 (j mod 2)
-    static constexpr uint32_t kColO = 256;  // O (fp32) at columns 256 .. 256 + D
-    static constexpr uint32_t kColP = 384;  // P_j (bf16 pairs) at columns 384 + 64 (j mod 2)
+    static constexpr uint32_t kColS = 0;    // S_t (fp32) at 128 t; P_t (bf16 pairs) over its first 64
+    static constexpr uint32_t kColO = 256;  // O_t (fp32) at 256 + 128 t
     static constexpr uint32_t kIdescQK = mma_idesc_bf16(128, kPrefillKeys, false);
     static constexpr uint32_t kIdescPV = mma_idesc_bf16(128, D, true);
     static_assert(kSmemBytes <= 232448, "shared memory");
-    static_assert(kColO + D <= kColP, "TMEM columns");
+    static_assert(kPrefillQTiles == 2, "two query tiles per CTA");
 };
 
 struct Smem {
@@ -89,10 +93,10 @@ __device__ __forceinline__ uint32_t low_bits_through(int x) {
     return x >= 31 ? 0xffffffffu : (x < 0 ? 0u : ((2u << x) - 1u));
 }
 
-// The producer warp: Q once, then K_j and V_j of every key tile into the ring
-// (load u = 2 j is K_j, u = 2 j + 1 is V_j, slot u mod kSlots).  Lane 0 waits
-// and issues the copies; the warp fills the table of tile keys and pages and
-// zeroes the tail rows.
+// The producer warp: both query tiles once, then K_j and V_j of every key tile
+// into the ring (load u = 2 j is K_j, u = 2 j + 1 is V_j, slot u mod kSlots).
+// Lane 0 waits and issues the copies; the warp fills the table of tile keys
+// and pages and zeroes the tail rows.
 template <int D>
 __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* qmap,
                                 const PrefillArgs& a, const Smem& sm, int g, int pos_lo, int t0,
@@ -101,10 +105,12 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
     if (lane == 0) {
         prefetch_tmap(pool_map);
         prefetch_tmap(qmap);
-        mbar_arrive_expect_tx(sm.bar<D>(C::kBarQ), C::kColBlocks * a.BP * a.G * 128);
-        for (int cb = 0; cb < C::kColBlocks; ++cb)
-            tma_load_3d(sm.base + C::kOffQ + cb * C::kBlockBytes, qmap, sm.bar<D>(C::kBarQ),
-                        cb * 64, g * a.G, pos_lo);
+        mbar_arrive_expect_tx(sm.bar<D>(C::kBarQ),
+                              kPrefillQTiles * C::kColBlocks * a.BP * a.G * 128);
+        for (int t = 0; t < kPrefillQTiles; ++t)
+            for (int cb = 0; cb < C::kColBlocks; ++cb)
+                tma_load_3d(sm.base + C::kOffQ + t * C::kQBytes + cb * C::kBlockBytes, qmap,
+                            sm.bar<D>(C::kBarQ), cb * 64, g * a.G, pos_lo + t * a.BP);
     }
     const int br = a.P < 64 ? a.P : 64;  // rows of one TMA box
     const int n_pieces = kPrefillKeys / br;  // <= 16
@@ -216,25 +222,33 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
     }
 }
 
-// S_j = Q K_j^T into S buffer j mod 2; releases K_j's slot when done.
+// S_t = Q_t K^T for the K tile in `slot`, into TMEM columns 128 t.
 template <int D>
-__device__ __forceinline__ bool issue_qk(const Smem& sm, uint32_t tmem, int j,
-                                         volatile int* abort_flag) {
+__device__ __forceinline__ void issue_qk(const Smem& sm, uint32_t tmem, int t, int slot) {
     using C = PreCfg<D>;
-    const int u = 2 * j, slot = u % C::kSlots;
-    if (!mbar_wait(sm.bar<D>(C::kBarFull + slot), (u / C::kSlots) & 1, abort_flag)) return false;
-    const uint32_t qa = sm.base + C::kOffQ;
+    const uint32_t qa = sm.base + C::kOffQ + t * C::kQBytes;
     const uint32_t ka = sm.base + C::kOffRing + slot * C::kSlotBytes;
-    const uint32_t dt = tmem + C::kColS + (uint32_t)(j & 1) * kPrefillKeys;
+    const uint32_t dt = tmem + C::kColS + (uint32_t)t * kPrefillKeys;
 #pragma unroll
     for (int ks = 0; ks < D / 16; ++ks) {
         const uint32_t off = (ks >> 2) * C::kBlockBytes + (ks & 3) * 32;
         mma_bf16_ss(dt, smem_desc_sw128(qa + off, 16, 1024), smem_desc_sw128(ka + off, 16, 1024),
                     C::kIdescQK, ks > 0);
     }
-    mma_commit(sm.bar<D>(C::kBarS + (j & 1)));
-    mma_commit(sm.bar<D>(C::kBarEmpty + slot));
-    return true;
+}
+
+// O_t += P_t V for the V tile in `slot`; P_t from TMEM over the first half of S_t.
+template <int D>
+__device__ __forceinline__ void issue_pv(const Smem& sm, uint32_t tmem, int t, int slot,
+                                         bool first) {
+    using C = PreCfg<D>;
+    const uint32_t pa = tmem + C::kColS + (uint32_t)t * kPrefillKeys;
+    const uint32_t va = sm.base + C::kOffRing + slot * C::kSlotBytes;
+#pragma unroll
+    for (int ks = 0; ks < kPrefillKeys / 16; ++ks)
+        mma_bf16_ts(tmem + C::kColO + (uint32_t)t * 128, pa + ks * 8,
+                    smem_desc_sw128(va + ks * 16 * 128, C::kBlockBytes, 1024), C::kIdescPV,
+                    (!first || ks > 0) ? 1u : 0u);
 }
 
 template <int D>
@@ -245,25 +259,45 @@ __device__ void prefill_mma(const PrefillArgs& a, const Smem& sm, uint32_t tmem,
     bool any = false;
     if (ok && T > 0) {
         tc_fence_after();
-        ok = issue_qk<D>(sm, tmem, 0, abort_flag);
-        any = ok;
+        const int k0 = 0;
+        ok = mbar_wait(sm.bar<D>(C::kBarFull + k0), 0, abort_flag);
+        if (ok) {
+            any = true;
+            issue_qk<D>(sm, tmem, 0, k0);
+            mma_commit(sm.bar<D>(C::kBarS + 0));
+            issue_qk<D>(sm, tmem, 1, k0);
+            mma_commit(sm.bar<D>(C::kBarS + 1));
+            mma_commit(sm.bar<D>(C::kBarEmpty + k0));
+        }
         for (int j = 0; ok && j < T; ++j) {
-            // S buffer (j + 1) mod 2 last held S_{j-1}, read before P_{j-1} was signalled
-            if (j + 1 < T && !(ok = issue_qk<D>(sm, tmem, j + 1, abort_flag))) break;
-            if (!(ok = mbar_wait(sm.bar<D>(C::kBarP + (j & 1)), (j >> 1) & 1, abort_flag))) break;
+            const int uv = 2 * j + 1, vslot = uv % C::kSlots;
+            const int uk = 2 * j + 2, kslot = uk % C::kSlots;
+            const bool more = j + 1 < T;
+            // tile a: O_a += P_a V_j, then S_a for the next key tile
+            if (!(ok = mbar_wait(sm.bar<D>(C::kBarP + 0), j & 1, abort_flag))) break;
             tc_fence_after();
-            const int u = 2 * j + 1, slot = u % C::kSlots;
-            if (!(ok = mbar_wait(sm.bar<D>(C::kBarFull + slot), (u / C::kSlots) & 1, abort_flag)))
+            if (!(ok = mbar_wait(sm.bar<D>(C::kBarFull + vslot), (uv / C::kSlots) & 1, abort_flag)))
                 break;
-            const uint32_t pa = tmem + C::kColP + (uint32_t)(j & 1) * (kPrefillKeys / 2);
-            const uint32_t va = sm.base + C::kOffRing + slot * C::kSlotBytes;
-#pragma unroll
-            for (int ks = 0; ks < kPrefillKeys / 16; ++ks)
-                mma_bf16_ts(tmem + C::kColO, pa + ks * 8,
-                            smem_desc_sw128(va + ks * 16 * 128, C::kBlockBytes, 1024), C::kIdescPV,
-                            (j > 0 || ks > 0) ? 1u : 0u);
-            mma_commit(sm.bar<D>(C::kBarPV + (j & 1)));
-            mma_commit(sm.bar<D>(C::kBarEmpty + slot));
+            issue_pv<D>(sm, tmem, 0, vslot, j == 0);
+            if (!more) mma_commit(sm.bar<D>(C::kBarO + 0));
+            if (more) {
+                if (!(ok = mbar_wait(sm.bar<D>(C::kBarFull + kslot), (uk / C::kSlots) & 1,
+                                     abort_flag)))
+                    break;
+                issue_qk<D>(sm, tmem, 0, kslot);
+                mma_commit(sm.bar<D>(C::kBarS + 0));
+            }
+            // tile b
+            if (!(ok = mbar_wait(sm.bar<D>(C::kBarP + 1), j & 1, abort_flag))) break;
+            tc_fence_after();
+            issue_pv<D>(sm, tmem, 1, vslot, j == 0);
+            mma_commit(sm.bar<D>(C::kBarEmpty + vslot));
+            if (!more) mma_commit(sm.bar<D>(C::kBarO + 1));
+            if (more) {
+                issue_qk<D>(sm, tmem, 1, kslot);
+                mma_commit(sm.bar<D>(C::kBarS + 1));
+                mma_commit(sm.bar<D>(C::kBarEmpty + kslot));
+            }
         }
     }
     if (!ok) {
@@ -288,17 +322,20 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, const v
     return ok;
 }
 
+// Softmax warpgroup of query tile t (one row per thread) and its epilogue.
 template <int D>
-__device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t tmem, int g,
+__device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t tmem, int t, int g,
                                 int pos_lo, int t0, int T, volatile int* abort_flag, int warp,
                                 int lane) {
     using C = PreCfg<D>;
     const int wq = warp & 3;
     const int row = wq * 32 + lane;
-    const int qi = pos_lo + row / a.G;
+    const int qi = pos_lo + t * a.BP + row / a.G;
     const bool valid = row < a.BP * a.G && qi < a.n_q;
     const int p_row = a.n - a.n_q + qi;
     const uint32_t tl = tmem + ((uint32_t)(wq * 32) << 16);
+    const uint32_t col_s = C::kColS + (uint32_t)t * kPrefillKeys;
+    const uint32_t col_o = C::kColO + (uint32_t)t * 128;
     const float sc = a.scale_log2;  // > 0 (the host raises a zero scale to a tiny one)
     float m_run = -INFINITY, l = 0.f;
     bool ok = true;
@@ -318,37 +355,36 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
         }
         const int key0 = w0.x;
         const uint32_t vis[4] = {(uint32_t)w0.z, (uint32_t)w0.w, (uint32_t)w1.x, (uint32_t)w1.y};
-        ok = warp_wait(sm.bar<D>(C::kBarS + (j & 1)), (j >> 1) & 1, abort_flag, lane);
+        ok = warp_wait(sm.bar<D>(C::kBarS + t), j & 1, abort_flag, lane);
         if (!ok) break;
         tc_fence_after();
-        // raw logits q.k (the scale is applied inside the exponent; it is > 0)
-        float x[kPrefillKeys];
-        {
-            uint32_t u[kPrefillKeys];
-#pragma unroll
-            for (int c = 0; c < kPrefillKeys / 32; ++c)
-                tmem_ld32(tl + C::kColS + (uint32_t)(j & 1) * kPrefillKeys + c * 32,
-                          *reinterpret_cast<uint32_t(*)[32]>(&u[c * 32]));
-            tmem_wait_ld();
-#pragma unroll
-            for (int c = 0; c < kPrefillKeys; ++c) x[c] = __uint_as_float(u[c]);
-        }
+        // Raw logits q.k (the scale is applied inside the exponent; it is > 0),
+        // taken 64 columns at a time to keep registers low: one pass for the
+        // row maximum, one for the weights.
         const int lim = p_row - key0;  // keys key0 + c with c <= lim are causal
-        if (!(valid && (w0.y & kPrefillTileFull) && lim >= kPrefillKeys - 1)) {
-#pragma unroll
-            for (int w = 0; w < 4; ++w) {
-                const uint32_t mw = valid ? (vis[w] & low_bits_through(lim - 32 * w)) : 0u;
-#pragma unroll
-                for (int c = 0; c < 32; ++c)
-                    if (!((mw >> c) & 1u)) x[32 * w + c] = -INFINITY;
-            }
-        }
-        // row maximum: eight independent chains, then a tree
+        const bool unmasked = valid && (w0.y & kPrefillTileFull) && lim >= kPrefillKeys - 1;
         float mx[8];
 #pragma unroll
-        for (int c = 0; c < 8; ++c) mx[c] = x[c];
+        for (int c = 0; c < 8; ++c) mx[c] = -INFINITY;
 #pragma unroll
-        for (int c = 8; c < kPrefillKeys; ++c) mx[c & 7] = fmaxf(mx[c & 7], x[c]);
+        for (int hh = 0; hh < 2; ++hh) {
+            uint32_t x[64];
+            tmem_ld32(tl + col_s + 64 * hh, *reinterpret_cast<uint32_t(*)[32]>(&x[0]));
+            tmem_ld32(tl + col_s + 64 * hh + 32, *reinterpret_cast<uint32_t(*)[32]>(&x[32]));
+            tmem_wait_ld();
+            if (!unmasked) {
+#pragma unroll
+                for (int w = 0; w < 2; ++w) {
+                    const int ww = 2 * hh + w;
+                    const uint32_t mw = valid ? (vis[ww] & low_bits_through(lim - 32 * ww)) : 0u;
+#pragma unroll
+                    for (int c = 0; c < 32; ++c)
+                        if (!((mw >> c) & 1u)) x[32 * w + c] = 0xff800000u;  // -inf
+                }
+            }
+#pragma unroll
+            for (int c = 0; c < 64; ++c) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(x[c]));
+        }
         const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
                                fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) * sc;
         const bool need = mt > m_run + 8.f;
@@ -359,57 +395,61 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
             l *= alpha;
         }
         if (j > 0 && __any_sync(0xffffffffu, need)) {
-            // O holds P_{j-1} V_{j-1} once that MMA is done: rescale it in place
-            ok = warp_wait(sm.bar<D>(C::kBarPV + ((j - 1) & 1)), ((j - 1) >> 1) & 1, abort_flag,
-                           lane);
-            if (!ok) break;
-            tc_fence_after();
+            // O_t holds the products up to key tile j - 1 (complete: S_t(j) was
+            // issued after them): rescale it in place
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
                 uint32_t o[32];
-                tmem_ld32(tl + C::kColO + c * 32, o);
+                tmem_ld32(tl + col_o + c * 32, o);
                 tmem_wait_ld();
 #pragma unroll
                 for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-                tmem_st32(tl + C::kColO + c * 32, o);
+                tmem_st32(tl + col_o + c * 32, o);
             }
-            tmem_wait_st();
         }
-        if (j >= 2) {
-            // P buffer (j mod 2) was last read by the MMAs of tile j - 2
-            ok = warp_wait(sm.bar<D>(C::kBarPV + (j & 1)), ((j - 2) >> 1) & 1, abort_flag, lane);
-            if (!ok) break;
-            tc_fence_after();
-        }
-        // weights 2^(s * scale - m), rounded to bf16 and stored to TMEM as the A
-        // operand of the value product; the normaliser sums the same rounded
-        // weights (eight chains), so the output is a weighted mean of V rows
-        // with weights summing to one
+        // weights 2^(s * scale - m), rounded to bf16 and stored to TMEM over the
+        // first half of S_t as the A operand of the value product (half hh of
+        // the keys goes to columns 32 hh .. +31, after that half of S was read);
+        // the normaliser sums the same rounded weights (eight chains), so the
+        // output is a weighted mean of V rows with weights summing to one
         const float nmu = m_run == -INFINITY ? 0.f : -m_run;
         float ls[8];
 #pragma unroll
         for (int c = 0; c < 8; ++c) ls[c] = 0.f;
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
+        for (int hh = 0; hh < 2; ++hh) {
+            uint32_t x[64];
+            tmem_ld32(tl + col_s + 64 * hh, *reinterpret_cast<uint32_t(*)[32]>(&x[0]));
+            tmem_ld32(tl + col_s + 64 * hh + 32, *reinterpret_cast<uint32_t(*)[32]>(&x[32]));
+            tmem_wait_ld();
+            if (!unmasked) {
+#pragma unroll
+                for (int w = 0; w < 2; ++w) {
+                    const int ww = 2 * hh + w;
+                    const uint32_t mw = valid ? (vis[ww] & low_bits_through(lim - 32 * ww)) : 0u;
+#pragma unroll
+                    for (int c = 0; c < 32; ++c)
+                        if (!((mw >> c) & 1u)) x[32 * w + c] = 0xff800000u;  // -inf
+                }
+            }
             uint32_t w[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-                const int c = 64 * h + 2 * i;
-                const __nv_bfloat162 hb = __floats2bfloat162_rn(exp2f(fmaf(x[c], sc, nmu)),
-                                                                exp2f(fmaf(x[c + 1], sc, nmu)));
+                const __nv_bfloat162 hb =
+                    __floats2bfloat162_rn(exp2f(fmaf(__uint_as_float(x[2 * i]), sc, nmu)),
+                                          exp2f(fmaf(__uint_as_float(x[2 * i + 1]), sc, nmu)));
                 w[i] = *reinterpret_cast<const uint32_t*>(&hb);
                 ls[(2 * i) & 7] += __uint_as_float(w[i] << 16);
                 ls[(2 * i + 1) & 7] += __uint_as_float(w[i] & 0xffff0000u);
             }
-            tmem_st32(tl + C::kColP + (uint32_t)(j & 1) * (kPrefillKeys / 2) + 32 * h, w);
+            tmem_st32(tl + col_s + 32 * hh, w);
         }
         l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
         tmem_wait_st();
         tc_fence_before();
-        mbar_arrive(sm.bar<D>(C::kBarP + (j & 1)));
+        mbar_arrive(sm.bar<D>(C::kBarP + t));
     }
-    if (ok && T > 0)
-        ok = warp_wait(sm.bar<D>(C::kBarPV + ((T - 1) & 1)), ((T - 1) >> 1) & 1, abort_flag, lane);
+    if (ok && T > 0) ok = warp_wait(sm.bar<D>(C::kBarO + t), 0, abort_flag, lane);
     if (!ok) {
         if (lane == 0) {
             set_error(a.err, kErrTimeout);
@@ -424,8 +464,9 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
     float* part_row = nullptr;
     uint8_t* out_row = nullptr;
     if (a.n_split > 1) {
-        part_row = a.part_o + ((size_t)blockIdx.x * kPrefillRows + row) * D;
-        if (valid) a.part_ml[(size_t)blockIdx.x * kPrefillRows + row] = lse2;
+        const size_t pr = ((size_t)blockIdx.x * kPrefillQTiles + t) * kPrefillRows + row;
+        part_row = a.part_o + pr * D;
+        if (valid) a.part_ml[pr] = lse2;
     } else {
         out_row = reinterpret_cast<uint8_t*>(a.out) +
                   ((size_t)qi * a.Hq + h) * D * (a.out_f32 ? 4 : 2);
@@ -435,7 +476,7 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
     for (int c = 0; c < D / 32; ++c) {
         uint32_t o[32];
         if (T > 0) {
-            tmem_ld32(tl + C::kColO + c * 32, o);
+            tmem_ld32(tl + col_o + c * 32, o);
             tmem_wait_ld();
         } else {
 #pragma unroll
@@ -468,7 +509,7 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
 }
 
 template <int D>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(320, 1)
     sq_prefill_kernel(const __grid_constant__ CUtensorMap pool_map,
                       const __grid_constant__ CUtensorMap qmap, const PrefillArgs a) {
     using C = PreCfg<D>;
@@ -481,12 +522,12 @@ __global__ void __launch_bounds__(192, 1)
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sm.ptr + C::kOffMisc + 4);
     int* sched = reinterpret_cast<int*>(sm.ptr + C::kOffMisc + 8);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // heaviest query tiles (latest positions) first
+    // heaviest CTA tiles (latest positions) first
     const int split = blockIdx.x % a.n_split;
     const int rest = blockIdx.x / a.n_split;
     const int g = rest % a.Hkv;
     const int qt = a.n_qt - 1 - rest / a.Hkv;
-    const int pos_lo = qt * a.BP;
+    const int pos_lo = qt * kPrefillQTiles * a.BP;
     if (threadIdx.x == 0) {
         mbar_init(sm.bar<D>(C::kBarQ), 1);
         for (int s = 0; s < C::kSlots; ++s) {
@@ -496,13 +537,13 @@ __global__ void __launch_bounds__(192, 1)
         for (int b = 0; b < 2; ++b) {
             mbar_init(sm.bar<D>(C::kBarS + b), 1);
             mbar_init(sm.bar<D>(C::kBarP + b), 128);
-            mbar_init(sm.bar<D>(C::kBarPV + b), 1);
+            mbar_init(sm.bar<D>(C::kBarO + b), 1);
         }
         mbar_init(sm.bar<D>(C::kBarVfix), 1);
         mbar_init(sm.bar<D>(C::kBarDone), 1);
         fence_mbar_init();
         *abort_flag = 0;
-        // key tiles up to the last query position, split evenly
+        // key tiles up to the CTA tile's last query position, split evenly
         const int lo = __ldg(&a.qt_tiles[qt]);
         const int t0 = (int)((int64_t)lo * split / a.n_split);
         sched[0] = t0;
@@ -523,7 +564,7 @@ __global__ void __launch_bounds__(192, 1)
         if (lane == 0) prefill_mma<D>(a, sm, tmem, T, abort_flag);
         __syncwarp();
     } else {
-        prefill_softmax<D>(a, sm, tmem, g, pos_lo, t0, T, abort_flag, warp, lane);
+        prefill_softmax<D>(a, sm, tmem, (warp - 2) >> 2, g, pos_lo, t0, T, abort_flag, warp, lane);
     }
     tc_fence_before();
     __syncthreads();
@@ -534,26 +575,31 @@ __global__ void __launch_bounds__(192, 1)
 }
 
 // Merges the key-range splits of each query row: weights 2^(lse_s - max).
+// One warp per (CTA tile, query tile, row).
 template <int D>
 __global__ void __launch_bounds__(256) sq_prefill_combine_kernel(const PrefillCombineArgs a) {
     const int gw = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
     const int lane = threadIdx.x & 31;
     const int units = a.n_qt * a.Hkv;
-    if (gw >= units * kPrefillRows) return;
-    const int rest = gw / kPrefillRows, row = gw % kPrefillRows;
+    constexpr int kRowsPerUnit = kPrefillQTiles * kPrefillRows;
+    if (gw >= units * kRowsPerUnit) return;
+    const int rest = gw / kRowsPerUnit, tr = gw % kRowsPerUnit;
+    const int t = tr / kPrefillRows, row = tr % kPrefillRows;
     const int g = rest % a.Hkv, qt = a.n_qt - 1 - rest / a.Hkv;
-    const int qi = qt * a.BP + row / a.G;
+    const int qi = (qt * kPrefillQTiles + t) * a.BP + row / a.G;
     if (row >= a.BP * a.G || qi >= a.n_q) return;
     const int h = g * a.G + row % a.G;
+    auto part = [&](int s) {
+        return (((size_t)rest * a.n_split + s) * kPrefillQTiles + t) * kPrefillRows + row;
+    };
     float M = -INFINITY;
-    for (int s = 0; s < a.n_split; ++s)
-        M = fmaxf(M, a.part_ml[((size_t)rest * a.n_split + s) * kPrefillRows + row]);
+    for (int s = 0; s < a.n_split; ++s) M = fmaxf(M, a.part_ml[part(s)]);
     float W = 0.f, acc[D / 32];
 #pragma unroll
     for (int e = 0; e < D / 32; ++e) acc[e] = 0.f;
     if (M != -INFINITY) {
         for (int s = 0; s < a.n_split; ++s) {
-            const size_t pr = ((size_t)rest * a.n_split + s) * kPrefillRows + row;
+            const size_t pr = part(s);
             const float ml = a.part_ml[pr];
             if (ml == -INFINITY) continue;
             const float w = exp2f(ml - M);
@@ -606,7 +652,7 @@ cudaError_t launch_prefill(const CUtensorMap& pool_map, const CUtensorMap& qmap,
 }
 
 cudaError_t launch_prefill_combine(const PrefillCombineArgs& a, int D, cudaStream_t st) {
-    const int64_t warps = (int64_t)a.n_qt * a.Hkv * kPrefillRows;
+    const int64_t warps = (int64_t)a.n_qt * a.Hkv * kPrefillQTiles * kPrefillRows;
     const unsigned grid = (unsigned)((warps * 32 + 255) / 256);
     if (grid == 0) return cudaSuccess;
     if (D == 128) dev::sq_prefill_combine_kernel<128><<<grid, 256, 0, st>>>(a);

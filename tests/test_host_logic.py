@@ -304,11 +304,11 @@ def test_prefill_plan_visibility_matches_brute_force(seed):
         assert got[0] == key0 and got[1] == full and list(got[2:]) == words
     assert info["visible_pairs"] == exp_pairs
     assert info["BP"] == 128 // G
-    assert info["n_qt"] == -(-n_q // (128 // G))
-    # each query tile reaches the listed tiles up to its last query position
-    BP = 128 // G
+    span = 2 * (128 // G)          # two query tiles per CTA
+    assert info["n_qt"] == -(-n_q // span)
+    # each CTA tile reaches the listed tiles up to its last query position
     for qt, cnt in enumerate(info["qt_tiles"]):
-        p_last = n - n_q + min((qt + 1) * BP, n_q) - 1
+        p_last = n - n_q + min((qt + 1) * span, n_q) - 1
         assert cnt == sum(1 for t in exp_tiles if t[0] <= p_last), qt
     units = info["n_qt"] * Hkv
     assert info["n_split"] >= 1
@@ -337,4 +337,4 @@ def test_prefill_plan_splits_short_query_blocks():
     rc, info, _ = plan_prefill(32, 8, 131072, 8, [])
     assert rc == 0 and info["n_qt"] == 1 and info["n_split"] == 19
     rc, info, _ = plan_prefill(32, 8, 32768, 32768, [(100, 5000)])
-    assert rc == 0 and info["n_split"] == 1 and info["n_qt"] == 1024
+    assert rc == 0 and info["n_split"] == 1 and info["n_qt"] == 512
