@@ -744,18 +744,19 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
         sb[i] = spans[i].end;
     }
     PrefillPlanHost plan;
-    int rc = plan_prefill(g, s->n, n_q, sa.data(), sb.data(), n_spans, c->num_sms, &plan);
+    int rc = plan_prefill(g, s->n, n_q, sa.data(), sb.data(), n_spans, c->num_sms, &plan,
+                          s->pages.data());
     if (rc != SQ_OK) return rc;
     cudaStream_t st = as_stream(stream);
     cudaError_t e;
-    // upload: key tiles, per-query-tile counts, then the page table
+    // upload: key tiles, per-CTA-tile counts, then the page of every piece
     const size_t tb = plan.tiles.size() * sizeof(PrefillTile);
     const size_t qb = plan.qt_tiles.size() * sizeof(int32_t);
-    const size_t pb = s->pages.size() * sizeof(int32_t);
+    const size_t pb = plan.tile_pages.size() * sizeof(int32_t);
     if (c->staging.size() < tb + qb + pb) c->staging.resize(tb + qb + pb);
     if (tb) std::memcpy(c->staging.data(), plan.tiles.data(), tb);
     std::memcpy(c->staging.data() + tb, plan.qt_tiles.data(), qb);
-    std::memcpy(c->staging.data() + tb + qb, s->pages.data(), pb);
+    if (pb) std::memcpy(c->staging.data() + tb + qb, plan.tile_pages.data(), pb);
     UploadSlot& slot = c->slots[c->next_slot];
     c->next_slot = (c->next_slot + 1) % kUploadSlots;
     rc = upload(c, slot, c->staging.data(), tb + qb + pb, stream);
@@ -800,9 +801,9 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
     PrefillArgs a;
     a.tiles = reinterpret_cast<const PrefillTile*>(slot.d);
     a.qt_tiles = reinterpret_cast<const int32_t*>(slot.d + tb);
-    a.page_ids = reinterpret_cast<const int32_t*>(slot.d + tb + qb);
+    a.tile_pages = reinterpret_cast<const int32_t*>(slot.d + tb + qb);
+    a.n_pieces = plan.n_pieces;
     a.n_tiles = (int32_t)plan.tiles.size();
-    a.n_pages_seq = (int32_t)s->pages.size();
     a.n = s->n;
     a.n_q = n_q;
     a.layer = layer;

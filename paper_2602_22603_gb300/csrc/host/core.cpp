@@ -554,7 +554,7 @@ void plan_serialize(const DecodePlanHost& p, const DecodePlanLayout& L, uint8_t*
 // plan carries the span part as one bit per key, per key tile.
 int plan_prefill(const Geometry& g, int32_t n, int32_t n_q, const int32_t* starts,
                  const int32_t* ends, int32_t n_spans, int32_t target_ctas,
-                 PrefillPlanHost* out) {
+                 PrefillPlanHost* out, const int32_t* pages) {
     *out = PrefillPlanHost();
     if (n < 1 || n_q < 1 || n_q > n) return kInvalidArg;
     std::vector<std::pair<int32_t, int32_t>> sp;
@@ -580,6 +580,17 @@ int plan_prefill(const Geometry& g, int32_t n, int32_t n_q, const int32_t* start
         if (!any) continue;
         tile.flags = full ? kPrefillTileFull : 0;
         out->tiles.push_back(tile);
+    }
+    // the page of each TMA box (min(P, 64) rows) of each listed tile
+    const int32_t br = std::min(g.P, 64);
+    out->n_pieces = kPrefillKeys / br;
+    if (pages) {
+        out->tile_pages.resize(out->tiles.size() * out->n_pieces);
+        for (size_t t = 0; t < out->tiles.size(); ++t)
+            for (int32_t i = 0; i < out->n_pieces; ++i) {
+                const int32_t key = out->tiles[t].key0 + i * br;
+                out->tile_pages[t * out->n_pieces + i] = key < n ? pages[key / g.P] : -1;
+            }
     }
     // visible keys of each query: the visible keys among 0 .. p
     int64_t seen = 0, pairs = 0;

@@ -180,6 +180,8 @@ void plan_serialize(const DecodePlanHost& p, const DecodePlanLayout& lay,
 struct PrefillPlanHost {
     std::vector<PrefillTile> tiles;   // key tiles with a visible key, increasing key0
     std::vector<int32_t> qt_tiles;    // per CTA tile: key tiles with key0 <= its last position
+    int32_t n_pieces = 0;             // TMA boxes (min(P, 64) rows) per key tile
+    std::vector<int32_t> tile_pages;  // [tiles][n_pieces] page of each piece, -1 past the end
     int32_t n = 0, n_q = 0;
     int32_t BP = 0;                   // query positions per query tile
     int32_t n_qt = 0;                 // CTA tiles (kPrefillQTiles query tiles each) per KV head
@@ -191,8 +193,10 @@ struct PrefillPlanHost {
 // tokens are the queries: validates the spans, builds the per-tile visibility
 // bitmaps, and splits each query tile's key range in n_split parts when the
 // query tiles alone would fill fewer than `target_ctas` CTAs.
+// `pages` (may be null) is the sequence's page table; with it the plan also
+// lists the page of every piece of every key tile.
 int plan_prefill(const Geometry& g, int32_t n, int32_t n_q, const int32_t* starts,
                  const int32_t* ends, int32_t n_spans, int32_t target_ctas,
-                 PrefillPlanHost* out);
+                 PrefillPlanHost* out, const int32_t* pages = nullptr);
 
 }  // namespace sq

@@ -48,8 +48,8 @@ cudaError_t launch_combine(const CombineArgs& a, int D, cudaStream_t st);
 struct PrefillArgs {
     const PrefillTile* tiles;   // key tiles with a visible key, increasing key0
     const int32_t* qt_tiles;    // [n_qt] key tiles each CTA tile reaches (a prefix of tiles)
-    const int32_t* page_ids;    // the sequence's page table
-    int32_t n_tiles, n_pages_seq;
+    const int32_t* tile_pages;  // [n_tiles][n_pieces] page of each min(P, 64)-row piece, -1 past the end
+    int32_t n_tiles, n_pieces;
     int32_t n, n_q;             // sequence tokens; queries = its last n_q tokens
     int32_t layer, Hq, Hkv, G, P, num_pages;
     int32_t BP;                 // query positions per query tile (kPrefillRows / G)

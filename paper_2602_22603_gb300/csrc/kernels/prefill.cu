@@ -139,9 +139,8 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
 #pragma unroll 1
             for (int idx = lane; idx < C::kMetaTiles * n_pieces; idx += 32) {
                 const int t = idx / n_pieces, i = idx - t * n_pieces;
-                if (tb + t >= T) continue;
-                const int key = meta_key0[t] + i * br;
-                meta_page[t * 16 + i] = key < a.n ? __ldg(&a.page_ids[key / a.P]) : -1;
+                if (tb + t < T)
+                    meta_page[t * 16 + i] = __ldg(&a.tile_pages[(size_t)(t0 + tb + t) * n_pieces + i]);
             }
             __syncwarp();
         }
@@ -311,6 +310,31 @@ __device__ void prefill_mma(const PrefillArgs& a, const Smem& sm, uint32_t tmem,
     }
 }
 
+// Packed fp32 pair helpers (sm_100 family): d = a * b + c on two lanes at once.
+__device__ __forceinline__ uint64_t f2pack(float lo, float hi) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+__device__ __forceinline__ void f2unpack(uint64_t v, float& lo, float& hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
 // One lane of the warp polls the barrier; the others wait at the shuffle.
 // Returns the warp-uniform result.
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, const volatile int* abort,
@@ -363,9 +387,10 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
         // row maximum, one for the weights.
         const int lim = p_row - key0;  // keys key0 + c with c <= lim are causal
         const bool unmasked = valid && (w0.y & kPrefillTileFull) && lim >= kPrefillKeys - 1;
-        float mx[8];
+        // row maximum: three-input max over four independent chains
+        float mx[4];
 #pragma unroll
-        for (int c = 0; c < 8; ++c) mx[c] = -INFINITY;
+        for (int c = 0; c < 4; ++c) mx[c] = -INFINITY;
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
             uint32_t x[64];
@@ -383,10 +408,14 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
                 }
             }
 #pragma unroll
-            for (int c = 0; c < 64; ++c) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(x[c]));
+            for (int c = 0; c < 64; c += 8) {
+                mx[0] = fmax3(mx[0], __uint_as_float(x[c]), __uint_as_float(x[c + 1]));
+                mx[1] = fmax3(mx[1], __uint_as_float(x[c + 2]), __uint_as_float(x[c + 3]));
+                mx[2] = fmax3(mx[2], __uint_as_float(x[c + 4]), __uint_as_float(x[c + 5]));
+                mx[3] = fmax3(mx[3], __uint_as_float(x[c + 6]), __uint_as_float(x[c + 7]));
+            }
         }
-        const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) * sc;
+        const float mt = fmaxf(fmax3(mx[0], mx[1], mx[2]), mx[3]) * sc;
         const bool need = mt > m_run + 8.f;
         float alpha = 1.f;
         if (need) {
@@ -407,15 +436,17 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
                 tmem_st32(tl + col_o + c * 32, o);
             }
         }
-        // weights 2^(s * scale - m), rounded to bf16 and stored to TMEM over the
-        // first half of S_t as the A operand of the value product (half hh of
-        // the keys goes to columns 32 hh .. +31, after that half of S was read);
-        // the normaliser sums the same rounded weights (eight chains), so the
-        // output is a weighted mean of V rows with weights summing to one
+        // weights 2^(s * scale - m) (arguments two at a time with a packed
+        // FMA), rounded to bf16 and stored to TMEM over the first half of S_t
+        // as the A operand of the value product (half hh of the keys goes to
+        // columns 32 hh .. +31, after that half of S was read); the normaliser
+        // sums the fp32 weights (four packed chains)
+        const uint64_t sc2 = f2pack(sc, sc);
         const float nmu = m_run == -INFINITY ? 0.f : -m_run;
-        float ls[8];
+        const uint64_t nmu2 = f2pack(nmu, nmu);
+        uint64_t ls2[4];
 #pragma unroll
-        for (int c = 0; c < 8; ++c) ls[c] = 0.f;
+        for (int c = 0; c < 4; ++c) ls2[c] = 0;
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
             uint32_t x[64];
@@ -435,16 +466,25 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
             uint32_t w[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-                const __nv_bfloat162 hb =
-                    __floats2bfloat162_rn(exp2f(fmaf(__uint_as_float(x[2 * i]), sc, nmu)),
-                                          exp2f(fmaf(__uint_as_float(x[2 * i + 1]), sc, nmu)));
+                float a0, a1;
+                f2unpack(ffma2(f2pack(__uint_as_float(x[2 * i]), __uint_as_float(x[2 * i + 1])),
+                               sc2, nmu2),
+                         a0, a1);
+                const float p0 = exp2f(a0), p1 = exp2f(a1);
+                ls2[i & 3] = fadd2(ls2[i & 3], f2pack(p0, p1));
+                const __nv_bfloat162 hb = __floats2bfloat162_rn(p0, p1);
                 w[i] = *reinterpret_cast<const uint32_t*>(&hb);
-                ls[(2 * i) & 7] += __uint_as_float(w[i] << 16);
-                ls[(2 * i + 1) & 7] += __uint_as_float(w[i] & 0xffff0000u);
             }
             tmem_st32(tl + col_s + 32 * hh, w);
         }
-        l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
+        {
+            float s0, s1, s2, s3, s4, s5, s6, s7;
+            f2unpack(ls2[0], s0, s1);
+            f2unpack(ls2[1], s2, s3);
+            f2unpack(ls2[2], s4, s5);
+            f2unpack(ls2[3], s6, s7);
+            l += ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
+        }
         tmem_wait_st();
         tc_fence_before();
         mbar_arrive(sm.bar<D>(C::kBarP + t));
