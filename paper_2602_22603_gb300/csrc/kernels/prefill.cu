@@ -64,11 +64,10 @@ struct PreCfg {
     static constexpr int kBarDone = kBarVfix + 1;       // every MMA of the CTA done
     static constexpr int kNumBars = kBarDone + 1;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
-    // producer's table of the next kMetaTiles key tiles: first key, then the
-    // page of each of up to 16 pieces
+    // producer's double-buffered table of key-tile records (int4 each)
     static constexpr int kMetaTiles = 16;
-    static constexpr int kOffMeta = kOffMisc + 32;
-    static constexpr int kMetaBytes = kMetaTiles * 17 * 4;
+    static constexpr int kOffMeta = (kOffMisc + 32 + 15) & ~15;  // int4 records: 16-byte aligned
+    static constexpr int kMetaBytes = 2 * kMetaTiles * 16;
     static constexpr int kSmemBytes = kOffMeta + kMetaBytes + 1024;  // + alignment slack
     static constexpr uint32_t kTmemCols = 512;
     static constexpr uint32_t kColS = 0;    // S_t (fp32) at 128 t; P_t (bf16 pairs) over its first 64
@@ -76,6 +75,7 @@ struct PreCfg {
     static constexpr uint32_t kIdescQK = mma_idesc_bf16(128, kPrefillKeys, false);
     static constexpr uint32_t kIdescPV = mma_idesc_bf16(128, D, true);
     static_assert(kSmemBytes <= 232448, "shared memory");
+    static_assert(kOffMeta % 16 == 0 && kOffRing % 1024 == 0 && kOffBar % 8 == 0, "alignment");
     static_assert(kPrefillQTiles == 2, "two query tiles per CTA");
 };
 
@@ -95,8 +95,13 @@ __device__ __forceinline__ uint32_t low_bits_through(int x) {
 
 // The producer warp: both query tiles once, then K_j and V_j of every key tile
 // into the ring (load u = 2 j is K_j, u = 2 j + 1 is V_j, slot u mod kSlots).
-// Lane 0 waits and issues the copies; the warp fills the table of tile keys
-// and pages and zeroes the tail rows.
+// The warp writes, for the key tiles of the next batch, a record of what the
+// copies need {first key, box mask, page of box 0, page of box 1} into a
+// double-buffered shared table half a batch ahead; lane 0 reads the record of
+// its next tile while the current one is in flight, so that between a free
+// slot and the copies that refill it there is only the barrier.  Boxes past
+// the second (pages of fewer than 64 tokens) take their page from global
+// memory.
 template <int D>
 __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* qmap,
                                 const PrefillArgs& a, const Smem& sm, int g, int pos_lo, int t0,
@@ -113,82 +118,93 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
                             sm.bar<D>(C::kBarQ), cb * 64, g * a.G, pos_lo + t * a.BP);
     }
     const int br = a.P < 64 ? a.P : 64;  // rows of one TMA box
-    const int n_pieces = kPrefillKeys / br;  // <= 16
+    const int n_pieces = a.n_pieces;      // <= 16
+    int4* table = reinterpret_cast<int4*>(sm.ptr + C::kOffMeta);  // [2][kMetaTiles]
+    // records of tiles [tb, tb + kMetaTiles) into table half `half`
+    auto fill = [&](int tb, int half) {
+        if (lane < C::kMetaTiles && tb + lane < T) {
+            const int t = t0 + tb + lane;
+            const int key0 = __ldg(&a.tiles[t].key0);
+            uint32_t pmask = 0;
+            int p0 = -1, p1 = -1;
+            for (int i = 0; i < n_pieces && key0 + i * br < a.n; ++i) {
+                const int32_t page = __ldg(&a.tile_pages[(size_t)t * n_pieces + i]);
+                if ((uint32_t)page < (uint32_t)a.num_pages) pmask |= 1u << i;
+                else set_error(a.err, kErrBounds);
+                if (i == 0) p0 = page;
+                if (i == 1) p1 = page;
+            }
+            table[half * C::kMetaTiles + lane] = make_int4(key0, (int)pmask, p0, p1);
+        }
+    };
+    fill(0, 0);
+    __syncwarp();
     int issued = 0;
     int tail_u = -1;          // the load that used the fix-up barrier
     bool tail_done = false;   // ... and was handed over on its slot's barrier
-    // The first key and the pages of the next kMetaTiles tiles are read into
-    // a small shared table ahead of use (rolled loops keep this warp's code
-    // small), so that no global-memory latency sits between a free slot and
-    // the copy that refills it.
-    int32_t* meta_key0 = reinterpret_cast<int32_t*>(sm.ptr + C::kOffMeta);
-    int32_t* meta_page = meta_key0 + C::kMetaTiles;  // [kMetaTiles][16]
-    int batch = -1;
-    int key0 = 0;
-    for (int u = 0; u < 2 * T; ++u) {
-        const int j = u >> 1;
-        const bool is_v = (u & 1) != 0;
-        const int slot = u % C::kSlots;
-        const int use = u / C::kSlots;
-        if (j / C::kMetaTiles != batch) {
-            batch = j / C::kMetaTiles;
-            const int tb = batch * C::kMetaTiles;
-            if (lane < C::kMetaTiles && tb + lane < T)
-                meta_key0[lane] = __ldg(&a.tiles[t0 + tb + lane].key0);
-            __syncwarp();
-#pragma unroll 1
-            for (int idx = lane; idx < C::kMetaTiles * n_pieces; idx += 32) {
-                const int t = idx / n_pieces, i = idx - t * n_pieces;
-                if (tb + t < T)
-                    meta_page[t * 16 + i] = __ldg(&a.tile_pages[(size_t)(t0 + tb + t) * n_pieces + i]);
-            }
+    int4 rec = make_int4(0, 0, -1, -1);
+    if (lane == 0 && T > 0) rec = table[0];
+    for (int j = 0; j < T; ++j) {
+        // the next batch's records, half a batch ahead of their use
+        if (j % C::kMetaTiles == C::kMetaTiles / 2 && (j / C::kMetaTiles + 1) * C::kMetaTiles < T) {
+            fill((j / C::kMetaTiles + 1) * C::kMetaTiles, (j / C::kMetaTiles + 1) & 1);
             __syncwarp();
         }
+        const int key0 = __shfl_sync(0xffffffffu, rec.x, 0);
+        const bool tail = key0 + kPrefillKeys > a.n;
         bool ok = true;
-        if (use > 0 && lane == 0)
-            ok = mbar_wait(sm.bar<D>(C::kBarEmpty + slot), (use - 1) & 1, abort_flag);
-        if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) {
+        for (int kv = 0; kv < 2; ++kv) {
+            const int u = 2 * j + kv;
+            const int slot = u % C::kSlots;
+            const int use = u / C::kSlots;
+            if (lane == 0) {
+                if (use > 0)
+                    ok = mbar_wait(sm.bar<D>(C::kBarEmpty + slot), (use - 1) & 1, abort_flag);
+                if (ok) {
+                    const uint32_t pmask = (uint32_t)rec.y;
+                    const uint32_t bytes = (uint32_t)__popc(pmask) * br * 128 * C::kColBlocks;
+                    const bool vfix = kv == 1 && tail;
+                    const uint32_t fb =
+                        vfix ? sm.bar<D>(C::kBarVfix) : sm.bar<D>(C::kBarFull + slot);
+                    mbar_arrive_expect_tx(fb, bytes);
+                    const uint32_t dst = sm.base + C::kOffRing + slot * C::kSlotBytes;
+                    const int head_row = (kv ? a.Hkv + g : g) * a.P;
+#pragma unroll 1
+                    for (int i = 0; i < n_pieces; ++i) {
+                        if (!((pmask >> i) & 1u)) continue;
+                        const int key = key0 + i * br;
+                        const int32_t page =
+                            i == 0 ? rec.z
+                                   : (i == 1 ? rec.w
+                                             : __ldg(&a.tile_pages[(size_t)(t0 + j) * n_pieces + i]));
+#pragma unroll
+                        for (int cb = 0; cb < C::kColBlocks; ++cb)
+                            tma_load_4d(dst + cb * C::kBlockBytes + i * br * 128, pool_map, fb,
+                                        cb * 64, head_row + key % a.P, page, a.layer);
+                    }
+                    // the next tile's record, read while these copies are in flight
+                    if (kv == 1 && j + 1 < T)
+                        rec = table[((j + 1) / C::kMetaTiles & 1) * C::kMetaTiles +
+                                    (j + 1) % C::kMetaTiles];
+                }
+            }
+            ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+            if (!ok) break;
+            issued = u + 1;
+        }
+        if (!ok) {
             if (lane == 0) {
                 set_error(a.err, kErrTimeout);
                 *abort_flag = 1;
             }
             break;
         }
-        const int mt = j % C::kMetaTiles;
-        key0 = meta_key0[mt];
-        const bool tail = is_v && key0 + kPrefillKeys > a.n;
-        const uint32_t dst = sm.base + C::kOffRing + slot * C::kSlotBytes;
-        if (lane == 0) {
-            // pieces that hold tokens of the sequence and a page inside the pool
-            uint32_t pmask = 0;
-#pragma unroll 1
-            for (int i = 0; i < n_pieces && key0 + i * br < a.n; ++i) {
-                if ((uint32_t)meta_page[mt * 16 + i] < (uint32_t)a.num_pages) pmask |= 1u << i;
-                else set_error(a.err, kErrBounds);
-            }
-            const uint32_t bytes = (uint32_t)__popc(pmask) * br * 128 * C::kColBlocks;
-            const uint32_t fb = tail ? sm.bar<D>(C::kBarVfix) : sm.bar<D>(C::kBarFull + slot);
-            mbar_arrive_expect_tx(fb, bytes);
-            const int head_row = (is_v ? a.Hkv + g : g) * a.P;
-#pragma unroll 1
-            for (int i = 0; i < n_pieces; ++i) {
-                if (!((pmask >> i) & 1u)) continue;
-                const int key = key0 + i * br;
-                const int32_t page = meta_page[mt * 16 + i];
-#pragma unroll
-                for (int cb = 0; cb < C::kColBlocks; ++cb)
-                    tma_load_4d(dst + cb * C::kBlockBytes + i * br * 128, pool_map, fb, cb * 64,
-                                head_row + key % a.P, page, a.layer);
-            }
-        }
-        __syncwarp();
-        issued = u + 1;
         if (tail) {
             // The last key tile: its V rows past the sequence's end hold stale
             // or never-written data.  Their weights are zero, but 0 * NaN is
             // not, so zero those rows before the MMAs read the slot.
+            const int u = 2 * j + 1, slot = u % C::kSlots;
             tail_u = u;
-            ok = true;
             if (lane == 0) ok = mbar_wait(sm.bar<D>(C::kBarVfix), 0, abort_flag);
             if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) {
                 if (lane == 0) {
@@ -387,104 +403,132 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
         // row maximum, one for the weights.
         const int lim = p_row - key0;  // keys key0 + c with c <= lim are causal
         const bool unmasked = valid && (w0.y & kPrefillTileFull) && lim >= kPrefillKeys - 1;
-        // row maximum: three-input max over four independent chains
-        float mx[4];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) mx[c] = -INFINITY;
-#pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-            uint32_t x[64];
-            tmem_ld32(tl + col_s + 64 * hh, *reinterpret_cast<uint32_t(*)[32]>(&x[0]));
-            tmem_ld32(tl + col_s + 64 * hh + 32, *reinterpret_cast<uint32_t(*)[32]>(&x[32]));
-            tmem_wait_ld();
-            if (!unmasked) {
-#pragma unroll
-                for (int w = 0; w < 2; ++w) {
-                    const int ww = 2 * hh + w;
-                    const uint32_t mw = valid ? (vis[ww] & low_bits_through(lim - 32 * ww)) : 0u;
-#pragma unroll
-                    for (int c = 0; c < 32; ++c)
-                        if (!((mw >> c) & 1u)) x[32 * w + c] = 0xff800000u;  // -inf
-                }
-            }
-#pragma unroll
-            for (int c = 0; c < 64; c += 8) {
-                mx[0] = fmax3(mx[0], __uint_as_float(x[c]), __uint_as_float(x[c + 1]));
-                mx[1] = fmax3(mx[1], __uint_as_float(x[c + 2]), __uint_as_float(x[c + 3]));
-                mx[2] = fmax3(mx[2], __uint_as_float(x[c + 4]), __uint_as_float(x[c + 5]));
-                mx[3] = fmax3(mx[3], __uint_as_float(x[c + 6]), __uint_as_float(x[c + 7]));
-            }
-        }
-        const float mt = fmaxf(fmax3(mx[0], mx[1], mx[2]), mx[3]) * sc;
-        const bool need = mt > m_run + 8.f;
-        float alpha = 1.f;
-        if (need) {
-            alpha = exp2f(m_run - mt);
-            m_run = mt;
-            l *= alpha;
-        }
-        if (j > 0 && __any_sync(0xffffffffu, need)) {
-            // O_t holds the products up to key tile j - 1 (complete: S_t(j) was
-            // issued after them): rescale it in place
-#pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
-                uint32_t o[32];
-                tmem_ld32(tl + col_o + c * 32, o);
-                tmem_wait_ld();
-#pragma unroll
-                for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-                tmem_st32(tl + col_o + c * 32, o);
-            }
-        }
-        // weights 2^(s * scale - m) (arguments two at a time with a packed
-        // FMA), rounded to bf16 and stored to TMEM over the first half of S_t
-        // as the A operand of the value product (half hh of the keys goes to
-        // columns 32 hh .. +31, after that half of S was read); the normaliser
-        // sums the fp32 weights (four packed chains)
+        // Weights 2^(s * scale - m) with the running maximum m, two arguments
+        // at a time with a packed FMA, rounded to bf16 into wt (32 words per
+        // 64 keys); the normaliser sums the fp32 weights (four packed chains).
+        // When `track` is set the pass also returns the tile's raw maximum.
+        // Nothing is stored: S stays intact until the weights are accepted.
         const uint64_t sc2 = f2pack(sc, sc);
-        const float nmu = m_run == -INFINITY ? 0.f : -m_run;
-        const uint64_t nmu2 = f2pack(nmu, nmu);
-        uint64_t ls2[4];
+        uint32_t wt[2][32];
+        auto weights = [&](float m, bool track, float& tile_max, float& tile_sum) {
+            const float nmu = m == -INFINITY ? 0.f : -m;
+            const uint64_t nmu2 = f2pack(nmu, nmu);
+            uint64_t ls2[4];
+            float mx[4];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) ls2[c] = 0;
+            for (int c = 0; c < 4; ++c) {
+                ls2[c] = 0;
+                mx[c] = -INFINITY;
+            }
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-            uint32_t x[64];
-            tmem_ld32(tl + col_s + 64 * hh, *reinterpret_cast<uint32_t(*)[32]>(&x[0]));
-            tmem_ld32(tl + col_s + 64 * hh + 32, *reinterpret_cast<uint32_t(*)[32]>(&x[32]));
-            tmem_wait_ld();
-            if (!unmasked) {
+            for (int hh = 0; hh < 2; ++hh) {
+                uint32_t x[64];
+                tmem_ld32(tl + col_s + 64 * hh, *reinterpret_cast<uint32_t(*)[32]>(&x[0]));
+                tmem_ld32(tl + col_s + 64 * hh + 32, *reinterpret_cast<uint32_t(*)[32]>(&x[32]));
+                tmem_wait_ld();
+                if (!unmasked) {
 #pragma unroll
-                for (int w = 0; w < 2; ++w) {
-                    const int ww = 2 * hh + w;
-                    const uint32_t mw = valid ? (vis[ww] & low_bits_through(lim - 32 * ww)) : 0u;
+                    for (int w = 0; w < 2; ++w) {
+                        const int ww = 2 * hh + w;
+                        const uint32_t mw = valid ? (vis[ww] & low_bits_through(lim - 32 * ww)) : 0u;
 #pragma unroll
-                    for (int c = 0; c < 32; ++c)
-                        if (!((mw >> c) & 1u)) x[32 * w + c] = 0xff800000u;  // -inf
+                        for (int c = 0; c < 32; ++c)
+                            if (!((mw >> c) & 1u)) x[32 * w + c] = 0xff800000u;  // -inf
+                    }
+                }
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const float x0 = __uint_as_float(x[2 * i]), x1 = __uint_as_float(x[2 * i + 1]);
+                    if (track) mx[i & 3] = fmax3(mx[i & 3], x0, x1);
+                    float a0, a1;
+                    f2unpack(ffma2(f2pack(x0, x1), sc2, nmu2), a0, a1);
+                    const float p0 = exp2f(a0), p1 = exp2f(a1);
+                    ls2[i & 3] = fadd2(ls2[i & 3], f2pack(p0, p1));
+                    const __nv_bfloat162 hb = __floats2bfloat162_rn(p0, p1);
+                    wt[hh][i] = *reinterpret_cast<const uint32_t*>(&hb);
                 }
             }
-            uint32_t w[32];
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-                float a0, a1;
-                f2unpack(ffma2(f2pack(__uint_as_float(x[2 * i]), __uint_as_float(x[2 * i + 1])),
-                               sc2, nmu2),
-                         a0, a1);
-                const float p0 = exp2f(a0), p1 = exp2f(a1);
-                ls2[i & 3] = fadd2(ls2[i & 3], f2pack(p0, p1));
-                const __nv_bfloat162 hb = __floats2bfloat162_rn(p0, p1);
-                w[i] = *reinterpret_cast<const uint32_t*>(&hb);
-            }
-            tmem_st32(tl + col_s + 32 * hh, w);
-        }
-        {
             float s0, s1, s2, s3, s4, s5, s6, s7;
             f2unpack(ls2[0], s0, s1);
             f2unpack(ls2[1], s2, s3);
             f2unpack(ls2[2], s4, s5);
             f2unpack(ls2[3], s6, s7);
-            l += ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
+            tile_sum = ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
+            tile_max = fmaxf(fmax3(mx[0], mx[1], mx[2]), mx[3]);
+        };
+        // The maximum is raised lazily, so most tiles keep it: take the
+        // weights with the current maximum and the tile maximum in one pass,
+        // and redo the tile only where a row's maximum grew by more than 2^8
+        // (or the row has seen no key yet).
+        float mt = -INFINITY, tsum = 0.f;
+        bool done = false;
+        if (__all_sync(0xffffffffu, m_run != -INFINITY)) {
+            float raw;
+            weights(m_run, true, raw, tsum);
+            mt = raw * sc;
+            done = !__any_sync(0xffffffffu, mt > m_run + 8.f);
+        } else {
+            // row maximum: three-input max over four independent chains
+            float mx[4];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) mx[c] = -INFINITY;
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {
+                uint32_t x[64];
+                tmem_ld32(tl + col_s + 64 * hh, *reinterpret_cast<uint32_t(*)[32]>(&x[0]));
+                tmem_ld32(tl + col_s + 64 * hh + 32, *reinterpret_cast<uint32_t(*)[32]>(&x[32]));
+                tmem_wait_ld();
+                if (!unmasked) {
+#pragma unroll
+                    for (int w = 0; w < 2; ++w) {
+                        const int ww = 2 * hh + w;
+                        const uint32_t mw = valid ? (vis[ww] & low_bits_through(lim - 32 * ww)) : 0u;
+#pragma unroll
+                        for (int c = 0; c < 32; ++c)
+                            if (!((mw >> c) & 1u)) x[32 * w + c] = 0xff800000u;  // -inf
+                    }
+                }
+#pragma unroll
+                for (int c = 0; c < 64; c += 8) {
+                    mx[0] = fmax3(mx[0], __uint_as_float(x[c]), __uint_as_float(x[c + 1]));
+                    mx[1] = fmax3(mx[1], __uint_as_float(x[c + 2]), __uint_as_float(x[c + 3]));
+                    mx[2] = fmax3(mx[2], __uint_as_float(x[c + 4]), __uint_as_float(x[c + 5]));
+                    mx[3] = fmax3(mx[3], __uint_as_float(x[c + 6]), __uint_as_float(x[c + 7]));
+                }
+            }
+            mt = fmaxf(fmax3(mx[0], mx[1], mx[2]), mx[3]) * sc;
         }
+        if (done) {
+            l += tsum;
+        } else {
+            const bool need = mt > m_run + 8.f;
+            float alpha = 1.f;
+            if (need) {
+                alpha = exp2f(m_run - mt);
+                m_run = mt;
+                l *= alpha;
+            }
+            if (j > 0 && __any_sync(0xffffffffu, need)) {
+                // O_t holds the products up to key tile j - 1 (complete: S_t(j)
+                // was issued after them): rescale it in place
+#pragma unroll
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t o[32];
+                    tmem_ld32(tl + col_o + c * 32, o);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i)
+                        o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+                    tmem_st32(tl + col_o + c * 32, o);
+                }
+            }
+            float unused;
+            weights(m_run, false, unused, tsum);
+            l += tsum;
+        }
+        // P_t over the first half of S_t: keys 64 hh .. +63 to columns 32 hh .. +31
+        tmem_st32(tl + col_s, wt[0]);
+        tmem_st32(tl + col_s + 32, wt[1]);
         tmem_wait_st();
         tc_fence_before();
         mbar_arrive(sm.bar<D>(C::kBarP + t));
