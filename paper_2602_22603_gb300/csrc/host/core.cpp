@@ -614,13 +614,27 @@ int plan_prefill(const Geometry& g, int32_t n, int32_t n_q, const int32_t* start
     }
     const int64_t units = (int64_t)out->n_qt * g.Hkv;
     const int32_t n_tiles = (int32_t)out->tiles.size();
+    // Split each CTA tile's key range when there are too few CTA tiles to
+    // fill the GPU: pick the split that minimises the estimated makespan,
+    // waves x (key tiles per CTA + a fixed per-CTA cost), CTAs running
+    // `target_ctas` at a time.
     int32_t split = 1;
-    if (units < target_ctas && n_tiles > 0) {
-        // at least kMinTiles key tiles per split, at most kMaxSplit splits
-        constexpr int32_t kMinTiles = 4, kMaxSplit = 64;
-        split = (int32_t)std::min<int64_t>((target_ctas + units - 1) / units,
-                                           std::max<int32_t>(1, n_tiles / kMinTiles));
-        split = std::max(1, std::min(split, kMaxSplit));
+    if (units < target_ctas && n_tiles > 0 && target_ctas > 0) {
+        constexpr int32_t kMaxSplit = 64;
+        constexpr double kCtaCost = 4.0;  // prologue + epilogue, in key tiles
+        double avg = 0;
+        for (int32_t c : out->qt_tiles) avg += c;
+        avg /= std::max<int32_t>(1, out->n_qt);
+        double best = 1e300;
+        for (int32_t sp = 1; sp <= kMaxSplit && sp <= n_tiles; ++sp) {
+            const int64_t ctas = units * sp;
+            const int64_t waves = (ctas + target_ctas - 1) / target_ctas;
+            const double cost = (double)waves * (avg / sp + kCtaCost);
+            if (cost < best - 1e-9) {
+                best = cost;
+                split = sp;
+            }
+        }
     }
     out->n_split = split;
     return kOk;

@@ -266,8 +266,10 @@ __device__ __forceinline__ void issue_pv(const Smem& sm, uint32_t tmem, int t, i
                     (!first || ks > 0) ? 1u : 0u);
 }
 
+// `two`: tile b holds query rows (false for short query blocks, whose rows
+// all fit in tile a; tile b's products are then skipped).
 template <int D>
-__device__ void prefill_mma(const PrefillArgs& a, const Smem& sm, uint32_t tmem, int T,
+__device__ void prefill_mma(const PrefillArgs& a, const Smem& sm, uint32_t tmem, int T, bool two,
                             volatile int* abort_flag) {
     using C = PreCfg<D>;
     bool ok = mbar_wait(sm.bar<D>(C::kBarQ), 0, abort_flag);
@@ -280,8 +282,10 @@ __device__ void prefill_mma(const PrefillArgs& a, const Smem& sm, uint32_t tmem,
             any = true;
             issue_qk<D>(sm, tmem, 0, k0);
             mma_commit(sm.bar<D>(C::kBarS + 0));
-            issue_qk<D>(sm, tmem, 1, k0);
-            mma_commit(sm.bar<D>(C::kBarS + 1));
+            if (two) {
+                issue_qk<D>(sm, tmem, 1, k0);
+                mma_commit(sm.bar<D>(C::kBarS + 1));
+            }
             mma_commit(sm.bar<D>(C::kBarEmpty + k0));
         }
         for (int j = 0; ok && j < T; ++j) {
@@ -295,13 +299,16 @@ __device__ void prefill_mma(const PrefillArgs& a, const Smem& sm, uint32_t tmem,
                 break;
             issue_pv<D>(sm, tmem, 0, vslot, j == 0);
             if (!more) mma_commit(sm.bar<D>(C::kBarO + 0));
+            if (!two) mma_commit(sm.bar<D>(C::kBarEmpty + vslot));
             if (more) {
                 if (!(ok = mbar_wait(sm.bar<D>(C::kBarFull + kslot), (uk / C::kSlots) & 1,
                                      abort_flag)))
                     break;
                 issue_qk<D>(sm, tmem, 0, kslot);
                 mma_commit(sm.bar<D>(C::kBarS + 0));
+                if (!two) mma_commit(sm.bar<D>(C::kBarEmpty + kslot));
             }
+            if (!two) continue;
             // tile b
             if (!(ok = mbar_wait(sm.bar<D>(C::kBarP + 1), j & 1, abort_flag))) break;
             tc_fence_after();
@@ -372,6 +379,23 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
     const int row = wq * 32 + lane;
     const int qi = pos_lo + t * a.BP + row / a.G;
     const bool valid = row < a.BP * a.G && qi < a.n_q;
+    // A warp none of whose rows is a query only keeps the barrier count: it
+    // waits for each S and signals its P without computing (its rows of P
+    // and O are never read back).
+    if (!__any_sync(0xffffffffu, valid)) {
+        for (int j = 0; j < T; ++j) {
+            if (!warp_wait(sm.bar<D>(C::kBarS + t), j & 1, abort_flag, lane)) {
+                if (lane == 0) {
+                    set_error(a.err, kErrTimeout);
+                    *abort_flag = 1;
+                }
+                return;
+            }
+            tc_fence_before();
+            mbar_arrive(sm.bar<D>(C::kBarP + t));
+        }
+        return;
+    }
     const int p_row = a.n - a.n_q + qi;
     const uint32_t tl = tmem + ((uint32_t)(wq * 32) << 16);
     const uint32_t col_s = C::kColS + (uint32_t)t * kPrefillKeys;
@@ -642,12 +666,14 @@ __global__ void __launch_bounds__(320, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
     const int t0 = sched[0], T = sched[1];
+    // tile b is empty when every query of the CTA tile fits in tile a
+    const bool two = pos_lo + a.BP < a.n_q;
     if (warp == 0) {
         prefill_produce<D>(&pool_map, &qmap, a, sm, g, pos_lo, t0, T, abort_flag, lane);
     } else if (warp == 1) {
-        if (lane == 0) prefill_mma<D>(a, sm, tmem, T, abort_flag);
+        if (lane == 0) prefill_mma<D>(a, sm, tmem, T, two, abort_flag);
         __syncwarp();
-    } else {
+    } else if (warp < 6 || two) {
         prefill_softmax<D>(a, sm, tmem, (warp - 2) >> 2, g, pos_lo, t0, T, abort_flag, warp, lane);
     }
     tc_fence_before();

@@ -315,7 +315,7 @@ def test_prefill_plan_visibility_matches_brute_force(seed):
     if units >= 152:
         assert info["n_split"] == 1
     else:
-        assert info["n_split"] <= max(1, len(exp_tiles) // 4)
+        assert info["n_split"] <= max(1, min(64, len(exp_tiles)))
 
 
 def test_prefill_plan_rejects_bad_input():
@@ -336,5 +336,11 @@ def test_prefill_plan_splits_short_query_blocks():
     from tests.hostlib import plan_prefill
     rc, info, _ = plan_prefill(32, 8, 131072, 8, [])
     assert rc == 0 and info["n_qt"] == 1 and info["n_split"] == 19
+    # 512 queries: 64 CTA tiles; the split fills its waves of 152 CTAs (not
+    # 3 splits = 192 CTAs, whose second wave is 26% full)
+    rc, info, _ = plan_prefill(32, 8, 131072, 512, [])
+    ctas = 64 * info["n_split"]
+    assert rc == 0 and info["n_qt"] == 8 and info["n_split"] > 1
+    assert ctas / (-(-ctas // 152) * 152) >= 0.9
     rc, info, _ = plan_prefill(32, 8, 32768, 32768, [(100, 5000)])
     assert rc == 0 and info["n_split"] == 1 and info["n_qt"] == 512
