@@ -292,18 +292,20 @@ __device__ void prefill_mma(const PrefillArgs& a, const Smem& sm, uint32_t tmem,
             const int uv = 2 * j + 1, vslot = uv % C::kSlots;
             const int uk = 2 * j + 2, kslot = uk % C::kSlots;
             const bool more = j + 1 < T;
+            // V_j and K_{j+1} have normally landed long ago; checking them before
+            // P_a keeps these barrier reads off the path from P_a to the MMAs
+            if (!(ok = mbar_wait(sm.bar<D>(C::kBarFull + vslot), (uv / C::kSlots) & 1, abort_flag)))
+                break;
+            if (more && !(ok = mbar_wait(sm.bar<D>(C::kBarFull + kslot), (uk / C::kSlots) & 1,
+                                         abort_flag)))
+                break;
             // tile a: O_a += P_a V_j, then S_a for the next key tile
             if (!(ok = mbar_wait(sm.bar<D>(C::kBarP + 0), j & 1, abort_flag))) break;
             tc_fence_after();
-            if (!(ok = mbar_wait(sm.bar<D>(C::kBarFull + vslot), (uv / C::kSlots) & 1, abort_flag)))
-                break;
             issue_pv<D>(sm, tmem, 0, vslot, j == 0);
             if (!more) mma_commit(sm.bar<D>(C::kBarO + 0));
             if (!two) mma_commit(sm.bar<D>(C::kBarEmpty + vslot));
             if (more) {
-                if (!(ok = mbar_wait(sm.bar<D>(C::kBarFull + kslot), (uk / C::kSlots) & 1,
-                                     abort_flag)))
-                    break;
                 issue_qk<D>(sm, tmem, 0, kslot);
                 mma_commit(sm.bar<D>(C::kBarS + 0));
                 if (!two) mma_commit(sm.bar<D>(C::kBarEmpty + kslot));
