@@ -68,7 +68,9 @@ struct PreCfg {
     static constexpr int kMetaTiles = 16;
     static constexpr int kOffMeta = (kOffMisc + 32 + 15) & ~15;  // int4 records: 16-byte aligned
     static constexpr int kMetaBytes = 2 * kMetaTiles * 16;
-    static constexpr int kSmemBytes = kOffMeta + kMetaBytes + 1024;  // + alignment slack
+    // dual-key mode: tile b's (max, normaliser) of each row, for the merge
+    static constexpr int kOffXchg = kOffMeta + kMetaBytes;
+    static constexpr int kSmemBytes = kOffXchg + kPrefillRows * 8 + 1024;  // + alignment slack
     static constexpr uint32_t kTmemCols = 512;
     static constexpr uint32_t kColS = 0;    // S_t (fp32) at 128 t; P_t (bf16 pairs) over its first 64
     static constexpr uint32_t kColO = 256;  // O_t (fp32) at 256 + 128 t
@@ -237,11 +239,12 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
     }
 }
 
-// S_t = Q_t K^T for the K tile in `slot`, into TMEM columns 128 t.
+// S_t = Q_q K^T for the K tile in `slot`, into TMEM columns 128 t (q = t
+// except in dual-key mode, where both tiles use query tile 0).
 template <int D>
-__device__ __forceinline__ void issue_qk(const Smem& sm, uint32_t tmem, int t, int slot) {
+__device__ __forceinline__ void issue_qk(const Smem& sm, uint32_t tmem, int t, int slot, int q = -1) {
     using C = PreCfg<D>;
-    const uint32_t qa = sm.base + C::kOffQ + t * C::kQBytes;
+    const uint32_t qa = sm.base + C::kOffQ + (q < 0 ? t : q) * C::kQBytes;
     const uint32_t ka = sm.base + C::kOffRing + slot * C::kSlotBytes;
     const uint32_t dt = tmem + C::kColS + (uint32_t)t * kPrefillKeys;
 #pragma unroll
@@ -266,15 +269,63 @@ __device__ __forceinline__ void issue_pv(const Smem& sm, uint32_t tmem, int t, i
                     (!first || ks > 0) ? 1u : 0u);
 }
 
+// Dual-key mode (every query of the CTA tile fits in tile a): both tiles
+// hold tile a's queries; tile a takes key tiles 0, 2, 4, ... and tile b the
+// odd ones, and the two results are merged at the end.
+template <int D>
+__device__ bool prefill_mma_dual(const Smem& sm, uint32_t tmem, int T, volatile int* abort_flag) {
+    using C = PreCfg<D>;
+    const int Tt[2] = {(T + 1) / 2, T / 2};
+    bool ok = true;
+    for (int t = 0; t < 2 && ok; ++t) {
+        // S_t(0) = Q_a K_t
+        const int u = 2 * t, slot = u % C::kSlots;
+        if (!(ok = mbar_wait(sm.bar<D>(C::kBarFull + slot), (u / C::kSlots) & 1, abort_flag))) break;
+        issue_qk<D>(sm, tmem, t, slot, 0);
+        mma_commit(sm.bar<D>(C::kBarS + t));
+        mma_commit(sm.bar<D>(C::kBarEmpty + slot));
+    }
+    for (int i = 0; ok && i < Tt[0]; ++i) {
+        for (int t = 0; t < 2; ++t) {
+            if (i >= Tt[t]) break;
+            const int j = 2 * i + t;  // key tile of this step
+            const int uv = 2 * j + 1, vslot = uv % C::kSlots;
+            const int uk = 2 * j + 4, kslot = uk % C::kSlots;  // K of key tile j + 2
+            const bool more = i + 1 < Tt[t];
+            if (!(ok = mbar_wait(sm.bar<D>(C::kBarFull + vslot), (uv / C::kSlots) & 1, abort_flag)))
+                break;
+            if (more && !(ok = mbar_wait(sm.bar<D>(C::kBarFull + kslot), (uk / C::kSlots) & 1,
+                                         abort_flag)))
+                break;
+            if (!(ok = mbar_wait(sm.bar<D>(C::kBarP + t), i & 1, abort_flag))) break;
+            tc_fence_after();
+            issue_pv<D>(sm, tmem, t, vslot, i == 0);
+            mma_commit(sm.bar<D>(C::kBarEmpty + vslot));
+            if (!more) mma_commit(sm.bar<D>(C::kBarO + t));
+            if (more) {
+                issue_qk<D>(sm, tmem, t, kslot, 0);
+                mma_commit(sm.bar<D>(C::kBarS + t));
+                mma_commit(sm.bar<D>(C::kBarEmpty + kslot));
+            }
+        }
+    }
+    return ok;
+}
+
 // `two`: tile b holds query rows (false for short query blocks, whose rows
-// all fit in tile a; tile b's products are then skipped).
+// all fit in tile a; tile b's products are then skipped, or, with `dual`, it
+// takes every other key tile).
 template <int D>
 __device__ void prefill_mma(const PrefillArgs& a, const Smem& sm, uint32_t tmem, int T, bool two,
-                            volatile int* abort_flag) {
+                            bool dual, volatile int* abort_flag) {
     using C = PreCfg<D>;
     bool ok = mbar_wait(sm.bar<D>(C::kBarQ), 0, abort_flag);
     bool any = false;
-    if (ok && T > 0) {
+    if (ok && T > 0 && dual) {
+        tc_fence_after();
+        any = true;
+        ok = prefill_mma_dual<D>(sm, tmem, T, abort_flag);
+    } else if (ok && T > 0) {
         tc_fence_after();
         const int k0 = 0;
         ok = mbar_wait(sm.bar<D>(C::kBarFull + k0), 0, abort_flag);
@@ -374,28 +425,34 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, const v
 // Softmax warpgroup of query tile t (one row per thread) and its epilogue.
 template <int D>
 __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t tmem, int t, int g,
-                                int pos_lo, int t0, int T, volatile int* abort_flag, int warp,
-                                int lane) {
+                                int pos_lo, int t0, int T_cta, bool dual, volatile int* abort_flag,
+                                int warp, int lane) {
     using C = PreCfg<D>;
     const int wq = warp & 3;
     const int row = wq * 32 + lane;
-    const int qi = pos_lo + t * a.BP + row / a.G;
+    // dual-key mode: both tiles hold tile a's queries, tile t takes key tiles
+    // t, t + 2, t + 4, ... of the CTA's range
+    const int qi = pos_lo + (dual ? 0 : t) * a.BP + row / a.G;
     const bool valid = row < a.BP * a.G && qi < a.n_q;
+    const int T = dual ? (T_cta + 1 - t) / 2 : T_cta;
+    const int kstep = dual ? 2 : 1, kfirst = dual ? t : 0;
+    float* xchg = reinterpret_cast<float*>(sm.ptr + C::kOffXchg);
     // A warp none of whose rows is a query only keeps the barrier count: it
     // waits for each S and signals its P without computing (its rows of P
     // and O are never read back).
     if (!__any_sync(0xffffffffu, valid)) {
+        bool wok = true;
         for (int j = 0; j < T; ++j) {
-            if (!warp_wait(sm.bar<D>(C::kBarS + t), j & 1, abort_flag, lane)) {
-                if (lane == 0) {
-                    set_error(a.err, kErrTimeout);
-                    *abort_flag = 1;
-                }
-                return;
-            }
+            if (wok) wok = warp_wait(sm.bar<D>(C::kBarS + t), j & 1, abort_flag, lane);
             tc_fence_before();
             mbar_arrive(sm.bar<D>(C::kBarP + t));
         }
+        if (!wok && lane == 0) {
+            set_error(a.err, kErrTimeout);
+            *abort_flag = 1;
+        }
+        // the merge of the two tiles' results meets all 256 threads, whatever happened
+        if (dual) named_bar_sync(3, 256);
         return;
     }
     const int p_row = a.n - a.n_q + qi;
@@ -407,7 +464,7 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
     bool ok = true;
     int4 n0 = make_int4(0, 0, 0, 0), n1 = n0;
     if (T > 0) {
-        const int4* tp = reinterpret_cast<const int4*>(a.tiles + t0);
+        const int4* tp = reinterpret_cast<const int4*>(a.tiles + t0 + kfirst);
         n0 = __ldg(tp);
         n1 = __ldg(tp + 1);
     }
@@ -415,7 +472,8 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
         // this tile's record; the next one is fetched while this tile is worked on
         const int4 w0 = n0, w1 = n1;
         if (j + 1 < T) {
-            const int4* tp = reinterpret_cast<const int4*>(a.tiles + t0 + j + 1);
+            const int4* tp =
+                reinterpret_cast<const int4*>(a.tiles + t0 + kfirst + (j + 1) * kstep);
             n0 = __ldg(tp);
             n1 = __ldg(tp + 1);
         }
@@ -560,6 +618,30 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
         mbar_arrive(sm.bar<D>(C::kBarP + t));
     }
     if (ok && T > 0) ok = warp_wait(sm.bar<D>(C::kBarO + t), 0, abort_flag, lane);
+    // dual-key mode: tile b hands its (max, normaliser) to tile a, which
+    // merges the two partial results of each row (weights 2^(m_t - max))
+    float wa = 1.f, wb = 0.f;
+    if (dual) {
+        if (t == 1) {
+            xchg[2 * row] = m_run;
+            xchg[2 * row + 1] = l;
+        }
+        named_bar_sync(3, 256);
+        if (t == 1) {
+            if (!ok && lane == 0) {
+                set_error(a.err, kErrTimeout);
+                *abort_flag = 1;
+            }
+            return;
+        }
+        if (ok) ok = warp_wait(sm.bar<D>(C::kBarO + 1), 0, abort_flag, lane);
+        const float mb = xchg[2 * row], lb = xchg[2 * row + 1];
+        const float M = fmaxf(m_run, mb);
+        wa = m_run == -INFINITY ? 0.f : exp2f(m_run - M);
+        wb = mb == -INFINITY ? 0.f : exp2f(mb - M);
+        l = l * wa + lb * wb;
+        m_run = M;
+    }
     if (!ok) {
         if (lane == 0) {
             set_error(a.err, kErrTimeout);
@@ -592,10 +674,19 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
 #pragma unroll
             for (int i = 0; i < 32; ++i) o[i] = 0u;
         }
-        if (!valid) continue;
         float f[32];
+        if (dual) {
+            uint32_t ob[32];
+            tmem_ld32(tl + C::kColO + 128 + c * 32, ob);
+            tmem_wait_ld();
 #pragma unroll
-        for (int i = 0; i < 32; ++i) f[i] = __uint_as_float(o[i]) * inv;
+            for (int i = 0; i < 32; ++i)
+                f[i] = (__uint_as_float(o[i]) * wa + __uint_as_float(ob[i]) * wb) * inv;
+        } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) f[i] = __uint_as_float(o[i]) * inv;
+        }
+        if (!valid) continue;
         if (part_row || a.out_f32) {
             float4* dst = reinterpret_cast<float4*>(part_row ? part_row + c * 32
                                                              : reinterpret_cast<float*>(out_row) + c * 32);
@@ -668,15 +759,18 @@ __global__ void __launch_bounds__(320, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
     const int t0 = sched[0], T = sched[1];
-    // tile b is empty when every query of the CTA tile fits in tile a
+    // tile b is empty when every query of the CTA tile fits in tile a; it then
+    // takes every other key tile of tile a's queries (dual-key mode)
     const bool two = pos_lo + a.BP < a.n_q;
+    const bool dual = !two && T >= 2;
     if (warp == 0) {
         prefill_produce<D>(&pool_map, &qmap, a, sm, g, pos_lo, t0, T, abort_flag, lane);
     } else if (warp == 1) {
-        if (lane == 0) prefill_mma<D>(a, sm, tmem, T, two, abort_flag);
+        if (lane == 0) prefill_mma<D>(a, sm, tmem, T, two, dual, abort_flag);
         __syncwarp();
-    } else if (warp < 6 || two) {
-        prefill_softmax<D>(a, sm, tmem, (warp - 2) >> 2, g, pos_lo, t0, T, abort_flag, warp, lane);
+    } else if (warp < 6 || two || dual) {
+        prefill_softmax<D>(a, sm, tmem, (warp - 2) >> 2, g, pos_lo, t0, T, dual, abort_flag, warp,
+                           lane);
     }
     tc_fence_before();
     __syncthreads();

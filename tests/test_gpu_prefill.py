@@ -204,3 +204,22 @@ def test_prefill_rejects_bad_arguments():
         assert c.sync_status() == sq.SQ_OK
     finally:
         p.close()
+
+
+@pytest.mark.parametrize("n,n_q,spans", [
+    (5 * 128 + 3, 5, [(10, 200)]),             # 6 key tiles: the two halves take 3 + 3
+    (7 * 128 + 1, 3, [(0, 600)]),              # 8 key tiles; rows see keys only past 600
+    (4 * 128, 8, [(0, 130), (260, 384)]),      # keys only in tiles 1 and 3 (one half)
+    (3 * 128 + 64, 1, []),                     # 4 key tiles, one query
+])
+def test_prefill_short_block_dual_key_split(n, n_q, spans):
+    # All queries of a CTA tile fit in its first query tile, so the second takes
+    # every other key tile and the two partial results are merged per row.
+    p = Pair(1, 32, 8, 128, 64, num_pages=n // 64 + 4, seed=n_q + 40)
+    try:
+        h = p.seq_new()
+        p.append(h, n)
+        check(p, h, 0, n_q, spans, seed=n + 1)
+        check(p, h, 0, n_q, spans, seed=n + 2, out_dtype=sq.SQ_OUT_BF16)
+    finally:
+        p.close()
