@@ -49,6 +49,27 @@ struct PlanEntry {
     uint64_t last_use = 0;
 };
 
+// Prefill plans, reused while the sequence (its version), the query count,
+// the spans and the CTA target stay the same: the layers of one step share
+// one plan, planned and uploaded once.
+constexpr int kPrefillPlanEntries = 4;
+struct PrefillPlanEntry {
+    bool valid = false;
+    int32_t seq = 0;
+    uint64_t version = 0;
+    int32_t n_q = 0;
+    int32_t target = 0;
+    std::vector<int32_t> spans;  // start, end pairs as passed
+    size_t tb = 0, qb = 0;       // bytes of the tile records, of the per-CTA-tile counts
+    int32_t n_tiles = 0, n_pieces = 0, BP = 0, n_qt = 0, n_split = 0;
+    int64_t visible_pairs = 0;
+    uint8_t* d = nullptr;  // [tiles][qt_tiles][tile_pages]
+    size_t cap = 0;
+    cudaEvent_t ev = nullptr;  // recorded after the last launch that used it
+    bool ev_recorded = false;
+    uint64_t last_use = 0;
+};
+
 struct UploadSlot {
     uint8_t* d = nullptr;
     size_t cap = 0;
@@ -89,6 +110,7 @@ struct sq_cache {
     cudaEvent_t pre_ev = nullptr;
     bool pre_ev_recorded = false;
     PlanEntry plans[kPlanCacheEntries];
+    PrefillPlanEntry pre_plans[kPrefillPlanEntries];
     uint64_t use_clock = 0;
     UploadSlot slots[kUploadSlots];
     int next_slot = 0;
@@ -363,6 +385,10 @@ int sq_cache_destroy(sq_cache* c) {
     if (!c) return SQ_ERR_BAD_HANDLE;
     cudaDeviceSynchronize();
     for (auto& p : c->plans) free_entry(p);
+    for (auto& p : c->pre_plans) {
+        if (p.d) cudaFree(p.d);
+        if (p.ev) cudaEventDestroy(p.ev);
+    }
     for (auto& s : c->slots) {
         if (s.d) cudaFree(s.d);
         if (s.ev) cudaEventDestroy(s.ev);
@@ -738,29 +764,87 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
         return SQ_ERR_INVALID_ARG;
     if (!(sm_scale >= 0.f) || sm_scale > 3.0e38f) return SQ_ERR_INVALID_ARG;
     if (n_spans < 0 || (n_spans > 0 && !spans)) return SQ_ERR_INVALID_ARG;
-    std::vector<int32_t> sa(n_spans), sb(n_spans);
+    std::vector<int32_t> key(2 * (size_t)n_spans);
     for (int32_t i = 0; i < n_spans; ++i) {
-        sa[i] = spans[i].start;
-        sb[i] = spans[i].end;
+        key[2 * i] = spans[i].start;
+        key[2 * i + 1] = spans[i].end;
     }
-    PrefillPlanHost plan;
-    int rc = plan_prefill(g, s->n, n_q, sa.data(), sb.data(), n_spans, c->num_sms, &plan,
-                          s->pages.data());
-    if (rc != SQ_OK) return rc;
     cudaStream_t st = as_stream(stream);
     cudaError_t e;
-    // upload: key tiles, per-CTA-tile counts, then the page of every piece
-    const size_t tb = plan.tiles.size() * sizeof(PrefillTile);
-    const size_t qb = plan.qt_tiles.size() * sizeof(int32_t);
-    const size_t pb = plan.tile_pages.size() * sizeof(int32_t);
-    if (c->staging.size() < tb + qb + pb) c->staging.resize(tb + qb + pb);
-    if (tb) std::memcpy(c->staging.data(), plan.tiles.data(), tb);
-    std::memcpy(c->staging.data() + tb, plan.qt_tiles.data(), qb);
-    if (pb) std::memcpy(c->staging.data() + tb + qb, plan.tile_pages.data(), pb);
-    UploadSlot& slot = c->slots[c->next_slot];
-    c->next_slot = (c->next_slot + 1) % kUploadSlots;
-    rc = upload(c, slot, c->staging.data(), tb + qb + pb, stream);
-    if (rc != SQ_OK) return rc;
+    PrefillPlanEntry* hit = nullptr;
+    for (auto& p : c->pre_plans)
+        if (p.valid && p.seq == seq && p.version == s->version && p.n_q == n_q &&
+            p.target == c->num_sms && p.spans == key) {
+            hit = &p;
+            break;
+        }
+    if (!hit) {
+        std::vector<int32_t> sa(n_spans), sb(n_spans);
+        for (int32_t i = 0; i < n_spans; ++i) {
+            sa[i] = key[2 * i];
+            sb[i] = key[2 * i + 1];
+        }
+        PrefillPlanHost plan;
+        int rc = plan_prefill(g, s->n, n_q, sa.data(), sb.data(), n_spans, c->num_sms, &plan,
+                              s->pages.data());
+        if (rc != SQ_OK) return rc;
+        // upload: key tiles, per-CTA-tile counts, then the page of every piece
+        const size_t tb = plan.tiles.size() * sizeof(PrefillTile);
+        const size_t qb = plan.qt_tiles.size() * sizeof(int32_t);
+        const size_t pb = plan.tile_pages.size() * sizeof(int32_t);
+        // least recently used entry
+        PrefillPlanEntry* victim = &c->pre_plans[0];
+        for (auto& p : c->pre_plans)
+            if (!p.valid || p.last_use < victim->last_use) victim = &p;
+        victim->valid = false;
+        if (!victim->ev) {
+            e = cudaEventCreateWithFlags(&victim->ev, cudaEventDisableTiming);
+            if (e != cudaSuccess) return cuda_status(e);
+        }
+        if (tb + qb + pb > victim->cap) {
+            if (victim->ev_recorded) cudaEventSynchronize(victim->ev);
+            if (victim->d) cudaFree(victim->d);
+            victim->d = nullptr;
+            victim->cap = 0;
+            victim->ev_recorded = false;
+            const size_t cap = std::max<size_t>((tb + qb + pb) * 5 / 4, 4096);
+            e = cudaMalloc(&victim->d, cap);
+            if (e != cudaSuccess) return cuda_status(e);
+            victim->cap = cap;
+        }
+        if (victim->ev_recorded) {
+            // the launches that read the old plan run before it is overwritten
+            e = cudaStreamWaitEvent(st, victim->ev, 0);
+            if (e != cudaSuccess) return cuda_status(e);
+        }
+        if (c->staging.size() < tb + qb + pb) c->staging.resize(tb + qb + pb);
+        if (tb) std::memcpy(c->staging.data(), plan.tiles.data(), tb);
+        std::memcpy(c->staging.data() + tb, plan.qt_tiles.data(), qb);
+        if (pb) std::memcpy(c->staging.data() + tb + qb, plan.tile_pages.data(), pb);
+        rc = staged_copy(c, victim->d, c->staging.data(), tb + qb + pb, stream);
+        if (rc != SQ_OK) return rc;
+        victim->seq = seq;
+        victim->version = s->version;
+        victim->n_q = n_q;
+        victim->target = c->num_sms;
+        victim->spans = key;
+        victim->tb = tb;
+        victim->qb = qb;
+        victim->n_tiles = (int32_t)plan.tiles.size();
+        victim->n_pieces = plan.n_pieces;
+        victim->BP = plan.BP;
+        victim->n_qt = plan.n_qt;
+        victim->n_split = plan.n_split;
+        victim->visible_pairs = plan.visible_pairs;
+        victim->valid = true;
+        hit = victim;
+    } else if (hit->ev_recorded) {
+        // its upload ran on the stream of the call that planned it
+        e = cudaStreamWaitEvent(st, hit->ev, 0);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    hit->last_use = ++c->use_clock;
+    const PrefillPlanEntry& plan = *hit;
     const int64_t grid = (int64_t)plan.n_qt * g.Hkv * plan.n_split;
     if (plan.n_split > 1) {
         const size_t need =
@@ -799,11 +883,11 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
         if (r != CUDA_SUCCESS) return SQ_ERR_INVALID_ARG;
     }
     PrefillArgs a;
-    a.tiles = reinterpret_cast<const PrefillTile*>(slot.d);
-    a.qt_tiles = reinterpret_cast<const int32_t*>(slot.d + tb);
-    a.tile_pages = reinterpret_cast<const int32_t*>(slot.d + tb + qb);
+    a.tiles = reinterpret_cast<const PrefillTile*>(plan.d);
+    a.qt_tiles = reinterpret_cast<const int32_t*>(plan.d + plan.tb);
+    a.tile_pages = reinterpret_cast<const int32_t*>(plan.d + plan.tb + plan.qb);
     a.n_pieces = plan.n_pieces;
-    a.n_tiles = (int32_t)plan.tiles.size();
+    a.n_tiles = plan.n_tiles;
     a.n = s->n;
     a.n_q = n_q;
     a.layer = layer;
@@ -848,9 +932,9 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
         if (e != cudaSuccess) return cuda_status(e);
         c->pre_ev_recorded = true;
     }
-    e = cudaEventRecord(slot.ev, st);
+    e = cudaEventRecord(hit->ev, st);
     if (e != cudaSuccess) return cuda_status(e);
-    slot.ev_recorded = true;
+    hit->ev_recorded = true;
     c->host->seq_mut(seq)->last_stream = stream;
     c->stats.prefill_calls += 1;
     c->stats.prefill_pairs += plan.visible_pairs;

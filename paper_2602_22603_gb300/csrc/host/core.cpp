@@ -2,6 +2,7 @@
 #include "core.hpp"
 
 #include <algorithm>
+#include <atomic>
 #include <cstring>
 #include <unordered_map>
 
@@ -79,7 +80,8 @@ bool PageAllocator::drop_ref(int32_t p) {
 }
 
 // ---------------------------------------------------------------------------
-static uint64_t g_version_counter = 1;
+// shared by every cache (of any thread): a version is never handed out twice
+static std::atomic<uint64_t> g_version_counter{1};
 
 HostCache::HostCache(const Geometry& g) : g_(g), alloc_(g.num_pages), seqs_(g.max_seqs) {
     free_slots_.reserve(g.max_seqs);

@@ -95,19 +95,37 @@ __device__ __forceinline__ uint32_t low_bits_through(int x) {
     return x >= 31 ? 0xffffffffu : (x < 0 ? 0u : ((2u << x) - 1u));
 }
 
-// The producer warp: both query tiles once, then K_j and V_j of every key tile
-// into the ring (load u = 2 j is K_j, u = 2 j + 1 is V_j, slot u mod kSlots).
-// The warp writes, for the key tiles of the next batch, a record of what the
-// copies need {first key, box mask, page of box 0, page of box 1} into a
-// double-buffered shared table half a batch ahead; lane 0 reads the record of
-// its next tile while the current one is in flight, so that between a free
-// slot and the copies that refill it there is only the barrier.  Boxes past
-// the second (pages of fewer than 64 tokens) take their page from global
-// memory.
+// Order of the K and V loads of a CTA's T key tiles, load u into ring slot
+// u mod kSlots.  Normally key tile by key tile: u = 2 j is K_j, u = 2 j + 1
+// is V_j.  In dual-key mode (tile a takes the even key tiles, tile b the odd
+// ones) the loads follow the order in which the MMA warp consumes them, so
+// that no tile waits in the ring for a later one: K_0, K_1, then V_j and
+// K_{j+2} in turn, and the last two V tiles.
+__device__ __forceinline__ void load_of(int u, int T, bool dual, int& j, int& kv) {
+    if (!dual) {
+        j = u >> 1;
+        kv = u & 1;
+    } else if (u < 2) {
+        j = u;
+        kv = 0;
+    } else if (u >= 2 * T - 2) {
+        j = u - T;
+        kv = 1;
+    } else {
+        j = ((u - 2) >> 1) + ((u & 1) ? 2 : 0);
+        kv = (u & 1) ? 0 : 1;
+    }
+}
+// The loads of K_j and V_j in dual-key mode (T >= 2).
+__device__ __forceinline__ int dual_load_k(int j) { return j < 2 ? j : 2 * j - 1; }
+__device__ __forceinline__ int dual_load_v(int j, int T) { return j < T - 1 ? 2 * j + 2 : 2 * T - 1; }
+
+// The producer warp: both query tiles once, then the K and V tiles of every
+// key tile into the ring in the order of load_of.
 template <int D>
 __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* qmap,
                                 const PrefillArgs& a, const Smem& sm, int g, int pos_lo, int t0,
-                                int T, volatile int* abort_flag, int lane) {
+                                int T, bool dual, volatile int* abort_flag, int lane) {
     using C = PreCfg<D>;
     if (lane == 0) {
         prefetch_tmap(pool_map);
@@ -141,59 +159,57 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
     };
     fill(0, 0);
     __syncwarp();
+    const int n_units = 2 * T;
+    int next_fill = 1;        // the record batch to fill next
     int issued = 0;
     int tail_u = -1;          // the load that used the fix-up barrier
     bool tail_done = false;   // ... and was handed over on its slot's barrier
     int4 rec = make_int4(0, 0, -1, -1);
-    if (lane == 0 && T > 0) rec = table[0];
-    for (int j = 0; j < T; ++j) {
-        // the next batch's records, half a batch ahead of their use
-        if (j % C::kMetaTiles == C::kMetaTiles / 2 && (j / C::kMetaTiles + 1) * C::kMetaTiles < T) {
-            fill((j / C::kMetaTiles + 1) * C::kMetaTiles, (j / C::kMetaTiles + 1) & 1);
+    if (lane == 0 && T > 0) rec = table[0];  // load 0 is of key tile 0 in both orders
+    int j = 0, kv = 0;
+    for (int u = 0; u < n_units; ++u) {
+        int jn = 0, kvn = 0;  // the next load's key tile
+        if (u + 1 < n_units) load_of(u + 1, T, dual, jn, kvn);
+        // the next batch's records, half a batch before their first use
+        if (u + 1 < n_units && next_fill * C::kMetaTiles < T &&
+            jn + C::kMetaTiles / 2 >= next_fill * C::kMetaTiles) {
+            fill(next_fill * C::kMetaTiles, next_fill & 1);
             __syncwarp();
+            ++next_fill;
         }
         const int key0 = __shfl_sync(0xffffffffu, rec.x, 0);
-        const bool tail = key0 + kPrefillKeys > a.n;
+        const bool vfix = kv == 1 && key0 + kPrefillKeys > a.n;
+        const int slot = u % C::kSlots;
+        const int use = u / C::kSlots;
         bool ok = true;
-        for (int kv = 0; kv < 2; ++kv) {
-            const int u = 2 * j + kv;
-            const int slot = u % C::kSlots;
-            const int use = u / C::kSlots;
-            if (lane == 0) {
-                if (use > 0)
-                    ok = mbar_wait(sm.bar<D>(C::kBarEmpty + slot), (use - 1) & 1, abort_flag);
-                if (ok) {
-                    const uint32_t pmask = (uint32_t)rec.y;
-                    const uint32_t bytes = (uint32_t)__popc(pmask) * br * 128 * C::kColBlocks;
-                    const bool vfix = kv == 1 && tail;
-                    const uint32_t fb =
-                        vfix ? sm.bar<D>(C::kBarVfix) : sm.bar<D>(C::kBarFull + slot);
-                    mbar_arrive_expect_tx(fb, bytes);
-                    const uint32_t dst = sm.base + C::kOffRing + slot * C::kSlotBytes;
-                    const int head_row = (kv ? a.Hkv + g : g) * a.P;
+        if (lane == 0) {
+            if (use > 0) ok = mbar_wait(sm.bar<D>(C::kBarEmpty + slot), (use - 1) & 1, abort_flag);
+            if (ok) {
+                const uint32_t pmask = (uint32_t)rec.y;
+                const uint32_t bytes = (uint32_t)__popc(pmask) * br * 128 * C::kColBlocks;
+                const uint32_t fb = vfix ? sm.bar<D>(C::kBarVfix) : sm.bar<D>(C::kBarFull + slot);
+                mbar_arrive_expect_tx(fb, bytes);
+                const uint32_t dst = sm.base + C::kOffRing + slot * C::kSlotBytes;
+                const int head_row = (kv ? a.Hkv + g : g) * a.P;
 #pragma unroll 1
-                    for (int i = 0; i < n_pieces; ++i) {
-                        if (!((pmask >> i) & 1u)) continue;
-                        const int key = key0 + i * br;
-                        const int32_t page =
-                            i == 0 ? rec.z
-                                   : (i == 1 ? rec.w
-                                             : __ldg(&a.tile_pages[(size_t)(t0 + j) * n_pieces + i]));
+                for (int i = 0; i < n_pieces; ++i) {
+                    if (!((pmask >> i) & 1u)) continue;
+                    const int key = key0 + i * br;
+                    const int32_t page =
+                        i == 0 ? rec.z
+                               : (i == 1 ? rec.w
+                                         : __ldg(&a.tile_pages[(size_t)(t0 + j) * n_pieces + i]));
 #pragma unroll
-                        for (int cb = 0; cb < C::kColBlocks; ++cb)
-                            tma_load_4d(dst + cb * C::kBlockBytes + i * br * 128, pool_map, fb,
-                                        cb * 64, head_row + key % a.P, page, a.layer);
-                    }
-                    // the next tile's record, read while these copies are in flight
-                    if (kv == 1 && j + 1 < T)
-                        rec = table[((j + 1) / C::kMetaTiles & 1) * C::kMetaTiles +
-                                    (j + 1) % C::kMetaTiles];
+                    for (int cb = 0; cb < C::kColBlocks; ++cb)
+                        tma_load_4d(dst + cb * C::kBlockBytes + i * br * 128, pool_map, fb,
+                                    cb * 64, head_row + key % a.P, page, a.layer);
                 }
+                // the next load's record, read while these copies are in flight
+                if (u + 1 < n_units && jn != j)
+                    rec = table[(jn / C::kMetaTiles & 1) * C::kMetaTiles + jn % C::kMetaTiles];
             }
-            ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-            if (!ok) break;
-            issued = u + 1;
         }
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
         if (!ok) {
             if (lane == 0) {
                 set_error(a.err, kErrTimeout);
@@ -201,11 +217,11 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
             }
             break;
         }
-        if (tail) {
-            // The last key tile: its V rows past the sequence's end hold stale
-            // or never-written data.  Their weights are zero, but 0 * NaN is
-            // not, so zero those rows before the MMAs read the slot.
-            const int u = 2 * j + 1, slot = u % C::kSlots;
+        issued = u + 1;
+        if (vfix) {
+            // V of the last key tile: its rows past the sequence's end hold
+            // stale or never-written data.  Their weights are zero, but 0 * NaN
+            // is not, so zero those rows before the MMAs read the slot.
             tail_u = u;
             if (lane == 0) ok = mbar_wait(sm.bar<D>(C::kBarVfix), 0, abort_flag);
             if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) {
@@ -227,6 +243,8 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
             if (lane == 0) mbar_arrive(sm.bar<D>(C::kBarFull + slot));
             tail_done = true;
         }
+        j = jn;
+        kv = kvn;
     }
     // Drain: every copy this CTA issued lands before the CTA exits (immediate
     // unless a consumer gave up early).
@@ -271,43 +289,40 @@ __device__ __forceinline__ void issue_pv(const Smem& sm, uint32_t tmem, int t, i
 
 // Dual-key mode (every query of the CTA tile fits in tile a): both tiles
 // hold tile a's queries; tile a takes key tiles 0, 2, 4, ... and tile b the
-// odd ones, and the two results are merged at the end.
+// odd ones, and the two results are merged at the end.  Key tile j's PV and
+// the QK of key tile j + 2 (into the same S columns) are issued in the order
+// of the loads, each as soon as its tile has landed.
 template <int D>
 __device__ bool prefill_mma_dual(const Smem& sm, uint32_t tmem, int T, volatile int* abort_flag) {
     using C = PreCfg<D>;
-    const int Tt[2] = {(T + 1) / 2, T / 2};
     bool ok = true;
     for (int t = 0; t < 2 && ok; ++t) {
-        // S_t(0) = Q_a K_t
-        const int u = 2 * t, slot = u % C::kSlots;
+        // S_t = Q_a K_t
+        const int u = dual_load_k(t), slot = u % C::kSlots;
         if (!(ok = mbar_wait(sm.bar<D>(C::kBarFull + slot), (u / C::kSlots) & 1, abort_flag))) break;
         issue_qk<D>(sm, tmem, t, slot, 0);
         mma_commit(sm.bar<D>(C::kBarS + t));
         mma_commit(sm.bar<D>(C::kBarEmpty + slot));
     }
-    for (int i = 0; ok && i < Tt[0]; ++i) {
-        for (int t = 0; t < 2; ++t) {
-            if (i >= Tt[t]) break;
-            const int j = 2 * i + t;  // key tile of this step
-            const int uv = 2 * j + 1, vslot = uv % C::kSlots;
-            const int uk = 2 * j + 4, kslot = uk % C::kSlots;  // K of key tile j + 2
-            const bool more = i + 1 < Tt[t];
-            if (!(ok = mbar_wait(sm.bar<D>(C::kBarFull + vslot), (uv / C::kSlots) & 1, abort_flag)))
-                break;
-            if (more && !(ok = mbar_wait(sm.bar<D>(C::kBarFull + kslot), (uk / C::kSlots) & 1,
-                                         abort_flag)))
-                break;
-            if (!(ok = mbar_wait(sm.bar<D>(C::kBarP + t), i & 1, abort_flag))) break;
-            tc_fence_after();
-            issue_pv<D>(sm, tmem, t, vslot, i == 0);
-            mma_commit(sm.bar<D>(C::kBarEmpty + vslot));
-            if (!more) mma_commit(sm.bar<D>(C::kBarO + t));
-            if (more) {
-                issue_qk<D>(sm, tmem, t, kslot, 0);
-                mma_commit(sm.bar<D>(C::kBarS + t));
-                mma_commit(sm.bar<D>(C::kBarEmpty + kslot));
-            }
+    for (int j = 0; ok && j < T; ++j) {
+        const int t = j & 1, i = j >> 1;
+        const int uv = dual_load_v(j, T), vslot = uv % C::kSlots;
+        if (!(ok = mbar_wait(sm.bar<D>(C::kBarFull + vslot), (uv / C::kSlots) & 1, abort_flag)))
+            break;
+        if (!(ok = mbar_wait(sm.bar<D>(C::kBarP + t), i & 1, abort_flag))) break;
+        tc_fence_after();
+        issue_pv<D>(sm, tmem, t, vslot, i == 0);
+        mma_commit(sm.bar<D>(C::kBarEmpty + vslot));
+        if (j + 2 >= T) {  // the last key tile of tile t
+            mma_commit(sm.bar<D>(C::kBarO + t));
+            continue;
         }
+        const int uk = dual_load_k(j + 2), kslot = uk % C::kSlots;
+        if (!(ok = mbar_wait(sm.bar<D>(C::kBarFull + kslot), (uk / C::kSlots) & 1, abort_flag)))
+            break;
+        issue_qk<D>(sm, tmem, t, kslot, 0);
+        mma_commit(sm.bar<D>(C::kBarS + t));
+        mma_commit(sm.bar<D>(C::kBarEmpty + kslot));
     }
     return ok;
 }
@@ -723,6 +738,8 @@ __global__ void __launch_bounds__(320, 1)
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sm.ptr + C::kOffMisc + 4);
     int* sched = reinterpret_cast<int*>(sm.ptr + C::kOffMisc + 8);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // the split-merging kernel that follows may be scheduled from here on
+    grid_launch_dependents();
     // heaviest CTA tiles (latest positions) first
     const int split = blockIdx.x % a.n_split;
     const int rest = blockIdx.x / a.n_split;
@@ -764,7 +781,7 @@ __global__ void __launch_bounds__(320, 1)
     const bool two = pos_lo + a.BP < a.n_q;
     const bool dual = !two && T >= 2;
     if (warp == 0) {
-        prefill_produce<D>(&pool_map, &qmap, a, sm, g, pos_lo, t0, T, abort_flag, lane);
+        prefill_produce<D>(&pool_map, &qmap, a, sm, g, pos_lo, t0, T, dual, abort_flag, lane);
     } else if (warp == 1) {
         if (lane == 0) prefill_mma<D>(a, sm, tmem, T, two, dual, abort_flag);
         __syncwarp();
@@ -781,9 +798,15 @@ __global__ void __launch_bounds__(320, 1)
 }
 
 // Merges the key-range splits of each query row: weights 2^(lse_s - max).
-// One warp per (CTA tile, query tile, row).
+// One warp per (CTA tile, query tile, row); the lanes take the splits' log-sum-
+// exps (up to 64 splits), then the partial outputs go through in batches of 8
+// whose loads are in flight together.
 template <int D>
 __global__ void __launch_bounds__(256) sq_prefill_combine_kernel(const PrefillCombineArgs a) {
+    constexpr int V = D / 32;  // output elements per lane
+    constexpr int U = 8;       // splits per batch of loads
+    // programmatic dependent of the prefill kernel: wait for its partials
+    grid_dependency_wait();
     const int gw = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
     const int lane = threadIdx.x & 31;
     const int units = a.n_qt * a.Hkv;
@@ -795,33 +818,70 @@ __global__ void __launch_bounds__(256) sq_prefill_combine_kernel(const PrefillCo
     const int qi = (qt * kPrefillQTiles + t) * a.BP + row / a.G;
     if (row >= a.BP * a.G || qi >= a.n_q) return;
     const int h = g * a.G + row % a.G;
-    auto part = [&](int s) {
-        return (((size_t)rest * a.n_split + s) * kPrefillQTiles + t) * kPrefillRows + row;
-    };
-    float M = -INFINITY;
-    for (int s = 0; s < a.n_split; ++s) M = fmaxf(M, a.part_ml[part(s)]);
-    float W = 0.f, acc[D / 32];
+    // partial row of split s: part0 + s * kRowsPerUnit
+    const size_t part0 = ((size_t)rest * a.n_split * kPrefillQTiles + t) * kPrefillRows + row;
+    const float ml0 = lane < a.n_split ? a.part_ml[part0 + (size_t)lane * kRowsPerUnit] : -INFINITY;
+    const float ml1 =
+        lane + 32 < a.n_split ? a.part_ml[part0 + (size_t)(lane + 32) * kRowsPerUnit] : -INFINITY;
+    float M = fmaxf(ml0, ml1);
 #pragma unroll
-    for (int e = 0; e < D / 32; ++e) acc[e] = 0.f;
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    float w0 = 0.f, w1 = 0.f;
     if (M != -INFINITY) {
-        for (int s = 0; s < a.n_split; ++s) {
-            const size_t pr = part(s);
-            const float ml = a.part_ml[pr];
-            if (ml == -INFINITY) continue;
-            const float w = exp2f(ml - M);
-            W += w;
-            const float* po = a.part_o + pr * D;
+        if (ml0 != -INFINITY) w0 = exp2f(ml0 - M);
+        if (ml1 != -INFINITY) w1 = exp2f(ml1 - M);
+    }
+    float W = w0 + w1;
 #pragma unroll
-            for (int e = 0; e < D / 32; ++e) acc[e] += w * po[lane + 32 * e];
+    for (int off = 16; off > 0; off >>= 1) W += __shfl_xor_sync(0xffffffffu, W, off);
+    float acc[V];
+#pragma unroll
+    for (int e = 0; e < V; ++e) acc[e] = 0.f;
+    for (int s0 = 0; W > 0.f && s0 < a.n_split; s0 += U) {
+        float w[U];
+        float vals[U][V];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int s = s0 + u;  // the same in every lane
+            const float ws = __shfl_sync(0xffffffffu, s < 32 ? w0 : w1, s & 31);
+            w[u] = s < a.n_split ? ws : 0.f;
+#pragma unroll
+            for (int e = 0; e < V; ++e) vals[u][e] = 0.f;
+            if (w[u] > 0.f) {  // an empty split's partial is not read
+                const float* po = a.part_o + (part0 + (size_t)s * kRowsPerUnit) * D + lane * V;
+                if constexpr (V == 4) {
+                    const float4 v = *reinterpret_cast<const float4*>(po);
+                    vals[u][0] = v.x; vals[u][1] = v.y; vals[u][2] = v.z; vals[u][3] = v.w;
+                } else {
+                    const float2 v = *reinterpret_cast<const float2*>(po);
+                    vals[u][0] = v.x; vals[u][1] = v.y;
+                }
+            }
         }
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+#pragma unroll
+            for (int e = 0; e < V; ++e) acc[e] += w[u] * vals[u][e];
     }
     const float inv = W > 0.f ? 1.f / W : 0.f;
-    const size_t o = ((size_t)qi * a.Hq + h) * D;
-#pragma unroll
-    for (int e = 0; e < D / 32; ++e) {
-        const float v = acc[e] * inv;
-        if (a.out_f32) reinterpret_cast<float*>(a.out)[o + lane + 32 * e] = v;
-        else reinterpret_cast<__nv_bfloat16*>(a.out)[o + lane + 32 * e] = __float2bfloat16_rn(v);
+    const size_t o = ((size_t)qi * a.Hq + h) * D + lane * V;
+    if (a.out_f32) {
+        float* out = reinterpret_cast<float*>(a.out) + o;
+        if constexpr (V == 4)
+            *reinterpret_cast<float4*>(out) =
+                make_float4(acc[0] * inv, acc[1] * inv, acc[2] * inv, acc[3] * inv);
+        else
+            *reinterpret_cast<float2*>(out) = make_float2(acc[0] * inv, acc[1] * inv);
+    } else {
+        __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.out) + o;
+        if constexpr (V == 4) {
+            uint2 u;
+            u.x = pack_bf16x2(acc[0] * inv, acc[1] * inv);
+            u.y = pack_bf16x2(acc[2] * inv, acc[3] * inv);
+            *reinterpret_cast<uint2*>(out) = u;
+        } else {
+            *reinterpret_cast<uint32_t*>(out) = pack_bf16x2(acc[0] * inv, acc[1] * inv);
+        }
     }
     if (lane == 0 && a.lse)
         a.lse[(size_t)qi * a.Hq + h] = W > 0.f ? (M + __log2f(W)) * 0.69314718055994531f : -INFINITY;
@@ -861,9 +921,18 @@ cudaError_t launch_prefill_combine(const PrefillCombineArgs& a, int D, cudaStrea
     const int64_t warps = (int64_t)a.n_qt * a.Hkv * kPrefillQTiles * kPrefillRows;
     const unsigned grid = (unsigned)((warps * 32 + 255) / 256);
     if (grid == 0) return cudaSuccess;
-    if (D == 128) dev::sq_prefill_combine_kernel<128><<<grid, 256, 0, st>>>(a);
-    else dev::sq_prefill_combine_kernel<64><<<grid, 256, 0, st>>>(a);
-    return cudaGetLastError();
+    // scheduled while the prefill kernel's last CTAs run; waits for them
+    cudaLaunchAttribute at;
+    at.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at.val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cfg.attrs = &at;
+    cfg.numAttrs = 1;
+    if (D == 128) return cudaLaunchKernelEx(&cfg, dev::sq_prefill_combine_kernel<128>, a);
+    return cudaLaunchKernelEx(&cfg, dev::sq_prefill_combine_kernel<64>, a);
 }
 
 }  // namespace sq

@@ -223,3 +223,33 @@ def test_prefill_short_block_dual_key_split(n, n_q, spans):
         check(p, h, 0, n_q, spans, seed=n + 2, out_dtype=sq.SQ_OUT_BF16)
     finally:
         p.close()
+
+
+def test_prefill_plan_reuse_follows_sequence_changes():
+    # a plan is reused across layers while the sequence, the query count and
+    # the spans are unchanged; every change (append, n_q, spans, eviction, a
+    # fork's copy-on-write) gives a new one, and more distinct plans than the
+    # cache holds cycle through it
+    p = Pair(2, 16, 4, 64, 16, num_pages=120, seed=12)
+    try:
+        h = p.seq_new()
+        p.append(h, 700)
+        s1, s2 = [(40, 90), (300, 420)], [(0, 10), (500, 650)]
+        check(p, h, 0, 100, s1, seed=1)
+        check(p, h, 1, 100, s1, seed=2)
+        p.append(h, 50)
+        check(p, h, 0, 100, s1, seed=3)
+        check(p, h, 0, 120, s1, seed=4)
+        check(p, h, 1, 120, s2, seed=5)
+        p.evict(h, [(200, 260)])
+        check(p, h, 0, 80, [], seed=6)
+        a = p.fork(h)
+        p.append(a, 10)
+        for layer in (0, 1):
+            check(p, a, layer, 30, [(5, 25)], seed=7 + layer)
+            check(p, h, layer, 30, [(5, 25)], seed=9 + layer)
+        for rep in range(2):
+            for n_q in (1, 7, 33, 64, 65, 129):
+                check(p, h, rep, n_q, s2, seed=20 + n_q)
+    finally:
+        p.close()
