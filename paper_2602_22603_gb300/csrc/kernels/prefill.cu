@@ -64,12 +64,8 @@ struct PreCfg {
     static constexpr int kBarDone = kBarVfix + 1;       // every MMA of the CTA done
     static constexpr int kNumBars = kBarDone + 1;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
-    // producer's double-buffered table of key-tile records (int4 each)
-    static constexpr int kMetaTiles = 16;
-    static constexpr int kOffMeta = (kOffMisc + 32 + 15) & ~15;  // int4 records: 16-byte aligned
-    static constexpr int kMetaBytes = 2 * kMetaTiles * 16;
     // dual-key mode: tile b's (max, normaliser) of each row, for the merge
-    static constexpr int kOffXchg = kOffMeta + kMetaBytes;
+    static constexpr int kOffXchg = (kOffMisc + 32 + 15) & ~15;
     static constexpr int kSmemBytes = kOffXchg + kPrefillRows * 8 + 1024;  // + alignment slack
     static constexpr uint32_t kTmemCols = 512;
     static constexpr uint32_t kColS = 0;    // S_t (fp32) at 128 t; P_t (bf16 pairs) over its first 64
@@ -77,7 +73,7 @@ struct PreCfg {
     static constexpr uint32_t kIdescQK = mma_idesc_bf16(128, kPrefillKeys, false);
     static constexpr uint32_t kIdescPV = mma_idesc_bf16(128, D, true);
     static_assert(kSmemBytes <= 232448, "shared memory");
-    static_assert(kOffMeta % 16 == 0 && kOffRing % 1024 == 0 && kOffBar % 8 == 0, "alignment");
+    static_assert(kOffXchg % 16 == 0 && kOffRing % 1024 == 0 && kOffBar % 8 == 0, "alignment");
     static_assert(kPrefillQTiles == 2, "two query tiles per CTA");
 };
 
@@ -120,109 +116,122 @@ __device__ __forceinline__ void load_of(int u, int T, bool dual, int& j, int& kv
 __device__ __forceinline__ int dual_load_k(int j) { return j < 2 ? j : 2 * j - 1; }
 __device__ __forceinline__ int dual_load_v(int j, int T) { return j < T - 1 ? 2 * j + 2 : 2 * T - 1; }
 
-// The producer warp: both query tiles once, then the K and V tiles of every
-// key tile into the ring in the order of load_of.
+// The producer warp: the query tiles once, then the K and V tiles of every key
+// tile into the ring in the order of load_of, two loads at a time: lanes 0
+// and 1 wait for their slots, arm their barriers and issue their copies
+// together, so that the shared-memory round trips of the two overlap.  What a
+// tile's copies need, {first key, page of box 0, page of box 1}, is held in
+// registers: lane l has the record of the window's key tile j = l (mod 32),
+// batches of 16 tiles alternating between the lower and the upper half-warp;
+// a batch is read from global memory about ten tiles before its first use and
+// moved into place a few tiles before it.  Boxes past the second (pages of
+// fewer than 64 tokens) take their page from global memory.
 template <int D>
 __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* qmap,
                                 const PrefillArgs& a, const Smem& sm, int g, int pos_lo, int t0,
-                                int T, bool dual, volatile int* abort_flag, int lane) {
+                                int T, bool two, bool dual, volatile int* abort_flag, int lane) {
     using C = PreCfg<D>;
     if (lane == 0) {
         prefetch_tmap(pool_map);
         prefetch_tmap(qmap);
-        mbar_arrive_expect_tx(sm.bar<D>(C::kBarQ),
-                              kPrefillQTiles * C::kColBlocks * a.BP * a.G * 128);
-        for (int t = 0; t < kPrefillQTiles; ++t)
+        const int nq = two ? 2 : 1;  // tile b is loaded only when it holds queries
+        mbar_arrive_expect_tx(sm.bar<D>(C::kBarQ), nq * C::kColBlocks * a.BP * a.G * 128);
+        for (int t = 0; t < nq; ++t)
             for (int cb = 0; cb < C::kColBlocks; ++cb)
                 tma_load_3d(sm.base + C::kOffQ + t * C::kQBytes + cb * C::kBlockBytes, qmap,
                             sm.bar<D>(C::kBarQ), cb * 64, g * a.G, pos_lo + t * a.BP);
     }
     const int br = a.P < 64 ? a.P : 64;  // rows of one TMA box
     const int n_pieces = a.n_pieces;      // <= 16
-    int4* table = reinterpret_cast<int4*>(sm.ptr + C::kOffMeta);  // [2][kMetaTiles]
-    // records of tiles [tb, tb + kMetaTiles) into table half `half`
-    auto fill = [&](int tb, int half) {
-        if (lane < C::kMetaTiles && tb + lane < T) {
-            const int t = t0 + tb + lane;
-            const int key0 = __ldg(&a.tiles[t].key0);
-            uint32_t pmask = 0;
-            int p0 = -1, p1 = -1;
-            for (int i = 0; i < n_pieces && key0 + i * br < a.n; ++i) {
-                const int32_t page = __ldg(&a.tile_pages[(size_t)t * n_pieces + i]);
-                if ((uint32_t)page < (uint32_t)a.num_pages) pmask |= 1u << i;
-                else set_error(a.err, kErrBounds);
-                if (i == 0) p0 = page;
-                if (i == 1) p1 = page;
-            }
-            table[half * C::kMetaTiles + lane] = make_int4(key0, (int)pmask, p0, p1);
+    constexpr int kBatch = 16;
+    // {first key, page of box 0, page of box 1} of key tile tb + lane % 16
+    auto load_rec = [&](int tb) {
+        int4 r = make_int4(0, -1, -1, 0);
+        const int jj = tb + (lane & (kBatch - 1));
+        if (jj < T) {
+            const size_t t = (size_t)(t0 + jj);
+            r.x = __ldg(&a.tiles[t].key0);
+            r.y = __ldg(&a.tile_pages[t * n_pieces]);
+            if (n_pieces > 1) r.z = __ldg(&a.tile_pages[t * n_pieces + 1]);
         }
+        return r;
     };
-    fill(0, 0);
-    __syncwarp();
+    int4 rec = make_int4(0, -1, -1, 0), pend = rec;
+    if (lane < kBatch) rec = load_rec(0);
+    int fill_b = 1;    // the next batch to read
+    int merge_b = -1;  // the batch read into `pend`, not yet in place
     const int n_units = 2 * T;
-    int next_fill = 1;        // the record batch to fill next
     int issued = 0;
     int tail_u = -1;          // the load that used the fix-up barrier
     bool tail_done = false;   // ... and was handed over on its slot's barrier
-    int4 rec = make_int4(0, 0, -1, -1);
-    if (lane == 0 && T > 0) rec = table[0];  // load 0 is of key tile 0 in both orders
-    int j = 0, kv = 0;
-    for (int u = 0; u < n_units; ++u) {
-        int jn = 0, kvn = 0;  // the next load's key tile
-        if (u + 1 < n_units) load_of(u + 1, T, dual, jn, kvn);
-        // the next batch's records, half a batch before their first use
-        if (u + 1 < n_units && next_fill * C::kMetaTiles < T &&
-            jn + C::kMetaTiles / 2 >= next_fill * C::kMetaTiles) {
-            fill(next_fill * C::kMetaTiles, next_fill & 1);
-            __syncwarp();
-            ++next_fill;
+    for (int u0 = 0; u0 < n_units; u0 += 2) {  // n_units is even
+        int j0, kv0, j1, kv1;
+        load_of(u0, T, dual, j0, kv0);
+        load_of(u0 + 1, T, dual, j1, kv1);
+        const int jmax = j0 > j1 ? j0 : j1;
+        if (merge_b >= 0 && jmax + 4 >= kBatch * merge_b) {
+            if ((lane >> 4) == (merge_b & 1)) rec = pend;
+            merge_b = -1;
         }
-        const int key0 = __shfl_sync(0xffffffffu, rec.x, 0);
-        const bool vfix = kv == 1 && key0 + kPrefillKeys > a.n;
+        if (merge_b < 0 && fill_b * kBatch < T && jmax + 10 >= kBatch * fill_b) {
+            if ((lane >> 4) == (fill_b & 1)) pend = load_rec(fill_b * kBatch);
+            merge_b = fill_b++;
+        }
+        const int u = u0 + (lane & 1);  // lanes 0 and 1 issue
+        const int j = (lane & 1) ? j1 : j0, kv = (lane & 1) ? kv1 : kv0;
+        const int key0 = __shfl_sync(0xffffffffu, rec.x, j & 31);
+        const int pg0 = __shfl_sync(0xffffffffu, rec.y, j & 31);
+        const int pg1 = __shfl_sync(0xffffffffu, rec.z, j & 31);
         const int slot = u % C::kSlots;
         const int use = u / C::kSlots;
+        const bool vfix = lane < 2 && kv == 1 && key0 + kPrefillKeys > a.n;
         bool ok = true;
-        if (lane == 0) {
-            if (use > 0) ok = mbar_wait(sm.bar<D>(C::kBarEmpty + slot), (use - 1) & 1, abort_flag);
-            if (ok) {
-                const uint32_t pmask = (uint32_t)rec.y;
-                const uint32_t bytes = (uint32_t)__popc(pmask) * br * 128 * C::kColBlocks;
-                const uint32_t fb = vfix ? sm.bar<D>(C::kBarVfix) : sm.bar<D>(C::kBarFull + slot);
-                mbar_arrive_expect_tx(fb, bytes);
-                const uint32_t dst = sm.base + C::kOffRing + slot * C::kSlotBytes;
-                const int head_row = (kv ? a.Hkv + g : g) * a.P;
-#pragma unroll 1
-                for (int i = 0; i < n_pieces; ++i) {
-                    if (!((pmask >> i) & 1u)) continue;
-                    const int key = key0 + i * br;
-                    const int32_t page =
-                        i == 0 ? rec.z
-                               : (i == 1 ? rec.w
-                                         : __ldg(&a.tile_pages[(size_t)(t0 + j) * n_pieces + i]));
-#pragma unroll
-                    for (int cb = 0; cb < C::kColBlocks; ++cb)
-                        tma_load_4d(dst + cb * C::kBlockBytes + i * br * 128, pool_map, fb,
-                                    cb * 64, head_row + key % a.P, page, a.layer);
-                }
-                // the next load's record, read while these copies are in flight
-                if (u + 1 < n_units && jn != j)
-                    rec = table[(jn / C::kMetaTiles & 1) * C::kMetaTiles + jn % C::kMetaTiles];
-            }
-        }
-        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-        if (!ok) {
+        if (lane < 2 && use > 0)
+            ok = mbar_wait(sm.bar<D>(C::kBarEmpty + slot), (use - 1) & 1, abort_flag);
+        // both slots free, or neither load is issued
+        if (!__all_sync(0xffffffffu, ok)) {
             if (lane == 0) {
                 set_error(a.err, kErrTimeout);
                 *abort_flag = 1;
             }
             break;
         }
-        issued = u + 1;
-        if (vfix) {
+        if (lane < 2) {
+            int nv = (a.n - key0 + br - 1) / br;  // boxes inside the sequence
+            nv = nv < n_pieces ? nv : n_pieces;
+            const uint32_t fb = vfix ? sm.bar<D>(C::kBarVfix) : sm.bar<D>(C::kBarFull + slot);
+            mbar_arrive_expect_tx(fb, (uint32_t)nv * br * 128 * C::kColBlocks);
+            const uint32_t dst = sm.base + C::kOffRing + slot * C::kSlotBytes;
+            const int head_row = (kv ? a.Hkv + g : g) * a.P;
+#pragma unroll 1
+            for (int i = 0; i < nv; ++i) {
+                int32_t page =
+                    i == 0 ? pg0
+                           : (i == 1 ? pg1
+                                     : __ldg(&a.tile_pages[(size_t)(t0 + j) * n_pieces + i]));
+                if ((uint32_t)page >= (uint32_t)a.num_pages) {
+                    // a page outside the pool: flagged; the box is read from
+                    // page 0 so that the barrier's byte count still completes
+                    set_error(a.err, kErrBounds);
+                    page = 0;
+                }
+                const int key = key0 + i * br;
+#pragma unroll
+                for (int cb = 0; cb < C::kColBlocks; ++cb)
+                    tma_load_4d(dst + cb * C::kBlockBytes + i * br * 128, pool_map, fb, cb * 64,
+                                head_row + key % a.P, page, a.layer);
+            }
+        }
+        issued = u0 + 2;
+        const uint32_t fix = __ballot_sync(0xffffffffu, vfix);
+        if (fix) {
             // V of the last key tile: its rows past the sequence's end hold
             // stale or never-written data.  Their weights are zero, but 0 * NaN
             // is not, so zero those rows before the MMAs read the slot.
-            tail_u = u;
+            const int src = __ffs(fix) - 1;
+            const int fslot = __shfl_sync(0xffffffffu, slot, src);
+            const int fkey0 = __shfl_sync(0xffffffffu, key0, src);
+            tail_u = u0 + src;
             if (lane == 0) ok = mbar_wait(sm.bar<D>(C::kBarVfix), 0, abort_flag);
             if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) {
                 if (lane == 0) {
@@ -231,20 +240,18 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
                 }
                 break;
             }
-            const int r0 = a.n - key0;  // 1 .. 127
+            const int r0 = a.n - fkey0;  // 1 .. 127
             const int chunks = (kPrefillKeys - r0) * 8;
-            uint8_t* vsp = sm.ptr + C::kOffRing + slot * C::kSlotBytes;
+            uint8_t* vsp = sm.ptr + C::kOffRing + fslot * C::kSlotBytes;
             for (int cb = 0; cb < C::kColBlocks; ++cb)
                 for (int c = lane; c < chunks; c += 32)
                     *reinterpret_cast<uint4*>(vsp + cb * C::kBlockBytes + (r0 + (c >> 3)) * 128 +
                                               (c & 7) * 16) = make_uint4(0, 0, 0, 0);
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) mbar_arrive(sm.bar<D>(C::kBarFull + slot));
+            if (lane == 0) mbar_arrive(sm.bar<D>(C::kBarFull + fslot));
             tail_done = true;
         }
-        j = jn;
-        kv = kvn;
     }
     // Drain: every copy this CTA issued lands before the CTA exits (immediate
     // unless a consumer gave up early).
@@ -781,7 +788,7 @@ __global__ void __launch_bounds__(320, 1)
     const bool two = pos_lo + a.BP < a.n_q;
     const bool dual = !two && T >= 2;
     if (warp == 0) {
-        prefill_produce<D>(&pool_map, &qmap, a, sm, g, pos_lo, t0, T, dual, abort_flag, lane);
+        prefill_produce<D>(&pool_map, &qmap, a, sm, g, pos_lo, t0, T, two, dual, abort_flag, lane);
     } else if (warp == 1) {
         if (lane == 0) prefill_mma<D>(a, sm, tmem, T, two, dual, abort_flag);
         __syncwarp();
