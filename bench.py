@@ -36,6 +36,7 @@ if ROOT not in sys.path:
 
 METRIC = "decode-attn tokens/s + achieved HBM GB/s at 128k ctx; span-evict GB/s"
 PREFILL_METRIC = "masked-prefill attention tokens/s at 32k ctx (all layers) + achieved bf16 TFLOP/s"
+AUX_METRIC = "aux-thread trigger prefill: K/V GB/s read over a 128k shared context (all layers)"
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -46,8 +47,12 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="sq", choices=["sq", "reference"])
     ap.add_argument("--workload", default="serving-128k",
-                    choices=["serving-128k", "large-ragged", "agent-32k", "trace", "prefill-32k"])
+                    choices=["serving-128k", "large-ragged", "agent-32k", "trace", "prefill-32k",
+                             "aux-trigger-128k"])
     ap.add_argument("--prefill-ctx", type=int, default=32768, help="prefill-32k: context tokens")
+    ap.add_argument("--aux-ctx", type=int, default=131072, help="aux-trigger-128k: context tokens")
+    ap.add_argument("--aux-queries", type=int, default=8,
+                    help="aux-trigger-128k: trigger-phrase tokens the aux thread prefills")
     ap.add_argument("--turns", type=int, default=50, help="trace: turns per agent")
     ap.add_argument("--requests", type=int, default=8)
     ap.add_argument("--ctx", type=int, default=131072)
@@ -99,10 +104,11 @@ def sources_hash(kernel: str) -> str:
     return m.hexdigest()[:16]
 
 
-def recorded_traffic_ratio(kernel: str):
+def recorded_traffic_ratio(kernel: str, workload: str = None):
     """DRAM traffic per algorithmic byte from the ncu capture summarised in
     profiles/, if that capture was taken of the current kernel sources
-    (else None)."""
+    (else None).  A kernel captured under several workloads tags each line
+    with `workload=`."""
     import re
     pdir = os.path.join(ROOT, "profiles")
     if not os.path.isdir(pdir):
@@ -113,9 +119,10 @@ def recorded_traffic_ratio(kernel: str):
             continue
         with open(os.path.join(pdir, name)) as f:
             for line in f:
-                mt = re.search(r"traffic: kernel=(\S+) ratio=([0-9.]+) sources_sha256=([0-9a-f]+)", line)
-                if mt and mt.group(1) == kernel and mt.group(3) == cur:
-                    return float(mt.group(2)), "profiles/" + name
+                mt = re.search(r"traffic: kernel=(\S+)(?: workload=(\S+))? ratio=([0-9.]+) "
+                               r"sources_sha256=([0-9a-f]+)", line)
+                if mt and mt.group(1) == kernel and mt.group(2) == workload and mt.group(4) == cur:
+                    return float(mt.group(3)), "profiles/" + name
     return None, None
 
 
@@ -921,7 +928,7 @@ def run_prefill(args, world, rank, local):
     achieved = flops / (mean_call / 1e3) / 1e12
     peak, peak_kind = tensor_peak()
     value = world * n * K / (total_ms / 1e3)
-    ratio, ratio_src = recorded_traffic_ratio("sq_prefill_kernel")
+    ratio, ratio_src = recorded_traffic_ratio("sq_prefill_kernel", "prefill-32k")
     kv_bytes = n * Hkv * D * 2 * 2                    # K and V of one layer
     res = {
         "metric": PREFILL_METRIC,
@@ -1042,6 +1049,205 @@ def prefill_cpu_baseline(bank, offs, sizes, q_offs, spans, L, Hq, Hkv, D, n, sca
             "cores": oatt.num_threads(), "kind": "oracle", "cpu_model": cpu_model(),
             "sample": f"the last {n_sample} queries of the {n}-token context, all {Hq} heads, at "
                       f"{len(layers)} of {L} layers; tokens/s = queries / (seconds per layer x {L})",
+            "seconds": round(total, 3)}
+
+
+def run_aux_trigger(args, world, rank, local):
+    """The auxiliary thread's spawn (Algorithm 1, Phase 2): fork the main
+    thread's 131,072-token context (8B-class GQA, 32 layers), append the
+    trigger phrase (8 tokens by default) and run its masked prefill over the
+    whole shared context at every layer, then release the fork.  One step =
+    one such spawn; the prefill reads every K/V row of the context once per
+    layer, so it is bound by HBM."""
+    import torch
+
+    import paper_2602_22603_gb300 as sq
+    from synthetic import AGENT_8B, Bank, sub_seed
+    torch.cuda.set_device(local)
+    sh = AGENT_8B
+    L, Hq, Hkv, D, P = args.layers, sh.num_q_heads, sh.num_kv_heads, sh.head_dim, sh.page_size
+    n0, n_q = args.aux_ctx, args.aux_queries
+    n = n0 + n_q
+    seed = args.seed + 1000 * rank
+    scale = 1.0 / math.sqrt(D)
+    cache = sq.Cache(L, Hq, Hkv, D, P, n // P + 64, max_seqs=4)
+    bank = Bank(1 << 28, sub_seed(seed, 1), device="cuda")
+    chunk = 4096
+    sizes = [chunk] * (n0 // chunk) + ([n0 % chunk] if n0 % chunk else [])
+    offs = bank.offsets(2 * len(sizes) + 2, L * chunk * Hkv * D, sub_seed(seed, 2))
+    m = cache.seq_new()
+    for i, c in enumerate(sizes):
+        cache.append_kv(m, c, bank.view(offs[2 * i], (L, c, Hkv, D)),
+                        bank.view(offs[2 * i + 1], (L, c, Hkv, D)))
+    trig_k = bank.view(offs[-2], (L, n_q, Hkv, D))
+    trig_v = bank.view(offs[-1], (L, n_q, Hkv, D))
+    q_offs = bank.offsets(L, n_q * Hq * D, sub_seed(seed, 4))
+    q_ptr = [bank.data.data_ptr() + 2 * int(o) for o in q_offs]
+    out = torch.empty(n_q, Hq, D, dtype=torch.bfloat16, device="cuda")
+    stream = torch.cuda.current_stream()
+    st_h = int(stream.cuda_stream)
+    torch.cuda.synchronize()
+
+    def step(evs=None):
+        a = cache.fork_aux(m)
+        cache.append_kv(a, n_q, trig_k, trig_v)
+        for layer in range(L):
+            if evs is not None:
+                evs[2 * layer].record(stream)
+            sq.sq_prefill_attention(cache.handle, a, layer, n_q, q_ptr[layer], out,
+                                    sq.SQ_OUT_BF16, None, scale, [], st_h)
+            if evs is not None:
+                evs[2 * layer + 1].record(stream)
+        cache.release(a)
+
+    K, W = args.steps, args.warmup
+    for _ in range(W):
+        step()
+    torch.cuda.synchronize()
+    assert cache.sync_status() == sq.SQ_OK
+    barrier(world)
+    clocks = ClockSampler(local)
+    time.sleep(0.4)
+    e_begin, e_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    call_evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2 * L)] for _ in range(K)]
+    e_begin.record(stream)
+    for t in range(K):
+        step(call_evs[t])
+    e_end.record(stream)
+    torch.cuda.synchronize()
+    clock_rec = clocks.stop()
+    assert cache.sync_status() == sq.SQ_OK
+    total_ms = max_over_ranks(e_begin.elapsed_time(e_end), world)
+    call_ms = [call_evs[t][2 * l].elapsed_time(call_evs[t][2 * l + 1]) for t in range(K) for l in range(L)]
+    mean_call = statistics.mean(call_ms)
+    kv_bytes = n * Hkv * D * 2 * 2                    # K and V of one layer, every row read once
+    value = world * kv_bytes * L * K / (total_ms / 1e3) / 1e9
+    achieved = kv_bytes / (mean_call / 1e3) / 1e9
+    hbm_peak, peak_kind = peaks()
+    ratio, ratio_src = recorded_traffic_ratio("sq_prefill_kernel", "aux-trigger-128k")
+    res = {
+        "metric": AUX_METRIC,
+        "value": round(value, 1),
+        "unit": "GB/s",
+        "n_gpus": world, "steps": K, "warmup": W,
+        "ms_per_step": round(total_ms / K, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) K/V and queries from a bank; no dataset)",
+        "config": {
+            "workload": (f"aux-trigger-128k: fork of a {n0}-token context, {n_q}-token trigger "
+                         f"phrase appended and prefilled over all {n} keys at {L} layers, fork "
+                         f"released; 32q/8kv, d128, page 64, bf16"),
+            "layers": L, "q_heads": Hq, "kv_heads": Hkv, "head_dim": D, "page_size": P,
+            "context_tokens": n0, "trigger_tokens": n_q, "sm_scale": scale,
+            "l2": "each call reads %.2f GB of distinct K/V (inputs larger than L2)" % (kv_bytes / 1e9),
+            "parallelism": "replicas" if world > 1 else "single GPU",
+        },
+        "aux_prefill": {
+            "us_per_call": round(mean_call * 1e3, 2),
+            "us_per_call_min": round(min(call_ms) * 1e3, 2),
+            "kv_gb_per_call": round(kv_bytes / 1e9, 4),
+            "step": "fork + append of the trigger tokens + one prefill call per layer + release",
+        },
+        "roofline": {
+            "bound": "hbm",
+            "kernel": "sq_prefill_kernel (+ sq_prefill_combine_kernel, timed together per call)",
+            "achieved": round(achieved, 1),
+            "peak": hbm_peak,
+            "peak_kind": peak_kind,
+            "unit": "GB/s",
+            "frac": round(achieved / hbm_peak, 4),
+            "traffic": int(ratio * kv_bytes) if ratio else None,
+            "traffic_source": (ratio_src + ": DRAM bytes per byte of the layer's K/V, from the "
+                               "capture") if ratio else None,
+            "algorithmic_bytes_per_launch": int(kv_bytes),
+        },
+        # per step: the append kernel, then per layer the prefill and the split merge
+        "gpu_launches": int(K * (1 + 2 * L)),
+        "clocks": clock_rec,
+    }
+    if not args.no_e2e:
+        # through the C ABI with host buffers: the trigger tokens' K/V and each
+        # layer's queries copied in from pinned memory, each layer's output back
+        tk_h, tv_h = trig_k.cpu().pin_memory(), trig_v.cpu().pin_memory()
+        tk_d, tv_d = torch.empty_like(trig_k), torch.empty_like(trig_v)
+        q_h = [bank.view(int(o), (n_q, Hq, D)).cpu().pin_memory() for o in q_offs]
+        q_d = torch.empty(n_q, Hq, D, dtype=torch.bfloat16, device="cuda")
+        out_h = torch.empty(L, n_q, Hq, D, dtype=torch.bfloat16).pin_memory()
+        Ke = min(K, 5)
+
+        def e2e_step():
+            a = cache.fork_aux(m)
+            tk_d.copy_(tk_h, non_blocking=True)
+            tv_d.copy_(tv_h, non_blocking=True)
+            cache.append_kv(a, n_q, tk_d, tv_d)
+            for layer in range(L):
+                q_d.copy_(q_h[layer], non_blocking=True)
+                cache.prefill_attention(a, layer, n_q, q_d, out, sq.SQ_OUT_BF16, None, scale, [])
+                out_h[layer].copy_(out, non_blocking=True)
+            cache.release(a)
+
+        e2e_step()
+        torch.cuda.synchronize()
+        barrier(world)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        w0 = time.perf_counter()
+        e0.record(stream)
+        for _ in range(Ke):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - w0
+        e_ms = max_over_ranks(max(e0.elapsed_time(e1), wall * 1e3), world)
+        res["e2e"] = {
+            "value": round(world * kv_bytes * L * Ke / (e_ms / 1e3) / 1e9, 1), "unit": "GB/s",
+            "h2d_bytes_per_step": int(2 * tk_h.numel() * 2 + L * n_q * Hq * D * 2),
+            "d2h_bytes_per_step": int(out_h.numel() * 2),
+            "steps": Ke,
+            "note": "per step: pinned trigger K/V and per-layer queries in, per-layer outputs out",
+        }
+    if not args.no_cpu and rank == 0 and world == 1:
+        res["cpu_baseline"] = aux_trigger_cpu_baseline(bank, offs, sizes, q_offs, L, Hq, Hkv, D,
+                                                       n0, n_q, scale)
+    cache.close()
+    return res
+
+
+def aux_trigger_cpu_baseline(bank, offs, sizes, q_offs, L, Hq, Hkv, D, n0, n_q, scale):
+    """The oracle as it stands (oracle/attention.c prefill, fp64, OpenMP) on
+    the host cores: the trigger tokens' prefill over the whole context at
+    every layer, every head (one step, about 10-15 s on 16 cores); GB/s = K/V
+    bytes of a layer / seconds per layer."""
+    import numpy as np
+
+    from oracle import attention as oatt
+    from synthetic import bf16_bits
+    host = bf16_bits(bank.data.cpu())
+    layers = range(L)
+    total = 0.0
+    n = n0 + n_q
+    for layer in layers:
+        ks, vs = [], []
+        for i, c in enumerate(sizes):
+            for which, dst in ((0, ks), (1, vs)):
+                o = int(offs[2 * i + which])
+                dst.append(host[o:o + L * c * Hkv * D].reshape(L, c, Hkv, D)[layer])
+        for which, dst in ((0, ks), (1, vs)):
+            o = int(offs[len(offs) - 2 + which])
+            dst.append(host[o:o + L * n_q * Hkv * D].reshape(L, n_q, Hkv, D)[layer])
+        k = np.ascontiguousarray(np.concatenate(ks))
+        v = np.ascontiguousarray(np.concatenate(vs))
+        qo = int(q_offs[layer])
+        q = host[qo:qo + n_q * Hq * D].reshape(n_q, Hq, D)
+        t0 = time.perf_counter()
+        oatt.prefill(np.ascontiguousarray(q), k, v, scale, [])
+        total += time.perf_counter() - t0
+    per_layer = total / len(layers)
+    kv_bytes = n * Hkv * D * 2 * 2
+    return {"value": round(kv_bytes / per_layer / 1e9, 4), "unit": "GB/s",
+            "cores": oatt.num_threads(), "kind": "oracle", "cpu_model": cpu_model(),
+            "sample": f"the {n_q} trigger queries over all {n} keys, all {Hq} heads, at "
+                      f"{len(layers)} of {L} layers; GB/s = K/V bytes of a layer / seconds per layer",
             "seconds": round(total, 3)}
 
 
@@ -1189,6 +1395,8 @@ def main():
         res = run_trace(args, world, rank, local)
     elif args.workload == "prefill-32k":
         res = run_prefill(args, world, rank, local)
+    elif args.workload == "aux-trigger-128k":
+        res = run_aux_trigger(args, world, rank, local)
     else:
         res = run_sq(args, world, rank, local)
     if rank == 0:
