@@ -427,6 +427,14 @@ __device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
     asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
     return d;
 }
+// 2^x as the single PTX instruction ex2.approx.ftz (relative error about
+// 2^-22).  Results below 2^-126 flush to zero: every row holds a weight of at
+// least 1 (its running maximum's), so they change its sums by under 2^-119.
+__device__ __forceinline__ float ex2_ftz(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
 __device__ __forceinline__ float fmax3(float a, float b, float c) {
     float d;
     asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
@@ -548,7 +556,7 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
                     if (track) mx[i & 3] = fmax3(mx[i & 3], x0, x1);
                     float a0, a1;
                     f2unpack(ffma2(f2pack(x0, x1), sc2, nmu2), a0, a1);
-                    const float p0 = exp2f(a0), p1 = exp2f(a1);
+                    const float p0 = ex2_ftz(a0), p1 = ex2_ftz(a1);
                     ls2[i & 3] = fadd2(ls2[i & 3], f2pack(p0, p1));
                     const __nv_bfloat162 hb = __floats2bfloat162_rn(p0, p1);
                     wt[hh][i] = *reinterpret_cast<const uint32_t*>(&hb);
