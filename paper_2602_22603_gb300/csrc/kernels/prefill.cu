@@ -272,11 +272,14 @@ __device__ __forceinline__ void issue_qk(const Smem& sm, uint32_t tmem, int t, i
     const uint32_t qa = sm.base + C::kOffQ + (q < 0 ? t : q) * C::kQBytes;
     const uint32_t ka = sm.base + C::kOffRing + slot * C::kSlotBytes;
     const uint32_t dt = tmem + C::kColS + (uint32_t)t * kPrefillKeys;
+    // descriptors built once and stepped per K step: the address field holds
+    // address / 16 in 14 bits and every address here is below 2^18 bytes, so
+    // adding offset / 16 cannot carry out of it
+    const uint64_t qd = smem_desc_sw128(qa, 16, 1024), kd = smem_desc_sw128(ka, 16, 1024);
 #pragma unroll
     for (int ks = 0; ks < D / 16; ++ks) {
-        const uint32_t off = (ks >> 2) * C::kBlockBytes + (ks & 3) * 32;
-        mma_bf16_ss(dt, smem_desc_sw128(qa + off, 16, 1024), smem_desc_sw128(ka + off, 16, 1024),
-                    C::kIdescQK, ks > 0);
+        const uint32_t off = ((ks >> 2) * C::kBlockBytes + (ks & 3) * 32) >> 4;
+        mma_bf16_ss(dt, qd + off, kd + off, C::kIdescQK, ks > 0);
     }
 }
 
@@ -287,11 +290,11 @@ __device__ __forceinline__ void issue_pv(const Smem& sm, uint32_t tmem, int t, i
     using C = PreCfg<D>;
     const uint32_t pa = tmem + C::kColS + (uint32_t)t * kPrefillKeys;
     const uint32_t va = sm.base + C::kOffRing + slot * C::kSlotBytes;
+    const uint64_t vd = smem_desc_sw128(va, C::kBlockBytes, 1024);
 #pragma unroll
     for (int ks = 0; ks < kPrefillKeys / 16; ++ks)
-        mma_bf16_ts(tmem + C::kColO + (uint32_t)t * 128, pa + ks * 8,
-                    smem_desc_sw128(va + ks * 16 * 128, C::kBlockBytes, 1024), C::kIdescPV,
-                    (!first || ks > 0) ? 1u : 0u);
+        mma_bf16_ts(tmem + C::kColO + (uint32_t)t * 128, pa + ks * 8, vd + (uint64_t)(ks * 128),
+                    C::kIdescPV, (!first || ks > 0) ? 1u : 0u);
 }
 
 // Dual-key mode (every query of the CTA tile fits in tile a): both tiles
