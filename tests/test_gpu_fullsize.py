@@ -172,3 +172,37 @@ def test_prefill_32k_full_size():
                 assert np.abs(got - exp_lse[0]).max() <= 1e-2, p
     finally:
         bp.close()
+
+
+def test_aux_trigger_prefill_128k_full_size():
+    """The aux thread's trigger prefill at the bench's size and launch
+    configuration: a fork of a 131,072-token context (32q/8kv, d128, P64)
+    appends 8 tokens and prefills them over all 131,080 keys (each KV head's
+    key range split across the SMs, dual-key mode, split merge).  Every output
+    row and log-sum-exp at two layers against the oracle, bf16 outputs too."""
+    L, Hq, Hkv, D, P = 2, 32, 8, 128, 64
+    n0, n_q = 131072, 8
+    bp = BankPair(L, Hq, Hkv, D, P, num_pages=n0 // P + 64, seed=5)
+    try:
+        m = bp.seq_new()
+        bp.fill(m, n0, 4096)
+        a = bp.fork(m)
+        bp.append(a, n_q)
+        scale = 1.0 / math.sqrt(D)
+        for layer in (0, 1):
+            q = bf16_normal((n_q, Hq, D), 500 + layer, device="cuda")
+            out = torch.empty(n_q, Hq, D, dtype=torch.float32, device="cuda")
+            out16 = torch.empty(n_q, Hq, D, dtype=torch.bfloat16, device="cuda")
+            lse = torch.empty(n_q, Hq, dtype=torch.float32, device="cuda")
+            bp.cache.prefill_attention(a, layer, n_q, q, out, sq.SQ_OUT_F32, lse, scale, [])
+            bp.cache.prefill_attention(a, layer, n_q, q, out16, sq.SQ_OUT_BF16, None, scale, [])
+            torch.cuda.synchronize()
+            assert bp.cache.sync_status() == sq.SQ_OK
+            K, V = bp.rows(a, layer)
+            assert K.shape[0] == n0 + n_q
+            exp, exp_lse = oatt.prefill(bf16_bits(q.cpu()), K, V, scale, [], want_lse=True)
+            assert_close(out, exp)
+            assert_close(out16, exp)
+            assert np.abs(lse.cpu().numpy().astype(np.float64) - exp_lse).max() <= 1e-2
+    finally:
+        bp.close()
