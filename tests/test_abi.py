@@ -58,3 +58,22 @@ def test_null_cache_is_rejected(libsq):
     out = ctypes.c_int32()
     assert libsq.sq_seq_new(None, ctypes.byref(out)) == sq.SQ_ERR_BAD_HANDLE
     assert libsq.sq_cache_destroy(None) == sq.SQ_ERR_BAD_HANDLE
+
+
+def test_binding_fails_loudly_without_the_library():
+    # a fresh interpreter whose package points at a library that does not
+    # exist: the first call raises instead of falling back to anything
+    import subprocess
+    import sys
+    code = (
+        "import paper_2602_22603_gb300 as sq\n"
+        "sq.LIB_PATH = '/nonexistent/libsq.so'\n"
+        "try:\n"
+        "    sq.lib()\n"
+        "except RuntimeError as e:\n"
+        "    print('raised', 'libsq.so not found' in str(e))\n"
+        "else:\n"
+        "    print('loaded')\n")
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, timeout=300,
+                       cwd=os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+    assert r.stdout.strip() == "raised True", r.stdout + r.stderr
