@@ -216,6 +216,15 @@ SQ_API int sq_release(sq_cache *cache, sq_seq seq, void *stream);
 SQ_API int sq_seq_info(sq_cache *cache, sq_seq seq, int32_t *n_tokens,
                 int32_t *n_pages);
 
+/* Position of the sequence's next token: the number of tokens ever appended
+ * to it, counting from its parent's at fork time.  Span eviction (Algorithm 1,
+ * clear_kv) lowers the token count but not this: the library stores keys after
+ * the rotary embedding and never re-rotates them, so kept keys keep the phase
+ * of their original positions and a new token continues after the last
+ * position handed out (a reading: the paper does not discuss positions after
+ * eviction).  Errors: BAD_HANDLE, INVALID_ARG (out is NULL). */
+SQ_API int sq_seq_next_pos(sq_cache *cache, sq_seq seq, int64_t *out);
+
 /* Copy the page table of `seq` into host_out[0 .. cap); *n_out = its length.
  * Errors: BAD_HANDLE, INVALID_ARG (cap too small). */
 SQ_API int sq_get_page_table(sq_cache *cache, sq_seq seq, int32_t *host_out,

@@ -90,6 +90,7 @@ _SIGS = {
                                             ctypes.POINTER(sq_span), _I32, _P]),
     "sq_release": (ctypes.c_int, [_P, _I32, _P]),
     "sq_seq_info": (ctypes.c_int, [_P, _I32, _I32P, _I32P]),
+    "sq_seq_next_pos": (ctypes.c_int, [_P, _I32, ctypes.POINTER(ctypes.c_int64)]),
     "sq_get_page_table": (ctypes.c_int, [_P, _I32, _I32P, _I32, _I32P]),
     "sq_page_refcount": (ctypes.c_int, [_P, _I32, _I32P]),
     "sq_free_pages": (ctypes.c_int, [_P, _I32P]),
@@ -240,6 +241,14 @@ def sq_seq_info(cache: int, seq: int) -> Tuple[int, int]:
     return n.value, p.value
 
 
+def sq_seq_next_pos(cache: int, seq: int) -> int:
+    """Position of the sequence's next token (tokens ever appended; eviction
+    does not lower it)."""
+    x = ctypes.c_int64()
+    _check(lib().sq_seq_next_pos(cache, seq, ctypes.byref(x)), "sq_seq_next_pos")
+    return x.value
+
+
 def sq_get_page_table(cache: int, seq: int) -> List[int]:
     _, npages = sq_seq_info(cache, seq)
     buf = (ctypes.c_int32 * max(1, npages))()
@@ -338,6 +347,7 @@ class Cache:
                                               sm_scale, spans, stream))
     release = lambda self, seq, stream=None: sq_release(self.handle, seq, stream)
     seq_info = lambda self, seq: sq_seq_info(self.handle, seq)
+    next_pos = lambda self, seq: sq_seq_next_pos(self.handle, seq)
     page_table = lambda self, seq: sq_get_page_table(self.handle, seq)
     page_refcount = lambda self, page: sq_page_refcount(self.handle, page)
     free_pages = lambda self: sq_free_pages(self.handle)

@@ -82,6 +82,11 @@ int sqh_seq_info(void* c, int32_t h, int32_t* n_tokens, int32_t* n_pages) {
     return kOk;
 }
 
+int64_t sqh_next_pos(void* c, int32_t h) {
+    const Seq* s = static_cast<HostCache*>(c)->seq(h);
+    return s ? s->next_pos : -1;
+}
+
 int sqh_page_table(void* c, int32_t h, int32_t* out, int32_t cap, int32_t* n_out) {
     const Seq* s = static_cast<HostCache*>(c)->seq(h);
     if (!s) return kBadHandle;

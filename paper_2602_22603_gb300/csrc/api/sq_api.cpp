@@ -972,6 +972,15 @@ int sq_seq_info(sq_cache* c, sq_seq seq, int32_t* n_tokens, int32_t* n_pages) {
     return SQ_OK;
 }
 
+int sq_seq_next_pos(sq_cache* c, sq_seq seq, int64_t* out) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    const Seq* s = c->host->seq(seq);
+    if (!s) return SQ_ERR_BAD_HANDLE;
+    if (!out) return SQ_ERR_INVALID_ARG;
+    *out = s->next_pos;
+    return SQ_OK;
+}
+
 int sq_get_page_table(sq_cache* c, sq_seq seq, int32_t* host_out, int32_t cap, int32_t* n_out) {
     if (!c) return SQ_ERR_BAD_HANDLE;
     const Seq* s = c->host->seq(seq);

@@ -117,6 +117,7 @@ int HostCache::seq_new(int32_t* handle) {
     s.gen = (s.gen % 2047) + 1;  // 1 .. 2047: handles stay positive
     s.n = 0;
     s.pages.clear();
+    s.next_pos = 0;
     s.version = g_version_counter++;
     s.last_stream = nullptr;
     *handle = (int32_t)((s.gen << 20) | (uint32_t)slot);
@@ -128,12 +129,14 @@ int HostCache::fork(int32_t parent, int32_t* child) {
     if (!ps) return kBadHandle;
     std::vector<int32_t> pages = ps->pages;
     int32_t n = ps->n;
+    const int64_t next_pos = ps->next_pos;
     void* st = ps->last_stream;
     int rc = seq_new(child);
     if (rc != kOk) return rc;
     Seq* cs = seq_mut(*child);
     cs->pages = std::move(pages);
     cs->n = n;
+    cs->next_pos = next_pos;
     cs->last_stream = st;
     for (int32_t p : cs->pages) alloc_.add_ref(p);
     return kOk;
@@ -175,6 +178,7 @@ int HostCache::append(int32_t h, int32_t n_new, AppendPlan* plan) {
     plan->first_page_index = n / P;
     plan->pages.assign(s->pages.begin() + n / P, s->pages.end());
     s->n = n + n_new;
+    s->next_pos += n_new;
     s->version = g_version_counter++;
     return kOk;
 }
@@ -193,6 +197,7 @@ void HostCache::undo_append(int32_t h, const AppendPlan& plan) {
         s->pages.back() = plan.cow_old;
     }
     s->n = plan.n0;
+    s->next_pos -= plan.n_new;
     s->version = g_version_counter++;
 }
 

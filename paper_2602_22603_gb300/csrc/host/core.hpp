@@ -79,6 +79,10 @@ struct Seq {
     int32_t n = 0;
     std::vector<int32_t> pages;
     uint64_t version = 0;  // bumped by every change of n or pages
+    // position of the next token: tokens ever appended (a fork starts from its
+    // parent's); eviction does not lower it, since kept keys keep the rotary
+    // phase of their original positions
+    int64_t next_pos = 0;
     void* last_stream = nullptr;
 };
 

@@ -34,6 +34,8 @@ def lib():
         L.sqh_release.argtypes = [P, I32]
         L.sqh_evict_tiles.argtypes = [P, I32, I32P, I32, I32, I32P, I32, I32P, I32, I32P, I32P]
         L.sqh_seq_info.argtypes = [P, I32, I32P, I32P]
+        L.sqh_next_pos.argtypes = [P, I32]
+        L.sqh_next_pos.restype = ctypes.c_int64
         L.sqh_page_table.argtypes = [P, I32, I32P, I32, I32P]
         L.sqh_refcount.argtypes = [P, I32]
         L.sqh_free_count.argtypes = [P]
@@ -113,6 +115,9 @@ class HostCache:
         n, p = ctypes.c_int32(), ctypes.c_int32()
         rc = lib().sqh_seq_info(self.h, h, ctypes.byref(n), ctypes.byref(p))
         return rc, n.value, p.value
+
+    def next_pos(self, h):
+        return lib().sqh_next_pos(self.h, h)
 
     def page_table(self, h):
         rc, n, npg = self.info(h)

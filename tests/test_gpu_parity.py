@@ -430,3 +430,23 @@ def test_many_sequences_in_one_call():
     rng.shuffle(seqs)
     _decode_check(p, seqs, 0, 0.0884, 3)
     p.close()
+
+
+def test_next_position_through_the_api():
+    # the same counter through the C ABI: appends advance it, a fork inherits
+    # it, eviction leaves it, a bad handle is refused
+    p = Pair(1, 16, 4, 64, 16, num_pages=40, seed=3)
+    try:
+        m = p.seq_new()
+        p.append(m, 100)
+        assert p.cache.next_pos(m) == 100
+        a = p.fork(m)
+        p.append(a, 5)
+        assert (p.cache.next_pos(a), p.cache.next_pos(m)) == (105, 100)
+        p.evict(m, [(0, 30)])
+        assert p.cache.seq_info(m)[0] == 70 and p.cache.next_pos(m) == 100
+        with pytest.raises(sq.SqError) as ei:
+            sq.sq_seq_next_pos(p.cache.handle, 123456789)
+        assert ei.value.code == sq.SQ_ERR_BAD_HANDLE
+    finally:
+        p.close()

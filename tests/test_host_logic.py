@@ -344,3 +344,28 @@ def test_prefill_plan_splits_short_query_blocks():
     assert ctas / (-(-ctas // 152) * 152) >= 0.9
     rc, info, _ = plan_prefill(32, 8, 32768, 32768, [(100, 5000)])
     assert rc == 0 and info["n_split"] == 1 and info["n_qt"] == 512
+
+
+def test_next_position_counts_appends_not_evictions():
+    # the position of a sequence's next token: every appended token advances
+    # it, a fork starts from its parent's, eviction leaves it (kept keys keep
+    # the rotary phase of their original positions), a refused append does not
+    hc = HostCache(1, 8, 2, 64, 16, 40)
+    rc, m = hc.seq_new()
+    assert rc == 0 and hc.next_pos(m) == 0
+    assert hc.append(m, 100) == 0
+    assert hc.next_pos(m) == 100
+    rc, a = hc.fork(m)
+    assert rc == 0 and hc.next_pos(a) == 100
+    assert hc.append(a, 7) == 0
+    assert (hc.next_pos(a), hc.next_pos(m)) == (107, 100)
+    rc, _ = hc.evict(m, [(10, 50), (60, 61)])
+    assert rc == 0
+    assert hc.info(m)[1] == 59 and hc.next_pos(m) == 100
+    assert hc.append(m, 1) == 0
+    assert (hc.info(m)[1], hc.next_pos(m)) == (60, 101)
+    assert hc.append(m, 16 * 40) != 0           # more pages than the pool holds
+    assert (hc.info(m)[1], hc.next_pos(m)) == (60, 101)
+    assert hc.release(a) == 0
+    rc, b = hc.seq_new()                         # a fresh handle starts at 0
+    assert rc == 0 and hc.next_pos(b) == 0
