@@ -96,11 +96,17 @@ KERNEL_SOURCES = {
 
 
 def sources_hash(kernel: str) -> str:
+    """Hash of a kernel's sources with comments and whitespace removed, so that
+    an edit of comments alone does not void a traffic capture."""
     import hashlib
+    import re
     m = hashlib.sha256()
     for rel in KERNEL_SOURCES[kernel]:
-        with open(os.path.join(ROOT, "paper_2602_22603_gb300", "csrc", rel), "rb") as f:
-            m.update(f.read())
+        with open(os.path.join(ROOT, "paper_2602_22603_gb300", "csrc", rel)) as f:
+            text = f.read()
+        text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", " ", text)
+        m.update(" ".join(text.split()).encode())
     return m.hexdigest()[:16]
 
 

@@ -29,8 +29,16 @@
 // shared-memory slots (K_0, V_0, K_1, ...); a K slot is released once both S
 // products are done, a V slot once both PV products are.
 //
-// Warp roles (320 threads): warp 0 loads (lane 0 issues the TMA copies), lane
-// 0 of warp 1 issues the MMAs and warp 1 owns the TMEM allocation, warps 2-5
+// Short query blocks: when a CTA tile's queries all fit in tile a, tile b's
+// warpgroup takes the same rows over every other key tile (dual-key mode, the
+// two results merged per row at the end, loads in the order the MMAs consume
+// them), and when there are fewer CTA tiles than SMs each tile's key range is
+// split over several CTAs whose normalised partial results a second kernel
+// merges.
+//
+// Warp roles (320 threads): warp 0 loads (lanes 0 and 1 issue the TMA copies,
+// two loads at a time), lane 0 of warp 1 issues the MMAs and warp 1 owns the
+// TMEM allocation, warps 2-5
 // are the softmax warpgroup of tile a and warps 6-9 that of tile b (warp w
 // reads TMEM lanes 32 (w mod 4) .. +31, one row per thread).  Every wait is
 // bounded; a wait that runs out sets the error word and the CTA winds down
