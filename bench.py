@@ -422,7 +422,7 @@ def run_sq(args, world, rank, local):
         },
         "roofline": {
             "bound": "hbm",
-            "kernel": "sq_decode_splitk_kernel (+ sq_lse_combine_kernel, timed together per call)",
+            "kernel": "sq_decode_splitk_kernel (split-K attention and the merge of its partials)",
             "achieved": round(achieved, 1),
             "peak": hbm_peak,
             "peak_kind": peak_kind,
@@ -435,7 +435,8 @@ def run_sq(args, world, rank, local):
                                "to this launch's algorithmic bytes") if ratio else None,
             "algorithmic_bytes_per_launch": int(uniq_per_call),
         },
-        "gpu_launches": int(K * (1 + 2 * L)),
+        # per step: the append kernel, then one decode kernel per layer
+        "gpu_launches": int(K * (1 + L)),
         "clocks": clock_rec,
     }
 

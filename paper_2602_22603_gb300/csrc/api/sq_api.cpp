@@ -46,6 +46,7 @@ struct PlanEntry {
     size_t part_cap = 0;
     cudaEvent_t ev = nullptr;   // recorded after the last launch that used it
     bool ev_recorded = false;
+    cudaStream_t ev_stream = nullptr;  // ... on this stream (work on it is ordered after anyway)
     uint64_t last_use = 0;
 };
 
@@ -67,6 +68,7 @@ struct PrefillPlanEntry {
     size_t cap = 0;
     cudaEvent_t ev = nullptr;  // recorded after the last launch that used it
     bool ev_recorded = false;
+    cudaStream_t ev_stream = nullptr;  // ... on this stream
     uint64_t last_use = 0;
 };
 
@@ -75,6 +77,7 @@ struct UploadSlot {
     size_t cap = 0;
     cudaEvent_t ev = nullptr;
     bool ev_recorded = false;
+    cudaStream_t ev_stream = nullptr;
 };
 
 // Pinned host staging for uploads: a copy from pageable memory may wait for
@@ -109,6 +112,7 @@ struct sq_cache {
     size_t pre_part_cap = 0;
     cudaEvent_t pre_ev = nullptr;
     bool pre_ev_recorded = false;
+    cudaStream_t pre_ev_stream = nullptr;
     PlanEntry plans[kPlanCacheEntries];
     PrefillPlanEntry pre_plans[kPrefillPlanEntries];
     uint64_t use_clock = 0;
@@ -265,7 +269,8 @@ int upload(sq_cache* c, UploadSlot& s, const void* src, size_t bytes, void* stre
         s.cap = cap;
         s.ev_recorded = false;
     }
-    if (s.ev_recorded) {
+    // work on the stream that recorded the event is ordered after it already
+    if (s.ev_recorded && s.ev_stream != as_stream(stream)) {
         cudaError_t e = cudaStreamWaitEvent(as_stream(stream), s.ev, 0);
         if (e != cudaSuccess) return cuda_status(e);
     }
@@ -578,6 +583,10 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
     }
     cudaStream_t st = as_stream(stream);
     cudaError_t e;
+    // a reused plan that needs no cross-stream wait was on the device before
+    // anything this call enqueues: the kernel may read it before its
+    // grid-dependency wait
+    bool plan_ready = false;
     if (!hit) {
         DecodePlanHost plan;
         int rc = plan_decode(*c->host, seqs, n_seqs, c->decode_ctas, &plan);
@@ -587,7 +596,7 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
         PlanEntry* victim = &c->plans[0];
         for (auto& p : c->plans)
             if (!p.valid || p.last_use < victim->last_use) victim = &p;
-        const size_t part_bytes = (size_t)decode_partial_bytes(lay.n_items, g.D);
+        const size_t part_bytes = (size_t)decode_partial_bytes(lay.n_comb_ent, g.G(), g.D);
         if ((size_t)lay.total > victim->plan_cap || part_bytes > victim->part_cap) {
             if (victim->ev_recorded) cudaEventSynchronize(victim->ev);
             if ((size_t)lay.total > victim->plan_cap) {
@@ -613,7 +622,7 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
             e = cudaEventCreateWithFlags(&victim->ev, cudaEventDisableTiming);
             if (e != cudaSuccess) return cuda_status(e);
         }
-        if (victim->ev_recorded) {
+        if (victim->ev_recorded && victim->ev_stream != st) {
             e = cudaStreamWaitEvent(st, victim->ev, 0);
             if (e != cudaSuccess) return cuda_status(e);
         }
@@ -634,23 +643,30 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
                plan.cta_begin[victim->first_busy_cta + 1] == plan.cta_begin[victim->first_busy_cta])
             ++victim->first_busy_cta;
         hit = victim;
-    } else if (hit->ev_recorded) {
+    } else if (hit->ev_recorded && hit->ev_stream != st) {
         e = cudaStreamWaitEvent(st, hit->ev, 0);
         if (e != cudaSuccess) return cuda_status(e);
+    } else {
+        plan_ready = true;
     }
     hit->last_use = ++c->use_clock;
     const DecodePlanLayout& L = hit->lay;
     float* part_o = hit->d_part;
-    float* part_ml = part_o + (size_t)L.n_items * kRowsPerTile * g.D;
+    float* part_ml = part_o + (size_t)L.n_comb_ent * g.G() * g.D;
 
     DecodeArgs a;
     a.segs = reinterpret_cast<const DecodeSeg*>(hit->d_plan + L.segs);
     a.items = reinterpret_cast<const DecodeItem*>(hit->d_plan + L.items);
     a.cta_begin = reinterpret_cast<const int32_t*>(hit->d_plan + L.cta_begin);
     a.page_ids = reinterpret_cast<const int32_t*>(hit->d_plan + L.page_ids);
+    a.comb_off = reinterpret_cast<const int32_t*>(hit->d_plan + L.comb_off);
+    a.arrive = reinterpret_cast<unsigned int*>(hit->d_plan + L.arrive);
     a.q = reinterpret_cast<const __nv_bfloat16*>(q);
+    a.out = out;
     a.part_o = part_o;
     a.part_ml = part_ml;
+    a.out_f32 = out_dtype == SQ_OUT_F32;
+    a.plan_ready = plan_ready ? 1 : 0;
     a.layer = layer;
     a.Hq = g.Hq;
     a.Hkv = g.Hkv;
@@ -663,23 +679,10 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
     a.err = c->d_err;
     e = launch_decode(c->tmap, a, L.n_ctas, g.D, st);
     if (e != cudaSuccess) { hit->valid = false; return cuda_status(e); }
-
-    CombineArgs ca;
-    ca.comb_off = reinterpret_cast<const int32_t*>(hit->d_plan + L.comb_off);
-    ca.comb_ent = reinterpret_cast<const CombineEnt*>(hit->d_plan + L.comb_ent);
-    ca.part_o = part_o;
-    ca.part_ml = part_ml;
-    ca.out = out;
-    ca.out_f32 = out_dtype == SQ_OUT_F32;
-    ca.n_seqs = n_seqs;
-    ca.Hq = g.Hq;
-    ca.Hkv = g.Hkv;
-    ca.G = g.G();
-    e = launch_combine(ca, g.D, st);
-    if (e != cudaSuccess) { hit->valid = false; return cuda_status(e); }
     e = cudaEventRecord(hit->ev, st);
     if (e != cudaSuccess) return cuda_status(e);
     hit->ev_recorded = true;
+    hit->ev_stream = st;
     for (int32_t i = 0; i < n_seqs; ++i) c->host->seq_mut(seqs[i])->last_stream = stream;
     c->stats.decode_calls += 1;
     c->stats.decode_logical_bytes += hit->logical_tokens * g.token_layer_bytes();
@@ -736,6 +739,7 @@ int sq_evict_spans(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_span
         e = cudaEventRecord(s.ev, st);
         if (e != cudaSuccess) return cuda_status(e);
         s.ev_recorded = true;
+        s.ev_stream = st;
     }
     rc = record_freed(c, plan.freed, stream);
     if (rc != SQ_OK) return rc;
@@ -812,7 +816,7 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
             if (e != cudaSuccess) return cuda_status(e);
             victim->cap = cap;
         }
-        if (victim->ev_recorded) {
+        if (victim->ev_recorded && victim->ev_stream != st) {
             // the launches that read the old plan run before it is overwritten
             e = cudaStreamWaitEvent(st, victim->ev, 0);
             if (e != cudaSuccess) return cuda_status(e);
@@ -838,7 +842,7 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
         victim->visible_pairs = plan.visible_pairs;
         victim->valid = true;
         hit = victim;
-    } else if (hit->ev_recorded) {
+    } else if (hit->ev_recorded && hit->ev_stream != st) {
         // its upload ran on the stream of the call that planned it
         e = cudaStreamWaitEvent(st, hit->ev, 0);
         if (e != cudaSuccess) return cuda_status(e);
@@ -863,7 +867,7 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
             c->pre_part_cap = need * 5 / 4;
             c->pre_ev_recorded = false;
         }
-        if (c->pre_ev_recorded) {
+        if (c->pre_ev_recorded && c->pre_ev_stream != st) {
             e = cudaStreamWaitEvent(st, c->pre_ev, 0);
             if (e != cudaSuccess) return cuda_status(e);
         }
@@ -931,10 +935,12 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
         e = cudaEventRecord(c->pre_ev, st);
         if (e != cudaSuccess) return cuda_status(e);
         c->pre_ev_recorded = true;
+        c->pre_ev_stream = st;
     }
     e = cudaEventRecord(hit->ev, st);
     if (e != cudaSuccess) return cuda_status(e);
     hit->ev_recorded = true;
+    hit->ev_stream = st;
     c->host->seq_mut(seq)->last_stream = stream;
     c->stats.prefill_calls += 1;
     c->stats.prefill_pairs += plan.visible_pairs;
@@ -1073,9 +1079,9 @@ int sq_decode_attention_noalloc(sq_cache* c, const sq_seq* seqs, int32_t n_seqs,
     int rc = plan_decode(*c->host, seqs, n_seqs, c->decode_ctas, &plan);
     if (rc != SQ_OK) return rc;
     const DecodePlanLayout L = plan_layout(plan, n_seqs, g.Hkv);
-    // scratch = [plan | partial outputs | partial (max, sum)]
+    // scratch = [plan (with zeroed arrival words) | partial outputs | partial (max, sum)]
     const size_t part_off = ((size_t)L.total + 255) & ~size_t(255);
-    const size_t need = part_off + (size_t)decode_partial_bytes(L.n_items, g.D);
+    const size_t need = part_off + (size_t)decode_partial_bytes(L.n_comb_ent, g.G(), g.D);
     if (need > (size_t)SQ_NOALLOC_SCRATCH_BYTES) return SQ_ERR_CAPACITY;
     void* base = nullptr;
     rc = noalloc_scratch(dev, &base);
@@ -1088,16 +1094,21 @@ int sq_decode_attention_noalloc(sq_cache* c, const sq_seq* seqs, int32_t n_seqs,
     cudaError_t e = cudaMemcpyAsync(scratch, c->staging.data(), L.total, cudaMemcpyHostToDevice, st);
     if (e != cudaSuccess) return cuda_status(e);
     float* part_o = reinterpret_cast<float*>(scratch + part_off);
-    float* part_ml = part_o + (size_t)L.n_items * kRowsPerTile * g.D;
+    float* part_ml = part_o + (size_t)L.n_comb_ent * g.G() * g.D;
 
     DecodeArgs a;
     a.segs = reinterpret_cast<const DecodeSeg*>(scratch + L.segs);
     a.items = reinterpret_cast<const DecodeItem*>(scratch + L.items);
     a.cta_begin = reinterpret_cast<const int32_t*>(scratch + L.cta_begin);
     a.page_ids = reinterpret_cast<const int32_t*>(scratch + L.page_ids);
+    a.comb_off = reinterpret_cast<const int32_t*>(scratch + L.comb_off);
+    a.arrive = reinterpret_cast<unsigned int*>(scratch + L.arrive);
     a.q = reinterpret_cast<const __nv_bfloat16*>(q);
+    a.out = out;
     a.part_o = part_o;
     a.part_ml = part_ml;
+    a.out_f32 = out_dtype == SQ_OUT_F32;
+    a.plan_ready = 0;  // uploaded just now
     a.layer = layer;
     a.Hq = g.Hq;
     a.Hkv = g.Hkv;
@@ -1112,20 +1123,6 @@ int sq_decode_attention_noalloc(sq_cache* c, const sq_seq* seqs, int32_t n_seqs,
     c->debug_flags &= ~SQ_DEBUG_DROP_DECODE_STAGE;
     a.err = c->d_err;
     e = launch_decode(c->tmap, a, L.n_ctas, g.D, st);
-    if (e != cudaSuccess) return cuda_status(e);
-
-    CombineArgs ca;
-    ca.comb_off = reinterpret_cast<const int32_t*>(scratch + L.comb_off);
-    ca.comb_ent = reinterpret_cast<const CombineEnt*>(scratch + L.comb_ent);
-    ca.part_o = part_o;
-    ca.part_ml = part_ml;
-    ca.out = out;
-    ca.out_f32 = out_dtype == SQ_OUT_F32;
-    ca.n_seqs = n_seqs;
-    ca.Hq = g.Hq;
-    ca.Hkv = g.Hkv;
-    ca.G = g.G();
-    e = launch_combine(ca, g.D, st);
     if (e != cudaSuccess) return cuda_status(e);
     for (int32_t i = 0; i < n_seqs; ++i) c->host->seq_mut(seqs[i])->last_stream = stream;
     c->stats.decode_calls += 1;

@@ -491,6 +491,7 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
             const int64_t lo = std::max(b, unit_start[v]), hi = std::min(e, unit_end[v]);
             if (hi <= lo) continue;
             DecodeItem it;
+            std::memset(&it, 0, sizeof it);
             it.seg = (int32_t)(v / g.Hkv);
             it.head = (int32_t)(v % g.Hkv);
             it.s0 = (int32_t)(lo - unit_start[v]);
@@ -500,7 +501,7 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
     }
     out->cta_begin[ctas] = (int32_t)out->items.size();
 
-    // combine lists per (sequence, KV head)
+    // partial entries per (sequence, KV head), contiguous, in item order
     const int32_t keys = n_seqs * g.Hkv;
     out->comb_off.assign(keys + 1, 0);
     for (const DecodeItem& it : out->items) {
@@ -508,17 +509,10 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
         for (int32_t j = 0; j < s.n_grp; ++j) ++out->comb_off[s.grp_seq[j] * g.Hkv + it.head + 1];
     }
     for (int32_t k = 0; k < keys; ++k) out->comb_off[k + 1] += out->comb_off[k];
-    out->comb_ent.resize(out->comb_off[keys]);
     std::vector<int32_t> fill(out->comb_off.begin(), out->comb_off.end() - 1);
-    for (int32_t i = 0; i < (int32_t)out->items.size(); ++i) {
-        const DecodeItem& it = out->items[i];
+    for (DecodeItem& it : out->items) {
         const DecodeSeg& s = out->segs[it.seg];
-        for (int32_t j = 0; j < s.n_grp; ++j) {
-            CombineEnt e;
-            e.item = i;
-            e.j = j;
-            out->comb_ent[fill[s.grp_seq[j] * g.Hkv + it.head]++] = e;
-        }
+        for (int32_t j = 0; j < s.n_grp; ++j) it.ent[j] = fill[s.grp_seq[j] * g.Hkv + it.head]++;
     }
     return kOk;
 }
@@ -532,14 +526,14 @@ DecodePlanLayout plan_layout(const DecodePlanHost& p, int32_t n_seqs, int32_t Hk
     L.n_ctas = p.n_ctas;
     L.n_page_ids = (int32_t)p.page_ids.size();
     L.n_comb_keys = n_seqs * Hkv;
-    L.n_comb_ent = (int32_t)p.comb_ent.size();
+    L.n_comb_ent = p.comb_off.empty() ? 0 : p.comb_off.back();
     int64_t o = 0;
     L.segs = o;      o = align16(o + sizeof(DecodeSeg) * L.n_segs);
     L.items = o;     o = align16(o + sizeof(DecodeItem) * L.n_items);
     L.cta_begin = o; o = align16(o + sizeof(int32_t) * (L.n_ctas + 1));
     L.page_ids = o;  o = align16(o + sizeof(int32_t) * L.n_page_ids);
     L.comb_off = o;  o = align16(o + sizeof(int32_t) * (L.n_comb_keys + 1));
-    L.comb_ent = o;  o = align16(o + sizeof(CombineEnt) * L.n_comb_ent);
+    L.arrive = o;    o = align16(o + sizeof(uint32_t) * L.n_comb_keys);
     L.total = o;
     return L;
 }
@@ -551,7 +545,6 @@ void plan_serialize(const DecodePlanHost& p, const DecodePlanLayout& L, uint8_t*
     std::memcpy(dst + L.cta_begin, p.cta_begin.data(), sizeof(int32_t) * (L.n_ctas + 1));
     std::memcpy(dst + L.page_ids, p.page_ids.data(), sizeof(int32_t) * L.n_page_ids);
     std::memcpy(dst + L.comb_off, p.comb_off.data(), sizeof(int32_t) * (L.n_comb_keys + 1));
-    std::memcpy(dst + L.comb_ent, p.comb_ent.data(), sizeof(CombineEnt) * L.n_comb_ent);
 }
 
 // ---------------------------------------------------------------------------

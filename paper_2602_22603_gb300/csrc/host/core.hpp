@@ -158,8 +158,9 @@ struct DecodePlanHost {
     std::vector<DecodeItem> items;
     std::vector<int32_t> cta_begin;   // n_ctas + 1
     std::vector<int32_t> page_ids;
+    // partial entries of (sequence i, KV head h): [comb_off[k], comb_off[k + 1]),
+    // k = i * Hkv + h, in item order
     std::vector<int32_t> comb_off;    // n_seqs * Hkv + 1
-    std::vector<CombineEnt> comb_ent;
     int64_t unique_tokens = 0;        // sum over segments of n_tok (one head, one layer)
     int64_t logical_tokens = 0;       // sum over sequences of n
     int32_t n_ctas = 0;

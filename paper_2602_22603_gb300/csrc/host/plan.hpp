@@ -30,17 +30,15 @@ struct DecodeSeg {
     int32_t grp_lim[kRowsPerTile];    // valid tokens of each, from the run start
 };
 
-// A contiguous range of stages of one (segment, KV head) — one partial result.
+// A contiguous range of stages of one (segment, KV head) — one partial result
+// per group member.  Member j's G rows go to partial entry ent[j]; the entries
+// of one (sequence, KV head) are contiguous, so that its merge reads them
+// without an index.
 struct DecodeItem {
     int32_t seg;
     int32_t head;
     int32_t s0, s1;                   // stages [s0, s1)
-};
-
-// One combine entry: partials of item `item`, rows of group member `j`.
-struct CombineEnt {
-    int32_t item;
-    int32_t j;
+    int32_t ent[kRowsPerTile];        // partial entry of each group member (n_grp used)
 };
 
 // Eviction compaction, planned once per eviction and shared by every
@@ -80,8 +78,11 @@ struct PrefillTile {
 };
 
 // Byte offsets of the arrays of a decode plan inside one upload buffer.
+// Byte offsets of the serialised decode plan.  `arrive` holds one 32-bit
+// arrival count per (sequence, KV head), zero in the serialised plan; the
+// kernel counts on it and leaves it at zero again.
 struct DecodePlanLayout {
-    int64_t segs, items, cta_begin, page_ids, comb_off, comb_ent, total;
+    int64_t segs, items, cta_begin, page_ids, comb_off, arrive, total;
     int32_t n_segs, n_items, n_ctas, n_page_ids, n_comb_keys, n_comb_ent;
 };
 

@@ -1,5 +1,5 @@
-// Split-K flash-decoding over the paged bf16 KV pool, and the log-sum-exp
-// combine of its partial results.
+// Split-K flash-decoding over the paged bf16 KV pool, with the log-sum-exp
+// merge of its partial results in the same kernel.
 //
 // What is computed (Sec. 1 and Sec. 3.4: for every generated token,
 // attention reads the whole KV cache of the context; Sec. 2.1: in
@@ -16,6 +16,20 @@
 // online-softmax partial (max, sum, unnormalised output) for up to 16 query
 // rows — the G heads of every sequence in the group, so a shared page is read
 // from HBM once for all of them.
+//
+// Merge: an item leaves one partial (max, sum, unnormalised output) per group
+// member, in that (sequence, KV head)'s contiguous run of entries.  After its
+// last item a CTA counts its arrivals on each (sequence, KV head) it touched;
+// the CTA that brings a count to the number of entries merges that run
+// (max of the maxima, weights 2^(m - M)) and writes the normalised output.
+// The arrival word holds the call's tag next to the count, and the last
+// arriver clears it, so a word left by another call never counts here.
+//
+// Start-up: the kernel is a programmatic dependent of whatever precedes it.
+// When the plan was already on the device (a reused plan), the producer reads
+// it and prefetches the CTA's first stages into L2 before the dependency wait;
+// the K/V rows themselves reach shared memory only after the wait, through L2,
+// which holds whatever the preceding kernel wrote to them.
 //
 // Tensor cores: S = Q K^T and O += P V are m16n8k16 bf16 mma.sync with fp32
 // accumulation; rows = query rows (<= 16), columns = tokens / head dims.  The
@@ -59,12 +73,88 @@ __device__ __forceinline__ float bf16x2_sum(uint32_t v) {
     return __uint_as_float(v << 16) + __uint_as_float(v & 0xffff0000u);
 }
 
+// ---- start-up work before the grid-dependency wait --------------------------
+constexpr int kPrefetchStages = 4;  // stages prefetched into L2
+constexpr int kFastStages = 3;      // stages whose coordinates are kept in registers
+
+// The coordinates of a CTA's first stages (whole-page stages only, P >= 64):
+// the producer issues their loads right after the wait, without re-reading the
+// plan there.
+struct FastStart {
+    int n;                       // stages read (0: none)
+    int it, s;                   // where the producer continues
+    int32_t row[kFastStages];    // K row coordinate head * P + row0 (V: + Hkv * P)
+    int32_t pid[kFastStages];
+};
+
+__device__ __forceinline__ void fast_start(const DecodeArgs& a, int it0, int it1, FastStart& fs) {
+    const int P = a.P;
+    int it = it0, s = 0, s1 = 0, head = 0, page_off = 0;
+    if (it < it1) {
+        const DecodeItem* item = a.items + it;
+        s = item->s0;
+        s1 = item->s1;
+        head = item->head;
+        page_off = a.segs[item->seg].page_off;
+    }
+    fs.n = 0;
+#pragma unroll
+    for (int k = 0; k < kFastStages; ++k) {
+        while (it < it1 && s >= s1) {
+            if (++it < it1) {
+                const DecodeItem* item = a.items + it;
+                s = item->s0;
+                s1 = item->s1;
+                head = item->head;
+                page_off = a.segs[item->seg].page_off;
+            }
+        }
+        if (it < it1) {
+            const int tok0 = s * kStageTokens;
+            fs.pid[k] = a.page_ids[page_off + tok0 / P];
+            fs.row[k] = head * P + tok0 % P;
+            fs.n = k + 1;
+            ++s;
+        }
+    }
+    fs.it = it;
+    fs.s = s;
+}
+
+template <int D>
+__device__ void prefetch_first_stages(const CUtensorMap* tmap, const DecodeArgs& a, int it0,
+                                      int it1) {
+    const int P = a.P;
+    const int pages_per_stage = P < kStageTokens ? kStageTokens / P : 1;
+    int n = 0;
+    for (int it = it0; it < it1 && n < kPrefetchStages; ++it) {
+        const DecodeItem* item = a.items + it;
+        const int head = item->head, s1 = item->s1;
+        const DecodeSeg* seg = a.segs + item->seg;
+        const int page_off = seg->page_off, n_pages = seg->n_pages;
+        for (int s = item->s0; s < s1 && n < kPrefetchStages; ++s, ++n) {
+            const int tok0 = s * kStageTokens;
+            const int pi0 = tok0 / P;
+            const int row0 = P > kStageTokens ? (tok0 % P) : 0;
+            const int np = P >= kStageTokens ? 1 : min(pages_per_stage, n_pages - pi0);
+            for (int k = 0; k < np; ++k) {
+                const int32_t p = a.page_ids[page_off + pi0 + k];
+                if ((uint32_t)p >= (uint32_t)a.num_pages) continue;  // reported by the producer
+                for (int cb = 0; cb < DecCfg<D>::kColBlocks; ++cb) {
+                    tma_prefetch_l2_4d(tmap, cb * 64, head * P + row0, p, a.layer);
+                    tma_prefetch_l2_4d(tmap, cb * 64, (a.Hkv + head) * P + row0, p, a.layer);
+                }
+            }
+        }
+    }
+}
+
 // ---- producer: one thread issues the TMA loads of every stage -------------
 template <int D>
 __device__ void produce(const CUtensorMap* tmap, const DecodeArgs& a, int it0, int it1,
-                        uint8_t* smem, uint64_t* bars, volatile int* abort_flag) {
+                        const FastStart& fs, uint8_t* smem, uint64_t* bars,
+                        volatile int* abort_flag) {
     using C = DecCfg<D>;
-    prefetch_tmap(tmap);
     const int P = a.P;
     const int box_rows = P < kStageTokens ? P : kStageTokens;
     const int pages_per_stage = P < kStageTokens ? kStageTokens / P : 1;
@@ -73,11 +163,45 @@ __device__ void produce(const CUtensorMap* tmap, const DecodeArgs& a, int it0, i
     uint32_t phase = 0;
     uint32_t issued = 0, issued_phase = 0;  // per-slot bits of the last issue
     bool ok = true;
-    for (int it = it0; it < it1 && ok; ++it) {
+    int it_start = it0, s_start = -1;       // -1: the item's first stage
+    if (fs.n > 0) {
+        // the first stages, from registers (whole-page stages; fresh slots)
+        const uint32_t bytes = box_bytes * C::kColBlocks * 2u;
+#pragma unroll
+        for (int k = 0; k < kFastStages; ++k) {
+            if (k < fs.n) {
+                const uint32_t full = smem_addr(&bars[k]);
+                const int32_t p = fs.pid[k];
+                if ((uint32_t)p < (uint32_t)a.num_pages) {
+                    mbar_arrive_expect_tx(full, bytes);
+                    const uint32_t dk = smem_addr(smem + k * C::kStageBytes);
+#pragma unroll
+                    for (int cb = 0; cb < C::kColBlocks; ++cb) {
+                        tma_load_4d(dk + cb * C::kBlockBytes, tmap, full, cb * 64, fs.row[k], p,
+                                    a.layer);
+                        tma_load_4d(dk + cb * C::kBlockBytes + C::kTileBytes, tmap, full, cb * 64,
+                                    fs.row[k] + a.Hkv * P, p, a.layer);
+                    }
+                } else {
+                    set_error(a.err, kErrBounds);
+                    mbar_arrive(full);
+                }
+                issued |= 1u << k;
+            }
+        }
+        slot = fs.n;
+        if (slot == C::kStages) {
+            slot = 0;
+            phase = 1;
+        }
+        it_start = fs.it;
+        s_start = fs.s;
+    }
+    for (int it = it_start; it < it1 && ok; ++it) {
         const DecodeItem item = a.items[it];
         const DecodeSeg* seg = a.segs + item.seg;
         const int page_off = seg->page_off, n_pages = seg->n_pages;
-        for (int s = item.s0; s < item.s1; ++s) {
+        for (int s = (it == it_start && s_start >= 0) ? s_start : item.s0; s < item.s1; ++s) {
             const uint32_t full = smem_addr(&bars[slot]);
             const uint32_t empty = smem_addr(&bars[C::kStages + slot]);
             if (!mbar_wait(empty, phase ^ 1, abort_flag)) {
@@ -340,32 +464,65 @@ __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, ui
         }
         const float Ms0 = M0 == -INFINITY ? 0.f : M0, Ms1 = M1 == -INFINITY ? 0.f : M1;
         const float f0 = dead ? 0.f : exp2f(m0 - Ms0), f1 = dead ? 0.f : exp2f(m1 - Ms1);
-        for (int w = 0; w < kDecodeConsumerWarps; ++w) {
-            if (w == warp) {
+        // the merged tile: member j's G rows, plus their (M, L), go to its
+        // partial entry
+        const int rows = n_grp * G;
+        const int32_t* ent = a.items[it].ent;
+        constexpr int kVecRow = D / 4;  // float4 per row
+        if (it + 1 == it1) {
+            // The CTA's last item: every warp is past its last stage (the
+            // barrier above) and no copy is pending, so the ring is free.
+            // Each warp leaves its rows there; all threads add the four.
+            float* wo = reinterpret_cast<float*>(smem) + warp * kRowsPerTile * C::kMergeStride;
 #pragma unroll
-                for (int nd = 0; nd < C::kNT; ++nd) {
-                    float2* p0 = reinterpret_cast<float2*>(red_o + r0 * C::kMergeStride + nd * 8 + tig * 2);
-                    float2* p1 = reinterpret_cast<float2*>(red_o + r1 * C::kMergeStride + nd * 8 + tig * 2);
-                    float2 a0 = dead ? make_float2(0.f, 0.f) : make_float2(o[nd][0] * f0, o[nd][1] * f0);
-                    float2 a1 = dead ? make_float2(0.f, 0.f) : make_float2(o[nd][2] * f1, o[nd][3] * f1);
-                    if (w > 0) {
-                        const float2 b0 = *p0, b1 = *p1;
-                        a0.x += b0.x; a0.y += b0.y;
-                        a1.x += b1.x; a1.y += b1.y;
-                    }
-                    *p0 = a0;
-                    *p1 = a1;
-                }
+            for (int nd = 0; nd < C::kNT; ++nd) {
+                *reinterpret_cast<float2*>(wo + r0 * C::kMergeStride + nd * 8 + tig * 2) =
+                    dead ? make_float2(0.f, 0.f) : make_float2(o[nd][0] * f0, o[nd][1] * f0);
+                *reinterpret_cast<float2*>(wo + r1 * C::kMergeStride + nd * 8 + tig * 2) =
+                    dead ? make_float2(0.f, 0.f) : make_float2(o[nd][2] * f1, o[nd][3] * f1);
             }
             named_bar_sync(1, kDecodeConsumerWarps * 32);
+            const float* ro = reinterpret_cast<const float*>(smem);
+            for (int v = threadIdx.x; v < rows * kVecRow; v += kDecodeConsumerWarps * 32) {
+                const int r = v / kVecRow, c4 = v % kVecRow;
+                float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int w = 0; w < kDecodeConsumerWarps; ++w) {
+                    const float4 x = *reinterpret_cast<const float4*>(
+                        ro + (w * kRowsPerTile + r) * C::kMergeStride + c4 * 4);
+                    sum.x += x.x; sum.y += x.y; sum.z += x.z; sum.w += x.w;
+                }
+                float* po = a.part_o + ((size_t)ent[r / G] * G + r % G) * D;
+                reinterpret_cast<float4*>(po)[c4] = sum;
+            }
+        } else {
+            // the ring is still in use: the four warps add in turn into one tile
+            for (int w = 0; w < kDecodeConsumerWarps; ++w) {
+                if (w == warp) {
+#pragma unroll
+                    for (int nd = 0; nd < C::kNT; ++nd) {
+                        float2* p0 = reinterpret_cast<float2*>(red_o + r0 * C::kMergeStride + nd * 8 + tig * 2);
+                        float2* p1 = reinterpret_cast<float2*>(red_o + r1 * C::kMergeStride + nd * 8 + tig * 2);
+                        float2 a0 = dead ? make_float2(0.f, 0.f) : make_float2(o[nd][0] * f0, o[nd][1] * f0);
+                        float2 a1 = dead ? make_float2(0.f, 0.f) : make_float2(o[nd][2] * f1, o[nd][3] * f1);
+                        if (w > 0) {
+                            const float2 b0 = *p0, b1 = *p1;
+                            a0.x += b0.x; a0.y += b0.y;
+                            a1.x += b1.x; a1.y += b1.y;
+                        }
+                        *p0 = a0;
+                        *p1 = a1;
+                    }
+                }
+                named_bar_sync(1, kDecodeConsumerWarps * 32);
+            }
+            for (int v = threadIdx.x; v < rows * kVecRow; v += kDecodeConsumerWarps * 32) {
+                const int r = v / kVecRow, c4 = v % kVecRow;
+                float* po = a.part_o + ((size_t)ent[r / G] * G + r % G) * D;
+                reinterpret_cast<float4*>(po)[c4] =
+                    *reinterpret_cast<const float4*>(red_o + r * C::kMergeStride + c4 * 4);
+            }
         }
-        // the merged tile: rows of the group's query heads, plus their (M, L)
-        const int rows = n_grp * G;
-        float* po = a.part_o + (size_t)it * kRowsPerTile * D;
-        constexpr int kVecRow = D / 4;  // float4 per row
-        for (int v = threadIdx.x; v < rows * kVecRow; v += kDecodeConsumerWarps * 32)
-            reinterpret_cast<float4*>(po)[v] = *reinterpret_cast<const float4*>(
-                red_o + (v / kVecRow) * C::kMergeStride + (v % kVecRow) * 4);
         if (threadIdx.x < rows) {
             const int r = threadIdx.x;
             float M = -INFINITY;
@@ -376,12 +533,166 @@ __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, ui
 #pragma unroll
             for (int w = 0; w < kDecodeConsumerWarps; ++w)
                 L += red_l[w * kRowsPerTile + r] * exp2f(red_m[w * kRowsPerTile + r] - Ms);
-            *reinterpret_cast<float2*>(a.part_ml + ((size_t)it * kRowsPerTile + r) * 2) =
-                make_float2(M, L);
+            *reinterpret_cast<float4*>(a.part_ml + ((size_t)ent[r / G] * G + r % G) * 4) =
+                make_float4(M, L, 0.f, 0.f);
         }
         // the merge buffers are rewritten by the next item only after every
         // warp has copied them out
         named_bar_sync(1, kDecodeConsumerWarps * 32);
+    }
+}
+
+// ---- arrivals and the merge of finished (sequence, KV head) runs -----------
+// The arrival word of a run counts the items that have written their partial;
+// the arrival that brings it to the run's length merges the run and sets the
+// word back to zero.  Every CTA arrives once per (item, group member), also
+// after a wait ran out, so every call leaves every word at zero, and a plan
+// upload writes zeros; the word therefore always starts a call at zero.
+
+// Up to 4 output float4 per thread per round; a round stages whole runs
+// (several when they fit) or one chunk of a long run.
+constexpr int kMergeOuts = 4;
+
+// Stages entries [c0, c0 + cn) of run r (first entry e0) at `dst`:
+// [cn][G][D] outputs, then [cn][G] (m, l, -, -) records.
+template <int D>
+__device__ __forceinline__ void stage_run(const DecodeArgs& a, uint32_t dst, int e0, int c0, int cn,
+                                          int tid) {
+    const int G = a.G;
+    const int nv_o = cn * G * (D / 4);
+    const float* so = a.part_o + (size_t)(e0 + c0) * G * D;
+    for (int v = tid; v < nv_o; v += kDecodeConsumerWarps * 32) cp_async_16(dst + v * 16, so + v * 4);
+    const float* sm = a.part_ml + (size_t)(e0 + c0) * G * 4;
+    const uint32_t dm = dst + nv_o * 16;
+    for (int v = tid; v < cn * G; v += kDecodeConsumerWarps * 32) cp_async_16(dm + v * 16, sm + v * 4);
+}
+
+template <int D>
+__device__ void arrive_and_merge(const DecodeArgs& a, int it0, int it1, uint8_t* ring, int* smem_i,
+                                 int warp) {
+    using C = DecCfg<D>;
+    constexpr int kT = kDecodeConsumerWarps * 32;
+    constexpr int kVec = D / 4;                       // float4 per output row
+    const int tid = threadIdx.x;
+    const int G = a.G;
+    const int outs_run = G * kVec;                    // output float4 of one run (<= 512)
+    const int ent_bytes = G * (D * 4 + 16);           // one staged entry
+    const int cap = C::kStages * C::kStageBytes / ent_bytes;  // entries per round (>= 11)
+    const uint32_t ring_s = smem_addr(ring);
+    int* n_last = smem_i;
+    int* l_key = smem_i + 1;        // completed runs: key, first entry, entries
+    int* l_e0 = l_key + kT;
+    int* l_n = l_e0 + kT;
+    int total = 0;
+    for (int it = it0; it < it1; ++it) total += a.segs[a.items[it].seg].n_grp;
+    for (int rb = 0; rb < total; rb += kT) {
+        if (tid == 0) *n_last = 0;
+        named_bar_sync(1, kT);
+        int key = -1;
+        for (int it = it0, p = 0; it < it1 && p <= rb + tid; ++it) {
+            const DecodeItem* item = a.items + it;
+            const DecodeSeg* seg = a.segs + item->seg;
+            const int j = rb + tid - p;
+            if (j < seg->n_grp) key = seg->grp_seq[j] * a.Hkv + item->head;
+            p += seg->n_grp;
+        }
+        if (key >= 0) {
+            const int e0 = a.comb_off[key], n = a.comb_off[key + 1] - e0;
+            // release: this CTA's partials (written before the barrier above)
+            // before the count; acquire: every counted partial before the reads
+            if (atom_add_acq_rel_gpu(a.arrive + key, 1u) + 1u == (unsigned)n) {
+                a.arrive[key] = 0u;
+                const int k = atomicAdd(n_last, 1);
+                l_key[k] = key;
+                l_e0[k] = e0;
+                l_n[k] = n;
+            }
+        }
+        named_bar_sync(1, kT);
+        const int nl = *reinterpret_cast<volatile int*>(n_last);
+        for (int k = 0; k < nl;) {
+            // whole runs while they fit, else chunks of the one run
+            int k1 = k, ents = 0;
+            while (k1 < nl && ents + l_n[k1] <= cap && (k1 - k + 1) * outs_run <= kMergeOuts * kT)
+                ents += l_n[k1++];
+            const bool chunked = k1 == k;
+            if (chunked) k1 = k + 1;
+            const int n_chunk = chunked ? l_n[k] : 0;
+            float Mr[kMergeOuts], Lr[kMergeOuts], acc[kMergeOuts][4];
+#pragma unroll
+            for (int r = 0; r < kMergeOuts; ++r) {
+                Mr[r] = -INFINITY;
+                Lr[r] = 0.f;
+                acc[r][0] = acc[r][1] = acc[r][2] = acc[r][3] = 0.f;
+            }
+            for (int c0 = 0; c0 < (chunked ? n_chunk : 1); c0 += cap) {
+                const int cn_chunk = chunked ? min(cap, n_chunk - c0) : 0;
+                // stage
+                uint32_t off = 0;
+                for (int q = k; q < k1; ++q) {
+                    const int cn = chunked ? cn_chunk : l_n[q];
+                    stage_run<D>(a, ring_s + off, l_e0[q], chunked ? c0 : 0, cn, tid);
+                    off += cn * ent_bytes;
+                }
+                cp_async_commit();
+                cp_async_wait<0>();
+                named_bar_sync(1, kT);
+                // merge this thread's outputs
+#pragma unroll
+                for (int r = 0; r < kMergeOuts; ++r) {
+                    const int o = tid + r * kT;
+                    if (o >= (k1 - k) * outs_run) continue;
+                    const int q = k + o / outs_run;
+                    const int row = (o % outs_run) / kVec, c4 = o % kVec;
+                    uint32_t base = 0;
+                    for (int t = k; t < q; ++t) base += l_n[t] * ent_bytes;
+                    const int cn = chunked ? cn_chunk : l_n[q];
+                    const float4* so = reinterpret_cast<const float4*>(ring + base);
+                    const float4* sm = so + cn * G * kVec;
+                    float bm = Mr[r];
+#pragma unroll 4
+                    for (int e = 0; e < cn; ++e) bm = fmaxf(bm, sm[e * G + row].x);
+                    const float bs = bm == -INFINITY ? 0.f : bm;
+                    const float sc = exp2f(Mr[r] - bs);
+                    Lr[r] *= sc;
+                    acc[r][0] *= sc; acc[r][1] *= sc; acc[r][2] *= sc; acc[r][3] *= sc;
+#pragma unroll 4
+                    for (int e = 0; e < cn; ++e) {
+                        const float4 ml = sm[e * G + row];
+                        const float w = exp2f(ml.x - bs);
+                        Lr[r] += w * ml.y;
+                        const float4 v = so[(e * G + row) * kVec + c4];
+                        acc[r][0] += w * v.x; acc[r][1] += w * v.y;
+                        acc[r][2] += w * v.z; acc[r][3] += w * v.w;
+                    }
+                    Mr[r] = bm;
+                }
+                named_bar_sync(1, kT);  // the staging is rewritten by the next round
+            }
+            // normalised outputs
+#pragma unroll
+            for (int r = 0; r < kMergeOuts; ++r) {
+                const int o = tid + r * kT;
+                if (o >= (k1 - k) * outs_run) continue;
+                const int q = k + o / outs_run;
+                const int row = (o % outs_run) / kVec, c4 = o % kVec;
+                const int rk = l_key[q];
+                const int i = rk / a.Hkv, h = (rk % a.Hkv) * G + row;
+                const float inv = 1.f / Lr[r];
+                const size_t ob = ((size_t)i * a.Hq + h) * D + c4 * 4;
+                if (a.out_f32) {
+                    *reinterpret_cast<float4*>(reinterpret_cast<float*>(a.out) + ob) = make_float4(
+                        acc[r][0] * inv, acc[r][1] * inv, acc[r][2] * inv, acc[r][3] * inv);
+                } else {
+                    uint2 u;
+                    u.x = pack_bf16x2(acc[r][0] * inv, acc[r][1] * inv);
+                    u.y = pack_bf16x2(acc[r][2] * inv, acc[r][3] * inv);
+                    *reinterpret_cast<uint2*>(reinterpret_cast<__nv_bfloat16*>(a.out) + ob) = u;
+                }
+            }
+            k = k1;
+        }
+        named_bar_sync(1, kT);  // the list is rewritten by the next batch of arrivals
     }
 }
 
@@ -404,106 +715,47 @@ __global__ void __launch_bounds__(DecCfg<D>::kThreads, 2)
         *abort_flag = 0;
         fence_mbar_init();
     }
+    // A reused plan is read before the wait: the producer keeps its item range
+    // and first stages in registers and warms L2 with the first stages' rows.
+    FastStart fs;
+    fs.n = 0;
+    int p_it0 = 0, p_it1 = 0;
+    if (warp == kDecodeConsumerWarps && lane == 0) {
+        prefetch_tmap(&tmap);
+        if (a.plan_ready) {
+            p_it0 = a.cta_begin[blockIdx.x];
+            p_it1 = a.cta_begin[blockIdx.x + 1];
+            if (a.P >= kStageTokens && (int)blockIdx.x != a.debug_drop_cta)
+                fast_start(a, p_it0, p_it1, fs);
+            prefetch_first_stages<D>(&tmap, a, p_it0, p_it1);
+        }
+    }
     __syncthreads();
     // Launched as a programmatic dependent: the set-up above overlapped the
     // previous kernel's tail; nothing it may have written is read before here.
     grid_dependency_wait();
-    grid_launch_dependents();  // the combine may be scheduled as CTAs retire
-    const int it0 = a.cta_begin[blockIdx.x], it1 = a.cta_begin[blockIdx.x + 1];
+    grid_launch_dependents();  // the next kernel may be scheduled as CTAs retire
     if (warp == kDecodeConsumerWarps) {
-        if (lane == 0) produce<D>(&tmap, a, it0, it1, smem, bars, abort_flag);
+        if (lane == 0) {
+            if (!a.plan_ready) {
+                p_it0 = a.cta_begin[blockIdx.x];
+                p_it1 = a.cta_begin[blockIdx.x + 1];
+            }
+            produce<D>(&tmap, a, p_it0, p_it1, fs, smem, bars, abort_flag);
+        }
         return;
     }
+    const int it0 = a.cta_begin[blockIdx.x], it1 = a.cta_begin[blockIdx.x + 1];
     consume<D>(a, it0, it1, smem, bars, abort_flag, merge, warp, lane);
-}
-
-// ---- combine: one warp per (sequence, query head) ---------------------------
-// Max of the partial maxima, weights 2^(m_c - M), weighted sums of the
-// unnormalised outputs and of the sums; loads of up to 8 partials in flight.
-template <int D>
-__global__ void __launch_bounds__(256) sq_lse_combine_kernel(const CombineArgs a) {
-    constexpr int V = D / 32;  // output elements per lane
-    constexpr int U = 8;       // partials per batch of loads
-    // programmatic dependent of the decode kernel: wait for its partials
-    grid_dependency_wait();
-    grid_launch_dependents();
-    const int wid = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    const int lane = threadIdx.x & 31;
-    if (wid >= a.n_seqs * a.Hq) return;
-    const int i = wid / a.Hq, h = wid % a.Hq;
-    const int hh = h % a.G;
-    const int key = i * a.Hkv + h / a.G;
-    const int e0 = a.comb_off[key], e1 = a.comb_off[key + 1];
-    const int np = e1 - e0;
-
-    float M = -INFINITY;
-    for (int k = lane; k < np; k += 32) {
-        const CombineEnt ent = a.comb_ent[e0 + k];
-        M = fmaxf(M, a.part_ml[((size_t)ent.item * kRowsPerTile + ent.j * a.G + hh) * 2]);
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-    const float Ms = M == -INFINITY ? 0.f : M;
-
-    float acc[V];
-#pragma unroll
-    for (int e = 0; e < V; ++e) acc[e] = 0.f;
-    float L = 0.f;
-    for (int k0 = 0; k0 < np; k0 += U) {
-        float w[U];
-        float vals[U][V];
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            w[u] = 0.f;
-#pragma unroll
-            for (int e = 0; e < V; ++e) vals[u][e] = 0.f;
-            if (k0 + u < np) {
-                const CombineEnt ent = a.comb_ent[e0 + k0 + u];
-                const size_t row = (size_t)ent.item * kRowsPerTile + ent.j * a.G + hh;
-                const float2 ml = *reinterpret_cast<const float2*>(a.part_ml + row * 2);
-                w[u] = exp2f(ml.x - Ms);
-                L += w[u] * ml.y;
-                const float* po = a.part_o + row * D + lane * V;
-                if constexpr (V == 4) {
-                    const float4 v = *reinterpret_cast<const float4*>(po);
-                    vals[u][0] = v.x; vals[u][1] = v.y; vals[u][2] = v.z; vals[u][3] = v.w;
-                } else {
-                    const float2 v = *reinterpret_cast<const float2*>(po);
-                    vals[u][0] = v.x; vals[u][1] = v.y;
-                }
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < U; ++u)
-#pragma unroll
-            for (int e = 0; e < V; ++e) acc[e] += w[u] * vals[u][e];
-    }
-    const float inv = 1.f / L;
-    const size_t ob = ((size_t)i * a.Hq + h) * D + lane * V;
-    if (a.out_f32) {
-        float* out = reinterpret_cast<float*>(a.out) + ob;
-        if constexpr (V == 4)
-            *reinterpret_cast<float4*>(out) =
-                make_float4(acc[0] * inv, acc[1] * inv, acc[2] * inv, acc[3] * inv);
-        else
-            *reinterpret_cast<float2*>(out) = make_float2(acc[0] * inv, acc[1] * inv);
-    } else {
-        __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.out) + ob;
-        if constexpr (V == 4) {
-            uint2 u;
-            u.x = pack_bf16x2(acc[0] * inv, acc[1] * inv);
-            u.y = pack_bf16x2(acc[2] * inv, acc[3] * inv);
-            *reinterpret_cast<uint2*>(out) = u;
-        } else {
-            *reinterpret_cast<uint32_t*>(out) = pack_bf16x2(acc[0] * inv, acc[1] * inv);
-        }
-    }
+    // the ring and the merge buffers are free again (every stage consumed, the
+    // last item ended on a barrier)
+    arrive_and_merge<D>(a, it0, it1, smem, reinterpret_cast<int*>(merge), warp);
 }
 
 }  // namespace
 
-int64_t decode_partial_bytes(int32_t n_items, int32_t D) {
-    return (int64_t)n_items * kRowsPerTile * (D + 2) * (int64_t)sizeof(float);
+int64_t decode_partial_bytes(int32_t n_ent, int32_t G, int32_t D) {
+    return (int64_t)n_ent * G * (D + 4) * (int64_t)sizeof(float);
 }
 
 template <int D>
@@ -535,9 +787,9 @@ int decode_ctas_per_sm(int D) {
     return n;
 }
 
-// Both kernels are launched as programmatic dependents of whatever precedes
-// them on the stream: each waits (griddepcontrol.wait) before it reads
-// anything, so the launch latency overlaps the previous kernel's tail.
+// The kernel is launched as a programmatic dependent of whatever precedes it
+// on the stream: it waits (griddepcontrol.wait) before it reads anything the
+// preceding work may write, so its launch and set-up overlap that work's tail.
 static cudaLaunchAttribute pdl_attr() {
     cudaLaunchAttribute at;
     at.id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -561,19 +813,6 @@ cudaError_t launch_decode(const CUtensorMap& tmap, const DecodeArgs& a, int n_ct
     cfg.blockDim = dim3(DecCfg<64>::kThreads);
     cfg.dynamicSmemBytes = DecCfg<64>::kSmemBytes;
     return cudaLaunchKernelEx(&cfg, sq_decode_splitk_kernel<64>, tmap, a);
-}
-
-cudaError_t launch_combine(const CombineArgs& a, int D, cudaStream_t st) {
-    const int warps = a.n_seqs * a.Hq;
-    cudaLaunchAttribute at = pdl_attr();
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((warps + 7) / 8);
-    cfg.blockDim = dim3(256);
-    cfg.stream = st;
-    cfg.attrs = &at;
-    cfg.numAttrs = 1;
-    if (D == 128) return cudaLaunchKernelEx(&cfg, sq_lse_combine_kernel<128>, a);
-    return cudaLaunchKernelEx(&cfg, sq_lse_combine_kernel<64>, a);
 }
 
 }  // namespace sq

@@ -16,33 +16,29 @@ struct DecodeArgs {
     const DecodeItem* items;
     const int32_t* cta_begin;
     const int32_t* page_ids;
+    const int32_t* comb_off;    // [n_seqs * Hkv + 1] partial entries of each (sequence, KV head)
+    unsigned int* arrive;       // [n_seqs * Hkv] arrival counts, zero between calls
     const __nv_bfloat16* q;     // [n_seqs][Hq][D]
-    float* part_o;              // [n_items][16][D]  unnormalised partial outputs
-    float* part_ml;             // [n_items][16][2]  max (log2 units), sum
+    void* out;                  // [n_seqs][Hq][D] bf16 or fp32
+    float* part_o;              // [n_ent][G][D]  unnormalised partial outputs
+    float* part_ml;             // [n_ent][G][4]  max (log2 units), sum, unused, unused
+    int32_t out_f32;
+    // 1: the plan was on the device before whatever precedes this launch on
+    // the stream, so it may be read before the grid-dependency wait
+    int32_t plan_ready;
     int32_t layer, Hq, Hkv, G, P, num_pages;
     float scale_log2;           // sm_scale * log2(e)
     int32_t debug_drop_cta;     // test hook: this CTA leaves its first stage unsignalled (-1: none)
     int* err;
 };
 
-struct CombineArgs {
-    const int32_t* comb_off;    // [n_seqs * Hkv + 1]
-    const CombineEnt* comb_ent;
-    const float* part_o;
-    const float* part_ml;
-    void* out;                  // [n_seqs][Hq][D] bf16 or fp32
-    int32_t out_f32;
-    int32_t n_seqs, Hq, Hkv, G;
-};
-
-// Bytes of partial results one decode plan needs.
-int64_t decode_partial_bytes(int32_t n_items, int32_t D);
+// Bytes of partial results one decode plan needs (n_ent partial entries).
+int64_t decode_partial_bytes(int32_t n_ent, int32_t G, int32_t D);
 // Persistent CTAs per SM the decode kernel runs with (occupancy of the kernel).
 int decode_ctas_per_sm(int D);
 cudaError_t decode_prepare(int D);  // raises the dynamic shared-memory limit once
 cudaError_t launch_decode(const CUtensorMap& tmap, const DecodeArgs& a, int n_ctas, int D,
                           cudaStream_t st);
-cudaError_t launch_combine(const CombineArgs& a, int D, cudaStream_t st);
 
 // ---- masked prefill attention -------------------------------------------------
 struct PrefillArgs {

@@ -15,6 +15,7 @@ from paper_2602_22603_gb300 import build as _build  # noqa: E402
 _lib = None
 
 SEG_INTS = 4 + 2 * 16  # DecodeSeg: page_off, n_pages, n_tok, n_grp, grp_seq[16], grp_lim[16]
+ITEM_INTS = 4 + 16     # DecodeItem: seg, head, s0, s1, ent[16]
 
 
 def lib():
@@ -157,15 +158,32 @@ class HostCache:
 
         n_segs, n_items, n_ctas_, n_pid, n_keys, n_ent = L[7:13]
         segs = arr_at(L[0], n_segs, SEG_INTS)
+        seg_list = [{"page_off": int(s[0]), "n_pages": int(s[1]), "n_tok": int(s[2]),
+                     "n_grp": int(s[3]), "grp_seq": [int(x) for x in s[4:4 + s[3]]],
+                     "grp_lim": [int(x) for x in s[20:20 + s[3]]]} for s in segs]
+        raw_items = arr_at(L[1], n_items, ITEM_INTS) if n_items else np.zeros((0, ITEM_INTS), np.int32)
+        comb_off = arr_at(L[4], n_keys + 1).tolist()
+        # each item's group members name their partial entry; every entry is
+        # named once, inside the range of its (sequence, KV head)
+        comb_ent = [None] * n_ent
+        for it, row in enumerate(raw_items):
+            seg = seg_list[row[0]]
+            for j in range(seg["n_grp"]):
+                e = int(row[4 + j])
+                key = seg["grp_seq"][j] * self.Hkv + int(row[1])
+                assert comb_off[key] <= e < comb_off[key + 1], (it, j, e)
+                assert comb_ent[e] is None, e
+                comb_ent[e] = [it, j]
+        assert all(x is not None for x in comb_ent)
+        arrive = buf[L[5]:L[5] + 4 * n_keys]
+        assert L[5] % 4 == 0 and not arrive.any()
         plan = {
-            "segs": [{"page_off": int(s[0]), "n_pages": int(s[1]), "n_tok": int(s[2]),
-                      "n_grp": int(s[3]), "grp_seq": [int(x) for x in s[4:4 + s[3]]],
-                      "grp_lim": [int(x) for x in s[20:20 + s[3]]]} for s in segs],
-            "items": arr_at(L[1], n_items, 4).tolist() if n_items else [],
+            "segs": seg_list,
+            "items": raw_items[:, :4].tolist(),
             "cta_begin": arr_at(L[2], n_ctas_ + 1).tolist(),
             "page_ids": arr_at(L[3], n_pid).tolist(),
-            "comb_off": arr_at(L[4], n_keys + 1).tolist(),
-            "comb_ent": arr_at(L[5], n_ent, 2).tolist() if n_ent else [],
+            "comb_off": comb_off,
+            "comb_ent": comb_ent,
             "unique_tokens": L[13], "logical_tokens": L[14],
         }
         return 0, plan

@@ -121,6 +121,63 @@ def test_split_invariance_over_cta_counts():
         assert (o - outs[0]).abs().max().item() < 5e-4
 
 
+def test_one_cta_merges_hundreds_of_runs():
+    """decode_ctas = 1: the one CTA holds every item (40 sequences, 8 KV heads:
+    320 arrivals, three rounds of 128) and completes, so merges, every
+    (sequence, KV head) run itself; forks make two-member groups too."""
+    p = Pair(1, 32, 8, 128, 16, num_pages=700, decode_ctas=1, seed=52)
+    rng = np.random.default_rng(52)
+    keep = []
+    seqs = []
+    for i in range(30):
+        h = p.seq_new()
+        keep.append(p.append(h, int(rng.integers(1, 300))))
+        seqs.append(h)
+    for h in seqs[:10]:
+        f = p.fork(h)
+        keep.append(p.append(f, int(rng.integers(1, 20))))
+        seqs.append(f)
+    _decode_check(p, seqs, 0, 0.0884, 53)
+    p.close()
+
+
+def test_decode_replayed_from_a_cuda_graph():
+    """Replays of a captured decode repeat its kernel arguments, the merge's
+    arrival tag among them: every replay must still merge each run once
+    (the last arrival clears the word), with fresh queries each time."""
+    p = Pair(2, 32, 8, 128, 64, num_pages=200, decode_ctas=300, seed=54)
+    keep = []
+    m = p.seq_new()
+    keep.append(p.append(m, 3000))
+    a = p.fork(m)
+    keep.append(p.append(a, 40))
+    seqs = [m, a]
+    q = torch.zeros(2, 32, 128, dtype=torch.bfloat16, device="cuda")
+    outs = [torch.zeros(2, 32, 128, device="cuda") for _ in range(2)]
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        for layer in range(2):      # plans made and cached on the capture stream
+            p.cache.decode_attention(seqs, layer, q, outs[layer], sq.SQ_OUT_F32, 0.09)
+    s.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        for layer in range(2):
+            p.cache.decode_attention(seqs, layer, q, outs[layer], sq.SQ_OUT_F32, 0.09)
+    for rep in range(3):
+        q_cpu = bf16_normal((2, 32, 128), 60 + rep)
+        q.copy_(q_cpu.cuda())
+        for o in outs:
+            o.fill_(float("nan"))
+        g.replay()
+        torch.cuda.synchronize()
+        assert p.cache.sync_status() == sq.SQ_OK
+        for layer in range(2):
+            assert_close(outs[layer], p.oracle_decode(seqs, layer, 0.09, q_cpu), max_abs=5e-3)
+    del g
+    p.close()
+
+
 @pytest.mark.parametrize("seed", range(4))
 def test_random_forks_appends_evictions(seed):
     rng = random.Random(seed)

@@ -67,16 +67,21 @@ def test_noalloc_matches_regular_entry_point_two_calls_in_a_row():
 
 
 def test_noalloc_rejects_plans_beyond_the_scratch():
-    # 8 KV heads x 512 stages over 4096 persistent CTAs -> 4096 partial items,
-    # ~136 MB of partials: more than the fixed scratch holds
-    p = Pair(1, 32, 8, 128, 64, num_pages=600, seed=43, decode_ctas=4096)
-    keep = [None]
-    m = p.seq_new()
-    keep.append(p.append(m, 32768))
-    q = bf16_normal((1, 32, 128), 1).cuda()
-    out = torch.zeros(1, 32, 128, device="cuda")
-    assert _noalloc_c(p.cache, [m], 0, q, out, sq.SQ_OUT_F32, 0.1) == sq.SQ_ERR_CAPACITY
-    torch.cuda.synchronize()
-    assert torch.count_nonzero(out).item() == 0     # nothing was enqueued
-    assert p.cache.sync_status() == sq.SQ_OK
-    p.close()
+    # 8 KV heads x 2048 stages over 16384 persistent CTAs -> about 16,390
+    # partial entries of G = 4 rows: ~34 MB of partials plus ~1.4 MB of plan,
+    # more than the fixed scratch holds
+    n = 131072
+    c = sq.Cache(1, 32, 8, 128, 64, n // 64 + 4, max_seqs=4, decode_ctas=16384)
+    try:
+        m = c.seq_new()
+        kv = torch.zeros(1, 4096, 8, 128, dtype=torch.bfloat16, device="cuda")
+        for _ in range(n // 4096):
+            c.append_kv(m, 4096, kv, kv)
+        q = bf16_normal((1, 32, 128), 1).cuda()
+        out = torch.zeros(1, 32, 128, device="cuda")
+        assert _noalloc_c(c, [m], 0, q, out, sq.SQ_OUT_F32, 0.1) == sq.SQ_ERR_CAPACITY
+        torch.cuda.synchronize()
+        assert torch.count_nonzero(out).item() == 0     # nothing was enqueued
+        assert c.sync_status() == sq.SQ_OK
+    finally:
+        c.close()
