@@ -387,15 +387,21 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
 
     // Group sequences holding the same physical page at the same logical
     // index into shared runs (depth-first over the prefix tree of pages).
+    // Every segment also records its family: the subtree of one first page
+    // (a request, its forks and whatever they added).
     struct Work {
         std::vector<int32_t> members;
         int32_t q;
+        int32_t fam;  // -1 at the root
     };
     std::vector<Work> stack;
+    std::vector<int32_t> seg_fam;
+    int32_t n_fam = 0;
     {
         Work root;
         for (int32_t i = 0; i < n_seqs; ++i) root.members.push_back(i);
         root.q = 0;
+        root.fam = -1;
         stack.push_back(std::move(root));
     }
     while (!stack.empty()) {
@@ -418,6 +424,7 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
         // process parts in order: push in reverse so the first is handled first
         std::vector<Work> next;
         for (auto& part : parts) {
+            const int32_t fam = w.fam >= 0 ? w.fam : n_fam++;
             const int32_t q0 = w.q;
             int32_t q_end = q0 + 1;
             const Seq* lead = ss[part[0]];
@@ -453,11 +460,13 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
                 for (int32_t q = q0; q < q_end; ++q) out->page_ids.push_back(sl->pages[q]);
                 out->unique_tokens += seg.n_tok;
                 out->segs.push_back(seg);
+                seg_fam.push_back(fam);
             }
             Work nw;
             for (int32_t i : part)
                 if ((int32_t)ss[i]->pages.size() > q_end) nw.members.push_back(i);
             nw.q = q_end;
+            nw.fam = fam;
             if (!nw.members.empty()) next.push_back(std::move(nw));
         }
         for (auto it = next.rbegin(); it != next.rend(); ++it) stack.push_back(std::move(*it));
@@ -466,18 +475,36 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
     // (segment, head) units and an even split of their cost over the
     // persistent CTAs.  On the cost line a unit occupies kUnitCostStages
     // (its start-up) followed by its stages; an item is the overlap of a
-    // CTA's share with a unit's stages.
+    // CTA's share with a unit's stages.  Units go family by family, head by
+    // head, each family's segments in tree order: a fork's own short tail
+    // follows the shared prefix of the same head, so it lands in the CTA that
+    // finishes that prefix instead of in a pile of tails at the end of the
+    // line (whose one CTA would then merge every fork's rows alone).
     const int32_t n_segs = (int32_t)out->segs.size();
+    std::vector<int32_t> by_fam(n_segs);
+    for (int32_t s = 0; s < n_segs; ++s) by_fam[s] = s;
+    std::stable_sort(by_fam.begin(), by_fam.end(),
+                     [&](int32_t x, int32_t y) { return seg_fam[x] < seg_fam[y]; });
+    std::vector<int32_t> unit_seg, unit_head;
+    for (int32_t b = 0; b < n_segs;) {
+        int32_t e = b;
+        while (e < n_segs && seg_fam[by_fam[e]] == seg_fam[by_fam[b]]) ++e;
+        for (int32_t h = 0; h < g.Hkv; ++h)
+            for (int32_t x = b; x < e; ++x) {
+                unit_seg.push_back(by_fam[x]);
+                unit_head.push_back(h);
+            }
+        b = e;
+    }
     std::vector<int64_t> unit_start;  // where the unit's stages begin on the cost line
     std::vector<int64_t> unit_end;
     int64_t total = 0;
-    for (int32_t s = 0; s < n_segs; ++s)
-        for (int32_t h = 0; h < g.Hkv; ++h) {
-            total += kUnitCostStages;
-            unit_start.push_back(total);
-            total += ceil_div(out->segs[s].n_tok, kStageTokens);
-            unit_end.push_back(total);
-        }
+    for (size_t v = 0; v < unit_seg.size(); ++v) {
+        total += kUnitCostStages;
+        unit_start.push_back(total);
+        total += ceil_div(out->segs[unit_seg[v]].n_tok, kStageTokens);
+        unit_end.push_back(total);
+    }
     const int64_t n_units = (int64_t)unit_start.size();
     const int32_t ctas = (int32_t)std::min<int64_t>(n_ctas, total - n_units * kUnitCostStages);
     out->n_ctas = ctas;
@@ -492,8 +519,8 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
             if (hi <= lo) continue;
             DecodeItem it;
             std::memset(&it, 0, sizeof it);
-            it.seg = (int32_t)(v / g.Hkv);
-            it.head = (int32_t)(v % g.Hkv);
+            it.seg = unit_seg[v];
+            it.head = unit_head[v];
             it.s0 = (int32_t)(lo - unit_start[v]);
             it.s1 = (int32_t)(hi - unit_start[v]);
             out->items.push_back(it);
@@ -512,7 +539,12 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
     std::vector<int32_t> fill(out->comb_off.begin(), out->comb_off.end() - 1);
     for (DecodeItem& it : out->items) {
         const DecodeSeg& s = out->segs[it.seg];
-        for (int32_t j = 0; j < s.n_grp; ++j) it.ent[j] = fill[s.grp_seq[j] * g.Hkv + it.head]++;
+        it.sole = 0;
+        for (int32_t j = 0; j < s.n_grp; ++j) {
+            const int32_t key = s.grp_seq[j] * g.Hkv + it.head;
+            it.ent[j] = fill[key]++;
+            if (out->comb_off[key + 1] - out->comb_off[key] == 1) it.sole |= 1 << j;
+        }
     }
     return kOk;
 }

@@ -33,11 +33,13 @@ struct DecodeSeg {
 // A contiguous range of stages of one (segment, KV head) — one partial result
 // per group member.  Member j's G rows go to partial entry ent[j]; the entries
 // of one (sequence, KV head) are contiguous, so that its merge reads them
-// without an index.
+// without an index.  A member whose (sequence, KV head) has this one entry
+// only (bit j of `sole`) gets its normalised output written directly.
 struct DecodeItem {
     int32_t seg;
     int32_t head;
     int32_t s0, s1;                   // stages [s0, s1)
+    int32_t sole;                     // bit j: member j's run is this item alone
     int32_t ent[kRowsPerTile];        // partial entry of each group member (n_grp used)
 };
 

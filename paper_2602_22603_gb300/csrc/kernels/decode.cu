@@ -57,7 +57,7 @@ struct DecCfg {
     // and one 16-row output tile
     static constexpr int kMergeStride = D + 8;  // floats per merge row (padded: fewer bank conflicts)
     static constexpr int kMergeBytes = 2 * kDecodeConsumerWarps * kRowsPerTile * 4 +
-                                       kRowsPerTile * kMergeStride * 4;
+                                       kRowsPerTile * kMergeStride * 4 + kRowsPerTile * 4;
     // + 1024 alignment slack + 256 for the mbarriers and flags
     static constexpr int kSmemBytes = kStages * kStageBytes + kMergeBytes + 1024 + 256;
     static constexpr int kNT = D / 8;   // 8-wide output column tiles
@@ -283,6 +283,7 @@ __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, ui
     float* red_m = merge;                                          // [4][16]
     float* red_l = merge + kDecodeConsumerWarps * kRowsPerTile;    // [4][16]
     float* red_o = merge + 2 * kDecodeConsumerWarps * kRowsPerTile;  // [16][kMergeStride]
+    float* red_sum = red_o + kRowsPerTile * C::kMergeStride;          // [16] merged row sums
     int slot = 0;
     uint32_t phase = 0;
     bool dead = false;  // warp-uniform: a wait ran out or the CTA aborted
@@ -465,10 +466,49 @@ __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, ui
         const float Ms0 = M0 == -INFINITY ? 0.f : M0, Ms1 = M1 == -INFINITY ? 0.f : M1;
         const float f0 = dead ? 0.f : exp2f(m0 - Ms0), f1 = dead ? 0.f : exp2f(m1 - Ms1);
         // the merged tile: member j's G rows, plus their (M, L), go to its
-        // partial entry
+        // partial entry; a member whose run is this item alone gets its
+        // normalised output instead
         const int rows = n_grp * G;
         const int32_t* ent = a.items[it].ent;
+        const int sole = a.items[it].sole;
         constexpr int kVecRow = D / 4;  // float4 per row
+        if (threadIdx.x < rows) {
+            const int r = threadIdx.x;
+            float M = -INFINITY;
+#pragma unroll
+            for (int w = 0; w < kDecodeConsumerWarps; ++w) M = fmaxf(M, red_m[w * kRowsPerTile + r]);
+            const float Ms = M == -INFINITY ? 0.f : M;
+            float L = 0.f;
+#pragma unroll
+            for (int w = 0; w < kDecodeConsumerWarps; ++w)
+                L += red_l[w * kRowsPerTile + r] * exp2f(red_m[w * kRowsPerTile + r] - Ms);
+            red_sum[r] = L;
+            if (!((sole >> (r / G)) & 1))
+                *reinterpret_cast<float4*>(a.part_ml + ((size_t)ent[r / G] * G + r % G) * 4) =
+                    make_float4(M, L, 0.f, 0.f);
+        }
+        // one row's float4 of the merged tile to its destination (read after
+        // a barrier that follows the red_sum writes)
+        auto put = [&](int r, int c4, float4 v) {
+            const int j = r / G;
+            if ((sole >> j) & 1) {
+                const float inv = 1.f / red_sum[r];
+                const size_t ob =
+                    ((size_t)seg->grp_seq[j] * a.Hq + item.head * G + r % G) * D + c4 * 4;
+                if (a.out_f32) {
+                    *reinterpret_cast<float4*>(reinterpret_cast<float*>(a.out) + ob) =
+                        make_float4(v.x * inv, v.y * inv, v.z * inv, v.w * inv);
+                } else {
+                    uint2 u;
+                    u.x = pack_bf16x2(v.x * inv, v.y * inv);
+                    u.y = pack_bf16x2(v.z * inv, v.w * inv);
+                    *reinterpret_cast<uint2*>(reinterpret_cast<__nv_bfloat16*>(a.out) + ob) = u;
+                }
+            } else {
+                float* po = a.part_o + ((size_t)ent[j] * G + r % G) * D;
+                reinterpret_cast<float4*>(po)[c4] = v;
+            }
+        };
         if (it + 1 == it1) {
             // The CTA's last item: every warp is past its last stage (the
             // barrier above) and no copy is pending, so the ring is free.
@@ -492,8 +532,7 @@ __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, ui
                         ro + (w * kRowsPerTile + r) * C::kMergeStride + c4 * 4);
                     sum.x += x.x; sum.y += x.y; sum.z += x.z; sum.w += x.w;
                 }
-                float* po = a.part_o + ((size_t)ent[r / G] * G + r % G) * D;
-                reinterpret_cast<float4*>(po)[c4] = sum;
+                put(r, c4, sum);
             }
         } else {
             // the ring is still in use: the four warps add in turn into one tile
@@ -518,23 +557,8 @@ __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, ui
             }
             for (int v = threadIdx.x; v < rows * kVecRow; v += kDecodeConsumerWarps * 32) {
                 const int r = v / kVecRow, c4 = v % kVecRow;
-                float* po = a.part_o + ((size_t)ent[r / G] * G + r % G) * D;
-                reinterpret_cast<float4*>(po)[c4] =
-                    *reinterpret_cast<const float4*>(red_o + r * C::kMergeStride + c4 * 4);
+                put(r, c4, *reinterpret_cast<const float4*>(red_o + r * C::kMergeStride + c4 * 4));
             }
-        }
-        if (threadIdx.x < rows) {
-            const int r = threadIdx.x;
-            float M = -INFINITY;
-#pragma unroll
-            for (int w = 0; w < kDecodeConsumerWarps; ++w) M = fmaxf(M, red_m[w * kRowsPerTile + r]);
-            const float Ms = M == -INFINITY ? 0.f : M;
-            float L = 0.f;
-#pragma unroll
-            for (int w = 0; w < kDecodeConsumerWarps; ++w)
-                L += red_l[w * kRowsPerTile + r] * exp2f(red_m[w * kRowsPerTile + r] - Ms);
-            *reinterpret_cast<float4*>(a.part_ml + ((size_t)ent[r / G] * G + r % G) * 4) =
-                make_float4(M, L, 0.f, 0.f);
         }
         // the merge buffers are rewritten by the next item only after every
         // warp has copied them out
@@ -593,7 +617,7 @@ __device__ void arrive_and_merge(const DecodeArgs& a, int it0, int it1, uint8_t*
             const DecodeItem* item = a.items + it;
             const DecodeSeg* seg = a.segs + item->seg;
             const int j = rb + tid - p;
-            if (j < seg->n_grp) key = seg->grp_seq[j] * a.Hkv + item->head;
+            if (j < seg->n_grp && !((item->sole >> j) & 1)) key = seg->grp_seq[j] * a.Hkv + item->head;
             p += seg->n_grp;
         }
         if (key >= 0) {

@@ -15,7 +15,7 @@ from paper_2602_22603_gb300 import build as _build  # noqa: E402
 _lib = None
 
 SEG_INTS = 4 + 2 * 16  # DecodeSeg: page_off, n_pages, n_tok, n_grp, grp_seq[16], grp_lim[16]
-ITEM_INTS = 4 + 16     # DecodeItem: seg, head, s0, s1, ent[16]
+ITEM_INTS = 5 + 16     # DecodeItem: seg, head, s0, s1, sole, ent[16]
 
 
 def lib():
@@ -169,11 +169,13 @@ class HostCache:
         for it, row in enumerate(raw_items):
             seg = seg_list[row[0]]
             for j in range(seg["n_grp"]):
-                e = int(row[4 + j])
+                e = int(row[5 + j])
                 key = seg["grp_seq"][j] * self.Hkv + int(row[1])
                 assert comb_off[key] <= e < comb_off[key + 1], (it, j, e)
                 assert comb_ent[e] is None, e
                 comb_ent[e] = [it, j]
+                # the sole bit marks exactly the one-entry runs
+                assert bool((int(row[4]) >> j) & 1) == (comb_off[key + 1] - comb_off[key] == 1)
         assert all(x is not None for x in comb_ent)
         arrive = buf[L[5]:L[5] + 4 * n_keys]
         assert L[5] % 4 == 0 and not arrive.any()
