@@ -198,6 +198,62 @@ def test_decode_plan_reads_shared_prefix_once():
     assert plan["logical_tokens"] == 4097 + 4104
 
 
+def test_decode_plan_spreads_fork_tails():
+    # 8 requests of 32,768 tokens, each with a fork holding an 8-token tail
+    # of its own (the aux trigger): 64 one-stage tail units among 64 prefix
+    # units of 512 stages.  Units go family by family, head by head, so each
+    # tail follows the prefix unit of its own head: no CTA holds more than a
+    # few tails, and each tail's CTA also holds the end of that prefix.
+    Hkv = 8
+    hc = HostCache(1, 32, Hkv, 128, 64, 8 * 520)
+    seqs = []
+    for _ in range(8):
+        rc, m = hc.seq_new()
+        assert hc.append(m, 32768) == 0
+        rc, a = hc.fork(m)
+        assert hc.append(a, 8) == 0
+        seqs += [m, a]
+    rc, plan = hc.plan_decode(seqs, 304)
+    assert rc == 0
+    _check_plan(hc, seqs, plan, 304, 4)
+    segs, items, cb = plan["segs"], plan["items"], plan["cta_begin"]
+    tails_per_cta = []
+    for c in range(len(cb) - 1):
+        its = items[cb[c]:cb[c + 1]]
+        tails = [it for it in its if segs[it[0]]["n_tok"] == 8]
+        tails_per_cta.append(len(tails))
+        for t in tails:
+            # the same CTA ends the shared prefix of the tail's head (or the
+            # tail starts the CTA right after it)
+            fork_seq = segs[t[0]]["grp_seq"][0]
+            prefix = [it for it in items[max(0, cb[c] - 1):cb[c + 1]]
+                      if segs[it[0]]["n_grp"] == 2 and fork_seq in segs[it[0]]["grp_seq"]
+                      and it[1] == t[1]]
+            assert prefix, (c, t)
+    assert sum(tails_per_cta) == 8 * Hkv
+    assert max(tails_per_cta) <= 2
+    # a fork's (sequence, head) run: its prefix entries and its tail; the
+    # tails are never alone, so no tail member is marked sole
+    assert all(len(plan["comb_ent"][plan["comb_off"][k]:plan["comb_off"][k + 1]]) > 1
+               for k in range(len(plan["comb_off"]) - 1))
+
+
+def test_decode_plan_marks_single_item_runs():
+    # many short sequences, one CTA: every (sequence, head) run is one item,
+    # so every member is marked sole (the parse of the plan checks the mark
+    # against the run lengths)
+    hc = HostCache(1, 16, 4, 64, 16, 400)
+    seqs = []
+    for n in (1, 5, 16, 17, 40):
+        rc, h = hc.seq_new()
+        assert hc.append(h, n) == 0
+        seqs.append(h)
+    rc, plan = hc.plan_decode(seqs, 1)
+    assert rc == 0
+    offs = plan["comb_off"]
+    assert all(offs[k + 1] - offs[k] == 1 for k in range(len(offs) - 1))
+
+
 def test_decode_plan_rejects_bad_input():
     hc = HostCache(1, 8, 2, 64, 16, 100)
     rc, m = hc.seq_new()
