@@ -483,20 +483,24 @@ def run_sq(args, world, rank, local):
             cache.release(a)
         torch.cuda.synchronize()
         st0 = cache.stats()
-        ev_ms = 0.0
-        per = []
+        # One eviction per request, enqueued back to back: the host planning
+        # of each call overlaps the GPU work of the one before (a GPU sleep
+        # covers the first), and the events between calls give each call's
+        # GPU time: copy-on-write copies and the compaction kernel.
+        span_list = [spec["spans"](seed, r, cache.seq_info(m)[0], P) for r, m in enumerate(mains)]
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(mains) + 1)]
+        b = []
+        torch.cuda._sleep(2_000_000)
+        evs[0].record(stream)
         for r, m in enumerate(mains):
-            n = cache.seq_info(m)[0]
-            spans = spec["spans"](seed, r, n, P)
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            b0 = cache.stats()["evict_bytes"]
-            e0.record(stream)
-            cache.evict_spans(m, spans)
-            e1.record(stream)
-            torch.cuda.synchronize()
-            ms = e0.elapsed_time(e1)
-            ev_ms += ms
-            per.append((cache.stats()["evict_bytes"] - b0) / (ms / 1e3) / 1e9)
+            b.append(cache.stats()["evict_bytes"])
+            cache.evict_spans(m, span_list[r])
+            evs[r + 1].record(stream)
+        torch.cuda.synchronize()
+        b.append(cache.stats()["evict_bytes"])
+        per_ms = [evs[r].elapsed_time(evs[r + 1]) for r in range(len(mains))]
+        ev_ms = sum(per_ms)
+        per = [(b[r + 1] - b[r]) / (per_ms[r] / 1e3) / 1e9 for r in range(len(mains))]
         st1 = cache.stats()
         ev_bytes = st1["evict_bytes"] - st0["evict_bytes"]
         assert cache.sync_status() == sq.SQ_OK
@@ -521,6 +525,7 @@ def run_sq(args, world, rank, local):
             "moved_rows": int(st1["evict_moved_rows"] - st0["evict_moved_rows"]),
             "per_request_gbs": [round(x, 1) for x in per],
             "calls": len(mains),
+            "timing": "GPU time per call, calls enqueued back to back (host planning overlapped)",
         }
         res["after_evict"] = {
             "tokens_per_s": round(world * S * K / (max_over_ranks(after["total_ms"], world) / 1e3), 3),
