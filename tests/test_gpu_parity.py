@@ -121,6 +121,30 @@ def test_split_invariance_over_cta_counts():
         assert (o - outs[0]).abs().max().item() < 5e-4
 
 
+@pytest.mark.parametrize("Hq,Hkv,D,P,ctas,n", [
+    (32, 2, 64, 32, 400, 9000),    # G = 16: runs of ~140 entries merge in chunks of 22
+    (6, 2, 128, 256, 200, 3000),   # G = 3: several runs per merge round (96 outputs each)
+    (8, 8, 64, 16, 300, 2000),     # G = 1, d = 64: 16 outputs per run, many runs per CTA
+    (16, 4, 64, 16, 1, 700),       # one CTA: every run is one item (direct outputs)
+])
+def test_merge_paths_across_shapes(Hq, Hkv, D, P, ctas, n):
+    """The in-kernel merge across group sizes, head dims and CTA counts: main
+    and fork share a prefix, each adds its own tail; every (sequence, KV head)
+    run is merged by the CTA that completes it (or written directly when it is
+    one item) and must equal the oracle."""
+    p = Pair(1, Hq, Hkv, D, P, num_pages=3 * (n // P) + 40, decode_ctas=ctas, seed=n + ctas)
+    keep = []
+    m = p.seq_new()
+    keep.append(p.append(m, n))
+    a = p.fork(m)
+    keep.append(p.append(a, 37))
+    keep.append(p.append(m, 5))
+    b = p.fork(a)
+    keep.append(p.append(b, 1))
+    _decode_check(p, [m, a, b], 0, 1.0 / math.sqrt(D), n + 1)
+    p.close()
+
+
 def test_one_cta_merges_hundreds_of_runs():
     """decode_ctas = 1: the one CTA holds every item (40 sequences, 8 KV heads:
     320 arrivals, three rounds of 128) and completes, so merges, every
