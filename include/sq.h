@@ -152,7 +152,9 @@ SQ_API int sq_fork_aux(sq_cache *cache, sq_seq parent, sq_seq *child_out);
  *   seqs: host, n_seqs distinct live handles, each with >= 1 token
  *   q:    device, bf16 [n_seqs][num_q_heads][head_dim]
  *   out:  device, [n_seqs][num_q_heads][head_dim], bf16 (SQ_OUT_BF16, round
- *         to nearest even) or fp32 (SQ_OUT_F32)
+ *         to nearest even) or fp32 (SQ_OUT_F32); must not overlap q (rows are
+ *         written while other rows' queries are still being read): an
+ *         overlap is INVALID_ARG
  * Sequences that share pages (a main thread and its forks) in one call read
  * each shared page once for all of them (Sec. 3.4, shared-context kernels).
  * Errors: BAD_HANDLE, INVALID_ARG, NO_MEMORY, CUDA. */
@@ -188,6 +190,7 @@ SQ_API int sq_evict_spans(sq_cache *cache, sq_seq seq, const sq_span *spans,
  *   lse: NULL, or device float [n_q][Hq], 4-byte aligned: the natural log of
  *        sum_j exp(sm_scale * q . K[j]) over the visible keys (for a backward
  *        pass or for merging with other key ranges);
+ *   q, out and lse must not overlap one another (INVALID_ARG);
  *   sm_scale: finite, >= 0;
  *   spans: host, n_spans half-open spans of current positions, any order;
  *          empty, overlapping or out-of-range spans are INVALID_ARG;

@@ -552,6 +552,14 @@ int sq_append_kv_batch(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, const vo
     return SQ_OK;
 }
 
+// True when the byte ranges [a, a + na) and [b, b + nb) share a byte.  The
+// attention calls write outputs while other CTAs still read the queries, so
+// an output that overlaps the queries (or the log-sum-exps either) is refused.
+static bool overlaps(const void* a, size_t na, const void* b, size_t nb) {
+    const uintptr_t x = reinterpret_cast<uintptr_t>(a), y = reinterpret_cast<uintptr_t>(b);
+    return na > 0 && nb > 0 && x < y + nb && y < x + na;
+}
+
 int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t layer,
                         const void* q, void* out, int32_t out_dtype, float sm_scale,
                         void* stream) {
@@ -564,6 +572,11 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
     if ((reinterpret_cast<uintptr_t>(q) & 15) || (reinterpret_cast<uintptr_t>(out) & 15))
         return SQ_ERR_INVALID_ARG;
     if (!(sm_scale == sm_scale)) return SQ_ERR_INVALID_ARG;
+    {
+        const size_t rows = (size_t)n_seqs * g.Hq * g.D;
+        if (overlaps(q, rows * 2, out, rows * (out_dtype == SQ_OUT_F32 ? 4 : 2)))
+            return SQ_ERR_INVALID_ARG;
+    }
     for (int32_t i = 0; i < n_seqs; ++i) {
         const Seq* s = c->host->seq(seqs[i]);
         if (!s) return SQ_ERR_BAD_HANDLE;
@@ -767,6 +780,13 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
         (reinterpret_cast<uintptr_t>(lse) & 3))
         return SQ_ERR_INVALID_ARG;
     if (!(sm_scale >= 0.f) || sm_scale > 3.0e38f) return SQ_ERR_INVALID_ARG;
+    {
+        const size_t rows = (size_t)n_q * g.Hq;
+        const size_t qb = rows * g.D * 2, ob = rows * g.D * (out_dtype == SQ_OUT_F32 ? 4 : 2);
+        const size_t lb = lse ? rows * 4 : 0;
+        if (overlaps(q, qb, out, ob) || overlaps(q, qb, lse, lb) || overlaps(out, ob, lse, lb))
+            return SQ_ERR_INVALID_ARG;
+    }
     if (n_spans < 0 || (n_spans > 0 && !spans)) return SQ_ERR_INVALID_ARG;
     std::vector<int32_t> key(2 * (size_t)n_spans);
     for (int32_t i = 0; i < n_spans; ++i) {
@@ -1072,6 +1092,11 @@ int sq_decode_attention_noalloc(sq_cache* c, const sq_seq* seqs, int32_t n_seqs,
     if ((reinterpret_cast<uintptr_t>(q) & 15) || (reinterpret_cast<uintptr_t>(out) & 15))
         return SQ_ERR_INVALID_ARG;
     if (!(sm_scale == sm_scale)) return SQ_ERR_INVALID_ARG;
+    {
+        const size_t rows = (size_t)n_seqs * g.Hq * g.D;
+        if (overlaps(q, rows * 2, out, rows * (out_dtype == SQ_OUT_F32 ? 4 : 2)))
+            return SQ_ERR_INVALID_ARG;
+    }
     int dev = -1;
     if (cudaGetDevice(&dev) != cudaSuccess) return SQ_ERR_CUDA;
     if (dev != c->device) return SQ_ERR_INVALID_ARG;

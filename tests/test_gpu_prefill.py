@@ -189,6 +189,8 @@ def test_prefill_rejects_bad_arguments():
             dict(n_q=101), dict(n_q=0), dict(layer=1), dict(spans=[(5, 5)]),
             dict(spans=[(5, 9), (8, 12)]), dict(spans=[(90, 101)]), dict(sm_scale=-1.0),
             dict(sm_scale=float("nan")), dict(out_dtype=7),
+            dict(out=q.view(torch.float32)[:5]),             # out overlaps q
+            dict(lse=out.view(-1)[:160]),                     # lse overlaps out
         ]
         for kw in bad:
             args = dict(seq=h, layer=0, n_q=10, q=q, out=out, out_dtype=sq.SQ_OUT_F32,

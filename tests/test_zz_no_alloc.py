@@ -66,6 +66,34 @@ def test_noalloc_matches_regular_entry_point_two_calls_in_a_row():
     p.close()
 
 
+def test_decode_rejects_output_over_queries():
+    # the merged rows of a call are written while other CTAs still read their
+    # queries, so both entry points refuse an output that overlaps q
+    p = Pair(1, 16, 4, 64, 16, num_pages=40, seed=45)
+    keep = [None]
+    m = p.seq_new()
+    keep.append(p.append(m, 300))
+    buf = torch.zeros(4096, dtype=torch.float32, device="cuda")     # 16 KiB
+    q = buf.view(torch.bfloat16)[:1024].view(1, 16, 64)               # bytes [0, 2048)
+    arr = (ctypes.c_int32 * 1)(m)
+    bad = [
+        (buf[256:256 + 1024].view(1, 16, 64), sq.SQ_OUT_F32),        # fp32 out from byte 1024
+        (q, sq.SQ_OUT_BF16),                                           # in place
+    ]
+    for out, dt in bad:
+        rc = sq.lib().sq_decode_attention(p.cache.handle, arr, 1, 0, q.data_ptr(), out.data_ptr(),
+                                          dt, ctypes.c_float(0.1),
+                                          torch.cuda.current_stream().cuda_stream)
+        assert rc == sq.SQ_ERR_INVALID_ARG
+        assert _noalloc_c(p.cache, [m], 0, q, out, dt, 0.1) == sq.SQ_ERR_INVALID_ARG
+    # adjacent (the output starts at q's end): accepted
+    out = buf[512:512 + 1024].view(1, 16, 64)
+    assert _noalloc_c(p.cache, [m], 0, q, out, sq.SQ_OUT_F32, 0.1) == sq.SQ_OK
+    torch.cuda.synchronize()
+    assert p.cache.sync_status() == sq.SQ_OK
+    p.close()
+
+
 def test_noalloc_rejects_plans_beyond_the_scratch():
     # 8 KV heads x 2048 stages over 16384 persistent CTAs -> about 16,390
     # partial entries of G = 4 rows: ~34 MB of partials plus ~1.4 MB of plan,
