@@ -825,12 +825,13 @@ __global__ void __launch_bounds__(320, 1)
 
 // Merges the key-range splits of each query row: weights 2^(lse_s - max).
 // One warp per (CTA tile, query tile, row); the lanes take the splits' log-sum-
-// exps (up to 64 splits), then the partial outputs go through in batches of 8
-// whose loads are in flight together.
+// exps (up to 64 splits).  The partial outputs of the first 24 splits are
+// loaded together with them, so a row of up to 24 splits costs one round trip;
+// an empty split's partial (never written) is read but selected away.
 template <int D>
 __global__ void __launch_bounds__(256) sq_prefill_combine_kernel(const PrefillCombineArgs a) {
     constexpr int V = D / 32;  // output elements per lane
-    constexpr int U = 8;       // splits per batch of loads
+    constexpr int U = 24;      // splits per batch of loads
     // programmatic dependent of the prefill kernel: wait for its partials
     grid_dependency_wait();
     const int gw = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
@@ -849,6 +850,26 @@ __global__ void __launch_bounds__(256) sq_prefill_combine_kernel(const PrefillCo
     const float ml0 = lane < a.n_split ? a.part_ml[part0 + (size_t)lane * kRowsPerUnit] : -INFINITY;
     const float ml1 =
         lane + 32 < a.n_split ? a.part_ml[part0 + (size_t)(lane + 32) * kRowsPerUnit] : -INFINITY;
+    float vals[U][V];
+    auto load = [&](int s0) {
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int s = s0 + u;  // the same in every lane
+#pragma unroll
+            for (int e = 0; e < V; ++e) vals[u][e] = 0.f;
+            if (s < a.n_split) {
+                const float* po = a.part_o + (part0 + (size_t)s * kRowsPerUnit) * D + lane * V;
+                if constexpr (V == 4) {
+                    const float4 v = *reinterpret_cast<const float4*>(po);
+                    vals[u][0] = v.x; vals[u][1] = v.y; vals[u][2] = v.z; vals[u][3] = v.w;
+                } else {
+                    const float2 v = *reinterpret_cast<const float2*>(po);
+                    vals[u][0] = v.x; vals[u][1] = v.y;
+                }
+            }
+        }
+    };
+    load(0);
     float M = fmaxf(ml0, ml1);
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
@@ -864,30 +885,16 @@ __global__ void __launch_bounds__(256) sq_prefill_combine_kernel(const PrefillCo
 #pragma unroll
     for (int e = 0; e < V; ++e) acc[e] = 0.f;
     for (int s0 = 0; W > 0.f && s0 < a.n_split; s0 += U) {
-        float w[U];
-        float vals[U][V];
+        if (s0 > 0) load(s0);
 #pragma unroll
         for (int u = 0; u < U; ++u) {
-            const int s = s0 + u;  // the same in every lane
+            const int s = s0 + u;
             const float ws = __shfl_sync(0xffffffffu, s < 32 ? w0 : w1, s & 31);
-            w[u] = s < a.n_split ? ws : 0.f;
+            if (s < a.n_split && ws > 0.f) {
 #pragma unroll
-            for (int e = 0; e < V; ++e) vals[u][e] = 0.f;
-            if (w[u] > 0.f) {  // an empty split's partial is not read
-                const float* po = a.part_o + (part0 + (size_t)s * kRowsPerUnit) * D + lane * V;
-                if constexpr (V == 4) {
-                    const float4 v = *reinterpret_cast<const float4*>(po);
-                    vals[u][0] = v.x; vals[u][1] = v.y; vals[u][2] = v.z; vals[u][3] = v.w;
-                } else {
-                    const float2 v = *reinterpret_cast<const float2*>(po);
-                    vals[u][0] = v.x; vals[u][1] = v.y;
-                }
+                for (int e = 0; e < V; ++e) acc[e] += ws * vals[u][e];
             }
         }
-#pragma unroll
-        for (int u = 0; u < U; ++u)
-#pragma unroll
-            for (int e = 0; e < V; ++e) acc[e] += w[u] * vals[u][e];
     }
     const float inv = W > 0.f ? 1.f / W : 0.f;
     const size_t o = ((size_t)qi * a.Hq + h) * D + lane * V;
