@@ -126,6 +126,7 @@ def test_split_invariance_over_cta_counts():
     (6, 2, 128, 256, 200, 3000),   # G = 3: several runs per merge round (96 outputs each)
     (8, 8, 64, 16, 300, 2000),     # G = 1, d = 64: 16 outputs per run, many runs per CTA
     (16, 4, 64, 16, 1, 700),       # one CTA: every run is one item (direct outputs)
+    (16, 1, 128, 64, 304, 5000),   # one KV head, G = 16: a run fills a round's 512 outputs
 ])
 def test_merge_paths_across_shapes(Hq, Hkv, D, P, ctas, n):
     """The in-kernel merge across group sizes, head dims and CTA counts: main
