@@ -484,13 +484,15 @@ def run_sq(args, world, rank, local):
         torch.cuda.synchronize()
         st0 = cache.stats()
         # One eviction per request, enqueued back to back: the host planning
-        # of each call overlaps the GPU work of the one before (a GPU sleep
-        # covers the first), and the events between calls give each call's
-        # GPU time: copy-on-write copies and the compaction kernel.
+        # of each call overlaps the GPU work of the one before (reads of the
+        # input bank keep the GPU busy while the first is planned), and the
+        # events between calls give each call's GPU time: copy-on-write
+        # copies and the compaction kernel.
         span_list = [spec["spans"](seed, r, cache.seq_info(m)[0], P) for r, m in enumerate(mains)]
         evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(mains) + 1)]
         b = []
-        torch.cuda._sleep(2_000_000)
+        for _ in range(4):
+            sq.sq_probe_read(cache.handle, bank.data, bank.data.numel() * 2, st_h)
         evs[0].record(stream)
         for r, m in enumerate(mains):
             b.append(cache.stats()["evict_bytes"])
