@@ -284,12 +284,15 @@ void free_entry(PlanEntry& p) {
     p = PlanEntry();
 }
 
-// Rows per eviction tile: the largest (up to 64, at most a page) for which
-// one CTA per (layer, K/V, head) plane still fits in one wave of resident CTAs.
+// Rows per eviction tile: 8 KiB copies (32 rows at d = 128, 64 at d = 64;
+// measured faster than 16 KiB and far faster than 4 KiB ones), at most a
+// page, and fewer if one CTA per (layer, K/V, head) plane would not fit in
+// one wave of resident CTAs.
 int choose_tile_rows(const sq_cache* c) {
     const int64_t planes = (int64_t)c->g.L * 2 * c->g.Hkv;
+    const int target = std::max(8, 8192 / (2 * c->g.D));
     int best = 0;
-    for (int tr = std::min(c->g.P, kStageTokens); tr >= 8; tr >>= 1) {
+    for (int tr = std::min(c->g.P, target); tr >= 8; tr >>= 1) {
         best = tr;
         if (planes <= (int64_t)c->num_sms * evict_ctas_per_sm(tr, c->g.D)) break;
     }

@@ -135,7 +135,7 @@ struct EvictArgs {
 cudaError_t launch_append(const AppendArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_append_batch(const AppendBatchArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_cow_copy(const CowArgs& a, int num_sms, cudaStream_t st);
-constexpr int kEvictStages = 3;
+constexpr int kEvictStages = 6;
 // Shared memory of one eviction CTA for a tile size.
 int evict_smem_bytes(int tile_rows, int D);
 // Resident eviction CTAs per SM for a tile size.
