@@ -1354,9 +1354,11 @@ def run_reference(args, world, rank):
     L, Hq, Hkv, D = args.layers, 32, 8, 128
     R, n = args.requests, args.ctx
     scale = 1.0 / math.sqrt(D)
-    bank = bf16_bits(Bank(1 << 27, sub_seed(args.seed, 11)).data)
-    rng = np.random.default_rng(sub_seed(args.seed, 12))
     row = Hkv * D
+    # room for a sequence's rows at any of many offsets (at least two
+    # sequences' worth, so the draw below never has an empty range)
+    bank = bf16_bits(Bank(max(1 << 27, 2 * n * row), sub_seed(args.seed, 11)).data)
+    rng = np.random.default_rng(sub_seed(args.seed, 12))
 
     def rows():
         o = int(rng.integers(0, (bank.size - n * row) // 8)) * 8
