@@ -18,18 +18,20 @@
 // from HBM once for all of them.
 //
 // Merge: an item leaves one partial (max, sum, unnormalised output) per group
-// member, in that (sequence, KV head)'s contiguous run of entries.  After its
+// member, in that (sequence, KV head)'s contiguous run of entries; a member
+// whose run is this one item gets its normalised output directly.  After its
 // last item a CTA counts its arrivals on each (sequence, KV head) it touched;
 // the CTA that brings a count to the number of entries merges that run
 // (max of the maxima, weights 2^(m - M)) and writes the normalised output.
-// The arrival word holds the call's tag next to the count, and the last
-// arriver clears it, so a word left by another call never counts here.
+// Counts are zero in every uploaded plan and the completing arrival resets
+// its count, so every call starts from zero.
 //
 // Start-up: the kernel is a programmatic dependent of whatever precedes it.
 // When the plan was already on the device (a reused plan), the producer reads
-// it and prefetches the CTA's first stages into L2 before the dependency wait;
-// the K/V rows themselves reach shared memory only after the wait, through L2,
-// which holds whatever the preceding kernel wrote to them.
+// its item range and first stages into registers and prefetches those stages
+// into L2 before the dependency wait; the K/V rows themselves reach shared
+// memory only after the wait, through L2, which holds whatever the preceding
+// kernel wrote to them.
 //
 // Tensor cores: S = Q K^T and O += P V are m16n8k16 bf16 mma.sync with fp32
 // accumulation; rows = query rows (<= 16), columns = tokens / head dims.  The
