@@ -787,15 +787,21 @@ __global__ void __launch_bounds__(320, 1)
         mbar_init(sm.bar<D>(C::kBarDone), 1);
         fence_mbar_init();
         *abort_flag = 0;
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_addr(tmem_slot), C::kTmemCols);
+        tmem_relinquish();
+    }
+    // Launched as a programmatic dependent: the set-up above overlapped the
+    // preceding kernel's tail; the plan, the queries and the pool are read
+    // only from here on.
+    grid_dependency_wait();
+    if (threadIdx.x == 0) {
         // key tiles up to the CTA tile's last query position, split evenly
         const int lo = __ldg(&a.qt_tiles[qt]);
         const int t0 = (int)((int64_t)lo * split / a.n_split);
         sched[0] = t0;
         sched[1] = (int)((int64_t)lo * (split + 1) / a.n_split) - t0;
-    }
-    if (warp == 1) {
-        tmem_alloc(smem_addr(tmem_slot), C::kTmemCols);
-        tmem_relinquish();
     }
     tc_fence_before();
     __syncthreads();
@@ -832,8 +838,10 @@ template <int D>
 __global__ void __launch_bounds__(256) sq_prefill_combine_kernel(const PrefillCombineArgs a) {
     constexpr int V = D / 32;  // output elements per lane
     constexpr int U = 24;      // splits per batch of loads
-    // programmatic dependent of the prefill kernel: wait for its partials
+    // programmatic dependent of the prefill kernel: wait for its partials;
+    // the next layer's prefill may then be scheduled
     grid_dependency_wait();
+    grid_launch_dependents();
     const int gw = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
     const int lane = threadIdx.x & 31;
     const int units = a.n_qt * a.Hkv;
@@ -941,13 +949,24 @@ cudaError_t launch_prefill(const CUtensorMap& pool_map, const CUtensorMap& qmap,
                            const PrefillArgs& a, int D, cudaStream_t st) {
     const unsigned grid = (unsigned)(a.n_qt * a.Hkv * a.n_split);
     if (grid == 0) return cudaSuccess;
-    if (D == 128)
-        dev::sq_prefill_kernel<128><<<grid, dev::PreCfg<128>::kThreads,
-                                      dev::PreCfg<128>::kSmemBytes, st>>>(pool_map, qmap, a);
-    else
-        dev::sq_prefill_kernel<64><<<grid, dev::PreCfg<64>::kThreads, dev::PreCfg<64>::kSmemBytes,
-                                     st>>>(pool_map, qmap, a);
-    return cudaGetLastError();
+    // a programmatic dependent of whatever precedes it: its barrier and tensor
+    // memory set-up overlaps that work's tail (it waits before any read)
+    cudaLaunchAttribute at;
+    at.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at.val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.stream = st;
+    cfg.attrs = &at;
+    cfg.numAttrs = 1;
+    if (D == 128) {
+        cfg.blockDim = dim3(dev::PreCfg<128>::kThreads);
+        cfg.dynamicSmemBytes = dev::PreCfg<128>::kSmemBytes;
+        return cudaLaunchKernelEx(&cfg, dev::sq_prefill_kernel<128>, pool_map, qmap, a);
+    }
+    cfg.blockDim = dim3(dev::PreCfg<64>::kThreads);
+    cfg.dynamicSmemBytes = dev::PreCfg<64>::kSmemBytes;
+    return cudaLaunchKernelEx(&cfg, dev::sq_prefill_kernel<64>, pool_map, qmap, a);
 }
 
 cudaError_t launch_prefill_combine(const PrefillCombineArgs& a, int D, cudaStream_t st) {
