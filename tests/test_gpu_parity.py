@@ -166,6 +166,36 @@ def test_one_cta_merges_hundreds_of_runs():
     p.close()
 
 
+def test_cached_plan_reused_across_streams():
+    """The same sequences decoded on stream A, then B, then A again: each later
+    call reuses the cached plan (its arrival counts and partial buffers too)
+    after waiting for the other stream's use of it, and every result equals
+    the oracle."""
+    p = Pair(2, 32, 8, 128, 64, num_pages=200, decode_ctas=300, seed=56)
+    keep = []
+    m = p.seq_new()
+    keep.append(p.append(m, 2500))
+    a = p.fork(m)
+    keep.append(p.append(a, 24))
+    seqs = [m, a]
+    sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+    sa.wait_stream(torch.cuda.current_stream())
+    sb.wait_stream(torch.cuda.current_stream())
+    checks = []
+    for i, st in enumerate((sa, sb, sa, sb, sb, sa)):
+        q_cpu, q = _q(700 + i, 2, 32, 128)
+        keep.append(q)
+        st.wait_stream(torch.cuda.current_stream())   # q was copied on the default stream
+        with torch.cuda.stream(st):
+            out = p.decode(seqs, i % 2, 0.09, q, sq.SQ_OUT_F32, st)
+        checks.append((out, i % 2, q_cpu))
+    torch.cuda.synchronize()
+    assert p.cache.sync_status() == sq.SQ_OK
+    for out, layer, q_cpu in checks:
+        assert_close(out, p.oracle_decode(seqs, layer, 0.09, q_cpu), max_abs=5e-3)
+    p.close()
+
+
 def test_decode_replayed_from_a_cuda_graph():
     """Replays of a captured decode repeat its kernel arguments, the merge's
     arrival tag among them: every replay must still merge each run once
