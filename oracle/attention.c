@@ -142,6 +142,51 @@ int oracle_decode_batch_f64(int n_seqs, const int *ns, int Hq, int Hkv, int d,
 }
 
 /*
+ * Quantities for the error analysis of a decode whose softmax weights each
+ * carry a small relative perturbation (for instance weights rounded to a
+ * narrower type before the PV product).  Not part of the method: the tests
+ * build their error budgets from them.  For query head h, KV head
+ * g = floor(h / G) and every dimension e, with w_t the exact softmax weights
+ * and o[h] the exact output (both exactly as oracle_decode_f64 computes them):
+ *   dev[h][e]  = sum_t w_t * |V[t][g][e] - o[h][e]|
+ *   absv[h][e] = sum_t w_t * |V[t][g][e]|
+ * out receives o.  Same shapes and return codes as oracle_decode_f64.
+ */
+int oracle_decode_dev_f64(int n, int Hq, int Hkv, int d, const uint16_t *q,
+                          const uint16_t *k, const uint16_t *v, double scale,
+                          const uint8_t *mask, double *out, double *dev,
+                          double *absv) {
+    if (n <= 0 || Hq <= 0 || Hkv <= 0 || d <= 0 || Hq % Hkv != 0) return -1;
+    int G = Hq / Hkv;
+    int status = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(min : status)
+    for (int h = 0; h < Hq; ++h) {
+        double *w = (double *)malloc(sizeof(double) * (size_t)n);
+        if (!w) { status = -2; continue; }
+        const int g = h / G;
+        double *o = out + (size_t)h * d;
+        int rc = one_head(n, Hkv, d, g, q + (size_t)h * d, k, v, scale, mask, o, w,
+                          NULL);
+        if (rc == 0) {
+            double *dv = dev + (size_t)h * d, *av = absv + (size_t)h * d;
+            for (int e = 0; e < d; ++e) { dv[e] = 0.0; av[e] = 0.0; }
+            for (int t = 0; t < n; ++t) {
+                if (w[t] == 0.0) continue;
+                const uint16_t *vt = v + ((size_t)t * Hkv + g) * d;
+                for (int e = 0; e < d; ++e) {
+                    const double x = widen_bf16(vt[e]);
+                    dv[e] += w[t] * fabs(x - o[e]);
+                    av[e] += w[t] * fabs(x);
+                }
+            }
+        }
+        free(w);
+        if (rc < status) status = rc;
+    }
+    return status;
+}
+
+/*
  * Masked prefill attention (Algorithm 2, BuildMask; Sec. 3.3: the auxiliary
  * training traces see the context with the closed cursors' tokens masked
  * out).  The last n_q tokens of a sequence of n tokens are the queries; query

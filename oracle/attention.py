@@ -46,6 +46,11 @@ def lib():
                 u16p, u16p, u16p, ctypes.c_double,
                 ctypes.POINTER(ctypes.c_uint8), f64p, f64p, f64p]
             L.oracle_decode_f64.restype = ctypes.c_int
+            L.oracle_decode_dev_f64.argtypes = [
+                ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                u16p, u16p, u16p, ctypes.c_double,
+                ctypes.POINTER(ctypes.c_uint8), f64p, f64p, f64p]
+            L.oracle_decode_dev_f64.restype = ctypes.c_int
             L.oracle_decode_batch_f64.argtypes = [
                 ctypes.c_int, ctypes.POINTER(ctypes.c_int), ctypes.c_int,
                 ctypes.c_int, ctypes.c_int, u16p,
@@ -114,6 +119,36 @@ def decode(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float,
     if want_lse:
         res.append(lse)
     return res[0] if len(res) == 1 else tuple(res)
+
+
+def decode_dev(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float,
+               mask: Optional[np.ndarray] = None):
+    """Decode attention of one sequence plus two weighted spreads of V used
+    by error analyses (not part of the method): returns (out, dev, absv),
+    each float64 [Hq, d], with dev[h, e] = sum_t w_t |V[t, g, e] - out[h, e]|
+    and absv[h, e] = sum_t w_t |V[t, g, e]| for the exact softmax weights w.
+    Arguments as for decode()."""
+    q = np.ascontiguousarray(q, dtype=np.uint16)
+    k = np.ascontiguousarray(k, dtype=np.uint16)
+    v = np.ascontiguousarray(v, dtype=np.uint16)
+    Hq, d = q.shape
+    n, Hkv, d2 = k.shape
+    assert d2 == d and v.shape == k.shape
+    out = np.zeros((Hq, d), dtype=np.float64)
+    dev = np.zeros((Hq, d), dtype=np.float64)
+    absv = np.zeros((Hq, d), dtype=np.float64)
+    m = None
+    if mask is not None:
+        m = np.ascontiguousarray(mask, dtype=np.uint8)
+        assert m.shape == (n,)
+    f64p = ctypes.POINTER(ctypes.c_double)
+    rc = lib().oracle_decode_dev_f64(
+        n, Hq, Hkv, d, _u16(q), _u16(k), _u16(v), float(scale),
+        m.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)) if m is not None else None,
+        out.ctypes.data_as(f64p), dev.ctypes.data_as(f64p), absv.ctypes.data_as(f64p))
+    if rc != 0:
+        raise ValueError(f"oracle_decode_dev_f64 rejected the input (rc={rc})")
+    return out, dev, absv
 
 
 def decode_batch(q: np.ndarray, ks: Sequence[np.ndarray], vs: Sequence[np.ndarray],

@@ -113,15 +113,19 @@ class BankPair:
             assert self.cache.seq_info(h)[0] == self.oracle.n_tokens(self.o[h])
         assert self.cache.free_pages() == self.oracle.free_count()
 
-    def check_plane(self, h, layer, kv, head):
-        """One (layer, K/V, head) plane of a sequence, read through the page
-        table from the device pool, equals the oracle's rows bit for bit."""
+    def check_planes(self, h, layer, planes=None):
+        """The listed (K/V, head) planes of one layer of a sequence (all
+        2 x Hkv of them by default), read through the page table from the
+        device pool, equal the oracle's rows bit for bit."""
+        if planes is None:
+            planes = [(kv, head) for kv in (0, 1) for head in range(self.Hkv)]
         torch.cuda.synchronize()
         pool = self.cache.pool_view()
         pt = torch.tensor(self.cache.page_table(h), dtype=torch.long, device="cuda")
         n = self.cache.seq_info(h)[0]
         j = torch.arange(n, device="cuda")
-        got = bf16_bits(pool[layer, pt[j // self.P], kv, head, j % self.P, :].cpu())
         K, V = self.rows(h, layer)
-        exp = (K if kv == 0 else V)[:, head, :]
-        assert np.array_equal(got, exp), (layer, kv, head)
+        for kv, head in planes:
+            got = bf16_bits(pool[layer, pt[j // self.P], kv, head, j % self.P, :].cpu())
+            exp = (K if kv == 0 else V)[:, head, :]
+            assert np.array_equal(got, exp), (layer, kv, head)

@@ -13,6 +13,7 @@ import paper_2602_22603_gb300 as sq
 from oracle import attention as oatt
 from oracle import cache_model as ocm
 from synthetic import bf16_bits, bf16_normal
+from tests.budget import decode_budget
 
 # Attention tolerance against the double-precision oracle (max / mean abs).
 MAX_ABS = 1e-2
@@ -147,6 +148,19 @@ class Pair:
         self.cache.decode_attention(list(seqs), layer, q, out, out_dtype, sm_scale, stream)
         return out
 
+    def oracle_decode_budget(self, seqs: Sequence[int], layer: int, sm_scale: float,
+                             q_cpu) -> Tuple[np.ndarray, np.ndarray]:
+        """The oracle's outputs [S, Hq, D] and the kernel's per-element error
+        budget for them (tests/budget.py)."""
+        qb = bf16_bits(q_cpu)
+        res, bud = [], []
+        for i, h in enumerate(seqs):
+            k, v = self.store.rows(self.oracle.tokens(self.o[h]), layer)
+            o, dev, absv = oatt.decode_dev(qb[i], k, v, sm_scale)
+            res.append(o)
+            bud.append(decode_budget(dev, absv, k.shape[0]))
+        return np.stack(res), np.stack(bud)
+
     def oracle_decode(self, seqs: Sequence[int], layer: int, sm_scale: float, q_cpu) -> np.ndarray:
         qb = bf16_bits(q_cpu)
         res = []
@@ -163,3 +177,13 @@ def assert_close(got: torch.Tensor, exp: np.ndarray, max_abs=MAX_ABS, mean_abs=M
     assert err.max() <= max_abs, f"max abs error {err.max():.3g}"
     assert err.mean() <= mean_abs, f"mean abs error {err.mean():.3g}"
     return float(err.max()), float(err.mean())
+
+
+def assert_budget(got: torch.Tensor, exp: np.ndarray, budget: np.ndarray):
+    """The contract's tolerance (max-abs 1e-2, mean-abs 1e-3) and, element by
+    element, the error budget the kernel's arithmetic allows (tests/budget.py)."""
+    e = assert_close(got, exp)
+    g = got.detach().float().cpu().numpy().astype(np.float64)
+    over = np.abs(g - exp) - budget
+    assert over.max() <= 0.0, f"error above its budget by {over.max():.3g}"
+    return e

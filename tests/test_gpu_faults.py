@@ -13,7 +13,7 @@ import torch
 
 import paper_2602_22603_gb300 as sq
 from synthetic import bf16_normal
-from tests.gpu_harness import Pair, assert_close
+from tests.gpu_harness import Pair, assert_budget, assert_close
 
 pytestmark = pytest.mark.gpu
 
@@ -48,7 +48,7 @@ def test_unsignalled_stage_times_out_and_context_survives():
     out2 = p.decode([m, a], 0, 0.125, q, sq.SQ_OUT_F32)
     torch.cuda.synchronize()
     assert p.cache.sync_status() == sq.SQ_OK
-    assert_close(out2, p.oracle_decode([m, a], 0, 0.125, q_cpu))
+    assert_budget(out2, *p.oracle_decode_budget([m, a], 0, 0.125, q_cpu))
     # and so do appends and evictions
     keep.append(p.append(m, 5))
     p.evict(m, [(100, 400)])

@@ -12,7 +12,7 @@ import torch
 
 import paper_2602_22603_gb300 as sq
 from synthetic import TINY, bf16_normal, random_spans, shuffled
-from tests.gpu_harness import MAX_ABS, MEAN_ABS, Pair, assert_close
+from tests.gpu_harness import MAX_ABS, MEAN_ABS, Pair, assert_budget, assert_close
 
 pytestmark = pytest.mark.gpu
 
@@ -32,12 +32,12 @@ def _q(seed, S, Hq, D):
 
 def _decode_check(p: Pair, seqs, layer, scale, seed):
     q_cpu, q = _q(seed, len(seqs), p.Hq, p.D)
-    exp = p.oracle_decode(seqs, layer, scale, q_cpu)
+    exp, budget = p.oracle_decode_budget(seqs, layer, scale, q_cpu)
     out32 = p.decode(seqs, layer, scale, q, sq.SQ_OUT_F32)
     out16 = p.decode(seqs, layer, scale, q, sq.SQ_OUT_BF16)
     torch.cuda.synchronize()
     assert p.cache.sync_status() == sq.SQ_OK
-    e32 = assert_close(out32, exp, max_abs=5e-3)
+    e32 = assert_budget(out32, exp, budget)
     e16 = assert_close(out16, exp)
     # the bf16 output is the fp32 output rounded to nearest even
     assert torch.equal(out16, out32.to(torch.bfloat16))
@@ -102,6 +102,7 @@ def test_split_invariance_over_cta_counts():
     """The same decode with 1 .. many persistent CTAs (so 1 .. many partials
     per sequence and head) agrees with the oracle and with itself."""
     outs = []
+    budget = None
     for ctas in (1, 2, 7, 64, 304, 1000):
         p = Pair(1, 32, 8, 128, 64, num_pages=600, decode_ctas=ctas, seed=3)
         keep = []
@@ -113,12 +114,14 @@ def test_split_invariance_over_cta_counts():
         q_cpu, q = _q(77, 2, 32, 128)
         out = p.decode([m, a], 0, 0.0884, q, sq.SQ_OUT_F32)
         torch.cuda.synchronize()
-        exp = p.oracle_decode([m, a], 0, 0.0884, q_cpu)
-        assert_close(out, exp, max_abs=5e-3)
+        exp, budget = p.oracle_decode_budget([m, a], 0, 0.0884, q_cpu)
+        assert_budget(out, exp, budget)
         outs.append(out.cpu())
         p.close()
+    # every split is within the budget of the exact result, so two splits
+    # are within twice the budget of each other
     for o in outs[1:]:
-        assert (o - outs[0]).abs().max().item() < 5e-4
+        assert np.all((o - outs[0]).abs().double().numpy() <= 2 * budget)
 
 
 @pytest.mark.parametrize("Hq,Hkv,D,P,ctas,n", [
@@ -192,7 +195,7 @@ def test_cached_plan_reused_across_streams():
     torch.cuda.synchronize()
     assert p.cache.sync_status() == sq.SQ_OK
     for out, layer, q_cpu in checks:
-        assert_close(out, p.oracle_decode(seqs, layer, 0.09, q_cpu), max_abs=5e-3)
+        assert_budget(out, *p.oracle_decode_budget(seqs, layer, 0.09, q_cpu))
     p.close()
 
 
@@ -228,7 +231,7 @@ def test_decode_replayed_from_a_cuda_graph():
         torch.cuda.synchronize()
         assert p.cache.sync_status() == sq.SQ_OK
         for layer in range(2):
-            assert_close(outs[layer], p.oracle_decode(seqs, layer, 0.09, q_cpu), max_abs=5e-3)
+            assert_budget(outs[layer], *p.oracle_decode_budget(seqs, layer, 0.09, q_cpu))
     del g
     p.close()
 
@@ -386,17 +389,17 @@ def test_two_streams_main_and_aux():
             q_cpu, q = _q(500 + step, 1, 32, 128)
             keep.append(q)
             out = p.decode([m], step % 2, 1.0, q, sq.SQ_OUT_F32, sa)
-            checks.append((out, p.oracle_decode([m], step % 2, 1.0, q_cpu)))
+            checks.append((out, p.oracle_decode_budget([m], step % 2, 1.0, q_cpu)))
         if step % 2 == 0:
             with torch.cuda.stream(sb):
                 keep.append(p.append(a, 1, sb))
                 q_cpu, q = _q(900 + step, 1, 32, 128)
                 keep.append(q)
                 out = p.decode([a], step % 2, 1.0, q, sq.SQ_OUT_F32, sb)
-                checks.append((out, p.oracle_decode([a], step % 2, 1.0, q_cpu)))
+                checks.append((out, p.oracle_decode_budget([a], step % 2, 1.0, q_cpu)))
     torch.cuda.synchronize()
-    for out, exp in checks:
-        assert_close(out, exp, max_abs=5e-3)
+    for out, (exp, budget) in checks:
+        assert_budget(out, exp, budget)
     p.release(a, sb)
     with torch.cuda.stream(sa):
         spans = random_spans(seed=4, n_spans=12, total=int(0.4 * 4096), lo=64, hi=4096, median=150)
