@@ -275,11 +275,14 @@ SQ_API int sq_stats(sq_cache *cache, sq_stats_t *out);
  * be reached from C.  This call allocates no device memory — no cudaMalloc,
  * no cudaFree, no library allocator.  The call's split-K plan and partial
  * results go to a fixed scratch array of SQ_NOALLOC_SCRATCH_BYTES that is
- * part of the library's device image: every GPU that loads the library holds
- * it until the process exits.
- *   - The first call on a device looks up the scratch's device address
- *     (cudaGetSymbolAddress, with the cache's device current); make that first
- *     call before any stream capture.
+ * part of the library's device image.
+ *   - sq_cache_create makes that array resident on the cache's device (its
+ *     device address is looked up there, which loads it; it then stays until
+ *     the process exits) and allocates two pinned host buffers of 2 MiB for
+ *     this call's plan uploads.  The call itself loads and allocates nothing
+ *     on the device.  If that set-up failed, the call returns its error.
+ *   - The plan is copied asynchronously from one of those pinned buffers; a
+ *     plan larger than 2 MiB is copied from pageable host memory instead.
  *   - The current device must be the cache's device (else INVALID_ARG).
  *   - A call whose plan and partials need more than SQ_NOALLOC_SCRATCH_BYTES
  *     (very many sequences, or a very large decode_ctas) returns
@@ -289,6 +292,8 @@ SQ_API int sq_stats(sq_cache *cache, sq_stats_t *out);
  *     (every value read is written first by the same call).  Calls whose GPU
  *     work overlaps — on different streams without ordering between them —
  *     race on the scratch: order them (one stream, or events).
+ *   - After a reset of the device (cudaDeviceReset) every cache of it is
+ *     gone with its context: destroy them and create new ones.
  * Errors: BAD_HANDLE, INVALID_ARG, CAPACITY, CUDA. */
 SQ_API int sq_decode_attention_noalloc(sq_cache *cache, const sq_seq *seqs, int32_t n_seqs,
                                        int32_t layer, const void *q, void *out,

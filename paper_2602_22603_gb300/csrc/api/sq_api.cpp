@@ -85,6 +85,11 @@ struct UploadSlot {
 // memory it is a plain asynchronous DMA.  A buffer is refilled only after the
 // copy that last used it has run.
 constexpr int kPinnedSlots = 8;
+// Pinned staging of sq_decode_attention_noalloc's plans, allocated with the
+// cache: two slots of 2 MiB (a decode plan of 16 sequences of 2^17 tokens is
+// ~0.2 MiB); a larger plan is copied from pageable memory instead.
+constexpr int kNoallocPinnedSlots = 2;
+constexpr size_t kNoallocPinnedBytes = 2u << 20;
 struct PinnedSlot {
     uint8_t* h = nullptr;
     size_t cap = 0;
@@ -121,6 +126,14 @@ struct sq_cache {
     PinnedSlot pinned[kPinnedSlots];
     int next_pinned = 0;
     std::vector<uint8_t> staging;
+    // sq_decode_attention_noalloc: the device address of the library's fixed
+    // scratch on this cache's device (resolved at creation; null if that
+    // failed, with the status kept), and pinned staging for its plan uploads,
+    // allocated at creation too
+    uint8_t* noalloc_base = nullptr;
+    int noalloc_status = SQ_OK;
+    PinnedSlot noalloc_pinned[kNoallocPinnedSlots];
+    int next_noalloc_pinned = 0;
     // pages freed by work on a stream become reusable elsewhere only after
     // that work: the stream that freed each free page, and one event per
     // stream recorded after its latest freeing operation
@@ -370,6 +383,10 @@ int sq_cache_create(const sq_config* cfg, sq_cache** out) {
     auto fail = [&](int code) {
         if (c->own_pool) cudaFree(c->pool);
         if (c->d_err) cudaFree(c->d_err);
+        for (auto& p : c->noalloc_pinned) {
+            if (p.h) cudaFreeHost(p.h);
+            if (p.ev) cudaEventDestroy(p.ev);
+        }
         return code;
     };
     // [0] device error word, [1] sink of the read probe
@@ -382,6 +399,28 @@ int sq_cache_create(const sq_config* cfg, sq_cache** out) {
     for (auto& s : c->slots) {
         e = cudaEventCreateWithFlags(&s.ev, cudaEventDisableTiming);
         if (e != cudaSuccess) return fail(cuda_status(e));
+    }
+    // The no-alloc decode's scratch: looking its address up loads its module
+    // on this device now, so that the decode call itself loads and allocates
+    // nothing.  A failure here only disables that call.
+    {
+        void* base = nullptr;
+        c->noalloc_status = noalloc_scratch(&base);
+        c->noalloc_base = static_cast<uint8_t*>(base);
+        if (c->noalloc_status != SQ_OK) cudaGetLastError();
+        for (auto& p : c->noalloc_pinned) {
+            if (c->noalloc_status != SQ_OK) break;
+            e = cudaEventCreateWithFlags(&p.ev, cudaEventDisableTiming);
+            if (e == cudaSuccess)
+                e = cudaHostAlloc(reinterpret_cast<void**>(&p.h), kNoallocPinnedBytes,
+                                  cudaHostAllocDefault);
+            if (e != cudaSuccess) {
+                cudaGetLastError();
+                c->noalloc_status = cuda_status(e);
+                break;
+            }
+            p.cap = kNoallocPinnedBytes;
+        }
     }
     e = cudaDeviceSynchronize();
     if (e != cudaSuccess) return fail(cuda_status(e));
@@ -402,6 +441,10 @@ int sq_cache_destroy(sq_cache* c) {
         if (s.ev) cudaEventDestroy(s.ev);
     }
     for (auto& p : c->pinned) {
+        if (p.h) cudaFreeHost(p.h);
+        if (p.ev) cudaEventDestroy(p.ev);
+    }
+    for (auto& p : c->noalloc_pinned) {
         if (p.h) cudaFreeHost(p.h);
         if (p.ev) cudaEventDestroy(p.ev);
     }
@@ -1103,6 +1146,7 @@ int sq_decode_attention_noalloc(sq_cache* c, const sq_seq* seqs, int32_t n_seqs,
     int dev = -1;
     if (cudaGetDevice(&dev) != cudaSuccess) return SQ_ERR_CUDA;
     if (dev != c->device) return SQ_ERR_INVALID_ARG;
+    if (c->noalloc_status != SQ_OK) return c->noalloc_status;
     DecodePlanHost plan;
     int rc = plan_decode(*c->host, seqs, n_seqs, c->decode_ctas, &plan);
     if (rc != SQ_OK) return rc;
@@ -1111,16 +1155,33 @@ int sq_decode_attention_noalloc(sq_cache* c, const sq_seq* seqs, int32_t n_seqs,
     const size_t part_off = ((size_t)L.total + 255) & ~size_t(255);
     const size_t need = part_off + (size_t)decode_partial_bytes(L.n_comb_ent, g.G(), g.D);
     if (need > (size_t)SQ_NOALLOC_SCRATCH_BYTES) return SQ_ERR_CAPACITY;
-    void* base = nullptr;
-    rc = noalloc_scratch(dev, &base);
-    if (rc != SQ_OK) return rc;
-    uint8_t* scratch = static_cast<uint8_t*>(base);
+    uint8_t* scratch = c->noalloc_base;
 
-    if (c->staging.size() < (size_t)L.total) c->staging.resize(L.total);
-    plan_serialize(plan, L, c->staging.data());
+    // The plan goes up from one of the cache's two pinned slots (an
+    // asynchronous copy; the slot is refilled only after its previous copy
+    // ran), or, if it is larger than a slot, from pageable memory.
     cudaStream_t st = as_stream(stream);
-    cudaError_t e = cudaMemcpyAsync(scratch, c->staging.data(), L.total, cudaMemcpyHostToDevice, st);
-    if (e != cudaSuccess) return cuda_status(e);
+    cudaError_t e;
+    if ((size_t)L.total <= kNoallocPinnedBytes) {
+        PinnedSlot& ps = c->noalloc_pinned[c->next_noalloc_pinned];
+        c->next_noalloc_pinned = (c->next_noalloc_pinned + 1) % kNoallocPinnedSlots;
+        if (ps.ev_recorded) {
+            e = cudaEventSynchronize(ps.ev);
+            if (e != cudaSuccess) return cuda_status(e);
+        }
+        plan_serialize(plan, L, ps.h);
+        e = cudaMemcpyAsync(scratch, ps.h, L.total, cudaMemcpyHostToDevice, st);
+        if (e != cudaSuccess) return cuda_status(e);
+        e = cudaEventRecord(ps.ev, st);
+        if (e != cudaSuccess) return cuda_status(e);
+        ps.ev_recorded = true;
+    } else {
+        // (a copy from pageable memory has taken its source when it returns)
+        std::vector<uint8_t> host(L.total);
+        plan_serialize(plan, L, host.data());
+        e = cudaMemcpyAsync(scratch, host.data(), L.total, cudaMemcpyHostToDevice, st);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
     float* part_o = reinterpret_cast<float*>(scratch + part_off);
     float* part_ml = part_o + (size_t)L.n_comb_ent * g.G() * g.D;
 

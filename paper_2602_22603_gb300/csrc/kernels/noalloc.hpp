@@ -3,9 +3,9 @@
 
 namespace sq {
 
-// Looks up (once per device; the device must be current) the device address
-// of the library's static scratch array.  Returns SQ_OK or SQ_ERR_CUDA /
-// SQ_ERR_UNSUPPORTED.  Allocates nothing.
-int noalloc_scratch(int device, void** ptr);
+// Looks up the device address of the library's static scratch array on the
+// current device (loading its module there if it is not loaded yet).
+// Returns SQ_OK or SQ_ERR_CUDA.
+int noalloc_scratch(void** ptr);
 
 }  // namespace sq

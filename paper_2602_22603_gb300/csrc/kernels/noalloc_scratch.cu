@@ -8,14 +8,15 @@
 // split-K plan and partial results of one decode call live in this
 // file-scope array instead of in buffers the library would allocate.
 //
-// The array is part of the library's device image: every GPU that loads the
-// library holds its SQ_NOALLOC_SCRATCH_BYTES until the process exits.  Host
-// code cannot use the symbol itself (on the host it names a stand-in, not a
-// device address), so its device address is looked up once per device with
-// cudaGetSymbolAddress, with that device current, and handed to the kernels.
+// The array belongs to this file's device module.  With lazy module loading
+// (the CUDA default) the module, and with it the array's
+// SQ_NOALLOC_SCRATCH_BYTES, is loaded on a device the first time anything in
+// it is used there, and then stays until the process exits.  Host code
+// cannot use the symbol itself (on the host it names a stand-in, not a
+// device address), so sq_cache_create looks its device address up with
+// cudaGetSymbolAddress, with the cache's device current, which is the
+// first use: the decode call itself then loads and allocates nothing.
 #include <cuda_runtime.h>
-
-#include <mutex>
 
 #include "noalloc.hpp"
 #include "sq.h"
@@ -25,22 +26,14 @@ namespace {
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[SQ_NOALLOC_SCRATCH_BYTES];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_mu;
-void* g_addr[kMaxDevices] = {};
-
 }  // namespace
 
-int noalloc_scratch(int device, void** ptr) {
-    if (device < 0 || device >= kMaxDevices) return SQ_ERR_UNSUPPORTED;
-    std::lock_guard<std::mutex> lock(g_mu);
-    if (!g_addr[device]) {
-        void* p = nullptr;
-        const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-        if (e != cudaSuccess || !p) return SQ_ERR_CUDA;
-        g_addr[device] = p;
-    }
-    *ptr = g_addr[device];
+int noalloc_scratch(void** ptr) {
+    *ptr = nullptr;
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess || !p) return SQ_ERR_CUDA;
+    *ptr = p;
     return SQ_OK;
 }
 
