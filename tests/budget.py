@@ -13,14 +13,15 @@ dbar = sum_t w_t d_t, so
 
 for every output element.  Rescaling by 2^(m_old - m_new) and the split-K
 merge multiply numerator and denominator by the same factors, so (1) holds
-for any split of the tokens.  u = 2^-9 is the unit roundoff of bf16 (8
-significant bits); it is raised by 2^-12 for the fp32 logits (a 128-term
-fp32 dot product and the scale perturb a weight by far less than 2^-12
-relatively) and the hardware exponential.  The remaining fp32 error is the
-accumulation of O and of the normaliser: at most one fp32 rounding (counted
-as 2^-22, two units, to cover truncating tensor-core accumulation) per
-64-token stage an item holds, plus a few for the merge, each relative to
-sum_t w_t |v_t|.
+for any split of the tokens.  u = 2^-8 is the unit roundoff of bf16: it
+keeps 8 significant bits, and rounding to nearest errs by at most half a
+unit in the last place, 2^-8 of the leading bit.  u is raised by 2^-12 for
+the fp32 logits (a 128-term fp32 dot product and the scale perturb a weight
+by far less than 2^-12 relatively) and the hardware exponential.  The
+remaining fp32 error is the accumulation of O and of the normaliser: at most
+one fp32 rounding (counted as 2^-22, two units, to cover truncating
+tensor-core accumulation) per 64-token stage an item holds, plus a few for
+the merge, each relative to sum_t w_t |v_t|.
 
 The oracle supplies sum_t w_t |v_t - o| (dev) and sum_t w_t |v_t| (absv).
 """
@@ -30,7 +31,7 @@ import math
 
 import numpy as np
 
-U_BF16 = 2.0 ** -9
+U_BF16 = 2.0 ** -8
 U_WEIGHT = U_BF16 + 2.0 ** -12   # bf16 rounding + fp32 logit / exp2 error
 U_ACC = 2.0 ** -22               # per fp32 accumulation step (2 ulps)
 STAGE_TOKENS = 64
