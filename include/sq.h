@@ -168,12 +168,30 @@ SQ_API int sq_decode_attention(sq_cache *cache, const sq_seq *seqs, int32_t n_se
  *   spans: host, n_spans half-open spans of current positions, any order;
  *          empty, overlapping or out-of-range spans are INVALID_ARG;
  *          n_spans == 0 is a no-op.
- * Pages whose contents change and that are shared with another sequence are
- * replaced by fresh pages (copy-on-write, increasing logical page order);
- * others are compacted in place; pages past the new end are released.
+ * The kept rows are packed into full pages (every page full but the last;
+ * a sequence that had partial pages from sq_evict_spans_ragged is packed
+ * too).  Pages whose contents change and that are shared with another
+ * sequence are replaced by fresh pages (copy-on-write, increasing logical
+ * page order); others are compacted in place; pages past the new end are
+ * released.
  * Errors: BAD_HANDLE, INVALID_ARG, NO_PAGES, NO_MEMORY, CUDA. */
 SQ_API int sq_evict_spans(sq_cache *cache, sq_seq seq, const sq_span *spans,
                    int32_t n_spans, void *stream);
+
+/* The same eviction (Algorithm 1 phase 1, C.clear_kv; same arguments, same
+ * logical result) with work proportional to the spans instead of the
+ * sequence: pages the spans do not touch keep their rows; each maximal run
+ * of touched pages (a window) has its kept rows packed from slot 0 of its
+ * first page, and its pages that are no longer needed leave the sequence by
+ * remapping alone, without a copy.  About P rows per span are copied.  The
+ * last page of each window may stay partial: every page then carries its own
+ * fill (sq_get_page_fill), which decode and prefill attention honour, and
+ * appends still go to the sequence's last page.  When a window's last page
+ * is written, its slots past the fill are set to zero.  Copy-on-write, page
+ * release and error behaviour as for sq_evict_spans.
+ * Errors: BAD_HANDLE, INVALID_ARG, NO_PAGES, NO_MEMORY, CUDA. */
+SQ_API int sq_evict_spans_ragged(sq_cache *cache, sq_seq seq, const sq_span *spans,
+                                 int32_t n_spans, void *stream);
 
 /* Masked prefill attention (Algorithm 2, BuildMask; Sec. 3.3): the
  * training-time counterpart of span eviction.  The last n_q tokens of `seq`
@@ -196,10 +214,14 @@ SQ_API int sq_evict_spans(sq_cache *cache, sq_seq seq, const sq_span *spans,
  *          empty, overlapping or out-of-range spans are INVALID_ARG;
  *          n_spans == 0 is plain causal attention.
  * A query that sees no token (every key up to it masked) gets a zero output
- * and lse = -infinity.  The sequence and the cache are not modified.  The
+ * and lse = -infinity.  On a sequence with partial pages (sq_evict_spans_ragged)
+ * the n_q queries must lie in consecutive page slots, that is no partial page
+ * may hold one of them but the last (true for rows appended after the last
+ * ragged eviction); otherwise UNSUPPORTED.  The sequence and the cache are
+ * not modified.  The
  * kernel runs on the tensor cores (bf16 products, fp32 accumulation; the
  * softmax weights are rounded to bf16 before the value product).
- * Errors: BAD_HANDLE, INVALID_ARG, NO_MEMORY, CUDA. */
+ * Errors: BAD_HANDLE, INVALID_ARG, UNSUPPORTED, NO_MEMORY, CUDA. */
 SQ_API int sq_prefill_attention(sq_cache *cache, sq_seq seq, int32_t layer, int32_t n_q,
                                 const void *q, void *out, int32_t out_dtype, float *lse,
                                 float sm_scale, const sq_span *spans, int32_t n_spans,
@@ -232,6 +254,14 @@ SQ_API int sq_seq_next_pos(sq_cache *cache, sq_seq seq, int64_t *out);
  * Errors: BAD_HANDLE, INVALID_ARG (cap too small). */
 SQ_API int sq_get_page_table(sq_cache *cache, sq_seq seq, int32_t *host_out,
                       int32_t cap, int32_t *n_out);
+
+/* Copy the fill of every page of `seq` (rows it holds, 1 .. page_size, in
+ * its first slots; the sequence's rows are the pages' filled slots in page
+ * order) into host_out[0 .. cap); *n_out = the page count.  Every page is
+ * full but the last unless sq_evict_spans_ragged left partial pages.
+ * Errors: BAD_HANDLE, INVALID_ARG (cap too small). */
+SQ_API int sq_get_page_fill(sq_cache *cache, sq_seq seq, int32_t *host_out,
+                            int32_t cap, int32_t *n_out);
 
 /* Reference count of a page (0 = free). */
 SQ_API int sq_page_refcount(sq_cache *cache, int32_t page, int32_t *out);

@@ -86,12 +86,14 @@ _SIGS = {
     "sq_append_kv_batch": (ctypes.c_int, [_P, _I32P, _I32, _P, _P, _P]),
     "sq_decode_attention": (ctypes.c_int, [_P, _I32P, _I32, _I32, _P, _P, _I32, ctypes.c_float, _P]),
     "sq_evict_spans": (ctypes.c_int, [_P, _I32, ctypes.POINTER(sq_span), _I32, _P]),
+    "sq_evict_spans_ragged": (ctypes.c_int, [_P, _I32, ctypes.POINTER(sq_span), _I32, _P]),
     "sq_prefill_attention": (ctypes.c_int, [_P, _I32, _I32, _I32, _P, _P, _I32, _P, ctypes.c_float,
                                             ctypes.POINTER(sq_span), _I32, _P]),
     "sq_release": (ctypes.c_int, [_P, _I32, _P]),
     "sq_seq_info": (ctypes.c_int, [_P, _I32, _I32P, _I32P]),
     "sq_seq_next_pos": (ctypes.c_int, [_P, _I32, ctypes.POINTER(ctypes.c_int64)]),
     "sq_get_page_table": (ctypes.c_int, [_P, _I32, _I32P, _I32, _I32P]),
+    "sq_get_page_fill": (ctypes.c_int, [_P, _I32, _I32P, _I32, _I32P]),
     "sq_page_refcount": (ctypes.c_int, [_P, _I32, _I32P]),
     "sq_free_pages": (ctypes.c_int, [_P, _I32P]),
     "sq_pool_ptr": (ctypes.c_int, [_P, ctypes.POINTER(_P)]),
@@ -221,6 +223,13 @@ def sq_evict_spans(cache: int, seq: int, spans: Sequence[Tuple[int, int]], strea
     _check(lib().sq_evict_spans(cache, seq, arr, len(spans), _stream(stream)), "sq_evict_spans")
 
 
+def sq_evict_spans_ragged(cache: int, seq: int, spans: Sequence[Tuple[int, int]],
+                          stream=None) -> None:
+    arr = (sq_span * max(1, len(spans)))(*[sq_span(int(a), int(b)) for a, b in spans])
+    _check(lib().sq_evict_spans_ragged(cache, seq, arr, len(spans), _stream(stream)),
+           "sq_evict_spans_ragged")
+
+
 def sq_prefill_attention(cache: int, seq: int, layer: int, n_q: int, q, out,
                          out_dtype: int = SQ_OUT_BF16, lse=None, sm_scale: float = 1.0,
                          spans: Sequence[Tuple[int, int]] = (), stream=None) -> None:
@@ -254,6 +263,14 @@ def sq_get_page_table(cache: int, seq: int) -> List[int]:
     buf = (ctypes.c_int32 * max(1, npages))()
     n = _I32()
     _check(lib().sq_get_page_table(cache, seq, buf, npages, ctypes.byref(n)), "sq_get_page_table")
+    return list(buf[: n.value])
+
+
+def sq_get_page_fill(cache: int, seq: int) -> List[int]:
+    _, npages = sq_seq_info(cache, seq)
+    buf = (ctypes.c_int32 * max(1, npages))()
+    n = _I32()
+    _check(lib().sq_get_page_fill(cache, seq, buf, npages, ctypes.byref(n)), "sq_get_page_fill")
     return list(buf[: n.value])
 
 
@@ -341,6 +358,8 @@ class Cache:
                         stream=None: sq_decode_attention(self.handle, seqs, layer, q, out,
                                                          out_dtype, sm_scale, stream))
     evict_spans = lambda self, seq, spans, stream=None: sq_evict_spans(self.handle, seq, spans, stream)
+    evict_spans_ragged = (lambda self, seq, spans, stream=None:
+                          sq_evict_spans_ragged(self.handle, seq, spans, stream))
     prefill_attention = (lambda self, seq, layer, n_q, q, out, out_dtype=SQ_OUT_BF16, lse=None,
                          sm_scale=1.0, spans=(), stream=None:
                          sq_prefill_attention(self.handle, seq, layer, n_q, q, out, out_dtype, lse,
@@ -349,6 +368,7 @@ class Cache:
     seq_info = lambda self, seq: sq_seq_info(self.handle, seq)
     next_pos = lambda self, seq: sq_seq_next_pos(self.handle, seq)
     page_table = lambda self, seq: sq_get_page_table(self.handle, seq)
+    page_fills = lambda self, seq: sq_get_page_fill(self.handle, seq)
     page_refcount = lambda self, page: sq_page_refcount(self.handle, page)
     free_pages = lambda self: sq_free_pages(self.handle)
     stats = lambda self: sq_stats(self.handle)

@@ -34,36 +34,39 @@ int sqh_append(void* c, int32_t h, int32_t n) {
     return static_cast<HostCache*>(c)->append(h, n, &p);
 }
 
-// stats_out (may be NULL): moved_rows, cow_pages, freed_pages, first_row, n_runs
-int sqh_evict(void* c, int32_t h, const int32_t* spans, int32_t n_spans, int64_t* stats_out) {
+// ragged: 0 dense, 1 ragged.  stats_out (may be NULL): moved_rows, cow_pages,
+// freed_pages, zeroed_rows, windows, number of moves.
+int sqh_evict(void* c, int32_t h, const int32_t* spans, int32_t n_spans, int32_t ragged,
+              int64_t* stats_out) {
     std::vector<int32_t> a(n_spans > 0 ? n_spans : 0), b(a.size());
     for (int32_t i = 0; i < n_spans; ++i) { a[i] = spans[2 * i]; b[i] = spans[2 * i + 1]; }
     EvictPlan p;
-    int rc = static_cast<HostCache*>(c)->evict(h, a.data(), b.data(), n_spans, &p);
+    int rc = static_cast<HostCache*>(c)->evict(h, a.data(), b.data(), n_spans, &p, ragged != 0);
     if (rc == kOk && stats_out) {
         stats_out[0] = p.moved_rows;
         stats_out[1] = (int64_t)p.cow_pages.size();
         stats_out[2] = (int64_t)p.freed.size();
-        stats_out[3] = p.first_row;
-        stats_out[4] = (int64_t)p.run_dst.size();
+        stats_out[3] = p.zeroed_rows;
+        stats_out[4] = p.windows;
+        stats_out[5] = (int64_t)p.moves.size();
     }
     return rc;
 }
 
 // Evicts and returns the compaction tiles (4 ints each: dst_page, dst_slot,
 // n_rows, piece_begin) and pieces (src_page, src_slot, n_rows, dst_row).
-int sqh_evict_tiles(void* c, int32_t h, const int32_t* spans, int32_t n_spans, int32_t tile_rows,
-                    int32_t* tiles_out, int32_t tiles_cap, int32_t* pieces_out,
+int sqh_evict_tiles(void* c, int32_t h, const int32_t* spans, int32_t n_spans, int32_t ragged,
+                    int32_t tile_rows, int32_t* tiles_out, int32_t tiles_cap, int32_t* pieces_out,
                     int32_t pieces_cap, int32_t* n_tiles, int32_t* n_pieces) {
     HostCache* hc = static_cast<HostCache*>(c);
     std::vector<int32_t> a(n_spans > 0 ? n_spans : 0), b(a.size());
     for (int32_t i = 0; i < n_spans; ++i) { a[i] = spans[2 * i]; b[i] = spans[2 * i + 1]; }
     EvictPlan p;
-    int rc = hc->evict(h, a.data(), b.data(), n_spans, &p);
+    int rc = hc->evict(h, a.data(), b.data(), n_spans, &p, ragged != 0);
     if (rc != kOk) return rc;
     std::vector<EvictTile> tiles;
     std::vector<EvictPiece> pieces;
-    evict_tiles(p, hc->geom().P, tile_rows, &tiles, &pieces);
+    evict_tiles(p, tile_rows, &tiles, &pieces);
     *n_tiles = (int32_t)tiles.size();
     *n_pieces = (int32_t)pieces.size();
     if ((int32_t)tiles.size() > tiles_cap || (int32_t)pieces.size() > pieces_cap) return kInvalidArg;
@@ -96,6 +99,37 @@ int sqh_page_table(void* c, int32_t h, int32_t* out, int32_t cap, int32_t* n_out
     return kOk;
 }
 
+int sqh_page_fill(void* c, int32_t h, int32_t* out, int32_t cap, int32_t* n_out) {
+    const Seq* s = static_cast<HostCache*>(c)->seq(h);
+    if (!s) return kBadHandle;
+    *n_out = (int32_t)s->fill.size();
+    if (cap < *n_out) return kInvalidArg;
+    std::memcpy(out, s->fill.data(), sizeof(int32_t) * s->fill.size());
+    return kOk;
+}
+
+// The slot-space spans and end a masked prefill of the last n_q rows of
+// sequence h uses (prefill_slot_spans); out receives start, end pairs.
+int sqh_prefill_slot_spans(void* c, int32_t h, int32_t n_q, const int32_t* spans,
+                           int32_t n_spans, int32_t* out, int32_t cap, int32_t* n_out,
+                           int32_t* n_slots) {
+    HostCache* hc = static_cast<HostCache*>(c);
+    const Seq* s = hc->seq(h);
+    if (!s) return kBadHandle;
+    std::vector<int32_t> a(n_spans > 0 ? n_spans : 0), b(a.size()), xa, xb;
+    for (int32_t i = 0; i < n_spans; ++i) { a[i] = spans[2 * i]; b[i] = spans[2 * i + 1]; }
+    int rc = prefill_slot_spans(*s, hc->geom().P, n_q, a.data(), b.data(), n_spans, &xa, &xb,
+                                n_slots);
+    if (rc != kOk) return rc;
+    *n_out = (int32_t)xa.size();
+    if (cap < *n_out) return kInvalidArg;
+    for (size_t i = 0; i < xa.size(); ++i) {
+        out[2 * i] = xa[i];
+        out[2 * i + 1] = xb[i];
+    }
+    return kOk;
+}
+
 int sqh_refcount(void* c, int32_t p) {
     HostCache* hc = static_cast<HostCache*>(c);
     if (p < 0 || p >= hc->geom().num_pages) return -1;
@@ -106,10 +140,10 @@ int sqh_free_count(void* c) { return static_cast<HostCache*>(c)->alloc().free_co
 
 int64_t sqh_peak_live_pages(void* c) { return static_cast<HostCache*>(c)->peak_live_pages(); }
 
-// Plans a decode call.  layout_out receives 16 int64 values:
+// Plans a decode call.  layout_out receives 17 int64 values:
 //   offsets segs, items, cta_begin, page_ids, comb_off, arrive, total,
 //   counts n_segs, n_items, n_ctas, n_page_ids, n_comb_keys, n_comb_ent,
-//   unique_tokens, logical_tokens, sizeof(DecodeSeg).
+//   unique_tokens, logical_tokens, sizeof(DecodeSeg), offset page_fill (-1: none).
 // If buf is non-NULL and buf_bytes >= total, the serialised plan is written.
 int sqh_plan_decode(void* c, const int32_t* handles, int32_t n, int32_t n_ctas,
                     int64_t* layout_out, uint8_t* buf, int64_t buf_bytes) {
@@ -118,9 +152,9 @@ int sqh_plan_decode(void* c, const int32_t* handles, int32_t n, int32_t n_ctas,
     int rc = plan_decode(*hc, handles, n, n_ctas, &p);
     if (rc != kOk) return rc;
     DecodePlanLayout L = plan_layout(p, n, hc->geom().Hkv);
-    int64_t v[16] = {L.segs, L.items, L.cta_begin, L.page_ids, L.comb_off, L.arrive, L.total,
+    int64_t v[17] = {L.segs, L.items, L.cta_begin, L.page_ids, L.comb_off, L.arrive, L.total,
                      L.n_segs, L.n_items, L.n_ctas, L.n_page_ids, L.n_comb_keys, L.n_comb_ent,
-                     p.unique_tokens, p.logical_tokens, (int64_t)sizeof(DecodeSeg)};
+                     p.unique_tokens, p.logical_tokens, (int64_t)sizeof(DecodeSeg), L.page_fill};
     std::memcpy(layout_out, v, sizeof v);
     if (buf) {
         if (buf_bytes < L.total) return kInvalidArg;

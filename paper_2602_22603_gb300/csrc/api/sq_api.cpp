@@ -502,7 +502,9 @@ int sq_append_kv(sq_cache* c, sq_seq seq, int32_t n_tokens, const void* k, const
         cudaError_t e = launch_cow_copy(ca, c->num_sms, st);
         if (e != cudaSuccess) return undo(cuda_status(e));
     }
-    const int64_t end = (int64_t)plan.n0 + plan.n_new;
+    // rows go to slot-space positions pos0 .. pos0 + n - 1 (the last page's
+    // free slots, then the fresh pages)
+    const int64_t end = (int64_t)plan.pos0 + plan.n_new;
     for (size_t b = 0; b < plan.pages.size(); b += kAppendMaxPages) {
         AppendArgs a;
         a.pool = c->pool;
@@ -514,11 +516,11 @@ int sq_append_kv(sq_cache* c, sq_seq seq, int32_t n_tokens, const void* k, const
         a.page_index0 = plan.first_page_index + (int32_t)b;
         a.n_pages = (int32_t)std::min<size_t>(kAppendMaxPages, plan.pages.size() - b);
         for (int i = 0; i < a.n_pages; ++i) a.pages[i] = plan.pages[b + i];
-        const int64_t pb = std::max<int64_t>(plan.n0, (int64_t)a.page_index0 * g.P);
+        const int64_t pb = std::max<int64_t>(plan.pos0, (int64_t)a.page_index0 * g.P);
         const int64_t pe = std::min<int64_t>(end, (int64_t)(a.page_index0 + a.n_pages) * g.P);
         if (pe <= pb) continue;
         a.pos0 = (int32_t)pb;
-        a.tok_begin = (int32_t)(pb - plan.n0);
+        a.tok_begin = (int32_t)(pb - plan.pos0);
         a.n_tok = (int32_t)(pe - pb);
         a.err = c->d_err;
         cudaError_t e = launch_append(a, c->num_sms, st);
@@ -583,8 +585,8 @@ int sq_append_kv_batch(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, const vo
         a.n = std::min(kAppendBatchMax, n_seqs - b);
         for (int32_t i = 0; i < a.n; ++i) {
             const AppendPlan& pl = plans[b + i];
-            a.page[i] = pl.pages[0];                 // the page holding position n0
-            a.slot[i] = pl.n0 % g.P;
+            a.page[i] = pl.pages[0];                 // the page holding slot position pos0
+            a.slot[i] = pl.pos0 % g.P;
         }
         a.err = c->d_err;
         cudaError_t e = launch_append_batch(a, c->num_sms, st);
@@ -720,6 +722,8 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
     a.page_ids = reinterpret_cast<const int32_t*>(hit->d_plan + L.page_ids);
     a.comb_off = reinterpret_cast<const int32_t*>(hit->d_plan + L.comb_off);
     a.arrive = reinterpret_cast<unsigned int*>(hit->d_plan + L.arrive);
+    a.page_fill = L.page_fill >= 0 ? reinterpret_cast<const int32_t*>(hit->d_plan + L.page_fill)
+                                   : nullptr;
     a.q = reinterpret_cast<const __nv_bfloat16*>(q);
     a.out = out;
     a.part_o = part_o;
@@ -749,8 +753,12 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
     return SQ_OK;
 }
 
-int sq_evict_spans(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_spans, void* stream) {
-    TraceRange trace_("sq_evict_spans");
+}  // extern "C"
+
+namespace {
+
+int evict_impl(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_spans, void* stream,
+               bool ragged) {
     if (!c) return SQ_ERR_BAD_HANDLE;
     if (!c->host->seq(seq)) return SQ_ERR_BAD_HANDLE;
     if (n_spans < 0 || (n_spans > 0 && !spans)) return SQ_ERR_INVALID_ARG;
@@ -761,7 +769,7 @@ int sq_evict_spans(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_span
         b[i] = spans[i].end;
     }
     EvictPlan plan;
-    int rc = c->host->evict(seq, a.data(), b.data(), n_spans, &plan);
+    int rc = c->host->evict(seq, a.data(), b.data(), n_spans, &plan, ragged);
     if (rc != SQ_OK) return rc;
     const Geometry& g = c->g;
     cudaStream_t st = as_stream(stream);
@@ -771,10 +779,10 @@ int sq_evict_spans(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_span
     };
     rc = fence_taken_pages(c, plan.cow_pages, stream);
     if (rc != SQ_OK) return undo(rc);
-    if (plan.first_row < plan.n_new) {
+    if (!plan.moves.empty()) {
         std::vector<EvictTile> tiles;
         std::vector<EvictPiece> pieces;
-        evict_tiles(plan, g.P, c->evict_tile_rows, &tiles, &pieces);
+        evict_tiles(plan, c->evict_tile_rows, &tiles, &pieces);
         const size_t tb = tiles.size() * sizeof(EvictTile);
         std::vector<uint8_t> buf(tb + pieces.size() * sizeof(EvictPiece));
         std::memcpy(buf.data(), tiles.data(), tb);
@@ -792,6 +800,7 @@ int sq_evict_spans(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_span
         ea.n_tiles = (int32_t)tiles.size();
         ea.n_pieces = (int32_t)pieces.size();
         ea.tile_rows = c->evict_tile_rows;
+        ea.zero_tiles = plan.zeroed_rows > 0 ? 1 : 0;
         ea.err = c->d_err;
         cudaError_t e = launch_evict(ea, st);
         if (e != cudaSuccess) return undo(cuda_status(e));
@@ -806,9 +815,25 @@ int sq_evict_spans(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_span
     c->stats.evict_calls += 1;
     c->stats.evicted_tokens += plan.evicted;
     c->stats.evict_moved_rows += plan.moved_rows;
-    c->stats.evict_bytes += 2 * plan.moved_rows * g.L * g.token_layer_bytes();
+    // rows copied are read and written, zeroed rows only written
+    c->stats.evict_bytes += (2 * plan.moved_rows + plan.zeroed_rows) * g.L * g.token_layer_bytes();
     c->stats.cow_pages += (int64_t)plan.cow_pages.size();
     return SQ_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int sq_evict_spans(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_spans, void* stream) {
+    TraceRange trace_("sq_evict_spans");
+    return evict_impl(c, seq, spans, n_spans, stream, false);
+}
+
+int sq_evict_spans_ragged(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_spans,
+                          void* stream) {
+    TraceRange trace_("sq_evict_spans_ragged");
+    return evict_impl(c, seq, spans, n_spans, stream, true);
 }
 
 int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, const void* q,
@@ -855,8 +880,21 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
             sb[i] = key[2 * i + 1];
         }
         PrefillPlanHost plan;
-        int rc = plan_prefill(g, s->n, n_q, sa.data(), sb.data(), n_spans, c->num_sms, &plan,
+        int rc;
+        if (has_partial_pages(*s, g.P)) {
+            // slot space: the spans mapped through the page fills, plus the
+            // unused slots of the partial pages
+            std::vector<int32_t> xa, xb;
+            int32_t n_slots = 0;
+            rc = prefill_slot_spans(*s, g.P, n_q, sa.data(), sb.data(), n_spans, &xa, &xb,
+                                    &n_slots);
+            if (rc != SQ_OK) return rc;
+            rc = plan_prefill(g, n_slots, n_q, xa.data(), xb.data(), (int32_t)xa.size(),
+                              c->num_sms, &plan, s->pages.data());
+        } else {
+            rc = plan_prefill(g, s->n, n_q, sa.data(), sb.data(), n_spans, c->num_sms, &plan,
                               s->pages.data());
+        }
         if (rc != SQ_OK) return rc;
         // upload: key tiles, per-CTA-tile counts, then the page of every piece
         const size_t tb = plan.tiles.size() * sizeof(PrefillTile);
@@ -958,7 +996,7 @@ int sq_prefill_attention(sq_cache* c, sq_seq seq, int32_t layer, int32_t n_q, co
     a.tile_pages = reinterpret_cast<const int32_t*>(plan.d + plan.tb + plan.qb);
     a.n_pieces = plan.n_pieces;
     a.n_tiles = plan.n_tiles;
-    a.n = s->n;
+    a.n = slot_end(*s, g.P);   // the slot-space end (s->n when every page but the last is full)
     a.n_q = n_q;
     a.layer = layer;
     a.Hq = g.Hq;
@@ -1061,6 +1099,17 @@ int sq_get_page_table(sq_cache* c, sq_seq seq, int32_t* host_out, int32_t cap, i
     if (n_out) *n_out = n;
     if (n > 0 && (!host_out || cap < n)) return SQ_ERR_INVALID_ARG;
     if (n > 0) std::memcpy(host_out, s->pages.data(), sizeof(int32_t) * n);
+    return SQ_OK;
+}
+
+int sq_get_page_fill(sq_cache* c, sq_seq seq, int32_t* host_out, int32_t cap, int32_t* n_out) {
+    if (!c) return SQ_ERR_BAD_HANDLE;
+    const Seq* s = c->host->seq(seq);
+    if (!s) return SQ_ERR_BAD_HANDLE;
+    const int32_t n = (int32_t)s->fill.size();
+    if (n_out) *n_out = n;
+    if (n > 0 && (!host_out || cap < n)) return SQ_ERR_INVALID_ARG;
+    if (n > 0) std::memcpy(host_out, s->fill.data(), sizeof(int32_t) * n);
     return SQ_OK;
 }
 
@@ -1192,6 +1241,8 @@ int sq_decode_attention_noalloc(sq_cache* c, const sq_seq* seqs, int32_t n_seqs,
     a.page_ids = reinterpret_cast<const int32_t*>(scratch + L.page_ids);
     a.comb_off = reinterpret_cast<const int32_t*>(scratch + L.comb_off);
     a.arrive = reinterpret_cast<unsigned int*>(scratch + L.arrive);
+    a.page_fill = L.page_fill >= 0 ? reinterpret_cast<const int32_t*>(scratch + L.page_fill)
+                                   : nullptr;
     a.q = reinterpret_cast<const __nv_bfloat16*>(q);
     a.out = out;
     a.part_o = part_o;

@@ -117,6 +117,7 @@ int HostCache::seq_new(int32_t* handle) {
     s.gen = (s.gen % 2047) + 1;  // 1 .. 2047: handles stay positive
     s.n = 0;
     s.pages.clear();
+    s.fill.clear();
     s.next_pos = 0;
     s.version = g_version_counter++;
     s.last_stream = nullptr;
@@ -128,6 +129,7 @@ int HostCache::fork(int32_t parent, int32_t* child) {
     const Seq* ps = seq(parent);
     if (!ps) return kBadHandle;
     std::vector<int32_t> pages = ps->pages;
+    std::vector<int32_t> fill = ps->fill;
     int32_t n = ps->n;
     const int64_t next_pos = ps->next_pos;
     void* st = ps->last_stream;
@@ -135,6 +137,7 @@ int HostCache::fork(int32_t parent, int32_t* child) {
     if (rc != kOk) return rc;
     Seq* cs = seq_mut(*child);
     cs->pages = std::move(pages);
+    cs->fill = std::move(fill);
     cs->n = n;
     cs->next_pos = next_pos;
     cs->last_stream = st;
@@ -151,12 +154,17 @@ int HostCache::append(int32_t h, int32_t n_new, AppendPlan* plan) {
     const int32_t n = s->n;
     plan->n0 = n;
     plan->n_new = n_new;
+    plan->pos0 = slot_end(*s, P);
+    plan->last_fill0 = s->pages.empty() ? 0 : s->fill.back();
     if (n_new == 0) return kOk;
     if ((int64_t)n + n_new >= (1LL << 31)) return kCapacity;
-    const int32_t new_np = ceil_div((int64_t)n + n_new, P);
+    // the last page's free slots take the first rows, then fresh pages
+    const int32_t room = s->pages.empty() ? 0 : P - s->fill.back();
+    const int64_t grow = n_new > room ? ((int64_t)n_new - room + P - 1) / P : 0;
+    const int64_t new_np = (int64_t)s->pages.size() + grow;
     if (new_np > g_.max_pages_per_seq) return kCapacity;
-    const bool cow = (n % P != 0) && alloc_.refcount(s->pages.back()) > 1;
-    const int32_t need = (cow ? 1 : 0) + new_np - (int32_t)s->pages.size();
+    const bool cow = room > 0 && alloc_.refcount(s->pages.back()) > 1;
+    const int64_t need = (cow ? 1 : 0) + grow;
     if (need > alloc_.free_count()) return kNoPages;
 
     if (cow) {
@@ -167,16 +175,24 @@ int HostCache::append(int32_t h, int32_t n_new, AppendPlan* plan) {
         plan->cow = true;
         plan->cow_old = old;
         plan->cow_new = fresh;
-        plan->cow_rows = n % P;
+        plan->cow_rows = s->fill.back();
         plan->taken.push_back(fresh);
     }
-    while ((int32_t)s->pages.size() < new_np) {
+    plan->first_page_index = plan->pos0 / P;
+    int32_t left = n_new;
+    if (room > 0) {
+        const int32_t k = std::min(room, left);
+        s->fill.back() += k;
+        left -= k;
+    }
+    while (left > 0) {
         int32_t p = take_lowest();
         s->pages.push_back(p);
+        s->fill.push_back(std::min(P, left));
+        left -= s->fill.back();
         plan->taken.push_back(p);
     }
-    plan->first_page_index = n / P;
-    plan->pages.assign(s->pages.begin() + n / P, s->pages.end());
+    plan->pages.assign(s->pages.begin() + plan->first_page_index, s->pages.end());
     s->n = n + n_new;
     s->next_pos += n_new;
     s->version = g_version_counter++;
@@ -186,11 +202,14 @@ int HostCache::append(int32_t h, int32_t n_new, AppendPlan* plan) {
 void HostCache::undo_append(int32_t h, const AppendPlan& plan) {
     Seq* s = seq_mut(h);
     if (!s || plan.n_new == 0) return;
-    const int32_t old_np = ceil_div(plan.n0, g_.P);
-    while ((int32_t)s->pages.size() > old_np) {
+    // pages before the append: pos0 = (pages - 1) * P + last fill
+    const int32_t keep = plan.last_fill0 > 0 ? (plan.pos0 - plan.last_fill0) / g_.P + 1 : 0;
+    while ((int32_t)s->pages.size() > keep) {
         alloc_.drop_ref(s->pages.back());
         s->pages.pop_back();
+        s->fill.pop_back();
     }
+    if (keep > 0) s->fill.back() = plan.last_fill0;
     if (plan.cow) {
         alloc_.drop_ref(plan.cow_new);
         alloc_.add_ref(plan.cow_old);
@@ -201,82 +220,202 @@ void HostCache::undo_append(int32_t h, const AppendPlan& plan) {
     s->version = g_version_counter++;
 }
 
+bool has_partial_pages(const Seq& s, int32_t P) {
+    for (size_t q = 0; q + 1 < s.fill.size(); ++q)
+        if (s.fill[q] != P) return true;
+    return false;
+}
+
+namespace {
+
+// A run of rows moving as one: destination page index / slot, source page
+// index / slot (indices into the sequence's page table before the eviction).
+struct Run {
+    int32_t dq, ds, sq, ss, n;
+};
+
+// Packs the kept logical rows `kept` (increasing, disjoint half-open ranges)
+// into consecutive slots from slot 0 of page index dq0, splitting at source
+// and destination page boundaries.  start[q] = first logical row of page q.
+void pack_rows(const std::vector<std::pair<int32_t, int32_t>>& kept,
+               const std::vector<int32_t>& start, int32_t P, int32_t dq0, std::vector<Run>* out) {
+    int64_t m = 0;  // destination index from slot 0 of page dq0
+    size_t q = 0;   // source page index, monotone
+    for (const auto& r : kept) {
+        int32_t j = r.first;
+        while (j < r.second) {
+            while (start[q + 1] <= j) ++q;
+            const int32_t ds = (int32_t)(m % P);
+            const int32_t n = std::min({r.second - j, start[q + 1] - j, P - ds});
+            out->push_back({dq0 + (int32_t)(m / P), ds, (int32_t)q, j - start[q], n});
+            j += n;
+            m += n;
+        }
+    }
+}
+
+}  // namespace
+
 int HostCache::evict(int32_t h, const int32_t* starts, const int32_t* ends,
-                     int32_t n_spans, EvictPlan* plan) {
+                     int32_t n_spans, EvictPlan* plan, bool ragged) {
     *plan = EvictPlan();
     Seq* s = seq_mut(h);
     if (!s) return kBadHandle;
     if (n_spans < 0) return kInvalidArg;
     const int32_t n = s->n;
     const int32_t P = g_.P;
+    plan->ragged = ragged;
     plan->n_old = n;
     plan->n_new = n;
-    plan->first_row = n;
     plan->old_pages = s->pages;
+    plan->old_fill = s->fill;
     plan->new_pages = s->pages;
+    plan->new_fill = s->fill;
     if (n_spans == 0) return kOk;
     if (!starts || !ends) return kInvalidArg;
 
     std::vector<std::pair<int32_t, int32_t>> sp;
     int rc = sorted_spans(n, starts, ends, n_spans, &sp);
     if (rc != kOk) return rc;
+    const int32_t np = (int32_t)s->pages.size();
+    std::vector<int32_t> start(np + 1, 0);
+    for (int32_t q = 0; q < np; ++q) start[q + 1] = start[q] + s->fill[q];
     int64_t removed = 0;
     for (auto& ab : sp) removed += ab.second - ab.first;
-    // kept runs
-    int32_t cur = 0, dst = 0;
-    for (auto& ab : sp) {
-        if (ab.first > cur) {
-            plan->run_dst.push_back(dst);
-            plan->run_src.push_back(cur);
-            plan->run_len.push_back(ab.first - cur);
-            dst += ab.first - cur;
+
+    // Windows: the whole table (dense), or the maximal runs of pages a span
+    // touches (ragged).  Each window's kept rows are packed from slot 0 of
+    // its first page.
+    struct Window {
+        int32_t qa, qb;                                 // page indices, inclusive
+        std::vector<std::pair<int32_t, int32_t>> kept;  // logical row ranges
+        int32_t used = 0;                               // pages that receive rows
+    };
+    std::vector<Window> win;
+    if (!ragged) {
+        win.push_back({0, np - 1, {}, 0});
+    } else {
+        std::vector<uint8_t> touched(np, 0);
+        int32_t q = 0;
+        for (auto& ab : sp) {
+            while (start[q + 1] <= ab.first) ++q;
+            int32_t e = q;
+            while (start[e + 1] < ab.second) ++e;
+            for (int32_t x = q; x <= e; ++x) touched[x] = 1;
         }
-        cur = ab.second;
+        for (q = 0; q < np;) {
+            if (!touched[q]) {
+                ++q;
+                continue;
+            }
+            int32_t e = q;
+            while (e + 1 < np && touched[e + 1]) ++e;
+            win.push_back({q, e, {}, 0});
+            q = e + 1;
+        }
     }
-    if (n > cur) {
-        plan->run_dst.push_back(dst);
-        plan->run_src.push_back(cur);
-        plan->run_len.push_back(n - cur);
-        dst += n - cur;
+    size_t si = 0;
+    for (Window& w : win) {
+        int32_t cur = start[w.qa];
+        const int32_t end = start[w.qb + 1];
+        while (si < sp.size() && sp[si].second <= cur) ++si;
+        size_t k = si;
+        while (cur < end) {
+            if (k < sp.size() && sp[k].first < end) {
+                if (sp[k].first > cur) w.kept.push_back({cur, sp[k].first});
+                cur = std::max(cur, sp[k].second);
+                ++k;
+            } else {
+                w.kept.push_back({cur, end});
+                cur = end;
+            }
+        }
     }
-    const int32_t n2 = (int32_t)(n - removed);
-    const int32_t new_np = ceil_div(n2, P);
-    const int32_t a0 = sp[0].first;
-    const int32_t qc = a0 / P;
-    const bool any_change = n2 > a0;  // some kept row moves
-    // copy-on-write needs
+
+    // runs, and which destination pages change
+    std::vector<std::vector<Run>> runs(win.size());
+    std::vector<uint8_t> changed(np, 0);
+    std::vector<int32_t> dest_fill(np, 0);
+    for (size_t wi = 0; wi < win.size(); ++wi) {
+        Window& w = win[wi];
+        pack_rows(w.kept, start, P, w.qa, &runs[wi]);
+        int64_t r = 0;
+        for (auto& kr : w.kept) r += kr.second - kr.first;
+        w.used = (int32_t)((r + P - 1) / P);
+        for (int32_t i = 0; i < w.used; ++i)
+            dest_fill[w.qa + i] = (int32_t)std::min<int64_t>(P, r - (int64_t)i * P);
+        for (const Run& x : runs[wi])
+            if (x.dq != x.sq || x.ds != x.ss) changed[x.dq] = 1;
+    }
+    // the last page of a ragged window is also written when its unused
+    // slots are zeroed, which happens only if its rows change anyway
     int32_t need = 0;
-    if (any_change)
-        for (int32_t q = qc; q < new_np; ++q)
-            if (alloc_.refcount(s->pages[q]) > 1) ++need;
+    for (const Window& w : win)
+        for (int32_t i = 0; i < w.used; ++i)
+            if (changed[w.qa + i] && alloc_.refcount(s->pages[w.qa + i]) > 1) ++need;
     if (need > alloc_.free_count()) return kNoPages;
 
     // commit
-    std::vector<int32_t> new_pages(s->pages.begin(), s->pages.begin() + new_np);
-    int64_t moved = 0;
-    if (any_change) {
-        for (int32_t q = qc; q < new_np; ++q) {
-            const int32_t row_end = std::min<int64_t>((int64_t)q * P + P, n2);
-            if (alloc_.refcount(s->pages[q]) > 1) {
-                new_pages[q] = take_lowest();
-                plan->cow_pages.push_back(new_pages[q]);
-                moved += row_end - (int64_t)q * P;
-            } else {
-                moved += row_end - std::max<int64_t>((int64_t)q * P, a0);
+    std::vector<int32_t> page_at(s->pages);   // destination page of each page index
+    for (const Window& w : win)
+        for (int32_t i = 0; i < w.used; ++i) {
+            const int32_t q = w.qa + i;
+            if (changed[q] && alloc_.refcount(s->pages[q]) > 1) {
+                page_at[q] = take_lowest();
+                plan->cow_pages.push_back(page_at[q]);
             }
         }
-        for (int32_t q = qc; q < new_np; ++q)
-            if (new_pages[q] != s->pages[q]) alloc_.drop_ref(s->pages[q]);
+    for (size_t wi = 0; wi < win.size(); ++wi) {
+        const Window& w = win[wi];
+        for (const Run& x : runs[wi]) {
+            const bool fresh = page_at[x.dq] != s->pages[x.dq];
+            if (!fresh && x.dq == x.sq && x.ds == x.ss) continue;  // rows stay where they are
+            plan->moves.push_back({page_at[x.dq], x.ds, s->pages[x.sq], x.ss, x.n});
+            plan->moved_rows += x.n;
+        }
+        if (ragged && w.used > 0) {
+            const int32_t q = w.qa + w.used - 1;
+            const bool fresh = page_at[q] != s->pages[q];
+            if ((changed[q] || fresh) && dest_fill[q] < P) {
+                plan->moves.push_back({page_at[q], dest_fill[q], -1, 0, P - dest_fill[q]});
+                plan->zeroed_rows += P - dest_fill[q];
+            }
+        }
     }
-    for (size_t q = new_np; q < s->pages.size(); ++q)
-        if (alloc_.drop_ref(s->pages[q])) plan->freed.push_back(s->pages[q]);
-    plan->new_pages = new_pages;
-    plan->n_new = n2;
-    plan->first_row = any_change ? qc * P : n2;
-    plan->moved_rows = moved;
+    // references: replaced originals and the pages that leave
+    std::vector<int32_t> pages, fill;
+    pages.reserve(np);
+    fill.reserve(np);
+    size_t wi = 0;
+    for (int32_t q = 0; q < np;) {
+        if (wi < win.size() && win[wi].qa == q) {
+            const Window& w = win[wi];
+            for (int32_t i = 0; i <= w.qb - w.qa; ++i) {
+                const int32_t x = w.qa + i;
+                if (i < w.used) {
+                    if (page_at[x] != s->pages[x]) alloc_.drop_ref(s->pages[x]);
+                    pages.push_back(page_at[x]);
+                    fill.push_back(dest_fill[x]);
+                } else if (alloc_.drop_ref(s->pages[x])) {
+                    plan->freed.push_back(s->pages[x]);
+                }
+            }
+            q = w.qb + 1;
+            ++wi;
+        } else {
+            pages.push_back(s->pages[q]);
+            fill.push_back(s->fill[q]);
+            ++q;
+        }
+    }
+    plan->new_pages = pages;
+    plan->new_fill = fill;
+    plan->n_new = (int32_t)(n - removed);
     plan->evicted = (int32_t)removed;
-    s->pages = std::move(new_pages);
-    s->n = n2;
+    plan->windows = ragged ? (int32_t)win.size() : 1;
+    s->pages = std::move(pages);
+    s->fill = std::move(fill);
+    s->n = plan->n_new;
     s->version = g_version_counter++;
     return kOk;
 }
@@ -284,19 +423,15 @@ int HostCache::evict(int32_t h, const int32_t* starts, const int32_t* ends,
 void HostCache::undo_evict(int32_t h, const EvictPlan& plan) {
     Seq* s = seq_mut(h);
     if (!s || plan.n_new == plan.n_old) return;
-    // trailing pages back
-    for (size_t q = plan.new_pages.size(); q < plan.old_pages.size(); ++q) {
-        int32_t p = plan.old_pages[q];
+    // every page of the old table gains its holder back before the new
+    // table's pages lose theirs, so no page shared by both passes zero
+    for (int32_t p : plan.old_pages) {
         if (alloc_.refcount(p) == 0) alloc_.take(p);
         else alloc_.add_ref(p);
     }
-    for (size_t q = 0; q < plan.new_pages.size(); ++q) {
-        if (plan.new_pages[q] != plan.old_pages[q]) {
-            alloc_.drop_ref(plan.new_pages[q]);
-            alloc_.add_ref(plan.old_pages[q]);
-        }
-    }
+    for (int32_t p : plan.new_pages) alloc_.drop_ref(p);
     s->pages = plan.old_pages;
+    s->fill = plan.old_fill;
     s->n = plan.n_old;
     s->version = g_version_counter++;
 }
@@ -314,53 +449,30 @@ int HostCache::release(int32_t h, std::vector<int32_t>* freed) {
     return kOk;
 }
 
-void evict_tiles(const EvictPlan& p, int32_t P, int32_t tile_rows,
-                 std::vector<EvictTile>* tiles, std::vector<EvictPiece>* pieces) {
+void evict_tiles(const EvictPlan& p, int32_t tile_rows, std::vector<EvictTile>* tiles,
+                 std::vector<EvictPiece>* pieces) {
     tiles->clear();
     pieces->clear();
-    if (p.first_row >= p.n_new) return;
-    size_t r = 0;  // current kept run (monotone in the destination row)
-    const int32_t first_q = p.first_row / P;
-    const int32_t new_np = (int32_t)p.new_pages.size();
-    for (int32_t q = first_q; q < new_np; ++q) {
-        const int32_t page_begin = q * P;
-        const int32_t row_end = std::min<int64_t>((int64_t)page_begin + P, p.n_new);
-        const bool fresh = p.new_pages[q] != p.old_pages[q];
-        int32_t row = page_begin;
-        if (!fresh) {
-            // skip destination rows that keep their row (kept[j] == j)
-            while (row < row_end) {
-                while (r + 1 < p.run_dst.size() && p.run_dst[r + 1] <= row) ++r;
-                const int32_t src = p.run_src[r] + (row - p.run_dst[r]);
-                if (src != row) break;
-                // the whole rest of this run keeps its rows
-                row = std::min<int32_t>(row_end, p.run_dst[r] + p.run_len[r]);
+    EvictTile* open = nullptr;   // the tile being filled
+    bool open_zero = false;
+    for (const EvictMove& m : p.moves) {
+        const bool zero = m.src_page < 0;
+        int32_t done = 0;
+        while (done < m.n) {
+            const int32_t dst_slot = m.dst_slot + done;
+            // continue the open tile when this move extends it in place
+            const bool cont = open && open_zero == zero && open->dst_page == m.dst_page &&
+                              open->dst_slot + open->n_rows == dst_slot &&
+                              open->n_rows < tile_rows;
+            if (!cont) {
+                tiles->push_back({m.dst_page, dst_slot, 0, (int32_t)pieces->size()});
+                open = &tiles->back();
+                open_zero = zero;
             }
-        }
-        while (row < row_end) {
-            const int32_t t_end = std::min(row_end, row + tile_rows);
-            EvictTile t;
-            t.dst_page = p.new_pages[q];
-            t.dst_slot = row - page_begin;
-            t.n_rows = t_end - row;
-            t.piece_begin = (int32_t)pieces->size();
-            int32_t j = row;
-            while (j < t_end) {
-                while (r + 1 < p.run_dst.size() && p.run_dst[r + 1] <= j) ++r;
-                const int32_t src = p.run_src[r] + (j - p.run_dst[r]);
-                const int32_t run_left = p.run_dst[r] + p.run_len[r] - j;
-                const int32_t page_left = P - src % P;
-                const int32_t n = std::min({t_end - j, run_left, page_left});
-                EvictPiece pc;
-                pc.src_page = p.old_pages[src / P];
-                pc.src_slot = src % P;
-                pc.n_rows = n;
-                pc.dst_row = j - row;
-                pieces->push_back(pc);
-                j += n;
-            }
-            tiles->push_back(t);
-            row = t_end;
+            const int32_t k = std::min(m.n - done, tile_rows - open->n_rows);
+            if (!zero) pieces->push_back({m.src_page, m.src_slot + done, k, open->n_rows});
+            open->n_rows += k;
+            done += k;
         }
     }
 }
@@ -374,6 +486,7 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
     const Geometry& g = c.geom();
     if (n_seqs < 1 || !handles || n_ctas < 1) return kInvalidArg;
     std::vector<const Seq*> ss(n_seqs);
+    bool ragged = false;
     for (int32_t i = 0; i < n_seqs; ++i) {
         ss[i] = c.seq(handles[i]);
         if (!ss[i]) return kBadHandle;
@@ -381,12 +494,15 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
         for (int32_t j = 0; j < i; ++j)
             if (ss[j] == ss[i]) return kInvalidArg;
         out->logical_tokens += ss[i]->n;
+        ragged = ragged || has_partial_pages(*ss[i], g.P);
     }
     const int32_t P = g.P;
     const int32_t max_grp = kRowsPerTile / g.G();
 
-    // Group sequences holding the same physical page at the same logical
-    // index into shared runs (depth-first over the prefix tree of pages).
+    // Group sequences holding the same physical page, with the same fill, at
+    // the same page index into shared runs (depth-first over the prefix tree
+    // of pages).  (Two holders of one page can see different fills after a
+    // ragged eviction of one of them; they read that page separately.)
     // Every segment also records its family: the subtree of one first page
     // (a request, its forks and whatever they added).
     struct Work {
@@ -409,14 +525,14 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
         stack.pop_back();
         // partition by the page held at w.q (first-seen order)
         std::vector<std::vector<int32_t>> parts;
-        std::vector<int32_t> part_page;
+        std::vector<std::pair<int32_t, int32_t>> part_page;  // (page, fill)
         for (int32_t i : w.members) {
             if ((int32_t)ss[i]->pages.size() <= w.q) continue;
-            int32_t p = ss[i]->pages[w.q];
+            const std::pair<int32_t, int32_t> key{ss[i]->pages[w.q], ss[i]->fill[w.q]};
             size_t k = 0;
-            while (k < part_page.size() && part_page[k] != p) ++k;
+            while (k < part_page.size() && part_page[k] != key) ++k;
             if (k == part_page.size()) {
-                part_page.push_back(p);
+                part_page.push_back(key);
                 parts.emplace_back();
             }
             parts[k].push_back(i);
@@ -433,7 +549,8 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
                 bool same = true;
                 for (int32_t i : part) {
                     if ((int32_t)ss[i]->pages.size() <= q_end ||
-                        ss[i]->pages[q_end] != lead->pages[q_end]) {
+                        ss[i]->pages[q_end] != lead->pages[q_end] ||
+                        ss[i]->fill[q_end] != lead->fill[q_end]) {
                         same = false;
                         break;
                     }
@@ -450,15 +567,21 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
                 seg.n_tok = 0;
                 for (int32_t j = 0; j < seg.n_grp; ++j) {
                     int32_t i = part[b + j];
-                    int64_t lim = std::min<int64_t>((int64_t)ss[i]->n - (int64_t)q0 * P,
+                    // slot-space limit of this member inside the run
+                    int64_t lim = std::min<int64_t>((int64_t)slot_end(*ss[i], P) - (int64_t)q0 * P,
                                                     (int64_t)seg.n_pages * P);
                     seg.grp_seq[j] = i;
                     seg.grp_lim[j] = (int32_t)lim;
                     seg.n_tok = std::max(seg.n_tok, (int32_t)lim);
                 }
                 const Seq* sl = ss[part[b]];
-                for (int32_t q = q0; q < q_end; ++q) out->page_ids.push_back(sl->pages[q]);
-                out->unique_tokens += seg.n_tok;
+                for (int32_t q = q0; q < q_end; ++q) {
+                    out->page_ids.push_back(sl->pages[q]);
+                    if (ragged) out->page_fill.push_back(sl->fill[q]);
+                    // rows read: the filled slots below the run's limit
+                    const int64_t below = (int64_t)seg.n_tok - (int64_t)(q - q0) * P;
+                    out->unique_tokens += std::max<int64_t>(0, std::min<int64_t>(sl->fill[q], below));
+                }
                 out->segs.push_back(seg);
                 seg_fam.push_back(fam);
             }
@@ -566,6 +689,11 @@ DecodePlanLayout plan_layout(const DecodePlanHost& p, int32_t n_seqs, int32_t Hk
     L.page_ids = o;  o = align16(o + sizeof(int32_t) * L.n_page_ids);
     L.comb_off = o;  o = align16(o + sizeof(int32_t) * (L.n_comb_keys + 1));
     L.arrive = o;    o = align16(o + sizeof(uint32_t) * L.n_comb_keys);
+    if (!p.page_fill.empty()) {
+        L.page_fill = o; o = align16(o + sizeof(int32_t) * L.n_page_ids);
+    } else {
+        L.page_fill = -1;
+    }
     L.total = o;
     return L;
 }
@@ -577,6 +705,8 @@ void plan_serialize(const DecodePlanHost& p, const DecodePlanLayout& L, uint8_t*
     std::memcpy(dst + L.cta_begin, p.cta_begin.data(), sizeof(int32_t) * (L.n_ctas + 1));
     std::memcpy(dst + L.page_ids, p.page_ids.data(), sizeof(int32_t) * L.n_page_ids);
     std::memcpy(dst + L.comb_off, p.comb_off.data(), sizeof(int32_t) * (L.n_comb_keys + 1));
+    if (L.page_fill >= 0)
+        std::memcpy(dst + L.page_fill, p.page_fill.data(), sizeof(int32_t) * L.n_page_ids);
 }
 
 // ---------------------------------------------------------------------------
@@ -669,6 +799,50 @@ int plan_prefill(const Geometry& g, int32_t n, int32_t n_q, const int32_t* start
         }
     }
     out->n_split = split;
+    return kOk;
+}
+
+int prefill_slot_spans(const Seq& s, int32_t P, int32_t n_q, const int32_t* starts,
+                       const int32_t* ends, int32_t n_spans, std::vector<int32_t>* a_out,
+                       std::vector<int32_t>* b_out, int32_t* n_slots) {
+    a_out->clear();
+    b_out->clear();
+    std::vector<std::pair<int32_t, int32_t>> sp;
+    int rc = sorted_spans(s.n, starts, ends, n_spans, &sp);
+    if (rc != kOk) return rc;
+    const int32_t np = (int32_t)s.pages.size();
+    *n_slots = slot_end(s, P);
+    if (n_q < 1 || n_q > s.n) return kInvalidArg;
+    std::vector<int32_t> start(np + 1, 0);
+    for (int32_t q = 0; q < np; ++q) start[q + 1] = start[q] + s.fill[q];
+    // the queries must sit in consecutive slots: the slot of row n - n_q is
+    // n_slots - n_q exactly when no unused slot lies between
+    {
+        const int32_t j = s.n - n_q;
+        int32_t q = (int32_t)(std::upper_bound(start.begin(), start.end(), j) - start.begin()) - 1;
+        if (q * P + (j - start[q]) != *n_slots - n_q) return kUnsupported;
+    }
+    // spans and unused slots, in slot order, adjacent ranges merged
+    std::vector<std::pair<int32_t, int32_t>> r;
+    auto add = [&](int32_t a, int32_t b) {
+        if (a >= b) return;
+        if (!r.empty() && r.back().second == a) r.back().second = b;
+        else r.push_back({a, b});
+    };
+    size_t k = 0;
+    for (int32_t q = 0; q < np; ++q) {
+        // the span parts inside page q
+        while (k < sp.size() && sp[k].second <= start[q]) ++k;
+        for (size_t x = k; x < sp.size() && sp[x].first < start[q + 1]; ++x) {
+            const int32_t a = std::max(sp[x].first, start[q]), b = std::min(sp[x].second, start[q + 1]);
+            add(q * P + (a - start[q]), q * P + (b - start[q]));
+        }
+        if (q + 1 < np) add(q * P + s.fill[q], (q + 1) * P);
+    }
+    for (auto& ab : r) {
+        a_out->push_back(ab.first);
+        b_out->push_back(ab.second);
+    }
     return kOk;
 }
 

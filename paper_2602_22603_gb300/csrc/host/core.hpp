@@ -12,6 +12,16 @@
 //     replaced by a fresh page (increasing logical order), others are
 //     compacted in place; pages past the new end lose a reference;
 //   * release: every page loses a reference.
+//
+// Page fills: each page of a sequence holds `fill` rows (1 .. P) in its
+// first slots; the logical rows are the pages' filled slots in order.  All
+// pages are full but the last (the dense layout, logical j in slot j % P of
+// pages[j / P]) unless a ragged eviction left partial pages: it packs only
+// the runs of pages the spans touch (windows), each from slot 0 of its first
+// page, drops the window pages it no longer needs by remapping, and leaves
+// every other page as it was.  Kernels address rows in SLOT SPACE, position
+// q * P + slot for slot `slot` of page index q, which keeps the logical
+// order; a sequence's slot-space end is (pages - 1) * P + last fill.
 #pragma once
 
 #include <stdint.h>
@@ -78,6 +88,7 @@ struct Seq {
     uint32_t gen = 0;
     int32_t n = 0;
     std::vector<int32_t> pages;
+    std::vector<int32_t> fill;  // rows held by each page, 1 .. P (sum = n)
     uint64_t version = 0;  // bumped by every change of n or pages
     // position of the next token: tokens ever appended (a fork starts from its
     // parent's); eviction does not lower it, since kept keys keep the rotary
@@ -86,8 +97,17 @@ struct Seq {
     void* last_stream = nullptr;
 };
 
+// Slot-space end of a sequence: (pages - 1) * P + last fill (0 when empty).
+inline int32_t slot_end(const Seq& s, int32_t P) {
+    return s.pages.empty() ? 0 : ((int32_t)s.pages.size() - 1) * P + s.fill.back();
+}
+// True when some page other than the last holds fewer than P rows.
+bool has_partial_pages(const Seq& s, int32_t P);
+
 struct AppendPlan {
     int32_t n0 = 0, n_new = 0;
+    int32_t pos0 = 0;        // slot-space position of the first new row
+    int32_t last_fill0 = 0;  // fill of the last page before (0: no page)
     bool cow = false;
     int32_t cow_old = -1, cow_new = -1, cow_rows = 0;
     int32_t first_page_index = 0;  // logical index of the page holding n0
@@ -95,18 +115,29 @@ struct AppendPlan {
     std::vector<int32_t> taken;    // pages newly taken (cow page first)
 };
 
+// One contiguous piece of an eviction's row movement: n rows from slots
+// src_slot .. of page src_page to slots dst_slot .. of page dst_page, or n
+// zero rows when src_page is -1.
+struct EvictMove {
+    int32_t dst_page, dst_slot, src_page, src_slot, n;
+};
+
 struct EvictPlan {
     int32_t n_old = 0, n_new = 0;
-    int32_t first_row = 0;             // first destination row that may change
-    std::vector<int32_t> old_pages;    // page table before
-    std::vector<int32_t> new_pages;    // page table after (length ceil(n_new / P))
-    std::vector<int32_t> run_dst;      // kept runs: destination start (increasing)
-    std::vector<int32_t> run_src;      //            source start
-    std::vector<int32_t> run_len;      //            length (> 0)
+    bool ragged = false;
+    std::vector<int32_t> old_pages, old_fill;   // page table before
+    std::vector<int32_t> new_pages, new_fill;   // page table after
+    // Row movement in increasing destination (slot-space) order.  Every
+    // source of a move lies at a slot-space position >= its destination's,
+    // inside the same window, so performing the moves in order (each one's
+    // reads before its writes) compacts in place.
+    std::vector<EvictMove> moves;
     std::vector<int32_t> cow_pages;    // fresh pages taken (increasing logical page)
     std::vector<int32_t> freed;        // pages whose count reached zero
-    int64_t moved_rows = 0;            // destination rows that are written
+    int64_t moved_rows = 0;            // rows copied
+    int64_t zeroed_rows = 0;           // unused slots set to zero (ragged windows)
     int32_t evicted = 0;
+    int32_t windows = 0;               // runs of pages packed
 };
 
 class HostCache {
@@ -121,9 +152,10 @@ class HostCache {
     // restores the state if the device work cannot be enqueued.
     int append(int32_t h, int32_t n_new, AppendPlan* plan);
     void undo_append(int32_t h, const AppendPlan& plan);
-    // Validates spans, plans and commits an eviction.
+    // Validates spans, plans and commits an eviction: dense (the kept rows
+    // packed into full pages) or ragged (only the touched windows packed).
     int evict(int32_t h, const int32_t* starts, const int32_t* ends,
-              int32_t n_spans, EvictPlan* plan);
+              int32_t n_spans, EvictPlan* plan, bool ragged = false);
     void undo_evict(int32_t h, const EvictPlan& plan);
     int release(int32_t h, std::vector<int32_t>* freed);
 
@@ -142,14 +174,14 @@ class HostCache {
     int64_t peak_live_ = 0;
 };
 
-// Splits the rows an eviction writes into tiles of at most `tile_rows`
-// rows inside one destination page, in increasing logical order, and each
-// tile into contiguous source pieces (a piece never crosses a kept-run or a
-// source-page boundary).  Every source of a tile lies at a logical position
-// >= the tile's first destination row, so processing tiles in order, each
-// tile's reads before its writes, compacts in place.
-void evict_tiles(const EvictPlan& p, int32_t P, int32_t tile_rows,
-                 std::vector<EvictTile>* tiles, std::vector<EvictPiece>* pieces);
+// Splits an eviction's moves into tiles of at most `tile_rows` contiguous
+// destination rows of one page, in order, and each copy tile into its
+// contiguous source pieces; a tile of zero rows has no pieces.  Every
+// source of a tile lies at a slot-space position >= the tile's first
+// destination row, so processing tiles in order, each tile's reads before
+// its writes, compacts in place.
+void evict_tiles(const EvictPlan& p, int32_t tile_rows, std::vector<EvictTile>* tiles,
+                 std::vector<EvictPiece>* pieces);
 
 // ---- decode planning -------------------------------------------------------
 
@@ -158,10 +190,14 @@ struct DecodePlanHost {
     std::vector<DecodeItem> items;
     std::vector<int32_t> cta_begin;   // n_ctas + 1
     std::vector<int32_t> page_ids;
+    // rows held by each page of page_ids; filled only when some sequence of
+    // the call has a partial page before its last (else every page is full
+    // up to the members' limits)
+    std::vector<int32_t> page_fill;
     // partial entries of (sequence i, KV head h): [comb_off[k], comb_off[k + 1]),
     // k = i * Hkv + h, in item order
     std::vector<int32_t> comb_off;    // n_seqs * Hkv + 1
-    int64_t unique_tokens = 0;        // sum over segments of n_tok (one head, one layer)
+    int64_t unique_tokens = 0;        // distinct rows read (one head, one layer)
     int64_t logical_tokens = 0;       // sum over sequences of n
     int32_t n_ctas = 0;
 };
@@ -199,9 +235,20 @@ struct PrefillPlanHost {
 // bitmaps, and splits each query tile's key range in n_split parts when the
 // query tiles alone would fill fewer than `target_ctas` CTAs.
 // `pages` (may be null) is the sequence's page table; with it the plan also
-// lists the page of every piece of every key tile.
+// lists the page of every piece of every key tile.  Positions are slot-space
+// positions: for a sequence with partial pages, n is its slot-space end and
+// the spans include its unused slots (see prefill_slot_spans).
 int plan_prefill(const Geometry& g, int32_t n, int32_t n_q, const int32_t* starts,
                  const int32_t* ends, int32_t n_spans, int32_t target_ctas,
                  PrefillPlanHost* out, const int32_t* pages = nullptr);
+
+// Slot-space form of a masked prefill over sequence `s`: validates the
+// logical spans against s.n, maps them to slot-space ranges, adds the unused
+// slots of every partial page before the last, and returns the slot-space
+// end.  The last n_q rows must occupy consecutive slots (no partial page
+// among the pages holding them, but the last); otherwise kUnsupported.
+int prefill_slot_spans(const Seq& s, int32_t P, int32_t n_q, const int32_t* starts,
+                       const int32_t* ends, int32_t n_spans, std::vector<int32_t>* a_out,
+                       std::vector<int32_t>* b_out, int32_t* n_slots);
 
 }  // namespace sq

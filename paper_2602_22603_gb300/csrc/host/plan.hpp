@@ -46,12 +46,13 @@ struct DecodeItem {
 // Eviction compaction, planned once per eviction and shared by every
 // (layer, K/V, head) plane: destination tiles (contiguous rows of one page, in
 // increasing logical order) and, per tile, the contiguous source pieces that
-// fill it.
+// fill it.  A tile without pieces writes zeros (the unused slots of a page
+// that a ragged eviction leaves partial).
 struct EvictTile {
     int32_t dst_page;
     int32_t dst_slot;     // first destination slot in the page
     int32_t n_rows;       // rows written (<= tile capacity)
-    int32_t piece_begin;  // pieces [piece_begin, next tile's piece_begin)
+    int32_t piece_begin;  // pieces [piece_begin, next tile's piece_begin); none: zero rows
 };
 
 struct EvictPiece {
@@ -83,8 +84,9 @@ struct PrefillTile {
 // Byte offsets of the serialised decode plan.  `arrive` holds one 32-bit
 // arrival count per (sequence, KV head), zero in the serialised plan; the
 // kernel counts on it and leaves it at zero again.
+// `page_fill` is -1 when the plan carries no page fills.
 struct DecodePlanLayout {
-    int64_t segs, items, cta_begin, page_ids, comb_off, arrive, total;
+    int64_t segs, items, cta_begin, page_ids, comb_off, arrive, page_fill, total;
     int32_t n_segs, n_items, n_ctas, n_page_ids, n_comb_keys, n_comb_ent;
 };
 

@@ -33,6 +33,11 @@
 // memory only after the wait, through L2, which holds whatever the preceding
 // kernel wrote to them.
 //
+// Page fills: after a ragged eviction a page may hold fewer rows than it has
+// slots (its rows first, then zeros or rows once appended).  Stages are in
+// slot space (page index x P + slot); the plan then carries every page's
+// fill, and the rows past a page's fill get no weight.
+//
 // Tensor cores: S = Q K^T and O += P V are m16n8k16 bf16 mma.sync with fp32
 // accumulation; rows = query rows (<= 16), columns = tokens / head dims.  The
 // contraction is tiny (G x d per token) and the kernel is HBM-bound, so the
@@ -323,6 +328,24 @@ __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, ui
         for (int s = item.s0; s < item.s1; ++s) {
             const uint32_t full = smem_addr(&bars[slot]);
             const uint32_t empty = smem_addr(&bars[C::kStages + slot]);
+            // Pages a ragged eviction left partial: bit r of vm says whether
+            // row r of this warp's 16 holds a row of its page (read before
+            // the wait, off the critical path).  The unused slots hold zeros
+            // or rows once appended, so only their scores are masked.
+            uint32_t vm = 0xffffu;
+            if (a.page_fill) {
+                const int t0 = s * kStageTokens + warp * 16;  // segment slot position
+                const int P = a.P;
+                const int pq0 = t0 / P, pq1 = (t0 + 15) / P;  // pq1 = pq0 + 1 only for P = 8
+                const int f0 = pq0 < seg->n_pages ? __ldg(&a.page_fill[seg->page_off + pq0]) : 0;
+                const int f1 = pq1 < seg->n_pages ? __ldg(&a.page_fill[seg->page_off + pq1]) : 0;
+                vm = 0u;
+#pragma unroll
+                for (int r = 0; r < 16; ++r) {
+                    const int t = t0 + r;
+                    vm |= (uint32_t)(t % P < (t / P == pq0 ? f0 : f1)) << r;
+                }
+            }
             if (!dead) {
                 const bool ok = mbar_wait(full, phase, abort_flag);
                 if (!__all_sync(0xffffffffu, ok)) {
@@ -363,8 +386,9 @@ __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, ui
 #pragma unroll
                     for (int e = 0; e < 2; ++e) {
                         const int tk = tbase + nt * 8 + tig * 2 + e;
-                        x[nt][e] = tk < lim0 ? sc[nt][e] * a.scale_log2 : -INFINITY;
-                        x[nt][2 + e] = tk < lim1 ? sc[nt][2 + e] * a.scale_log2 : -INFINITY;
+                        const bool rv = (vm >> (nt * 8 + tig * 2 + e)) & 1u;
+                        x[nt][e] = tk < lim0 && rv ? sc[nt][e] * a.scale_log2 : -INFINITY;
+                        x[nt][2 + e] = tk < lim1 && rv ? sc[nt][2 + e] * a.scale_log2 : -INFINITY;
                         mx0 = fmaxf(mx0, x[nt][e]);
                         mx1 = fmaxf(mx1, x[nt][2 + e]);
                     }

@@ -109,15 +109,27 @@ __global__ void __launch_bounds__(256) sq_cow_copy_kernel(const CowArgs a) {
 // and (b) the loads issued ahead for later tiles read positions past every
 // row written so far.  Copy-on-write destination pages are fresh pages that
 // hold no source row.  No inter-CTA wait is needed.
+//
+// A tile without pieces writes zeros: the unused slots of a page that a
+// ragged eviction leaves partial.  Its store reads a zero tile that the
+// CTA's warp clears once; it writes only past the rows its window kept, and
+// later tiles read only later windows' pages.
 __global__ void __launch_bounds__(32) sq_evict_compact_kernel(const EvictArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    if (threadIdx.x != 0) return;
     constexpr int S = kEvictStages;
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
     const uint32_t row_bytes = (uint32_t)a.D * 2u;
     const uint32_t tile_bytes = (uint32_t)a.tile_rows * row_bytes;
-    uint64_t* full = reinterpret_cast<uint64_t*>(smem + S * tile_bytes);
+    uint8_t* zero = smem + S * tile_bytes;   // the zero tile (a.zero_tiles only)
+    if (a.zero_tiles) {
+        for (uint32_t i = threadIdx.x * 16u; i < tile_bytes; i += blockDim.x * 16u)
+            *reinterpret_cast<uint4*>(zero + i) = make_uint4(0, 0, 0, 0);
+        fence_proxy_async_smem();  // the bulk stores read it through the async proxy
+        __syncwarp();
+    }
+    if (threadIdx.x != 0) return;
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + (S + (a.zero_tiles ? 1 : 0)) * tile_bytes);
     const int plane = blockIdx.x;
     const int head = plane % a.Hkv;
     const int kv = (plane / a.Hkv) % 2;
@@ -173,10 +185,13 @@ __global__ void __launch_bounds__(32) sq_evict_compact_kernel(const EvictArgs a)
         }
         fence_proxy_async_smem();
         const EvictTile tl = a.tiles[t];
+        const int pe = t + 1 < T ? __ldg(&a.tiles[t + 1].piece_begin) : a.n_pieces;
+        const bool zeros = tl.piece_begin == pe;  // no pieces: a tile of zeros
         if ((uint64_t)tl.dst_page < (uint64_t)a.num_pages && tl.dst_slot >= 0 && tl.n_rows > 0 &&
-            tl.n_rows <= a.tile_rows && tl.dst_slot + tl.n_rows <= a.P) {
+            tl.n_rows <= a.tile_rows && tl.dst_slot + tl.n_rows <= a.P && (!zeros || a.zero_tiles)) {
             bulk_store(base + tl.dst_page * page_stride + (int64_t)tl.dst_slot * row_bytes,
-                       smem_addr(smem + slot * tile_bytes), (uint32_t)tl.n_rows * row_bytes);
+                       smem_addr(zeros ? zero : smem + slot * tile_bytes),
+                       (uint32_t)tl.n_rows * row_bytes);
         } else {
             set_error(a.err, kErrBounds);
         }
@@ -227,8 +242,8 @@ cudaError_t launch_cow_copy(const CowArgs& a, int num_sms, cudaStream_t st) {
     return cudaGetLastError();
 }
 
-int evict_smem_bytes(int tile_rows, int D) {
-    return kEvictStages * tile_rows * D * 2 + kEvictStages * 8 + 128;
+int evict_smem_bytes(int tile_rows, int D, bool zero_tiles) {
+    return (kEvictStages + (zero_tiles ? 1 : 0)) * tile_rows * D * 2 + kEvictStages * 8 + 128;
 }
 
 int evict_ctas_per_sm(int tile_rows, int D) {
@@ -244,13 +259,14 @@ int evict_ctas_per_sm(int tile_rows, int D) {
 cudaError_t evict_prepare() {
     return cudaFuncSetAttribute(sq_evict_compact_kernel,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                evict_smem_bytes(kStageTokens, 128));
+                                evict_smem_bytes(kStageTokens, 128, true));
 }
 
 cudaError_t launch_evict(const EvictArgs& a, cudaStream_t st) {
     const int blocks = a.L * 2 * a.Hkv;
     if (blocks == 0 || a.n_tiles == 0) return cudaSuccess;
-    sq_evict_compact_kernel<<<blocks, 32, evict_smem_bytes(a.tile_rows, a.D), st>>>(a);
+    sq_evict_compact_kernel<<<blocks, 32, evict_smem_bytes(a.tile_rows, a.D, a.zero_tiles != 0),
+                              st>>>(a);
     return cudaGetLastError();
 }
 

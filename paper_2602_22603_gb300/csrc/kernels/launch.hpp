@@ -16,6 +16,9 @@ struct DecodeArgs {
     const DecodeItem* items;
     const int32_t* cta_begin;
     const int32_t* page_ids;
+    // rows held by each page of page_ids, or null when every page of the
+    // call is full up to the members' limits (no sequence with partial pages)
+    const int32_t* page_fill;
     const int32_t* comb_off;    // [n_seqs * Hkv + 1] partial entries of each (sequence, KV head)
     unsigned int* arrive;       // [n_seqs * Hkv] arrival counts, zero between calls
     const __nv_bfloat16* q;     // [n_seqs][Hq][D]
@@ -129,6 +132,7 @@ struct EvictArgs {
     const EvictPiece* pieces;   // their contiguous source pieces
     int32_t n_tiles, n_pieces;
     int32_t tile_rows;          // rows a tile holds at most
+    int32_t zero_tiles;         // 1: some tiles (those without pieces) write zeros
     int* err;
 };
 
@@ -136,8 +140,9 @@ cudaError_t launch_append(const AppendArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_append_batch(const AppendBatchArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_cow_copy(const CowArgs& a, int num_sms, cudaStream_t st);
 constexpr int kEvictStages = 6;
-// Shared memory of one eviction CTA for a tile size.
-int evict_smem_bytes(int tile_rows, int D);
+// Shared memory of one eviction CTA for a tile size (plus one zero tile when
+// the plan zeroes rows).
+int evict_smem_bytes(int tile_rows, int D, bool zero_tiles = false);
 // Resident eviction CTAs per SM for a tile size.
 int evict_ctas_per_sm(int tile_rows, int D);
 cudaError_t evict_prepare();  // raises the dynamic shared-memory limit once

@@ -12,6 +12,7 @@ import torch
 import paper_2602_22603_gb300 as sq
 from oracle import cache_model as ocm
 from synthetic import Bank, bf16_bits, sub_seed
+from tests.gpu_harness import row_slots
 
 
 class BankPair:
@@ -62,9 +63,12 @@ class BankPair:
             self.append(h, k)
             n -= k
 
-    def evict(self, h, spans, stream=None):
-        r = self.oracle.evict(self.o[h], spans)
-        self.cache.evict_spans(h, spans, stream)
+    def evict(self, h, spans, stream=None, ragged=False):
+        r = self.oracle.evict(self.o[h], spans, mode="ragged" if ragged else "dense")
+        if ragged:
+            self.cache.evict_spans_ragged(h, spans, stream)
+        else:
+            self.cache.evict_spans(h, spans, stream)
         return r
 
     def release(self, h, stream=None):
@@ -110,6 +114,7 @@ class BankPair:
     def check_tables(self, handles: Sequence[int]):
         for h in handles:
             assert self.cache.page_table(h) == self.oracle.page_table(self.o[h])
+            assert self.cache.page_fills(h) == self.oracle.page_fills(self.o[h])
             assert self.cache.seq_info(h)[0] == self.oracle.n_tokens(self.o[h])
         assert self.cache.free_pages() == self.oracle.free_count()
 
@@ -121,11 +126,9 @@ class BankPair:
             planes = [(kv, head) for kv in (0, 1) for head in range(self.Hkv)]
         torch.cuda.synchronize()
         pool = self.cache.pool_view()
-        pt = torch.tensor(self.cache.page_table(h), dtype=torch.long, device="cuda")
-        n = self.cache.seq_info(h)[0]
-        j = torch.arange(n, device="cuda")
+        page, slot = row_slots(self.cache, h)
         K, V = self.rows(h, layer)
         for kv, head in planes:
-            got = bf16_bits(pool[layer, pt[j // self.P], kv, head, j % self.P, :].cpu())
+            got = bf16_bits(pool[layer, page, kv, head, slot, :].cpu())
             exp = (K if kv == 0 else V)[:, head, :]
             assert np.array_equal(got, exp), (layer, kv, head)

@@ -53,11 +53,11 @@ class Pair:
     """One library cache and one oracle cache, kept in lockstep."""
 
     def __init__(self, L, Hq, Hkv, D, P, num_pages, max_seqs=64, decode_ctas=0, seed=0,
-                 k_scale=1.0):
+                 k_scale=1.0, physical=False):
         self.L, self.Hq, self.Hkv, self.D, self.P = L, Hq, Hkv, D, P
         self.cache = sq.Cache(L, Hq, Hkv, D, P, num_pages, max_seqs=max_seqs,
                               decode_ctas=decode_ctas)
-        self.oracle = ocm.OracleCache(num_pages, P)
+        self.oracle = ocm.OracleCache(num_pages, P, physical=physical)
         self.store = RowStore(L, Hkv, D)
         self.o: Dict[int, int] = {}     # library handle -> oracle sequence id
         self.seed = seed
@@ -82,6 +82,8 @@ class Pair:
         return h
 
     def append(self, h: int, n: int, stream=None):
+        if n == 0:
+            return None
         s = self._next_seed()
         k = bf16_normal((self.L, n, self.Hkv, self.D), s, scale=self.k_scale)
         v = bf16_normal((self.L, n, self.Hkv, self.D), s + 50000)
@@ -104,9 +106,12 @@ class Pair:
         self.cache.append_kv_batch(list(hs), kd, vd, stream)
         return kd, vd
 
-    def evict(self, h: int, spans, stream=None):
-        r = self.oracle.evict(self.o[h], spans)
-        self.cache.evict_spans(h, spans, stream)
+    def evict(self, h: int, spans, stream=None, ragged=False):
+        r = self.oracle.evict(self.o[h], spans, mode="ragged" if ragged else "dense")
+        if ragged:
+            self.cache.evict_spans_ragged(h, spans, stream)
+        else:
+            self.cache.evict_spans(h, spans, stream)
         return r
 
     def release(self, h: int, stream=None):
@@ -117,6 +122,7 @@ class Pair:
     def check_tables(self):
         for h, o in self.o.items():
             assert self.cache.page_table(h) == self.oracle.page_table(o)
+            assert self.cache.page_fills(h) == self.oracle.page_fills(o)
             assert self.cache.seq_info(h)[0] == self.oracle.n_tokens(o)
         assert self.cache.free_pages() == self.oracle.free_count()
         for p in range(self.oracle.num_pages):
@@ -127,10 +133,7 @@ class Pair:
         the library's page table, equals the row the oracle says is there."""
         torch.cuda.synchronize()
         pool = self.cache.pool_view()
-        pt = torch.tensor(self.cache.page_table(h), dtype=torch.long, device="cuda")
-        n = self.cache.seq_info(h)[0]
-        j = torch.arange(n, device="cuda")
-        page, slot = pt[j // self.P], j % self.P
+        page, slot = row_slots(self.cache, h)
         toks = self.oracle.tokens(self.o[h])
         for layer in (layers if layers is not None else range(self.L)):
             for kv in (0, 1):
@@ -139,6 +142,17 @@ class Pair:
                 ek, ev = self.store.rows(toks, layer)
                 exp = ek if kv == 0 else ev
                 assert np.array_equal(got, exp), f"layer {layer} kv {kv}"
+
+    def check_zero_slots(self):
+        """Every slot the (physical) oracle says was set to zero holds zero
+        bits in the device pool, in every layer, K and V, and head."""
+        torch.cuda.synchronize()
+        pool = self.cache.pool_view()
+        for p, slots in self.oracle.phys.items():
+            z = [t for t, x in enumerate(slots) if x == ocm.ZERO]
+            if z:
+                got = pool[:, p, :, :, z, :]
+                assert not torch.any(got.view(torch.int16) != 0).item(), (p, z)
 
     def decode(self, seqs: Sequence[int], layer: int, sm_scale: float, q: torch.Tensor,
                out_dtype=sq.SQ_OUT_F32, stream=None) -> torch.Tensor:
@@ -168,6 +182,17 @@ class Pair:
             k, v = self.store.rows(self.oracle.tokens(self.o[h]), layer)
             res.append(oatt.decode(qb[i], k, v, sm_scale))
         return np.stack(res)
+
+
+def row_slots(cache, h):
+    """(page, slot) of every row of sequence h in logical order, as CUDA
+    long tensors, through the library's page table and page fills."""
+    pt = cache.page_table(h)
+    fills = cache.page_fills(h)
+    page = np.repeat(np.asarray(pt, dtype=np.int64), fills)
+    slot = np.concatenate([np.arange(f, dtype=np.int64) for f in fills]) if fills else \
+        np.zeros(0, dtype=np.int64)
+    return torch.from_numpy(page).cuda(), torch.from_numpy(slot).cuda()
 
 
 def assert_close(got: torch.Tensor, exp: np.ndarray, max_abs=MAX_ABS, mean_abs=MEAN_ABS):

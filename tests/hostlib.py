@@ -31,9 +31,12 @@ def lib():
         L.sqh_seq_new.argtypes = [P, I32P]
         L.sqh_fork.argtypes = [P, I32, I32P]
         L.sqh_append.argtypes = [P, I32, I32]
-        L.sqh_evict.argtypes = [P, I32, I32P, I32, I64P]
+        L.sqh_evict.argtypes = [P, I32, I32P, I32, I32, I64P]
         L.sqh_release.argtypes = [P, I32]
-        L.sqh_evict_tiles.argtypes = [P, I32, I32P, I32, I32, I32P, I32, I32P, I32, I32P, I32P]
+        L.sqh_evict_tiles.argtypes = [P, I32, I32P, I32, I32, I32, I32P, I32, I32P, I32, I32P,
+                                      I32P]
+        L.sqh_page_fill.argtypes = [P, I32, I32P, I32, I32P]
+        L.sqh_prefill_slot_spans.argtypes = [P, I32, I32, I32P, I32, I32P, I32, I32P, I32P]
         L.sqh_seq_info.argtypes = [P, I32, I32P, I32P]
         L.sqh_next_pos.argtypes = [P, I32]
         L.sqh_next_pos.restype = ctypes.c_int64
@@ -89,20 +92,20 @@ class HostCache:
     def append(self, h, n):
         return lib().sqh_append(self.h, h, n)
 
-    def evict(self, h, spans):
+    def evict(self, h, spans, ragged=False):
         arr = (ctypes.c_int32 * max(2, 2 * len(spans)))(*[int(x) for ab in spans for x in ab])
-        st = (ctypes.c_int64 * 5)()
-        rc = lib().sqh_evict(self.h, h, arr, len(spans), st)
+        st = (ctypes.c_int64 * 6)()
+        rc = lib().sqh_evict(self.h, h, arr, len(spans), int(ragged), st)
         return rc, {"moved_rows": st[0], "cow_pages": st[1], "freed": st[2],
-                    "first_row": st[3], "n_runs": st[4]}
+                    "zeroed_rows": st[3], "windows": st[4], "n_moves": st[5]}
 
-    def evict_tiles(self, h, spans, tile_rows, cap=100000):
+    def evict_tiles(self, h, spans, tile_rows, ragged=False, cap=100000):
         arr = (ctypes.c_int32 * max(2, 2 * len(spans)))(*[int(x) for ab in spans for x in ab])
         tiles = np.zeros(4 * cap, dtype=np.int32)
         pieces = np.zeros(4 * cap, dtype=np.int32)
         nt, npc = ctypes.c_int32(), ctypes.c_int32()
         i32p = ctypes.POINTER(ctypes.c_int32)
-        rc = lib().sqh_evict_tiles(self.h, h, arr, len(spans), tile_rows,
+        rc = lib().sqh_evict_tiles(self.h, h, arr, len(spans), int(ragged), tile_rows,
                                    tiles.ctypes.data_as(i32p), cap, pieces.ctypes.data_as(i32p),
                                    cap, ctypes.byref(nt), ctypes.byref(npc))
         if rc != 0:
@@ -128,6 +131,25 @@ class HostCache:
         assert lib().sqh_page_table(self.h, h, buf, npg, ctypes.byref(m)) == 0
         return list(buf[:m.value])
 
+    def page_fill(self, h):
+        rc, n, npg = self.info(h)
+        assert rc == 0
+        buf = (ctypes.c_int32 * max(1, npg))()
+        m = ctypes.c_int32()
+        assert lib().sqh_page_fill(self.h, h, buf, npg, ctypes.byref(m)) == 0
+        return list(buf[:m.value])
+
+    def prefill_slot_spans(self, h, n_q, spans, cap=1 << 16):
+        """(rc, slot-space spans, slot-space end) of a masked prefill."""
+        arr = (ctypes.c_int32 * max(2, 2 * len(spans)))(*[int(x) for ab in spans for x in ab])
+        out = (ctypes.c_int32 * (2 * cap))()
+        m, ns = ctypes.c_int32(), ctypes.c_int32()
+        rc = lib().sqh_prefill_slot_spans(self.h, h, n_q, arr, len(spans), out, cap,
+                                          ctypes.byref(m), ctypes.byref(ns))
+        if rc != 0:
+            return rc, None, None
+        return 0, [(out[2 * i], out[2 * i + 1]) for i in range(m.value)], ns.value
+
     def refcount(self, p):
         return lib().sqh_refcount(self.h, p)
 
@@ -139,7 +161,7 @@ class HostCache:
 
     def plan_decode(self, handles, n_ctas):
         arr = (ctypes.c_int32 * len(handles))(*handles)
-        lay = (ctypes.c_int64 * 16)()
+        lay = (ctypes.c_int64 * 17)()
         rc = lib().sqh_plan_decode(self.h, arr, len(handles), n_ctas, lay, None, 0)
         if rc != 0:
             return rc, None
@@ -187,5 +209,6 @@ class HostCache:
             "comb_off": comb_off,
             "comb_ent": comb_ent,
             "unique_tokens": L[13], "logical_tokens": L[14],
+            "page_fill": arr_at(L[16], n_pid).tolist() if L[16] >= 0 else None,
         }
         return 0, plan

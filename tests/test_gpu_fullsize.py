@@ -221,3 +221,50 @@ def test_aux_trigger_prefill_128k_full_size():
             assert np.abs(lse.cpu().numpy().astype(np.float64) - exp_lse).max() <= 1e-2
     finally:
         bp.close()
+
+
+def test_serving_128k_ragged_eviction_full_size():
+    """The serving workload's requests at full length (8 x 131,072 tokens,
+    32q/8kv, d128, P64; two layers) evicted by ragged packing with the
+    bench's spans (20-65% of each request in 10-40 spans): page tables and
+    fills bit-exact, every plane of both layers of every request bit-exact,
+    a few P rows copied per span, and decode of all 16 sequences (each request
+    re-forked, Algorithm 1's next trigger) at both layers against the oracle."""
+    L, Hq, Hkv, D, P = 2, 32, 8, 128, 64
+    R, ctx = 8, 131072
+    bp = BankPair(L, Hq, Hkv, D, P, num_pages=R * (ctx // P + 4) + R * 4 + 64, seed=6)
+    try:
+        scale = 1.0 / math.sqrt(D)
+        mains = []
+        for r in range(R):
+            m = bp.seq_new()
+            bp.fill(m, ctx, 8192)
+            mains.append(m)
+        moved, spans_total = 0, 0
+        for r, m in enumerate(mains):
+            n = bp.cache.seq_info(m)[0]
+            spans = request_spans(0, r, n, P)
+            res = bp.evict(m, spans, ragged=True)
+            assert res["moved_rows"] <= 2 * P * len(spans)
+            moved += res["moved_rows"]
+            spans_total += len(spans)
+        st = bp.cache.stats()
+        assert st["evict_moved_rows"] == moved
+        bp.check_tables(mains)
+        for m in mains:
+            assert any(f < P for f in bp.cache.page_fills(m)[:-1])
+            for layer in range(L):
+                bp.check_planes(m, layer)
+        auxs = []
+        for m in mains:
+            a = bp.fork(m)
+            bp.append(a, 8)
+            auxs.append(a)
+        seqs = [x for pair in zip(mains, auxs) for x in pair]
+        for h in seqs:
+            bp.append(h, 1)
+        bp.check_tables(seqs)
+        for layer in range(L):
+            _decode_and_check(bp, seqs, layer, scale, 700 + layer, None)
+    finally:
+        bp.close()

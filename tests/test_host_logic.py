@@ -31,6 +31,7 @@ def random_spans(rng, n, k):
 def compare_state(hc, oc, pairs):
     for h, o in pairs.items():
         assert hc.page_table(h) == oc.page_table(o)
+        assert hc.page_fill(h) == oc.page_fills(o)
         assert hc.info(h)[1] == oc.n_tokens(o)
     assert hc.free_count() == oc.free_count()
     for p in range(oc.num_pages):
@@ -73,12 +74,16 @@ def test_page_tables_match_oracle_bit_exact(seed):
             spans = random_spans(rng, oc.n_tokens(o), rng.choice([1, 2, 4, 9]))
             if rng.random() < 0.1 and spans:
                 spans.append((spans[0][0], spans[0][0] + 1))  # overlap -> rejected
-            rc, st = hc.evict(h, spans)
-            orc, ost = oracle_call(oc.evict, o, spans)
+            ragged = rng.random() < 0.5
+            rc, st = hc.evict(h, spans, ragged)
+            orc, ost = oracle_call(oc.evict, o, spans, "ragged" if ragged else "dense")
             assert rc == orc, (spans, rc, orc)
             if rc == 0 and spans:
                 assert st["moved_rows"] == ost["moved_rows"]
                 assert st["cow_pages"] == ost["cow_pages"]
+                if ragged:
+                    assert st["zeroed_rows"] == ost["zeroed_rows"]
+                    assert st["windows"] == ost["windows"]
         else:
             assert hc.release(h) == 0
             oc.release(o)
@@ -120,9 +125,21 @@ def _check_plan(hc, handles, plan, n_ctas, G):
         assert 1 <= s["n_grp"] <= 16 // G
         assert max(s["grp_lim"]) == s["n_tok"] and min(s["grp_lim"]) > 0
         assert s["n_tok"] <= s["n_pages"] * P
-    # every (sequence, head) covers its tokens exactly once, through its own pages
+    # every (sequence, head) covers its slots exactly once, through its own
+    # pages (slot space: page index x P + slot; rows = filled slots)
     tables = [hc.page_table(h) for h in handles]
-    ns = [hc.info(h)[1] for h in handles]
+    fills = [hc.page_fill(h) for h in handles]
+    ends = [(len(f) - 1) * P + f[-1] for f in fills]
+    ragged = any(x < P for f in fills for x in f[:-1])
+    assert (plan["page_fill"] is not None) == ragged
+    if ragged:
+        for s in segs:
+            pids = plan["page_ids"][s["page_off"]:s["page_off"] + s["n_pages"]]
+            pf = plan["page_fill"][s["page_off"]:s["page_off"] + s["n_pages"]]
+            for j in range(s["n_grp"]):
+                i = s["grp_seq"][j]
+                q0 = tables[i].index(pids[0])
+                assert fills[i][q0:q0 + s["n_pages"]] == pf
     for i in range(len(handles)):
         for head in range(Hkv):
             key = i * Hkv + head
@@ -146,7 +163,7 @@ def _check_plan(hc, handles, plan, n_ctas, G):
             for a, b in covered:
                 assert a == pos
                 pos = b
-            assert pos == ns[i]
+            assert pos == ends[i]
 
 
 @pytest.mark.parametrize("seed", range(10))
@@ -171,7 +188,7 @@ def test_decode_plan_covers_every_token_once(seed):
         assert hc.append(h, rng.randint(0, 2 * P)) == 0
         if rng.random() < 0.5:
             n = hc.info(h)[1]
-            hc.evict(h, random_spans(rng, n, 3))
+            hc.evict(h, random_spans(rng, n, 3), ragged=rng.random() < 0.5)
     rng.shuffle(seqs)
     for n_ctas in (1, 3, 152, 304, 5000):
         rc, plan = hc.plan_decode(seqs, n_ctas)
@@ -289,19 +306,29 @@ def test_evict_tiles_compact_in_place(seed):
         k = rng.randint(0, P)
         hc.append(m, k)
         oc.append(om, k)
+    # a first ragged eviction leaves partial pages for the one under test
+    if rng.random() < 0.5:
+        pre = random_spans(rng, oc.n_tokens(om), 4)
+        assert hc.evict(m, pre, ragged=True)[0] == 0
+        oc.evict(om, pre, mode="ragged")
+    ragged = rng.random() < 0.5
     n = oc.n_tokens(om)
     spans = random_spans(rng, n, rng.choice([1, 3, 8, 20]))
     # physical state before, as {page: [token ids]}
     phys = {p: list(v) for p, v in oc.phys.items()}
-    rc, tiles, pieces = hc.evict_tiles(m, spans, tile_rows)
-    oc.evict(om, spans)
+    rc, tiles, pieces = hc.evict_tiles(m, spans, tile_rows, ragged)
+    oc.evict(om, spans, mode="ragged" if ragged else "dense")
     assert rc == 0
     written = set()
     for t in range(len(tiles)):
         dpage, dslot, nrows, pb = (int(x) for x in tiles[t])
         pe = int(tiles[t + 1][3]) if t + 1 < len(tiles) else len(pieces)
         assert 0 < nrows <= tile_rows and dslot + nrows <= P
-        buf = [None] * nrows
+        if pe == pb:                      # a tile of zeros
+            assert ragged
+            buf = [ocm.ZERO] * nrows
+        else:
+            buf = [None] * nrows
         for k in range(pb, pe):
             spage, sslot, pn, drow = (int(x) for x in pieces[k])
             assert 0 < pn and sslot + pn <= P and drow + pn <= nrows
@@ -312,13 +339,21 @@ def test_evict_tiles_compact_in_place(seed):
         for i in range(nrows):
             phys.setdefault(dpage, [-1] * P)[dslot + i] = buf[i]
             written.add((dpage, dslot + i))
-    pt = hc.page_table(m)
-    assert pt == oc.page_table(om)
-    got = [phys[pt[j // P]][j % P] for j in range(oc.n_tokens(om))]
-    assert got == oc.tokens(om)
+
+    def read(h):
+        rows = []
+        for pg, f in zip(hc.page_table(h), hc.page_fill(h)):
+            rows.extend(phys[pg][:f])
+        return rows
+
+    assert hc.page_table(m) == oc.page_table(om)
+    assert hc.page_fill(m) == oc.page_fills(om)
+    assert read(m) == oc.tokens(om)
+    # every slot the oracle holds, unused ones included, as the tiles left it
+    for pg in hc.page_table(m):
+        assert phys[pg] == oc.phys[pg], pg
     for a, oa in forks:
-        apt = hc.page_table(a)
-        assert [phys[apt[j // P]][j % P] for j in range(oc.n_tokens(oa))] == oc.tokens(oa)
+        assert read(a) == oc.tokens(oa)
 
 
 # ---------------------------------------------------------------------------
@@ -425,3 +460,51 @@ def test_next_position_counts_appends_not_evictions():
     assert hc.release(a) == 0
     rc, b = hc.seq_new()                         # a fresh handle starts at 0
     assert rc == 0 and hc.next_pos(b) == 0
+
+
+@pytest.mark.parametrize("seed", range(10))
+def test_prefill_slot_spans_on_partial_pages(seed):
+    """A masked prefill over a sequence with partial pages runs in slot space:
+    the masked slots are exactly the slots of the spans' rows plus the unused
+    slots of every page but the last, the end is (pages - 1) x P + last fill,
+    and queries that a partial page would split are refused."""
+    rng = random.Random(900 + seed)
+    P = rng.choice([8, 16, 64])
+    hc = HostCache(1, 8, 2, 64, P, 3000)
+    oc = ocm.OracleCache(3000, P)
+    rc, m = hc.seq_new()
+    om = oc.seq_new()
+    n0 = rng.randint(4 * P, 30 * P)
+    hc.append(m, n0)
+    oc.append(om, n0)
+    pre = random_spans(rng, n0, rng.choice([1, 3, 6]))
+    assert hc.evict(m, pre, ragged=True)[0] == 0
+    oc.evict(om, pre, mode="ragged")
+    tail = rng.randint(1, 3 * P)
+    hc.append(m, tail)
+    oc.append(om, tail)
+    n = oc.n_tokens(om)
+    fills = oc.page_fills(om)
+    slot_of = [q * P + t for q, f in enumerate(fills) for t in range(f)]
+    end = (len(fills) - 1) * P + fills[-1]
+    spans = random_spans(rng, n - tail, rng.choice([0, 1, 4]))
+    for n_q in (1, tail, min(n, tail + rng.randint(1, 4 * P)), n):
+        rc, sl, n_slots = hc.prefill_slot_spans(m, n_q, spans)
+        contiguous = slot_of[n - n_q] == end - n_q
+        if not contiguous:
+            assert rc == -8            # unsupported
+            continue
+        assert rc == 0 and n_slots == end
+        masked = set()
+        for a, b in spans:
+            masked.update(slot_of[j] for j in range(a, b))
+        for q, f in enumerate(fills[:-1]):
+            masked.update(range(q * P + f, (q + 1) * P))
+        got = set()
+        prev = -1
+        for a, b in sl:
+            assert prev < a < b        # sorted, disjoint, not touching (merged)
+            prev = b
+            got.update(range(a, b))
+        assert got == masked
+    assert hc.prefill_slot_spans(m, tail, [(0, n + 1)])[0] == -1   # bad span
