@@ -61,6 +61,10 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--ragged", action="store_true",
+                    help="trace: evict with sq_evict_spans_ragged")
+    ap.add_argument("--no-sub", action="store_true",
+                    help="serving-128k at one GPU: skip the other workloads' sub-records")
     return ap.parse_args()
 
 
@@ -288,13 +292,17 @@ def run_sq(args, world, rank, local):
     offs = bank.offsets(sum(n_chunks) * 2, chunk_elems, sub_seed(seed, 2))
     first_off = [2 * sum(n_chunks[:r]) for r in range(R)]
     mains, auxs = [], []
-    for r in range(R):
+
+    def build_request(r):
         m = cache.seq_new()
         for c in range(n_chunks[r]):
             i = first_off[r] + 2 * c
             cache.append_kv(m, chunk, bank.view(offs[i], (L, chunk, Hkv, D)),
                             bank.view(offs[i + 1], (L, chunk, Hkv, D)))
-        mains.append(m)
+        return m
+
+    for r in range(R):
+        mains.append(build_request(r))
     tok_elems = L * Hkv * D
     small = bank.offsets(8192, 2 * 8 * tok_elems, sub_seed(seed, 3))
     small_i = [0]
@@ -488,7 +496,8 @@ def run_sq(args, world, rank, local):
         # input bank keep the GPU busy while the first is planned), and the
         # events between calls give each call's GPU time: copy-on-write
         # copies and the compaction kernel.
-        span_list = [spec["spans"](seed, r, cache.seq_info(m)[0], P) for r, m in enumerate(mains)]
+        pre_lengths = [cache.seq_info(m)[0] for m in mains]
+        span_list = [spec["spans"](seed, r, pre_lengths[r], P) for r in range(len(mains))]
         evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(mains) + 1)]
         b = []
         for _ in range(4):
@@ -537,6 +546,70 @@ def run_sq(args, world, rank, local):
         }
         st = cache.stats()
         res["peak_live_pages"] = st["peak_live_pages"]
+
+        # ---- ragged-page eviction of the same requests and spans ---------------
+        # The requests are rebuilt from the same bank rows to the same length,
+        # the same spans are evicted by ragged packing (only the pages the spans
+        # touch), and decode runs again over the partial pages.
+        lengths = pre_lengths
+        for h in mains + auxs:
+            cache.release(h)
+        torch.cuda.synchronize()
+        mains[:] = [build_request(r) for r in range(R)]
+        extra_rows = bank.offsets(64, 2 * 64 * tok_elems, sub_seed(seed, 7))
+        xi = 0
+        for r, m in enumerate(mains):
+            k_extra = lengths[r] - ctxs[r]
+            while k_extra > 0:
+                c = min(k_extra, 64)
+                o = int(extra_rows[xi % len(extra_rows)])
+                xi += 1
+                cache.append_kv(m, c, bank_ptr + 2 * o, bank_ptr + 2 * (o + 64 * tok_elems))
+                k_extra -= c
+        assert [cache.seq_info(m)[0] for m in mains] == lengths
+        torch.cuda.synchronize()
+        st0 = cache.stats()
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(mains) + 1)]
+        for _ in range(4):
+            sq.sq_probe_read(cache.handle, bank.data, bank.data.numel() * 2, st_h)
+        evs[0].record(stream)
+        for r, m in enumerate(mains):
+            cache.evict_spans_ragged(m, span_list[r])
+            evs[r + 1].record(stream)
+        torch.cuda.synchronize()
+        rg_ms = evs[0].elapsed_time(evs[len(mains)])
+        st1 = cache.stats()
+        assert cache.sync_status() == sq.SQ_OK
+        rg_bytes = st1["evict_bytes"] - st0["evict_bytes"]
+        partial = sum(sum(1 for f in cache.page_fills(m)[:-1] if f < P) for m in mains)
+        fork_all()
+        seqs[:] = [x for pair in zip(mains, auxs) for x in pair]
+        set_seqs()
+        torch.cuda.synchronize()
+        after_rg = timed_decode(K, W)
+        pc = after_rg["attn_ms"] / after_rg["calls"]
+        up = after_rg["unique_bytes"] / after_rg["calls"]
+        res["evict_ragged"] = {
+            "call": "sq_evict_spans_ragged",
+            "ms_total": round(rg_ms, 4),
+            "ms_total_dense": res["evict"]["ms_total"],
+            "moved_rows": int(st1["evict_moved_rows"] - st0["evict_moved_rows"]),
+            "moved_rows_dense": res["evict"]["moved_rows"],
+            "algorithmic_bytes": int(rg_bytes),
+            "gbs": round(rg_bytes / (rg_ms / 1e3) / 1e9, 1),
+            "spans": sum(len(x) for x in span_list),
+            "partial_pages_left": int(partial),
+            "calls": len(mains),
+            "timing": "GPU time of the calls enqueued back to back",
+        }
+        res["after_evict_ragged"] = {
+            "tokens_per_s": round(world * S * K / (max_over_ranks(after_rg["total_ms"], world) / 1e3), 3),
+            "attn_ms_per_call": round(pc, 5),
+            "unique_gb_per_call": round(up / 1e9, 4),
+            "hbm_gbs_unique": round(up / (pc / 1e3) / 1e9, 1),
+            "frac_of_%s_peak" % peak_kind: round(up / (pc / 1e3) / 1e9 / hbm_peak, 4),
+            "unique_gb_per_call_dense": res["after_evict"]["unique_gb_per_call"],
+        }
 
     # ---- CPU oracle on a bounded sample (rank 0, N = 1) ----------------------
     if not args.no_cpu and rank == 0 and world == 1 and args.workload == "serving-128k":
@@ -632,6 +705,27 @@ def run_agent(args, world, rank, local):
     tokens = steps_main + done_aux
     uniq = st1["decode_unique_bytes"] - st0["decode_unique_bytes"]
     calls = st1["decode_calls"] - st0["decode_calls"]
+    # per-call device time: the main thread's steps alone on one stream, the
+    # 32 layer calls of each step back to back between two events
+    Kc = 32
+    evc = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(Kc)]
+    sa_h = int(sa.cuda_stream)
+    c0 = cache.stats()
+    for t in range(Kc):
+        k, v = rows(1)
+        cache.append_kv(main, 1, k, v, sa_h)
+        evc[t][0].record(sa)
+        for layer in range(L):
+            sq.sq_decode_attention(cache.handle, arr[main], layer, qp[main][layer],
+                                   op[main][layer], sq.SQ_OUT_BF16, 1.0, sa_h)
+        evc[t][1].record(sa)
+    torch.cuda.synchronize()
+    c1 = cache.stats()
+    call_ms = sum(a.elapsed_time(b) for a, b in evc) / (Kc * L)
+    call_bytes = (c1["decode_unique_bytes"] - c0["decode_unique_bytes"]) / (c1["decode_calls"] -
+                                                                             c0["decode_calls"])
+    call_gbs = call_bytes / (call_ms / 1e3) / 1e9
     # eviction, after releasing the aux (Algorithm 1 order)
     cache.release(aux, int(sb.cuda_stream))
     n = cache.seq_info(main)[0]
@@ -667,10 +761,52 @@ def run_agent(args, world, rank, local):
         "evict": {"gbs": round(ev_bytes / (ev_ms / 1e3) / 1e9, 1), "ms": round(ev_ms, 4),
                   "algorithmic_bytes": int(ev_bytes),
                   "frac_of_%s_peak" % peak_kind: round(ev_bytes / (ev_ms / 1e3) / 1e9 / hbm_peak, 4)},
+        "roofline": {
+            "bound": "hbm",
+            "kernel": "sq_decode_splitk_kernel, one 32,768-token sequence per call",
+            "achieved": round(call_gbs, 1), "peak": hbm_peak, "peak_kind": peak_kind,
+            "unit": "GB/s", "frac": round(call_gbs / hbm_peak, 4),
+            "algorithmic_bytes_per_launch": int(call_bytes),
+            "ms_per_call": round(call_ms, 5),
+            "timing": "CUDA events around the 32 layer calls of a main-thread step, "
+                      "calls back to back on one stream, 32 steps",
+            "traffic": None,
+        },
         "clocks": clock_rec,
     }
+    if not args.no_cpu and rank == 0 and world == 1:
+        res["cpu_baseline"] = agent_cpu_baseline(kbank, vbank, ko, vo, chunk, n0, L, Hq, Hkv, D,
+                                                 q[main])
     cache.close()
     return res
+
+
+def agent_cpu_baseline(kbank, vbank, ko, vo, chunk, n0, L, Hq, Hkv, D, q):
+    """The oracle as it stands (oracle/attention.c decode, fp64, OpenMP) on
+    the host cores: one main-thread decode step of the agent workload, the
+    query of every layer over the 32,768-token context at all 32 layers;
+    tokens/s = 1 / seconds of the step."""
+    import numpy as np
+
+    from oracle import attention as oatt
+    from synthetic import bf16_bits
+    hk, hv = bf16_bits(kbank.data.cpu()), bf16_bits(vbank.data.cpu())
+    qb = bf16_bits(q.cpu())
+    ce = L * chunk * Hkv * D
+    total = 0.0
+    for layer in range(L):
+        k = np.ascontiguousarray(np.concatenate(
+            [hk[int(o):int(o) + ce].reshape(L, chunk, Hkv, D)[layer] for o in ko]))
+        v = np.ascontiguousarray(np.concatenate(
+            [hv[int(o):int(o) + ce].reshape(L, chunk, Hkv, D)[layer] for o in vo]))
+        t0 = time.perf_counter()
+        oatt.decode(np.ascontiguousarray(qb[layer, 0]), k, v, 1.0)
+        total += time.perf_counter() - t0
+    return {"value": round(1.0 / total, 4), "unit": "tokens/s", "cores": oatt.num_threads(),
+            "kind": "oracle", "cpu_model": cpu_model(),
+            "sample": f"one main-thread decode step: the {n0}-token context, all {Hq} heads, "
+                      f"all {L} layers",
+            "seconds": round(total, 3)}
 
 
 def run_trace(args, world, rank, local):
@@ -754,7 +890,10 @@ def run_trace(args, world, rank, local):
                         break
                     chosen.append(old[int(j)])
                     cov += old[int(j)][2] - old[int(j)][1]
-                cache.evict_spans(m, [(s, e) for _, s, e in chosen], sh_)
+                if args.ragged:
+                    cache.evict_spans_ragged(m, [(s, e) for _, s, e in chosen], sh_)
+                else:
+                    cache.evict_spans(m, [(s, e) for _, s, e in chosen], sh_)
                 # shift the positions of the responses that stay
                 gone = sorted((s, e) for _, s, e in chosen)
                 keep = []
@@ -800,12 +939,14 @@ def run_trace(args, world, rank, local):
     torch.cuda.synchronize()
     wall = time.perf_counter() - w0
     clock_rec = clocks.stop()
+    step_append_ms = 0.0   # batched one-row appends of the decode steps (their launch gap included)
     for e in ev_list:
         if e[0] == "append":
             times["append"] += e[1].elapsed_time(e[2])
         elif len(e) == 2:
             times["eviction"] += e[0].elapsed_time(e[1])
         else:
+            step_append_ms += e[0].elapsed_time(e[1])
             times["append"] += e[0].elapsed_time(e[1])
             times["attention"] += e[1].elapsed_time(e[2])
     st1 = cache.stats()
@@ -834,9 +975,23 @@ def run_trace(args, world, rank, local):
             "peak_tokens_all_agents": int(peak_tokens),
             "peak_live_pages": int(st1["peak_live_pages"]),
             "final_tokens_per_agent": [cache.seq_info(m)[0] for m in mains],
+            # the new token's K/V append and its gap to the first layer's
+            # attention, as a share of the decode steps' GPU time
+            "step_append_share": round(step_append_ms / (step_append_ms + times["attention"]), 5),
+            "step_append_us": round(1e3 * step_append_ms / (T * 256), 3),
+            "evict_call": "sq_evict_spans_ragged" if args.ragged else "sq_evict_spans",
+        },
+        "roofline": {
+            "bound": "hbm", "kernel": "sq_decode_splitk_kernel (all decode calls of the trace)",
+            "achieved": round((st1["decode_unique_bytes"] - st0["decode_unique_bytes"]) /
+                              (times["attention"] / 1e3) / 1e9, 1),
+            "peak": peaks()[0], "peak_kind": peaks()[1], "unit": "GB/s",
+            "timing": "CUDA events around each step's 32 layer calls",
+            "traffic": None,
         },
         "clocks": clock_rec,
     }
+    res["roofline"]["frac"] = round(res["roofline"]["achieved"] / res["roofline"]["peak"], 4)
     cache.close()
     return res
 
@@ -1395,6 +1550,46 @@ def run_reference(args, world, rank):
     }
 
 
+# The other workloads, measured in the same process after the headline one
+# (its cache closed first), so that one default run records every workload:
+# (workload, overrides of the command-line arguments).
+SUB_WORKLOADS = [
+    ("large-ragged", {"steps": 5, "warmup": 3, "no_cpu": True, "no_e2e": True}),
+    ("agent-32k", {}),
+    ("trace", {"turns": 16, "ragged": True}),
+    ("prefill-32k", {"steps": 3, "warmup": 3, "no_cpu": True, "no_e2e": True}),
+    ("aux-trigger-128k", {"steps": 10, "warmup": 3, "no_cpu": True, "no_e2e": True}),
+]
+SUB_DROP = ("metric", "data", "n_gpus", "higher_is_better", "scaling", "vs_baseline", "dtype",
+            "gpu_launches", "e2e")
+
+
+def run_sub_records(args, rank, local):
+    import gc
+
+    import torch
+    runners = {"large-ragged": run_sq, "agent-32k": run_agent, "trace": run_trace,
+               "prefill-32k": run_prefill, "aux-trigger-128k": run_aux_trigger}
+    out = {}
+    for name, over in SUB_WORKLOADS:
+        a = argparse.Namespace(**vars(args))
+        a.workload = name
+        for k, v in over.items():
+            setattr(a, k, v)
+        gc.collect()
+        torch.cuda.empty_cache()
+        try:
+            r = runners[name](a, 1, rank, local)
+        except Exception as e:  # a failed sub-record is reported, not fatal
+            out[name] = {"error": f"{type(e).__name__}: {e}"}
+            continue
+        rec = {k: v for k, v in r.items() if k not in SUB_DROP}
+        rec["note"] = ("measured in the same process after the headline workload, whose cache "
+                       "was closed first; steps and warm-up as listed")
+        out[name] = rec
+    return out
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -1415,6 +1610,8 @@ def main():
         res = run_aux_trigger(args, world, rank, local)
     else:
         res = run_sq(args, world, rank, local)
+        if args.workload == "serving-128k" and world == 1 and not args.no_sub:
+            res["sub_records"] = run_sub_records(args, rank, local)
     if rank == 0:
         print(json.dumps(res), flush=True)
     if world > 1:

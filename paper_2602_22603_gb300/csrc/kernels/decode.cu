@@ -334,16 +334,19 @@ __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, ui
             // or rows once appended, so only their scores are masked.
             uint32_t vm = 0xffffu;
             if (a.page_fill) {
-                const int t0 = s * kStageTokens + warp * 16;  // segment slot position
+                // P is a power of two >= 8 and the 16 rows start at a multiple
+                // of 16: one page holds them all (P >= 16), or two (P = 8)
                 const int P = a.P;
-                const int pq0 = t0 / P, pq1 = (t0 + 15) / P;  // pq1 = pq0 + 1 only for P = 8
-                const int f0 = pq0 < seg->n_pages ? __ldg(&a.page_fill[seg->page_off + pq0]) : 0;
-                const int f1 = pq1 < seg->n_pages ? __ldg(&a.page_fill[seg->page_off + pq1]) : 0;
-                vm = 0u;
-#pragma unroll
-                for (int r = 0; r < 16; ++r) {
-                    const int t = t0 + r;
-                    vm |= (uint32_t)(t % P < (t / P == pq0 ? f0 : f1)) << r;
+                const int t0 = s * kStageTokens + warp * 16;  // segment slot position
+                const int pq = t0 >> (__ffs(P) - 1);
+                const int f0 = pq < seg->n_pages ? __ldg(&a.page_fill[seg->page_off + pq]) : 0;
+                if (P >= 16) {
+                    const int v = min(max(f0 - (t0 & (P - 1)), 0), 16);
+                    vm = (uint32_t)((1u << v) - 1u);   // v = 16 gives 0xffff
+                } else {
+                    const int f1 =
+                        pq + 1 < seg->n_pages ? __ldg(&a.page_fill[seg->page_off + pq + 1]) : 0;
+                    vm = ((1u << min(f0, 8)) - 1u) | (((1u << min(f1, 8)) - 1u) << 8);
                 }
             }
             if (!dead) {
