@@ -589,8 +589,13 @@ def run_sq(args, world, rank, local):
         after_rg = timed_decode(K, W)
         pc = after_rg["attn_ms"] / after_rg["calls"]
         up = after_rg["unique_bytes"] / after_rg["calls"]
+        rg_ratio, rg_src = recorded_traffic_ratio("sq_evict_compact_kernel", "ragged")
+        dr_ratio, dr_src = recorded_traffic_ratio("sq_decode_splitk_kernel", "ragged")
         res["evict_ragged"] = {
             "call": "sq_evict_spans_ragged",
+            "kernel": "sq_evict_compact_kernel",
+            "traffic_per_call": int(rg_ratio * rg_bytes / len(mains)) if rg_ratio else None,
+            "traffic_source": rg_src,
             "ms_total": round(rg_ms, 4),
             "ms_total_dense": res["evict"]["ms_total"],
             "moved_rows": int(st1["evict_moved_rows"] - st0["evict_moved_rows"]),
@@ -609,6 +614,8 @@ def run_sq(args, world, rank, local):
             "hbm_gbs_unique": round(up / (pc / 1e3) / 1e9, 1),
             "frac_of_%s_peak" % peak_kind: round(up / (pc / 1e3) / 1e9 / hbm_peak, 4),
             "unique_gb_per_call_dense": res["after_evict"]["unique_gb_per_call"],
+            "traffic_per_call": int(dr_ratio * up) if dr_ratio else None,
+            "traffic_source": dr_src,
         }
 
     # ---- CPU oracle on a bounded sample (rank 0, N = 1) ----------------------
