@@ -9,6 +9,7 @@
 
 #include <algorithm>
 #include <cstring>
+#include <deque>
 #include <memory>
 #include <new>
 #include <unordered_map>
@@ -40,6 +41,12 @@ struct PlanEntry {
     DecodePlanLayout lay{};
     int64_t unique_tokens = 0, logical_tokens = 0;
     int32_t first_busy_cta = 0;  // lowest CTA with work (target of the test hook)
+    // write tickets of the plan's pages (fixed while the plan is valid: a
+    // write to a page changes the version of every sequence holding it): the
+    // kDecodeMaxUnsafe newest (ticket, page) pairs and the newest ticket of
+    // all other pages
+    std::vector<std::pair<uint64_t, int32_t>> tick_top;
+    uint64_t tick_rest = 0;
     uint8_t* d_plan = nullptr;
     size_t plan_cap = 0;
     float* d_part = nullptr;
@@ -140,6 +147,15 @@ struct sq_cache {
     std::vector<void*> freed_on;
     std::vector<uint8_t> fenced;
     std::unordered_map<void*, cudaEvent_t> free_event;
+    // Writes to the pool by the library's kernels: every append, copy-on-write
+    // and eviction takes a ticket, stamps the pages it writes and records an
+    // event; write_done is the newest ticket whose work, and all before it,
+    // is known complete.
+    uint64_t write_seq = 0, write_done = 0;
+    bool early_ok = true;
+    std::vector<uint64_t> page_ticket;
+    std::deque<std::pair<uint64_t, cudaEvent_t>> write_pending;
+    std::vector<cudaEvent_t> write_events;  // recycled
     int32_t debug_flags = 0;
     sq_stats_t stats;
 };
@@ -234,6 +250,48 @@ int record_freed(sq_cache* c, const std::vector<int32_t>& freed, void* stream) {
         c->fenced[p] = 1;
     }
     return SQ_OK;
+}
+
+// Stamps the pages a pool-writing launch just enqueued on `stream` writes.
+// If the event cannot be recorded, decode stops loading anything before its
+// dependency wait for the rest of the cache's life.
+void note_writes(sq_cache* c, const int32_t* pages, size_t n, void* stream) {
+    if (n == 0 || !c->early_ok) return;
+    const uint64_t t = ++c->write_seq;
+    for (size_t i = 0; i < n; ++i)
+        if (pages[i] >= 0 && pages[i] < c->g.num_pages) c->page_ticket[pages[i]] = t;
+    cudaEvent_t ev;
+    if (!c->write_events.empty()) {
+        ev = c->write_events.back();
+        c->write_events.pop_back();
+    } else if (cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) != cudaSuccess) {
+        cudaGetLastError();
+        c->early_ok = false;
+        return;
+    }
+    if (cudaEventRecord(ev, as_stream(stream)) != cudaSuccess) {
+        cudaGetLastError();
+        c->write_events.push_back(ev);
+        c->early_ok = false;
+        return;
+    }
+    c->write_pending.push_back({t, ev});
+}
+
+// Advances write_done over the writes whose events have completed, in
+// ticket order (a write still running holds back every later ticket).
+void poll_writes(sq_cache* c) {
+    while (!c->write_pending.empty()) {
+        const cudaError_t q = cudaEventQuery(c->write_pending.front().second);
+        if (q == cudaErrorNotReady) break;
+        if (q != cudaSuccess) {   // leave the ticket pending; the error surfaces elsewhere
+            cudaGetLastError();
+            break;
+        }
+        c->write_done = c->write_pending.front().first;
+        c->write_events.push_back(c->write_pending.front().second);
+        c->write_pending.pop_front();
+    }
 }
 
 // Asynchronous host -> device copy of `bytes` from `src` through a pinned
@@ -354,6 +412,7 @@ int sq_cache_create(const sq_config* cfg, sq_cache** out) {
     if (!c->host) return SQ_ERR_NO_MEMORY;
     c->freed_on.assign(g.num_pages, nullptr);
     c->fenced.assign(g.num_pages, 0);
+    c->page_ticket.assign(g.num_pages, 0);
     std::memset(&c->stats, 0, sizeof c->stats);
     cudaError_t e = cudaGetDevice(&c->device);
     if (e != cudaSuccess) return cuda_status(e);
@@ -449,6 +508,8 @@ int sq_cache_destroy(sq_cache* c) {
         if (p.ev) cudaEventDestroy(p.ev);
     }
     for (auto& kv : c->free_event) cudaEventDestroy(kv.second);
+    for (auto& w : c->write_pending) cudaEventDestroy(w.second);
+    for (cudaEvent_t ev : c->write_events) cudaEventDestroy(ev);
     if (c->pre_part) cudaFree(c->pre_part);
     if (c->pre_ev) cudaEventDestroy(c->pre_ev);
     if (c->d_err) cudaFree(c->d_err);
@@ -526,6 +587,7 @@ int sq_append_kv(sq_cache* c, sq_seq seq, int32_t n_tokens, const void* k, const
         cudaError_t e = launch_append(a, c->num_sms, st);
         if (e != cudaSuccess) return undo(cuda_status(e));
     }
+    note_writes(c, plan.pages.data(), plan.pages.size(), stream);
     c->host->seq_mut(seq)->last_stream = stream;
     c->stats.appended_tokens += n_tokens;
     if (plan.cow) c->stats.cow_pages += 1;
@@ -591,6 +653,11 @@ int sq_append_kv_batch(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, const vo
         a.err = c->d_err;
         cudaError_t e = launch_append_batch(a, c->num_sms, st);
         if (e != cudaSuccess) return undo(n_seqs, cuda_status(e));
+    }
+    {
+        std::vector<int32_t> written(n_seqs);
+        for (int32_t i = 0; i < n_seqs; ++i) written[i] = plans[i].pages[0];
+        note_writes(c, written.data(), written.size(), stream);
     }
     for (int32_t i = 0; i < n_seqs; ++i) {
         c->host->seq_mut(seqs[i])->last_stream = stream;
@@ -703,6 +770,18 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
         while (victim->first_busy_cta + 1 < (int32_t)plan.cta_begin.size() &&
                plan.cta_begin[victim->first_busy_cta + 1] == plan.cta_begin[victim->first_busy_cta])
             ++victim->first_busy_cta;
+        {
+            std::vector<std::pair<uint64_t, int32_t>> tk(plan.page_ids.size());
+            for (size_t i = 0; i < tk.size(); ++i)
+                tk[i] = {c->page_ticket[plan.page_ids[i]], plan.page_ids[i]};
+            const size_t top = std::min<size_t>(kDecodeMaxUnsafe, tk.size());
+            std::partial_sort(tk.begin(), tk.begin() + top, tk.end(),
+                              [](const std::pair<uint64_t, int32_t>& x,
+                                 const std::pair<uint64_t, int32_t>& y) { return x.first > y.first; });
+            victim->tick_top.assign(tk.begin(), tk.begin() + top);
+            victim->tick_rest = 0;
+            for (size_t i = top; i < tk.size(); ++i) victim->tick_rest = std::max(victim->tick_rest, tk[i].first);
+        }
         hit = victim;
     } else if (hit->ev_recorded && hit->ev_stream != st) {
         e = cudaStreamWaitEvent(st, hit->ev, 0);
@@ -738,6 +817,19 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
     a.num_pages = g.num_pages;
     a.scale_log2 = sm_scale * 1.4426950408889634f;
     a.debug_drop_cta = (c->debug_flags & SQ_DEBUG_DROP_DECODE_STAGE) ? hit->first_busy_cta : -1;
+    a.kv_early = 0;
+    a.n_unsafe = 0;
+    if (plan_ready && c->early_ok) {
+        // every write to the plan's pages outside its newest few is complete:
+        // the kernel may load its first stages before its dependency wait,
+        // except from the pages whose writes may still be running
+        poll_writes(c);
+        if (hit->tick_rest <= c->write_done) {
+            a.kv_early = 1;
+            for (const auto& tp : hit->tick_top)
+                if (tp.first > c->write_done) a.unsafe[a.n_unsafe++] = tp.second;
+        }
+    }
     c->debug_flags &= ~SQ_DEBUG_DROP_DECODE_STAGE;
     a.err = c->d_err;
     e = launch_decode(c->tmap, a, L.n_ctas, g.D, st);
@@ -808,6 +900,10 @@ int evict_impl(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_spans, v
         if (e != cudaSuccess) return cuda_status(e);
         s.ev_recorded = true;
         s.ev_stream = st;
+        std::vector<int32_t> written;
+        for (const EvictMove& m : plan.moves)
+            if (written.empty() || written.back() != m.dst_page) written.push_back(m.dst_page);
+        note_writes(c, written.data(), written.size(), stream);
     }
     rc = record_freed(c, plan.freed, stream);
     if (rc != SQ_OK) return rc;
@@ -1260,6 +1356,8 @@ int sq_decode_attention_noalloc(sq_cache* c, const sq_seq* seqs, int32_t n_seqs,
     while (busy + 1 < (int32_t)plan.cta_begin.size() && plan.cta_begin[busy + 1] == plan.cta_begin[busy])
         ++busy;
     a.debug_drop_cta = (c->debug_flags & SQ_DEBUG_DROP_DECODE_STAGE) ? busy : -1;
+    a.kv_early = 0;   // the plan was uploaded just now (read after the wait)
+    a.n_unsafe = 0;
     c->debug_flags &= ~SQ_DEBUG_DROP_DECODE_STAGE;
     a.err = c->d_err;
     e = launch_decode(c->tmap, a, L.n_ctas, g.D, st);

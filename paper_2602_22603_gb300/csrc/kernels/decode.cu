@@ -89,6 +89,7 @@ constexpr int kFastStages = 3;      // stages whose coordinates are kept in regi
 // plan there.
 struct FastStart {
     int n;                       // stages read (0: none)
+    int early;                   // of them, issued before the grid-dependency wait
     int it, s;                   // where the producer continues
     int32_t row[kFastStages];    // K row coordinate head * P + row0 (V: + Hkv * P)
     int32_t pid[kFastStages];
@@ -157,6 +158,30 @@ __device__ void prefetch_first_stages(const CUtensorMap* tmap, const DecodeArgs&
 }
 
 // ---- producer: one thread issues the TMA loads of every stage -------------
+// Issues the loads of fast stage k (whole-page stage, ring slot k).
+template <int D>
+__device__ __forceinline__ void issue_fast_stage(const CUtensorMap* tmap, const DecodeArgs& a,
+                                                 const FastStart& fs, int k, uint8_t* smem,
+                                                 uint64_t* bars) {
+    using C = DecCfg<D>;
+    const uint32_t bytes = (uint32_t)kStageTokens * 128u * C::kColBlocks * 2u;
+    const uint32_t full = smem_addr(&bars[k]);
+    const int32_t p = fs.pid[k];
+    if ((uint32_t)p < (uint32_t)a.num_pages) {
+        mbar_arrive_expect_tx(full, bytes);
+        const uint32_t dk = smem_addr(smem + k * C::kStageBytes);
+#pragma unroll
+        for (int cb = 0; cb < C::kColBlocks; ++cb) {
+            tma_load_4d(dk + cb * C::kBlockBytes, tmap, full, cb * 64, fs.row[k], p, a.layer);
+            tma_load_4d(dk + cb * C::kBlockBytes + C::kTileBytes, tmap, full, cb * 64,
+                        fs.row[k] + a.Hkv * a.P, p, a.layer);
+        }
+    } else {
+        set_error(a.err, kErrBounds);
+        mbar_arrive(full);
+    }
+}
+
 template <int D>
 __device__ void produce(const CUtensorMap* tmap, const DecodeArgs& a, int it0, int it1,
                         const FastStart& fs, uint8_t* smem, uint64_t* bars,
@@ -172,27 +197,12 @@ __device__ void produce(const CUtensorMap* tmap, const DecodeArgs& a, int it0, i
     bool ok = true;
     int it_start = it0, s_start = -1;       // -1: the item's first stage
     if (fs.n > 0) {
-        // the first stages, from registers (whole-page stages; fresh slots)
-        const uint32_t bytes = box_bytes * C::kColBlocks * 2u;
+        // the first stages, from registers (whole-page stages; fresh slots);
+        // the first fs.early of them were issued before the dependency wait
 #pragma unroll
         for (int k = 0; k < kFastStages; ++k) {
             if (k < fs.n) {
-                const uint32_t full = smem_addr(&bars[k]);
-                const int32_t p = fs.pid[k];
-                if ((uint32_t)p < (uint32_t)a.num_pages) {
-                    mbar_arrive_expect_tx(full, bytes);
-                    const uint32_t dk = smem_addr(smem + k * C::kStageBytes);
-#pragma unroll
-                    for (int cb = 0; cb < C::kColBlocks; ++cb) {
-                        tma_load_4d(dk + cb * C::kBlockBytes, tmap, full, cb * 64, fs.row[k], p,
-                                    a.layer);
-                        tma_load_4d(dk + cb * C::kBlockBytes + C::kTileBytes, tmap, full, cb * 64,
-                                    fs.row[k] + a.Hkv * P, p, a.layer);
-                    }
-                } else {
-                    set_error(a.err, kErrBounds);
-                    mbar_arrive(full);
-                }
+                if (k >= fs.early) issue_fast_stage<D>(tmap, a, fs, k, smem, bars);
                 issued |= 1u << k;
             }
         }
@@ -772,6 +782,7 @@ __global__ void __launch_bounds__(DecCfg<D>::kThreads, 2)
     // and first stages in registers and warms L2 with the first stages' rows.
     FastStart fs;
     fs.n = 0;
+    fs.early = 0;
     int p_it0 = 0, p_it1 = 0;
     if (warp == kDecodeConsumerWarps && lane == 0) {
         prefetch_tmap(&tmap);
@@ -784,8 +795,22 @@ __global__ void __launch_bounds__(DecCfg<D>::kThreads, 2)
         }
     }
     __syncthreads();
+    // Pages no in-flight work writes (the host checked every library write to
+    // them is complete; the kernels before this one write no other pool
+    // memory) may be loaded before the wait: the first stages stream in while
+    // the previous kernel finishes.  Stop at the first stage in a page that
+    // may still be written; the rest go out after the wait, in order.
+    if (warp == kDecodeConsumerWarps && lane == 0 && a.kv_early && fs.n > 0) {
+        for (int k = 0; k < fs.n; ++k) {
+            bool unsafe = false;
+            for (int u = 0; u < a.n_unsafe; ++u) unsafe |= a.unsafe[u] == fs.pid[k];
+            if (unsafe) break;
+            issue_fast_stage<D>(&tmap, a, fs, k, smem, bars);
+            fs.early = k + 1;
+        }
+    }
     // Launched as a programmatic dependent: the set-up above overlapped the
-    // previous kernel's tail; nothing it may have written is read before here.
+    // previous kernel's tail; nothing else it may have written is read before here.
     grid_dependency_wait();
     grid_launch_dependents();  // the next kernel may be scheduled as CTAs retire
     if (warp == kDecodeConsumerWarps) {

@@ -11,6 +11,10 @@
 namespace sq {
 
 // ---- decode attention -------------------------------------------------------
+// Pages whose K/V may still be being written when a decode call starts, at
+// most this many per call (see DecodeArgs::kv_early).
+constexpr int kDecodeMaxUnsafe = 32;
+
 struct DecodeArgs {
     const DecodeSeg* segs;
     const DecodeItem* items;
@@ -32,6 +36,13 @@ struct DecodeArgs {
     int32_t layer, Hq, Hkv, G, P, num_pages;
     float scale_log2;           // sm_scale * log2(e)
     int32_t debug_drop_cta;     // test hook: this CTA leaves its first stage unsignalled (-1: none)
+    // 1: every library write to the plan's pages except those in unsafe[] is
+    // known complete (the host polled its events), so a CTA may load its
+    // first stages before the grid-dependency wait, overlapping the previous
+    // kernel's tail, up to its first stage in one of those pages
+    int32_t kv_early;
+    int32_t n_unsafe;
+    int32_t unsafe[kDecodeMaxUnsafe];
     int* err;
 };
 

@@ -565,3 +565,33 @@ def test_next_position_through_the_api():
         assert ei.value.code == sq.SQ_ERR_BAD_HANDLE
     finally:
         p.close()
+
+
+def test_decode_steps_reuse_plans_with_early_loads():
+    """Decode steps as a model runs them: one batched append, then every
+    layer's call on one stream.  Every call after a step's first reuses the
+    step's plan and loads its first stages before its dependency wait (the
+    pages the step's append wrote are excluded until that append is known
+    complete); each output must equal the oracle."""
+    L = 6
+    p = Pair(L, 32, 8, 128, 64, num_pages=900, seed=88)
+    keep = []
+    m = p.seq_new()
+    keep.append(p.append(m, 20000))
+    a = p.fork(m)
+    keep.append(p.append(a, 30))
+    seqs = [m, a]
+    checks = []
+    for step in range(3):
+        keep.append(p.append_batch(seqs))
+        for layer in range(L):
+            q_cpu, q = _q(900 + 10 * step + layer, 2, 32, 128)
+            keep.append(q)
+            out = p.decode(seqs, layer, 0.09, q, sq.SQ_OUT_F32)
+            checks.append((out, layer, q_cpu, [p.oracle.n_tokens(p.o[h]) for h in seqs]))
+        torch.cuda.synchronize()
+        for out, layer, q_cpu, ns in checks:
+            assert_budget(out, *p.oracle_decode_budget(seqs, layer, 0.09, q_cpu))
+        checks.clear()
+    assert p.cache.sync_status() == sq.SQ_OK
+    p.close()
