@@ -54,10 +54,13 @@ int sqh_evict(void* c, int32_t h, const int32_t* spans, int32_t n_spans, int32_t
 }
 
 // Evicts and returns the compaction tiles (4 ints each: dst_page, dst_slot,
-// n_rows, piece_begin) and pieces (src_page, src_slot, n_rows, dst_row).
+// n_rows, piece_begin) and pieces (src_page, src_slot, n_rows, dst_row), and
+// the chunks of windows (chunk_out[0 .. n_chunks], tile indices) that the
+// library would run in parallel CTAs with `max_chunks`.
 int sqh_evict_tiles(void* c, int32_t h, const int32_t* spans, int32_t n_spans, int32_t ragged,
                     int32_t tile_rows, int32_t* tiles_out, int32_t tiles_cap, int32_t* pieces_out,
-                    int32_t pieces_cap, int32_t* n_tiles, int32_t* n_pieces) {
+                    int32_t pieces_cap, int32_t* n_tiles, int32_t* n_pieces, int32_t max_chunks,
+                    int32_t* chunk_out, int32_t chunk_cap, int32_t* n_chunks) {
     HostCache* hc = static_cast<HostCache*>(c);
     std::vector<int32_t> a(n_spans > 0 ? n_spans : 0), b(a.size());
     for (int32_t i = 0; i < n_spans; ++i) { a[i] = spans[2 * i]; b[i] = spans[2 * i + 1]; }
@@ -66,12 +69,18 @@ int sqh_evict_tiles(void* c, int32_t h, const int32_t* spans, int32_t n_spans, i
     if (rc != kOk) return rc;
     std::vector<EvictTile> tiles;
     std::vector<EvictPiece> pieces;
-    evict_tiles(p, tile_rows, &tiles, &pieces);
+    std::vector<int32_t> window_tile, chunk;
+    evict_tiles(p, tile_rows, &tiles, &pieces, &window_tile);
+    evict_chunks(window_tile, (int32_t)tiles.size(), max_chunks, 4, &chunk);
     *n_tiles = (int32_t)tiles.size();
     *n_pieces = (int32_t)pieces.size();
-    if ((int32_t)tiles.size() > tiles_cap || (int32_t)pieces.size() > pieces_cap) return kInvalidArg;
+    *n_chunks = (int32_t)chunk.size() - 1;
+    if ((int32_t)tiles.size() > tiles_cap || (int32_t)pieces.size() > pieces_cap ||
+        (int32_t)chunk.size() > chunk_cap)
+        return kInvalidArg;
     std::memcpy(tiles_out, tiles.data(), tiles.size() * sizeof(EvictTile));
     std::memcpy(pieces_out, pieces.data(), pieces.size() * sizeof(EvictPiece));
+    std::memcpy(chunk_out, chunk.data(), chunk.size() * sizeof(int32_t));
     return kOk;
 }
 

@@ -874,11 +874,21 @@ int evict_impl(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_spans, v
     if (!plan.moves.empty()) {
         std::vector<EvictTile> tiles;
         std::vector<EvictPiece> pieces;
-        evict_tiles(plan, c->evict_tile_rows, &tiles, &pieces);
+        std::vector<int32_t> window_tile, chunk;
+        evict_tiles(plan, c->evict_tile_rows, &tiles, &pieces, &window_tile);
+        // Independent windows (ragged eviction) run as chunks in parallel
+        // CTAs, up to about four waves of resident CTAs over all planes
+        const int64_t planes = (int64_t)g.L * 2 * g.Hkv;
+        const int64_t resident =
+            (int64_t)c->num_sms * evict_ctas_per_sm(c->evict_tile_rows, g.D);
+        const int32_t max_chunks = (int32_t)std::max<int64_t>(1, 4 * resident / planes);
+        evict_chunks(window_tile, (int32_t)tiles.size(), max_chunks, 4, &chunk);
         const size_t tb = tiles.size() * sizeof(EvictTile);
-        std::vector<uint8_t> buf(tb + pieces.size() * sizeof(EvictPiece));
+        const size_t pcb = pieces.size() * sizeof(EvictPiece);
+        std::vector<uint8_t> buf(tb + pcb + chunk.size() * sizeof(int32_t));
         std::memcpy(buf.data(), tiles.data(), tb);
-        std::memcpy(buf.data() + tb, pieces.data(), pieces.size() * sizeof(EvictPiece));
+        std::memcpy(buf.data() + tb, pieces.data(), pcb);
+        std::memcpy(buf.data() + tb + pcb, chunk.data(), chunk.size() * sizeof(int32_t));
         UploadSlot& s = c->slots[c->next_slot];
         c->next_slot = (c->next_slot + 1) % kUploadSlots;
         rc = upload(c, s, buf.data(), buf.size(), stream);
@@ -893,6 +903,8 @@ int evict_impl(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_spans, v
         ea.n_pieces = (int32_t)pieces.size();
         ea.tile_rows = c->evict_tile_rows;
         ea.zero_tiles = plan.zeroed_rows > 0 ? 1 : 0;
+        ea.n_chunks = (int32_t)chunk.size() - 1;
+        ea.chunk = ea.n_chunks > 1 ? reinterpret_cast<const int32_t*>(s.d + tb + pcb) : nullptr;
         ea.err = c->d_err;
         cudaError_t e = launch_evict(ea, st);
         if (e != cudaSuccess) return undo(cuda_status(e));

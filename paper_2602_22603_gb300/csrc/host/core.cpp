@@ -370,14 +370,14 @@ int HostCache::evict(int32_t h, const int32_t* starts, const int32_t* ends,
         for (const Run& x : runs[wi]) {
             const bool fresh = page_at[x.dq] != s->pages[x.dq];
             if (!fresh && x.dq == x.sq && x.ds == x.ss) continue;  // rows stay where they are
-            plan->moves.push_back({page_at[x.dq], x.ds, s->pages[x.sq], x.ss, x.n});
+            plan->moves.push_back({page_at[x.dq], x.ds, s->pages[x.sq], x.ss, x.n, (int32_t)wi});
             plan->moved_rows += x.n;
         }
         if (ragged && w.used > 0) {
             const int32_t q = w.qa + w.used - 1;
             const bool fresh = page_at[q] != s->pages[q];
             if ((changed[q] || fresh) && dest_fill[q] < P) {
-                plan->moves.push_back({page_at[q], dest_fill[q], -1, 0, P - dest_fill[q]});
+                plan->moves.push_back({page_at[q], dest_fill[q], -1, 0, P - dest_fill[q], (int32_t)wi});
                 plan->zeroed_rows += P - dest_fill[q];
             }
         }
@@ -450,13 +450,21 @@ int HostCache::release(int32_t h, std::vector<int32_t>* freed) {
 }
 
 void evict_tiles(const EvictPlan& p, int32_t tile_rows, std::vector<EvictTile>* tiles,
-                 std::vector<EvictPiece>* pieces) {
+                 std::vector<EvictPiece>* pieces, std::vector<int32_t>* window_tile) {
     tiles->clear();
     pieces->clear();
+    if (window_tile) window_tile->clear();
     EvictTile* open = nullptr;   // the tile being filled
     bool open_zero = false;
+    int32_t window = -1;
     for (const EvictMove& m : p.moves) {
         const bool zero = m.src_page < 0;
+        if (m.window != window) {
+            // a new window starts a new tile
+            window = m.window;
+            open = nullptr;
+            if (window_tile) window_tile->push_back((int32_t)tiles->size());
+        }
         int32_t done = 0;
         while (done < m.n) {
             const int32_t dst_slot = m.dst_slot + done;
@@ -475,6 +483,22 @@ void evict_tiles(const EvictPlan& p, int32_t tile_rows, std::vector<EvictTile>* 
             done += k;
         }
     }
+}
+
+void evict_chunks(const std::vector<int32_t>& window_tile, int32_t n_tiles, int32_t max_chunks,
+                  int32_t min_tiles, std::vector<int32_t>* chunk) {
+    chunk->assign(1, 0);
+    const int32_t nw = (int32_t)window_tile.size();
+    int32_t want = std::min<int32_t>(max_chunks, nw);
+    if (min_tiles > 0) want = std::min<int32_t>(want, std::max<int32_t>(1, n_tiles / min_tiles));
+    // cut at the window start nearest each even share of the tiles
+    int32_t w = 1;
+    for (int32_t c = 1; c < want && w < nw; ++c) {
+        const int64_t target = (int64_t)n_tiles * c / want;
+        while (w < nw && window_tile[w] < target) ++w;
+        if (w < nw && window_tile[w] > chunk->back()) chunk->push_back(window_tile[w++]);
+    }
+    chunk->push_back(n_tiles);
 }
 
 // ---------------------------------------------------------------------------

@@ -120,6 +120,7 @@ struct AppendPlan {
 // zero rows when src_page is -1.
 struct EvictMove {
     int32_t dst_page, dst_slot, src_page, src_slot, n;
+    int32_t window;   // the window (run of packed pages) the move belongs to
 };
 
 struct EvictPlan {
@@ -180,8 +181,16 @@ class HostCache {
 // source of a tile lies at a slot-space position >= the tile's first
 // destination row, so processing tiles in order, each tile's reads before
 // its writes, compacts in place.
+// `window_tile` (may be null) receives the index of each window's first
+// tile: windows share no page, so their tiles may run in any order.
 void evict_tiles(const EvictPlan& p, int32_t tile_rows, std::vector<EvictTile>* tiles,
-                 std::vector<EvictPiece>* pieces);
+                 std::vector<EvictPiece>* pieces, std::vector<int32_t>* window_tile = nullptr);
+
+// Groups consecutive windows into at most `max_chunks` chunks of about equal
+// tile counts, at least `min_tiles` tiles each (but the last): chunk c is
+// tiles [chunk[c], chunk[c + 1]).  One chunk when there is one window.
+void evict_chunks(const std::vector<int32_t>& window_tile, int32_t n_tiles, int32_t max_chunks,
+                  int32_t min_tiles, std::vector<int32_t>* chunk);
 
 // ---- decode planning -------------------------------------------------------
 

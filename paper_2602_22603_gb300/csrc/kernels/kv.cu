@@ -110,8 +110,10 @@ __global__ void __launch_bounds__(256) sq_cow_copy_kernel(const CowArgs a) {
 // row written so far.  Copy-on-write destination pages are fresh pages that
 // hold no source row.  No inter-CTA wait is needed.
 //
-// A tile without pieces writes zeros: the unused slots of a page that a
-// ragged eviction leaves partial.  Its store reads a zero tile that the
+// A ragged eviction's windows share no page, so the tile list is cut at
+// window starts into chunks that separate CTAs of one plane run in parallel;
+// each chunk keeps the in-order rule above.  A tile without pieces writes
+// zeros: the unused slots of a page that a ragged eviction leaves partial.  Its store reads a zero tile that the
 // CTA's warp clears once; it writes only past the rows its window kept, and
 // later tiles read only later windows' pages.
 __global__ void __launch_bounds__(32) sq_evict_compact_kernel(const EvictArgs a) {
@@ -130,7 +132,16 @@ __global__ void __launch_bounds__(32) sq_evict_compact_kernel(const EvictArgs a)
     }
     if (threadIdx.x != 0) return;
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + (S + (a.zero_tiles ? 1 : 0)) * tile_bytes);
-    const int plane = blockIdx.x;
+    // CTA = (chunk of independent windows, plane); tiles [tb, te) of the list
+    const int planes = a.L * 2 * a.Hkv;
+    const int plane = blockIdx.x % planes;
+    const int ch = blockIdx.x / planes;
+    const int tb = a.chunk ? __ldg(&a.chunk[ch]) : 0;
+    const int te = a.chunk ? __ldg(&a.chunk[ch + 1]) : a.n_tiles;
+    if (tb < 0 || te > a.n_tiles || tb > te) {
+        set_error(a.err, kErrBounds);
+        return;
+    }
     const int head = plane % a.Hkv;
     const int kv = (plane / a.Hkv) % 2;
     const int layer = plane / (2 * a.Hkv);
@@ -140,12 +151,13 @@ __global__ void __launch_bounds__(32) sq_evict_compact_kernel(const EvictArgs a)
     for (int s = 0; s < S; ++s) mbar_init(smem_addr(&full[s]), 1);
     fence_mbar_init();
 
-    auto issue_loads = [&](int t) {
+    auto issue_loads = [&](int t) {   // t: index in the chunk
         const int slot = t % S;
+        const int g = tb + t;
         const uint32_t bar = smem_addr(&full[slot]);
         const uint32_t dst0 = smem_addr(smem + slot * tile_bytes);
-        const int pb = __ldg(&a.tiles[t].piece_begin);
-        const int pe = t + 1 < a.n_tiles ? __ldg(&a.tiles[t + 1].piece_begin) : a.n_pieces;
+        const int pb = __ldg(&a.tiles[g].piece_begin);
+        const int pe = g + 1 < a.n_tiles ? __ldg(&a.tiles[g + 1].piece_begin) : a.n_pieces;
         uint32_t bytes = 0;
         for (int k = pb; k < pe; ++k) {
             const EvictPiece pc = a.pieces[k];
@@ -174,7 +186,7 @@ __global__ void __launch_bounds__(32) sq_evict_compact_kernel(const EvictArgs a)
         }
     };
 
-    const int T = a.n_tiles;
+    const int T = te - tb;
     for (int t = 0; t < S - 1 && t < T; ++t) issue_loads(t);
     int t = 0;
     for (; t < T; ++t) {
@@ -184,8 +196,9 @@ __global__ void __launch_bounds__(32) sq_evict_compact_kernel(const EvictArgs a)
             break;
         }
         fence_proxy_async_smem();
-        const EvictTile tl = a.tiles[t];
-        const int pe = t + 1 < T ? __ldg(&a.tiles[t + 1].piece_begin) : a.n_pieces;
+        const int g = tb + t;
+        const EvictTile tl = a.tiles[g];
+        const int pe = g + 1 < a.n_tiles ? __ldg(&a.tiles[g + 1].piece_begin) : a.n_pieces;
         const bool zeros = tl.piece_begin == pe;  // no pieces: a tile of zeros
         if ((uint64_t)tl.dst_page < (uint64_t)a.num_pages && tl.dst_slot >= 0 && tl.n_rows > 0 &&
             tl.n_rows <= a.tile_rows && tl.dst_slot + tl.n_rows <= a.P && (!zeros || a.zero_tiles)) {
@@ -263,7 +276,7 @@ cudaError_t evict_prepare() {
 }
 
 cudaError_t launch_evict(const EvictArgs& a, cudaStream_t st) {
-    const int blocks = a.L * 2 * a.Hkv;
+    const int blocks = a.L * 2 * a.Hkv * (a.chunk ? a.n_chunks : 1);
     if (blocks == 0 || a.n_tiles == 0) return cudaSuccess;
     sq_evict_compact_kernel<<<blocks, 32, evict_smem_bytes(a.tile_rows, a.D, a.zero_tiles != 0),
                               st>>>(a);

@@ -144,6 +144,10 @@ struct EvictArgs {
     int32_t n_tiles, n_pieces;
     int32_t tile_rows;          // rows a tile holds at most
     int32_t zero_tiles;         // 1: some tiles (those without pieces) write zeros
+    // null, or [n_chunks + 1] tile indices: chunk c (tiles [chunk[c],
+    // chunk[c + 1]), whole windows) of every plane runs in its own CTA
+    const int32_t* chunk;
+    int32_t n_chunks;
     int* err;
 };
 

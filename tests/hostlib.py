@@ -34,7 +34,7 @@ def lib():
         L.sqh_evict.argtypes = [P, I32, I32P, I32, I32, I64P]
         L.sqh_release.argtypes = [P, I32]
         L.sqh_evict_tiles.argtypes = [P, I32, I32P, I32, I32, I32, I32P, I32, I32P, I32, I32P,
-                                      I32P]
+                                      I32P, I32, I32P, I32, I32P]
         L.sqh_page_fill.argtypes = [P, I32, I32P, I32, I32P]
         L.sqh_prefill_slot_spans.argtypes = [P, I32, I32, I32P, I32, I32P, I32, I32P, I32P]
         L.sqh_seq_info.argtypes = [P, I32, I32P, I32P]
@@ -99,18 +99,25 @@ class HostCache:
         return rc, {"moved_rows": st[0], "cow_pages": st[1], "freed": st[2],
                     "zeroed_rows": st[3], "windows": st[4], "n_moves": st[5]}
 
-    def evict_tiles(self, h, spans, tile_rows, ragged=False, cap=100000):
+    def evict_tiles(self, h, spans, tile_rows, ragged=False, cap=100000, max_chunks=1,
+                    want_chunks=False):
         arr = (ctypes.c_int32 * max(2, 2 * len(spans)))(*[int(x) for ab in spans for x in ab])
         tiles = np.zeros(4 * cap, dtype=np.int32)
         pieces = np.zeros(4 * cap, dtype=np.int32)
-        nt, npc = ctypes.c_int32(), ctypes.c_int32()
+        chunks = np.zeros(cap, dtype=np.int32)
+        nt, npc, nch = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
         i32p = ctypes.POINTER(ctypes.c_int32)
         rc = lib().sqh_evict_tiles(self.h, h, arr, len(spans), int(ragged), tile_rows,
                                    tiles.ctypes.data_as(i32p), cap, pieces.ctypes.data_as(i32p),
-                                   cap, ctypes.byref(nt), ctypes.byref(npc))
+                                   cap, ctypes.byref(nt), ctypes.byref(npc), max_chunks,
+                                   chunks.ctypes.data_as(i32p), cap, ctypes.byref(nch))
         if rc != 0:
-            return rc, None, None
-        return 0, tiles[:4 * nt.value].reshape(-1, 4), pieces[:4 * npc.value].reshape(-1, 4)
+            return (rc, None, None, None) if want_chunks else (rc, None, None)
+        t = tiles[:4 * nt.value].reshape(-1, 4)
+        pc = pieces[:4 * npc.value].reshape(-1, 4)
+        if want_chunks:
+            return 0, t, pc, chunks[:nch.value + 1].tolist()
+        return 0, t, pc
 
     def release(self, h):
         return lib().sqh_release(self.h, h)

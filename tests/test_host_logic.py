@@ -316,11 +316,39 @@ def test_evict_tiles_compact_in_place(seed):
     spans = random_spans(rng, n, rng.choice([1, 3, 8, 20]))
     # physical state before, as {page: [token ids]}
     phys = {p: list(v) for p, v in oc.phys.items()}
-    rc, tiles, pieces = hc.evict_tiles(m, spans, tile_rows, ragged)
+    max_chunks = rng.choice([1, 2, 5, 64])
+    rc, tiles, pieces, chunks = hc.evict_tiles(m, spans, tile_rows, ragged, max_chunks=max_chunks,
+                                               want_chunks=True)
     oc.evict(om, spans, mode="ragged" if ragged else "dense")
     assert rc == 0
-    written = set()
+    # chunks cover the tiles in order; a dense eviction is one chunk
+    assert chunks[0] == 0 and chunks[-1] == len(tiles) and chunks == sorted(set(chunks))
+    assert len(chunks) - 1 <= max(1, max_chunks)
+    if not ragged:
+        assert len(chunks) == 2 or len(tiles) == 0
+    # chunks run in any order (here: last first), each in order, against
+    # one pool; chunk c's tiles read no slot another chunk writes
+    order = []
+    for c in reversed(range(len(chunks) - 1)):
+        order.extend(range(chunks[c], chunks[c + 1]))
+    chunk_of = {}
+    for c in range(len(chunks) - 1):
+        for t in range(chunks[c], chunks[c + 1]):
+            chunk_of[t] = c
+    writes = {}
     for t in range(len(tiles)):
+        dpage, dslot, nrows, _ = (int(x) for x in tiles[t])
+        for i in range(nrows):
+            writes[(dpage, dslot + i)] = chunk_of[t]
+    for t in range(len(tiles)):
+        pb = int(tiles[t][3])
+        pe = int(tiles[t + 1][3]) if t + 1 < len(tiles) else len(pieces)
+        for k in range(pb, pe):
+            spage, sslot, pn, _ = (int(x) for x in pieces[k])
+            for i in range(pn):
+                assert writes.get((spage, sslot + i), chunk_of[t]) == chunk_of[t]
+    written = set()
+    for t in order:
         dpage, dslot, nrows, pb = (int(x) for x in tiles[t])
         pe = int(tiles[t + 1][3]) if t + 1 < len(tiles) else len(pieces)
         assert 0 < nrows <= tile_rows and dslot + nrows <= P
