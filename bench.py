@@ -1014,14 +1014,15 @@ def prefill_tile_flops(n, n_q, spans, G, Hkv, D):
     """FLOPs the tile loop issues (every 128 x 128 tile it computes, masked
     parts included) for one call: 4 x 128 x 128 x D per (query tile, key
     tile) pair; a CTA's two query tiles both run over the key tiles its
-    later tile reaches."""
+    later tile reaches.  Key tiles (pages of 64 tokens): the 64-key boxes
+    holding a visible key, two by two."""
     import numpy as np
     vis = np.ones(n, dtype=bool)
     for a, b in spans:
         vis[a:b] = False
-    n_kt = (n + 127) // 128
-    tile_has = np.array([vis[t * 128:(t + 1) * 128].any() for t in range(n_kt)])
-    key0 = np.nonzero(tile_has)[0] * 128
+    n_box = (n + 63) // 64
+    box_has = np.array([vis[b * 64:(b + 1) * 64].any() for b in range(n_box)])
+    key0 = (np.nonzero(box_has)[0] * 64)[::2]
     span = 2 * (128 // G)
     n_qt = (n_q + span - 1) // span
     total = 0

@@ -173,15 +173,16 @@ int sqh_plan_decode(void* c, const int32_t* handles, int32_t n, int32_t n_ctas,
 }
 
 // Plans a masked prefill over a sequence of n tokens (G = Hq / Hkv; spans as
-// start, end pairs).  info_out receives 6 int64 values: n_tiles, BP, n_qt,
-// n_split, visible_pairs, sizeof(PrefillTile).  If tiles_out is non-NULL,
-// up to `cap` tiles are written as 6 int32 each: key0, flags, vis[4]; if
-// qt_out is non-NULL, up to qt_cap per-query-tile tile counts.
-int sqh_plan_prefill(int32_t Hq, int32_t Hkv, int32_t n, int32_t n_q, const int32_t* spans,
-                     int32_t n_spans, int32_t target_ctas, int64_t* info_out, int32_t* tiles_out,
-                     int32_t cap, int32_t* qt_out, int32_t qt_cap) {
+// start, end pairs; page size P).  info_out receives 6 int64 values: n_tiles,
+// BP, n_qt, n_split, visible_pairs, sizeof(PrefillTile).  If tiles_out is
+// non-NULL, up to `cap` tiles are written as 7 int32 each: key0, flags,
+// vis[4], key0b; if qt_out is non-NULL, up to qt_cap per-query-tile counts.
+int sqh_plan_prefill(int32_t Hq, int32_t Hkv, int32_t P, int32_t n, int32_t n_q,
+                     const int32_t* spans, int32_t n_spans, int32_t target_ctas,
+                     int64_t* info_out, int32_t* tiles_out, int32_t cap, int32_t* qt_out,
+                     int32_t qt_cap) {
     Geometry g;
-    g.L = 1; g.Hq = Hq; g.Hkv = Hkv; g.D = 128; g.P = 64;
+    g.L = 1; g.Hq = Hq; g.Hkv = Hkv; g.D = 128; g.P = P;
     g.num_pages = 1; g.max_seqs = 1; g.max_pages_per_seq = 1;
     if (Hkv < 1 || Hq % Hkv != 0) return kInvalidArg;
     std::vector<int32_t> a(n_spans > 0 ? n_spans : 0), b(a.size());
@@ -199,10 +200,11 @@ int sqh_plan_prefill(int32_t Hq, int32_t Hkv, int32_t n, int32_t n_q, const int3
         const int32_t m = std::min<int32_t>(cap, (int32_t)p.tiles.size());
         for (int32_t i = 0; i < m; ++i) {
             const PrefillTile& t = p.tiles[i];
-            int32_t* o = tiles_out + 6 * i;
+            int32_t* o = tiles_out + 7 * i;
             o[0] = t.key0;
             o[1] = t.flags;
             for (int w = 0; w < 4; ++w) o[2 + w] = (int32_t)t.vis[w];
+            o[6] = t.key0b;
         }
     }
     if (qt_out) {

@@ -754,27 +754,55 @@ int plan_prefill(const Geometry& g, int32_t n, int32_t n_q, const int32_t* start
     }
     for (auto& ab : sp)
         for (int32_t j = ab.first; j < ab.second; ++j) vis[j >> 5] &= ~(1u << (j & 31));
-    for (int32_t t = 0; t < n_kt; ++t) {
-        PrefillTile tile{};
-        tile.key0 = t * kPrefillKeys;
-        bool any = false, full = true;
-        for (int w = 0; w < 4; ++w) {
-            tile.vis[w] = vis[(size_t)t * 4 + w];
-            any |= tile.vis[w] != 0;
-            full &= tile.vis[w] == 0xffffffffu;
+    auto box_full = [&](int32_t b) {   // 64 keys from b, all in the sequence and visible
+        return vis[(b >> 5)] == 0xffffffffu && vis[(b >> 5) + 1] == 0xffffffffu;
+    };
+    if (g.P >= 64) {
+        // the 64-key boxes with a visible key, two by two
+        std::vector<int32_t> boxes;
+        for (int32_t b = 0; b < n; b += 64)
+            if (vis[b >> 5] | vis[(b >> 5) + 1]) boxes.push_back(b);
+        for (size_t i = 0; i < boxes.size(); i += 2) {
+            PrefillTile tile{};
+            tile.key0 = boxes[i];
+            tile.key0b = i + 1 < boxes.size() ? boxes[i + 1] : kPrefillNoKeys;
+            tile.vis[0] = vis[tile.key0 >> 5];
+            tile.vis[1] = vis[(tile.key0 >> 5) + 1];
+            if (i + 1 < boxes.size()) {
+                tile.vis[2] = vis[tile.key0b >> 5];
+                tile.vis[3] = vis[(tile.key0b >> 5) + 1];
+            }
+            const bool full = i + 1 < boxes.size() && box_full(tile.key0) && box_full(tile.key0b);
+            tile.flags = full ? kPrefillTileFull : 0;
+            out->tiles.push_back(tile);
         }
-        if (!any) continue;
-        tile.flags = full ? kPrefillTileFull : 0;
-        out->tiles.push_back(tile);
+    } else {
+        for (int32_t t = 0; t < n_kt; ++t) {
+            PrefillTile tile{};
+            tile.key0 = t * kPrefillKeys;
+            tile.key0b = tile.key0 + 64;
+            bool any = false, full = true;
+            for (int w = 0; w < 4; ++w) {
+                tile.vis[w] = vis[(size_t)t * 4 + w];
+                any |= tile.vis[w] != 0;
+                full &= tile.vis[w] == 0xffffffffu;
+            }
+            if (!any) continue;
+            tile.flags = full ? kPrefillTileFull : 0;
+            out->tiles.push_back(tile);
+        }
     }
-    // the page of each TMA box (min(P, 64) rows) of each listed tile
+    // the page of each TMA box (min(P, 64) rows) of each listed tile: the
+    // first half's boxes from key0, the second half's from key0b
     const int32_t br = std::min(g.P, 64);
     out->n_pieces = kPrefillKeys / br;
     if (pages) {
+        const int32_t half = out->n_pieces / 2;
         out->tile_pages.resize(out->tiles.size() * out->n_pieces);
         for (size_t t = 0; t < out->tiles.size(); ++t)
             for (int32_t i = 0; i < out->n_pieces; ++i) {
-                const int32_t key = out->tiles[t].key0 + i * br;
+                const int64_t key = i < half ? (int64_t)out->tiles[t].key0 + i * br
+                                             : (int64_t)out->tiles[t].key0b + (i - half) * br;
                 out->tile_pages[t * out->n_pieces + i] = key < n ? pages[key / g.P] : -1;
             }
     }

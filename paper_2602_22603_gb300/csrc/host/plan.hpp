@@ -72,12 +72,21 @@ constexpr int kPrefillKeys = 128;
 constexpr int kPrefillQTiles = 2;
 constexpr int32_t kPrefillTileFull = 1;  // every key of the tile exists and is visible
 
-// One key tile that holds at least one visible key of the sequence.
+// One key tile that holds at least one visible key of the sequence: two
+// halves of 64 keys, each 64 consecutive positions starting at a multiple of
+// 64 (key0, key0b).  With pages of >= 64 tokens the halves are the visible
+// 64-key boxes of the sequence taken two by two, so a box that a span covers
+// entirely is skipped even when its neighbour is not; with smaller pages the
+// tile is 128 aligned keys (key0b = key0 + 64).  A missing second half has
+// key0b = kPrefillNoKeys (past any sequence).
+constexpr int32_t kPrefillNoKeys = 0x7fffffc0;
 struct PrefillTile {
-    int32_t key0;      // first key position (a multiple of kPrefillKeys)
+    int32_t key0;      // first key of the lower half
     int32_t flags;     // kPrefillTileFull or 0
-    uint32_t vis[4];   // bit c of word w: key key0 + 32 w + c exists and lies in no span
-    int32_t pad[2];
+    uint32_t vis[4];   // bit c of word w: key (w < 2 ? key0 : key0b) + 32 (w % 2) + c
+                       // exists and lies in no span
+    int32_t key0b;     // first key of the upper half
+    int32_t pad;
 };
 
 // Byte offsets of the arrays of a decode plan inside one upload buffer.

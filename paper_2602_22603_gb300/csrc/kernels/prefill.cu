@@ -152,19 +152,21 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
     const int br = a.P < 64 ? a.P : 64;  // rows of one TMA box
     const int n_pieces = a.n_pieces;      // <= 16
     constexpr int kBatch = 16;
-    // {first key, page of box 0, page of box 1} of key tile tb + lane % 16
+    // {first key of each half, page of box 0, page of box 1} of key tile
+    // tb + lane % 16 (x = key0, y = page 0, z = page 1, w = key0b)
     auto load_rec = [&](int tb) {
-        int4 r = make_int4(0, -1, -1, 0);
+        int4 r = make_int4(0, -1, -1, kPrefillNoKeys);
         const int jj = tb + (lane & (kBatch - 1));
         if (jj < T) {
             const size_t t = (size_t)(t0 + jj);
             r.x = __ldg(&a.tiles[t].key0);
+            r.w = __ldg(&a.tiles[t].key0b);
             r.y = __ldg(&a.tile_pages[t * n_pieces]);
             if (n_pieces > 1) r.z = __ldg(&a.tile_pages[t * n_pieces + 1]);
         }
         return r;
     };
-    int4 rec = make_int4(0, -1, -1, 0), pend = rec;
+    int4 rec = make_int4(0, -1, -1, kPrefillNoKeys), pend = rec;
     if (lane < kBatch) rec = load_rec(0);
     int fill_b = 1;    // the next batch to read
     int merge_b = -1;  // the batch read into `pend`, not yet in place
@@ -190,9 +192,14 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
         const int key0 = __shfl_sync(0xffffffffu, rec.x, j & 31);
         const int pg0 = __shfl_sync(0xffffffffu, rec.y, j & 31);
         const int pg1 = __shfl_sync(0xffffffffu, rec.z, j & 31);
+        const int key0b = __shfl_sync(0xffffffffu, rec.w, j & 31);
+        // rows of the tile inside the sequence (only the last tile has fewer
+        // than 128): the lower half's, then the upper half's
+        const int rows_b = key0b < a.n ? min(64, a.n - key0b) : 0;
+        const int rows = rows_b > 0 ? 64 + rows_b : min(64, a.n - key0);
         const int slot = u % C::kSlots;
         const int use = u / C::kSlots;
-        const bool vfix = lane < 2 && kv == 1 && key0 + kPrefillKeys > a.n;
+        const bool vfix = lane < 2 && kv == 1 && rows < kPrefillKeys;
         bool ok = true;
         if (lane < 2 && use > 0)
             ok = mbar_wait(sm.bar<D>(C::kBarEmpty + slot), (use - 1) & 1, abort_flag);
@@ -205,8 +212,7 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
             break;
         }
         if (lane < 2) {
-            int nv = (a.n - key0 + br - 1) / br;  // boxes inside the sequence
-            nv = nv < n_pieces ? nv : n_pieces;
+            const int nv = (rows + br - 1) / br;  // boxes inside the sequence (a prefix)
             const uint32_t fb = vfix ? sm.bar<D>(C::kBarVfix) : sm.bar<D>(C::kBarFull + slot);
             mbar_arrive_expect_tx(fb, (uint32_t)nv * br * 128 * C::kColBlocks);
             const uint32_t dst = sm.base + C::kOffRing + slot * C::kSlotBytes;
@@ -223,7 +229,8 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
                     set_error(a.err, kErrBounds);
                     page = 0;
                 }
-                const int key = key0 + i * br;
+                const int half = n_pieces / 2;
+                const int key = i < half ? key0 + i * br : key0b + (i - half) * br;
 #pragma unroll
                 for (int cb = 0; cb < C::kColBlocks; ++cb)
                     tma_load_4d(dst + cb * C::kBlockBytes + i * br * 128, pool_map, fb, cb * 64,
@@ -238,7 +245,7 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
             // is not, so zero those rows before the MMAs read the slot.
             const int src = __ffs(fix) - 1;
             const int fslot = __shfl_sync(0xffffffffu, slot, src);
-            const int fkey0 = __shfl_sync(0xffffffffu, key0, src);
+            const int frows = __shfl_sync(0xffffffffu, rows, src);
             tail_u = u0 + src;
             if (lane == 0) ok = mbar_wait(sm.bar<D>(C::kBarVfix), 0, abort_flag);
             if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) {
@@ -248,7 +255,7 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
                 }
                 break;
             }
-            const int r0 = a.n - fkey0;  // 1 .. 127
+            const int r0 = frows;  // 1 .. 127
             const int chunks = (kPrefillKeys - r0) * 8;
             uint8_t* vsp = sm.ptr + C::kOffRing + fslot * C::kSlotBytes;
             for (int cb = 0; cb < C::kColBlocks; ++cb)
@@ -526,8 +533,10 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
         // Raw logits q.k (the scale is applied inside the exponent; it is > 0),
         // taken 64 columns at a time to keep registers low: one pass for the
         // row maximum, one for the weights.
-        const int lim = p_row - key0;  // keys key0 + c with c <= lim are causal
-        const bool unmasked = valid && (w0.y & kPrefillTileFull) && lim >= kPrefillKeys - 1;
+        // keys key0 + c (lower half) and key0b + c (upper half) with c <= lim,
+        // c <= limb are causal
+        const int lim = p_row - key0, limb = p_row - w1.z;
+        const bool unmasked = valid && (w0.y & kPrefillTileFull) && lim >= 63 && limb >= 63;
         // Weights 2^(s * scale - m) with the running maximum m, two arguments
         // at a time with a packed FMA, rounded to bf16 into wt (32 words per
         // 64 keys); the normaliser sums the fp32 weights (four packed chains).
@@ -555,7 +564,8 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
 #pragma unroll
                     for (int w = 0; w < 2; ++w) {
                         const int ww = 2 * hh + w;
-                        const uint32_t mw = valid ? (vis[ww] & low_bits_through(lim - 32 * ww)) : 0u;
+                        const uint32_t mw =
+                            valid ? (vis[ww] & low_bits_through((ww < 2 ? lim : limb) - 32 * (ww & 1))) : 0u;
 #pragma unroll
                         for (int c = 0; c < 32; ++c)
                             if (!((mw >> c) & 1u)) x[32 * w + c] = 0xff800000u;  // -inf
@@ -607,7 +617,8 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
 #pragma unroll
                     for (int w = 0; w < 2; ++w) {
                         const int ww = 2 * hh + w;
-                        const uint32_t mw = valid ? (vis[ww] & low_bits_through(lim - 32 * ww)) : 0u;
+                        const uint32_t mw =
+                            valid ? (vis[ww] & low_bits_through((ww < 2 ? lim : limb) - 32 * (ww & 1))) : 0u;
 #pragma unroll
                         for (int c = 0; c < 32; ++c)
                             if (!((mw >> c) & 1u)) x[32 * w + c] = 0xff800000u;  // -inf

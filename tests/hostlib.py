@@ -47,24 +47,26 @@ def lib():
         L.sqh_peak_live_pages.restype = ctypes.c_int64
         L.sqh_plan_decode.argtypes = [P, I32P, I32, I32, I64P, ctypes.POINTER(ctypes.c_uint8),
                                       ctypes.c_int64]
-        L.sqh_plan_prefill.argtypes = [I32, I32, I32, I32, I32P, I32, I32, I64P, I32P, I32, I32P,
-                                       I32]
+        L.sqh_plan_prefill.argtypes = [I32, I32, I32, I32, I32, I32P, I32, I32, I64P, I32P, I32,
+                                       I32P, I32]
         _lib = L
     return _lib
 
 
-def plan_prefill(Hq, Hkv, n, n_q, spans, target_ctas=152, cap=1 << 16):
-    """(rc, info dict, tiles [k, 6] int64 array of key0, flags, vis[4])."""
+def plan_prefill(Hq, Hkv, n, n_q, spans, target_ctas=152, cap=1 << 16, P=64):
+    """(rc, info dict, tiles [k, 7] int64 array of key0, flags, vis[4], key0b)."""
     arr = (ctypes.c_int32 * max(2, 2 * len(spans)))(*[int(x) for ab in spans for x in ab])
     info = (ctypes.c_int64 * 6)()
-    tiles = (ctypes.c_int32 * (6 * cap))()
+    tiles = (ctypes.c_int32 * (7 * cap))()
     qt = (ctypes.c_int32 * cap)()
-    rc = lib().sqh_plan_prefill(Hq, Hkv, n, n_q, arr, len(spans), target_ctas, info, tiles, cap,
-                                qt, cap)
+    rc = lib().sqh_plan_prefill(Hq, Hkv, P, n, n_q, arr, len(spans), target_ctas, info, tiles,
+                                cap, qt, cap)
     d = dict(zip(("n_tiles", "BP", "n_qt", "n_split", "visible_pairs", "tile_bytes"), list(info)))
     d["qt_tiles"] = list(qt[: d["n_qt"]]) if rc == 0 else []
-    t = np.frombuffer(tiles, dtype=np.int32).reshape(-1, 6)[: d["n_tiles"] if rc == 0 else 0]
-    return rc, d, t.astype(np.int64) & 0xffffffff
+    t = np.frombuffer(tiles, dtype=np.int32).reshape(-1, 7)[: d["n_tiles"] if rc == 0 else 0]
+    t = t.astype(np.int64)
+    t[:, 1:6] &= 0xffffffff
+    return rc, d, t
 
 
 class HostCache:

@@ -387,17 +387,36 @@ def test_evict_tiles_compact_in_place(seed):
 # ---------------------------------------------------------------------------
 # masked prefill planning (Algorithm 2, BuildMask)
 # ---------------------------------------------------------------------------
-def _brute_prefill_plan(n, n_q, spans):
+NO_KEYS = 0x7fffffc0
+
+
+def _brute_prefill_plan(n, n_q, spans, P=64):
+    """Key tiles by their definition: with pages of >= 64 tokens, the 64-key
+    boxes holding a visible key, two by two; otherwise aligned 128-key tiles
+    holding one.  Each as (key0, full, vis words, key0b)."""
     removed = [False] * n
     for a, b in spans:
         for j in range(a, b):
             removed[j] = True
+
+    def bits_of(base):
+        return [base + c < n and not removed[base + c] for c in range(64)]
+
     tiles = []
-    for key0 in range(0, n, 128):
-        bits = [key0 + c < n and not removed[key0 + c] for c in range(128)]
-        if any(bits):
+    if P >= 64:
+        boxes = [b for b in range(0, n, 64) if any(bits_of(b))]
+        for i in range(0, len(boxes), 2):
+            lo = boxes[i]
+            hi = boxes[i + 1] if i + 1 < len(boxes) else NO_KEYS
+            bits = bits_of(lo) + (bits_of(hi) if hi != NO_KEYS else [False] * 64)
             words = [sum(1 << c for c in range(32) if bits[32 * w + c]) for w in range(4)]
-            tiles.append((key0, int(all(bits)), words))
+            tiles.append((lo, int(all(bits)), words, hi))
+    else:
+        for key0 in range(0, n, 128):
+            bits = bits_of(key0) + bits_of(key0 + 64)
+            if any(bits):
+                words = [sum(1 << c for c in range(32) if bits[32 * w + c]) for w in range(4)]
+                tiles.append((key0, int(all(bits)), words, key0 + 64))
     pairs = sum(sum(1 for j in range(p + 1) if not removed[j]) for p in range(n - n_q, n))
     return tiles, pairs
 
@@ -414,13 +433,14 @@ def test_prefill_plan_visibility_matches_brute_force(seed):
     cuts = sorted(rng.sample(range(n + 1), min(2 * k, n + 1)))
     spans = [(cuts[i], cuts[i + 1]) for i in range(0, len(cuts) - 1, 2) if cuts[i] < cuts[i + 1]]
     rng.shuffle(spans)
-    rc, info, tiles = plan_prefill(G * Hkv, Hkv, n, n_q, spans)
+    P = rng.choice([16, 64, 256])
+    rc, info, tiles = plan_prefill(G * Hkv, Hkv, n, n_q, spans, P=P)
     assert rc == 0
-    exp_tiles, exp_pairs = _brute_prefill_plan(n, n_q, spans)
+    exp_tiles, exp_pairs = _brute_prefill_plan(n, n_q, spans, P)
     assert info["tile_bytes"] == 32
     assert info["n_tiles"] == len(exp_tiles)
-    for got, (key0, full, words) in zip(tiles, exp_tiles):
-        assert got[0] == key0 and got[1] == full and list(got[2:]) == words
+    for got, (key0, full, words, key0b) in zip(tiles, exp_tiles):
+        assert got[0] == key0 and got[1] == full and list(got[2:6]) == words and got[6] == key0b
     assert info["visible_pairs"] == exp_pairs
     assert info["BP"] == 128 // G
     span = 2 * (128 // G)          # two query tiles per CTA
@@ -536,3 +556,18 @@ def test_prefill_slot_spans_on_partial_pages(seed):
             got.update(range(a, b))
         assert got == masked
     assert hc.prefill_slot_spans(m, tail, [(0, n + 1)])[0] == -1   # bad span
+
+
+def test_prefill_tiles_skip_boxes_a_span_covers():
+    """With 64-token pages a key tile pairs the visible 64-key boxes: a box
+    that a span covers entirely costs no tile half, even when its aligned
+    128-key neighbour is visible."""
+    from tests.hostlib import plan_prefill
+    rc, info, tiles = plan_prefill(8, 2, 512, 512, [(64, 128), (256, 384)], P=64)
+    assert rc == 0
+    # visible boxes 0, 128, 192, 384, 448 -> tiles (0, 128), (192, 384), (448, -)
+    assert [(int(t[0]), int(t[6])) for t in tiles] == [(0, 128), (192, 384), (448, NO_KEYS)]
+    assert all(int(t[1]) == 1 for t in tiles[:2]) and int(tiles[2][1]) == 0
+    # the same spans with 16-token pages keep aligned 128-key tiles
+    rc, info, tiles = plan_prefill(8, 2, 512, 512, [(64, 128), (256, 384)], P=16)
+    assert [int(t[0]) for t in tiles] == [0, 128, 384]
