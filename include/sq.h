@@ -289,6 +289,10 @@ typedef struct {
     int64_t prefill_calls;
     int64_t prefill_pairs;       /* visible (query, key) pairs per query head,
                                     summed over prefill calls */
+    int64_t decode_early_calls;  /* decode calls that loaded their first stages before
+                                    waiting for the preceding kernel */
+    int64_t decode_early_held;   /* pages those calls left for after the wait (a write
+                                    to them not yet known complete) */
 } sq_stats_t;
 
 SQ_API int sq_stats(sq_cache *cache, sq_stats_t *out);

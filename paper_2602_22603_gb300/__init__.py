@@ -58,7 +58,8 @@ class sq_stats_t(ctypes.Structure):
     _fields_ = [(name, ctypes.c_int64) for name in (
         "live_pages", "peak_live_pages", "decode_calls", "decode_logical_bytes",
         "decode_unique_bytes", "evict_calls", "evicted_tokens", "evict_moved_rows",
-        "evict_bytes", "appended_tokens", "cow_pages", "prefill_calls", "prefill_pairs")]
+        "evict_bytes", "appended_tokens", "cow_pages", "prefill_calls", "prefill_pairs",
+        "decode_early_calls", "decode_early_held")]
 
     def as_dict(self):
         return {name: int(getattr(self, name)) for name, _ in self._fields_}

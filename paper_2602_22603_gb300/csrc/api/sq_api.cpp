@@ -828,6 +828,8 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
             a.kv_early = 1;
             for (const auto& tp : hit->tick_top)
                 if (tp.first > c->write_done) a.unsafe[a.n_unsafe++] = tp.second;
+            c->stats.decode_early_calls += 1;
+            c->stats.decode_early_held += a.n_unsafe;
         }
     }
     c->debug_flags &= ~SQ_DEBUG_DROP_DECODE_STAGE;

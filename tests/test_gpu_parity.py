@@ -582,6 +582,7 @@ def test_decode_steps_reuse_plans_with_early_loads():
     keep.append(p.append(a, 30))
     seqs = [m, a]
     checks = []
+    st0 = p.cache.stats()
     for step in range(3):
         keep.append(p.append_batch(seqs))
         for layer in range(L):
@@ -593,5 +594,9 @@ def test_decode_steps_reuse_plans_with_early_loads():
         for out, layer, q_cpu, ns in checks:
             assert_budget(out, *p.oracle_decode_budget(seqs, layer, 0.09, q_cpu))
         checks.clear()
+    st1 = p.cache.stats()
+    # the calls after each step's first reused the plan and loaded early (in
+    # steps 1 and 2 at least: every earlier write had completed by then)
+    assert st1["decode_early_calls"] - st0["decode_early_calls"] >= 2 * (L - 1)
     assert p.cache.sync_status() == sq.SQ_OK
     p.close()
