@@ -747,6 +747,7 @@ def run_agent(args, world, rank, local):
     ev_bytes = cache.stats()["evict_bytes"] - b0
     assert cache.sync_status() == sq.SQ_OK
     hbm_peak, peak_kind = peaks()
+    tr_ratio, tr_src = recorded_traffic_ratio("sq_decode_splitk_kernel", "agent-32k")
     res = {
         "metric": METRIC, "value": round(tokens / wall, 3), "unit": "tokens/s",
         "n_gpus": 1, "steps": steps_main, "warmup": args.warmup,
@@ -777,7 +778,10 @@ def run_agent(args, world, rank, local):
             "ms_per_call": round(call_ms, 5),
             "timing": "CUDA events around the 32 layer calls of a main-thread step, "
                       "calls back to back on one stream, 32 steps",
-            "traffic": None,
+            "traffic": int(tr_ratio * call_bytes) if tr_ratio else None,
+            "traffic_source": (tr_src + ": DRAM bytes per algorithmic byte of captured calls of "
+                               "this workload, times this call's algorithmic bytes")
+                              if tr_ratio else None,
         },
         "clocks": clock_rec,
     }
@@ -959,6 +963,10 @@ def run_trace(args, world, rank, local):
     st1 = cache.stats()
     assert cache.sync_status() == sq.SQ_OK
     busy = sum(times.values())
+    tr_ratio, tr_src = recorded_traffic_ratio("sq_decode_splitk_kernel",
+                                              "ragged" if args.ragged else None)
+    call_bytes = (st1["decode_unique_bytes"] - st0["decode_unique_bytes"]) / max(
+        1, st1["decode_calls"] - st0["decode_calls"])
     res = {
         "metric": METRIC, "value": round(decoded / wall, 3), "unit": "tokens/s", "n_gpus": 1,
         "steps": T * 256, "warmup": 0, "ms_per_step": round(wall * 1e3 / (T * 256), 4),
@@ -994,7 +1002,11 @@ def run_trace(args, world, rank, local):
                               (times["attention"] / 1e3) / 1e9, 1),
             "peak": peaks()[0], "peak_kind": peaks()[1], "unit": "GB/s",
             "timing": "CUDA events around each step's 32 layer calls",
-            "traffic": None,
+            "traffic": int(tr_ratio * call_bytes) if tr_ratio else None,
+            "traffic_source": (tr_src + ": small-case DRAM bytes per algorithmic byte of the same "
+                               "kernel (%s), times the mean call's algorithmic bytes"
+                               % ("partial pages after a ragged eviction" if args.ragged
+                                  else "dense pages")) if tr_ratio else None,
         },
         "clocks": clock_rec,
     }
