@@ -236,10 +236,10 @@ def test_decode_replayed_from_a_cuda_graph():
     p.close()
 
 
-@pytest.mark.parametrize("seed", range(4))
+@pytest.mark.parametrize("seed", range(5))
 def test_random_forks_appends_evictions(seed):
     rng = random.Random(seed)
-    P = rng.choice([16, 64])
+    P = (8, 16, 32, 64, 256)[seed]
     D = rng.choice([64, 128])
     G = rng.choice([1, 4, 8])
     Hkv = rng.choice([1, 2, 4])

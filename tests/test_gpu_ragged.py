@@ -75,10 +75,10 @@ def test_tiny_workload_ragged():
     p.close()
 
 
-@pytest.mark.parametrize("seed", range(6))
+@pytest.mark.parametrize("seed", range(12))
 def test_random_ops_with_ragged_evictions(seed):
     rng = random.Random(seed)
-    P = rng.choice([8, 16, 64, 128])
+    P = (8, 16, 32, 64, 128, 256)[seed % 6]   # every page size twice
     D = rng.choice([64, 128])
     G = rng.choice([1, 4, 8])
     Hkv = 2
