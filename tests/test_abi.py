@@ -77,3 +77,39 @@ def test_binding_fails_loudly_without_the_library():
     r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, timeout=300,
                        cwd=os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
     assert r.stdout.strip() == "raised True", r.stdout + r.stderr
+
+
+_CTYPES = {"int32_t": ctypes.c_int32, "int64_t": ctypes.c_int64, "uint32_t": ctypes.c_uint32,
+           "float": ctypes.c_float, "void*": ctypes.c_void_p}
+
+
+def header_struct(name):
+    """Fields of `typedef struct { ... } name;` in include/sq.h, as (type, field)
+    pairs in declaration order (one declaration per line; comments dropped)."""
+    text = re.sub(r"/\*.*?\*/", " ", open(HEADER).read(), flags=re.S)
+    m = re.search(r"typedef\s+struct\s*\{([^}]*)\}\s*" + name + r"\s*;", text)
+    assert m, name
+    out = []
+    for decl in m.group(1).split(";"):
+        decl = " ".join(decl.split())
+        if not decl:
+            continue
+        mt = re.fullmatch(r"(\w+)\s*(\*?)\s*(\w+)", decl)
+        assert mt, decl
+        out.append((mt.group(1) + mt.group(2), mt.group(3)))
+    return out
+
+
+@pytest.mark.parametrize("c_name,py_struct", [("sq_config", sq.sq_config), ("sq_span", sq.sq_span),
+                                               ("sq_stats_t", sq.sq_stats_t)])
+def test_binding_structs_match_the_header(c_name, py_struct):
+    """The binding's ctypes structures have the header's fields, in order and
+    of the same types, so that a call that fills one (sq_stats copies the
+    whole struct) never writes past the caller's buffer."""
+    fields = header_struct(c_name)
+    assert [f for _, f in fields] == [n for n, _ in py_struct._fields_]
+    # the same field types in the same order give the same layout: ctypes lays
+    # a Structure out by the platform's C rules
+    for (ctype, fname), (_, pytype) in zip(fields, py_struct._fields_):
+        assert ctypes.sizeof(_CTYPES[ctype]) == ctypes.sizeof(pytype), fname
+        assert ctypes.alignment(_CTYPES[ctype]) == ctypes.alignment(pytype), fname
