@@ -113,3 +113,53 @@ def test_binding_structs_match_the_header(c_name, py_struct):
     for (ctype, fname), (_, pytype) in zip(fields, py_struct._fields_):
         assert ctypes.sizeof(_CTYPES[ctype]) == ctypes.sizeof(pytype), fname
         assert ctypes.alignment(_CTYPES[ctype]) == ctypes.alignment(pytype), fname
+
+
+def _c_kind(decl):
+    """Class of a C parameter or return type: ptr, i32, i64, f32 or size."""
+    decl = " ".join(decl.replace("const", " ").split())
+    if "*" in decl:
+        return "ptr"
+    base = decl.split()[0]
+    return {"int": "i32", "int32_t": "i32", "sq_seq": "i32", "int64_t": "i64", "float": "f32",
+            "size_t": "size"}[base]
+
+
+def _py_kind(t):
+    if t in (ctypes.c_void_p, ctypes.c_char_p) or hasattr(t, "_type_") and issubclass(
+            t, ctypes._Pointer):
+        return "ptr"
+    if t in (ctypes.c_int32, ctypes.c_int):
+        return "i32"
+    if t is ctypes.c_int64:
+        return "i64"
+    if t is ctypes.c_float:
+        return "f32"
+    if t is ctypes.c_size_t:
+        return "size"
+    raise AssertionError(t)
+
+
+def header_prototypes():
+    text = re.sub(r"/\*.*?\*/", " ", open(HEADER).read(), flags=re.S)
+    out = {}
+    for m in re.finditer(r"^SQ_API\s+([\w\s\*]*?)\b(sq_\w+)\s*\(([^)]*)\)\s*;", text, flags=re.M):
+        params = [p.strip() for p in m.group(3).split(",") if p.strip() and p.strip() != "void"]
+        # drop each parameter's name: the type is everything before the last word
+        types = [re.sub(r"\b\w+\s*$", "", p).strip() or p for p in params]
+        out[m.group(2)] = (m.group(1).strip(), types)
+    return out
+
+
+def test_binding_signatures_match_the_header():
+    """Every declared function has the binding's argument count, and each
+    argument and the result the same class (pointer, 32/64-bit integer,
+    float, size_t), so that ctypes marshals the call as C expects."""
+    protos = header_prototypes()
+    assert set(protos) == set(declared_functions())
+    for name, (ret, params) in protos.items():
+        res, args = sq._SIGS[name]
+        assert len(args) == len(params), name
+        assert _py_kind(res) == _c_kind(ret), name
+        for i, (p, a) in enumerate(zip(params, args)):
+            assert _c_kind(p) == _py_kind(a), (name, i, p)
