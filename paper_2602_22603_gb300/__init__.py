@@ -59,7 +59,7 @@ class sq_stats_t(ctypes.Structure):
         "live_pages", "peak_live_pages", "decode_calls", "decode_logical_bytes",
         "decode_unique_bytes", "evict_calls", "evicted_tokens", "evict_moved_rows",
         "evict_bytes", "appended_tokens", "cow_pages", "prefill_calls", "prefill_pairs",
-        "decode_early_calls", "decode_early_held")]
+        "decode_early_calls", "decode_early_held", "decode_plans_built")]
 
     def as_dict(self):
         return {name: int(getattr(self, name)) for name, _ in self._fields_}

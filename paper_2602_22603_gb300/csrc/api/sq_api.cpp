@@ -531,6 +531,83 @@ int sq_fork_aux(sq_cache* c, sq_seq parent, sq_seq* child_out) {
     return c->host->fork(parent, child_out);
 }
 
+// Cached decode plans an append leaves valid.  An append that stays inside
+// a sequence's last page (no new page, no copy-on-write) and inside its last
+// 64-token stage changes, for a plan holding that sequence, only the
+// sequence's length: the stages, the CTA split and every page stay as they
+// were.  The append kernel then rewrites that length in the plan, after the
+// plan's last decode on the same stream, and the plan takes the sequence's new
+// version.  Plans last used on another stream, plans with page fills, and
+// pages of fewer than 64 tokens (a stage spans pages) are rebuilt instead.
+struct LenUpdate {
+    PlanEntry* e;
+    int32_t i;     // call-local index of the sequence in the plan
+    int32_t val;   // its new end in slot space
+};
+
+static void plan_len_updates(sq_cache* c, sq_seq seq, const AppendPlan& ap, uint64_t old_version,
+                             cudaStream_t st, std::vector<LenUpdate>* out) {
+    if (c->g.P % kStageTokens != 0 || ap.cow || !ap.taken.empty() || ap.n_new < 1) return;
+    const int64_t e0 = ap.pos0, e1 = (int64_t)ap.pos0 + ap.n_new;
+    if ((e0 + kStageTokens - 1) / kStageTokens != (e1 + kStageTokens - 1) / kStageTokens) return;
+    for (auto& e : c->plans) {
+        if (!e.valid || e.lay.page_fill >= 0 || !e.ev_recorded || e.ev_stream != st) continue;
+        for (size_t i = 0; i < e.handles.size(); ++i)
+            if (e.handles[i] == seq && e.versions[i] == old_version)
+                out->push_back({&e, (int32_t)i, (int32_t)e1});
+    }
+}
+
+// Up to kAppendLenMax of `ups` (from index `from`) into the kernel's list;
+// returns how many were taken.
+static size_t fill_lens(const std::vector<LenUpdate>& ups, size_t from, AppendLens* l) {
+    l->n = 0;
+    size_t k = from;
+    for (; k < ups.size() && l->n < kAppendLenMax; ++k) {
+        const LenUpdate& u = ups[k];
+        l->ptr[l->n] = reinterpret_cast<int32_t*>(u.e->d_plan + u.e->lay.seq_len) + u.i;
+        l->val[l->n] = u.val;
+        ++l->n;
+    }
+    return k - from;
+}
+
+// After the append's launches: the updated plans take the sequence's new
+// version, count its new rows, list the written page among their newest
+// writes, and count the append as their last use on the stream.
+static void plan_len_apply(sq_cache* c, const LenUpdate& u, uint64_t new_version, int32_t n_new,
+                           int32_t page, cudaStream_t st) {
+    PlanEntry& e = *u.e;
+    e.versions[u.i] = new_version;
+    e.unique_tokens += n_new;
+    e.logical_tokens += n_new;
+    const uint64_t t = c->page_ticket[page];
+    bool found = false;
+    for (auto& tp : e.tick_top)
+        if (tp.second == page) {
+            tp.first = std::max(tp.first, t);
+            found = true;
+        }
+    if (!found) {
+        e.tick_top.push_back({t, page});
+        if (e.tick_top.size() > (size_t)kDecodeMaxUnsafe) {
+            auto oldest = std::min_element(
+                e.tick_top.begin(), e.tick_top.end(),
+                [](const std::pair<uint64_t, int32_t>& x, const std::pair<uint64_t, int32_t>& y) {
+                    return x.first < y.first;
+                });
+            e.tick_rest = std::max(e.tick_rest, oldest->first);
+            e.tick_top.erase(oldest);
+        }
+    }
+    // the plan's buffer is written by this append: it is reused (or replaced)
+    // only after it
+    if (cudaEventRecord(e.ev, st) != cudaSuccess) {
+        cudaGetLastError();
+        e.valid = false;
+    }
+}
+
 int sq_append_kv(sq_cache* c, sq_seq seq, int32_t n_tokens, const void* k, const void* v,
                  void* stream) {
     TraceRange trace_("sq_append_kv");
@@ -541,6 +618,7 @@ int sq_append_kv(sq_cache* c, sq_seq seq, int32_t n_tokens, const void* k, const
     if (!k || !v || (reinterpret_cast<uintptr_t>(k) & 15) || (reinterpret_cast<uintptr_t>(v) & 15))
         return SQ_ERR_INVALID_ARG;
     AppendPlan plan;
+    const uint64_t old_version = c->host->seq(seq)->version;
     int rc = c->host->append(seq, n_tokens, &plan);
     if (rc != SQ_OK) return rc;
     const Geometry& g = c->g;
@@ -549,6 +627,9 @@ int sq_append_kv(sq_cache* c, sq_seq seq, int32_t n_tokens, const void* k, const
         c->host->undo_append(seq, plan);
         return code;
     };
+    std::vector<LenUpdate> ups;
+    plan_len_updates(c, seq, plan, old_version, st, &ups);
+    size_t n_ups = 0;  // of them, passed to the kernel
     rc = fence_taken_pages(c, plan.taken, stream);
     if (rc != SQ_OK) return undo(rc);
     if (plan.cow) {
@@ -583,11 +664,17 @@ int sq_append_kv(sq_cache* c, sq_seq seq, int32_t n_tokens, const void* k, const
         a.pos0 = (int32_t)pb;
         a.tok_begin = (int32_t)(pb - plan.pos0);
         a.n_tok = (int32_t)(pe - pb);
+        a.lens.n = 0;
+        if (b == 0) n_ups = fill_lens(ups, 0, &a.lens);  // an in-page append is one launch
         a.err = c->d_err;
         cudaError_t e = launch_append(a, c->num_sms, st);
         if (e != cudaSuccess) return undo(cuda_status(e));
     }
     note_writes(c, plan.pages.data(), plan.pages.size(), stream);
+    {
+        const uint64_t nv = c->host->seq(seq)->version;
+        for (size_t k = 0; k < n_ups; ++k) plan_len_apply(c, ups[k], nv, plan.n_new, plan.pages[0], st);
+    }
     c->host->seq_mut(seq)->last_stream = stream;
     c->stats.appended_tokens += n_tokens;
     if (plan.cow) c->stats.cow_pages += 1;
@@ -614,12 +701,20 @@ int sq_append_kv_batch(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, const vo
         return code;
     };
     std::vector<int32_t> taken;
+    std::vector<uint64_t> old_versions(n_seqs);
     for (int32_t i = 0; i < n_seqs; ++i) {
+        old_versions[i] = c->host->seq(seqs[i])->version;
         int rc = c->host->append(seqs[i], 1, &plans[i]);
         if (rc != SQ_OK) return undo(i, rc);
         taken.insert(taken.end(), plans[i].taken.begin(), plans[i].taken.end());
     }
     cudaStream_t st = as_stream(stream);
+    // the plans each sequence's append leaves valid, and which of them the
+    // launch writing that sequence's row could take
+    std::vector<std::vector<LenUpdate>> ups(n_seqs);
+    std::vector<size_t> n_ups(n_seqs, 0);
+    for (int32_t i = 0; i < n_seqs; ++i)
+        plan_len_updates(c, seqs[i], plans[i], old_versions[i], st, &ups[i]);
     int rc = fence_taken_pages(c, taken, stream);
     if (rc != SQ_OK) return undo(n_seqs, rc);
     for (int32_t i = 0; i < n_seqs; ++i) {
@@ -645,10 +740,22 @@ int sq_append_kv_batch(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, const vo
         a.n_total = n_seqs;
         a.row0 = b;
         a.n = std::min(kAppendBatchMax, n_seqs - b);
+        AppendLens& l = a.lens;
+        l.n = 0;
         for (int32_t i = 0; i < a.n; ++i) {
             const AppendPlan& pl = plans[b + i];
             a.page[i] = pl.pages[0];                 // the page holding slot position pos0
             a.slot[i] = pl.pos0 % g.P;
+            // a sequence's plan updates go all into this launch, or none do
+            if (l.n + ups[b + i].size() <= (size_t)kAppendLenMax) {
+                AppendLens part;
+                n_ups[b + i] = fill_lens(ups[b + i], 0, &part);
+                for (int32_t k = 0; k < part.n; ++k) {
+                    l.ptr[l.n] = part.ptr[k];
+                    l.val[l.n] = part.val[k];
+                    ++l.n;
+                }
+            }
         }
         a.err = c->d_err;
         cudaError_t e = launch_append_batch(a, c->num_sms, st);
@@ -658,6 +765,11 @@ int sq_append_kv_batch(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, const vo
         std::vector<int32_t> written(n_seqs);
         for (int32_t i = 0; i < n_seqs; ++i) written[i] = plans[i].pages[0];
         note_writes(c, written.data(), written.size(), stream);
+    }
+    for (int32_t i = 0; i < n_seqs; ++i) {
+        const uint64_t nv = c->host->seq(seqs[i])->version;
+        for (size_t k = 0; k < n_ups[i]; ++k)
+            plan_len_apply(c, ups[i][k], nv, 1, plans[i].pages[0], st);
     }
     for (int32_t i = 0; i < n_seqs; ++i) {
         c->host->seq_mut(seqs[i])->last_stream = stream;
@@ -758,6 +870,7 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
         plan_serialize(plan, lay, c->staging.data());
         int urc = staged_copy(c, victim->d_plan, c->staging.data(), lay.total, stream);
         if (urc != SQ_OK) { victim->valid = false; return urc; }
+        c->stats.decode_plans_built += 1;
         victim->valid = true;
         victim->n_ctas = c->decode_ctas;
         victim->handles.assign(seqs, seqs + n_seqs);
@@ -801,6 +914,7 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
     a.page_ids = reinterpret_cast<const int32_t*>(hit->d_plan + L.page_ids);
     a.comb_off = reinterpret_cast<const int32_t*>(hit->d_plan + L.comb_off);
     a.arrive = reinterpret_cast<unsigned int*>(hit->d_plan + L.arrive);
+    a.seq_len = reinterpret_cast<const int32_t*>(hit->d_plan + L.seq_len);
     a.page_fill = L.page_fill >= 0 ? reinterpret_cast<const int32_t*>(hit->d_plan + L.page_fill)
                                    : nullptr;
     a.q = reinterpret_cast<const __nv_bfloat16*>(q);
@@ -1351,6 +1465,7 @@ int sq_decode_attention_noalloc(sq_cache* c, const sq_seq* seqs, int32_t n_seqs,
     a.page_ids = reinterpret_cast<const int32_t*>(scratch + L.page_ids);
     a.comb_off = reinterpret_cast<const int32_t*>(scratch + L.comb_off);
     a.arrive = reinterpret_cast<unsigned int*>(scratch + L.arrive);
+    a.seq_len = reinterpret_cast<const int32_t*>(scratch + L.seq_len);
     a.page_fill = L.page_fill >= 0 ? reinterpret_cast<const int32_t*>(scratch + L.page_fill)
                                    : nullptr;
     a.q = reinterpret_cast<const __nv_bfloat16*>(q);

@@ -519,6 +519,7 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
             if (ss[j] == ss[i]) return kInvalidArg;
         out->logical_tokens += ss[i]->n;
         ragged = ragged || has_partial_pages(*ss[i], g.P);
+        out->seq_len.push_back((int32_t)slot_end(*ss[i], g.P));
     }
     const int32_t P = g.P;
     const int32_t max_grp = kRowsPerTile / g.G();
@@ -589,6 +590,7 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
                 seg.n_pages = q_end - q0;
                 seg.n_grp = (int32_t)std::min<size_t>(max_grp, part.size() - b);
                 seg.n_tok = 0;
+                seg.q0 = q0;
                 for (int32_t j = 0; j < seg.n_grp; ++j) {
                     int32_t i = part[b + j];
                     // slot-space limit of this member inside the run
@@ -718,6 +720,8 @@ DecodePlanLayout plan_layout(const DecodePlanHost& p, int32_t n_seqs, int32_t Hk
     } else {
         L.page_fill = -1;
     }
+    L.n_seqs = n_seqs;
+    L.seq_len = o;   o = align16(o + sizeof(int32_t) * n_seqs);
     L.total = o;
     return L;
 }
@@ -731,6 +735,7 @@ void plan_serialize(const DecodePlanHost& p, const DecodePlanLayout& L, uint8_t*
     std::memcpy(dst + L.comb_off, p.comb_off.data(), sizeof(int32_t) * (L.n_comb_keys + 1));
     if (L.page_fill >= 0)
         std::memcpy(dst + L.page_fill, p.page_fill.data(), sizeof(int32_t) * L.n_page_ids);
+    std::memcpy(dst + L.seq_len, p.seq_len.data(), sizeof(int32_t) * L.n_seqs);
 }
 
 // ---------------------------------------------------------------------------

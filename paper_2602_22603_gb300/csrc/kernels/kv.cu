@@ -17,8 +17,15 @@ __device__ __forceinline__ int64_t row_offset(int64_t num_pages, int Hkv, int P,
     return (((((int64_t)layer * num_pages + page) * 2 + kv) * Hkv + head) * P + slot) * (int64_t)D;
 }
 
+// The new lengths of the appended sequences, into the cached decode plans
+// that stay valid (block 0; read by later kernels of the stream).
+__device__ __forceinline__ void write_lens(const AppendLens& l) {
+    if (blockIdx.x == 0 && threadIdx.x < l.n) *l.ptr[threadIdx.x] = l.val[threadIdx.x];
+}
+
 // ---- append (Algorithm 1: C <- C + R, C <- C + O) ---------------------------
 __global__ void __launch_bounds__(256) sq_append_kv_kernel(const AppendArgs a) {
+    write_lens(a.lens);
     const int vpr = a.D / 8;  // 16-byte vectors per row
     const int64_t total = (int64_t)a.L * a.n_tok * 2 * a.Hkv * vpr;
     for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
@@ -44,6 +51,7 @@ __global__ void __launch_bounds__(256) sq_append_kv_kernel(const AppendArgs a) {
 
 // ---- one new token for each of a batch of sequences --------------------------
 __global__ void __launch_bounds__(256) sq_append_kv_batch_kernel(const AppendBatchArgs a) {
+    write_lens(a.lens);
     const int vpr = a.D / 8;
     const int64_t total = (int64_t)a.L * a.n * 2 * a.Hkv * vpr;
     for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;

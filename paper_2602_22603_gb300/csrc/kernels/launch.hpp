@@ -25,6 +25,10 @@ struct DecodeArgs {
     const int32_t* page_fill;
     const int32_t* comb_off;    // [n_seqs * Hkv + 1] partial entries of each (sequence, KV head)
     unsigned int* arrive;       // [n_seqs * Hkv] arrival counts, zero between calls
+    // [n_seqs] each sequence's end in slot space; an append kernel may have
+    // rewritten it since the plan was uploaded, so it is read after the
+    // grid-dependency wait
+    const int32_t* seq_len;
     const __nv_bfloat16* q;     // [n_seqs][Hq][D]
     void* out;                  // [n_seqs][Hq][D] bf16 or fp32
     float* part_o;              // [n_ent][G][D]  unnormalised partial outputs
@@ -94,6 +98,15 @@ cudaError_t launch_prefill_combine(const PrefillCombineArgs& a, int D, cudaStrea
 // ---- append / copy-on-write / eviction --------------------------------------
 constexpr int kAppendMaxPages = 64;
 
+// Sequence lengths in cached decode plans that an append rewrites (in stream
+// order, by block 0): plans that the append leaves valid (see the API layer).
+constexpr int kAppendLenMax = 32;
+struct AppendLens {
+    int32_t n;
+    int32_t* ptr[kAppendLenMax];
+    int32_t val[kAppendLenMax];
+};
+
 struct AppendArgs {
     __nv_bfloat16* pool;
     const __nv_bfloat16* k;     // [L][n_total][Hkv][D]
@@ -107,6 +120,7 @@ struct AppendArgs {
     int32_t page_index0;        // logical page index of pages[0]
     int32_t n_pages;
     int32_t pages[kAppendMaxPages];
+    AppendLens lens;
     int* err;
 };
 
@@ -124,6 +138,7 @@ struct AppendBatchArgs {
     int32_t n;                  // rows this launch writes
     int32_t page[kAppendBatchMax];
     int32_t slot[kAppendBatchMax];
+    AppendLens lens;
     int* err;
 };
 

@@ -583,7 +583,12 @@ def test_decode_steps_reuse_plans_with_early_loads():
     seqs = [m, a]
     checks = []
     st0 = p.cache.stats()
+    rebuilds = 0
     for step in range(3):
+        # a plan is built for the first step, and again only when an append
+        # opens a page (P = 64: also a 64-token stage) of some sequence
+        if step == 0 or any(p.oracle.n_tokens(p.o[h]) % 64 == 0 for h in seqs):
+            rebuilds += 1
         keep.append(p.append_batch(seqs))
         for layer in range(L):
             q_cpu, q = _q(900 + 10 * step + layer, 2, 32, 128)
@@ -598,5 +603,38 @@ def test_decode_steps_reuse_plans_with_early_loads():
     # the calls after each step's first reused the plan and loaded early (in
     # steps 1 and 2 at least: every earlier write had completed by then)
     assert st1["decode_early_calls"] - st0["decode_early_calls"] >= 2 * (L - 1)
+    # the batched appends inside both sequences' last pages kept the plan
+    # (the fork's third append opens a page: 20,032 rows before it)
+    assert st1["decode_plans_built"] - st0["decode_plans_built"] == rebuilds == 2
+    assert p.cache.sync_status() == sq.SQ_OK
+    p.close()
+
+
+@pytest.mark.parametrize("P", [64, 128])
+def test_decode_plan_survives_in_page_appends(P):
+    """One-token appends (sq_append_kv) between decode steps: an append
+    inside the sequence's last page and 64-token stage keeps the cached plan
+    (the append kernel rewrites the sequence's length in it), one that opens
+    a page or a stage has it rebuilt; every output equals the oracle."""
+    L = 3
+    p = Pair(L, 16, 4, 64, P, num_pages=400, seed=91)
+    keep = []
+    m = p.seq_new()
+    keep.append(p.append(m, 4 * 64 + 58))   # the 6th step's append starts at 320
+    st0 = p.cache.stats()
+    rebuilds = 1                             # the first step plans
+    for step in range(10):
+        n_before = p.oracle.n_tokens(p.o[m])
+        if step > 0 and n_before % 64 == 0:  # a new 64-token stage (for P = 64 a new page)
+            rebuilds += 1
+        keep.append(p.append(m, 1))
+        for layer in range(L):
+            q_cpu, q = _q(1300 + 10 * step + layer, 1, 16, 64)
+            keep.append(q)
+            out = p.decode([m], layer, 0.125, q, sq.SQ_OUT_F32)
+            torch.cuda.synchronize()
+            assert_budget(out, *p.oracle_decode_budget([m], layer, 0.125, q_cpu))
+    st1 = p.cache.stats()
+    assert st1["decode_plans_built"] - st0["decode_plans_built"] == rebuilds == 2
     assert p.cache.sync_status() == sq.SQ_OK
     p.close()
