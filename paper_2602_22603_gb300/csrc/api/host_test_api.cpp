@@ -149,11 +149,10 @@ int sqh_free_count(void* c) { return static_cast<HostCache*>(c)->alloc().free_co
 
 int64_t sqh_peak_live_pages(void* c) { return static_cast<HostCache*>(c)->peak_live_pages(); }
 
-// Plans a decode call.  layout_out receives 18 int64 values:
+// Plans a decode call.  layout_out receives 17 int64 values:
 //   offsets segs, items, cta_begin, page_ids, comb_off, arrive, total,
 //   counts n_segs, n_items, n_ctas, n_page_ids, n_comb_keys, n_comb_ent,
-//   unique_tokens, logical_tokens, sizeof(DecodeSeg), offset page_fill (-1: none),
-//   offset seq_len.
+//   unique_tokens, logical_tokens, sizeof(DecodeSeg), offset page_fill (-1: none).
 // If buf is non-NULL and buf_bytes >= total, the serialised plan is written.
 int sqh_plan_decode(void* c, const int32_t* handles, int32_t n, int32_t n_ctas,
                     int64_t* layout_out, uint8_t* buf, int64_t buf_bytes) {
@@ -162,10 +161,9 @@ int sqh_plan_decode(void* c, const int32_t* handles, int32_t n, int32_t n_ctas,
     int rc = plan_decode(*hc, handles, n, n_ctas, &p);
     if (rc != kOk) return rc;
     DecodePlanLayout L = plan_layout(p, n, hc->geom().Hkv);
-    int64_t v[18] = {L.segs, L.items, L.cta_begin, L.page_ids, L.comb_off, L.arrive, L.total,
+    int64_t v[17] = {L.segs, L.items, L.cta_begin, L.page_ids, L.comb_off, L.arrive, L.total,
                      L.n_segs, L.n_items, L.n_ctas, L.n_page_ids, L.n_comb_keys, L.n_comb_ent,
-                     p.unique_tokens, p.logical_tokens, (int64_t)sizeof(DecodeSeg), L.page_fill,
-                     L.seq_len};
+                     p.unique_tokens, p.logical_tokens, (int64_t)sizeof(DecodeSeg), L.page_fill};
     std::memcpy(layout_out, v, sizeof v);
     if (buf) {
         if (buf_bytes < L.total) return kInvalidArg;

@@ -8,6 +8,7 @@
 #include <nvtx3/nvToolsExt.h>
 
 #include <algorithm>
+#include <cstddef>
 #include <cstring>
 #include <deque>
 #include <memory>
@@ -47,6 +48,9 @@ struct PlanEntry {
     // all other pages
     std::vector<std::pair<uint64_t, int32_t>> tick_top;
     uint64_t tick_rest = 0;
+    // per call-local sequence: the segment holding its last page when that
+    // segment has it alone (else -1), and the slot-space start of that run
+    std::vector<int32_t> tail_seg, tail_base;
     uint8_t* d_plan = nullptr;
     size_t plan_cap = 0;
     float* d_part = nullptr;
@@ -533,16 +537,19 @@ int sq_fork_aux(sq_cache* c, sq_seq parent, sq_seq* child_out) {
 
 // Cached decode plans an append leaves valid.  An append that stays inside
 // a sequence's last page (no new page, no copy-on-write) and inside its last
-// 64-token stage changes, for a plan holding that sequence, only the
-// sequence's length: the stages, the CTA split and every page stay as they
-// were.  The append kernel then rewrites that length in the plan, after the
-// plan's last decode on the same stream, and the plan takes the sequence's new
-// version.  Plans last used on another stream, plans with page fills, and
-// pages of fewer than 64 tokens (a stage spans pages) are rebuilt instead.
+// 64-token stage changes, for a plan holding that sequence, only the row
+// limit of the run holding that page: the stages, the CTA split and every
+// page stay as they were.  The page is the sequence's alone (else it would
+// have been copied on write), so that run's segment has it as its one member
+// and the limit is two words of the segment (its token count and the member's
+// limit).  The append kernel rewrites them, after the plan's last decode on
+// the same stream, and the plan takes the sequence's new version.  Plans
+// last used on another stream, plans with page fills, and pages of fewer than
+// 64 tokens (a stage spans pages) are rebuilt instead.
 struct LenUpdate {
     PlanEntry* e;
     int32_t i;     // call-local index of the sequence in the plan
-    int32_t val;   // its new end in slot space
+    int32_t val;   // the new row limit of its last run (end in slot space - run start)
 };
 
 static void plan_len_updates(sq_cache* c, sq_seq seq, const AppendPlan& ap, uint64_t old_version,
@@ -553,21 +560,24 @@ static void plan_len_updates(sq_cache* c, sq_seq seq, const AppendPlan& ap, uint
     for (auto& e : c->plans) {
         if (!e.valid || e.lay.page_fill >= 0 || !e.ev_recorded || e.ev_stream != st) continue;
         for (size_t i = 0; i < e.handles.size(); ++i)
-            if (e.handles[i] == seq && e.versions[i] == old_version)
-                out->push_back({&e, (int32_t)i, (int32_t)e1});
+            if (e.handles[i] == seq && e.versions[i] == old_version && e.tail_seg[i] >= 0)
+                out->push_back({&e, (int32_t)i, (int32_t)(e1 - e.tail_base[i])});
     }
 }
 
-// Up to kAppendLenMax of `ups` (from index `from`) into the kernel's list;
-// returns how many were taken.
+// The kernel's writes for `ups` (from index `from`): the run's token count
+// and its one member's limit, two words each, as many as fit; returns how
+// many updates were taken.
 static size_t fill_lens(const std::vector<LenUpdate>& ups, size_t from, AppendLens* l) {
     l->n = 0;
     size_t k = from;
-    for (; k < ups.size() && l->n < kAppendLenMax; ++k) {
+    for (; k < ups.size() && l->n + 2 <= kAppendLenMax; ++k) {
         const LenUpdate& u = ups[k];
-        l->ptr[l->n] = reinterpret_cast<int32_t*>(u.e->d_plan + u.e->lay.seq_len) + u.i;
-        l->val[l->n] = u.val;
-        ++l->n;
+        uint8_t* seg = u.e->d_plan + u.e->lay.segs + sizeof(DecodeSeg) * u.e->tail_seg[u.i];
+        l->ptr[l->n] = reinterpret_cast<int32_t*>(seg + offsetof(DecodeSeg, n_tok));
+        l->val[l->n++] = u.val;
+        l->ptr[l->n] = reinterpret_cast<int32_t*>(seg + offsetof(DecodeSeg, grp_lim));
+        l->val[l->n++] = u.val;
     }
     return k - from;
 }
@@ -747,7 +757,7 @@ int sq_append_kv_batch(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, const vo
             a.page[i] = pl.pages[0];                 // the page holding slot position pos0
             a.slot[i] = pl.pos0 % g.P;
             // a sequence's plan updates go all into this launch, or none do
-            if (l.n + ups[b + i].size() <= (size_t)kAppendLenMax) {
+            if (l.n + 2 * ups[b + i].size() <= (size_t)kAppendLenMax) {
                 AppendLens part;
                 n_ups[b + i] = fill_lens(ups[b + i], 0, &part);
                 for (int32_t k = 0; k < part.n; ++k) {
@@ -879,6 +889,15 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
         victim->lay = lay;
         victim->unique_tokens = plan.unique_tokens;
         victim->logical_tokens = plan.logical_tokens;
+        victim->tail_seg.assign(n_seqs, -1);
+        victim->tail_base.assign(n_seqs, 0);
+        for (size_t s = 0; s < plan.segs.size(); ++s) {
+            const DecodeSeg& sg = plan.segs[s];
+            if (sg.n_grp == 1 && (sg.tail & 1)) {
+                victim->tail_seg[sg.grp_seq[0]] = (int32_t)s;
+                victim->tail_base[sg.grp_seq[0]] = sg.q0 * g.P;
+            }
+        }
         victim->first_busy_cta = 0;
         while (victim->first_busy_cta + 1 < (int32_t)plan.cta_begin.size() &&
                plan.cta_begin[victim->first_busy_cta + 1] == plan.cta_begin[victim->first_busy_cta])
@@ -914,7 +933,6 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
     a.page_ids = reinterpret_cast<const int32_t*>(hit->d_plan + L.page_ids);
     a.comb_off = reinterpret_cast<const int32_t*>(hit->d_plan + L.comb_off);
     a.arrive = reinterpret_cast<unsigned int*>(hit->d_plan + L.arrive);
-    a.seq_len = reinterpret_cast<const int32_t*>(hit->d_plan + L.seq_len);
     a.page_fill = L.page_fill >= 0 ? reinterpret_cast<const int32_t*>(hit->d_plan + L.page_fill)
                                    : nullptr;
     a.q = reinterpret_cast<const __nv_bfloat16*>(q);
@@ -1465,7 +1483,6 @@ int sq_decode_attention_noalloc(sq_cache* c, const sq_seq* seqs, int32_t n_seqs,
     a.page_ids = reinterpret_cast<const int32_t*>(scratch + L.page_ids);
     a.comb_off = reinterpret_cast<const int32_t*>(scratch + L.comb_off);
     a.arrive = reinterpret_cast<unsigned int*>(scratch + L.arrive);
-    a.seq_len = reinterpret_cast<const int32_t*>(scratch + L.seq_len);
     a.page_fill = L.page_fill >= 0 ? reinterpret_cast<const int32_t*>(scratch + L.page_fill)
                                    : nullptr;
     a.q = reinterpret_cast<const __nv_bfloat16*>(q);

@@ -519,7 +519,6 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
             if (ss[j] == ss[i]) return kInvalidArg;
         out->logical_tokens += ss[i]->n;
         ragged = ragged || has_partial_pages(*ss[i], g.P);
-        out->seq_len.push_back((int32_t)slot_end(*ss[i], g.P));
     }
     const int32_t P = g.P;
     const int32_t max_grp = kRowsPerTile / g.G();
@@ -599,6 +598,7 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
                     seg.grp_seq[j] = i;
                     seg.grp_lim[j] = (int32_t)lim;
                     seg.n_tok = std::max(seg.n_tok, (int32_t)lim);
+                    if ((int32_t)ss[i]->pages.size() == q_end) seg.tail |= 1 << j;
                 }
                 const Seq* sl = ss[part[b]];
                 for (int32_t q = q0; q < q_end; ++q) {
@@ -720,8 +720,6 @@ DecodePlanLayout plan_layout(const DecodePlanHost& p, int32_t n_seqs, int32_t Hk
     } else {
         L.page_fill = -1;
     }
-    L.n_seqs = n_seqs;
-    L.seq_len = o;   o = align16(o + sizeof(int32_t) * n_seqs);
     L.total = o;
     return L;
 }
@@ -735,7 +733,6 @@ void plan_serialize(const DecodePlanHost& p, const DecodePlanLayout& L, uint8_t*
     std::memcpy(dst + L.comb_off, p.comb_off.data(), sizeof(int32_t) * (L.n_comb_keys + 1));
     if (L.page_fill >= 0)
         std::memcpy(dst + L.page_fill, p.page_fill.data(), sizeof(int32_t) * L.n_page_ids);
-    std::memcpy(dst + L.seq_len, p.seq_len.data(), sizeof(int32_t) * L.n_seqs);
 }
 
 // ---------------------------------------------------------------------------

@@ -206,7 +206,6 @@ struct DecodePlanHost {
     // partial entries of (sequence i, KV head h): [comb_off[k], comb_off[k + 1]),
     // k = i * Hkv + h, in item order
     std::vector<int32_t> comb_off;    // n_seqs * Hkv + 1
-    std::vector<int32_t> seq_len;     // each sequence's end in slot space
     int64_t unique_tokens = 0;        // distinct rows read (one head, one layer)
     int64_t logical_tokens = 0;       // sum over sequences of n
     int32_t n_ctas = 0;

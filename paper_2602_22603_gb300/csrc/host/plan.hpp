@@ -29,6 +29,8 @@ struct DecodeSeg {
     int32_t grp_seq[kRowsPerTile];    // call-local sequence indices
     int32_t grp_lim[kRowsPerTile];    // valid tokens of each, from the run start
     int32_t q0;                       // page index of the run's first page in its members
+    int32_t tail;                     // bit j: the run holds member j's last page (the
+                                      // others' limit is the whole run)
 };
 
 // A contiguous range of stages of one (segment, KV head) — one partial result
@@ -95,13 +97,9 @@ struct PrefillTile {
 // arrival count per (sequence, KV head), zero in the serialised plan; the
 // kernel counts on it and leaves it at zero again.
 // `page_fill` is -1 when the plan carries no page fills.
-// `seq_len` holds each call-local sequence's end in slot space (page index x P
-// + slot, one past its last row); the kernel takes every member's limit in a
-// run from it, so an append inside a sequence's last page and stage can keep
-// the plan by rewriting that one word.
 struct DecodePlanLayout {
-    int64_t segs, items, cta_begin, page_ids, comb_off, arrive, page_fill, seq_len, total;
-    int32_t n_segs, n_items, n_ctas, n_page_ids, n_comb_keys, n_comb_ent, n_seqs;
+    int64_t segs, items, cta_begin, page_ids, comb_off, arrive, page_fill, total;
+    int32_t n_segs, n_items, n_ctas, n_page_ids, n_comb_keys, n_comb_ent;
 };
 
 }  // namespace sq

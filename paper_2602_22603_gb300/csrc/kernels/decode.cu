@@ -311,14 +311,9 @@ __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, ui
         const int n_grp = seg->n_grp;
         const int j0 = r0 / G, j1 = r1 / G;
         const bool v0 = j0 < n_grp, v1 = j1 < n_grp;
-        // each member's rows in the run: its end in slot space, from the
-        // run's first slot, within the run's pages
-        const int run_slots = seg->n_pages * a.P, run0 = seg->q0 * a.P;
-        auto lim_of = [&](int j) { return min(a.seq_len[seg->grp_seq[j]] - run0, run_slots); };
-        const int lim0 = v0 ? lim_of(j0) : 0;
-        const int lim1 = v1 ? lim_of(j1) : 0;
-        int n_tok = 0;
-        for (int j = 0; j < n_grp; ++j) n_tok = max(n_tok, lim_of(j));
+        const int lim0 = v0 ? seg->grp_lim[j0] : 0;
+        const int lim1 = v1 ? seg->grp_lim[j1] : 0;
+        const int n_tok = seg->n_tok;
 
         uint32_t qa[C::kKS][4];
         {

@@ -25,10 +25,6 @@ struct DecodeArgs {
     const int32_t* page_fill;
     const int32_t* comb_off;    // [n_seqs * Hkv + 1] partial entries of each (sequence, KV head)
     unsigned int* arrive;       // [n_seqs * Hkv] arrival counts, zero between calls
-    // [n_seqs] each sequence's end in slot space; an append kernel may have
-    // rewritten it since the plan was uploaded, so it is read after the
-    // grid-dependency wait
-    const int32_t* seq_len;
     const __nv_bfloat16* q;     // [n_seqs][Hq][D]
     void* out;                  // [n_seqs][Hq][D] bf16 or fp32
     float* part_o;              // [n_ent][G][D]  unnormalised partial outputs
@@ -98,8 +94,9 @@ cudaError_t launch_prefill_combine(const PrefillCombineArgs& a, int D, cudaStrea
 // ---- append / copy-on-write / eviction --------------------------------------
 constexpr int kAppendMaxPages = 64;
 
-// Sequence lengths in cached decode plans that an append rewrites (in stream
-// order, by block 0): plans that the append leaves valid (see the API layer).
+// Words of cached decode plans that an append rewrites (in stream order, by
+// block 0): the row limit of the run holding the appended sequence's last
+// page, in plans that the append leaves valid (see the API layer).
 constexpr int kAppendLenMax = 32;
 struct AppendLens {
     int32_t n;

@@ -14,7 +14,7 @@ from paper_2602_22603_gb300 import build as _build  # noqa: E402
 
 _lib = None
 
-SEG_INTS = 4 + 2 * 16 + 1  # DecodeSeg: page_off, n_pages, n_tok, n_grp, grp_seq[16], grp_lim[16], q0
+SEG_INTS = 4 + 2 * 16 + 2  # DecodeSeg: page_off, n_pages, n_tok, n_grp, grp_seq[16], grp_lim[16], q0, tail
 ITEM_INTS = 5 + 16     # DecodeItem: seg, head, s0, s1, sole, ent[16]
 
 
@@ -170,7 +170,7 @@ class HostCache:
 
     def plan_decode(self, handles, n_ctas):
         arr = (ctypes.c_int32 * len(handles))(*handles)
-        lay = (ctypes.c_int64 * 18)()
+        lay = (ctypes.c_int64 * 17)()
         rc = lib().sqh_plan_decode(self.h, arr, len(handles), n_ctas, lay, None, 0)
         if rc != 0:
             return rc, None
@@ -191,7 +191,8 @@ class HostCache:
         segs = arr_at(L[0], n_segs, SEG_INTS)
         seg_list = [{"page_off": int(s[0]), "n_pages": int(s[1]), "n_tok": int(s[2]),
                      "n_grp": int(s[3]), "grp_seq": [int(x) for x in s[4:4 + s[3]]],
-                     "grp_lim": [int(x) for x in s[20:20 + s[3]]], "q0": int(s[36])} for s in segs]
+                     "grp_lim": [int(x) for x in s[20:20 + s[3]]], "q0": int(s[36]),
+                     "tail": int(s[37])} for s in segs]
         raw_items = arr_at(L[1], n_items, ITEM_INTS) if n_items else np.zeros((0, ITEM_INTS), np.int32)
         comb_off = arr_at(L[4], n_keys + 1).tolist()
         # each item's group members name their partial entry; every entry is
@@ -219,6 +220,5 @@ class HostCache:
             "comb_ent": comb_ent,
             "unique_tokens": L[13], "logical_tokens": L[14],
             "page_fill": arr_at(L[16], n_pid).tolist() if L[16] >= 0 else None,
-            "seq_len": arr_at(L[17], len(handles)).tolist(),
         }
         return 0, plan

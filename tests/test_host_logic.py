@@ -155,10 +155,17 @@ def _check_plan(hc, handles, plan, n_ctas, G):
                 q0 = tables[i].index(pids[0])
                 assert tables[i][q0:q0 + s["n_pages"]] == pids
                 lim = s["grp_lim"][j]
-                # the kernel's limit: the sequence's end from the run's first
-                # slot, within the run's pages
-                assert s["q0"] == q0 and plan["seq_len"][i] == ends[i]
-                assert min(plan["seq_len"][i] - q0 * P, s["n_pages"] * P) == lim
+                # the limit is the sequence's end from the run's first slot,
+                # within the run's pages (an append inside the last page
+                # rewrites it this way in a kept plan)
+                assert s["q0"] == q0
+                assert min(ends[i] - q0 * P, s["n_pages"] * P) == lim
+                # the tail bit: the run holds the member's last page; the
+                # others' limit is the whole run
+                is_tail = q0 + s["n_pages"] == len(tables[i])
+                assert bool((s["tail"] >> j) & 1) == is_tail
+                if not is_tail:
+                    assert lim == s["n_pages"] * P
                 lo, hi = s0 * STAGE, min(s1 * STAGE, lim)
                 if hi > lo:
                     covered.append((q0 * P + lo, q0 * P + hi))
