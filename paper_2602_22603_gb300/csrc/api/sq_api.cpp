@@ -49,8 +49,9 @@ struct PlanEntry {
     std::vector<std::pair<uint64_t, int32_t>> tick_top;
     uint64_t tick_rest = 0;
     // per call-local sequence: the segment holding its last page when that
-    // segment has it alone (else -1), and the slot-space start of that run
-    std::vector<int32_t> tail_seg, tail_base;
+    // segment has it alone (else -1), the slot-space start of that run, and
+    // the last page's entry in page_fill (plans with page fills)
+    std::vector<int32_t> tail_seg, tail_base, tail_fill;
     uint8_t* d_plan = nullptr;
     size_t plan_cap = 0;
     float* d_part = nullptr;
@@ -543,13 +544,15 @@ int sq_fork_aux(sq_cache* c, sq_seq parent, sq_seq* child_out) {
 // have been copied on write), so that run's segment has it as its one member
 // and the limit is two words of the segment (its token count and the member's
 // limit).  The append kernel rewrites them, after the plan's last decode on
-// the same stream, and the plan takes the sequence's new version.  Plans
-// last used on another stream, plans with page fills, and pages of fewer than
-// 64 tokens (a stage spans pages) are rebuilt instead.
+// the same stream, and the plan takes the sequence's new version; a plan
+// with page fills also gets the last page's new fill.  Plans last used on
+// another stream, and pages of fewer than 64 tokens (a stage spans pages),
+// are rebuilt instead.
 struct LenUpdate {
     PlanEntry* e;
     int32_t i;     // call-local index of the sequence in the plan
     int32_t val;   // the new row limit of its last run (end in slot space - run start)
+    int32_t fill;  // the new fill of its last page
 };
 
 static void plan_len_updates(sq_cache* c, sq_seq seq, const AppendPlan& ap, uint64_t old_version,
@@ -557,27 +560,36 @@ static void plan_len_updates(sq_cache* c, sq_seq seq, const AppendPlan& ap, uint
     if (c->g.P % kStageTokens != 0 || ap.cow || !ap.taken.empty() || ap.n_new < 1) return;
     const int64_t e0 = ap.pos0, e1 = (int64_t)ap.pos0 + ap.n_new;
     if ((e0 + kStageTokens - 1) / kStageTokens != (e1 + kStageTokens - 1) / kStageTokens) return;
+    const int32_t fill = (int32_t)(e1 - (int64_t)ap.first_page_index * c->g.P);
     for (auto& e : c->plans) {
-        if (!e.valid || e.lay.page_fill >= 0 || !e.ev_recorded || e.ev_stream != st) continue;
+        if (!e.valid || !e.ev_recorded || e.ev_stream != st) continue;
         for (size_t i = 0; i < e.handles.size(); ++i)
             if (e.handles[i] == seq && e.versions[i] == old_version && e.tail_seg[i] >= 0)
-                out->push_back({&e, (int32_t)i, (int32_t)(e1 - e.tail_base[i])});
+                out->push_back({&e, (int32_t)i, (int32_t)(e1 - e.tail_base[i]), fill});
     }
 }
 
-// The kernel's writes for `ups` (from index `from`): the run's token count
-// and its one member's limit, two words each, as many as fit; returns how
-// many updates were taken.
+// Words the kernel rewrites for one update: the run's token count, its one
+// member's limit, and (plans with page fills) the last page's fill.
+static int update_words(const LenUpdate& u) { return u.e->lay.page_fill >= 0 ? 3 : 2; }
+
+// The kernel's writes for `ups` (from index `from`), as many updates as fit
+// whole; returns how many were taken.
 static size_t fill_lens(const std::vector<LenUpdate>& ups, size_t from, AppendLens* l) {
     l->n = 0;
     size_t k = from;
-    for (; k < ups.size() && l->n + 2 <= kAppendLenMax; ++k) {
+    for (; k < ups.size() && l->n + update_words(ups[k]) <= kAppendLenMax; ++k) {
         const LenUpdate& u = ups[k];
         uint8_t* seg = u.e->d_plan + u.e->lay.segs + sizeof(DecodeSeg) * u.e->tail_seg[u.i];
         l->ptr[l->n] = reinterpret_cast<int32_t*>(seg + offsetof(DecodeSeg, n_tok));
         l->val[l->n++] = u.val;
         l->ptr[l->n] = reinterpret_cast<int32_t*>(seg + offsetof(DecodeSeg, grp_lim));
         l->val[l->n++] = u.val;
+        if (u.e->lay.page_fill >= 0) {
+            l->ptr[l->n] = reinterpret_cast<int32_t*>(u.e->d_plan + u.e->lay.page_fill) +
+                           u.e->tail_fill[u.i];
+            l->val[l->n++] = u.fill;
+        }
     }
     return k - from;
 }
@@ -757,7 +769,9 @@ int sq_append_kv_batch(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, const vo
             a.page[i] = pl.pages[0];                 // the page holding slot position pos0
             a.slot[i] = pl.pos0 % g.P;
             // a sequence's plan updates go all into this launch, or none do
-            if (l.n + 2 * ups[b + i].size() <= (size_t)kAppendLenMax) {
+            int words = 0;
+            for (const LenUpdate& u : ups[b + i]) words += update_words(u);
+            if (l.n + words <= kAppendLenMax) {
                 AppendLens part;
                 n_ups[b + i] = fill_lens(ups[b + i], 0, &part);
                 for (int32_t k = 0; k < part.n; ++k) {
@@ -891,11 +905,13 @@ int sq_decode_attention(sq_cache* c, const sq_seq* seqs, int32_t n_seqs, int32_t
         victim->logical_tokens = plan.logical_tokens;
         victim->tail_seg.assign(n_seqs, -1);
         victim->tail_base.assign(n_seqs, 0);
+        victim->tail_fill.assign(n_seqs, 0);
         for (size_t s = 0; s < plan.segs.size(); ++s) {
             const DecodeSeg& sg = plan.segs[s];
             if (sg.n_grp == 1 && (sg.tail & 1)) {
                 victim->tail_seg[sg.grp_seq[0]] = (int32_t)s;
                 victim->tail_base[sg.grp_seq[0]] = sg.q0 * g.P;
+                victim->tail_fill[sg.grp_seq[0]] = sg.page_off + sg.n_pages - 1;
             }
         }
         victim->first_busy_cta = 0;

@@ -210,3 +210,38 @@ def test_ragged_prefill():
     # one row fewer starts on the next page: accepted
     _prefill_check(p, m, 0, n_q - fills[qs], [], 401, scale)
     p.close()
+
+
+def test_decode_plan_survives_in_page_appends_after_ragged_eviction():
+    """After a ragged eviction (partial pages before the last), one-token
+    appends inside the last page keep the cached plan: the append kernel
+    rewrites the last run's limit and the last page's fill in it.  An append
+    that opens a page has the plan rebuilt; every output equals the oracle."""
+    L, P = 2, 64
+    p = Pair(L, 16, 4, 64, P, num_pages=300, seed=95, physical=True)
+    keep = []
+    m = p.seq_new()
+    keep.append(p.append(m, 14 * P + 20))
+    p.evict(m, [(100, 150), (400, 420), (880, 900)], ragged=True)
+    fills = p.cache.page_fills(m)
+    assert min(fills[:-1]) < P                      # partial pages before the last
+    st0 = p.cache.stats()
+    rebuilds = 0
+    for step in range(P + 4):                       # long enough to open a page
+        f = p.cache.page_fills(m)
+        if step == 0 or f[-1] == P:                 # first plan, or the append opens a page
+            rebuilds += 1
+        keep.append(p.append(m, 1))
+        for layer in range(L):
+            q_cpu, q = bf16_normal((1, 16, 64), 1500 + 7 * step + layer), None
+            q = q_cpu.cuda()
+            keep.append(q)
+            out = p.decode([m], layer, 0.125, q, sq.SQ_OUT_F32)
+            torch.cuda.synchronize()
+            assert_budget(out, *p.oracle_decode_budget([m], layer, 0.125, q_cpu))
+    st1 = p.cache.stats()
+    assert st1["decode_plans_built"] - st0["decode_plans_built"] == rebuilds
+    assert rebuilds >= 2
+    p.check_tables()
+    assert p.cache.sync_status() == sq.SQ_OK
+    p.close()
