@@ -120,6 +120,10 @@ SQ_API int sq_seq_new(sq_cache *cache, sq_seq *out);
  * If the sequence's last page is partial and shared with another sequence it
  * is first copied (copy-on-write); then fresh pages are taken, lowest free id
  * first, in increasing logical order.  n_tokens == 0 is a no-op.
+ * Cached decode plans holding `seq`, last used on `stream`, stay valid when
+ * the rows fit in the last page and its 64-token stage (pages of >= 64
+ * tokens): the launch rewrites the plan's row limit for the sequence, so the
+ * next sq_decode_attention on `stream` reuses the plan without an upload.
  * Errors: BAD_HANDLE, INVALID_ARG, NO_PAGES, CAPACITY, CUDA. */
 SQ_API int sq_append_kv(sq_cache *cache, sq_seq seq, int32_t n_tokens, const void *k,
                  const void *v, void *stream);
@@ -129,8 +133,9 @@ SQ_API int sq_append_kv(sq_cache *cache, sq_seq seq, int32_t n_tokens, const voi
  *   seqs: host, n_seqs distinct live handles
  *   k, v: device, bf16, contiguous [num_layers][n_seqs][num_kv_heads][head_dim]:
  *         row i belongs to seqs[i]
- * Same page rules as sq_append_kv, sequence by sequence in the order given;
- * all or nothing: on any error no sequence changes.
+ * Same page rules (and the same reuse of cached decode plans) as
+ * sq_append_kv, sequence by sequence in the order given; all or nothing: on
+ * any error no sequence changes.
  * Errors: BAD_HANDLE, INVALID_ARG, NO_PAGES, CAPACITY, CUDA. */
 SQ_API int sq_append_kv_batch(sq_cache *cache, const sq_seq *seqs, int32_t n_seqs,
                               const void *k, const void *v, void *stream);
