@@ -298,9 +298,11 @@ typedef struct {
                                     waiting for the preceding kernel */
     int64_t decode_early_held;   /* pages those calls left for after the wait (a write
                                     to them not yet known complete) */
-    int64_t decode_plans_built;  /* decode calls that planned and uploaded a plan (the
-                                    others reused a cached one, also after appends that
-                                    stayed inside a sequence's last page and stage) */
+    int64_t decode_plans_built;  /* sq_decode_attention calls that planned and uploaded a
+                                    plan (the others reused a cached one, also after
+                                    appends that stayed inside a sequence's last page and
+                                    stage); sq_decode_attention_noalloc plans every call
+                                    and is not counted here */
 } sq_stats_t;
 
 SQ_API int sq_stats(sq_cache *cache, sq_stats_t *out);
