@@ -268,3 +268,62 @@ def test_serving_128k_ragged_eviction_full_size():
             _decode_and_check(bp, seqs, layer, scale, 700 + layer, None)
     finally:
         bp.close()
+
+
+def test_d64_long_contexts_decode_evict_prefill():
+    """The d = 64 kernels (a six-stage decode ring, the 64-column prefill
+    tiles) at long contexts: 2 requests x 49,152 tokens + forks, G = 8, P = 64,
+    every sequence decoded at two layers; request 0 loses 30% in 10 spans while
+    its fork is alive (copy-on-write), tables and planes checked, decode again;
+    then a masked prefill of its last 4,096 tokens at one layer, sampled rows
+    with their log-sum-exp against the oracle."""
+    L, Hq, Hkv, D, P = 4, 32, 4, 64, 64
+    R, ctx = 2, 49152
+    # the eviction with the fork alive copies most of a request's pages on write
+    bp = BankPair(L, Hq, Hkv, D, P, num_pages=2 * R * (ctx // P + 4) + 256, seed=6)
+    try:
+        scale = 1.0 / math.sqrt(D)
+        mains, auxs = [], []
+        for r in range(R):
+            m = bp.seq_new()
+            bp.fill(m, ctx, 4096)
+            mains.append(m)
+            a = bp.fork(m)
+            bp.append(a, 8)
+            auxs.append(a)
+        seqs = [x for pair in zip(mains, auxs) for x in pair]
+        for layer in (0, L - 1):
+            _decode_and_check(bp, seqs, layer, scale, 700 + layer, None)
+        n = bp.cache.seq_info(mains[0])[0]
+        spans = shuffled(random_spans(33, 10, int(0.3 * n), P, n, median=1200), 2)
+        bp.evict(mains[0], spans)                   # the fork still holds the old pages
+        bp.check_tables(seqs)
+        bp.check_planes(mains[0], 1)
+        bp.check_planes(auxs[0], 2)
+        for h in seqs:
+            bp.append(h, 1)
+        for layer in (1, 2):
+            _decode_and_check(bp, seqs, layer, scale, 800 + layer, None)
+        # masked prefill of request 1's last 4,096 tokens
+        m = mains[1]
+        n = bp.cache.seq_info(m)[0]
+        n_q = 4096
+        pspans = shuffled(random_spans(34, 6, 6000, P, n - n_q, median=900), 3)
+        q = bf16_normal((n_q, Hq, D), 900, device="cuda")
+        out = torch.empty(n_q, Hq, D, dtype=torch.float32, device="cuda")
+        lse = torch.empty(n_q, Hq, dtype=torch.float32, device="cuda")
+        bp.cache.prefill_attention(m, 3, n_q, q, out, sq.SQ_OUT_F32, lse, scale, pspans)
+        torch.cuda.synchronize()
+        assert bp.cache.sync_status() == sq.SQ_OK
+        qb = bf16_bits(q.cpu())
+        K, V = bp.rows(m, 3)
+        for i in (0, 1, 7, 8, 63, 64, 2047, n_q - 9, n_q - 1):
+            p = n - n_q + i
+            vis = [(a, min(b, p + 1)) for a, b in pspans if a < p + 1]
+            exp, exp_lse = oatt.prefill(qb[i:i + 1], K[:p + 1], V[:p + 1], scale, vis,
+                                        want_lse=True)
+            assert_close(out[i:i + 1], exp)
+            got = lse[i].cpu().numpy().astype(np.float64)
+            assert np.abs(got - exp_lse[0]).max() <= 1e-2, i
+    finally:
+        bp.close()
