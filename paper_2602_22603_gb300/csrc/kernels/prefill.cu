@@ -24,8 +24,9 @@
 // and tcgen05.mma operations of one thread execute in issue order.  The same
 // order means that when S_t(j) is ready, PV_t(j-1) is complete, so a
 // warpgroup may rescale O_t then without another wait.  The running maximum
-// is raised lazily: O is rescaled only when a row's maximum grows by more than
-// 2^8, so the weights stay below 256.  K and V stream through one ring of
+// is raised lazily: a key tile's weights are taken with the current maximum
+// and accepted while every row's sum of them stays at most 2^16 (so does each
+// weight); only then is a maximum raised and O rescaled.  K and V stream through one ring of
 // shared-memory slots (K_0, V_0, K_1, ...); a K slot is released once both S
 // products are done, a V slot once both PV products are.
 //
@@ -440,10 +441,13 @@ __device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
     asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
     return d;
 }
-__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
-    uint64_t d;
-    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-    return d;
+// lo += the low bf16 of w, hi += its high bf16 (mixed-precision adds: the
+// bf16 operands are exact in fp32).
+__device__ __forceinline__ void add_bf16x2_f32(uint32_t w, float& lo, float& hi) {
+    asm("{\n\t.reg .b16 l16, h16;\n\tmov.b32 {l16, h16}, %2;\n\t"
+        "add.rn.f32.bf16 %0, l16, %0;\n\tadd.rn.f32.bf16 %1, h16, %1;\n\t}"
+        : "+f"(lo), "+f"(hi)
+        : "r"(w));
 }
 // 2^x as the single PTX instruction ex2.approx.ftz (relative error about
 // 2^-22).  Results below 2^-126 flush to zero: every row holds a weight of at
@@ -459,15 +463,11 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
     return d;
 }
 
-// One lane of the warp polls the barrier; the others wait at the shuffle.
-// Returns the warp-uniform result.
-__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, const volatile int* abort,
-                                          int lane) {
-    bool ok = true;
-    if (lane == 0) ok = mbar_wait(bar, parity, abort);
-    ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-    __syncwarp();
-    return ok;
+// Every lane of the warp polls the barrier (one instruction for the warp,
+// no hand-on from a polling lane: a softmax warp sees its S ready sooner);
+// returns the warp-uniform result.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, const volatile int* abort) {
+    return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort));
 }
 
 // Softmax warpgroup of query tile t (one row per thread) and its epilogue.
@@ -491,7 +491,7 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
     if (!__any_sync(0xffffffffu, valid)) {
         bool wok = true;
         for (int j = 0; j < T; ++j) {
-            if (wok) wok = warp_wait(sm.bar<D>(C::kBarS + t), j & 1, abort_flag, lane);
+            if (wok) wok = warp_wait(sm.bar<D>(C::kBarS + t), j & 1, abort_flag);
             tc_fence_before();
             mbar_arrive(sm.bar<D>(C::kBarP + t));
         }
@@ -527,7 +527,7 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
         }
         const int key0 = w0.x;
         const uint32_t vis[4] = {(uint32_t)w0.z, (uint32_t)w0.w, (uint32_t)w1.x, (uint32_t)w1.y};
-        ok = warp_wait(sm.bar<D>(C::kBarS + t), j & 1, abort_flag, lane);
+        ok = warp_wait(sm.bar<D>(C::kBarS + t), j & 1, abort_flag);
         if (!ok) break;
         tc_fence_after();
         // Raw logits q.k (the scale is applied inside the exponent; it is > 0),
@@ -539,21 +539,16 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
         const bool unmasked = valid && (w0.y & kPrefillTileFull) && lim >= 63 && limb >= 63;
         // Weights 2^(s * scale - m) with the running maximum m, two arguments
         // at a time with a packed FMA, rounded to bf16 into wt (32 words per
-        // 64 keys); the normaliser sums the fp32 weights (four packed chains).
-        // When `track` is set the pass also returns the tile's raw maximum.
+        // 64 keys).  The normaliser sums the same rounded weights that the PV
+        // product takes (eight fp32 chains), so the output is a convex
+        // combination of the V rows whatever the rounding.
         // Nothing is stored: S stays intact until the weights are accepted.
         const uint64_t sc2 = f2pack(sc, sc);
         uint32_t wt[2][32];
-        auto weights = [&](float m, bool track, float& tile_max, float& tile_sum) {
+        auto weights = [&](float m, float& tile_sum) {
             const float nmu = m == -INFINITY ? 0.f : -m;
             const uint64_t nmu2 = f2pack(nmu, nmu);
-            uint64_t ls2[4];
-            float mx[4];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                ls2[c] = 0;
-                mx[c] = -INFINITY;
-            }
+            float ls[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int hh = 0; hh < 2; ++hh) {
                 uint32_t x[64];
@@ -574,35 +569,28 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
                     const float x0 = __uint_as_float(x[2 * i]), x1 = __uint_as_float(x[2 * i + 1]);
-                    if (track) mx[i & 3] = fmax3(mx[i & 3], x0, x1);
                     float a0, a1;
                     f2unpack(ffma2(f2pack(x0, x1), sc2, nmu2), a0, a1);
-                    const float p0 = ex2_ftz(a0), p1 = ex2_ftz(a1);
-                    ls2[i & 3] = fadd2(ls2[i & 3], f2pack(p0, p1));
-                    const __nv_bfloat162 hb = __floats2bfloat162_rn(p0, p1);
+                    const __nv_bfloat162 hb = __floats2bfloat162_rn(ex2_ftz(a0), ex2_ftz(a1));
                     wt[hh][i] = *reinterpret_cast<const uint32_t*>(&hb);
+                    add_bf16x2_f32(wt[hh][i], ls[2 * (i & 3)], ls[2 * (i & 3) + 1]);
                 }
             }
-            float s0, s1, s2, s3, s4, s5, s6, s7;
-            f2unpack(ls2[0], s0, s1);
-            f2unpack(ls2[1], s2, s3);
-            f2unpack(ls2[2], s4, s5);
-            f2unpack(ls2[3], s6, s7);
-            tile_sum = ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
-            tile_max = fmaxf(fmax3(mx[0], mx[1], mx[2]), mx[3]);
+            tile_sum = ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
         };
         // The maximum is raised lazily, so most tiles keep it: take the
-        // weights with the current maximum and the tile maximum in one pass,
-        // and redo the tile only where a row's maximum grew by more than 2^8
-        // (or the row has seen no key yet).
+        // weights with the current maximum and accept them when no row's sum
+        // exceeds 2^16, which bounds every weight; no maximum is needed for
+        // that.  Otherwise (or when a row has seen no key yet) find the tile's
+        // maximum and redo the tile with it wherever it exceeds the running
+        // one by more than 2^8.
         float mt = -INFINITY, tsum = 0.f;
         bool done = false;
         if (__all_sync(0xffffffffu, m_run != -INFINITY)) {
-            float raw;
-            weights(m_run, true, raw, tsum);
-            mt = raw * sc;
-            done = !__any_sync(0xffffffffu, mt > m_run + 8.f);
-        } else {
+            weights(m_run, tsum);
+            done = !__any_sync(0xffffffffu, tsum > 65536.f);
+        }
+        if (!done) {
             // row maximum: three-input max over four independent chains
             float mx[4];
 #pragma unroll
@@ -658,8 +646,7 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
                     tmem_st32(tl + col_o + c * 32, o);
                 }
             }
-            float unused;
-            weights(m_run, false, unused, tsum);
+            weights(m_run, tsum);
             l += tsum;
         }
         // P_t over the first half of S_t: keys 64 hh .. +63 to columns 32 hh .. +31
@@ -669,7 +656,7 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
         tc_fence_before();
         mbar_arrive(sm.bar<D>(C::kBarP + t));
     }
-    if (ok && T > 0) ok = warp_wait(sm.bar<D>(C::kBarO + t), 0, abort_flag, lane);
+    if (ok && T > 0) ok = warp_wait(sm.bar<D>(C::kBarO + t), 0, abort_flag);
     // dual-key mode: tile b hands its (max, normaliser) to tile a, which
     // merges the two partial results of each row (weights 2^(m_t - max))
     float wa = 1.f, wb = 0.f;
@@ -686,7 +673,7 @@ __device__ void prefill_softmax(const PrefillArgs& a, const Smem& sm, uint32_t t
             }
             return;
         }
-        if (ok) ok = warp_wait(sm.bar<D>(C::kBarO + 1), 0, abort_flag, lane);
+        if (ok) ok = warp_wait(sm.bar<D>(C::kBarO + 1), 0, abort_flag);
         const float mb = xchg[2 * row], lb = xchg[2 * row + 1];
         const float M = fmaxf(m_run, mb);
         wa = m_run == -INFINITY ? 0.f : exp2f(m_run - M);

@@ -12,7 +12,8 @@ import torch
 import paper_2602_22603_gb300 as sq
 from oracle import attention as oatt
 from synthetic import bf16_bits, bf16_normal, random_spans
-from tests.gpu_harness import Pair, assert_close
+from tests.budget import decode_budget
+from tests.gpu_harness import Pair, assert_budget, assert_close
 
 pytestmark = pytest.mark.gpu
 
@@ -43,11 +44,33 @@ def oracle_prefill(p: Pair, h, layer, q_cpu, spans, scale):
     return oatt.prefill(bf16_bits(q_cpu), k, v, scale, spans, want_lse=True)
 
 
+def check_budget_rows(p: Pair, h, layer, q_cpu, out, spans, scale, rows):
+    """Element by element within the error budget of the bf16 softmax weights
+    (tests/budget.py): the normaliser sums the same rounded weights the PV
+    product takes, so each output row is a convex combination of V rows, as in
+    decode.  Query row r at position n - n_q + r is decode over the keys it
+    sees; rows that see no key are left to the exact check."""
+    k, v = p.store.rows(p.oracle.tokens(p.o[h]), layer)
+    n, n_q = k.shape[0], q_cpu.shape[0]
+    qb = bf16_bits(q_cpu)
+    got = out.detach().float().cpu()
+    for r in rows:
+        pos = n - n_q + r
+        mask = oatt.removed_mask(pos + 1, spans)
+        if mask.all():
+            continue
+        exp, dev, absv = oatt.decode_dev(qb[r], k[:pos + 1], v[:pos + 1], scale, mask)
+        assert_budget(got[r], exp, decode_budget(dev, absv, pos + 1))
+
+
 def check(p, h, layer, n_q, spans, seed, scale=None, out_dtype=sq.SQ_OUT_F32):
     scale = scale if scale is not None else 1.0 / math.sqrt(p.D)
     q_cpu, out, lse = run_prefill(p, h, layer, n_q, spans, seed, scale, out_dtype)
     exp, exp_lse = oracle_prefill(p, h, layer, q_cpu, spans, scale)
     assert_close(out, exp)
+    if out_dtype == sq.SQ_OUT_F32:
+        rows = sorted(set(np.linspace(0, n_q - 1, min(n_q, 40)).round().astype(int).tolist()))
+        check_budget_rows(p, h, layer, q_cpu, out, spans, scale, rows)
     got_lse = lse.cpu().numpy().astype(np.float64)
     fin = np.isfinite(exp_lse)
     assert np.array_equal(np.isfinite(got_lse), fin)
@@ -109,6 +132,28 @@ def test_prefill_split_key_ranges():
         spans = random_spans(4, 10, 1200, 0, 3000, median=120)
         check(p, h, 0, 8, spans, seed=3)
         check(p, h, 0, 8, [], seed=4, out_dtype=sq.SQ_OUT_BF16)
+    finally:
+        p.close()
+
+
+@pytest.mark.parametrize("Hq,Hkv,D,P,n,n_q,scale", [
+    (32, 8, 128, 64, 1100, 1100, 0.35),   # maxima grow a few powers of two: kept, weights > 1
+    (32, 8, 128, 64, 1100, 1100, 1.0),    # grow by ~10: some tiles redone with a raised maximum
+    (32, 8, 128, 64, 1100, 1100, 4.0),    # grow far past 2^16: raised on most tiles
+    (16, 4, 64, 16, 700, 700, 1.5),       # d = 64
+    (32, 8, 128, 64, 3000, 8, 4.0),       # short block: dual-key halves and split key ranges
+])
+def test_prefill_running_maximum_under_growing_logits(Hq, Hkv, D, P, n, n_q, scale):
+    # Large softmax scales make each row's maximum grow from key tile to key
+    # tile.  A tile's weights are kept with the old maximum while every row's
+    # sum of them stays at most 2^16; past that the tile is redone with the
+    # raised maximum and O rescaled.  Both, and the mix of rows in one warp
+    # taking either, must give the softmax over all visible keys.
+    p = Pair(1, Hq, Hkv, D, P, num_pages=(n + P - 1) // P + 8, seed=n + 5)
+    try:
+        h = p.seq_new()
+        p.append(h, n)
+        check(p, h, 0, n_q, spans_for(n, 3, n + 1), seed=n + 2, scale=scale)
     finally:
         p.close()
 
