@@ -126,10 +126,11 @@ __device__ __forceinline__ int dual_load_k(int j) { return j < 2 ? j : 2 * j - 1
 __device__ __forceinline__ int dual_load_v(int j, int T) { return j < T - 1 ? 2 * j + 2 : 2 * T - 1; }
 
 // The producer warp: the query tiles once, then the K and V tiles of every key
-// tile into the ring in the order of load_of, two loads at a time: lanes 0
-// and 1 wait for their slots, arm their barriers and issue their copies
-// together, so that the shared-memory round trips of the two overlap.  What a
-// tile's copies need, {first key, page of box 0, page of box 1}, is held in
+// tile into the ring in the order of load_of, two loads at a time: the whole
+// warp waits for both slots, then lanes 0 and 1 arm their barriers and issue
+// their copies together, so that the shared-memory round trips of the two
+// overlap.  What a tile's copies need, {first key, page of box 0, page of box
+// 1}, is held in
 // registers: lane l has the record of the window's key tile j = l (mod 32),
 // batches of 16 tiles alternating between the lower and the upper half-warp;
 // a batch is read from global memory about ten tiles before its first use and
@@ -199,11 +200,16 @@ __device__ void prefill_produce(const CUtensorMap* pool_map, const CUtensorMap* 
         const int rows_b = key0b < a.n ? min(64, a.n - key0b) : 0;
         const int rows = rows_b > 0 ? 64 + rows_b : min(64, a.n - key0);
         const int slot = u % C::kSlots;
-        const int use = u / C::kSlots;
         const bool vfix = lane < 2 && kv == 1 && rows < kPrefillKeys;
+        // every lane polls both slots' barriers in turn: warp-uniform waits,
+        // so no lane waits at the vote below for two polling lanes
         bool ok = true;
-        if (lane < 2 && use > 0)
-            ok = mbar_wait(sm.bar<D>(C::kBarEmpty + slot), (use - 1) & 1, abort_flag);
+        if (u0 >= C::kSlots)
+            ok = mbar_wait(sm.bar<D>(C::kBarEmpty + u0 % C::kSlots), (u0 / C::kSlots - 1) & 1,
+                           abort_flag);
+        if (ok && u0 + 1 >= C::kSlots)
+            ok = mbar_wait(sm.bar<D>(C::kBarEmpty + (u0 + 1) % C::kSlots),
+                           ((u0 + 1) / C::kSlots - 1) & 1, abort_flag);
         // both slots free, or neither load is issued
         if (!__all_sync(0xffffffffu, ok)) {
             if (lane == 0) {
