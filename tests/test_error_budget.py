@@ -13,6 +13,8 @@ parity tests assert element by element.
    (the GPU split-invariance test asserts exactly that).
 3. At the shapes the GPU tests use, the simulated error stays below 5e-3
    (max) and 5e-4 (mean), and the budget itself below the contract's 1e-2.
+4. The masked prefill kernel's lazy maximum (weights kept with an old
+   maximum up to a row sum of 2^16, or redone after a raise) keeps bound (1).
 """
 import math
 
@@ -125,3 +127,68 @@ def test_budget_bounds_simulated_rounding(n, G, d):
     for s in sims[1:]:
         assert np.all(np.abs(s - sims[0]) <= 2 * budget)
     assert budget.max() < 1e-2
+
+
+def simulate_prefill_row(x, vf, tile=128, force=None):
+    """The masked prefill kernel's weights for one query row, in float64
+    elsewhere: key tiles of `tile` keys; a tile's weights 2^(x - m) with the
+    running maximum m are rounded to bf16 and accepted while their (rounded)
+    sum stays at most 2^16; otherwise the tile's maximum raises m where it
+    grew by more than 2^8, O and the normaliser are rescaled and the tile is
+    redone.  `force` (a generator) sometimes takes the second path although
+    the row's own sum was small, as a row does when another row of its warp
+    needs it.  Returns (output, accepted tiles whose largest weight exceeded
+    1, raises after the first tile)."""
+    m, l = -math.inf, 0.0
+    o = np.zeros(vf.shape[1])
+    above_one = raises = 0
+    for a in range(0, len(x), tile):
+        xt = x[a:a + tile]
+        if m != -math.inf:
+            pr = torch.from_numpy(np.exp2(xt - m)).to(torch.bfloat16).double().numpy()
+            if pr.sum() <= 2.0 ** 16 and not (force is not None and force.random() < 0.1):
+                above_one += int(pr.max() > 1.0)
+                l += pr.sum()
+                o += pr @ vf[a:a + tile]
+                continue
+        mt = xt.max()
+        if mt > m + 8.0:
+            alpha = 0.0 if m == -math.inf else 2.0 ** (m - mt)
+            raises += int(m != -math.inf)
+            m = mt
+            l *= alpha
+            o *= alpha
+        pr = torch.from_numpy(np.exp2(xt - m)).to(torch.bfloat16).double().numpy()
+        l += pr.sum()
+        o += pr @ vf[a:a + tile]
+    return o / l, above_one, raises
+
+
+@pytest.mark.parametrize("scale,regime", [(0.35, "kept"), (1.0, "both"), (4.0, "raised")])
+def test_prefill_lazy_maximum_keeps_the_budget(scale, regime):
+    # Queries of the last positions of a 1,100-token sequence with logits
+    # whose maxima grow from key tile to key tile.  Weights kept with an old
+    # maximum (up to a row sum of 2^16) and weights redone after a raise are
+    # rounded alike, and the normaliser sums the rounded weights, so the
+    # output stays a convex combination of V rows: bound (1) of
+    # tests/budget.py holds whatever the maximum was.
+    n, d = 1100, 128
+    rng = np.random.default_rng(int(scale * 100))
+    tot_above = tot_raises = 0
+    for row in range(12):
+        q, k, v = qkv(row * 17 + int(scale * 10), n, 1, 1, d)
+        kf, vf = widen(k)[:, 0, :], widen(v)[:, 0, :]
+        x = (kf @ widen(q)[0]) * scale * math.log2(math.e)
+        exact, dev, _ = oatt.decode_dev(q, k, v, scale)
+        sim, above, raises = simulate_prefill_row(x, vf, force=rng if row % 3 == 2 else None)
+        tot_above += above
+        tot_raises += raises
+        bound = U_BF16 / (1 - U_BF16) * dev[0] + 1e-12
+        assert np.all(np.abs(sim - exact[0]) <= bound)
+    # the regimes the GPU test's scales are meant to reach
+    if regime in ("kept", "both"):
+        assert tot_above > 0
+    if regime in ("both", "raised"):
+        assert tot_raises > 0
+    if regime == "kept":
+        assert tot_raises == 0
