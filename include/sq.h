@@ -78,7 +78,10 @@ typedef struct {
                                   pool; else caller memory of sq_pool_bytes() bytes,
                                   256-byte aligned, owned by the caller */
     int32_t decode_ctas;       /* 0 = automatic (SMs x resident CTAs per SM); else the
-                                  number of persistent CTAs decode attention uses */
+                                  number of persistent CTAs decode attention uses
+                                  (a decode call that would split one sequence's KV
+                                  head over more than 65,535 of them returns
+                                  SQ_ERR_CAPACITY) */
 } sq_config;
 
 enum {
@@ -162,7 +165,7 @@ SQ_API int sq_fork_aux(sq_cache *cache, sq_seq parent, sq_seq *child_out);
  *         overlap is INVALID_ARG
  * Sequences that share pages (a main thread and its forks) in one call read
  * each shared page once for all of them (Sec. 3.4, shared-context kernels).
- * Errors: BAD_HANDLE, INVALID_ARG, NO_MEMORY, CUDA. */
+ * Errors: BAD_HANDLE, INVALID_ARG, CAPACITY, NO_MEMORY, CUDA. */
 SQ_API int sq_decode_attention(sq_cache *cache, const sq_seq *seqs, int32_t n_seqs,
                         int32_t layer, const void *q, void *out,
                         int32_t out_dtype, float sm_scale, void *stream);

@@ -684,7 +684,11 @@ int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
         const DecodeSeg& s = out->segs[it.seg];
         for (int32_t j = 0; j < s.n_grp; ++j) ++out->comb_off[s.grp_seq[j] * g.Hkv + it.head + 1];
     }
-    for (int32_t k = 0; k < keys; ++k) out->comb_off[k + 1] += out->comb_off[k];
+    for (int32_t k = 0; k < keys; ++k) {
+        // the kernel counts a run's entries in 16 bits
+        if (out->comb_off[k + 1] > kMaxRunEntries) return kCapacity;
+        out->comb_off[k + 1] += out->comb_off[k];
+    }
     std::vector<int32_t> fill(out->comb_off.begin(), out->comb_off.end() - 1);
     for (DecodeItem& it : out->items) {
         const DecodeSeg& s = out->segs[it.seg];

@@ -211,11 +211,16 @@ struct DecodePlanHost {
     int32_t n_ctas = 0;
 };
 
+// Most partial results one (sequence, KV head) may have in a decode call:
+// the kernel counts a run's arrivals in 16 bits.
+constexpr int32_t kMaxRunEntries = 65535;
+
 // Plans one decode call over the given sequences (each with n >= 1):
 // groups sequences that hold the same physical page at the same logical
 // index into shared runs, splits every (run, KV head) into stages of
 // kStageTokens tokens and deals the stages out evenly to `n_ctas`
-// persistent CTAs.
+// persistent CTAs.  kCapacity if a (sequence, KV head) would get more than
+// kMaxRunEntries partial results (more CTAs than that on one sequence).
 int plan_decode(const HostCache& c, const int32_t* handles, int32_t n_seqs,
                 int32_t n_ctas, DecodePlanHost* out);
 

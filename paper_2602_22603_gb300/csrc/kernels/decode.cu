@@ -606,11 +606,32 @@ __device__ void consume(const DecodeArgs& a, int it0, int it1, uint8_t* smem, ui
 }
 
 // ---- arrivals and the merge of finished (sequence, KV head) runs -----------
-// The arrival word of a run counts the items that have written their partial;
-// the arrival that brings it to the run's length merges the run and sets the
-// word back to zero.  Every CTA arrives once per (item, group member), also
-// after a wait ran out, so every call leaves every word at zero, and a plan
-// upload writes zeros; the word therefore always starts a call at zero.
+// The arrival word of a run holds two counts.  Its low half counts the items
+// that finished (a relaxed add, the claim); the claim that brings it to the
+// run's length makes its CTA the merger.  Every other CTA then publishes its
+// partial with a release add to the high half, and the merger, instead of
+// releasing its own partial first (a GPU-scope fence on its critical path),
+// waits with acquire loads until the high half counts the other entries; its
+// own partial it reads back within the CTA.  The merger sets the word back to
+// zero.  Every CTA claims once per (item, group member), also after a wait ran
+// out, so every call leaves every word at zero, and a plan upload writes
+// zeros; the word therefore always starts a call at zero.  A run holds at
+// most 65,535 entries (the planner's limit), so the halves never carry.
+
+// GPU-scope atomics of the arrival protocol.
+__device__ __forceinline__ unsigned atom_add_relaxed_gpu(unsigned* p, unsigned v) {
+    unsigned old;
+    asm volatile("atom.relaxed.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+__device__ __forceinline__ void red_add_release_gpu(unsigned* p, unsigned v) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned* p) {
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
 
 // Up to 4 output float4 per thread per round; a round stages whole runs
 // (several when they fit) or one chunk of a long run.
@@ -661,9 +682,25 @@ __device__ void arrive_and_merge(const DecodeArgs& a, int it0, int it1, uint8_t*
         }
         if (key >= 0) {
             const int e0 = a.comb_off[key], n = a.comb_off[key + 1] - e0;
-            // release: this CTA's partials (written before the barrier above)
-            // before the count; acquire: every counted partial before the reads
-            if (atom_add_acq_rel_gpu(a.arrive + key, 1u) + 1u == (unsigned)n) {
+            // claim; a CTA that does not complete the run releases its
+            // partials (written before the barrier above) to the merger, which
+            // acquires every other entry's before its reads (its own were
+            // written within the CTA)
+            const unsigned old = atom_add_relaxed_gpu(a.arrive + key, 1u);
+            const bool merger = (old & 0xffffu) + 1u == (unsigned)n;
+            if (!merger) {
+                red_add_release_gpu(a.arrive + key, 0x10000u);
+            } else {
+                const uint64_t t0 = globaltimer_ns();
+                for (uint32_t spin = 1;; ++spin) {
+                    if ((ld_acquire_gpu(a.arrive + key) >> 16) == (unsigned)(n - 1)) break;
+                    if ((spin & 31) == 0 && globaltimer_ns() - t0 > kWaitLimitNs) {
+                        set_error(a.err, kErrTimeout);
+                        break;
+                    }
+                }
+            }
+            if (merger) {
                 a.arrive[key] = 0u;
                 const int k = atomicAdd(n_last, 1);
                 l_key[k] = key;

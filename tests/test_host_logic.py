@@ -291,6 +291,21 @@ def test_decode_plan_rejects_bad_input():
     assert hc.plan_decode([m, 999], 10)[0] == -2     # bad handle
 
 
+def test_decode_plan_limits_entries_per_run():
+    # The kernel counts a run's arrivals in 16 bits: one KV head of one
+    # sequence may have at most 65,535 partial results.  66,000 stages of 64
+    # tokens dealt to 66,000 CTAs give ~65,998 (the unit's start-up share
+    # leaves the first CTAs without stages): SQ_ERR_CAPACITY.  65,000 CTAs
+    # are accepted.
+    n = 66000 * 64
+    hc = HostCache(1, 1, 1, 64, 64, n // 64 + 4, max_pages_per_seq=n // 64 + 4)
+    rc, m = hc.seq_new()
+    assert hc.append(m, n) == 0
+    assert hc.plan_decode([m], 66000)[0] == -4      # SQ_ERR_CAPACITY
+    rc, plan = hc.plan_decode([m], 65000)
+    assert rc == 0
+
+
 @pytest.mark.parametrize("seed", range(20))
 def test_evict_tiles_compact_in_place(seed):
     """Replaying the compaction tiles in order — each tile's reads before its
