@@ -118,6 +118,7 @@ struct sq_cache {
     int num_sms = 0;
     int decode_ctas = 0;
     int evict_tile_rows = 0;
+    int evict_stages = 0;
     __nv_bfloat16* pool = nullptr;
     bool own_pool = false;
     size_t pool_bytes = 0;
@@ -364,15 +365,14 @@ void free_entry(PlanEntry& p) {
 // measured faster than 16 KiB and far faster than 4 KiB ones), at most a
 // page, and fewer if one CTA per (layer, K/V, head) plane would not fit in
 // one wave of resident CTAs.
-int choose_tile_rows(const sq_cache* c) {
+// Eviction CTA shape: 8 KiB tiles (at most a page) and a ring depth by the
+// CTAs (one per (layer, K/V, head) plane) an SM gets.  Measured on dense
+// evictions: at most one per SM runs best with 6 slots (more copies in
+// flight per CTA), 512 planes on 152 SMs with 3, 1,280 planes with 4.
+void choose_evict_shape(sq_cache* c) {
     const int64_t planes = (int64_t)c->g.L * 2 * c->g.Hkv;
-    const int target = std::max(8, 8192 / (2 * c->g.D));
-    int best = 0;
-    for (int tr = std::min(c->g.P, target); tr >= 8; tr >>= 1) {
-        best = tr;
-        if (planes <= (int64_t)c->num_sms * evict_ctas_per_sm(tr, c->g.D)) break;
-    }
-    return best;
+    c->evict_tile_rows = std::min(c->g.P, std::max(8, 8192 / (2 * c->g.D)));
+    c->evict_stages = planes <= c->num_sms ? 6 : (planes <= 4LL * c->num_sms ? 3 : 4);
 }
 
 }  // namespace
@@ -430,7 +430,7 @@ int sq_cache_create(const sq_config* cfg, sq_cache** out) {
     if (e != cudaSuccess) return cuda_status(e);
     e = prefill_prepare(g.D);
     if (e != cudaSuccess) return cuda_status(e);
-    c->evict_tile_rows = choose_tile_rows(c.get());
+    choose_evict_shape(c.get());
     c->pool_bytes = pool_bytes_of(g);
     if (cfg->kv_pool) {
         c->pool = reinterpret_cast<__nv_bfloat16*>(cfg->kv_pool);
@@ -1030,7 +1030,7 @@ int evict_impl(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_spans, v
         // CTAs, up to about four waves of resident CTAs over all planes
         const int64_t planes = (int64_t)g.L * 2 * g.Hkv;
         const int64_t resident =
-            (int64_t)c->num_sms * evict_ctas_per_sm(c->evict_tile_rows, g.D);
+            (int64_t)c->num_sms * evict_ctas_per_sm(c->evict_tile_rows, g.D, c->evict_stages);
         const int32_t max_chunks = (int32_t)std::max<int64_t>(1, 4 * resident / planes);
         evict_chunks(window_tile, (int32_t)tiles.size(), max_chunks, 4, &chunk);
         const size_t tb = tiles.size() * sizeof(EvictTile);
@@ -1052,6 +1052,7 @@ int evict_impl(sq_cache* c, sq_seq seq, const sq_span* spans, int32_t n_spans, v
         ea.n_tiles = (int32_t)tiles.size();
         ea.n_pieces = (int32_t)pieces.size();
         ea.tile_rows = c->evict_tile_rows;
+        ea.stages = c->evict_stages;
         ea.zero_tiles = plan.zeroed_rows > 0 ? 1 : 0;
         ea.n_chunks = (int32_t)chunk.size() - 1;
         ea.chunk = ea.n_chunks > 1 ? reinterpret_cast<const int32_t*>(s.d + tb + pcb) : nullptr;

@@ -124,9 +124,9 @@ __global__ void __launch_bounds__(256) sq_cow_copy_kernel(const CowArgs a) {
 // zeros: the unused slots of a page that a ragged eviction leaves partial.  Its store reads a zero tile that the
 // CTA's warp clears once; it writes only past the rows its window kept, and
 // later tiles read only later windows' pages.
+template <int S>  // ring slots
 __global__ void __launch_bounds__(32) sq_evict_compact_kernel(const EvictArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    constexpr int S = kEvictStages;
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
     const uint32_t row_bytes = (uint32_t)a.D * 2u;
@@ -263,32 +263,50 @@ cudaError_t launch_cow_copy(const CowArgs& a, int num_sms, cudaStream_t st) {
     return cudaGetLastError();
 }
 
-int evict_smem_bytes(int tile_rows, int D, bool zero_tiles) {
-    return (kEvictStages + (zero_tiles ? 1 : 0)) * tile_rows * D * 2 + kEvictStages * 8 + 128;
+int evict_smem_bytes(int tile_rows, int D, int stages, bool zero_tiles) {
+    return (stages + (zero_tiles ? 1 : 0)) * tile_rows * D * 2 + stages * 8 + 128;
 }
 
-int evict_ctas_per_sm(int tile_rows, int D) {
+// The ring depths built: 3, 4 and 6 slots (the host's choices).
+template <typename F>
+static cudaError_t with_evict_kernel(int stages, F f) {
+    switch (stages) {
+        case 3: return f(sq_evict_compact_kernel<3>);
+        case 4: return f(sq_evict_compact_kernel<4>);
+        case 6: return f(sq_evict_compact_kernel<6>);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+int evict_ctas_per_sm(int tile_rows, int D, int stages) {
     int n = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, sq_evict_compact_kernel, 32,
-                                                      evict_smem_bytes(tile_rows, D)) !=
-            cudaSuccess ||
-        n < 1)
-        return 1;
-    return n;
+    const cudaError_t e = with_evict_kernel(stages, [&](auto kernel) {
+        return cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel, 32,
+                                                             evict_smem_bytes(tile_rows, D, stages));
+    });
+    return e != cudaSuccess || n < 1 ? 1 : n;
 }
 
 cudaError_t evict_prepare() {
-    return cudaFuncSetAttribute(sq_evict_compact_kernel,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                evict_smem_bytes(kStageTokens, 128, true));
+    for (int stages : {3, 4, 6}) {
+        const cudaError_t e = with_evict_kernel(stages, [&](auto kernel) {
+            return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        evict_smem_bytes(kStageTokens, 128, stages, true));
+        });
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 cudaError_t launch_evict(const EvictArgs& a, cudaStream_t st) {
     const int blocks = a.L * 2 * a.Hkv * (a.chunk ? a.n_chunks : 1);
     if (blocks == 0 || a.n_tiles == 0) return cudaSuccess;
-    sq_evict_compact_kernel<<<blocks, 32, evict_smem_bytes(a.tile_rows, a.D, a.zero_tiles != 0),
-                              st>>>(a);
-    return cudaGetLastError();
+    const int smem = evict_smem_bytes(a.tile_rows, a.D, a.stages, a.zero_tiles != 0);
+    const cudaError_t e = with_evict_kernel(a.stages, [&](auto kernel) {
+        kernel<<<blocks, 32, smem, st>>>(a);
+        return cudaSuccess;
+    });
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace sq

@@ -155,6 +155,7 @@ struct EvictArgs {
     const EvictPiece* pieces;   // their contiguous source pieces
     int32_t n_tiles, n_pieces;
     int32_t tile_rows;          // rows a tile holds at most
+    int32_t stages;             // shared-memory ring slots: 3, 4 or 6
     int32_t zero_tiles;         // 1: some tiles (those without pieces) write zeros
     // null, or [n_chunks + 1] tile indices: chunk c (tiles [chunk[c],
     // chunk[c + 1]), whole windows) of every plane runs in its own CTA
@@ -166,12 +167,11 @@ struct EvictArgs {
 cudaError_t launch_append(const AppendArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_append_batch(const AppendBatchArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_cow_copy(const CowArgs& a, int num_sms, cudaStream_t st);
-constexpr int kEvictStages = 6;
-// Shared memory of one eviction CTA for a tile size (plus one zero tile when
-// the plan zeroes rows).
-int evict_smem_bytes(int tile_rows, int D, bool zero_tiles = false);
-// Resident eviction CTAs per SM for a tile size.
-int evict_ctas_per_sm(int tile_rows, int D);
+// Shared memory of one eviction CTA for a tile size and ring depth (plus one
+// zero tile when the plan zeroes rows).
+int evict_smem_bytes(int tile_rows, int D, int stages, bool zero_tiles = false);
+// Resident eviction CTAs per SM for a tile size and ring depth.
+int evict_ctas_per_sm(int tile_rows, int D, int stages);
 cudaError_t evict_prepare();  // raises the dynamic shared-memory limit once
 cudaError_t launch_evict(const EvictArgs& a, cudaStream_t st);
 
