@@ -270,6 +270,39 @@ def test_serving_128k_ragged_eviction_full_size():
         bp.close()
 
 
+@pytest.mark.parametrize("L,ctx", [(32, 16384), (80, 8192)])
+def test_eviction_ring_depths_many_planes(L, ctx):
+    """Dense and ragged evictions with 32 and 80 layers of 8 KV heads (512 and
+    1,280 (layer, K/V, head) planes: a cache on 152 SMs drives them with a
+    ring of 3 and of 4 tiles; the small caches of the other tests use 6).
+    Two requests, each with a fork alive while its request is evicted (the
+    changed shared pages are copied on write); page tables and fills
+    bit-exact, every plane of three layers of every sequence bit-exact, then
+    decode of all four sequences against the oracle."""
+    Hq, Hkv, D, P = 32, 8, 128, 64
+    bp = BankPair(L, Hq, Hkv, D, P, num_pages=4 * (ctx // P + 4) + 64, seed=L)
+    try:
+        mains, auxs = [], []
+        for r in range(2):
+            m = bp.seq_new()
+            bp.fill(m, ctx, 1024)   # chunks that fit the bank at 80 layers
+            mains.append(m)
+            auxs.append(bp.fork(m))
+        for r, m in enumerate(mains):
+            spans = request_spans(L, r, ctx, P)
+            bp.evict(m, spans, ragged=(r == 1))
+        seqs = mains + auxs
+        bp.check_tables(seqs)
+        for h in seqs:
+            for layer in (0, L // 2, L - 1):
+                bp.check_planes(h, layer)
+        for h in seqs:
+            bp.append(h, 1)
+        _decode_and_check(bp, seqs, L - 1, 1.0 / math.sqrt(D), 900 + L, None)
+    finally:
+        bp.close()
+
+
 def test_d64_long_contexts_decode_evict_prefill():
     """The d = 64 kernels (a six-stage decode ring, the 64-column prefill
     tiles) at long contexts: 2 requests x 49,152 tokens + forks, G = 8, P = 64,
