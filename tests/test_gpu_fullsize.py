@@ -270,16 +270,17 @@ def test_serving_128k_ragged_eviction_full_size():
         bp.close()
 
 
-@pytest.mark.parametrize("L,ctx", [(32, 16384), (80, 8192)])
-def test_eviction_ring_depths_many_planes(L, ctx):
+@pytest.mark.parametrize("L,D,ctx", [(32, 128, 16384), (80, 128, 8192), (32, 64, 16384)])
+def test_eviction_ring_depths_many_planes(L, D, ctx):
     """Dense and ragged evictions with 32 and 80 layers of 8 KV heads (512 and
     1,280 (layer, K/V, head) planes: a cache on 152 SMs drives them with a
-    ring of 3 and of 4 tiles; the small caches of the other tests use 6).
-    Two requests, each with a fork alive while its request is evicted (the
-    changed shared pages are copied on write); page tables and fills
-    bit-exact, every plane of three layers of every sequence bit-exact, then
-    decode of all four sequences against the oracle."""
-    Hq, Hkv, D, P = 32, 8, 128, 64
+    ring of 3 and of 4 tiles; the small caches of the other tests use 6), at
+    d = 128 (32-row tiles) and d = 64 (64-row tiles).  Two requests, each with
+    a fork alive while its request is evicted (the changed shared pages are
+    copied on write); page tables and fills bit-exact, every plane of three
+    layers of every sequence bit-exact, then decode of all four sequences
+    against the oracle."""
+    Hq, Hkv, P = 32, 8, 64
     bp = BankPair(L, Hq, Hkv, D, P, num_pages=4 * (ctx // P + 4) + 64, seed=L)
     try:
         mains, auxs = [], []
