@@ -228,7 +228,8 @@ SQ_API int sq_evict_spans_ragged(sq_cache *cache, sq_seq seq, const sq_span *spa
  * ragged eviction); otherwise UNSUPPORTED.  The sequence and the cache are
  * not modified.  The
  * kernel runs on the tensor cores (bf16 products, fp32 accumulation; the
- * softmax weights are rounded to bf16 before the value product).
+ * softmax weights are rounded to bf16 before the value product, and the
+ * normaliser sums the same rounded weights).
  * Errors: BAD_HANDLE, INVALID_ARG, UNSUPPORTED, NO_MEMORY, CUDA. */
 SQ_API int sq_prefill_attention(sq_cache *cache, sq_seq seq, int32_t layer, int32_t n_q,
                                 const void *q, void *out, int32_t out_dtype, float *lse,
