@@ -154,6 +154,11 @@ int64_t sqh_peak_live_pages(void* c) { return static_cast<HostCache*>(c)->peak_l
 //   counts n_segs, n_items, n_ctas, n_page_ids, n_comb_keys, n_comb_ent,
 //   unique_tokens, logical_tokens, sizeof(DecodeSeg), offset page_fill (-1: none).
 // If buf is non-NULL and buf_bytes >= total, the serialised plan is written.
+// The eviction CTA shape the library picks: tile rows for (P, D) and ring
+// slots for (planes, SMs).
+int32_t sqh_evict_tile_rows(int32_t P, int32_t D) { return evict_tile_rows_for(P, D); }
+int32_t sqh_evict_stages(int64_t planes, int32_t num_sms) { return evict_stages_for(planes, num_sms); }
+
 int sqh_plan_decode(void* c, const int32_t* handles, int32_t n, int32_t n_ctas,
                     int64_t* layout_out, uint8_t* buf, int64_t buf_bytes) {
     HostCache* hc = static_cast<HostCache*>(c);

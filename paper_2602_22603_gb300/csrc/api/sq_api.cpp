@@ -369,18 +369,12 @@ void free_entry(PlanEntry& p) {
     p = PlanEntry();
 }
 
-// Rows per eviction tile: 8 KiB copies (32 rows at d = 128, 64 at d = 64;
-// measured faster than 16 KiB and far faster than 4 KiB ones), at most a
-// page, and fewer if one CTA per (layer, K/V, head) plane would not fit in
-// one wave of resident CTAs.
-// Eviction CTA shape: 8 KiB tiles (at most a page) and a ring depth by the
-// CTAs (one per (layer, K/V, head) plane) an SM gets.  Measured on dense
-// evictions: at most one per SM runs best with 6 slots (more copies in
-// flight per CTA), 512 planes on 152 SMs with 3, 1,280 planes with 4.
+// Eviction CTA shape (evict_tile_rows_for, evict_stages_for) and the CTAs
+// of it resident on the device at once.
 void choose_evict_shape(sq_cache* c) {
     const int64_t planes = (int64_t)c->g.L * 2 * c->g.Hkv;
-    c->evict_tile_rows = std::min(c->g.P, std::max(8, 8192 / (2 * c->g.D)));
-    c->evict_stages = planes <= c->num_sms ? 6 : (planes <= 4LL * c->num_sms ? 3 : 4);
+    c->evict_tile_rows = evict_tile_rows_for(c->g.P, c->g.D);
+    c->evict_stages = evict_stages_for(planes, c->num_sms);
     c->evict_resident =
         (int64_t)c->num_sms * evict_ctas_per_sm(c->evict_tile_rows, c->g.D, c->evict_stages);
 }

@@ -485,6 +485,14 @@ void evict_tiles(const EvictPlan& p, int32_t tile_rows, std::vector<EvictTile>* 
     }
 }
 
+int32_t evict_tile_rows_for(int32_t P, int32_t D) {
+    return std::min(P, std::max(8, 8192 / (2 * D)));
+}
+
+int32_t evict_stages_for(int64_t planes, int32_t num_sms) {
+    return planes <= num_sms ? 6 : (planes <= 4LL * num_sms ? 3 : 4);
+}
+
 void evict_chunks(const std::vector<int32_t>& window_tile, int32_t n_tiles, int32_t max_chunks,
                   int32_t min_tiles, std::vector<int32_t>* chunk) {
     chunk->assign(1, 0);

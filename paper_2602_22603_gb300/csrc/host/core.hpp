@@ -186,6 +186,14 @@ class HostCache {
 void evict_tiles(const EvictPlan& p, int32_t tile_rows, std::vector<EvictTile>* tiles,
                  std::vector<EvictPiece>* pieces, std::vector<int32_t>* window_tile = nullptr);
 
+// Eviction CTA shape: rows of an 8 KiB tile (at most a page, at least 8;
+// 8 KiB copies measured faster than 16 KiB ones and far faster than 4 KiB
+// ones), and ring slots by the (layer, K/V, head) planes each SM gets: 6 when
+// there is at most one per SM, 3 up to four per SM, 4 beyond (measured on
+// dense evictions of 128, 512 and 1,280 planes on 152 SMs).
+int32_t evict_tile_rows_for(int32_t P, int32_t D);
+int32_t evict_stages_for(int64_t planes, int32_t num_sms);
+
 // Groups consecutive windows into at most `max_chunks` chunks of about equal
 // tile counts, at least `min_tiles` tiles each (but the last): chunk c is
 // tiles [chunk[c], chunk[c + 1]).  One chunk when there is one window.

@@ -47,6 +47,10 @@ def lib():
         L.sqh_peak_live_pages.restype = ctypes.c_int64
         L.sqh_plan_decode.argtypes = [P, I32P, I32, I32, I64P, ctypes.POINTER(ctypes.c_uint8),
                                       ctypes.c_int64]
+        L.sqh_evict_tile_rows.argtypes = [I32, I32]
+        L.sqh_evict_tile_rows.restype = ctypes.c_int32
+        L.sqh_evict_stages.argtypes = [ctypes.c_int64, I32]
+        L.sqh_evict_stages.restype = ctypes.c_int32
         L.sqh_plan_prefill.argtypes = [I32, I32, I32, I32, I32, I32P, I32, I32, I64P, I32P, I32,
                                        I32P, I32]
         _lib = L

@@ -6,7 +6,7 @@ import random
 import pytest
 
 from oracle import cache_model as ocm
-from tests.hostlib import HostCache
+from tests.hostlib import HostCache, lib
 
 CODES = {ocm.InvalidArg: -1, ocm.BadHandle: -2, ocm.NoPages: -3, ocm.Capacity: -4}
 STAGE = 64  # tokens per decode stage
@@ -597,3 +597,16 @@ def test_prefill_tiles_skip_boxes_a_span_covers():
     # the same spans with 16-token pages keep aligned 128-key tiles
     rc, info, tiles = plan_prefill(8, 2, 512, 512, [(64, 128), (256, 384)], P=16)
     assert [int(t[0]) for t in tiles] == [0, 128, 384]
+
+
+def test_evict_shape_rule():
+    # 8 KiB tiles, at most a page; ring slots by the planes per SM
+    L_ = lib()
+    assert L_.sqh_evict_tile_rows(64, 128) == 32
+    assert L_.sqh_evict_tile_rows(64, 64) == 64
+    assert L_.sqh_evict_tile_rows(16, 128) == 16
+    assert L_.sqh_evict_tile_rows(8, 64) == 8
+    assert L_.sqh_evict_tile_rows(256, 64) == 64
+    for planes, stages in ((1, 6), (128, 6), (152, 6), (153, 3), (512, 3), (608, 3), (609, 4),
+                           (1280, 4), (100000, 4)):
+        assert L_.sqh_evict_stages(planes, 152) == stages, planes
